@@ -1,0 +1,408 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each pin is chosen so that a plausible mistake in the oracle fails it:
+a dropped [CLS] key, '>' instead of '>=', a non-causal or wrong Stage-II key
+set, mean instead of max over text tokens, a register counted as a
+candidate, a per-sample instead of per-segment Stage-I threshold, a wrong
+head average, a reordered or lossy gather.
+"""
+
+from __future__ import annotations
+
+import math
+from decimal import Decimal, getcontext
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import occam_oracle as O
+from synth import tiny_batch
+from tests._fixtures import worked_example
+
+
+# ----------------------------------------------------------------------------- worked example
+
+@pytest.mark.parametrize("case", [0, 1, 2])
+def test_worked_example_hand_derived(case):
+    """Hand-derived example (tests/golden/worked_example.json; Eqs. 4-8)."""
+    batch, g = worked_example()
+    c = g["cases"][case]
+    out = O.prune(batch, g["lambda1"], c["lambda2"])
+    e = math.e
+    Z1 = 3 + e + e * e
+    np.testing.assert_allclose(out["s1"], [e / Z1, 1 / Z1, e * e / Z1, 1 / Z1], rtol=1e-14)
+    np.testing.assert_allclose(out["ref1"], [1 / Z1], rtol=1e-14)
+    assert out["keep1"].astype(int).tolist() == c["keep1"]
+    s2_r0 = e / (e + 3)
+    s2_r2 = e * e / (3 + e + e * e)
+    ref2 = (1 / (e + 3) + 1 / (3 + e + e * e)) / 2
+    np.testing.assert_allclose(out["s2"][[0, 2]], [s2_r0, s2_r2], rtol=1e-14)
+    assert out["s2"][1] == 0.0  # pruned in Stage I: never scored in Stage II
+    np.testing.assert_allclose(out["ref2"], [ref2], rtol=1e-14)
+    assert out["keep2"].astype(int).tolist() == c["keep2"]
+    assert int(out["count_vis"][0]) == c["count_vis"]
+    assert out["out_index"].tolist() == c["out_index"]
+    assert out["count_out"].tolist() == [len(c["out_index"])]
+
+
+# ----------------------------------------------------------------------------- P1 softmax
+
+def test_softmax_rows_sum_to_one():
+    rng = np.random.default_rng(0)
+    x = rng.normal(size=(50, 77)) * 20
+    A = O.softmax(x, axis=1)
+    np.testing.assert_allclose(A.sum(axis=1), 1.0, atol=1e-12)
+    assert (A >= 0).all()
+    # shift invariance and the textbook formula on a small row
+    row = np.array([0.5, -1.0, 2.0])
+    ref = np.exp(row) / np.exp(row).sum()
+    np.testing.assert_allclose(O.softmax(row), ref, rtol=1e-15)
+    np.testing.assert_allclose(O.softmax(row + 1000.0), ref, rtol=1e-12)
+
+
+def test_stage1_mass_conservation():
+    """Without k_cls every segment's s1 sums to 1; with it, to 1 - A(cls)."""
+    b = tiny_batch(B=2, segs=3, P=(6, 9), R=2, M=(3, 2), seed=3)
+    m = b["meta"]
+    s1, _ = O.stage1_cls(b["q_cls"], None, b["K1"], m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"])
+    for s in range(m["S_tot"]):
+        a, z = m["seg_off_host"][s], m["seg_off_host"][s + 1]
+        assert abs(s1[a:z].sum() - 1.0) < 1e-12
+    s1c, _ = O.stage1_cls(b["q_cls"], b["k_cls"], b["K1"], m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"])
+    for s in range(m["S_tot"]):
+        a, z = m["seg_off_host"][s], m["seg_off_host"][s + 1]
+        assert s1c[a:z].sum() < 1.0 - 1e-6
+    # mutual: the average over queries of row-stochastic rows sums to 1
+    bm = tiny_batch(B=2, segs=1, P=(7, 4), R=2, M=(2, 2), stage1="mutual", seed=4)
+    mm = bm["meta"]
+    s1m, _ = O.stage1_mutual(bm["Q1"], bm["K1"], mm["seg_off_host"], mm["reg_idx_host"], mm["reg_off_host"])
+    for s in range(mm["S_tot"]):
+        a, z = mm["seg_off_host"][s], mm["seg_off_host"][s + 1]
+        assert abs(s1m[a:z].sum() - 1.0) < 1e-12
+
+
+def test_stage2_mass_without_text_keys_and_one_token():
+    """text_keys='none', M=1: sum_vis s2 + R * ref2 = 1 over the S1 rows."""
+    b = tiny_batch(B=2, segs=2, P=(5, 6), R=2, M=(1, 1), seed=5)
+    m = b["meta"]
+    is_reg = O.register_mask(m["total_rows"], m["reg_idx_host"])
+    keep1 = np.ones(m["total_rows"], bool)
+    s2, ref2 = O.stage2_scores(b["Q_text"], b["K_text"], b["K2"], keep1, is_reg,
+                               m["row_off_host"], m["text_off_host"], text_keys="none")
+    for bb in range(m["B"]):
+        a, z = m["row_off_host"][bb], m["row_off_host"][bb + 1]
+        R_b = int(is_reg[a:z].sum())
+        assert abs(s2[a:z][~is_reg[a:z]].sum() + R_b * ref2[bb] - 1.0) < 1e-12
+
+
+# ----------------------------------------------------------------------------- P2 / P12 uniform
+
+def _zero(t):
+    return torch.zeros_like(t)
+
+
+def test_stage1_cls_zero_query_is_uniform_and_ties_keep():
+    b = tiny_batch(B=2, segs=2, P=(5, 8), R=3, M=(2, 3), seed=6)
+    b["q_cls"] = _zero(b["q_cls"])
+    m = b["meta"]
+    s1, ref1 = O.stage1_cls(b["q_cls"], b["k_cls"], b["K1"], m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"])
+    for s in range(m["S_tot"]):
+        a, z = m["seg_off_host"][s], m["seg_off_host"][s + 1]
+        np.testing.assert_allclose(s1[a:z], 1.0 / (z - a + 1), rtol=1e-15)  # +1: the [CLS] key
+    out_eq = O.prune(b, 1.0, 0.0)
+    out_gt = O.prune(b, 1.0 + 2.0 ** -20, 0.0)
+    is_reg = out_eq["is_reg"]
+    assert out_eq["keep1"][~is_reg].all()          # equality keeps (>=)
+    assert not out_gt["keep1"][~is_reg].any()
+    assert out_gt["keep1"][is_reg].all()           # the register always stays in S1
+
+
+def test_stage1_mutual_zero_query_is_uniform():
+    b = tiny_batch(B=2, segs=1, P=(6, 9), R=2, M=(2, 2), stage1="mutual", seed=7)
+    b["Q1"] = _zero(b["Q1"])
+    m = b["meta"]
+    s1, ref1 = O.stage1_mutual(b["Q1"], b["K1"], m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"])
+    for s in range(m["S_tot"]):
+        a, z = m["seg_off_host"][s], m["seg_off_host"][s + 1]
+        np.testing.assert_allclose(s1[a:z], 1.0 / (z - a), rtol=1e-14)
+    out = O.prune(b, 1.0, 0.0)
+    assert out["keep1"].all()
+    out = O.prune(b, 1.0 + 1e-9, 0.0)
+    assert not out["keep1"][~out["is_reg"]].any()
+
+
+# ----------------------------------------------------------------------------- P3 Stage II closed form
+
+def _harmonic(n):
+    return sum(1.0 / k for k in range(1, n + 1))
+
+
+@pytest.mark.parametrize("M", [1, 3, 7])
+def test_stage2_zero_query_closed_form(M):
+    """Q_text = 0: A_j is uniform over n image keys + (j+1) causal text keys.
+
+    s2(v) = 1/(n+1) (its max, at j = 0); s2(r) = (H_{n+M} - H_n) / M.
+    """
+    b = tiny_batch(B=2, segs=2, P=(4, 6), R=2, M=(M, M), seed=8)
+    b["Q_text"] = _zero(b["Q_text"])
+    m = b["meta"]
+    is_reg = O.register_mask(m["total_rows"], m["reg_idx_host"])
+    rng = np.random.default_rng(1)
+    keep1 = rng.random(m["total_rows"]) < 0.6
+    s2, ref2 = O.stage2_scores(b["Q_text"], b["K_text"], b["K2"], keep1, is_reg,
+                               m["row_off_host"], m["text_off_host"])
+    for bb in range(m["B"]):
+        a, z = m["row_off_host"][bb], m["row_off_host"][bb + 1]
+        sel = (keep1[a:z] & ~is_reg[a:z])
+        n = int(sel.sum() + is_reg[a:z].sum())
+        np.testing.assert_allclose(s2[a:z][sel], 1.0 / (n + 1), rtol=1e-14)
+        assert (s2[a:z][~sel & ~is_reg[a:z]] == 0).all()
+        np.testing.assert_allclose(ref2[bb], (_harmonic(n + M) - _harmonic(n)) / M, rtol=1e-13)
+
+
+# ----------------------------------------------------------------------------- P4 heads
+
+def test_identical_heads_equal_single_head():
+    b1 = tiny_batch(B=1, segs=2, P=(6,), R=2, M=(4,), H1=1, H2=1, seed=9)
+    bH = dict(b1)
+    for k in ("q_cls", "k_cls", "K1", "Q_text", "K_text", "K2"):
+        bH[k] = b1[k].repeat(1, 3, 1)
+    o1 = O.prune(b1, 0.7, 1.1)
+    oH = O.prune(bH, 0.7, 1.1)
+    for k in ("s1", "ref1", "s2", "ref2"):
+        np.testing.assert_allclose(oH[k], o1[k], rtol=1e-13)
+    assert (oH["keep2"] == o1["keep2"]).all()
+
+
+# ----------------------------------------------------------------------------- P5 two keys
+
+@pytest.mark.parametrize("dl", [-2, 0, 1, 3])
+def test_two_key_threshold(dl):
+    """One visual key, one register, integer logits: keep iff lambda <= exp(l_v - l_r)."""
+    q = torch.tensor([[[2.0, 0, 0, 0]]]).to(torch.bfloat16)          # scale 1/2 -> logit = k[0]
+    K1 = torch.tensor([[[float(dl), 1, 2, 3]], [[0.0, -1, 5, 2]]]).to(torch.bfloat16)
+    seg_off = np.array([0, 2])
+    s1, ref1 = O.stage1_cls(q, None, K1, seg_off, np.array([1]), np.array([0, 1]))
+    ratio = math.exp(dl)
+    assert abs(s1[0] / ref1[0] - ratio) < 1e-12 * ratio
+    is_reg = np.array([False, True])
+    for lam, want in ((ratio * (1 - 1e-9), True), (ratio * (1 + 1e-9), False)):
+        keep = O.threshold(s1, np.full(2, ref1[0]), lam, is_reg)
+        assert bool(keep[0]) == want and bool(keep[1])
+
+
+# ----------------------------------------------------------------------------- P6 threshold set
+
+def test_kept_set_is_top_count_per_segment_and_sample():
+    b = tiny_batch(B=3, segs=3, P=(20, 13, 31), R=2, M=(5, 9, 2), seed=10)
+    out = O.prune(b, 0.9, 1.2)
+    m = b["meta"]
+    is_reg = out["is_reg"]
+    for s in range(m["S_tot"]):
+        a, z = m["seg_off_host"][s], m["seg_off_host"][s + 1]
+        vis = np.arange(a, z)[~is_reg[a:z]]
+        k = int(out["keep1"][vis].sum())
+        top = set(vis[np.argsort(-out["s1"][vis], kind="stable")[:k]].tolist())
+        assert top == set(vis[out["keep1"][vis]].tolist())
+    for bb in range(m["B"]):
+        a, z = m["row_off_host"][bb], m["row_off_host"][bb + 1]
+        cand = np.arange(a, z)[out["keep1"][a:z] & ~is_reg[a:z]]
+        k = int(out["keep2"][cand].sum())
+        top = set(cand[np.argsort(-out["s2"][cand], kind="stable")[:k]].tolist())
+        assert top == set(cand[out["keep2"][cand]].tolist())
+
+
+# ----------------------------------------------------------------------------- P7 monotone
+
+def test_counts_monotone_in_lambda():
+    b = tiny_batch(B=2, segs=2, P=(25, 18), R=2, M=(6, 4), seed=11)
+    c1 = [O.prune(b, l1, 0.0)["n1_vis"].sum() for l1 in np.linspace(0, 2.5, 11)]
+    assert all(x >= y for x, y in zip(c1, c1[1:]))
+    assert c1[0] == 25 * 2 + 18 * 2
+    base = O.prune(b, 0.8, 0.0)
+    c2 = [O.prune(b, 0.8, l2, keep1_override=base["keep1"])["count_vis"].sum()
+          for l2 in np.linspace(0, 4, 13)]
+    assert all(x >= y for x, y in zip(c2, c2[1:]))
+    assert c2[0] == base["n1_vis"].sum()
+
+
+# ----------------------------------------------------------------------------- P8-P10 compaction
+
+def test_lambda_zero_copies_everything():
+    b = tiny_batch(B=2, segs=2, P=(5, 7), R=2, M=(3, 4), seed=12)
+    out = O.prune(b, 0.0, 0.0)
+    n = b["meta"]["total_rows"]
+    assert out["out_index"].tolist() == list(range(n))
+    for name in ("hidden", "K2", "V"):
+        raw = b[name].reshape(n, -1).view(torch.int16).numpy()
+        assert (out["gathered"][name] == raw).all()
+
+
+def test_gather_equals_boolean_mask_indexing():
+    b = tiny_batch(B=3, segs=2, P=(9, 4, 12), R=2, M=(3, 6, 2), seed=13)
+    out = O.prune(b, 0.8, 1.1)
+    m = b["meta"]
+    keep = out["keep2"]
+    hid = b["hidden"].float().numpy()
+    got = b["hidden"].view(torch.int16).numpy()[out["out_index"]]
+    pos = 0
+    for bb in range(m["B"]):
+        a, z = m["row_off_host"][bb], m["row_off_host"][bb + 1]
+        want = hid[a:z][keep[a:z]]                       # numpy boolean-mask indexing
+        n = want.shape[0]
+        assert out["count_out"][bb] == n and out["out_off"][bb] == pos
+        np.testing.assert_array_equal(
+            torch.from_numpy(got[pos:pos + n]).view(torch.bfloat16).float().numpy(), want)
+        assert (np.diff(out["out_index"][pos:pos + n]) > 0).all()   # order preserved
+        pos += n
+    assert out["out_off"][-1] == pos == keep.sum()
+
+
+@pytest.mark.parametrize("keep_registers", [True, False])
+def test_registers_are_never_candidates(keep_registers):
+    b = tiny_batch(B=2, segs=3, P=(6, 5), R=3, M=(2, 3), seed=14)
+    out = O.prune(b, 0.0, 0.0, keep_registers=keep_registers)
+    is_reg = out["is_reg"]
+    assert out["count_vis"].sum() == (~is_reg).sum()
+    assert bool(np.isin(np.nonzero(is_reg)[0], out["out_index"]).all()) == keep_registers
+    assert not np.isin(np.nonzero(is_reg)[0], out["out_index"]).any() or keep_registers
+    assert out["count_out"].sum() == (~is_reg).sum() + (is_reg.sum() if keep_registers else 0)
+
+
+# ----------------------------------------------------------------------------- P13 scale invariance
+
+def test_threshold_scale_invariant():
+    rng = np.random.default_rng(2)
+    s = rng.random(100)
+    ref = np.full(100, 0.4)
+    is_reg = np.zeros(100, bool)
+    is_reg[[3, 50]] = True
+    base = O.threshold(s, ref, 1.3, is_reg)
+    for c in (1e-3, 0.5, 7.0):
+        assert (O.threshold(s * c, ref * c, 1.3, is_reg) == base).all()
+
+
+# ----------------------------------------------------------------------------- P11 brute force
+
+def _dexp(x):
+    return x.exp()
+
+
+def _brute_stage1_cls(q, kc, K, seg_off, reg_idx, reg_off):
+    H, d = len(K[0]), len(K[0][0])
+    sc = Decimal(1) / Decimal(d).sqrt()
+    s1 = [Decimal(0)] * len(K)
+    ref = []
+    for s in range(len(seg_off) - 1):
+        rows = range(seg_off[s], seg_off[s + 1])
+        for h in range(H):
+            dot = lambda a, b: sum(Decimal(x) * Decimal(y) for x, y in zip(a, b))  # noqa: E731
+            logits = {r: dot(q[s][h], K[r][h]) * sc for r in rows}
+            z = sum(_dexp(v) for v in logits.values())
+            if kc is not None:
+                z += _dexp(dot(q[s][h], kc[s][h]) * sc)
+            for r in rows:
+                s1[r] += _dexp(logits[r]) / z / H
+        regs = reg_idx[reg_off[s]:reg_off[s + 1]]
+        ref.append(sum(s1[r] for r in regs) / len(regs))
+    return s1, ref
+
+
+def _brute_stage1_mutual(Q, K, seg_off, reg_idx, reg_off):
+    H, d = len(K[0]), len(K[0][0])
+    sc = Decimal(1) / Decimal(d).sqrt()
+    s1 = [Decimal(0)] * len(K)
+    ref = []
+    dot = lambda a, b: sum(Decimal(x) * Decimal(y) for x, y in zip(a, b))  # noqa: E731
+    for s in range(len(seg_off) - 1):
+        rows = list(range(seg_off[s], seg_off[s + 1]))
+        n = len(rows)
+        for h in range(H):
+            for u in rows:
+                e = {v: _dexp(dot(Q[u][h], K[v][h]) * sc) for v in rows}
+                z = sum(e.values())
+                for v in rows:
+                    s1[v] += e[v] / z / H / n
+        regs = reg_idx[reg_off[s]:reg_off[s + 1]]
+        ref.append(sum(s1[r] for r in regs) / len(regs))
+    return s1, ref
+
+
+def _brute_stage2(Q, Kt, K, keep1, is_reg, row_off, text_off):
+    H, d = len(K[0]), len(K[0][0])
+    sc = Decimal(1) / Decimal(d).sqrt()
+    dot = lambda a, b: sum(Decimal(x) * Decimal(y) for x, y in zip(a, b))  # noqa: E731
+    s2 = [Decimal(0)] * len(K)
+    ref2 = []
+    for b in range(len(row_off) - 1):
+        S1 = [r for r in range(row_off[b], row_off[b + 1]) if keep1[r] or is_reg[r]]
+        texts = list(range(text_off[b], text_off[b + 1]))
+        M = len(texts)
+        regsum = Decimal(0)
+        regs = [r for r in S1 if is_reg[r]]
+        best = {r: Decimal(0) for r in S1}
+        for jj, j in enumerate(texts):
+            p = {r: Decimal(0) for r in S1}
+            for h in range(H):
+                e = {r: _dexp(dot(Q[j][h], K[r][h]) * sc) for r in S1}
+                z = sum(e.values()) + sum(_dexp(dot(Q[j][h], Kt[t][h]) * sc) for t in texts[:jj + 1])
+                for r in S1:
+                    p[r] += e[r] / z / H
+            for r in S1:
+                best[r] = max(best[r], p[r])
+            regsum += sum(p[r] for r in regs) / len(regs)
+        for r in S1:
+            if not is_reg[r]:
+                s2[r] = best[r]
+        ref2.append(regsum / M)
+    return s2, ref2
+
+
+def _lists(t):
+    return t.float().tolist()
+
+
+def test_brute_force_decimal_tiny():
+    """Every score recomputed with 50-digit decimals; all lambda breakpoints checked."""
+    getcontext().prec = 50
+    b = tiny_batch(B=2, segs=2, P=(3, 4), R=1, M=(2, 3), H1=2, d1=4, H2=2, d2=4, seed=15)
+    m = b["meta"]
+    out = O.prune(b, 0.9, 1.0)
+    s1, ref1 = _brute_stage1_cls(_lists(b["q_cls"]), _lists(b["k_cls"]), _lists(b["K1"]),
+                                 m["seg_off_host"].tolist(), m["reg_idx_host"].tolist(), m["reg_off_host"].tolist())
+    np.testing.assert_allclose(out["s1"], [float(x) for x in s1], rtol=1e-14)
+    np.testing.assert_allclose(out["ref1"], [float(x) for x in ref1], rtol=1e-14)
+    is_reg = out["is_reg"]
+    s2, ref2 = _brute_stage2(_lists(b["Q_text"]), _lists(b["K_text"]), _lists(b["K2"]), out["keep1"].tolist(),
+                             is_reg.tolist(), m["row_off_host"].tolist(), m["text_off_host"].tolist())
+    np.testing.assert_allclose(out["s2"], [float(x) for x in s2], rtol=1e-14, atol=0)
+    np.testing.assert_allclose(out["ref2"], [float(x) for x in ref2], rtol=1e-14)
+    # Stage-I count as a step function of lambda1: it drops exactly at each ratio
+    seg_of_row = np.repeat(np.arange(m["S_tot"]), np.diff(m["seg_off_host"]))
+    ratios = sorted(float(s1[r] / ref1[seg_of_row[r]]) for r in range(m["total_rows"]) if not is_reg[r])
+    for i, x in enumerate(ratios):
+        n_at = O.prune(b, x * (1 - 1e-12), 0.0)["n1_vis"].sum()
+        n_after = O.prune(b, x * (1 + 1e-12), 0.0)["n1_vis"].sum()
+        assert n_at == len(ratios) - i and n_after == len(ratios) - i - 1
+
+
+def test_brute_force_decimal_mutual():
+    getcontext().prec = 50
+    b = tiny_batch(B=2, segs=1, P=(4, 3), R=2, M=(2, 2), H1=2, d1=4, stage1="mutual", seed=16)
+    m = b["meta"]
+    s1, ref1 = O.stage1_mutual(b["Q1"], b["K1"], m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"])
+    bs1, bref = _brute_stage1_mutual(_lists(b["Q1"]), _lists(b["K1"]), m["seg_off_host"].tolist(),
+                                     m["reg_idx_host"].tolist(), m["reg_off_host"].tolist())
+    np.testing.assert_allclose(s1, [float(x) for x in bs1], rtol=1e-14)
+    np.testing.assert_allclose(ref1, [float(x) for x in bref], rtol=1e-14)
+
+
+def test_head_reduce_reading_differs_from_alternative():
+    """The 'max over (text, head)' reading is a different function (flag works)."""
+    b = tiny_batch(B=1, segs=2, P=(8,), R=2, M=(5,), H2=4, seed=17)
+    a = O.prune(b, 0.0, 1.0)
+    c = O.prune(b, 0.0, 1.0, head_reduce="max")
+    vis = ~a["is_reg"]
+    assert (c["s2"][vis] >= a["s2"][vis] - 1e-15).all()
+    assert (c["s2"][vis] > a["s2"][vis] * (1 + 1e-6)).any()
