@@ -1,0 +1,450 @@
+"""Throughput of the OccamToken prune path (score -> threshold -> compact).
+
+One step = one fused occam_prune call (Stage-I [CLS] scores and threshold,
+Stage-II text scores and threshold, compaction and gather of the kept hidden /
+K / V rows) over one batch of the LLaVA-NeXT-shaped workload: 64 images x
+5 crops x (576 visual + 4 register rows), text lengths 16..256, synthetic
+seeded inputs resident in HBM (about 5 GB per step: larger than L2, so no
+flush is needed between steps).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line. With N > 1 (torchrun) every rank runs an independent
+replica of the batch ("replicas only": samples are independent and nothing
+is exchanged); value = images processed by all ranks / max-over-ranks time.
+The reference arm (--impl reference) times the CPU oracle, as it stands, on a
+bounded sample of the same workload on this machine's host cores.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+WORKLOAD = "llavanext_b64"
+METRIC = "pruned images/sec (score+threshold+compact) at 1 GB300; achieved HBM GB/s vs peak"
+UNIT = "images/s"
+FALLBACK_HBM_GBS = 6800.0
+SPEC_HBM_GBS = 8000.0
+KERNEL_SOURCES = {
+    "stage1": "stage1.cu", "stage1_finalize": "stage1.cu", "s1_list_plan": "stage2.cu",
+    "stage2_stats": "stage2.cu", "stage2_scores": "stage2.cu", "scan": "compact.cu", "gather": "compact.cu",
+}
+
+
+# ----------------------------------------------------------------------------- helpers
+
+def _dist():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d.get("hbm_gbs", FALLBACK_HBM_GBS)), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """Samples SM clocks / throttle reasons with nvidia-smi while running."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict | None:
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _traffic_from_profiles(kernel: str):
+    """dram bytes per launch of `kernel` from a committed ncu summary, if the
+    kernel source is unchanged since it was taken; else None."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{WORKLOAD}.md")
+    if not os.path.exists(path):
+        return None
+    txt = open(path).read()
+    vals = {}
+    for line in txt.splitlines():
+        line = line.strip().strip("`")
+        if "=" in line and line.split("=")[0].strip() in ("dram_bytes_per_launch", "source_sha"):
+            k, v = line.split("=", 1)
+            vals[k.strip()] = v.strip()
+    if "dram_bytes_per_launch" not in vals or "source_sha" not in vals:
+        return None
+    src = os.path.join(ROOT, "paper_2605_29657_gb300", "csrc", KERNEL_SOURCES[kernel])
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    if sha != vals["source_sha"]:
+        return None
+    return float(vals["dram_bytes_per_launch"])
+
+
+def algorithmic_bytes(meta: dict, n1_total: int, kept_total: int) -> dict:
+    """Bytes each kernel must move per launch (what the method needs, not the
+    dense work it avoids), from this run's actual S1 sizes and kept rows."""
+    rows, S, T = meta["total_rows"], meta["S_tot"], meta["total_text"]
+    H1, d1, H2, d2, hid = meta["H1"], meta["d1"], meta["H2"], meta["d2"], meta["hidden"]
+    k1row = H1 * d1 * 2
+    k2row = H2 * d2 * 2
+    hrow = hid * 2                       # bytes of one hidden / V row (bf16)
+    b = {}
+    b["stage1"] = rows * k1row + 2 * S * k1row + rows * 8            # K1 once, q/k_cls, s1 write, s2 zero
+    b["stage1_finalize"] = rows * (4 + 1 + 1 + 4)                    # s1 read, role, keep1, list
+    b["s1_list_plan"] = n1_total * 8                                 # list copy
+    b["stage2_stats"] = n1_total * k2row + 2 * T * k2row + T * H2 * 8  # S1 keys, Q + K_text, stats
+    b["stage2_scores"] = n1_total * k2row + T * k2row + T * H2 * 8   # S1 keys, Q, stats
+    b["scan"] = rows * (1 + 1 + 4 + 1) + kept_total * 4              # keep1, role, s2, keep2, out_index
+    b["gather"] = kept_total * 2 * (2 * hrow + k2row)                # read + write hidden, K, V rows
+    # whole step, each byte once: K1, S1 keys, text Q/K, hidden+V of kept rows
+    # (their K rows were read for scoring), writes of the 3 gathered rows
+    step = (rows * k1row + 2 * S * k1row + n1_total * k2row + 2 * T * k2row
+            + kept_total * (2 * hrow) + kept_total * (2 * hrow + k2row) + rows + kept_total * 4)
+    b["step"] = step
+    return b
+
+
+def aggregate(ms_local: float, images_local: int, device=None):
+    """Max of the timed milliseconds and sum of the images over all ranks
+    (replicas: nothing else is exchanged)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms_local], dtype=torch.float64, device=device)
+    n = torch.tensor([images_local], dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t.item()), int(n.item())
+
+
+# ----------------------------------------------------------------------------- CPU oracle (baseline / reference arm)
+
+def _oracle_worker(args):
+    """Generates its own samples of the workload (untimed), then times the
+    oracle on them. Runs in a spawned process with single-threaded BLAS."""
+    seeds, = args
+    sys.path.insert(0, ROOT)
+    from oracle import occam_oracle as O
+    from synth import get_config, make_batch
+    w = get_config(WORKLOAD)
+    one = get_config(WORKLOAD, B=1)
+    batches = [make_batch(one, seed=int(s)) for s in seeds]
+    t0 = time.perf_counter()
+    for b in batches:
+        O.prune(b, w.lambda1, w.lambda2)
+    return time.perf_counter() - t0, len(batches)
+
+
+def oracle_throughput(n_workers: int, samples_per_worker: int, seed0: int, pool=None) -> dict:
+    import multiprocessing as mp
+    own = pool is None
+    if own:
+        pool = _make_pool(n_workers)
+    jobs = [([seed0 + 1000 + i * samples_per_worker + k for k in range(samples_per_worker)],)
+            for i in range(n_workers)]
+    res = pool.map(_oracle_worker, jobs)
+    if own:
+        pool.close()
+        pool.join()
+    wall = max(t for t, _ in res)
+    n = sum(k for _, k in res)
+    del mp
+    return {"value": n / wall, "unit": UNIT, "cores": n_workers, "kind": "oracle",
+            "sample": f"{n} samples of the {WORKLOAD} workload (each: 5 crops x 580 rows, text 16..256), "
+                      f"{samples_per_worker} per worker on {n_workers} single-threaded workers; "
+                      f"value = samples / slowest worker's oracle time",
+            "seconds": wall}
+
+
+def _make_pool(n):
+    import multiprocessing as mp
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[k] = "1"
+    return mp.get_context("spawn").Pool(n)
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def run_ours(args, rank, world, local):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2605_29657_gb300 as occ
+    from synth import get_config, make_batch
+
+    # host-core oracle pool first: spawn, before the first GPU call
+    n_workers = min(16, os.cpu_count() or 1)
+    pool = _make_pool(n_workers) if (rank == 0 and not args.no_cpu_baseline) else None
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    w = get_config(WORKLOAD)
+    batch = make_batch(w, device=dev, seed=w.seed + 0)  # every rank: its own replica of the batch
+    meta = batch["meta"]
+    layout = occ.BatchLayout.from_batch(batch, dev)
+    K2flat = batch["K2"].view(batch["K2"].shape[0], -1)
+    gather = (batch["hidden"], K2flat, batch["V"])
+    call = occ.PruneCall(layout, dict(mode="cls", q=batch["q_cls"], k_cls=batch["k_cls"], K1=batch["K1"]),
+                         dict(Q_text=batch["Q_text"], K_text=batch["K_text"], K2=batch["K2"]),
+                         w.lambda1, w.lambda2, keep_registers=True, gather=gather)
+    stream = torch.cuda.current_stream()
+    nk = len(occ.PruneCall.TRACE_NAMES) + 1
+
+    for _ in range(args.warmup):
+        call()
+    torch.cuda.synchronize()
+    st = call.status()
+    if st != 0:
+        raise RuntimeError(f"device status {st} after warm-up")
+    out = call.out
+    n1_total = int(out["n1_vis"].sum().item()) + int(meta["regs_per_seg"] * meta["S_tot"])
+    kept_total = int(out["out_off"][-1].item())
+    bytes_ = algorithmic_bytes(meta, n1_total, kept_total)
+
+    # traced steps: a spread of the timed steps record per-kernel events
+    n_traced = min(args.steps, 400)
+    traced_at = set(np.linspace(0, args.steps - 1, n_traced).astype(int).tolist())
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(n_traced)]
+    for evs in events:
+        for e in evs:
+            e.record(stream)
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    ti = 0
+    for i in range(args.steps):
+        if i in traced_at:
+            call.traced(events[ti])
+            ti += 1
+        else:
+            call()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    ms = t_start.elapsed_time(t_end)
+    st = call.status()
+    if st != 0:
+        raise RuntimeError(f"device status {st} after the timed steps")
+    per_kernel = {}
+    for j, name in enumerate(occ.PruneCall.TRACE_NAMES):
+        per_kernel[name] = float(np.mean([evs[j].elapsed_time(evs[j + 1]) for evs in events]))
+
+    ms_max, images = aggregate(ms, meta["B"] * args.steps, dev)
+    value = images / (ms_max / 1e3)
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        names = ["q_cls", "k_cls", "K1", "Q_text", "K_text", "K2", "hidden", "V"]
+        host = {k: batch[k].cpu().pin_memory() for k in names}
+        res_names = ["count_vis", "count_out", "out_off", "out_index"]
+        res_host = {k: torch.empty_like(out[k], device="cpu").pin_memory() for k in res_names}
+        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        d2h = sum(t.numel() * t.element_size() for t in res_host.values())
+
+        def e2e_step():
+            for k in names:
+                batch[k].copy_(host[k], non_blocking=True)
+            call()
+            for k in res_names:
+                res_host[k].copy_(out[k], non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        e_steps = max(3, min(10, args.steps // 100))
+        if world > 1:
+            dist.barrier()
+        a = torch.cuda.Event(enable_timing=True)
+        z = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(e_steps):
+            e2e_step()
+        z.record(stream)
+        torch.cuda.synchronize()
+        ems, e_images = aggregate(a.elapsed_time(z), meta["B"] * e_steps, dev)
+        e2e = {"value": e_images / (ems / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": e_steps}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return None
+
+    peak, peak_kind = _peaks()
+    dom = max(per_kernel, key=per_kernel.get)
+    achieved = bytes_[dom] / (per_kernel[dom] / 1e3) / 1e9
+    traffic = _traffic_from_profiles(dom)
+    roofline = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": traffic, "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
+                if peak_kind == "measured" else "fallback 6.8 TB/s",
+                "algorithmic_bytes_per_launch": bytes_[dom], "avg_launch_ms": per_kernel[dom]}
+    step_ms = ms_max / args.steps
+    step_gbs = bytes_["step"] / (step_ms / 1e3) / 1e9
+    cpu = None
+    if pool is not None:
+        cpu = oracle_throughput(n_workers, 4, 0, pool=pool)
+        pool.close()
+        pool.join()
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {
+            "workload": WORKLOAD, "B": meta["B"], "crops": meta["segs_per_sample"], "visual_per_crop": 576,
+            "registers_per_crop": meta["regs_per_seg"], "text_tokens": "16..256 (uniform)",
+            "H1xd1": f"{meta['H1']}x{meta['d1']}", "H2xd2": f"{meta['H2']}x{meta['d2']}", "hidden": meta["hidden"],
+            "lambda1": w.lambda1, "lambda2": w.lambda2, "accumulate": "fp32",
+            "parallelism": "replicas" if world > 1 else "single",
+            "l2": "inputs larger than L2 (about 5 GB resident per step); no flush",
+            "mean_n1_vis": float(out["n1_vis"].float().mean().item()),
+            "mean_count_vis": float(out["count_vis"].float().mean().item()),
+            "kept_rows_per_step": kept_total,
+            "algorithmic_bytes_per_step": bytes_["step"],
+            "step_algorithmic_GBps": step_gbs,
+            "step_frac_of_measured_hbm": step_gbs / peak,
+            "step_frac_of_8TBps": step_gbs / SPEC_HBM_GBS,
+            "per_kernel_ms": per_kernel,
+        },
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": 7 * args.steps,
+        "clocks": clocks,
+    }
+    if world > 1:
+        dist.destroy_process_group()
+    return line
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    n_workers = min(16, os.cpu_count() or 1)
+    pool = _make_pool(n_workers)
+    for i in range(args.warmup):
+        oracle_throughput(n_workers, 1, 10_000 + i, pool=pool)
+    vals, secs = [], 0.0
+    n = 0
+    for i in range(args.steps):
+        r = oracle_throughput(n_workers, 1, 20_000 + i * n_workers, pool=pool)
+        secs += r["seconds"]
+        n += n_workers
+    pool.close()
+    pool.join()
+    value = n / secs
+    del vals
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "B_per_step": n_workers,
+                   "note": "the CPU oracle (numpy float64) timed as it stands on this machine's host cores"},
+        "cpu_baseline": {"kind": "oracle", "cores": n_workers, "value": value, "unit": UNIT,
+                         "sample": f"each step: {n_workers} samples of the {WORKLOAD} workload, one per "
+                                   f"single-threaded worker"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    rank, world, local = _dist()
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        import paper_2605_29657_gb300.build as pb
+        pb.build()
+        line = run_ours(args, rank, world, local)
+    if line is not None and rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

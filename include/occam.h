@@ -1,0 +1,226 @@
+/*
+ * occam.h -- C ABI of the OccamToken prune path on GB300 (sm_103a).
+ *
+ * OccamToken keeps a visual token v of sample x when its attention score is
+ * at least lambda times the score of a test-time register token r that takes
+ * part in the same softmax (Sec. 3.2, Eq. 3):
+ *
+ *   Stage I  (vision encoder):  s1(v) = A_{cls->v} averaged over heads
+ *            (Sec. 3.4, Eq. 4; App. A, Eq. 10), or, without [CLS], the mean
+ *            attention v receives from all rows (Sec. 3.4, Eq. 6; App. A,
+ *            Eq. 13); S1 = {v : s1(v) >= lambda1 s1(r)} u {r} (Eq. 5).
+ *   Stage II (LLM layer l):     s2(v) = max_j A_{t_j->v},
+ *            s2(r) = mean_j A_{t_j->r} (Sec. 3.5, Eq. 7; App. A, Eqs. 15-16);
+ *            S2 = {v in S1\{r} : s2(v) >= lambda2 s2(r)} u {r} (Eq. 8).
+ *   Decoding continues on [S2; T] (Algorithm 1), so the kept rows of the
+ *   hidden states and of the layer's K/V are compacted (App. A, Eq. 21).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every pointer argument (except the descriptor structs themselves, the
+ *   src/dst/row_bytes arrays of a gather list, and the status out-argument of
+ *   occam_get_status) is a DEVICE pointer owned by the caller. The library
+ *   allocates no memory: scratch space comes from the caller's `workspace`,
+ *   of at least occam_workspace_size() bytes, 256-byte aligned.
+ * - bf16 tensors are dense row-major: [rows, H, d] (K1, Q1, K2),
+ *   [segments, H, d] (q_cls, k_cls), [text, H, d] (Q_text, K_text).
+ *   Their base addresses must be 16-byte aligned and H*d*2 a multiple of 16.
+ * - Rows are numbered sample-major, segment-major: sample b owns rows
+ *   [row_off[b], row_off[b+1]), segment s owns rows [seg_off[s], seg_off[s+1]),
+ *   segments of one sample are consecutive and tile the sample's rows.
+ *   A segment is one encoder pass (an image, a crop, a video frame) with its
+ *   own [CLS] query, softmax and registers; register rows are listed per
+ *   segment in reg_idx[reg_off[s] .. reg_off[s+1]).
+ * - Calls are asynchronous on the caller's stream and never synchronise it.
+ *   Host-side argument checks return an error code at once and launch
+ *   nothing. Errors found on the device (a capacity overflow, an empty text
+ *   query, a bounded wait that ran out) are recorded in a status word inside
+ *   the workspace; occam_get_status() reads and clears it.
+ * - No C++ exception crosses this boundary.
+ */
+#ifndef OCCAM_H
+#define OCCAM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* occam_stream_t; /* a cudaStream_t; NULL = legacy default stream */
+
+/* Return / status codes. */
+enum {
+  OCCAM_OK = 0,
+  OCCAM_ERR_INVALID_ARG = 1, /* bad size, null pointer, misaligned tensor, M_b = 0, R = 0 */
+  OCCAM_ERR_CAPACITY = 2,    /* more kept rows than capacity_rows: rows past capacity are not written */
+  OCCAM_ERR_CUDA = 3,        /* a CUDA launch failed (cudaGetLastError) */
+  OCCAM_ERR_TIMEOUT = 4,     /* a bounded device-side wait gave up */
+  OCCAM_ERR_UNSUPPORTED = 5, /* head count / head dim / size outside what the kernels are built for */
+  OCCAM_ERR_WORKSPACE = 6    /* workspace null, too small or not 256-byte aligned */
+};
+
+enum { OCCAM_STAGE1_CLS = 0, OCCAM_STAGE1_MUTUAL = 1 };
+enum { OCCAM_REF_SEGMENT = 0, OCCAM_REF_SAMPLE = 1 };
+enum { OCCAM_TEXT_KEYS_CAUSAL = 0, OCCAM_TEXT_KEYS_NONE = 1 };
+
+#define OCCAM_MAX_GATHER 8
+
+/* Batch layout. The arrays are device copies; the scalars are host values
+ * that must agree with them (they size the launches and the workspace). */
+typedef struct occam_batch {
+  int32_t B;               /* samples */
+  int32_t S_tot;           /* segments over the batch */
+  int64_t total_rows;      /* visual + register rows over the batch (< 2^31) */
+  int64_t total_text;      /* text tokens over the batch (< 2^31) */
+  int32_t max_seg_rows;    /* max rows of one segment */
+  int32_t max_sample_rows; /* max rows of one sample */
+  int32_t max_text;        /* max text tokens of one sample */
+  int32_t max_regs;        /* max registers of one segment */
+  const int64_t* row_off;    /* [B+1]   rows of sample b: [row_off[b], row_off[b+1]) */
+  const int64_t* seg_off;    /* [S_tot+1] rows of segment s */
+  const int32_t* seg_first;  /* [B+1]   segments of sample b: [seg_first[b], seg_first[b+1]) */
+  const int32_t* seg_sample; /* [S_tot] sample of segment s */
+  const int32_t* reg_idx;    /* [reg_off[S_tot]] global row ids of the register rows */
+  const int32_t* reg_off;    /* [S_tot+1] registers of segment s: reg_idx[reg_off[s] .. reg_off[s+1]) */
+  const int64_t* text_off;   /* [B+1]   text tokens of sample b: [text_off[b], text_off[b+1]) */
+} occam_batch;
+
+/* Stage-I inputs (Sec. 3.4). CLS: q = q_cls [S_tot,H1,d1]; k_cls [S_tot,H1,d1]
+ * or NULL (the [CLS] key is then left out of the softmax). MUTUAL: q = Q1
+ * [rows,H1,d1], k_cls ignored. K1 [rows,H1,d1]. Built for H1 = 16 with
+ * d1 = 64 (CLS) and d1 in {64, 72, 80} (MUTUAL). */
+typedef struct occam_stage1_args {
+  int32_t mode; /* OCCAM_STAGE1_CLS or OCCAM_STAGE1_MUTUAL */
+  int32_t H1;
+  int32_t d1;
+  const void* q;
+  const void* k_cls;
+  const void* K1;
+} occam_stage1_args;
+
+/* Stage-II inputs (Sec. 3.5): layer-l queries and keys. Q_text [total_text,H2,d2];
+ * K_text [total_text,H2,d2] or NULL (= OCCAM_TEXT_KEYS_NONE: the text keys are
+ * left out of the softmax); K2 [rows,H2,d2], read only at S1 rows. Built for
+ * d2 = 128 and 1 <= H2 <= 64. */
+typedef struct occam_stage2_args {
+  int32_t H2;
+  int32_t d2;
+  const void* Q_text;
+  const void* K_text;
+  const void* K2;
+} occam_stage2_args;
+
+/* Size of the scratch workspace every entry point needs for this batch and
+ * these head counts. Returns OCCAM_OK and writes *bytes. */
+int occam_workspace_size(const occam_batch* batch, int32_t H1, int32_t H2, size_t* bytes);
+
+/* Reads and clears the device status word of `workspace` (synchronises
+ * `stream`). *status receives OCCAM_OK or the first device-side error code
+ * recorded since the last call. */
+int occam_get_status(void* workspace, int32_t* status, occam_stream_t stream);
+
+/* Stage-I scores (Sec. 3.4, Eqs. 4 and 6; App. A, Eqs. 10 and 13).
+ * s1 [total_rows] fp32: head-averaged attention each row receives;
+ * ref1 [S_tot] fp32: the mean of s1 over the segment's registers (the
+ * reference s1(r); with one register it is exactly the paper's). */
+int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, float* s1,
+                       float* ref1, void* workspace, size_t workspace_bytes, occam_stream_t stream);
+
+/* Register-anchored threshold (Eq. 3; Stage I Eq. 5, Stage II Eq. 8).
+ * keep[row] = 1 for a visual row with s[row] >= lambda * ref[unit(row)] and
+ * (prev_keep == NULL or prev_keep[row] != 0); unit = segment (ref_scope =
+ * OCCAM_REF_SEGMENT, ref [S_tot]) or sample (OCCAM_REF_SAMPLE, ref [B]).
+ * Register rows are not candidates: keep[reg] = keep_registers.
+ * count_vis [B] (int32, may be NULL) receives the kept visual rows per sample. */
+int occam_threshold(const occam_batch* batch, const float* s, const float* ref, int32_t ref_scope,
+                    float lambda, const uint8_t* prev_keep, int32_t keep_registers, uint8_t* keep,
+                    int32_t* count_vis, void* workspace, size_t workspace_bytes, occam_stream_t stream);
+
+/* Stage-II scores (Sec. 3.5, Eq. 7; App. A, Eqs. 15-16). keep1 [total_rows]
+ * u8 marks the visual rows of S1 (register rows are always in S1). For
+ * sample b and text token j, per head, the softmax runs over the S1 rows of
+ * b and the text keys 0..j (causal); the per-head probabilities are averaged
+ * over heads. s2 [total_rows] fp32 = max over j for visual S1 rows, 0 for
+ * every other row; ref2 [B] fp32 = the mean over the sample's registers of
+ * the mean over j. */
+int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, const uint8_t* keep1,
+                       float* s2, float* ref2, void* workspace, size_t workspace_bytes,
+                       occam_stream_t stream);
+
+/* Order-preserving stream compaction of the rows with keep[row] != 0
+ * (Algorithm 1: decoding continues on [S2; T]). out_index [capacity_rows]
+ * int32 receives the kept global row ids in ascending order (hence sample-
+ * major), count_out [B] int32 the kept rows per sample and out_off [B+1]
+ * int64 their exclusive prefix (out_off[B] = total kept). For each of the
+ * n_tensors gather tensors t (0 <= n_tensors <= OCCAM_MAX_GATHER; host arrays
+ * of device pointers), row out_off[b]+k of dst[t] becomes an exact copy of
+ * the k-th kept row of src[t]; row_bytes[t] is the row size (multiple of 16,
+ * pointers 16-byte aligned). If more than capacity_rows rows are kept,
+ * nothing is written past capacity_rows, the device status records
+ * OCCAM_ERR_CAPACITY, and counts and offsets are still exact. */
+int occam_compact(const occam_batch* batch, const uint8_t* keep, int32_t n_tensors,
+                  const void* const* src, const int64_t* row_bytes, void* const* dst,
+                  int64_t capacity_rows, int32_t* out_index, int32_t* count_out, int64_t* out_off,
+                  void* workspace, size_t workspace_bytes, occam_stream_t stream);
+
+/* The fused path: Stage-I scores -> Stage-I threshold (per segment,
+ * lambda1; registers always in S1) -> Stage-II scores over S1 -> Stage-II
+ * threshold (per sample, lambda2) -> compaction and gather. Per-sample
+ * budgets are outputs, never inputs (App. A: no hard token budget). */
+typedef struct occam_prune_args {
+  occam_batch batch;
+  occam_stage1_args stage1;
+  occam_stage2_args stage2;
+  float lambda1;
+  float lambda2;
+  int32_t keep_registers; /* 1: register rows are emitted (the paper keeps r); 0: visual rows only */
+  int32_t n_tensors;      /* gather list, as in occam_compact */
+  const void* src[OCCAM_MAX_GATHER];
+  int64_t row_bytes[OCCAM_MAX_GATHER];
+  void* dst[OCCAM_MAX_GATHER];
+  int64_t capacity_rows;
+} occam_prune_args;
+
+/* Outputs of occam_prune. Required: keep2 [total_rows] u8 (S2, registers =
+ * keep_registers), out_index [capacity_rows] int32, count_vis [B] int32
+ * (kept visual rows = the sample's budget |S2 \ {r}|), count_out [B] int32,
+ * out_off [B+1] int64. Optional (NULL to skip): keep1 [total_rows] u8 (S1,
+ * registers = 1), s1 [total_rows], ref1 [S_tot], s2 [total_rows], ref2 [B]
+ * (fp32), n1_vis [B] int32 (visual rows of S1). */
+typedef struct occam_prune_out {
+  uint8_t* keep2;
+  int32_t* out_index;
+  int32_t* count_vis;
+  int32_t* count_out;
+  int64_t* out_off;
+  uint8_t* keep1;
+  float* s1;
+  float* ref1;
+  float* s2;
+  float* ref2;
+  int32_t* n1_vis;
+} occam_prune_out;
+
+int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
+                size_t workspace_bytes, occam_stream_t stream);
+
+/* occam_prune that also records caller-created CUDA events (cudaEvent_t,
+ * passed as void*) on `stream` between its steps, for per-kernel timing:
+ * events[0] after the initial zeroing, then one after each kernel in launch
+ * order ([CLS] or mutual scoring, Stage-I finalize, S1 list + work plan,
+ * Stage-II statistics, Stage-II scores, compaction scan, gather). Mutual
+ * scoring is two kernels timed together. Extra events are left unrecorded;
+ * missing ones are skipped. Results are identical to occam_prune. */
+int occam_prune_traced(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
+                       size_t workspace_bytes, occam_stream_t stream, void* const* events, int32_t n_events);
+
+/* Library version string (static storage). */
+const char* occam_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OCCAM_H */

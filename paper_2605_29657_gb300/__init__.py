@@ -1,0 +1,28 @@
+"""OccamToken prune path for GB300 (sm_103a).
+
+Register-anchored relative evidence testing over visual tokens: Stage-I
+[CLS]/mutual scores, the per-segment register threshold, Stage-II text scores,
+the per-sample register threshold, and order-preserving compaction of the
+kept rows -- all in the CUDA kernels of liboccam.so, reached through its C ABI
+(include/occam.h). This package is the thin Python binding of that ABI.
+"""
+
+from ._lib import (  # noqa: F401
+    OCCAM_REF_SAMPLE,
+    OCCAM_REF_SEGMENT,
+    OCCAM_STAGE1_CLS,
+    OCCAM_STAGE1_MUTUAL,
+    BatchLayout,
+    OccamError,
+    PruneCall,
+    alloc_workspace,
+    library,
+    occam_compact,
+    occam_get_status,
+    occam_prune,
+    occam_score_stage1,
+    occam_score_stage2,
+    occam_threshold,
+    occam_version,
+    occam_workspace_size,
+)

@@ -1,0 +1,522 @@
+// api.cu -- the C ABI of include/occam.h: host-side validation, workspace
+// carve-up and kernel launches. Nothing here allocates memory.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <mutex>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+using namespace occam;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
+  WsLayout L{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + (bytes ? bytes : 1));
+    return o;
+  };
+  const int64_t rows = b->total_rows, S = b->S_tot, B = b->B, T = b->total_text;
+  L.status = take(4);
+  L.counters = take(CNT_SLOTS * 4);
+  L.role = take(rows);
+  L.keep1 = take(rows);
+  L.s1 = take(rows * 4);
+  L.s2 = take(rows * 4);
+  L.ref1 = take(S * 4);
+  L.s1_list = take(rows * 4);
+  L.n1_seg = take(S * 4);
+  L.dense = take(rows * 4);
+  L.n1 = take(B * 4);
+  L.n1_vis = take(B * 4);
+  const int64_t tps = cdiv(b->max_text, kTextTile);
+  const int64_t nhg = cdiv(H2 > 0 ? H2 : 1, kHeadGroup);
+  const int64_t chmax = cdiv(b->max_sample_rows, kKeyChunk);
+  L.maxA = B * tps * nhg;
+  L.maxB = B * tps * chmax;
+  L.itemsA = take(L.maxA * 16);
+  L.itemsB = take(L.maxB * 16);
+  L.itemB_off = take((B + 1) * 4);
+  L.stats2 = take(T * (H2 > 0 ? H2 : 1) * 8);
+  L.refpart = take(L.maxB * 4);
+  L.ref2 = take(B * 4);
+  L.tau2 = take(B * 4);
+  L.done = take(B * 4);
+  L.scan_tiles = cdiv(rows, kScanTile);
+  L.scan_state = take(L.scan_tiles * 8);
+  L.stats1_rows = rows;
+  L.stats1 = take(rows * (H1 > 0 ? H1 : 1) * 8);
+  L.total = off;
+  return L;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<unsigned char*>(ws) + off);
+}
+
+int check_batch(const occam_batch* b) {
+  if (!b) return OCCAM_ERR_INVALID_ARG;
+  if (b->B < 1 || b->S_tot < b->B || b->total_rows < 1 || b->total_rows >= (int64_t(1) << 31) ||
+      b->total_text < 0 || b->total_text >= (int64_t(1) << 31) || b->max_seg_rows < 1 ||
+      b->max_sample_rows < b->max_seg_rows || b->max_text < 0 || b->max_regs < 1)
+    return OCCAM_ERR_INVALID_ARG;
+  if (!b->row_off || !b->seg_off || !b->seg_first || !b->seg_sample || !b->reg_idx || !b->reg_off ||
+      !b->text_off)
+    return OCCAM_ERR_INVALID_ARG;
+  return OCCAM_OK;
+}
+
+int check_ws(const occam_batch* b, int H1, int H2, void* ws, size_t bytes, WsLayout* L) {
+  *L = ws_layout(b, H1, H2);
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0 || bytes < L->total)
+    return OCCAM_ERR_WORKSPACE;
+  return OCCAM_OK;
+}
+
+BatchDev dev_batch(const occam_batch* b) {
+  BatchDev d;
+  d.B = b->B;
+  d.S_tot = b->S_tot;
+  d.total_rows = b->total_rows;
+  d.total_text = b->total_text;
+  d.row_off = b->row_off;
+  d.seg_off = b->seg_off;
+  d.seg_first = b->seg_first;
+  d.seg_sample = b->seg_sample;
+  d.reg_idx = b->reg_idx;
+  d.reg_off = b->reg_off;
+  d.text_off = b->text_off;
+  return d;
+}
+
+int num_sms() {
+  static int n = 0;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  });
+  return n;
+}
+
+void set_smem_attrs() {
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaFuncSetAttribute(stage1_cls_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         stage1_cls_smem_bytes());
+    cudaFuncSetAttribute(s2_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_stats_smem_bytes());
+    cudaFuncSetAttribute(s2_scores_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_scores_smem_bytes());
+  });
+}
+
+int cuda_ok() {
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? OCCAM_OK : OCCAM_ERR_CUDA;
+}
+
+#define OCCAM_TRY(x)                \
+  do {                              \
+    int _rc = (x);                  \
+    if (_rc != OCCAM_OK) return _rc; \
+  } while (0)
+
+#define OCCAM_CUDA(x)                                    \
+  do {                                                   \
+    if ((x) != cudaSuccess) return OCCAM_ERR_CUDA;       \
+  } while (0)
+
+int check_stage1(const occam_batch* b, const occam_stage1_args* a) {
+  if (!a || !a->q || !a->K1) return OCCAM_ERR_INVALID_ARG;
+  if (!aligned16(a->q) || !aligned16(a->K1) || (a->k_cls && !aligned16(a->k_cls))) return OCCAM_ERR_INVALID_ARG;
+  if (a->mode == OCCAM_STAGE1_CLS) {
+    if (a->H1 != 16 || a->d1 != 64) return OCCAM_ERR_UNSUPPORTED;
+    if (b->max_seg_rows > kMaxClusterCls * kMaxClsRowsPerCta) return OCCAM_ERR_UNSUPPORTED;
+  } else if (a->mode == OCCAM_STAGE1_MUTUAL) {
+    if (a->H1 < 1 || a->H1 > 64) return OCCAM_ERR_UNSUPPORTED;
+    if (a->d1 != 64 && a->d1 != 72 && a->d1 != 80) return OCCAM_ERR_UNSUPPORTED;
+    if (b->max_seg_rows > 65535 * kMutQTile) return OCCAM_ERR_UNSUPPORTED;
+  } else {
+    return OCCAM_ERR_INVALID_ARG;
+  }
+  return OCCAM_OK;
+}
+
+int check_stage2(const occam_stage2_args* a) {
+  if (!a || !a->Q_text || !a->K2) return OCCAM_ERR_INVALID_ARG;
+  if (a->d2 != 128 || a->H2 < 1 || a->H2 > 64) return OCCAM_ERR_UNSUPPORTED;
+  if (!aligned16(a->Q_text) || !aligned16(a->K2) || (a->K_text && !aligned16(a->K_text)))
+    return OCCAM_ERR_INVALID_ARG;
+  return OCCAM_OK;
+}
+
+int check_gather(int n, const void* const* src, const int64_t* rb, void* const* dst) {
+  if (n < 0 || n > OCCAM_MAX_GATHER) return OCCAM_ERR_INVALID_ARG;
+  for (int t = 0; t < n; ++t) {
+    if (!src || !dst || !rb || !src[t] || !dst[t] || rb[t] <= 0 || (rb[t] & 15) || !aligned16(src[t]) ||
+        !aligned16(dst[t]))
+      return OCCAM_ERR_INVALID_ARG;
+  }
+  return OCCAM_OK;
+}
+
+// Optional CUDA events recorded between the kernels of one call (for live
+// per-kernel timing by the caller). mark() records the next event, if any.
+struct Trace {
+  cudaEvent_t* ev = nullptr;
+  int n = 0;
+  int* next = nullptr;
+  void mark(cudaStream_t st) const {
+    if (ev && next && *next < n) cudaEventRecord(ev[(*next)++], st);
+  }
+};
+
+// ---------------------------------------------------------------- launch helpers
+
+int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const WsLayout& L, void* ws,
+                         float* s1, float* s2_zero, cudaStream_t st, Trace trace = Trace()) {
+  const BatchDev bt = dev_batch(b);
+  int* status = at<int>(ws, L.status);
+  if (a->mode == OCCAM_STAGE1_CLS) {
+    Stage1ClsParams p;
+    p.bt = bt;
+    p.q_cls = static_cast<const __nv_bfloat16*>(a->q);
+    p.k_cls = static_cast<const __nv_bfloat16*>(a->k_cls);
+    p.K1 = static_cast<const __nv_bfloat16*>(a->K1);
+    p.scale = (float)(1.0 / std::sqrt((double)a->d1));
+    p.s1 = s1;
+    p.s2_zero = s2_zero;
+    p.status = status;
+    int C = (int)cdiv(b->max_seg_rows, 160);
+    C = C < 1 ? 1 : (C > kMaxClusterCls ? kMaxClusterCls : C);
+    while (cdiv(b->max_seg_rows, C) > kMaxClsRowsPerCta && C < kMaxClusterCls) ++C;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(b->S_tot * C));
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = stage1_cls_smem_bytes();
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    OCCAM_CUDA(cudaLaunchKernelEx(&cfg, stage1_cls_kernel, p));
+    trace.mark(st);
+  } else {
+    MutualParams p;
+    p.bt = bt;
+    p.H = a->H1;
+    p.Q = static_cast<const __nv_bfloat16*>(a->q);
+    p.K = static_cast<const __nv_bfloat16*>(a->K1);
+    p.scale = (float)(1.0 / std::sqrt((double)a->d1));
+    p.stats = at<float2>(ws, L.stats1);
+    p.s1 = s1;
+    p.s2_zero = s2_zero;
+    launch_mutual(p, a->d1, b->S_tot, b->max_seg_rows, st);
+    trace.mark(st);
+  }
+  return cuda_ok();
+}
+
+int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, const float* s1, const uint8_t* keep_in,
+                     float lambda1, int do_threshold, float* ref1, uint8_t* keep1, int32_t* n1_vis,
+                     cudaStream_t st, Trace trace = Trace()) {
+  Stage1FinalizeParams p;
+  p.bt = dev_batch(b);
+  p.s1 = s1;
+  p.keep_in = keep_in;
+  p.lambda1 = lambda1;
+  p.do_threshold = do_threshold;
+  p.ref1 = ref1;
+  p.role = at<uint8_t>(ws, L.role);
+  p.keep1 = keep1;
+  p.s1_list = at<int32_t>(ws, L.s1_list);
+  p.n1_seg = at<int32_t>(ws, L.n1_seg);
+  p.n1_vis = n1_vis;
+  p.status = at<int>(ws, L.status);
+  stage1_finalize_kernel<<<b->S_tot, 256, 0, st>>>(p);
+  trace.mark(st);
+  return cuda_ok();
+}
+
+int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayout& L, void* ws, float* s2,
+                  float* ref2, float lambda2, cudaStream_t st, Trace trace = Trace()) {
+  Stage2Params p;
+  p.bt = dev_batch(b);
+  p.H = a->H2;
+  p.Q = static_cast<const __nv_bfloat16*>(a->Q_text);
+  p.Kt = static_cast<const __nv_bfloat16*>(a->K_text);
+  p.K = static_cast<const __nv_bfloat16*>(a->K2);
+  p.scale = (float)(1.0 / std::sqrt((double)a->d2));
+  p.role = at<uint8_t>(ws, L.role);
+  p.s1_list = at<int32_t>(ws, L.s1_list);
+  p.n1_seg = at<int32_t>(ws, L.n1_seg);
+  p.dense = at<int32_t>(ws, L.dense);
+  p.n1 = at<int32_t>(ws, L.n1);
+  p.itemsA = at<int4>(ws, L.itemsA);
+  p.itemsB = at<int4>(ws, L.itemsB);
+  p.itemB_off = at<int32_t>(ws, L.itemB_off);
+  p.counters = at<int32_t>(ws, L.counters);
+  p.maxA = L.maxA;
+  p.maxB = L.maxB;
+  p.stats = at<float2>(ws, L.stats2);
+  p.s2 = s2;
+  p.refpart = at<float>(ws, L.refpart);
+  p.done = at<int32_t>(ws, L.done);
+  p.ref2 = ref2;
+  p.tau2 = at<float>(ws, L.tau2);
+  p.lambda2 = lambda2;
+  p.status = at<int>(ws, L.status);
+  s2_dense_plan_kernel<<<b->B, 256, 0, st>>>(p, 1);
+  trace.mark(st);
+  const int sms = num_sms();
+  const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);
+  const int gB = (int)std::min<int64_t>(L.maxB, sms);
+  if (gA > 0) s2_stats_kernel<<<gA, 128, s2_stats_smem_bytes(), st>>>(p);
+  trace.mark(st);
+  if (gB > 0) s2_scores_kernel<<<gB, 256, s2_scores_smem_bytes(), st>>>(p);
+  trace.mark(st);
+  return cuda_ok();
+}
+
+int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, const uint8_t* keep_in,
+                   const uint8_t* keep1, const float* s2, int keep_registers, uint8_t* keep_out, int n_tensors,
+                   const void* const* src, const int64_t* row_bytes, void* const* dst, int64_t capacity,
+                   int32_t* out_index, int32_t* count_out, int32_t* count_vis, int64_t* out_off,
+                   cudaStream_t st, bool do_memsets = true, Trace trace = Trace()) {
+  ScanParams p;
+  p.bt = dev_batch(b);
+  p.mode = mode;
+  p.keep_in = keep_in;
+  p.role = (mode == 1) ? at<uint8_t>(ws, L.role) : nullptr;
+  p.keep1 = keep1;
+  p.s2 = s2;
+  p.tau2 = at<float>(ws, L.tau2);
+  p.keep_registers = keep_registers;
+  p.keep_out = keep_out;
+  p.capacity = capacity;
+  p.out_index = out_index;
+  p.count_out = count_out;
+  p.count_vis = count_vis;
+  p.out_off = out_off;
+  p.tile_state = at<unsigned long long>(ws, L.scan_state);
+  p.ticket = at<int32_t>(ws, L.counters) + CNT_SCAN_TICKET;
+  p.ntiles = L.scan_tiles;
+  p.status = at<int>(ws, L.status);
+  if (do_memsets) {
+    OCCAM_CUDA(cudaMemsetAsync(p.tile_state, 0, L.scan_tiles * 8, st));
+    OCCAM_CUDA(cudaMemsetAsync(p.ticket, 0, 4, st));
+    OCCAM_CUDA(cudaMemsetAsync(count_out, 0, b->B * 4, st));
+    if (count_vis) OCCAM_CUDA(cudaMemsetAsync(count_vis, 0, b->B * 4, st));
+  }
+  scan_kernel<<<(unsigned)L.scan_tiles, 256, 0, st>>>(p);
+  trace.mark(st);
+  if (n_tensors > 0) {
+    GatherParams g;
+    g.n_tensors = n_tensors;
+    for (int t = 0; t < OCCAM_MAX_GATHER; ++t) {
+      g.src[t] = t < n_tensors ? static_cast<const unsigned char*>(src[t]) : nullptr;
+      g.dst[t] = t < n_tensors ? static_cast<unsigned char*>(dst[t]) : nullptr;
+      g.row_bytes[t] = t < n_tensors ? row_bytes[t] : 0;
+    }
+    g.out_index = out_index;
+    g.out_off = out_off;
+    g.B = b->B;
+    g.capacity = capacity;
+    gather_kernel<<<num_sms() * 4, 256, 0, st>>>(g);
+  }
+  trace.mark(st);
+  return cuda_ok();
+}
+
+int mark_roles(const occam_batch* b, const WsLayout& L, void* ws, cudaStream_t st) {
+  uint8_t* role = at<uint8_t>(ws, L.role);
+  OCCAM_CUDA(cudaMemsetAsync(role, 0, b->total_rows, st));
+  roles_scatter_kernel<<<64, 256, 0, st>>>(dev_batch(b), role);
+  return cuda_ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* occam_version(void) { return "occam-gb300 0.1 (sm_103a)"; }
+
+int occam_workspace_size(const occam_batch* batch, int32_t H1, int32_t H2, size_t* bytes) {
+  OCCAM_TRY(check_batch(batch));
+  if (!bytes) return OCCAM_ERR_INVALID_ARG;
+  *bytes = ws_layout(batch, H1, H2).total;
+  return OCCAM_OK;
+}
+
+int occam_get_status(void* workspace, int32_t* status, occam_stream_t stream) {
+  if (!workspace || !status) return OCCAM_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int32_t v = 0;
+  OCCAM_CUDA(cudaMemcpyAsync(&v, workspace, 4, cudaMemcpyDeviceToHost, st));
+  OCCAM_CUDA(cudaMemsetAsync(workspace, 0, 4, st));
+  OCCAM_CUDA(cudaStreamSynchronize(st));
+  *status = v;
+  return OCCAM_OK;
+}
+
+int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, float* s1, float* ref1,
+                       void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  OCCAM_TRY(check_batch(batch));
+  OCCAM_TRY(check_stage1(batch, args));
+  if (!s1) return OCCAM_ERR_INVALID_ARG;
+  WsLayout L;
+  OCCAM_TRY(check_ws(batch, args->H1, 1, workspace, workspace_bytes, &L));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  set_smem_attrs();
+  OCCAM_TRY(launch_stage1_scores(batch, args, L, workspace, s1, nullptr, st));
+  OCCAM_TRY(launch_finalize1(batch, L, workspace, s1, nullptr, 0.f, 0, ref1, nullptr, nullptr, st));
+  return OCCAM_OK;
+}
+
+int occam_threshold(const occam_batch* batch, const float* s, const float* ref, int32_t ref_scope, float lambda,
+                    const uint8_t* prev_keep, int32_t keep_registers, uint8_t* keep, int32_t* count_vis,
+                    void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  OCCAM_TRY(check_batch(batch));
+  if (!s || !ref || !keep) return OCCAM_ERR_INVALID_ARG;
+  if (ref_scope != OCCAM_REF_SEGMENT && ref_scope != OCCAM_REF_SAMPLE) return OCCAM_ERR_INVALID_ARG;
+  if (!(lambda == lambda)) return OCCAM_ERR_INVALID_ARG;
+  WsLayout L;
+  OCCAM_TRY(check_ws(batch, 1, 1, workspace, workspace_bytes, &L));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  OCCAM_TRY(mark_roles(batch, L, workspace, st));
+  if (count_vis) OCCAM_CUDA(cudaMemsetAsync(count_vis, 0, batch->B * 4, st));
+  ThresholdParams p;
+  p.bt = dev_batch(batch);
+  p.s = s;
+  p.ref = ref;
+  p.ref_scope = ref_scope;
+  p.lambda = lambda;
+  p.prev_keep = prev_keep;
+  p.keep_registers = keep_registers;
+  p.role = at<uint8_t>(workspace, L.role);
+  p.keep = keep;
+  p.count_vis = count_vis;
+  threshold_kernel<<<(unsigned)cdiv(batch->total_rows, 256), 256, 0, st>>>(p);
+  return cuda_ok();
+}
+
+int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, const uint8_t* keep1, float* s2,
+                       float* ref2, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  OCCAM_TRY(check_batch(batch));
+  OCCAM_TRY(check_stage2(args));
+  if (!keep1 || !s2 || !ref2) return OCCAM_ERR_INVALID_ARG;
+  WsLayout L;
+  OCCAM_TRY(check_ws(batch, 1, args->H2, workspace, workspace_bytes, &L));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  set_smem_attrs();
+  OCCAM_TRY(mark_roles(batch, L, workspace, st));
+  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(workspace, L.counters), 0, CNT_SLOTS * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(workspace, L.done), 0, batch->B * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(workspace, L.n1_vis), 0, batch->B * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(s2, 0, batch->total_rows * 4, st));
+  // S1 lists from the given mask (registers always in S1)
+  Stage1FinalizeParams f;
+  f.bt = dev_batch(batch);
+  f.s1 = nullptr;
+  f.keep_in = keep1;
+  f.lambda1 = 0.f;
+  f.do_threshold = 1;
+  f.ref1 = nullptr;
+  f.role = at<uint8_t>(workspace, L.role);
+  f.keep1 = nullptr;
+  f.s1_list = at<int32_t>(workspace, L.s1_list);
+  f.n1_seg = at<int32_t>(workspace, L.n1_seg);
+  f.n1_vis = at<int32_t>(workspace, L.n1_vis);
+  f.status = at<int>(workspace, L.status);
+  stage1_finalize_kernel<<<batch->S_tot, 256, 0, st>>>(f);
+  OCCAM_TRY(cuda_ok());
+  return launch_stage2(batch, args, L, workspace, s2, ref2, 1.0f, st);
+}
+
+int occam_compact(const occam_batch* batch, const uint8_t* keep, int32_t n_tensors, const void* const* src,
+                  const int64_t* row_bytes, void* const* dst, int64_t capacity_rows, int32_t* out_index,
+                  int32_t* count_out, int64_t* out_off, void* workspace, size_t workspace_bytes,
+                  occam_stream_t stream) {
+  OCCAM_TRY(check_batch(batch));
+  if (!keep || !count_out || !out_off || capacity_rows < 0 || (capacity_rows > 0 && !out_index))
+    return OCCAM_ERR_INVALID_ARG;
+  OCCAM_TRY(check_gather(n_tensors, src, row_bytes, dst));
+  WsLayout L;
+  OCCAM_TRY(check_ws(batch, 1, 1, workspace, workspace_bytes, &L));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  return launch_compact(batch, L, workspace, 0, keep, nullptr, nullptr, 0, nullptr, n_tensors, src, row_bytes,
+                        dst, capacity_rows, out_index, count_out, nullptr, out_off, st);
+}
+
+static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
+                      size_t workspace_bytes, occam_stream_t stream, Trace trace) {
+  if (!args || !out) return OCCAM_ERR_INVALID_ARG;
+  const occam_batch* b = &args->batch;
+  OCCAM_TRY(check_batch(b));
+  OCCAM_TRY(check_stage1(b, &args->stage1));
+  OCCAM_TRY(check_stage2(&args->stage2));
+  OCCAM_TRY(check_gather(args->n_tensors, args->src, args->row_bytes, args->dst));
+  if (!out->keep2 || !out->count_vis || !out->count_out || !out->out_off || args->capacity_rows < 0 ||
+      (args->capacity_rows > 0 && !out->out_index))
+    return OCCAM_ERR_INVALID_ARG;
+  if (!(args->lambda1 == args->lambda1) || !(args->lambda2 == args->lambda2)) return OCCAM_ERR_INVALID_ARG;
+  WsLayout L;
+  OCCAM_TRY(check_ws(b, args->stage1.H1, args->stage2.H2, workspace, workspace_bytes, &L));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  set_smem_attrs();
+  void* ws = workspace;
+  float* s1 = out->s1 ? out->s1 : at<float>(ws, L.s1);
+  float* s2 = out->s2 ? out->s2 : at<float>(ws, L.s2);
+  uint8_t* keep1 = out->keep1 ? out->keep1 : at<uint8_t>(ws, L.keep1);
+  int32_t* n1_vis = out->n1_vis ? out->n1_vis : at<int32_t>(ws, L.n1_vis);
+  float* ref2 = out->ref2 ? out->ref2 : at<float>(ws, L.ref2);
+  // every zero-initialised accumulator of the call, up front
+  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(ws, L.counters), 0, CNT_SLOTS * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(ws, L.done), 0, b->B * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(n1_vis, 0, b->B * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(at<unsigned long long>(ws, L.scan_state), 0, L.scan_tiles * 8, st));
+  OCCAM_CUDA(cudaMemsetAsync(out->count_out, 0, b->B * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(out->count_vis, 0, b->B * 4, st));
+  trace.mark(st);
+  OCCAM_TRY(launch_stage1_scores(b, &args->stage1, L, ws, s1, s2, st, trace));
+  OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, st, trace));
+  OCCAM_TRY(launch_stage2(b, &args->stage2, L, ws, s2, ref2, args->lambda2, st, trace));
+  return launch_compact(b, L, ws, 1, nullptr, keep1, s2, args->keep_registers, out->keep2, args->n_tensors,
+                        args->src, args->row_bytes, args->dst, args->capacity_rows, out->out_index,
+                        out->count_out, out->count_vis, out->out_off, st, false, trace);
+}
+
+int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
+                size_t workspace_bytes, occam_stream_t stream) {
+  return prune_impl(args, out, workspace, workspace_bytes, stream, Trace());
+}
+
+int occam_prune_traced(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
+                       size_t workspace_bytes, occam_stream_t stream, void* const* events, int32_t n_events) {
+  if (n_events < 0 || (n_events > 0 && !events)) return OCCAM_ERR_INVALID_ARG;
+  int next = 0;
+  Trace t;
+  t.ev = reinterpret_cast<cudaEvent_t*>(const_cast<void**>(events));
+  t.n = n_events;
+  t.next = &next;
+  return prune_impl(args, out, workspace, workspace_bytes, stream, t);
+}
+
+}  // extern "C"

@@ -1,0 +1,141 @@
+// kernels.cuh -- kernel parameter blocks and declarations (internal).
+#pragma once
+
+#include "common.cuh"
+
+namespace occam {
+
+constexpr int kMaxClsRowsPerCta = 512;  // rows of one segment handled by one CTA of a [CLS] cluster
+constexpr int kMaxClusterCls = 8;       // portable cluster size
+
+struct Stage1ClsParams {
+  BatchDev bt;
+  const __nv_bfloat16* q_cls;
+  const __nv_bfloat16* k_cls;  // nullable
+  const __nv_bfloat16* K1;
+  float scale;
+  float* s1;
+  float* s2_zero;  // nullable: zeroed per row (Stage-II max accumulator)
+  int* status;
+};
+
+struct Stage1FinalizeParams {
+  BatchDev bt;
+  const float* s1;          // nullable when keep_in is given
+  const uint8_t* keep_in;   // nullable: S1 membership of visual rows given instead of tested
+  float lambda1;
+  int do_threshold;
+  float* ref1;       // nullable
+  uint8_t* role;
+  uint8_t* keep1;
+  int32_t* s1_list;  // per segment, at seg_off[s]
+  int32_t* n1_seg;
+  int32_t* n1_vis;   // [B], accumulated
+  int* status;
+};
+
+struct MutualParams {
+  BatchDev bt;
+  int H;
+  const __nv_bfloat16* Q;
+  const __nv_bfloat16* K;
+  float scale;
+  float2* stats;  // [rows, H] (max in log2 units, 1/sum)
+  float* s1;
+  float* s2_zero;
+};
+
+struct ThresholdParams {
+  BatchDev bt;
+  const float* s;
+  const float* ref;
+  int ref_scope;
+  float lambda;
+  const uint8_t* prev_keep;
+  int keep_registers;
+  const uint8_t* role;
+  uint8_t* keep;
+  int32_t* count_vis;
+};
+
+struct Stage2Params {
+  BatchDev bt;
+  int H;  // H2, d2 = 128
+  const __nv_bfloat16* Q;   // [total_text, H, 128]
+  const __nv_bfloat16* Kt;  // nullable
+  const __nv_bfloat16* K;   // [rows, H, 128]
+  float scale;
+  const uint8_t* role;
+  const int32_t* s1_list;   // per segment lists
+  const int32_t* n1_seg;
+  int32_t* dense;           // per sample dense S1 list at row_off[b]
+  int32_t* n1;              // [B]
+  int4* itemsA;             // (b, j0, head group, -)
+  int4* itemsB;             // (b, j0, key chunk, item index within sample)
+  int32_t* itemB_off;       // [B+1]
+  int32_t* counters;
+  int64_t maxA, maxB;
+  float2* stats;            // [total_text, H] (max in log2 units, 1/sum)
+  float* s2;                // atomicMax accumulator, zeroed beforehand
+  float* refpart;           // [maxB]
+  int32_t* done;            // [B] finished score items per sample (zeroed)
+  float* ref2;              // [B]
+  float* tau2;              // [B]
+  float lambda2;
+  int* status;
+};
+
+struct ScanParams {
+  BatchDev bt;
+  int mode;                  // 0: keep from `keep_in`; 1: fused Stage-II threshold
+  const uint8_t* keep_in;
+  const uint8_t* role;
+  const uint8_t* keep1;
+  const float* s2;
+  const float* tau2;
+  int keep_registers;
+  uint8_t* keep_out;         // nullable
+  int64_t capacity;
+  int32_t* out_index;
+  int32_t* count_out;        // [B] accumulated (zeroed)
+  int32_t* count_vis;        // [B] accumulated (zeroed), nullable
+  int64_t* out_off;          // [B+1]
+  unsigned long long* tile_state;
+  int32_t* ticket;
+  int64_t ntiles;
+  int* status;
+};
+
+struct GatherParams {
+  int n_tensors;
+  const unsigned char* src[OCCAM_MAX_GATHER];
+  unsigned char* dst[OCCAM_MAX_GATHER];
+  int64_t row_bytes[OCCAM_MAX_GATHER];
+  const int32_t* out_index;
+  const int64_t* out_off;    // total kept = out_off[B]
+  int B;
+  int64_t capacity;
+};
+
+// stage1.cu
+__global__ void stage1_cls_kernel(Stage1ClsParams p);
+int stage1_cls_smem_bytes();
+__global__ void stage1_finalize_kernel(Stage1FinalizeParams p);
+int mutual_colsum_smem_bytes(int DP);
+void launch_mutual(const MutualParams& p, int d1, int S_tot, int max_seg_rows, cudaStream_t st);
+__global__ void roles_scatter_kernel(BatchDev bt, uint8_t* role);
+__global__ void threshold_kernel(ThresholdParams p);
+
+// stage2.cu
+__global__ void s2_dense_plan_kernel(Stage2Params p, int build_dense);
+__global__ void s2_stats_kernel(Stage2Params p);
+__global__ void s2_scores_kernel(Stage2Params p);
+int s2_scores_smem_bytes();
+int s2_stats_smem_bytes();
+
+// compact.cu
+__global__ void scan_kernel(ScanParams p);
+__global__ void gather_kernel(GatherParams p);
+__global__ void offsets_fix_kernel(ScanParams p);
+
+}  // namespace occam

@@ -1,0 +1,363 @@
+// stage2.cu -- Stage II of OccamToken (Sec. 3.5): text-to-vision scores at
+// LLM layer l. For sample b and text token j, per head h, the softmax runs
+// over the S1 rows of b (visual survivors and registers) and the text keys
+// 0..j; p[j, v] is the per-head probability averaged over heads;
+// s2(v) = max_j p[j, v], s2(r) = mean over registers and over j (Eq. 7;
+// App. A, Eqs. 15-16), and tau2 = lambda2 * s2(r) (Eq. 8).
+//
+// Work is split in two passes so that any S1 size and any text length fit:
+//   stats  (item = sample, 64 text rows, 8 heads): per (j, h) the softmax
+//          max and sum over all keys, online over 64-key chunks;
+//   scores (item = sample, 64 text rows, 128 S1 keys): for every head the
+//          probabilities of the chunk's keys, accumulated over heads in
+//          registers, then the column max over j (atomicMax on the fp32 bit
+//          pattern -- exact and order-free because p >= 0) and the
+//          registers' column sums (written per item and reduced in a fixed
+//          order by the sample's last item, so ref2 is deterministic).
+// QK^T runs on the tensor cores (mma.sync m16n8k16, bf16 in, fp32
+// accumulate); operands are staged in shared memory by cp.async.
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace occam {
+
+namespace s2k {
+constexpr int D = 128;
+constexpr int LD = D + 8;  // padded smem row (272 B): conflict-free ldmatrix
+constexpr int KT = 64;     // keys per stats chunk
+}  // namespace s2k
+
+// ---------------------------------------------------------------------------
+// Dense per-sample S1 lists + work plan. Grid: one CTA per sample; the last
+// CTA to finish builds the item lists of both passes.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) s2_dense_plan_kernel(Stage2Params p, int build_dense) {
+  __shared__ int tmp[40];
+  __shared__ int is_last;
+  const int b = blockIdx.x, tid = threadIdx.x;
+  if (build_dense) {
+    const int sf = p.bt.seg_first[b], sl = p.bt.seg_first[b + 1];
+    const int64_t rbase = p.bt.row_off[b];
+    int base = 0;
+    for (int s = sf; s < sl; ++s) {
+      const int cnt = p.n1_seg[s];
+      const int64_t so = p.bt.seg_off[s];
+      for (int k = tid; k < cnt; k += blockDim.x) p.dense[rbase + base + k] = p.s1_list[so + k];
+      base += cnt;
+    }
+    if (tid == 0) p.n1[b] = base;
+  }
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) is_last = (atomicAdd(&p.counters[CNT_DENSE_DONE], 1) == (int)gridDim.x - 1);
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
+  int runA = 0, runB = 0;
+  for (int b0 = 0; b0 < p.bt.B; b0 += blockDim.x) {
+    const int bb = b0 + tid;
+    int nA = 0, nB = 0, tiles = 0, nch = 0;
+    if (bb < p.bt.B) {
+      const int M = (int)(p.bt.text_off[bb + 1] - p.bt.text_off[bb]);
+      const int n1 = *((volatile int32_t*)&p.n1[bb]);
+      tiles = (M + kTextTile - 1) / kTextTile;
+      nch = (n1 + kKeyChunk - 1) / kKeyChunk;
+      nA = tiles * nhg;
+      nB = tiles * nch;
+      if (M == 0) {
+        set_status(p.status, OCCAM_ERR_INVALID_ARG);
+        p.ref2[bb] = 0.f;
+        p.tau2[bb] = 0.f;
+      }
+    }
+    int totA, totB;
+    const int offA = runA + block_exclusive_scan(nA, tmp, &totA);
+    const int offB = runB + block_exclusive_scan(nB, tmp, &totB);
+    if (bb < p.bt.B) {
+      for (int i = 0; i < nA; ++i)
+        if (offA + i < p.maxA) p.itemsA[offA + i] = make_int4(bb, (i / nhg) * kTextTile, i % nhg, 0);
+      for (int i = 0; i < nB; ++i)
+        if (offB + i < p.maxB) p.itemsB[offB + i] = make_int4(bb, (i / nch) * kTextTile, i % nch, i);
+      p.itemB_off[bb] = offB;
+    }
+    runA += totA;
+    runB += totB;
+  }
+  if (tid == 0) {
+    p.itemB_off[p.bt.B] = runB;
+    if (runA > p.maxA || runB > p.maxB) set_status(p.status, OCCAM_ERR_CAPACITY);
+    p.counters[CNT_NA] = (int)(runA < p.maxA ? runA : p.maxA);
+    p.counters[CNT_NB] = (int)(runB < p.maxB ? runB : p.maxB);
+  }
+}
+
+// copy one 64- or 128-key chunk of head h into sdst[key][0..128) (stride LD)
+__device__ __forceinline__ void s2_load_keys(__nv_bfloat16* sdst, const Stage2Params& p, int b, int64_t t0,
+                                             int n_img, int total, int k0, int nkeys_tile, int h, int tid,
+                                             int nthreads) {
+  using namespace s2k;
+  const int64_t rbase = p.bt.row_off[b];
+  const int64_t HD = (int64_t)p.H * D;
+  for (int i = tid; i < nkeys_tile * 16; i += nthreads) {
+    const int kr = i >> 4, v = i & 15;
+    const int kk = k0 + kr;
+    const __nv_bfloat16* src = p.K;
+    int bytes = 0;
+    if (kk < n_img) {
+      src = p.K + (int64_t)p.dense[rbase + kk] * HD + (int64_t)h * D + v * 8;
+      bytes = 16;
+    } else if (kk < total) {
+      src = p.Kt + (t0 + (kk - n_img)) * HD + (int64_t)h * D + v * 8;
+      bytes = 16;
+    }
+    cp_async16_zfill(sdst + kr * LD + v * 8, src, bytes);
+  }
+}
+
+__device__ __forceinline__ void s2_load_queries(__nv_bfloat16* sdst, const Stage2Params& p, int64_t trow0,
+                                                int nq, int h, int tid, int nthreads) {
+  using namespace s2k;
+  const int64_t HD = (int64_t)p.H * D;
+  for (int i = tid; i < kTextTile * 16; i += nthreads) {
+    const int r = i >> 4, v = i & 15;
+    const bool ok = r < nq;
+    const __nv_bfloat16* src = ok ? p.Q + (trow0 + r) * HD + (int64_t)h * D + v * 8 : p.Q;
+    cp_async16_zfill(sdst + r * LD + v * 8, src, ok ? 16 : 0);
+  }
+}
+
+template <int NT>
+__device__ __forceinline__ void warp_qk128(float (&S)[NT][4], const __nv_bfloat16* sQ, int q_row0,
+                                           const __nv_bfloat16* sK, int k_row0, int lane) {
+  using namespace s2k;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) S[nt][0] = S[nt][1] = S[nt][2] = S[nt][3] = 0.f;
+#pragma unroll
+  for (int kk = 0; kk < D / 16; ++kk) {
+    uint32_t a[4];
+    ldmatrix_x4(a, sQ + (q_row0 + (lane & 7) + ((lane >> 3) & 1) * 8) * LD + kk * 16 + ((lane >> 4) & 1) * 8);
+#pragma unroll
+    for (int nt = 0; nt < NT; nt += 2) {
+      uint32_t bq[4];
+      ldmatrix_x4(bq, sK + (k_row0 + nt * 8 + (lane & 7) + ((lane >> 4) & 1) * 8) * LD + kk * 16 +
+                          ((lane >> 3) & 1) * 8);
+      mma_bf16_16816(S[nt], a, bq[0], bq[1]);
+      mma_bf16_16816(S[nt + 1], a, bq[2], bq[3]);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// pass 1: softmax statistics per (text row, head)
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(128) s2_stats_kernel(Stage2Params p) {
+  using namespace s2k;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_raw);  // [64][LD]
+  __nv_bfloat16* sK = sQ + kTextTile * LD;                          // [2][KT][LD]
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nA = p.counters[CNT_NA];
+  const float c = p.scale * 1.4426950408889634f;
+  for (int it = blockIdx.x; it < nA; it += gridDim.x) {
+    const int4 item = p.itemsA[it];
+    const int b = item.x, j0 = item.y, hg = item.z;
+    const int64_t t0 = p.bt.text_off[b];
+    const int M = (int)(p.bt.text_off[b + 1] - t0);
+    const int nq = min(kTextTile, M - j0);
+    const int n_img = p.n1[b];
+    const int n_txt = p.Kt ? min(j0 + kTextTile, M) : 0;
+    const int total = n_img + n_txt;
+    const int nchunks = (total + KT - 1) / KT;
+    const int jA = j0 + warp * 16 + (lane >> 2), jB = jA + 8;
+    const int hend = min(p.H, (hg + 1) * kHeadGroup);
+    for (int h = hg * kHeadGroup; h < hend; ++h) {
+      s2_load_queries(sQ, p, t0 + j0, nq, h, tid, 128);
+      s2_load_keys(sK, p, b, t0, n_img, total, 0, KT, h, tid, 128);
+      cp_async_commit();
+      float m[2] = {-INFINITY, -INFINITY}, z[2] = {0.f, 0.f};
+      for (int kc = 0; kc < nchunks; ++kc) {
+        if (kc + 1 < nchunks) s2_load_keys(sK + ((kc + 1) & 1) * KT * LD, p, b, t0, n_img, total, (kc + 1) * KT, KT, h, tid, 128);
+        cp_async_commit();
+        cp_async_wait<1>();
+        __syncthreads();
+        float S[8][4];
+        warp_qk128<8>(S, sQ, warp * 16, sK + (kc & 1) * KT * LD, 0, lane);
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          const int j = half ? jB : jA;
+          float cm = -INFINITY;
+#pragma unroll
+          for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int key = kc * KT + nt * 8 + (lane & 3) * 2 + e;
+              const bool valid = key < n_img || (key < total && key - n_img <= j);
+              const float x = valid ? S[nt][half * 2 + e] * c : -INFINITY;
+              S[nt][half * 2 + e] = x;
+              cm = fmaxf(cm, x);
+            }
+          cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 1));
+          cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 2));
+          const float mn = fmaxf(m[half], cm);
+          float acc = 0.f;
+          if (mn != -INFINITY) {
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+              for (int e = 0; e < 2; ++e) acc += exp2f(S[nt][half * 2 + e] - mn);
+          }
+          acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+          acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+          z[half] = (m[half] == -INFINITY ? 0.f : z[half] * exp2f(m[half] - mn)) + acc;
+          m[half] = mn;
+        }
+        __syncthreads();
+      }
+      if ((lane & 3) == 0) {
+        if (jA < M) p.stats[(t0 + jA) * p.H + h] = make_float2(m[0], 1.0f / z[0]);
+        if (jB < M) p.stats[(t0 + jB) * p.H + h] = make_float2(m[1], 1.0f / z[1]);
+      }
+    }
+  }
+}
+
+int s2_stats_smem_bytes() { return (kTextTile + 2 * s2k::KT) * s2k::LD * 2; }
+
+// ---------------------------------------------------------------------------
+// pass 2: head-averaged probabilities of 128 S1 keys for 64 text rows
+// ---------------------------------------------------------------------------
+namespace s2s {
+constexpr int kQBytes = kTextTile * s2k::LD * 2;      // 17408
+constexpr int kKBytes = kKeyChunk * s2k::LD * 2;      // 34816
+constexpr int kMaxH = 64;
+constexpr int kSmem = 2 * kQBytes + 2 * kKBytes + kTextTile * kMaxH * 8 + 2 * 4 * kKeyChunk * 4 +
+                      kKeyChunk * 8 + 64;
+}  // namespace s2s
+
+int s2_scores_smem_bytes() { return s2s::kSmem; }
+
+__global__ void __launch_bounds__(256, 1) s2_scores_kernel(Stage2Params p) {
+  using namespace s2k;
+  using namespace s2s;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_raw);                       // [2][64][LD]
+  __nv_bfloat16* sK = reinterpret_cast<__nv_bfloat16*>(smem_raw + 2 * kQBytes);         // [2][128][LD]
+  float2* sst = reinterpret_cast<float2*>(smem_raw + 2 * kQBytes + 2 * kKBytes);        // [64][H]
+  float* cmax = reinterpret_cast<float*>(sst + kTextTile * kMaxH);                      // [4][128]
+  float* csum = cmax + 4 * kKeyChunk;                                                   // [4][128]
+  int* krow = reinterpret_cast<int*>(csum + 4 * kKeyChunk);                             // [128]
+  int* kreg = krow + kKeyChunk;                                                         // [128]
+  __shared__ float red[kKeyChunk];
+  __shared__ int last_flag;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int rb = warp & 3, kh = warp >> 2;
+  const int nB = p.counters[CNT_NB];
+  const float c = p.scale * 1.4426950408889634f;
+  const float invH = 1.0f / (float)p.H;
+  for (int it = blockIdx.x; it < nB; it += gridDim.x) {
+    const int4 item = p.itemsB[it];
+    const int b = item.x, j0 = item.y, kc = item.z;
+    const int64_t t0 = p.bt.text_off[b];
+    const int M = (int)(p.bt.text_off[b + 1] - t0);
+    const int nq = min(kTextTile, M - j0);
+    const int n_img = p.n1[b];
+    const int k0 = kc * kKeyChunk;
+    const int nk = min(kKeyChunk, n_img - k0);
+    const int64_t rbase = p.bt.row_off[b];
+    for (int i = tid; i < kTextTile * p.H; i += 256) {
+      const int r = i / p.H, h = i - r * p.H;
+      sst[r * p.H + h] = (r < nq) ? p.stats[(t0 + j0 + r) * p.H + h] : make_float2(0.f, 0.f);
+    }
+    for (int i = tid; i < kKeyChunk; i += 256) {
+      const int row = (i < nk) ? p.dense[rbase + k0 + i] : -1;
+      krow[i] = row;
+      kreg[i] = (row >= 0) ? (int)p.role[row] : 0;
+    }
+    // operands of head 0
+    s2_load_queries(sQ, p, t0 + j0, nq, 0, tid, 256);
+    s2_load_keys(sK, p, b, t0, n_img, n_img, k0, kKeyChunk, 0, tid, 256);
+    cp_async_commit();
+    float P[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) P[nt][0] = P[nt][1] = P[nt][2] = P[nt][3] = 0.f;
+    const int rowA = rb * 16 + (lane >> 2), rowB = rowA + 8;
+    const bool vA = rowA < nq, vB = rowB < nq;
+    for (int h = 0; h < p.H; ++h) {
+      const int buf = h & 1;
+      if (h + 1 < p.H) {
+        s2_load_queries(sQ + (buf ^ 1) * kTextTile * LD, p, t0 + j0, nq, h + 1, tid, 256);
+        s2_load_keys(sK + (buf ^ 1) * kKeyChunk * LD, p, b, t0, n_img, n_img, k0, kKeyChunk, h + 1, tid, 256);
+      }
+      cp_async_commit();
+      cp_async_wait<1>();
+      __syncthreads();
+      float S[8][4];
+      warp_qk128<8>(S, sQ + buf * kTextTile * LD, rb * 16, sK + buf * kKeyChunk * LD, kh * 64, lane);
+      const float2 sa = sst[rowA * p.H + h], sb = sst[rowB * p.H + h];
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          if (vA) P[nt][e] += exp2f(fmaf(S[nt][e], c, -sa.x)) * sa.y;
+          if (vB) P[nt][2 + e] += exp2f(fmaf(S[nt][2 + e], c, -sb.x)) * sb.y;
+        }
+      __syncthreads();
+    }
+    // column max / sum over this item's text rows
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        float mx = fmaxf(vA ? P[nt][e] : 0.f, vB ? P[nt][2 + e] : 0.f);
+        float sm = (vA ? P[nt][e] : 0.f) + (vB ? P[nt][2 + e] : 0.f);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+        sm += __shfl_xor_sync(0xffffffffu, sm, 4);
+        sm += __shfl_xor_sync(0xffffffffu, sm, 8);
+        sm += __shfl_xor_sync(0xffffffffu, sm, 16);
+        if ((lane >> 2) == 0) {
+          const int col = kh * 64 + nt * 8 + (lane & 3) * 2 + e;
+          cmax[rb * kKeyChunk + col] = mx;
+          csum[rb * kKeyChunk + col] = sm;
+        }
+      }
+    __syncthreads();
+    if (tid < kKeyChunk) {
+      float rs = 0.f;
+      if (tid < nk) {
+        const float mx = fmaxf(fmaxf(cmax[tid], cmax[kKeyChunk + tid]),
+                               fmaxf(cmax[2 * kKeyChunk + tid], cmax[3 * kKeyChunk + tid])) * invH;
+        if (kreg[tid]) {
+          rs = ((csum[tid] + csum[kKeyChunk + tid]) + (csum[2 * kKeyChunk + tid] + csum[3 * kKeyChunk + tid])) * invH;
+        } else {
+          atomicMax(reinterpret_cast<int*>(&p.s2[krow[tid]]), __float_as_int(mx));
+        }
+      }
+      red[tid] = rs;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      float acc = 0.f;
+      for (int i = 0; i < kKeyChunk; ++i) acc += red[i];
+      p.refpart[it] = acc;
+      __threadfence();
+      const int nitems = p.itemB_off[b + 1] - p.itemB_off[b];
+      last_flag = (atomicAdd(&p.done[b], 1) == nitems - 1);
+    }
+    __syncthreads();
+    if (last_flag && tid == 0) {
+      __threadfence();
+      float acc = 0.f;
+      for (int i = p.itemB_off[b]; i < p.itemB_off[b + 1]; ++i) acc += *((volatile float*)&p.refpart[i]);
+      const int R = p.bt.reg_off[p.bt.seg_first[b + 1]] - p.bt.reg_off[p.bt.seg_first[b]];
+      const float r2 = (R > 0 && M > 0) ? acc / ((float)R * (float)M) : 0.f;
+      p.ref2[b] = r2;
+      p.tau2[b] = p.lambda2 * r2;
+    }
+    __syncthreads();
+  }
+}
+
+}  // namespace occam

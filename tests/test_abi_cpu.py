@@ -1,0 +1,100 @@
+"""Host-side checks that need no GPU: the library builds, loads, exports
+every entry point include/occam.h declares, and its host validation works."""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import shutil
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("nvcc not available")
+    from paper_2605_29657_gb300 import build
+    build.build()
+    import paper_2605_29657_gb300 as occ
+    return occ.library()
+
+
+def declared_functions():
+    txt = open(os.path.join(ROOT, "include", "occam.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(occam_\w+)\s*\(", txt, re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for want in ("occam_score_stage1", "occam_threshold", "occam_score_stage2", "occam_compact",
+                 "occam_prune", "occam_workspace_size", "occam_get_status"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def _host_batch(B=2, S=4, rows=40, text=10):
+    import paper_2605_29657_gb300 as occ
+    fake = 0x1000
+    return occ._lib.CBatch(B, S, rows, text, 10, 20, 7, 2, fake, fake, fake, fake, fake, fake, fake)
+
+
+def test_workspace_size_host_only(lib):
+    import paper_2605_29657_gb300 as occ
+    n = ctypes.c_size_t(0)
+    b = _host_batch()
+    assert lib.occam_workspace_size(ctypes.byref(b), 16, 32, ctypes.byref(n)) == 0
+    small = n.value
+    assert small > 0 and small % 256 == 0
+    b2 = _host_batch(rows=4000)
+    assert lib.occam_workspace_size(ctypes.byref(b2), 16, 32, ctypes.byref(n)) == 0
+    assert n.value > small
+    bad = _host_batch(B=0)
+    assert lib.occam_workspace_size(ctypes.byref(bad), 16, 32, ctypes.byref(n)) == occ._lib.OCCAM_ERR_INVALID_ARG
+
+
+def test_invalid_arguments_rejected_on_host(lib):
+    import paper_2605_29657_gb300 as occ
+    assert lib.occam_prune(None, None, None, 0, None) == occ._lib.OCCAM_ERR_INVALID_ARG
+    a = occ._lib.CPruneArgs()
+    a.batch = _host_batch()
+    a.stage1 = occ._lib.CStage1(0, 16, 48, 0x1000, None, 0x1000)   # d1 = 48 is not built
+    a.stage2 = occ._lib.CStage2(32, 128, 0x1000, 0x1000, 0x1000)
+    o = occ._lib.CPruneOut()
+    assert lib.occam_prune(ctypes.byref(a), ctypes.byref(o), None, 0, None) != 0
+    a.stage1 = occ._lib.CStage1(0, 16, 64, 0x1001, None, 0x1000)   # misaligned q
+    assert lib.occam_prune(ctypes.byref(a), ctypes.byref(o), None, 0, None) == occ._lib.OCCAM_ERR_INVALID_ARG
+    assert lib.occam_get_status(None, None, None) == occ._lib.OCCAM_ERR_INVALID_ARG
+
+
+def test_layout_validation_host_only():
+    import paper_2605_29657_gb300 as occ
+    ok = occ.BatchLayout([0, 10, 25], [0, 4, 10, 25], [2, 3, 9, 24], [0, 2, 3, 4], [0, 3, 5], device="cpu")
+    assert ok.B == 2 and ok.S_tot == 3 and ok.max_seg_rows == 15 and ok.max_sample_rows == 15
+    assert ok.host["seg_first"].tolist() == [0, 2, 3]
+    assert ok.host["seg_sample"].tolist() == [0, 0, 1]
+    with pytest.raises(occ.OccamError):   # a sample without text
+        occ.BatchLayout([0, 10, 25], [0, 10, 25], [9, 24], [0, 1, 2], [0, 3, 3], device="cpu")
+    with pytest.raises(occ.OccamError):   # a segment without registers
+        occ.BatchLayout([0, 10, 25], [0, 10, 25], [9], [0, 1, 1], [0, 3, 5], device="cpu")
+    with pytest.raises(occ.OccamError):   # segments that do not tile the samples
+        occ.BatchLayout([0, 10, 25], [0, 12, 25], [9, 24], [0, 1, 2], [0, 3, 5], device="cpu")
+
+
+def test_no_cpu_fallback_without_device():
+    import torch
+    import paper_2605_29657_gb300 as occ
+    if torch.cuda.is_available():
+        pytest.skip("has a GPU")
+    lay = occ.BatchLayout([0, 10], [0, 10], [9], [0, 1], [0, 3], device="cpu")
+    x = torch.zeros(10, 16, 64, dtype=torch.bfloat16)
+    with pytest.raises(occ.OccamError):
+        occ.occam_score_stage1(lay, occ.OCCAM_STAGE1_CLS, x[:1], x)

@@ -1,0 +1,181 @@
+"""CUDA path (through the C ABI) against the CPU oracle on seeded inputs.
+
+Sizes are small enough for the oracle to finish in seconds but span several
+tiles of every kernel (Stage-II text tiles of 64 rows and key chunks of 128,
+[CLS] cluster shares, 2,048-row scan tiles) with ragged tails.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import occam_oracle as O
+from synth import get_config, make_batch, tiny_batch
+from tests.gpu_helpers import check_prune, close, run_prune
+
+pytestmark = pytest.mark.gpu
+
+H = dict(H1=16, d1=64, H2=32, d2=128)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__ as g
+    g.build()
+    assert torch.cuda.is_available()
+
+
+def _tiny(**kw):
+    args = dict(H, hidden=256, beta1=2.0, sinks=("count", 1))
+    args.update(kw)
+    return tiny_batch(**args)
+
+
+CASES = [
+    # (name, tiny_batch kwargs, lambda1, lambda2)
+    ("one_segment_small", dict(B=1, segs=1, P=(9,), R=1, M=(3,), seed=1), 0.5, 1.0),
+    ("ragged_three", dict(B=3, segs=2, P=(5, 37, 130), R=2, M=(1, 7, 70), seed=2), 0.4, 1.1),
+    ("text_tiles", dict(B=2, segs=3, P=(200, 90), R=4, M=(64, 129), seed=3), 0.3, 1.3),
+    ("key_chunks", dict(B=2, segs=1, P=(700, 300), R=3, M=(20, 5), seed=4), 0.05, 1.2),
+    ("scan_tiles", dict(B=5, segs=2, P=(500, 333, 612, 47, 401), R=4, M=(9, 33, 65, 2, 17), seed=5), 0.2, 1.05),
+]
+
+
+@pytest.mark.parametrize("name,kw,l1,l2", CASES, ids=[c[0] for c in CASES])
+def test_prune_cls_matches_oracle(name, kw, l1, l2):
+    b = _tiny(**kw)
+    gpu = run_prune(b, l1, l2)
+    assert gpu["status"] == 0
+    rep = check_prune(b, gpu, l1, l2)
+    assert rep["kept"] > 0
+
+
+@pytest.mark.parametrize("d1", [72, 64])
+def test_prune_mutual_matches_oracle(d1):
+    b = _tiny(B=3, segs=1, P=(60, 301, 150), R=4, M=(5, 90, 64), stage1="mutual", d1=d1, seed=6,
+              query_bias=0.5, beta1=2.0)
+    gpu = run_prune(b, 0.5, 1.1)
+    assert gpu["status"] == 0
+    check_prune(b, gpu, 0.5, 1.1)
+
+
+@pytest.mark.parametrize("name", ["llava15_b1", "llavanext_b8"])
+def test_small_workloads(name):
+    w = get_config(name)
+    b = make_batch(w)
+    gpu = run_prune(b, w.lambda1, w.lambda2)
+    assert gpu["status"] == 0
+    rep = check_prune(b, gpu, w.lambda1, w.lambda2)
+    print(name, rep)
+
+
+# ----------------------------------------------------------------------------- edge cases
+
+def test_lambda_zero_keeps_everything_and_copies_bits():
+    b = _tiny(B=2, segs=2, P=(30, 11), R=2, M=(4, 9), seed=7)
+    gpu = run_prune(b, 0.0, 0.0)
+    check_prune(b, gpu, 0.0, 0.0)
+    n = b["meta"]["total_rows"]
+    assert gpu["out_index"][:n].tolist() == list(range(n))
+    for t, name in zip(gpu["gathered"], ("hidden", "K2", "V")):
+        src = b[name].reshape(n, -1)
+        assert torch.equal(t[:n].view(torch.int16), src.view(torch.int16))
+
+
+def test_empty_stage1_keeps_only_registers():
+    b = _tiny(B=2, segs=2, P=(20, 13), R=3, M=(5, 6), seed=8)
+    gpu = run_prune(b, 1e9, 1.0)
+    check_prune(b, gpu, 1e9, 1.0)
+    assert gpu["count_vis"].tolist() == [0, 0]
+    assert gpu["n1_vis"].tolist() == [0, 0]
+    assert gpu["count_out"].tolist() == [6, 6]
+
+
+@pytest.mark.parametrize("keep_registers", [False, True])
+def test_keep_registers_flag(keep_registers):
+    b = _tiny(B=2, segs=2, P=(25, 40), R=2, M=(8, 3), seed=9)
+    gpu = run_prune(b, 0.3, 1.0, keep_registers=keep_registers)
+    check_prune(b, gpu, 0.3, 1.0, keep_registers=keep_registers)
+
+
+def test_capacity_overflow_reports_and_stays_in_bounds():
+    b = _tiny(B=2, segs=1, P=(50, 60), R=2, M=(4, 4), seed=10)
+    cap = 7
+    gpu = run_prune(b, 0.0, 0.0, capacity_rows=cap)
+    assert gpu["status"] == 2  # OCCAM_ERR_CAPACITY
+    check_prune(b, gpu, 0.0, 0.0, capacity_rows=cap)
+    assert int(gpu["out_off"][-1]) == b["meta"]["total_rows"]
+
+
+def test_text_keys_none():
+    b = _tiny(B=2, segs=1, P=(40, 70), R=2, M=(12, 3), seed=11)
+    gpu = run_prune(b, 0.3, 1.0, text_keys=False)
+    check_prune(b, gpu, 0.3, 1.0, text_keys="none")
+
+
+def test_deterministic_across_calls():
+    b = _tiny(B=3, segs=2, P=(100, 57, 220), R=3, M=(70, 5, 130), seed=12)
+    a = run_prune(b, 0.2, 1.2)
+    c = run_prune(b, 0.2, 1.2)
+    for k in ("s1", "ref1", "s2", "ref2", "keep1", "keep2", "out_index", "count_out", "out_off"):
+        assert np.array_equal(a[k], c[k]), k
+
+
+# ----------------------------------------------------------------------------- standalone entry points
+
+def test_standalone_entry_points():
+    import paper_2605_29657_gb300 as occ
+
+    b = _tiny(B=3, segs=2, P=(33, 80, 7), R=2, M=(6, 70, 2), seed=13)
+    m = b["meta"]
+    dev = torch.device("cuda")
+    layout = occ.BatchLayout.from_batch(b, dev)
+    g = {k: b[k].to(dev) for k in ("q_cls", "k_cls", "K1", "Q_text", "K_text", "K2", "hidden")}
+    s1, ref1 = occ.occam_score_stage1(layout, occ.OCCAM_STAGE1_CLS, g["q_cls"], g["K1"], k_cls=g["k_cls"])
+    os1, oref1 = O.stage1_cls(b["q_cls"], b["k_cls"], b["K1"], m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"])
+    close("s1", s1.cpu().numpy(), os1)
+    close("ref1", ref1.cpu().numpy(), oref1)
+    # threshold on the oracle's own scores (fp32 copies): exact outside the band
+    is_reg = O.register_mask(m["total_rows"], m["reg_idx_host"])
+    seg_of_row = np.repeat(np.arange(m["S_tot"]), np.diff(m["seg_off_host"]))
+    s_t = torch.tensor(os1, dtype=torch.float32, device=dev)
+    r_t = torch.tensor(oref1, dtype=torch.float32, device=dev)
+    keep, cnt = occ.occam_threshold(layout, s_t, r_t, occ.OCCAM_REF_SEGMENT, 0.6, keep_registers=True)
+    s32 = s_t.cpu().numpy().astype(np.float64)
+    tau32 = (np.float32(0.6) * r_t.cpu().numpy())[seg_of_row].astype(np.float64)
+    want = ((s32 >= tau32) & ~is_reg) | is_reg
+    assert np.array_equal(keep.cpu().numpy().astype(bool), want)
+    assert cnt.cpu().tolist() == [int((want & ~is_reg)[a:z].sum()) for a, z in zip(m["row_off_host"][:-1], m["row_off_host"][1:])]
+    # Stage II on a given S1 mask
+    rng = np.random.default_rng(0)
+    keep1 = (rng.random(m["total_rows"]) < 0.5) | is_reg
+    k1 = torch.tensor(keep1.astype(np.uint8), device=dev)
+    s2, ref2 = occ.occam_score_stage2(layout, g["Q_text"], g["K2"], k1, K_text=g["K_text"])
+    os2, oref2 = O.stage2_scores(b["Q_text"], b["K_text"], b["K2"], keep1, is_reg, m["row_off_host"], m["text_off_host"])
+    close("s2", s2.cpu().numpy(), os2)
+    close("ref2", ref2.cpu().numpy(), oref2)
+    # compaction of a random mask with one gather tensor
+    mask = rng.random(m["total_rows"]) < 0.3
+    mk = torch.tensor(mask.astype(np.uint8), device=dev)
+    res = occ.occam_compact(layout, mk, tensors=(g["hidden"],))
+    oi, oc, oo, og = O.compact(mask, m["row_off_host"], [b["hidden"].view(torch.int16).numpy()])
+    n = int(oo[-1])
+    assert res["out_index"][:n].cpu().tolist() == oi.tolist()
+    assert res["count_out"].cpu().tolist() == oc.tolist()
+    assert res["out_off"].cpu().tolist() == oo.tolist()
+    assert np.array_equal(res["gathered"][0][:n].cpu().view(torch.int16).numpy(), og[0])
+
+
+def test_invalid_arguments_raise():
+    import paper_2605_29657_gb300 as occ
+
+    b = _tiny(B=1, segs=1, P=(10,), R=1, M=(2,), seed=14)
+    dev = torch.device("cuda")
+    layout = occ.BatchLayout.from_batch(b, dev)
+    g = {k: b[k].to(dev) for k in ("q_cls", "K1")}
+    with pytest.raises(occ.OccamError):
+        occ.occam_score_stage1(layout, occ.OCCAM_STAGE1_CLS, g["q_cls"], g["K1"][:, :8].contiguous())
+    with pytest.raises(occ.OccamError):
+        occ.occam_score_stage1(layout, occ.OCCAM_STAGE1_CLS, g["q_cls"].float(), g["K1"])
