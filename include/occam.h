@@ -21,7 +21,10 @@
  *   src/dst/row_bytes arrays of a gather list, and the status out-argument of
  *   occam_get_status) is a DEVICE pointer owned by the caller. The library
  *   allocates no memory: scratch space comes from the caller's `workspace`,
- *   of at least occam_workspace_size() bytes, 256-byte aligned.
+ *   of at least occam_workspace_size() bytes, 256-byte aligned, zero-filled
+ *   by the caller before its first use (the library keeps it consistent
+ *   afterwards). One workspace serves one call at a time: calls that share
+ *   a workspace must be ordered (same stream, or synchronised).
  * - bf16 tensors are dense row-major: [rows, H, d] (K1, Q1, K2),
  *   [segments, H, d] (q_cls, k_cls), [text, H, d] (Q_text, K_text).
  *   Their base addresses must be 16-byte aligned and H*d*2 a multiple of 16.

@@ -202,8 +202,9 @@ def occam_workspace_size(layout: BatchLayout, H1: int, H2: int) -> int:
 
 
 def alloc_workspace(layout: BatchLayout, H1: int = 16, H2: int = 32) -> torch.Tensor:
+    """A zero-filled, 256-byte aligned workspace (zero-filled before its first use, as the ABI requires)."""
     n = occam_workspace_size(layout, H1, H2)
-    ws = torch.empty(n + 256, dtype=torch.uint8, device=layout.device)
+    ws = torch.zeros(n + 256, dtype=torch.uint8, device=layout.device)
     off = (-ws.data_ptr()) % 256
     return ws[off:off + n]
 
