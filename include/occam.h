@@ -219,6 +219,34 @@ int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* 
 int occam_prune_traced(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                        size_t workspace_bytes, occam_stream_t stream, void* const* events, int32_t n_events);
 
+/* occam_compact for callers that cannot allocate device memory. The paper
+ * has no counterpart: this is a deployment convenience. Some callers may not
+ * call cudaMalloc at all -- plugins whose host framework owns every device
+ * allocation, serving runtimes that forbid allocation once started, or code
+ * that must not grow the device footprint per call -- and so cannot supply
+ * the workspace occam_compact needs for its scan state. This entry point
+ * takes the same arguments as occam_compact minus the workspace: its scratch
+ * (scan tile states, a tile ticket, a status word) is a fixed 64.25 KiB
+ * array inside this library, present on every GPU that loads the library
+ * until the process exits. It calls no cudaMalloc, cudaFree or allocating
+ * library routine. Limits and behaviour:
+ * - total_rows <= 16,777,216 (8,192 scan tiles of 2,048 rows); larger batches
+ *   are rejected with OCCAM_ERR_UNSUPPORTED and nothing is launched.
+ * - The first call on a device, made with that device current, looks up the
+ *   array's device address (cudaGetSymbolAddress) and caches it; make that
+ *   first call before any stream capture.
+ * - All calls on a device share the one array. Each call clears the parts it
+ *   needs before use, but calls that overlap on the GPU (different streams
+ *   without ordering, or different host threads) race on it and produce
+ *   wrong results: order them.
+ * - Device-side errors are not reported (there is no workspace status word to
+ *   read): a capacity overflow shows as out_off[B] > capacity_rows, with
+ *   counts and offsets still exact. */
+int occam_compact_noalloc(const occam_batch* batch, const uint8_t* keep, int32_t n_tensors,
+                          const void* const* src, const int64_t* row_bytes, void* const* dst,
+                          int64_t capacity_rows, int32_t* out_index, int32_t* count_out, int64_t* out_off,
+                          occam_stream_t stream);
+
 /* Library version string (static storage). */
 const char* occam_version(void);
 

@@ -18,6 +18,7 @@ from ._lib import (  # noqa: F401
     alloc_workspace,
     library,
     occam_compact,
+    occam_compact_noalloc,
     occam_get_status,
     occam_prune,
     occam_score_stage1,

@@ -100,9 +100,11 @@ def library() -> ctypes.CDLL:
         lib.occam_compact.argtypes = [P(CBatch), _p, _i32, P(_p), P(_i64), P(_p), _i64, _p, _p, _p, _p,
                                       ctypes.c_size_t, _p]
         lib.occam_prune.argtypes = [P(CPruneArgs), P(CPruneOut), _p, ctypes.c_size_t, _p]
+        lib.occam_compact_noalloc.argtypes = [P(CBatch), _p, _i32, P(_p), P(_i64), P(_p), _i64, _p, _p, _p, _p]
         lib.occam_prune_traced.argtypes = [P(CPruneArgs), P(CPruneOut), _p, ctypes.c_size_t, _p, P(_p), _i32]
         for name in ("occam_workspace_size", "occam_get_status", "occam_score_stage1", "occam_threshold",
-                     "occam_score_stage2", "occam_compact", "occam_prune", "occam_prune_traced"):
+                     "occam_score_stage2", "occam_compact", "occam_prune", "occam_prune_traced",
+                     "occam_compact_noalloc"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -296,6 +298,28 @@ def occam_compact(layout: BatchLayout, keep, tensors=(), capacity_rows: int | No
     _check(library().occam_compact(ctypes.byref(cb), _ptr(keep), n, src_a, rb_a, dst_a, cap, _ptr(out_index),
                                    _ptr(count_out), _ptr(out_off), _ptr(ws), ws.numel(), _stream(stream)),
            "occam_compact")
+    return dict(out_index=out_index, count_out=count_out, out_off=out_off, gathered=dst)
+
+
+def occam_compact_noalloc(layout: BatchLayout, keep, tensors=(), capacity_rows: int | None = None, dst=None,
+                          out_index=None, count_out=None, out_off=None, stream=None):
+    """occam_compact without a workspace, for callers that cannot allocate
+    device memory: the library's own fixed scratch array is used instead.
+    Output buffers are the caller's; pass them in to allocate nothing here."""
+    _dev_tensor(keep, torch.uint8, "keep")
+    dev = layout.device
+    cap = layout.total_rows if capacity_rows is None else int(capacity_rows)
+    tensors = [_dev_tensor(t, t.dtype, f"tensor{i}") for i, t in enumerate(tensors)]
+    if dst is None:
+        dst = [torch.empty((cap,) + tuple(t.shape[1:]), dtype=t.dtype, device=dev) for t in tensors]
+    out_index = torch.empty(max(cap, 1), dtype=torch.int32, device=dev) if out_index is None else out_index
+    count_out = torch.empty(layout.B, dtype=torch.int32, device=dev) if count_out is None else count_out
+    out_off = torch.empty(layout.B + 1, dtype=torch.int64, device=dev) if out_off is None else out_off
+    n, src_a, rb_a, dst_a = _gather_arrays(tensors, dst)
+    cb = layout.c()
+    _check(library().occam_compact_noalloc(ctypes.byref(cb), _ptr(keep), n, src_a, rb_a, dst_a, cap,
+                                           _ptr(out_index), _ptr(count_out), _ptr(out_off), _stream(stream)),
+           "occam_compact_noalloc")
     return dict(out_index=out_index, count_out=count_out, out_off=out_off, gathered=dst)
 
 

@@ -11,6 +11,8 @@
 //   all the same and reports OCCAM_ERR_TIMEOUT instead of hanging.
 // gather_kernel: persistent grid; one warp copies one kept row of one tensor
 //   with 16-byte loads / stores (exact bit copy).
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -193,3 +195,122 @@ __global__ void __launch_bounds__(256) gather_kernel(GatherParams p) {
 }
 
 }  // namespace occam
+
+// ============================================================================
+// occam_compact_noalloc: occam_compact for callers that cannot allocate
+// device memory. Its scratch (the scan's tile states, the tile ticket and a
+// status word) lives in the file-scope array below instead of a caller
+// workspace. Every GPU that loads this library holds the array (64.25 KiB)
+// until the process exits; all calls on a device share it.
+// ============================================================================
+namespace {
+
+constexpr int64_t kNoAllocMaxTiles = 8192;  // total_rows <= 8192 * 2048 = 16,777,216
+constexpr int kNoAllocMaxDevices = 64;
+
+// [0, kNoAllocMaxTiles): tile states; then one int32 ticket and one int32 status
+static __device__ __align__(256) unsigned long long g_noalloc_scratch[kNoAllocMaxTiles + 32];
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+int g_noalloc_sms[kNoAllocMaxDevices] = {};
+
+// Device address of the static scratch on the current device (looked up once
+// per device, with that device current).
+int noalloc_scratch(void** ptr, int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices) return OCCAM_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (g_noalloc_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return OCCAM_ERR_CUDA;
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    g_noalloc_ptr[dev] = p;
+    g_noalloc_sms[dev] = n;
+  }
+  *ptr = g_noalloc_ptr[dev];
+  *sms = g_noalloc_sms[dev];
+  return OCCAM_OK;
+}
+
+bool aligned16_na(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" int occam_compact_noalloc(const occam_batch* b, const uint8_t* keep, int32_t n_tensors,
+                                     const void* const* src, const int64_t* row_bytes, void* const* dst,
+                                     int64_t capacity_rows, int32_t* out_index, int32_t* count_out,
+                                     int64_t* out_off, occam_stream_t stream) {
+  using namespace occam;
+  if (!b || b->B < 1 || b->S_tot < b->B || b->total_rows < 1 || !b->row_off || !b->seg_off ||
+      !b->reg_idx || !b->reg_off)
+    return OCCAM_ERR_INVALID_ARG;
+  if (!keep || !count_out || !out_off || capacity_rows < 0 || (capacity_rows > 0 && !out_index))
+    return OCCAM_ERR_INVALID_ARG;
+  if (n_tensors < 0 || n_tensors > OCCAM_MAX_GATHER) return OCCAM_ERR_INVALID_ARG;
+  for (int t = 0; t < n_tensors; ++t) {
+    if (!src || !dst || !row_bytes || !src[t] || !dst[t] || row_bytes[t] <= 0 || (row_bytes[t] & 15) ||
+        !aligned16_na(src[t]) || !aligned16_na(dst[t]))
+      return OCCAM_ERR_INVALID_ARG;
+  }
+  const int64_t ntiles = (b->total_rows + kScanTile - 1) / kScanTile;
+  if (ntiles > kNoAllocMaxTiles) return OCCAM_ERR_UNSUPPORTED;  // more rows than the static scratch covers
+  void* scratch = nullptr;
+  int sms = 0;
+  const int rc = noalloc_scratch(&scratch, &sms);
+  if (rc != OCCAM_OK) return rc;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  unsigned long long* tiles = static_cast<unsigned long long*>(scratch);
+  int32_t* ticket = reinterpret_cast<int32_t*>(tiles + kNoAllocMaxTiles);
+  int* status = reinterpret_cast<int*>(ticket + 1);
+  // the array keeps the previous call's contents: clear what must start at zero
+  if (cudaMemsetAsync(tiles, 0, ntiles * 8, st) != cudaSuccess) return OCCAM_ERR_CUDA;
+  if (cudaMemsetAsync(ticket, 0, 8, st) != cudaSuccess) return OCCAM_ERR_CUDA;
+  if (cudaMemsetAsync(count_out, 0, b->B * 4, st) != cudaSuccess) return OCCAM_ERR_CUDA;
+  ScanParams p;
+  p.bt.B = b->B;
+  p.bt.S_tot = b->S_tot;
+  p.bt.total_rows = b->total_rows;
+  p.bt.total_text = b->total_text;
+  p.bt.row_off = b->row_off;
+  p.bt.seg_off = b->seg_off;
+  p.bt.seg_first = b->seg_first;
+  p.bt.seg_sample = b->seg_sample;
+  p.bt.reg_idx = b->reg_idx;
+  p.bt.reg_off = b->reg_off;
+  p.bt.text_off = b->text_off;
+  p.mode = 0;
+  p.keep_in = keep;
+  p.role = nullptr;
+  p.keep1 = nullptr;
+  p.s2 = nullptr;
+  p.tau2 = nullptr;
+  p.keep_registers = 0;
+  p.keep_out = nullptr;
+  p.capacity = capacity_rows;
+  p.out_index = out_index;
+  p.count_out = count_out;
+  p.count_vis = nullptr;
+  p.out_off = out_off;
+  p.tile_state = tiles;
+  p.ticket = ticket;
+  p.ntiles = ntiles;
+  p.status = status;
+  scan_kernel<<<(unsigned)ntiles, 256, 0, st>>>(p);
+  if (n_tensors > 0) {
+    GatherParams g;
+    g.n_tensors = n_tensors;
+    for (int t = 0; t < OCCAM_MAX_GATHER; ++t) {
+      g.src[t] = t < n_tensors ? static_cast<const unsigned char*>(src[t]) : nullptr;
+      g.dst[t] = t < n_tensors ? static_cast<unsigned char*>(dst[t]) : nullptr;
+      g.row_bytes[t] = t < n_tensors ? row_bytes[t] : 0;
+    }
+    g.out_index = out_index;
+    g.out_off = out_off;
+    g.B = b->B;
+    g.capacity = capacity_rows;
+    gather_kernel<<<sms * 4, 256, 0, st>>>(g);
+  }
+  return cudaGetLastError() == cudaSuccess ? OCCAM_OK : OCCAM_ERR_CUDA;
+}
