@@ -432,7 +432,10 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="synthetic workload to time (default: the LLaVA-NeXT batch-64 throughput workload)")
     args = ap.parse_args()
+    globals()["WORKLOAD"] = args.workload
     if args.warmup < 3:
         args.warmup = 3
     rank, world, local = _dist()
