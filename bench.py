@@ -41,7 +41,7 @@ FALLBACK_HBM_GBS = 6800.0
 SPEC_HBM_GBS = 8000.0
 KERNEL_SOURCES = {
     "stage1": "stage1.cu", "stage1_finalize": "stage1.cu", "s1_list_plan": "stage2.cu",
-    "stage2_stats": "stage2.cu", "stage2_scores": "stage2.cu", "scan": "compact.cu", "gather": "compact.cu",
+    "stage2_fused": "stage2_tc.cu", "stage2_twopass": "stage2.cu", "scan": "compact.cu", "gather": "compact.cu",
 }
 
 
@@ -155,8 +155,8 @@ def algorithmic_bytes(meta: dict, n1_total: int, kept_total: int) -> dict:
     b["stage1"] = rows * k1row + 2 * S * k1row + rows * 8            # K1 once, q/k_cls, s1 write, s2 zero
     b["stage1_finalize"] = rows * (4 + 1 + 1 + 4)                    # s1 read, role, keep1, list
     b["s1_list_plan"] = n1_total * 8                                 # list copy
-    b["stage2_stats"] = n1_total * k2row + 2 * T * k2row + T * H2 * 8  # S1 keys, Q + K_text, stats
-    b["stage2_scores"] = n1_total * k2row + T * k2row + T * H2 * 8   # S1 keys, Q, stats
+    b["stage2_fused"] = n1_total * k2row + 2 * T * k2row               # S1 keys once, Q + K_text
+    b["stage2_twopass"] = 2 * n1_total * k2row + 3 * T * k2row + 2 * T * H2 * 8  # both passes
     b["scan"] = rows * (1 + 1 + 4 + 1) + kept_total * 4              # keep1, role, s2, keep2, out_index
     b["gather"] = kept_total * 2 * (2 * hrow + k2row)                # read + write hidden, K, V rows
     # whole step, each byte once: K1, S1 keys, text Q/K, hidden+V of kept rows
@@ -384,7 +384,7 @@ def run_ours(args, rank, world, local):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 7 * args.steps,
+        "gpu_launches": 8 * args.steps,
         "clocks": clocks,
     }
     if world > 1:

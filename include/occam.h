@@ -211,11 +211,13 @@ int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* 
 
 /* occam_prune that also records caller-created CUDA events (cudaEvent_t,
  * passed as void*) on `stream` between its steps, for per-kernel timing:
- * events[0] after the initial zeroing, then one after each kernel in launch
- * order ([CLS] or mutual scoring, Stage-I finalize, S1 list + work plan,
- * Stage-II statistics, Stage-II scores, compaction scan, gather). Mutual
- * scoring is two kernels timed together. Extra events are left unrecorded;
- * missing ones are skipped. Results are identical to occam_prune. */
+ * events[0] after the initial zeroing, then one after each step in launch
+ * order: [CLS] or mutual scoring, Stage-I finalize, S1 list + work plan,
+ * fused tensor-core Stage II, two-pass Stage II (statistics and scores
+ * kernels, for the samples the fused kernel does not take), compaction scan,
+ * gather. Mutual scoring and the two-pass Stage II are two kernels each,
+ * timed together. Extra events are left unrecorded; missing ones are
+ * skipped. Results are identical to occam_prune. */
 int occam_prune_traced(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                        size_t workspace_bytes, occam_stream_t stream, void* const* events, int32_t n_events);
 

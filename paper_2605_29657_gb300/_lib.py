@@ -393,7 +393,7 @@ class PruneCall:
                                      self.ws.numel(), _stream(stream)), "occam_prune")
         return self.out
 
-    TRACE_NAMES = ("stage1", "stage1_finalize", "s1_list_plan", "stage2_stats", "stage2_scores", "scan", "gather")
+    TRACE_NAMES = ("stage1", "stage1_finalize", "s1_list_plan", "stage2_fused", "stage2_twopass", "scan", "gather")
 
     def traced(self, events, stream=None) -> dict:
         """As __call__, recording ``events`` (torch.cuda.Event, enable_timing) between the kernels."""

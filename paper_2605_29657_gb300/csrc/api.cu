@@ -1,8 +1,12 @@
 // api.cu -- the C ABI of include/occam.h: host-side validation, workspace
 // carve-up and kernel launches. Nothing here allocates memory.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cstdlib>
+#include <cstring>
 #include <mutex>
 
 #include "common.cuh"
@@ -46,11 +50,15 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   const int64_t chmax = cdiv(b->max_sample_rows, kKeyChunk);
   L.maxA = B * tps * nhg;
   L.maxB = B * tps * chmax;
+  L.maxF = B * cdiv(b->max_text, 128);
+  L.maxSlots = L.maxB + L.maxF * kFusedSlotsPerItem;
   L.itemsA = take(L.maxA * 16);
   L.itemsB = take(L.maxB * 16);
+  L.itemsF = take(L.maxF * 16);
   L.itemB_off = take((B + 1) * 4);
+  L.slot_off = take((B + 1) * 4);
   L.stats2 = take(T * (H2 > 0 ? H2 : 1) * 8);
-  L.refpart = take(L.maxB * 4);
+  L.refpart = take(L.maxSlots * 4);
   L.ref2 = take(B * 4);
   L.tau2 = take(B * 4);
   L.done = take(B * 4);
@@ -117,11 +125,49 @@ int num_sms() {
 void set_smem_attrs() {
   static std::once_flag once;
   std::call_once(once, [] {
+    cudaFuncSetAttribute(s2_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes());
     cudaFuncSetAttribute(stage1_cls_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          stage1_cls_smem_bytes());
     cudaFuncSetAttribute(s2_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_stats_smem_bytes());
     cudaFuncSetAttribute(s2_scores_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_scores_smem_bytes());
   });
+}
+
+// cuTensorMapEncodeTiled from the driver, looked up once.
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+// 2-D bf16 map over a [rows, cols] row-major tensor, 128-byte swizzle, box
+// of 64 columns x box_rows rows.
+bool encode_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, uint32_t box_rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t gstride[1] = {(cuuint64_t)(cols * 2)};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Stage-II path selection: the fused tensor-core kernel for every sample that
+// fits it (default), or the two-pass kernels for all samples when
+// OCCAM_STAGE2_PATH=twopass (used to test both paths on the same inputs).
+bool fused_enabled() {
+  const char* e = std::getenv("OCCAM_STAGE2_PATH");
+  return !(e && std::strcmp(e, "twopass") == 0);
 }
 
 int cuda_ok() {
@@ -283,13 +329,58 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
   p.tau2 = at<float>(ws, L.tau2);
   p.lambda2 = lambda2;
   p.status = at<int>(ws, L.status);
+  const bool fused = fused_enabled() && L.maxF > 0 && b->total_text > 0;
+  p.itemsF = at<int4>(ws, L.itemsF);
+  p.slot_off = at<int32_t>(ws, L.slot_off);
+  p.maxF = L.maxF;
+  p.use_fused = fused ? 1 : 0;
   s2_dense_plan_kernel<<<b->B, 256, 0, st>>>(p, 1);
   trace.mark(st);
   const int sms = num_sms();
+  if (fused) {
+    CUtensorMap mq, mk, mkt;
+    const int64_t cols = (int64_t)a->H2 * 128;
+    const void* kt = a->K_text ? a->K_text : a->Q_text;
+    if (!encode_map(&mq, a->Q_text, b->total_text, cols, 128) || !encode_map(&mk, a->K2, b->total_rows, cols, 1) ||
+        !encode_map(&mkt, kt, b->total_text, cols, 1))
+      return OCCAM_ERR_CUDA;
+    Stage2TcParams q;
+    q.bt = p.bt;
+    q.H = a->H2;
+    q.scale_log2 = p.scale * 1.4426950408889634f;
+    q.has_text = a->K_text ? 1 : 0;
+    q.dense = p.dense;
+    q.n1 = p.n1;
+    q.role = p.role;
+    q.items = p.itemsF;
+    q.counters = p.counters;
+    q.s2 = s2;
+    q.refpart = p.refpart;
+    q.slot_off = p.slot_off;
+    q.done = p.done;
+    q.ref2 = ref2;
+    q.tau2 = p.tau2;
+    q.lambda2 = lambda2;
+    q.status = p.status;
+    const int ncl = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / kFusedCluster));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(ncl * kFusedCluster));
+    cfg.blockDim = dim3(192);
+    cfg.dynamicSmemBytes = s2_fused_smem_bytes();
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kFusedCluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    OCCAM_CUDA(cudaLaunchKernelEx(&cfg, s2_fused_kernel, mq, mk, mkt, q));
+  }
+  trace.mark(st);
   const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);
   const int gB = (int)std::min<int64_t>(L.maxB, sms);
   if (gA > 0) s2_stats_kernel<<<gA, 128, s2_stats_smem_bytes(), st>>>(p);
-  trace.mark(st);
   if (gB > 0) s2_scores_kernel<<<gB, 256, s2_scores_smem_bytes(), st>>>(p);
   trace.mark(st);
   return cuda_ok();

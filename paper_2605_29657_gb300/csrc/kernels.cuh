@@ -1,10 +1,16 @@
 // kernels.cuh -- kernel parameter blocks and declarations (internal).
 #pragma once
 
+#include <cuda.h>
+
 #include "common.cuh"
 
 namespace occam {
 
+constexpr int kFusedCluster = 4;        // CTAs per cluster of the fused tcgen05 Stage-II kernel
+constexpr int kFusedMaxOwnImg = 384;    // S1 keys one of its CTAs can hold (TMEM columns)
+constexpr int kFusedMaxOwnTxt = 256;    // text keys one of its CTAs can take
+constexpr int kFusedSlotsPerItem = kFusedCluster * 4;  // s2(r) partials per item (one per epilogue warp)
 constexpr int kMaxClsRowsPerCta = 512;  // rows of one segment handled by one CTA of a [CLS] cluster
 constexpr int kMaxClusterCls = 8;       // portable cluster size
 
@@ -79,6 +85,10 @@ struct Stage2Params {
   float* s2;                // atomicMax accumulator, zeroed beforehand
   float* refpart;           // [maxB]
   int32_t* done;            // [B] finished score items per sample (zeroed)
+  int4* itemsF;             // fused items (b, j0, slot, -)
+  int use_fused;            // route eligible samples to the fused tensor-core kernel
+  int32_t* slot_off;        // [B+1] partial-slot range of each sample
+  int64_t maxF;
   float* ref2;              // [B]
   float* tau2;              // [B]
   float lambda2;
@@ -117,6 +127,26 @@ struct GatherParams {
   int64_t capacity;
 };
 
+struct Stage2TcParams {
+  BatchDev bt;
+  int H;
+  float scale_log2;
+  int has_text;
+  const int32_t* dense;
+  const int32_t* n1;
+  const uint8_t* role;
+  const int4* items;
+  const int32_t* counters;
+  float* s2;
+  float* refpart;
+  const int32_t* slot_off;
+  int32_t* done;
+  float* ref2;
+  float* tau2;
+  float lambda2;
+  int* status;
+};
+
 // stage1.cu
 __global__ void stage1_cls_kernel(Stage1ClsParams p);
 int stage1_cls_smem_bytes();
@@ -132,6 +162,11 @@ __global__ void s2_stats_kernel(Stage2Params p);
 __global__ void s2_scores_kernel(Stage2Params p);
 int s2_scores_smem_bytes();
 int s2_stats_smem_bytes();
+
+// stage2_tc.cu
+__global__ void s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
+                                const __grid_constant__ CUtensorMap mapKt, Stage2TcParams p);
+int s2_fused_smem_bytes();
 
 // compact.cu
 __global__ void scan_kernel(ScanParams p);

@@ -54,41 +54,60 @@ __global__ void __launch_bounds__(256) s2_dense_plan_kernel(Stage2Params p, int 
   if (!is_last) return;
   __threadfence();
   const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
-  int runA = 0, runB = 0;
+  int runA = 0, runB = 0, runF = 0, runS = 0;
   for (int b0 = 0; b0 < p.bt.B; b0 += blockDim.x) {
     const int bb = b0 + tid;
-    int nA = 0, nB = 0, tiles = 0, nch = 0;
+    int nA = 0, nB = 0, nF = 0, tiles = 0, nch = 0, tiles128 = 0;
     if (bb < p.bt.B) {
       const int M = (int)(p.bt.text_off[bb + 1] - p.bt.text_off[bb]);
       const int n1 = *((volatile int32_t*)&p.n1[bb]);
-      tiles = (M + kTextTile - 1) / kTextTile;
-      nch = (n1 + kKeyChunk - 1) / kKeyChunk;
-      nA = tiles * nhg;
-      nB = tiles * nch;
+      // the fused tensor-core kernel takes a sample when its S1 keys and its
+      // causal text keys fit the cluster's TMEM / shared memory
+      const bool fused = p.use_fused && n1 <= kFusedCluster * kFusedMaxOwnImg &&
+                         M <= kFusedCluster * kFusedMaxOwnTxt && M > 0;
+      if (fused) {
+        tiles128 = (M + 127) / 128;
+        nF = tiles128;
+      } else {
+        tiles = (M + kTextTile - 1) / kTextTile;
+        nch = (n1 + kKeyChunk - 1) / kKeyChunk;
+        nA = tiles * nhg;
+        nB = tiles * nch;
+      }
       if (M == 0) {
         set_status(p.status, OCCAM_ERR_INVALID_ARG);
         p.ref2[bb] = 0.f;
         p.tau2[bb] = 0.f;
       }
     }
-    int totA, totB;
+    const int nS = nF * kFusedSlotsPerItem + nB;  // s2(r) partial slots of this sample
+    int totA, totB, totF, totS;
     const int offA = runA + block_exclusive_scan(nA, tmp, &totA);
     const int offB = runB + block_exclusive_scan(nB, tmp, &totB);
+    const int offF = runF + block_exclusive_scan(nF, tmp, &totF);
+    const int offS = runS + block_exclusive_scan(nS, tmp, &totS);
     if (bb < p.bt.B) {
       for (int i = 0; i < nA; ++i)
         if (offA + i < p.maxA) p.itemsA[offA + i] = make_int4(bb, (i / nhg) * kTextTile, i % nhg, 0);
       for (int i = 0; i < nB; ++i)
-        if (offB + i < p.maxB) p.itemsB[offB + i] = make_int4(bb, (i / nch) * kTextTile, i % nch, i);
+        if (offB + i < p.maxB) p.itemsB[offB + i] = make_int4(bb, (i / nch) * kTextTile, i % nch, offS + i);
+      for (int i = 0; i < nF; ++i)
+        if (offF + i < p.maxF) p.itemsF[offF + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem, 0);
       p.itemB_off[bb] = offB;
+      p.slot_off[bb] = offS;
     }
     runA += totA;
     runB += totB;
+    runF += totF;
+    runS += totS;
   }
   if (tid == 0) {
     p.itemB_off[p.bt.B] = runB;
-    if (runA > p.maxA || runB > p.maxB) set_status(p.status, OCCAM_ERR_CAPACITY);
+    p.slot_off[p.bt.B] = runS;
+    if (runA > p.maxA || runB > p.maxB || runF > p.maxF) set_status(p.status, OCCAM_ERR_CAPACITY);
     p.counters[CNT_NA] = (int)(runA < p.maxA ? runA : p.maxA);
     p.counters[CNT_NB] = (int)(runB < p.maxB ? runB : p.maxB);
+    p.counters[CNT_NF] = (int)(runF < p.maxF ? runF : p.maxF);
   }
 }
 
@@ -257,7 +276,7 @@ __global__ void __launch_bounds__(256, 1) s2_scores_kernel(Stage2Params p) {
   const float invH = 1.0f / (float)p.H;
   for (int it = blockIdx.x; it < nB; it += gridDim.x) {
     const int4 item = p.itemsB[it];
-    const int b = item.x, j0 = item.y, kc = item.z;
+    const int b = item.x, j0 = item.y, kc = item.z, slot = item.w;
     const int64_t t0 = p.bt.text_off[b];
     const int M = (int)(p.bt.text_off[b + 1] - t0);
     const int nq = min(kTextTile, M - j0);
@@ -341,16 +360,16 @@ __global__ void __launch_bounds__(256, 1) s2_scores_kernel(Stage2Params p) {
     if (tid == 0) {
       float acc = 0.f;
       for (int i = 0; i < kKeyChunk; ++i) acc += red[i];
-      p.refpart[it] = acc;
+      p.refpart[slot] = acc;
       __threadfence();
-      const int nitems = p.itemB_off[b + 1] - p.itemB_off[b];
-      last_flag = (atomicAdd(&p.done[b], 1) == nitems - 1);
+      const int nslots = p.slot_off[b + 1] - p.slot_off[b];
+      last_flag = (atomicAdd(&p.done[b], 1) == nslots - 1);
     }
     __syncthreads();
     if (last_flag && tid == 0) {
       __threadfence();
       float acc = 0.f;
-      for (int i = p.itemB_off[b]; i < p.itemB_off[b + 1]; ++i) acc += *((volatile float*)&p.refpart[i]);
+      for (int i = p.slot_off[b]; i < p.slot_off[b + 1]; ++i) acc += *((volatile float*)&p.refpart[i]);
       const int R = p.bt.reg_off[p.bt.seg_first[b + 1]] - p.bt.reg_off[p.bt.seg_first[b]];
       const float r2 = (R > 0 && M > 0) ? acc / ((float)R * (float)M) : 0.f;
       p.ref2[b] = r2;

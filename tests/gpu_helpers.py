@@ -29,7 +29,21 @@ def to_device(batch: dict, dev) -> dict:
 
 
 def run_prune(batch: dict, lam1: float, lam2: float, keep_registers: bool = True, dev="cuda",
-              capacity_rows=None, gather=True, text_keys: bool = True, g=None):
+              capacity_rows=None, gather=True, text_keys: bool = True, g=None, path: str = "auto"):
+    """path: "auto" (fused tensor-core Stage II where it fits) or "twopass"."""
+    import os
+    old = os.environ.get("OCCAM_STAGE2_PATH")
+    os.environ["OCCAM_STAGE2_PATH"] = path
+    try:
+        return _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g)
+    finally:
+        if old is None:
+            os.environ.pop("OCCAM_STAGE2_PATH", None)
+        else:
+            os.environ["OCCAM_STAGE2_PATH"] = old
+
+
+def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g):
     import paper_2605_29657_gb300 as occ
 
     m = batch["meta"]

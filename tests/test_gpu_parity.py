@@ -40,16 +40,30 @@ CASES = [
     ("text_tiles", dict(B=2, segs=3, P=(200, 90), R=4, M=(64, 129), seed=3), 0.3, 1.3),
     ("key_chunks", dict(B=2, segs=1, P=(700, 300), R=3, M=(20, 5), seed=4), 0.05, 1.2),
     ("scan_tiles", dict(B=5, segs=2, P=(500, 333, 612, 47, 401), R=4, M=(9, 33, 65, 2, 17), seed=5), 0.2, 1.05),
+    # fused tensor-core Stage II: text tiles of 128 rows, chunk edges at 64 keys per CTA
+    ("fused_text_edges", dict(B=4, segs=1, P=(252, 60, 300, 5), R=4, M=(128, 129, 256, 1), seed=21), 0.0, 1.1),
+    ("fused_max_keys", dict(B=1, segs=2, P=(760,), R=4, M=(40,), seed=22), 0.0, 1.2),
+    # one sample above the fused kernel's S1 limit (two-pass), one below (fused)
+    ("mixed_paths", dict(B=2, segs=1, P=(1700, 200), R=3, M=(70, 90), seed=23), 0.0, 1.1),
 ]
 
 
+@pytest.mark.parametrize("path", ["auto", "twopass"])
 @pytest.mark.parametrize("name,kw,l1,l2", CASES, ids=[c[0] for c in CASES])
-def test_prune_cls_matches_oracle(name, kw, l1, l2):
+def test_prune_cls_matches_oracle(name, kw, l1, l2, path):
     b = _tiny(**kw)
-    gpu = run_prune(b, l1, l2)
+    gpu = run_prune(b, l1, l2, path=path)
     assert gpu["status"] == 0
     rep = check_prune(b, gpu, l1, l2)
     assert rep["kept"] > 0
+
+
+def test_registers_only_s1():
+    """Stage I keeps no visual row: S1 = registers (some CTAs of a cluster own no keys)."""
+    b = _tiny(B=2, segs=1, P=(30, 9), R=1, M=(5, 140), seed=24)
+    gpu = run_prune(b, 1e9, 1.0)
+    assert gpu["status"] == 0
+    check_prune(b, gpu, 1e9, 1.0)
 
 
 @pytest.mark.parametrize("d1", [72, 64])
@@ -109,9 +123,10 @@ def test_capacity_overflow_reports_and_stays_in_bounds():
     assert int(gpu["out_off"][-1]) == b["meta"]["total_rows"]
 
 
-def test_text_keys_none():
+@pytest.mark.parametrize("path", ["auto", "twopass"])
+def test_text_keys_none(path):
     b = _tiny(B=2, segs=1, P=(40, 70), R=2, M=(12, 3), seed=11)
-    gpu = run_prune(b, 0.3, 1.0, text_keys=False)
+    gpu = run_prune(b, 0.3, 1.0, text_keys=False, path=path)
     check_prune(b, gpu, 0.3, 1.0, text_keys="none")
 
 
