@@ -347,6 +347,8 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     Stage2TcParams q;
     q.bt = p.bt;
     q.H = a->H2;
+    q.K = static_cast<const __nv_bfloat16*>(a->K2);
+    q.Kt = static_cast<const __nv_bfloat16*>(kt);
     q.scale_log2 = p.scale * 1.4426950408889634f;
     q.has_text = a->K_text ? 1 : 0;
     q.dense = p.dense;
@@ -365,7 +367,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     const int ncl = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / kFusedCluster));
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(ncl * kFusedCluster));
-    cfg.blockDim = dim3(192);
+    cfg.blockDim = dim3(s2_fused_threads());
     cfg.dynamicSmemBytes = s2_fused_smem_bytes();
     cfg.stream = st;
     cudaLaunchAttribute attr[1];

@@ -10,7 +10,8 @@ namespace occam {
 constexpr int kFusedCluster = 4;        // CTAs per cluster of the fused tcgen05 Stage-II kernel
 constexpr int kFusedMaxOwnImg = 384;    // S1 keys one of its CTAs can hold (TMEM columns)
 constexpr int kFusedMaxOwnTxt = 256;    // text keys one of its CTAs can take
-constexpr int kFusedSlotsPerItem = kFusedCluster * 4;  // s2(r) partials per item (one per epilogue warp)
+constexpr int kFusedEpiWarps = 8;       // epilogue warps per CTA of the fused kernel
+constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedEpiWarps;  // s2(r) partials per item (one per epilogue warp)
 constexpr int kMaxClsRowsPerCta = 512;  // rows of one segment handled by one CTA of a [CLS] cluster
 constexpr int kMaxClusterCls = 8;       // portable cluster size
 
@@ -130,6 +131,8 @@ struct GatherParams {
 struct Stage2TcParams {
   BatchDev bt;
   int H;
+  const __nv_bfloat16* K;   // [rows, H, 128]
+  const __nv_bfloat16* Kt;  // [total_text, H, 128] (any valid pointer when has_text == 0)
   float scale_log2;
   int has_text;
   const int32_t* dense;
@@ -167,6 +170,7 @@ int s2_stats_smem_bytes();
 __global__ void s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
                                 const __grid_constant__ CUtensorMap mapKt, Stage2TcParams p);
 int s2_fused_smem_bytes();
+int s2_fused_threads();
 
 // compact.cu
 __global__ void scan_kernel(ScanParams p);

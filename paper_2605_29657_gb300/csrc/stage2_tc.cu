@@ -9,15 +9,16 @@
 // Work item = (sample, tile of 128 text rows), processed by one cluster of 4
 // CTAs. The text rows are the 128 TMEM lanes; each CTA owns a quarter of the
 // sample's S1 keys and of the causal text keys. Per head:
-//   1. the producer warp loads the head's 128 x 128 query tile (TMA, 128-byte
-//      swizzle) and streams the CTA's key rows in 64-key chunks with TMA
-//      gather4 (S1 rows are gathered by index straight from K2: pruned rows
-//      are never read);
+//   1. three producer warps stream the CTA's key rows in 64-key chunks with
+//      16-byte cp.async into the 128-byte-swizzled operand layout (S1 rows
+//      are gathered by index straight from K2: pruned rows are never read),
+//      and the head's 128 x 128 query tile arrives by TMA;
 //   2. the MMA warp computes S = Q K^T per chunk into a TMEM buffer;
-//   3. the four epilogue warps (one thread per text row) keep the row's
-//      running softmax max / sum over the CTA's keys, then exchange them
-//      with the three peer CTAs through distributed shared memory, so every
-//      CTA holds the exact per-row max and sum over all keys of the head;
+//   3. eight epilogue warps (two per TMEM lane quadrant, one thread per text
+//      row, taking alternate chunks) keep the row's running softmax max / sum
+//      over their chunks, then exchange them with every epilogue warp of the
+//      cluster through distributed shared memory, so every CTA holds the
+//      exact per-row max and sum over all keys of the head;
 //   4. the image chunks are multiplied again (S is recomputed from shared
 //      memory) and exp(l - max) / sum is accumulated into the head-summed
 //      probabilities P, which live in TMEM for the whole item.
@@ -41,7 +42,11 @@ constexpr int PMAX = kFusedMaxOwnImg;  // max S1 keys per CTA (P columns)
 constexpr int TMAX = kFusedMaxOwnTxt;  // max text keys per CTA
 constexpr int QBYTES = QR * 256;       // one head's query tile: 2 K-blocks x 128 rows x 128 B
 constexpr int KBYTES = KC * 256;       // one chunk: 2 K-blocks x 64 rows x 128 B
-constexpr int THREADS = 192;           // warp 0 producer, warp 1 MMA, warps 2-5 epilogue
+constexpr int NPROD = 3;               // producer warps (0-2); warp 3 issues MMAs; then the epilogue warps
+constexpr int MMA_WARP = NPROD;
+constexpr int EPI_WARP0 = NPROD + 1;
+constexpr int NEPI = kFusedEpiWarps;   // two per TMEM lane quadrant; half h takes chunks with (index & 1) == h
+constexpr int THREADS = (NPROD + 1 + NEPI) * 32;
 constexpr uint32_t IDESC = tc::idesc_bf16(128, KC);
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int S_COL = 0;               // two S buffers of KC columns
@@ -53,7 +58,7 @@ struct Smem {
   uint8_t q[2][QBYTES];
   uint8_t k[NST][KBYTES];
   int32_t kidx[2][PMAX + TMAX];
-  float2 xch[2][C][QR];
+  float2 xch[2][C][2][QR];
   uint8_t kreg[2][PMAX];
   uint64_t kfull[NST], kempty[NST], qfull[2], qempty[2], sfull[2], sempty[2], xbar[2], iready[2], idone[2], mdone;
   uint32_t tmem_base;
@@ -63,6 +68,7 @@ struct Smem {
 }  // namespace s2f
 
 int s2_fused_smem_bytes() { return (int)sizeof(s2f::Smem) + 1024; }
+int s2_fused_threads() { return s2f::THREADS; }
 
 namespace {
 
@@ -124,15 +130,15 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   volatile int* abort = &sm.abort;
 
   if (tid == 0) {
-    for (int i = 0; i < NST; ++i) { tc::bar_init(&sm.kfull[i], 1); tc::bar_init(&sm.kempty[i], 1); }
+    for (int i = 0; i < NST; ++i) { tc::bar_init(&sm.kfull[i], NPROD * 32); tc::bar_init(&sm.kempty[i], 1); }
     for (int i = 0; i < 2; ++i) {
       tc::bar_init(&sm.qfull[i], 1);
       tc::bar_init(&sm.qempty[i], 1);
       tc::bar_init(&sm.sfull[i], 1);
       tc::bar_init(&sm.sempty[i], 4);
-      tc::bar_init(&sm.xbar[i], 4 * C);
-      tc::bar_init(&sm.iready[i], 1);
-      tc::bar_init(&sm.idone[i], 4);
+      tc::bar_init(&sm.xbar[i], NEPI * C);
+      tc::bar_init(&sm.iready[i], NPROD * 32);
+      tc::bar_init(&sm.idone[i], NEPI);
     }
     tc::bar_init(&sm.mdone, 1);
     sm.abort = 0;
@@ -143,7 +149,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     tc::prefetch_map(&mapK);
     tc::prefetch_map(&mapKt);
   }
-  if (warp == 1) tc::tmem_alloc(&sm.tmem_base, TMEM_COLS);
+  if (warp == MMA_WARP) tc::tmem_alloc(&sm.tmem_base, TMEM_COLS);
   tc::fence_before();
   __syncthreads();
   tc::fence_after();
@@ -152,68 +158,77 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   const uint32_t tmem = sm.tmem_base;
   const int H = p.H;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ producer
+  if (warp < NPROD) {
+    // ------------------------------------------------------------ producers
+    // 96 threads; piece q = pt + 96 i (q < 1024) of a chunk is 16 bytes of key
+    // row (q >> 4), head slice bytes 16 * (q & 15); it lands at the row's
+    // 128-byte line of its K-block with the 16-byte chunk index XOR (row & 7).
+    const int pt = tid;
     uint32_t qcnt = 0, kcnt = 0;
     int ii = 0;
+    const int64_t HD = (int64_t)H * 128;
     for (int item = cid; item < nF; item += ncl, ++ii) {
       const ItemGeom g = item_geom(p, p.items[item], rank);
       const int ib = ii & 1;
-      // lane 0 decides, the warp follows (no divergent exits around __syncwarp)
-      int go = 0;
-      if (lane == 0) {
-        go = !*abort && tc::bar_wait(&sm.idone[ib], ((ii >> 1) & 1) ^ 1, abort, kLimitNs);
-        if (!go && !*abort) fail(sm, p.status);
-      }
-      if (!__shfl_sync(0xffffffffu, go, 0)) break;
-      for (int i = lane; i < g.own_img; i += 32) {
+      if (*abort || !tc::bar_wait(&sm.idone[ib], ((ii >> 1) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
+      for (int i = pt; i < g.own_img; i += NPROD * 32) {
         const int row = p.dense[g.rbase + g.img0 + i];
         sm.kidx[ib][i] = row;
         sm.kreg[ib][i] = p.role[row];
       }
-      for (int i = lane; i < g.own_txt; i += 32) sm.kidx[ib][PMAX + i] = (int)(g.t0 + g.txt0 + i);
-      __syncwarp();
-      if (lane == 0) {
-        tc::bar_arrive(&sm.iready[ib]);
-        const int nch = 2 * g.nic + g.ntc;
-        for (int h = 0; h < H && !*abort; ++h) {
+      for (int i = pt; i < g.own_txt; i += NPROD * 32) sm.kidx[ib][PMAX + i] = (int)(g.t0 + g.txt0 + i);
+      tc::bar_arrive(&sm.iready[ib]);
+      if (!tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
+      const int nch = 2 * g.nic + g.ntc;
+      bool ok = true;
+      for (int h = 0; h < H && ok; ++h) {
+        if (pt == 0) {
           const int qb = qcnt & 1;
-          if (!tc::bar_wait(&sm.qempty[qb], ((qcnt >> 1) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-          tc::bar_expect_tx(&sm.qfull[qb], QBYTES);
-          tc::tma_load_2d(sm.q[qb], &mapQ, h * 128, (int)(g.t0 + g.j0), &sm.qfull[qb]);
-          tc::tma_load_2d(sm.q[qb] + QBYTES / 2, &mapQ, h * 128 + 64, (int)(g.t0 + g.j0), &sm.qfull[qb]);
-          ++qcnt;
-          for (int ci = 0; ci < nch; ++ci) {
-            const int st = kcnt % NST;
-            if (!tc::bar_wait(&sm.kempty[st], ((kcnt / NST) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-            const bool is_txt = (ci >= g.nic) && (ci < g.nic + g.ntc);
-            const int c = ci < g.nic ? ci : (is_txt ? ci - g.nic : ci - g.nic - g.ntc);
-            const int* rows = is_txt ? &sm.kidx[ib][PMAX + c * KC] : &sm.kidx[ib][c * KC];
-            const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
-            const CUtensorMap* map = is_txt ? &mapKt : &mapK;
-            tc::bar_expect_tx(&sm.kfull[st], KBYTES);
-#pragma unroll 1
-            for (int kb = 0; kb < 2; ++kb) {
-#pragma unroll 4
-              for (int r4 = 0; r4 < KC / 4; ++r4) {
-                const int r = r4 * 4;
-                const int y0 = rows[min(r, nv - 1)], y1 = rows[min(r + 1, nv - 1)];
-                const int y2 = rows[min(r + 2, nv - 1)], y3 = rows[min(r + 3, nv - 1)];
-                tc::tma_gather4(sm.k[st] + kb * (KBYTES / 2) + r * 128, map, h * 128 + kb * 64, y0, y1, y2, y3,
-                                &sm.kfull[st]);
-              }
-            }
-            ++kcnt;
+          if (!tc::bar_wait(&sm.qempty[qb], ((qcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
+            fail(sm, p.status);
+            ok = false;
+          } else {
+            tc::bar_expect_tx(&sm.qfull[qb], QBYTES);
+            tc::tma_load_2d(sm.q[qb], &mapQ, h * 128, (int)(g.t0 + g.j0), &sm.qfull[qb]);
+            tc::tma_load_2d(sm.q[qb] + QBYTES / 2, &mapQ, h * 128 + 64, (int)(g.t0 + g.j0), &sm.qfull[qb]);
           }
         }
+        ++qcnt;
+        for (int ci = 0; ci < nch && ok; ++ci) {
+          const int st = kcnt % NST;
+          if (!tc::bar_wait(&sm.kempty[st], ((kcnt / NST) & 1) ^ 1, abort, kLimitNs)) {
+            fail(sm, p.status);
+            ok = false;
+            break;
+          }
+          const bool is_txt = (ci >= g.nic) && (ci < g.nic + g.ntc);
+          const int c = ci < g.nic ? ci : (is_txt ? ci - g.nic : ci - g.nic - g.ntc);
+          const int* rows = is_txt ? &sm.kidx[ib][PMAX + c * KC] : &sm.kidx[ib][c * KC];
+          const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
+          const __nv_bfloat16* base = is_txt ? p.Kt : p.K;
+          uint8_t* dst = sm.k[st];
+#pragma unroll
+          for (int i = 0; i < (KC * 16 + NPROD * 32 - 1) / (NPROD * 32); ++i) {
+            const int q = pt + NPROD * 32 * i;
+            if (q >= KC * 16) break;
+            const int key = q >> 4, c16 = q & 15;
+            const int kb = c16 >> 3, cc = c16 & 7;
+            const bool v = key < nv;
+            const __nv_bfloat16* src = base + (v ? (int64_t)rows[key] * HD + h * 128 + c16 * 8 : 0);
+            tc::cp_async16(dst + kb * (KBYTES / 2) + key * 128 + ((cc ^ (key & 7)) << 4), src, v ? 16 : 0);
+          }
+          tc::cp_async_arrive(&sm.kfull[st]);
+          ++kcnt;
+        }
       }
-      __syncwarp();
+      if (!ok) break;
     }
-    if (lane == 0) {
+    if (pt == 0) {
       sm.issued_k = kcnt;
       sm.issued_q = qcnt;
     }
-  } else if (warp == 1) {
+    asm volatile("cp.async.wait_all;" ::: "memory");
+  } else if (warp == MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       uint32_t qcnt = 0, kcnt = 0, scnt = 0;
@@ -231,6 +246,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
               fail(sm, p.status);
               break;
             }
+            tc::fence_proxy_async();
             tc::fence_after();
             const uint32_t d = tmem + S_COL + sb * KC;
             const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[st]);
@@ -255,13 +271,15 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     }
     __syncwarp();
   } else {
-    // ------------------------------------------------------------ epilogue (warps 2-5)
-    const int ew = warp - 2;            // 0..3
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - EPI_WARP0;    // 0..NEPI-1
+    const int half = ew >> 2;           // which chunks (index parity) this warp takes
     const int quad = warp & 3;          // TMEM lane quadrant this warp may access
     const int j = quad * 32 + lane;     // text row of this thread inside the tile
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const float sl2 = p.scale_log2;
     const float invH = 1.0f / (float)H;
+    const uint32_t sbuf = tmem + lane_base + S_COL + half * KC;
     uint32_t scnt = 0, xcnt = 0;
     int ii = 0;
     for (int item = cid; item < nF; item += ncl, ++ii) {
@@ -269,47 +287,60 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       const int ib = ii & 1;
       if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, nullptr, kLimitNs))) { fail(sm, p.status); break; }
       const bool vrow = g.j0 + j < g.M;
+      const bool wvalid = __any_sync(0xffffffffu, vrow);  // warp-uniform: any real text row here
       const int jj = g.j0 + j;
       bool ok = true;
+      uint32_t pstart = 0;  // chunk counter at the start of the last P pass
       for (int h = 0; h < H && ok; ++h) {
-        // ---- statistics over the CTA's keys
+        // ---- statistics over this warp's chunks of the CTA's keys
         float m = -INFINITY, z = 0.f;
-        for (int ci = 0; ci < g.nic + g.ntc; ++ci) {
-          const int sb = scnt & 1;
-          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[sb], (scnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
-          tc::fence_after();
-          uint32_t v[64];
-          tc::tmem_ld64(tmem + lane_base + S_COL + sb * KC, v);
-          tc::tmem_wait_ld();
-          tc::fence_before();
-          __syncwarp();
-          if (lane == 0) tc::bar_arrive(&sm.sempty[sb]);
-          ++scnt;
-          if (vrow) {
-            const bool is_txt = ci >= g.nic;
-            const int c = is_txt ? ci - g.nic : ci;
-            const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
-            const int tbase = g.txt0 + c * KC;  // sample-relative text index of column 0
-            const int lim = is_txt ? min(nv, jj - tbase + 1) : nv;
-            float cm = -INFINITY;
+        for (int ci = 0; ci < g.nic + g.ntc; ++ci, ++scnt) {
+          if ((int)(scnt & 1) != half) continue;
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[half], (scnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
+          const bool is_txt = ci >= g.nic;
+          const int c = is_txt ? ci - g.nic : ci;
+          const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
+          const int tbase = g.txt0 + c * KC;  // sample-relative text index of column 0
+          const int lim = vrow ? (is_txt ? min(nv, jj - tbase + 1) : nv) : 0;
 #pragma unroll
-            for (int col = 0; col < 64; ++col)
-              if (col < lim) cm = fmaxf(cm, __uint_as_float(v[col]) * sl2);
-            if (cm != -INFINITY) {
-              const float mn = fmaxf(m, cm);
-              float acc = 0.f;
+          for (int hf = 0; hf < 2; ++hf) {
+            uint32_t v[32];
+            if (wvalid) {
+              tc::fence_after();
+              tc::tmem_ld32(sbuf + hf * 32, v);
+              tc::tmem_wait_ld();
+            }
+            if (hf == 1) {
+              tc::fence_before();
+              __syncwarp();
+              if (lane == 0) tc::bar_arrive(&sm.sempty[half]);
+            }
+            const int l2 = lim - hf * 32;  // valid columns in this half
+            if (l2 > 0) {
+              float cm0 = -INFINITY, cm1 = -INFINITY;
 #pragma unroll
-              for (int col = 0; col < 64; ++col)
-                if (col < lim) acc += exp2f(__uint_as_float(v[col]) * sl2 - mn);
-              z = (m == -INFINITY ? 0.f : z * exp2f(m - mn)) + acc;
+              for (int col = 0; col < 32; col += 2) {
+                if (col < l2) cm0 = fmaxf(cm0, __uint_as_float(v[col]));
+                if (col + 1 < l2) cm1 = fmaxf(cm1, __uint_as_float(v[col + 1]));
+              }
+              const float mn = fmaxf(m, fmaxf(cm0, cm1) * sl2);
+              float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+              for (int col = 0; col < 32; col += 4) {
+                if (col < l2) a0 += tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -mn));
+                if (col + 1 < l2) a1 += tc::ex2(fmaf(__uint_as_float(v[col + 1]), sl2, -mn));
+                if (col + 2 < l2) a2 += tc::ex2(fmaf(__uint_as_float(v[col + 2]), sl2, -mn));
+                if (col + 3 < l2) a3 += tc::ex2(fmaf(__uint_as_float(v[col + 3]), sl2, -mn));
+              }
+              z = (m == -INFINITY ? 0.f : z * tc::ex2(m - mn)) + ((a0 + a1) + (a2 + a3));
               m = mn;
             }
           }
         }
         if (!ok) break;
-        // ---- exchange (max, sum) with the cluster
+        // ---- exchange (max, sum) with every epilogue warp of the cluster
         const int slot = xcnt & 1;
-        for (int r = 0; r < C; ++r) tc::st_cluster_f2(&sm.xch[slot][rank][j], (uint32_t)r, m, z);
+        for (int r = 0; r < C; ++r) tc::st_cluster_f2(&sm.xch[slot][rank][half][j], (uint32_t)r, m, z);
         __syncwarp();
         if (lane == 0)
           for (int r = 0; r < C; ++r) tc::bar_arrive_remote(&sm.xbar[slot], (uint32_t)r);
@@ -317,65 +348,84 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         ++xcnt;
         float Mx = -INFINITY;
 #pragma unroll
-        for (int r = 0; r < C; ++r) Mx = fmaxf(Mx, sm.xch[slot][r][j].x);
+        for (int r = 0; r < C; ++r)
+          Mx = fmaxf(Mx, fmaxf(sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x));
         float Z = 0.f;
 #pragma unroll
-        for (int r = 0; r < C; ++r) {
-          const float2 e = sm.xch[slot][r][j];
-          if (e.y > 0.f) Z += e.y * exp2f(e.x - Mx);
-        }
+        for (int r = 0; r < C; ++r)
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            const float2 e = sm.xch[slot][r][hh][j];
+            if (e.y > 0.f) Z += e.y * tc::ex2(e.x - Mx);
+          }
         const float f = (Z > 0.f) ? 1.0f / Z : 0.f;
         // ---- probabilities of the CTA's S1 keys, summed over heads in TMEM
-        for (int c = 0; c < g.nic; ++c) {
-          const int sb = scnt & 1;
-          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[sb], (scnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
-          tc::fence_after();
-          uint32_t v[64];
-          tc::tmem_ld64(tmem + lane_base + S_COL + sb * KC, v);
-          tc::tmem_wait_ld();
-          tc::fence_before();
-          __syncwarp();
-          if (lane == 0) tc::bar_arrive(&sm.sempty[sb]);
-          ++scnt;
-          const int nv = min(KC, g.own_img - c * KC);
+        pstart = scnt;
+        for (int c = 0; c < g.nic; ++c, ++scnt) {
+          if ((int)(scnt & 1) != half) continue;
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[half], (scnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
           const uint32_t pa = tmem + lane_base + P_COL + c * KC;
-          uint32_t w[64];
-          if (h > 0) {
-            tc::tmem_ld64(pa, w);
-            tc::tmem_wait_ld();
-          }
+          const int nv = min(KC, g.own_img - c * KC);
+          const float mf = vrow ? Mx : INFINITY;   // rows past M contribute 0
+          // two halves of 32 columns keep the live registers down
 #pragma unroll
-          for (int col = 0; col < 64; ++col) {
-            const float pv = (vrow && col < nv) ? exp2f(__uint_as_float(v[col]) * sl2 - Mx) * f : 0.f;
-            w[col] = __float_as_uint(h > 0 ? __uint_as_float(w[col]) + pv : pv);
+          for (int hf = 0; hf < 2; ++hf) {
+            uint32_t v[32], w[32];
+            if (wvalid) {
+              tc::fence_after();
+              tc::tmem_ld32(sbuf + hf * 32, v);
+              if (h > 0) tc::tmem_ld32(pa + hf * 32, w);
+              tc::tmem_wait_ld();
+            }
+            if (hf == 1) {  // the S buffer is free once both halves are in registers
+              tc::fence_before();
+              __syncwarp();
+              if (lane == 0) tc::bar_arrive(&sm.sempty[half]);
+            }
+            if (wvalid) {
+#pragma unroll
+              for (int col = 0; col < 32; ++col) {
+                const float pv = (hf * 32 + col < nv) ? tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -mf)) * f : 0.f;
+                w[col] = __float_as_uint(h > 0 ? __uint_as_float(w[col]) + pv : pv);
+              }
+              tc::tmem_st32(pa + hf * 32, w);
+            }
           }
-          tc::tmem_st64(pa, w);
         }
-        tc::tmem_wait_st();
+        if (wvalid) tc::tmem_wait_st();
+        // order this warp's P stores before the next head's exchange arrival
+        tc::fence_before();
       }
       if (!ok) { fail(sm, p.status); break; }
-      // ---- column reductions of P over this warp's 32 valid rows: column max
-      // -> s2 (atomicMax), register columns -> this warp's partial of s2(r)
+      // ---- column reductions of P over this warp's 32 rows, for the chunks
+      // this warp wrote in the last head (so no other warp's stores are
+      // involved): column max -> s2 (atomicMax), register columns -> this
+      // warp's partial of s2(r)
       float regacc = 0.f;
-      for (int c = 0; c < g.nic; ++c) {
-        uint32_t w[64];
-        tc::tmem_ld64(tmem + lane_base + P_COL + c * KC, w);
-        tc::tmem_wait_ld();
-        const int nv = min(KC, g.own_img - c * KC);
+      if (wvalid) {
+        tc::fence_after();
+        for (int c = (int)((pstart + half) & 1); c < g.nic; c += 2) {
+          const int nv = min(KC, g.own_img - c * KC);
+          for (int hf = 0; hf < 2; ++hf) {
+            uint32_t w[32];
+            tc::tmem_ld32(tmem + lane_base + P_COL + c * KC + hf * 32, w);
+            tc::tmem_wait_ld();
 #pragma unroll
-        for (int col = 0; col < 64; ++col) {
-          const float x = vrow ? __uint_as_float(w[col]) : 0.f;
-          const float mx = warp_max_f(x);
-          const float su = warp_sum_f(x);
-          if (lane == 0 && col < nv) {
-            const int key = c * KC + col;
-            if (sm.kreg[ib][key]) regacc += su * invH;
-            else atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(mx * invH));
+            for (int col = 0; col < 32; ++col) {
+              const float x = vrow ? __uint_as_float(w[col]) : 0.f;
+              const float mx = warp_max_f(x);
+              const float su = warp_sum_f(x);
+              if (lane == 0 && hf * 32 + col < nv) {
+                const int key = c * KC + hf * 32 + col;
+                if (sm.kreg[ib][key]) regacc += su * invH;
+                else atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(mx * invH));
+              }
+            }
           }
         }
       }
       if (lane == 0) {
-        p.refpart[g.slot + rank * 4 + ew] = regacc;
+        p.refpart[g.slot + rank * NEPI + ew] = regacc;
         __threadfence();
         const int nslots = p.slot_off[g.b + 1] - p.slot_off[g.b];
         if (atomicAdd(&p.done[g.b], 1) == nslots - 1) {
@@ -397,17 +447,15 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   tc::fence_before();
   __syncthreads();
   if (sm.abort && tid == 0) {
-    // drain the last copies issued into each buffer (the earlier ones were
-    // consumed): this CTA's shared memory must outlive them
-    const uint32_t k1 = sm.issued_k, q1 = sm.issued_q;
-    for (uint32_t i = (k1 > NST ? k1 - NST : 0); i < k1; ++i)
-      tc::bar_wait(&sm.kfull[i % NST], (i / NST) & 1, nullptr, kLimitNs / 8);
+    // drain the last query-tile copies (TMA) issued into each buffer; the
+    // producers' cp.async copies were drained by cp.async.wait_all
+    const uint32_t q1 = sm.issued_q;
     for (uint32_t i = (q1 > 2 ? q1 - 2 : 0); i < q1; ++i)
       tc::bar_wait(&sm.qfull[i & 1], (i >> 1) & 1, nullptr, kLimitNs / 8);
   }
   __syncthreads();
   tc::fence_after();
-  if (warp == 1) tc::tmem_dealloc(tmem, TMEM_COLS);
+  if (warp == MMA_WARP) tc::tmem_dealloc(tmem, TMEM_COLS);
   // peers may still write into this CTA's exchange buffers until here
   tc::cluster_sync_all();
 }
