@@ -51,10 +51,11 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   L.maxA = B * tps * nhg;
   L.maxB = B * tps * chmax;
   L.maxF = B * cdiv(b->max_text, 128);
-  L.maxSlots = L.maxB + L.maxF * kFusedSlotsPerItem;
+  L.maxSlots = L.maxB + L.maxF * kFusedSlotsPerItem8;
   L.itemsA = take(L.maxA * 16);
   L.itemsB = take(L.maxB * 16);
   L.itemsF = take(L.maxF * 16);
+  L.itemsF8 = take(L.maxF * 16);
   L.itemB_off = take((B + 1) * 4);
   L.slot_off = take((B + 1) * 4);
   L.stats2 = take(T * (H2 > 0 ? H2 : 1) * 8);
@@ -125,7 +126,6 @@ int num_sms() {
 void set_smem_attrs() {
   static std::once_flag once;
   std::call_once(once, [] {
-    cudaFuncSetAttribute(s2_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes());
     cudaFuncSetAttribute(stage1_cls_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          stage1_cls_smem_bytes());
     cudaFuncSetAttribute(s2_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_stats_smem_bytes());
@@ -331,6 +331,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
   p.status = at<int>(ws, L.status);
   const bool fused = fused_enabled() && L.maxF > 0 && b->total_text > 0;
   p.itemsF = at<int4>(ws, L.itemsF);
+  p.itemsF8 = at<int4>(ws, L.itemsF8);
   p.slot_off = at<int32_t>(ws, L.slot_off);
   p.maxF = L.maxF;
   p.use_fused = fused ? 1 : 0;
@@ -364,20 +365,12 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     q.tau2 = p.tau2;
     q.lambda2 = lambda2;
     q.status = p.status;
-    const int ncl = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / kFusedCluster));
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(ncl * kFusedCluster));
-    cfg.blockDim = dim3(s2_fused_threads());
-    cfg.dynamicSmemBytes = s2_fused_smem_bytes();
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = kFusedCluster;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    OCCAM_CUDA(cudaLaunchKernelEx(&cfg, s2_fused_kernel, mq, mk, mkt, q));
+    const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
+    if (launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
+    q.items = p.itemsF8;
+    const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
+    if (launch_fused(8, mq, mk, mkt, q, ncl8, st) != 0) return OCCAM_ERR_CUDA;
+
   }
   trace.mark(st);
   const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);

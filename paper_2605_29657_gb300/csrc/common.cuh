@@ -179,13 +179,13 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
 // Workspace carve-up (byte offsets from the workspace base; see ws_layout()).
 struct WsLayout {
   size_t status, counters, role, keep1, s1, s2, ref1, s1_list, n1_seg, dense, n1, n1_vis;
-  size_t itemsA, itemsB, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, stats1, itemsF, slot_off;
+  size_t itemsA, itemsB, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, stats1, itemsF, itemsF8, slot_off;
   size_t total;
   int64_t maxA, maxB, maxF, maxSlots, scan_tiles, stats1_rows;
 };
 
 // counters block (int32 slots)
-enum { CNT_DENSE_DONE = 0, CNT_SCAN_TICKET = 1, CNT_NA = 2, CNT_NB = 3, CNT_NF = 4, CNT_SLOTS = 5 };
+enum { CNT_DENSE_DONE = 0, CNT_SCAN_TICKET = 1, CNT_NA = 2, CNT_NB = 3, CNT_NF = 4, CNT_NF8 = 5, CNT_SLOTS = 6 };
 
 constexpr int kTextTile = 64;    // Stage-II text rows per item
 constexpr int kHeadGroup = 8;    // Stage-II heads per stats item

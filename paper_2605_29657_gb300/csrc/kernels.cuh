@@ -7,11 +7,12 @@
 
 namespace occam {
 
-constexpr int kFusedCluster = 4;        // CTAs per cluster of the fused tcgen05 Stage-II kernel
-constexpr int kFusedMaxOwnImg = 384;    // S1 keys one of its CTAs can hold (TMEM columns)
+constexpr int kFusedCluster = 4;        // CTAs per cluster of the fused tcgen05 Stage-II kernel (C = 8 variant for larger S1)
+constexpr int kFusedMaxOwnImg = 192;    // S1 keys one of its CTAs can hold (two TMEM buffers of this many columns)
 constexpr int kFusedMaxOwnTxt = 256;    // text keys one of its CTAs can take
 constexpr int kFusedEpiWarps = 8;       // epilogue warps per CTA of the fused kernel
-constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedEpiWarps;  // s2(r) partials per item (one per epilogue warp)
+constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedEpiWarps;  // s2(r) partials per C=4 item (one per epilogue warp)
+constexpr int kFusedSlotsPerItem8 = 8 * kFusedEpiWarps;             // and per C=8 item
 constexpr int kMaxClsRowsPerCta = 512;  // rows of one segment handled by one CTA of a [CLS] cluster
 constexpr int kMaxClusterCls = 8;       // portable cluster size
 
@@ -86,7 +87,8 @@ struct Stage2Params {
   float* s2;                // atomicMax accumulator, zeroed beforehand
   float* refpart;           // [maxB]
   int32_t* done;            // [B] finished score items per sample (zeroed)
-  int4* itemsF;             // fused items (b, j0, slot, -)
+  int4* itemsF;             // fused items for 4-CTA clusters (b, j0, slot, -)
+  int4* itemsF8;            // fused items for 8-CTA clusters
   int use_fused;            // route eligible samples to the fused tensor-core kernel
   int32_t* slot_off;        // [B+1] partial-slot range of each sample
   int64_t maxF;
@@ -167,9 +169,9 @@ int s2_scores_smem_bytes();
 int s2_stats_smem_bytes();
 
 // stage2_tc.cu
-__global__ void s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
-                                const __grid_constant__ CUtensorMap mapKt, Stage2TcParams p);
-int s2_fused_smem_bytes();
+int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt,
+                 const Stage2TcParams& q, int nclusters, cudaStream_t st);
+int s2_fused_smem_bytes(int C);
 int s2_fused_threads();
 
 // compact.cu

@@ -6,27 +6,32 @@
 // of q_{j,h} k^T / sqrt(d2); P[j, v] = sum_h A_{j,h}(v); s2(v) = max_j P[j, v] / H
 // for visual S1 rows and the registers' sum_j P[j, r] / H for s2(r).
 //
-// Work item = (sample, tile of 128 text rows), processed by one cluster of 4
-// CTAs. The text rows are the 128 TMEM lanes; each CTA owns a quarter of the
-// sample's S1 keys and of the causal text keys. Per head:
+// Work item = (sample, tile of 128 text rows), processed by one cluster of C
+// CTAs (C = 4, or 8 for samples with more S1 keys). The text rows are the 128
+// TMEM lanes; each CTA owns 1/C of the sample's S1 keys and of the causal
+// text keys. Per head:
 //   1. three producer warps stream the CTA's key rows in 64-key chunks with
 //      16-byte cp.async into the 128-byte-swizzled operand layout (S1 rows
-//      are gathered by index straight from K2: pruned rows are never read),
-//      and the head's 128 x 128 query tile arrives by TMA;
-//   2. the MMA warp computes S = Q K^T per chunk into a TMEM buffer;
+//      are gathered by index straight from K2: pruned rows are never read,
+//      every key row is read once per text tile); the head's 128 x 128 query
+//      tile arrives by TMA;
+//   2. one thread issues S = Q K^T per chunk (tcgen05.mma, bf16 in, fp32 in
+//      TMEM); S1-key chunks land in a per-head TMEM buffer E (two buffers,
+//      alternating by head), text-key chunks in a scratch TMEM buffer;
 //   3. eight epilogue warps (two per TMEM lane quadrant, one thread per text
-//      row, taking alternate chunks) keep the row's running softmax max / sum
-//      over their chunks, then exchange them with every epilogue warp of the
-//      cluster through distributed shared memory, so every CTA holds the
-//      exact per-row max and sum over all keys of the head;
-//   4. the image chunks are multiplied again (S is recomputed from shared
-//      memory) and exp(l - max) / sum is accumulated into the head-summed
-//      probabilities P, which live in TMEM for the whole item.
-// After the last head every CTA reduces its P columns over the valid rows:
+//      row, each taking one 32-column half of every chunk) turn S into
+//      exp2(l - cmax) (cmax: the half-chunk's row max, kept in shared
+//      memory), write it back over S in E, and keep the row's running
+//      softmax max / sum;
+//   4. the (max, sum) pairs are exchanged with every epilogue warp of the
+//      cluster through distributed shared memory. The exchange of head h is
+//      awaited only after head h+1's statistics, so its latency is hidden;
+//   5. then every warp adds exp2(cmax - max) / sum * E to the head-summed
+//      probabilities P of its 96 S1-key columns, which live in registers for
+//      the whole item.
+// After the last head every warp reduces its P columns over its 32 rows:
 // column max -> s2 (atomicMax on the fp32 bit pattern, exact and order-free
 // since P >= 0), register columns -> a partial of s2(r) reduced in fixed order.
-// Each key row of K2 is read from HBM once per text tile; the second pass
-// over a head's chunks hits L2.
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc5.cuh"
@@ -34,40 +39,48 @@
 namespace occam {
 
 namespace s2f {
-constexpr int C = kFusedCluster;       // CTAs per cluster
 constexpr int QR = 128;                // text rows per item (TMEM lanes)
 constexpr int KC = 64;                 // keys per chunk (MMA N)
 constexpr int NST = 4;                 // key-chunk ring stages
-constexpr int PMAX = kFusedMaxOwnImg;  // max S1 keys per CTA (P columns)
+constexpr int PMAX = kFusedMaxOwnImg;  // max S1 keys per CTA
+constexpr int NIC_MAX = PMAX / KC;     // S1-key chunks per CTA
 constexpr int TMAX = kFusedMaxOwnTxt;  // max text keys per CTA
 constexpr int QBYTES = QR * 256;       // one head's query tile: 2 K-blocks x 128 rows x 128 B
 constexpr int KBYTES = KC * 256;       // one chunk: 2 K-blocks x 64 rows x 128 B
 constexpr int NPROD = 3;               // producer warps (0-2); warp 3 issues MMAs; then the epilogue warps
 constexpr int MMA_WARP = NPROD;
 constexpr int EPI_WARP0 = NPROD + 1;
-constexpr int NEPI = kFusedEpiWarps;   // two per TMEM lane quadrant; half h takes chunks with (index & 1) == h
+constexpr int NEPI = kFusedEpiWarps;   // two per TMEM lane quadrant
+constexpr int PCOLS = PMAX / 2;        // P columns per epilogue warp (registers)
 constexpr int THREADS = (NPROD + 1 + NEPI) * 32;
+constexpr int NXS = 4;                 // exchange slots (the exchange runs one head behind)
 constexpr uint32_t IDESC = tc::idesc_bf16(128, KC);
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int S_COL = 0;               // two S buffers of KC columns
-constexpr int P_COL = 2 * KC;          // P: PMAX columns
+constexpr int S_COL = 0;               // two scratch buffers (text-key chunks), KC columns each
+constexpr int E_COL = 2 * KC;          // two E buffers (by head parity), PMAX columns each
+static_assert(E_COL + 2 * PMAX <= (int)TMEM_COLS, "TMEM budget");
+static_assert(PMAX % (2 * 32) == 0 && PCOLS % 32 == 0, "P columns split into 32-column pieces");
 constexpr uint64_t kLimitNs = 2000000000ull;
-static_assert(P_COL + PMAX <= (int)TMEM_COLS, "TMEM budget");
 
+template <int C>
 struct Smem {
   uint8_t q[2][QBYTES];
   uint8_t k[NST][KBYTES];
   int32_t kidx[2][PMAX + TMAX];
-  float2 xch[2][C][2][QR];
+  float2 xch[NXS][C][2][QR];          // (max, sum) per (slot, CTA, epilogue half, row)
+  float cmx[2][NIC_MAX][2][QR];       // half-chunk row max (log2 units) per (head parity, chunk, half, row)
   uint8_t kreg[2][PMAX];
-  uint64_t kfull[NST], kempty[NST], qfull[2], qempty[2], sfull[2], sempty[2], xbar[2], iready[2], idone[2], mdone;
+  uint64_t kfull[NST], kempty[NST], qfull[2], qempty[2], sfull[2], sempty[2], efree[2], xbar[NXS], iready[2],
+      idone[2], mdone;
   uint32_t tmem_base;
   int abort;
-  uint32_t issued_k, issued_q;  // producer's final counters (for the drain after an abort)
+  uint32_t issued_q;
 };
 }  // namespace s2f
 
-int s2_fused_smem_bytes() { return (int)sizeof(s2f::Smem) + 1024; }
+int s2_fused_smem_bytes(int C) {
+  return (int)(C == 8 ? sizeof(s2f::Smem<8>) : sizeof(s2f::Smem<4>)) + 1024;
+}
 int s2_fused_threads() { return s2f::THREADS; }
 
 namespace {
@@ -77,6 +90,7 @@ struct ItemGeom {
   int64_t rbase, t0;
 };
 
+template <int C>
 __device__ __forceinline__ ItemGeom item_geom(const Stage2TcParams& p, int4 it, int rank) {
   using namespace s2f;
   ItemGeom g;
@@ -99,7 +113,8 @@ __device__ __forceinline__ ItemGeom item_geom(const Stage2TcParams& p, int4 it, 
   return g;
 }
 
-__device__ __forceinline__ void fail(s2f::Smem& sm, int* status) {
+template <class SM>
+__device__ __forceinline__ void fail(SM& sm, int* status) {
   sm.abort = 1;
   set_status(status, OCCAM_ERR_TIMEOUT);
 }
@@ -117,17 +132,20 @@ __device__ __forceinline__ float warp_sum_f(float v) {
 
 }  // namespace
 
+template <int C>
 __global__ void __launch_bounds__(s2f::THREADS, 1)
     s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
                     const __grid_constant__ CUtensorMap mapKt, Stage2TcParams p) {
   using namespace s2f;
   extern __shared__ unsigned char smem_raw[];
-  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Smem<C>& sm = *reinterpret_cast<Smem<C>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rank = (int)tc::cluster_rank();
-  const int nF = p.counters[CNT_NF];
+  const int nF = p.counters[C == 8 ? CNT_NF8 : CNT_NF];
   const int cid = (int)tc::cluster_id_x(), ncl = (int)tc::nclusters_x();
   volatile int* abort = &sm.abort;
+  (void)mapK;
+  (void)mapKt;
 
   if (tid == 0) {
     for (int i = 0; i < NST; ++i) { tc::bar_init(&sm.kfull[i], NPROD * 32); tc::bar_init(&sm.kempty[i], 1); }
@@ -135,19 +153,17 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       tc::bar_init(&sm.qfull[i], 1);
       tc::bar_init(&sm.qempty[i], 1);
       tc::bar_init(&sm.sfull[i], 1);
-      tc::bar_init(&sm.sempty[i], 4);
-      tc::bar_init(&sm.xbar[i], NEPI * C);
+      tc::bar_init(&sm.sempty[i], NEPI);
+      tc::bar_init(&sm.efree[i], NEPI);
       tc::bar_init(&sm.iready[i], NPROD * 32);
       tc::bar_init(&sm.idone[i], NEPI);
     }
+    for (int i = 0; i < NXS; ++i) tc::bar_init(&sm.xbar[i], NEPI * C);
     tc::bar_init(&sm.mdone, 1);
     sm.abort = 0;
-    sm.issued_k = 0;
     sm.issued_q = 0;
     tc::bar_fence_init();
     tc::prefetch_map(&mapQ);
-    tc::prefetch_map(&mapK);
-    tc::prefetch_map(&mapKt);
   }
   if (warp == MMA_WARP) tc::tmem_alloc(&sm.tmem_base, TMEM_COLS);
   tc::fence_before();
@@ -168,7 +184,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     int ii = 0;
     const int64_t HD = (int64_t)H * 128;
     for (int item = cid; item < nF; item += ncl, ++ii) {
-      const ItemGeom g = item_geom(p, p.items[item], rank);
+      const ItemGeom g = item_geom<C>(p, p.items[item], rank);
       const int ib = ii & 1;
       if (*abort || !tc::bar_wait(&sm.idone[ib], ((ii >> 1) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
       for (int i = pt; i < g.own_img; i += NPROD * 32) {
@@ -179,7 +195,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       for (int i = pt; i < g.own_txt; i += NPROD * 32) sm.kidx[ib][PMAX + i] = (int)(g.t0 + g.txt0 + i);
       tc::bar_arrive(&sm.iready[ib]);
       if (!tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-      const int nch = 2 * g.nic + g.ntc;
+      const int nch = g.nic + g.ntc;
       bool ok = true;
       for (int h = 0; h < H && ok; ++h) {
         if (pt == 0) {
@@ -201,8 +217,8 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             ok = false;
             break;
           }
-          const bool is_txt = (ci >= g.nic) && (ci < g.nic + g.ntc);
-          const int c = ci < g.nic ? ci : (is_txt ? ci - g.nic : ci - g.nic - g.ntc);
+          const bool is_txt = ci < g.ntc;  // text chunks first: they do not wait for an E buffer
+          const int c = is_txt ? ci : ci - g.ntc;
           const int* rows = is_txt ? &sm.kidx[ib][PMAX + c * KC] : &sm.kidx[ib][c * KC];
           const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
           const __nv_bfloat16* base = is_txt ? p.Kt : p.K;
@@ -210,12 +226,13 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
 #pragma unroll
           for (int i = 0; i < (KC * 16 + NPROD * 32 - 1) / (NPROD * 32); ++i) {
             const int q = pt + NPROD * 32 * i;
-            if (q >= KC * 16) break;
-            const int key = q >> 4, c16 = q & 15;
-            const int kb = c16 >> 3, cc = c16 & 7;
-            const bool v = key < nv;
-            const __nv_bfloat16* src = base + (v ? (int64_t)rows[key] * HD + h * 128 + c16 * 8 : 0);
-            tc::cp_async16(dst + kb * (KBYTES / 2) + key * 128 + ((cc ^ (key & 7)) << 4), src, v ? 16 : 0);
+            if (q < KC * 16) {
+              const int key = q >> 4, c16 = q & 15;
+              const int kb = c16 >> 3, cc = c16 & 7;
+              const bool v = key < nv;
+              const __nv_bfloat16* src = base + (v ? (int64_t)rows[key] * HD + h * 128 + c16 * 8 : 0);
+              tc::cp_async16(dst + kb * (KBYTES / 2) + key * 128 + ((cc ^ (key & 7)) << 4), src, v ? 16 : 0);
+            }
           }
           tc::cp_async_arrive(&sm.kfull[st]);
           ++kcnt;
@@ -223,22 +240,26 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       }
       if (!ok) break;
     }
-    if (pt == 0) {
-      sm.issued_k = kcnt;
-      sm.issued_q = qcnt;
-    }
+    if (pt == 0) sm.issued_q = qcnt;
     asm volatile("cp.async.wait_all;" ::: "memory");
   } else if (warp == MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      uint32_t qcnt = 0, kcnt = 0, scnt = 0;
+      uint32_t qcnt = 0, kcnt = 0, scnt = 0, hk = 0;
       for (int item = cid; item < nF && !*abort; item += ncl) {
-        const ItemGeom g = item_geom(p, p.items[item], rank);
-        const int nch = 2 * g.nic + g.ntc;
-        for (int h = 0; h < H && !*abort; ++h) {
+        const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+        const int nch = g.nic + g.ntc;
+        for (int h = 0; h < H && !*abort; ++h, ++hk) {
           const int qb = qcnt & 1;
           if (!tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
+          const uint32_t ebuf = tmem + E_COL + (hk & 1) * PMAX;
           for (int ci = 0; ci < nch; ++ci) {
+            // E[hk & 1] is free once the probabilities of head hk - 2 were read out of it
+            if (ci == g.ntc && hk >= 2 &&
+                !tc::bar_wait(&sm.efree[hk & 1], ((hk - 2) >> 1) & 1, abort, kLimitNs)) {
+              fail(sm, p.status);
+              break;
+            }
             const int st = kcnt % NST;
             const int sb = scnt & 1;
             if (!tc::bar_wait(&sm.kfull[st], (kcnt / NST) & 1, abort, kLimitNs) ||
@@ -248,7 +269,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             }
             tc::fence_proxy_async();
             tc::fence_after();
-            const uint32_t d = tmem + S_COL + sb * KC;
+            const uint32_t d = ci >= g.ntc ? ebuf + (ci - g.ntc) * KC : tmem + S_COL + sb * KC;
             const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[st]);
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
@@ -273,159 +294,167 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   } else {
     // ------------------------------------------------------------ epilogue
     const int ew = warp - EPI_WARP0;    // 0..NEPI-1
-    const int half = ew >> 2;           // which chunks (index parity) this warp takes
+    const int half = ew >> 2;           // chunk parity this warp takes; also its P column half
     const int quad = warp & 3;          // TMEM lane quadrant this warp may access
     const int j = quad * 32 + lane;     // text row of this thread inside the tile
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const float sl2 = p.scale_log2;
     const float invH = 1.0f / (float)H;
-    const uint32_t sbuf = tmem + lane_base + S_COL + half * KC;
-    uint32_t scnt = 0, xcnt = 0;
+    uint32_t scnt = 0, hk = 0;
     int ii = 0;
     for (int item = cid; item < nF; item += ncl, ++ii) {
-      const ItemGeom g = item_geom(p, p.items[item], rank);
+      const ItemGeom g = item_geom<C>(p, p.items[item], rank);
       const int ib = ii & 1;
       if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, nullptr, kLimitNs))) { fail(sm, p.status); break; }
       const bool vrow = g.j0 + j < g.M;
       const bool wvalid = __any_sync(0xffffffffu, vrow);  // warp-uniform: any real text row here
       const int jj = g.j0 + j;
-      bool ok = true;
-      uint32_t pstart = 0;  // chunk counter at the start of the last P pass
-      for (int h = 0; h < H && ok; ++h) {
-        // ---- statistics over this warp's chunks of the CTA's keys
-        float m = -INFINITY, z = 0.f;
-        for (int ci = 0; ci < g.nic + g.ntc; ++ci, ++scnt) {
-          if ((int)(scnt & 1) != half) continue;
-          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[half], (scnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
-          const bool is_txt = ci >= g.nic;
-          const int c = is_txt ? ci - g.nic : ci;
-          const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
-          const int tbase = g.txt0 + c * KC;  // sample-relative text index of column 0
-          const int lim = vrow ? (is_txt ? min(nv, jj - tbase + 1) : nv) : 0;
+      float P[PCOLS / 32][32];
 #pragma unroll
-          for (int hf = 0; hf < 2; ++hf) {
-            uint32_t v[32];
+      for (int a = 0; a < PCOLS / 32; ++a)
+#pragma unroll
+        for (int b2 = 0; b2 < 32; ++b2) P[a][b2] = 0.f;
+      bool ok = true;
+      for (int step = 0; step <= H && ok; ++step) {
+        const uint32_t hcur = hk + step;  // global index of head `step` of this item
+        if (step < H) {
+          // ---- statistics of head `step` over this warp's chunks
+          const int eb = hcur & 1;
+          float m = -INFINITY, z = 0.f;
+          for (int ci = 0; ci < g.nic + g.ntc; ++ci, ++scnt) {
+            const int sb = scnt & 1;
+            if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[sb], (scnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
+            const bool is_txt = ci < g.ntc;
+            const int c = is_txt ? ci : ci - g.ntc;
+            const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
+            const int tbase = g.txt0 + c * KC + half * 32;  // sample-relative text index of this half's column 0
+            // valid columns of this warp's half of the chunk
+            const int lim = vrow ? (is_txt ? min(nv - half * 32, jj - tbase + 1) : nv - half * 32) : 0;
+            const uint32_t sa = lane_base + half * 32 + (is_txt ? tmem + S_COL + sb * KC : tmem + E_COL + eb * PMAX + c * KC);
             if (wvalid) {
               tc::fence_after();
-              tc::tmem_ld32(sbuf + hf * 32, v);
+              uint32_t v[32];
+              tc::tmem_ld32(sa, v);
               tc::tmem_wait_ld();
-            }
-            if (hf == 1) {
-              tc::fence_before();
-              __syncwarp();
-              if (lane == 0) tc::bar_arrive(&sm.sempty[half]);
-            }
-            const int l2 = lim - hf * 32;  // valid columns in this half
-            if (l2 > 0) {
-              float cm0 = -INFINITY, cm1 = -INFINITY;
+              float c0 = -INFINITY, c1 = -INFINITY;
 #pragma unroll
               for (int col = 0; col < 32; col += 2) {
-                if (col < l2) cm0 = fmaxf(cm0, __uint_as_float(v[col]));
-                if (col + 1 < l2) cm1 = fmaxf(cm1, __uint_as_float(v[col + 1]));
+                if (col < lim) c0 = fmaxf(c0, __uint_as_float(v[col]));
+                if (col + 1 < lim) c1 = fmaxf(c1, __uint_as_float(v[col + 1]));
               }
-              const float mn = fmaxf(m, fmaxf(cm0, cm1) * sl2);
-              float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+              const float cm = fmaxf(c0, c1) * sl2;
+              float a0 = 0.f, a1 = 0.f;
 #pragma unroll
-              for (int col = 0; col < 32; col += 4) {
-                if (col < l2) a0 += tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -mn));
-                if (col + 1 < l2) a1 += tc::ex2(fmaf(__uint_as_float(v[col + 1]), sl2, -mn));
-                if (col + 2 < l2) a2 += tc::ex2(fmaf(__uint_as_float(v[col + 2]), sl2, -mn));
-                if (col + 3 < l2) a3 += tc::ex2(fmaf(__uint_as_float(v[col + 3]), sl2, -mn));
+              for (int col = 0; col < 32; col += 2) {
+                const float e0 = (col < lim) ? tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -cm)) : 0.f;
+                const float e1 = (col + 1 < lim) ? tc::ex2(fmaf(__uint_as_float(v[col + 1]), sl2, -cm)) : 0.f;
+                a0 += e0;
+                a1 += e1;
+                v[col] = __float_as_uint(e0);
+                v[col + 1] = __float_as_uint(e1);
               }
-              z = (m == -INFINITY ? 0.f : z * tc::ex2(m - mn)) + ((a0 + a1) + (a2 + a3));
-              m = mn;
+              if (!is_txt) {
+                tc::tmem_st32(sa, v);  // E <- exp2(l - cmax); completion awaited before the exchange
+                sm.cmx[eb][c][half][j] = cm;
+              }
+              if (cm != -INFINITY) {
+                const float mn = fmaxf(m, cm);
+                z = (m == -INFINITY ? 0.f : z * tc::ex2(m - mn)) + (a0 + a1) * tc::ex2(cm - mn);
+                m = mn;
+              }
             }
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) tc::bar_arrive(&sm.sempty[sb]);
           }
+          if (wvalid) tc::tmem_wait_st();
+          tc::fence_before();
+          if (!ok) break;
+          // ---- post this head's (max, sum) to every epilogue warp of the cluster
+          const int slot = hcur & (NXS - 1);
+          for (int r = 0; r < C; ++r) tc::st_cluster_f2(&sm.xch[slot][rank][half][j], (uint32_t)r, m, z);
+          __syncwarp();
+          if (lane == 0)
+            for (int r = 0; r < C; ++r) tc::bar_arrive_remote(&sm.xbar[slot], (uint32_t)r);
         }
-        if (!ok) break;
-        // ---- exchange (max, sum) with every epilogue warp of the cluster
-        const int slot = xcnt & 1;
-        for (int r = 0; r < C; ++r) tc::st_cluster_f2(&sm.xch[slot][rank][half][j], (uint32_t)r, m, z);
-        __syncwarp();
-        if (lane == 0)
-          for (int r = 0; r < C; ++r) tc::bar_arrive_remote(&sm.xbar[slot], (uint32_t)r);
-        if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (xcnt >> 1) & 1, nullptr, kLimitNs, true))) { ok = false; break; }
-        ++xcnt;
-        float Mx = -INFINITY;
+        if (step >= 1) {
+          // ---- probabilities of head step-1, added into P
+          const uint32_t hp = hcur - 1;
+          const int slot = hp & (NXS - 1);
+          const int eb = hp & 1;
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (hp / NXS) & 1, nullptr, kLimitNs, true))) { ok = false; break; }
+          if (wvalid) {
+            float Mx = -INFINITY;
 #pragma unroll
-        for (int r = 0; r < C; ++r)
-          Mx = fmaxf(Mx, fmaxf(sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x));
-        float Z = 0.f;
+            for (int r = 0; r < C; ++r)
+              Mx = fmaxf(Mx, fmaxf(sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x));
+            float Z = 0.f;
 #pragma unroll
-        for (int r = 0; r < C; ++r)
+            for (int r = 0; r < C; ++r)
 #pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            const float2 e = sm.xch[slot][r][hh][j];
-            if (e.y > 0.f) Z += e.y * tc::ex2(e.x - Mx);
-          }
-        const float f = (Z > 0.f) ? 1.0f / Z : 0.f;
-        // ---- probabilities of the CTA's S1 keys, summed over heads in TMEM
-        pstart = scnt;
-        for (int c = 0; c < g.nic; ++c, ++scnt) {
-          if ((int)(scnt & 1) != half) continue;
-          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[half], (scnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
-          const uint32_t pa = tmem + lane_base + P_COL + c * KC;
-          const int nv = min(KC, g.own_img - c * KC);
-          const float mf = vrow ? Mx : INFINITY;   // rows past M contribute 0
-          // two halves of 32 columns keep the live registers down
-#pragma unroll
-          for (int hf = 0; hf < 2; ++hf) {
-            uint32_t v[32], w[32];
-            if (wvalid) {
-              tc::fence_after();
-              tc::tmem_ld32(sbuf + hf * 32, v);
-              if (h > 0) tc::tmem_ld32(pa + hf * 32, w);
-              tc::tmem_wait_ld();
-            }
-            if (hf == 1) {  // the S buffer is free once both halves are in registers
-              tc::fence_before();
-              __syncwarp();
-              if (lane == 0) tc::bar_arrive(&sm.sempty[half]);
-            }
-            if (wvalid) {
-#pragma unroll
-              for (int col = 0; col < 32; ++col) {
-                const float pv = (hf * 32 + col < nv) ? tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -mf)) * f : 0.f;
-                w[col] = __float_as_uint(h > 0 ? __uint_as_float(w[col]) + pv : pv);
+              for (int hh = 0; hh < 2; ++hh) {
+                const float2 e = sm.xch[slot][r][hh][j];
+                if (e.y > 0.f) Z += e.y * tc::ex2(e.x - Mx);
               }
-              tc::tmem_st32(pa + hf * 32, w);
+            const float invZ = (vrow && Z > 0.f) ? 1.0f / Z : 0.f;
+            tc::fence_after();
+#pragma unroll
+            for (int pc = 0; pc < PCOLS / 32; ++pc) {
+              const int col0 = half * PCOLS + pc * 32;
+              const int c = col0 / KC;
+              if (c < g.nic) {
+                const float cmc = sm.cmx[eb][c][(col0 / 32) & 1][j];
+                const float f = (invZ > 0.f && cmc != -INFINITY) ? tc::ex2(cmc - Mx) * invZ : 0.f;
+                uint32_t v[32];
+                tc::tmem_ld32(tmem + lane_base + E_COL + eb * PMAX + col0, v);
+                tc::tmem_wait_ld();
+#pragma unroll
+                for (int col = 0; col < 32; ++col) P[pc][col] = fmaf(__uint_as_float(v[col]), f, P[pc][col]);
+              }
             }
           }
+          tc::fence_before();
+          __syncwarp();
+          if (lane == 0) tc::bar_arrive(&sm.efree[eb]);
         }
-        if (wvalid) tc::tmem_wait_st();
-        // order this warp's P stores before the next head's exchange arrival
-        tc::fence_before();
       }
+      hk += H;
       if (!ok) { fail(sm, p.status); break; }
-      // ---- column reductions of P over this warp's 32 rows, for the chunks
-      // this warp wrote in the last head (so no other warp's stores are
-      // involved): column max -> s2 (atomicMax), register columns -> this
-      // warp's partial of s2(r)
+      // ---- column reductions of P over this warp's 32 rows: column max ->
+      // s2 (atomicMax), register columns -> this warp's partial of s2(r)
       float regacc = 0.f;
       if (wvalid) {
-        tc::fence_after();
-        for (int c = (int)((pstart + half) & 1); c < g.nic; c += 2) {
-          const int nv = min(KC, g.own_img - c * KC);
-          for (int hf = 0; hf < 2; ++hf) {
-            uint32_t w[32];
-            tc::tmem_ld32(tmem + lane_base + P_COL + c * KC + hf * 32, w);
-            tc::tmem_wait_ld();
 #pragma unroll
-            for (int col = 0; col < 32; ++col) {
-              const float x = vrow ? __uint_as_float(w[col]) : 0.f;
-              const float mx = warp_max_f(x);
-              const float su = warp_sum_f(x);
-              if (lane == 0 && hf * 32 + col < nv) {
-                const int key = c * KC + hf * 32 + col;
-                if (sm.kreg[ib][key]) regacc += su * invH;
-                else atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(mx * invH));
-              }
+        for (int pc = 0; pc < PCOLS / 32; ++pc) {
+          // transpose-reduce over the 32 rows of this warp: afterwards lane l
+          // holds the max and the sum of column (pc * 32 + l) -- 31 shuffles each
+          float mx[32], su[32];
+#pragma unroll
+          for (int col = 0; col < 32; ++col) mx[col] = su[col] = vrow ? P[pc][col] : 0.f;
+#pragma unroll
+          for (int sft = 16; sft >= 1; sft >>= 1) {
+            const bool up = (lane & sft) != 0;
+#pragma unroll
+            for (int i = 0; i < sft; ++i) {
+              const float sm_send = up ? mx[i] : mx[i + sft];
+              const float sm_keep = up ? mx[i + sft] : mx[i];
+              const float ss_send = up ? su[i] : su[i + sft];
+              const float ss_keep = up ? su[i + sft] : su[i];
+              mx[i] = fmaxf(sm_keep, __shfl_xor_sync(0xffffffffu, sm_send, sft));
+              su[i] = ss_keep + __shfl_xor_sync(0xffffffffu, ss_send, sft);
             }
           }
+          const int key = half * PCOLS + pc * 32 + lane;
+          float rc = 0.f;
+          if (key < g.own_img) {
+            if (sm.kreg[ib][key]) rc = su[0] * invH;
+            else atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(mx[0] * invH));
+          }
+          regacc += warp_sum_f(rc);
         }
       }
       if (lane == 0) {
-        p.refpart[g.slot + rank * NEPI + ew] = regacc;
+        p.refpart[g.slot + rank * NEPI + ew] = regacc;  // C * NEPI slots per item
         __threadfence();
         const int nslots = p.slot_off[g.b + 1] - p.slot_off[g.b];
         if (atomicAdd(&p.done[g.b], 1) == nslots - 1) {
@@ -458,6 +487,31 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   if (warp == MMA_WARP) tc::tmem_dealloc(tmem, TMEM_COLS);
   // peers may still write into this CTA's exchange buffers until here
   tc::cluster_sync_all();
+}
+
+int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt,
+                 const Stage2TcParams& q, int nclusters, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(nclusters * C));
+  cfg.blockDim = dim3(s2f::THREADS);
+  cfg.dynamicSmemBytes = s2_fused_smem_bytes(C);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e;
+  if (C == 8) {
+    cudaFuncSetAttribute(s2_fused_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(8));
+    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<8>, mq, mk, mkt, q);
+  } else {
+    cudaFuncSetAttribute(s2_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(4));
+    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<4>, mq, mk, mkt, q);
+  }
+  return e == cudaSuccess ? 0 : 1;
 }
 
 }  // namespace occam

@@ -42,7 +42,9 @@ CASES = [
     ("scan_tiles", dict(B=5, segs=2, P=(500, 333, 612, 47, 401), R=4, M=(9, 33, 65, 2, 17), seed=5), 0.2, 1.05),
     # fused tensor-core Stage II: text tiles of 128 rows, chunk edges at 64 keys per CTA
     ("fused_text_edges", dict(B=4, segs=1, P=(252, 60, 300, 5), R=4, M=(128, 129, 256, 1), seed=21), 0.0, 1.1),
-    ("fused_max_keys", dict(B=1, segs=2, P=(760,), R=4, M=(40,), seed=22), 0.0, 1.2),
+    ("fused_max_keys", dict(B=1, segs=1, P=(764,), R=4, M=(40,), seed=22), 0.0, 1.2),
+    # 8-CTA clusters: S1 above 768 keys, up to their limit of 1536
+    ("fused_c8", dict(B=2, segs=1, P=(1000, 1532), R=4, M=(130, 33), seed=25), 0.0, 1.15),
     # one sample above the fused kernel's S1 limit (two-pass), one below (fused)
     ("mixed_paths", dict(B=2, segs=1, P=(1700, 200), R=3, M=(70, 90), seed=23), 0.0, 1.1),
 ]
