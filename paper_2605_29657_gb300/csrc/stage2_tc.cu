@@ -16,19 +16,20 @@
 //      every key row is read once per text tile); the head's 128 x 128 query
 //      tile arrives by TMA;
 //   2. one thread issues S = Q K^T per chunk (tcgen05.mma, bf16 in, fp32 in
-//      TMEM); S1-key chunks land in a per-head TMEM buffer E (two buffers,
-//      alternating by head), text-key chunks in a scratch TMEM buffer;
+//      TMEM): text-key chunks into a two-deep scratch ring, S1-key chunks
+//      into a per-head TMEM buffer E (two buffers, alternating by head);
 //   3. eight epilogue warps (two per TMEM lane quadrant, one thread per text
-//      row, each taking one 32-column half of every chunk) turn S into
-//      exp2(l - cmax) (cmax: the half-chunk's row max, kept in shared
-//      memory), write it back over S in E, and keep the row's running
-//      softmax max / sum;
-//   4. the (max, sum) pairs are exchanged with every epilogue warp of the
-//      cluster through distributed shared memory. The exchange of head h is
+//      row) each own one 32-column half of every chunk. A warp turns its
+//      logits into exp2(l - cmax) (cmax: the row max of that half-chunk, kept
+//      in a register), writes them back over S1-key logits in E, and keeps
+//      the row's running softmax max / sum;
+//   4. the (max, sum) pairs go to every epilogue warp of the cluster with
+//      asynchronous distributed-shared-memory stores that complete on an
+//      mbarrier of the receiving CTA (no fences). The exchange of head h is
 //      awaited only after head h+1's statistics, so its latency is hidden;
-//   5. then every warp adds exp2(cmax - max) / sum * E to the head-summed
-//      probabilities P of its 96 S1-key columns, which live in registers for
-//      the whole item.
+//   5. then every warp adds exp2(cmax - max) / sum * E over its own columns to
+//      the head-summed probabilities P, which live in registers for the
+//      whole item.
 // After the last head every warp reduces its P columns over its 32 rows:
 // column max -> s2 (atomicMax on the fp32 bit pattern, exact and order-free
 // since P >= 0), register columns -> a partial of s2(r) reduced in fixed order.
@@ -51,7 +52,6 @@ constexpr int NPROD = 3;               // producer warps (0-2); warp 3 issues MM
 constexpr int MMA_WARP = NPROD;
 constexpr int EPI_WARP0 = NPROD + 1;
 constexpr int NEPI = kFusedEpiWarps;   // two per TMEM lane quadrant
-constexpr int PCOLS = PMAX / 2;        // P columns per epilogue warp (registers)
 constexpr int THREADS = (NPROD + 1 + NEPI) * 32;
 constexpr int NXS = 4;                 // exchange slots (the exchange runs one head behind)
 constexpr uint32_t IDESC = tc::idesc_bf16(128, KC);
@@ -59,19 +59,19 @@ constexpr uint32_t TMEM_COLS = 512;
 constexpr int S_COL = 0;               // two scratch buffers (text-key chunks), KC columns each
 constexpr int E_COL = 2 * KC;          // two E buffers (by head parity), PMAX columns each
 static_assert(E_COL + 2 * PMAX <= (int)TMEM_COLS, "TMEM budget");
-static_assert(PMAX % (2 * 32) == 0 && PCOLS % 32 == 0, "P columns split into 32-column pieces");
+static_assert(PMAX % KC == 0, "E buffers hold whole chunks");
 constexpr uint64_t kLimitNs = 2000000000ull;
 
 template <int C>
 struct Smem {
+  static constexpr uint32_t XBYTES = C * NEPI * 32 * 8;  // exchange bytes one CTA receives per head
   uint8_t q[2][QBYTES];
   uint8_t k[NST][KBYTES];
   int32_t kidx[2][PMAX + TMAX];
   float2 xch[NXS][C][2][QR];          // (max, sum) per (slot, CTA, epilogue half, row)
-  float cmx[2][NIC_MAX][2][QR];       // half-chunk row max (log2 units) per (head parity, chunk, half, row)
   uint8_t kreg[2][PMAX];
-  uint64_t kfull[NST], kempty[NST], qfull[2], qempty[2], sfull[2], sempty[2], efree[2], xbar[NXS], iready[2],
-      idone[2], mdone;
+  uint64_t kfull[NST], kempty[NST], qfull[2], qempty[2], sfull[2], sempty[2], efull[2][NIC_MAX], efree[2],
+      xbar[NXS], iready[2], idone[2], mdone;
   uint32_t tmem_base;
   int abort;
   uint32_t issued_q;
@@ -119,15 +119,79 @@ __device__ __forceinline__ void fail(SM& sm, int* status) {
   set_status(status, OCCAM_ERR_TIMEOUT);
 }
 
-__device__ __forceinline__ float warp_max_f(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
 __device__ __forceinline__ float warp_sum_f(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
+}
+
+// Statistics of one thread's row over a 32-column half-chunk of logits at
+// TMEM address sa (warp-collective): cm = max of the first `lim` columns in
+// log2 units (-inf if none), a = sum over them of exp2(l * sl2 - cm). With
+// STORE the exponentials (0 past lim) are written back over the logits; the
+// caller waits for that store before the values are read again.
+template <bool STORE>
+__device__ __forceinline__ void half_stats(uint32_t sa, int lim, float sl2, float& cm, float& a) {
+  cm = -INFINITY;
+  a = 0.f;
+  if (__all_sync(0xffffffffu, lim <= 0)) return;
+  const bool full = __all_sync(0xffffffffu, lim >= 32);
+  uint32_t v[32];
+  tc::fence_after();
+  tc::tmem_ld32(sa, v);
+  tc::tmem_wait_ld();
+  if (full) {
+    float t[11];
+#pragma unroll
+    for (int i = 0; i < 10; ++i)
+      t[i] = tc::fmax3(__uint_as_float(v[3 * i]), __uint_as_float(v[3 * i + 1]), __uint_as_float(v[3 * i + 2]));
+    t[10] = fmaxf(__uint_as_float(v[30]), __uint_as_float(v[31]));
+    const float mx = fmaxf(tc::fmax3(tc::fmax3(t[0], t[1], t[2]), tc::fmax3(t[3], t[4], t[5]), tc::fmax3(t[6], t[7], t[8])),
+                           fmaxf(t[9], t[10]));
+    cm = mx * sl2;
+    const float2 sc = make_float2(sl2, sl2), off = make_float2(-cm, -cm);
+    float2 acc0 = make_float2(0.f, 0.f), acc1 = acc0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), sc, off);
+      x.x = tc::ex2(x.x);
+      x.y = tc::ex2(x.y);
+      if (i & 1) acc1 = __fadd2_rn(acc1, x);
+      else acc0 = __fadd2_rn(acc0, x);
+      v[2 * i] = __float_as_uint(x.x);
+      v[2 * i + 1] = __float_as_uint(x.y);
+    }
+    a = (acc0.x + acc0.y) + (acc1.x + acc1.y);
+  } else {
+    float c0 = -INFINITY, c1 = -INFINITY;
+#pragma unroll
+    for (int col = 0; col < 32; col += 2) {
+      if (col < lim) c0 = fmaxf(c0, __uint_as_float(v[col]));
+      if (col + 1 < lim) c1 = fmaxf(c1, __uint_as_float(v[col + 1]));
+    }
+    cm = fmaxf(c0, c1) * sl2;
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int col = 0; col < 32; col += 2) {
+      const float e0 = (col < lim) ? tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -cm)) : 0.f;
+      const float e1 = (col + 1 < lim) ? tc::ex2(fmaf(__uint_as_float(v[col + 1]), sl2, -cm)) : 0.f;
+      a0 += e0;
+      a1 += e1;
+      v[col] = __float_as_uint(e0);
+      v[col + 1] = __float_as_uint(e1);
+    }
+    a = a0 + a1;
+  }
+  if (STORE) tc::tmem_st32(sa, v);
+}
+
+// merges a half-chunk's (cm, a) into the row's running softmax (m, z), log2 units
+__device__ __forceinline__ void online_merge(float& m, float& z, float cm, float a) {
+  if (cm != -INFINITY) {
+    const float mn = fmaxf(m, cm);
+    z = (m == -INFINITY ? 0.f : z * tc::ex2(m - mn)) + a * tc::ex2(cm - mn);
+    m = mn;
+  }
 }
 
 }  // namespace
@@ -154,15 +218,19 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       tc::bar_init(&sm.qempty[i], 1);
       tc::bar_init(&sm.sfull[i], 1);
       tc::bar_init(&sm.sempty[i], NEPI);
+      for (int c = 0; c < NIC_MAX; ++c) tc::bar_init(&sm.efull[i][c], 1);
       tc::bar_init(&sm.efree[i], NEPI);
       tc::bar_init(&sm.iready[i], NPROD * 32);
       tc::bar_init(&sm.idone[i], NEPI);
     }
-    for (int i = 0; i < NXS; ++i) tc::bar_init(&sm.xbar[i], NEPI * C);
+    // one local arrival (with the expected byte count) plus the peers'
+    // asynchronous stores complete each phase of an exchange slot
+    for (int i = 0; i < NXS; ++i) tc::bar_init(&sm.xbar[i], 1);
     tc::bar_init(&sm.mdone, 1);
     sm.abort = 0;
     sm.issued_q = 0;
     tc::bar_fence_init();
+    for (int i = 0; i < NXS; ++i) tc::bar_expect_tx(&sm.xbar[i], Smem<C>::XBYTES);
     tc::prefetch_map(&mapQ);
   }
   if (warp == MMA_WARP) tc::tmem_alloc(&sm.tmem_base, TMEM_COLS);
@@ -245,31 +313,35 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   } else if (warp == MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      uint32_t qcnt = 0, kcnt = 0, scnt = 0, hk = 0;
+      uint32_t qcnt = 0, kcnt = 0, tcnt = 0, hk = 0;
       for (int item = cid; item < nF && !*abort; item += ncl) {
         const ItemGeom g = item_geom<C>(p, p.items[item], rank);
         const int nch = g.nic + g.ntc;
         for (int h = 0; h < H && !*abort; ++h, ++hk) {
           const int qb = qcnt & 1;
           if (!tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-          const uint32_t ebuf = tmem + E_COL + (hk & 1) * PMAX;
-          for (int ci = 0; ci < nch; ++ci) {
-            // E[hk & 1] is free once the probabilities of head hk - 2 were read out of it
-            if (ci == g.ntc && hk >= 2 &&
-                !tc::bar_wait(&sm.efree[hk & 1], ((hk - 2) >> 1) & 1, abort, kLimitNs)) {
-              fail(sm, p.status);
-              break;
-            }
+          const int eb = hk & 1;
+          bool ok = true;
+          for (int ci = 0; ci < nch && ok; ++ci) {
+            const bool is_txt = ci < g.ntc;
             const int st = kcnt % NST;
-            const int sb = scnt & 1;
-            if (!tc::bar_wait(&sm.kfull[st], (kcnt / NST) & 1, abort, kLimitNs) ||
-                !tc::bar_wait(&sm.sempty[sb], ((scnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
+            uint32_t d;
+            if (is_txt) {
+              const int sb = tcnt & 1;
+              ok = tc::bar_wait(&sm.sempty[sb], ((tcnt >> 1) & 1) ^ 1, abort, kLimitNs);
+              d = tmem + S_COL + sb * KC;
+            } else {
+              // E[eb] is free once the probabilities of head hk - 2 were read out of it
+              if (ci == g.ntc && hk >= 2) ok = tc::bar_wait(&sm.efree[eb], ((hk - 2) >> 1) & 1, abort, kLimitNs);
+              d = tmem + E_COL + eb * PMAX + (ci - g.ntc) * KC;
+            }
+            if (ok) ok = tc::bar_wait(&sm.kfull[st], (kcnt / NST) & 1, abort, kLimitNs);
+            if (!ok) {
               fail(sm, p.status);
               break;
             }
             tc::fence_proxy_async();
             tc::fence_after();
-            const uint32_t d = ci >= g.ntc ? ebuf + (ci - g.ntc) * KC : tmem + S_COL + sb * KC;
             const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[st]);
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
@@ -277,11 +349,19 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
               tc::mma_bf16(d, tc::sdesc_sw128(qa + kb * (QBYTES / 2) + kk * 32),
                            tc::sdesc_sw128(kbase + kb * (KBYTES / 2) + kk * 32), IDESC, k > 0 ? 1u : 0u);
             }
-            tc::mma_commit(&sm.sfull[sb]);
+            if (is_txt) {
+              tc::mma_commit(&sm.sfull[tcnt & 1]);
+              ++tcnt;
+            } else {
+              tc::mma_commit(&sm.efull[eb][ci - g.ntc]);
+            }
             tc::mma_commit(&sm.kempty[st]);
             ++kcnt;
-            ++scnt;
           }
+          if (!ok) break;
+          // the E-chunk barriers of chunks this item does not use still
+          // complete once per head, so every barrier's phase follows the head index
+          for (int c = g.nic; c < NIC_MAX; ++c) tc::mma_commit(&sm.efull[eb][c]);
           tc::mma_commit(&sm.qempty[qb]);
           ++qcnt;
         }
@@ -294,13 +374,14 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   } else {
     // ------------------------------------------------------------ epilogue
     const int ew = warp - EPI_WARP0;    // 0..NEPI-1
-    const int half = ew >> 2;           // chunk parity this warp takes; also its P column half
+    const int half = ew >> 2;           // the 32-column half of every chunk this warp owns
     const int quad = warp & 3;          // TMEM lane quadrant this warp may access
     const int j = quad * 32 + lane;     // text row of this thread inside the tile
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const float sl2 = p.scale_log2;
     const float invH = 1.0f / (float)H;
-    uint32_t scnt = 0, hk = 0;
+    const bool armer = ew == 0 && lane == 0;  // re-arms the exchange slots of this CTA
+    uint32_t tcnt = 0, hk = 0;
     int ii = 0;
     for (int item = cid; item < nF; item += ncl, ++ii) {
       const ItemGeom g = item_geom<C>(p, p.items[item], rank);
@@ -309,76 +390,60 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       const bool vrow = g.j0 + j < g.M;
       const bool wvalid = __any_sync(0xffffffffu, vrow);  // warp-uniform: any real text row here
       const int jj = g.j0 + j;
-      float P[PCOLS / 32][32];
+      float P[NIC_MAX][32];
 #pragma unroll
-      for (int a = 0; a < PCOLS / 32; ++a)
+      for (int c = 0; c < NIC_MAX; ++c)
 #pragma unroll
-        for (int b2 = 0; b2 < 32; ++b2) P[a][b2] = 0.f;
+        for (int b2 = 0; b2 < 32; ++b2) P[c][b2] = 0.f;
+      float cmc[NIC_MAX], cmp[NIC_MAX];  // half-chunk maxima of the current / previous head
+#pragma unroll
+      for (int c = 0; c < NIC_MAX; ++c) cmc[c] = cmp[c] = -INFINITY;
       bool ok = true;
       for (int step = 0; step <= H && ok; ++step) {
         const uint32_t hcur = hk + step;  // global index of head `step` of this item
         if (step < H) {
-          // ---- statistics of head `step` over this warp's chunks
+          // ---- statistics of head `step`: text-key chunks, then S1-key chunks
           const int eb = hcur & 1;
           float m = -INFINITY, z = 0.f;
-          for (int ci = 0; ci < g.nic + g.ntc; ++ci, ++scnt) {
-            const int sb = scnt & 1;
-            if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[sb], (scnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
-            const bool is_txt = ci < g.ntc;
-            const int c = is_txt ? ci : ci - g.ntc;
-            const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
-            const int tbase = g.txt0 + c * KC + half * 32;  // sample-relative text index of this half's column 0
-            // valid columns of this warp's half of the chunk
-            const int lim = vrow ? (is_txt ? min(nv - half * 32, jj - tbase + 1) : nv - half * 32) : 0;
-            const uint32_t sa = lane_base + half * 32 + (is_txt ? tmem + S_COL + sb * KC : tmem + E_COL + eb * PMAX + c * KC);
+          for (int c = 0; c < g.ntc; ++c, ++tcnt) {
+            const int sb = tcnt & 1;
+            if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[sb], (tcnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
             if (wvalid) {
-              tc::fence_after();
-              uint32_t v[32];
-              tc::tmem_ld32(sa, v);
-              tc::tmem_wait_ld();
-              float c0 = -INFINITY, c1 = -INFINITY;
-#pragma unroll
-              for (int col = 0; col < 32; col += 2) {
-                if (col < lim) c0 = fmaxf(c0, __uint_as_float(v[col]));
-                if (col + 1 < lim) c1 = fmaxf(c1, __uint_as_float(v[col + 1]));
-              }
-              const float cm = fmaxf(c0, c1) * sl2;
-              float a0 = 0.f, a1 = 0.f;
-#pragma unroll
-              for (int col = 0; col < 32; col += 2) {
-                const float e0 = (col < lim) ? tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -cm)) : 0.f;
-                const float e1 = (col + 1 < lim) ? tc::ex2(fmaf(__uint_as_float(v[col + 1]), sl2, -cm)) : 0.f;
-                a0 += e0;
-                a1 += e1;
-                v[col] = __float_as_uint(e0);
-                v[col + 1] = __float_as_uint(e1);
-              }
-              if (!is_txt) {
-                tc::tmem_st32(sa, v);  // E <- exp2(l - cmax); completion awaited before the exchange
-                sm.cmx[eb][c][half][j] = cm;
-              }
-              if (cm != -INFINITY) {
-                const float mn = fmaxf(m, cm);
-                z = (m == -INFINITY ? 0.f : z * tc::ex2(m - mn)) + (a0 + a1) * tc::ex2(cm - mn);
-                m = mn;
-              }
+              const int nv = min(KC, g.own_txt - c * KC);
+              const int tbase = g.txt0 + c * KC + half * 32;  // sample-relative text index of this half's column 0
+              const int lim = vrow ? min(nv - half * 32, jj - tbase + 1) : 0;
+              float cm, a;
+              half_stats<false>(tmem + lane_base + S_COL + sb * KC + half * 32, lim, sl2, cm, a);
+              online_merge(m, z, cm, a);
             }
             tc::fence_before();
             __syncwarp();
             if (lane == 0) tc::bar_arrive(&sm.sempty[sb]);
+          }
+#pragma unroll
+          for (int c = 0; c < NIC_MAX; ++c) {
+            cmc[c] = -INFINITY;
+            if (ok && c < g.nic) {
+              if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.efull[eb][c], (hcur >> 1) & 1, nullptr, kLimitNs))) {
+                ok = false;
+              } else if (wvalid) {
+                const int lim = vrow ? min(KC, g.own_img - c * KC) - half * 32 : 0;
+                float a;
+                half_stats<true>(tmem + lane_base + E_COL + eb * PMAX + c * KC + half * 32, lim, sl2, cmc[c], a);
+                online_merge(m, z, cmc[c], a);
+              }
+            }
           }
           if (wvalid) tc::tmem_wait_st();
           tc::fence_before();
           if (!ok) break;
           // ---- post this head's (max, sum) to every epilogue warp of the cluster
           const int slot = hcur & (NXS - 1);
-          for (int r = 0; r < C; ++r) tc::st_cluster_f2(&sm.xch[slot][rank][half][j], (uint32_t)r, m, z);
-          __syncwarp();
-          if (lane == 0)
-            for (int r = 0; r < C; ++r) tc::bar_arrive_remote(&sm.xbar[slot], (uint32_t)r);
+#pragma unroll
+          for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][half][j], &sm.xbar[slot], (uint32_t)r, m, z);
         }
         if (step >= 1) {
-          // ---- probabilities of head step-1, added into P
+          // ---- probabilities of head step-1 over this warp's columns, added into P
           const uint32_t hp = hcur - 1;
           const int slot = hp & (NXS - 1);
           const int eb = hp & 1;
@@ -387,7 +452,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             float Mx = -INFINITY;
 #pragma unroll
             for (int r = 0; r < C; ++r)
-              Mx = fmaxf(Mx, fmaxf(sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x));
+              Mx = tc::fmax3(Mx, sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x);
             float Z = 0.f;
 #pragma unroll
             for (int r = 0; r < C; ++r)
@@ -399,24 +464,31 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             const float invZ = (vrow && Z > 0.f) ? 1.0f / Z : 0.f;
             tc::fence_after();
 #pragma unroll
-            for (int pc = 0; pc < PCOLS / 32; ++pc) {
-              const int col0 = half * PCOLS + pc * 32;
-              const int c = col0 / KC;
+            for (int c = 0; c < NIC_MAX; ++c) {
               if (c < g.nic) {
-                const float cmc = sm.cmx[eb][c][(col0 / 32) & 1][j];
-                const float f = (invZ > 0.f && cmc != -INFINITY) ? tc::ex2(cmc - Mx) * invZ : 0.f;
+                const float f = (invZ > 0.f && cmp[c] != -INFINITY) ? tc::ex2(cmp[c] - Mx) * invZ : 0.f;
                 uint32_t v[32];
-                tc::tmem_ld32(tmem + lane_base + E_COL + eb * PMAX + col0, v);
+                tc::tmem_ld32(tmem + lane_base + E_COL + eb * PMAX + c * KC + half * 32, v);
                 tc::tmem_wait_ld();
+                const float2 ff = make_float2(f, f);
 #pragma unroll
-                for (int col = 0; col < 32; ++col) P[pc][col] = fmaf(__uint_as_float(v[col]), f, P[pc][col]);
+                for (int i = 0; i < 16; ++i) {
+                  const float2 r2 = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), ff,
+                                               make_float2(P[c][2 * i], P[c][2 * i + 1]));
+                  P[c][2 * i] = r2.x;
+                  P[c][2 * i + 1] = r2.y;
+                }
               }
             }
           }
           tc::fence_before();
           __syncwarp();
           if (lane == 0) tc::bar_arrive(&sm.efree[eb]);
+          // the slot's phase for head hp is complete: arm it for head hp + NXS
+          if (armer) tc::bar_expect_tx(&sm.xbar[slot], Smem<C>::XBYTES);
         }
+#pragma unroll
+        for (int c = 0; c < NIC_MAX; ++c) cmp[c] = cmc[c];
       }
       hk += H;
       if (!ok) { fail(sm, p.status); break; }
@@ -425,32 +497,34 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       float regacc = 0.f;
       if (wvalid) {
 #pragma unroll
-        for (int pc = 0; pc < PCOLS / 32; ++pc) {
-          // transpose-reduce over the 32 rows of this warp: afterwards lane l
-          // holds the max and the sum of column (pc * 32 + l) -- 31 shuffles each
-          float mx[32], su[32];
+        for (int c = 0; c < NIC_MAX; ++c) {
+          if (c < g.nic) {
+            // transpose-reduce over the 32 rows of this warp: afterwards lane l
+            // holds the max and the sum of this warp's column l of chunk c
+            float mx[32], su[32];
 #pragma unroll
-          for (int col = 0; col < 32; ++col) mx[col] = su[col] = vrow ? P[pc][col] : 0.f;
+            for (int col = 0; col < 32; ++col) mx[col] = su[col] = vrow ? P[c][col] : 0.f;
 #pragma unroll
-          for (int sft = 16; sft >= 1; sft >>= 1) {
-            const bool up = (lane & sft) != 0;
+            for (int sft = 16; sft >= 1; sft >>= 1) {
+              const bool up = (lane & sft) != 0;
 #pragma unroll
-            for (int i = 0; i < sft; ++i) {
-              const float sm_send = up ? mx[i] : mx[i + sft];
-              const float sm_keep = up ? mx[i + sft] : mx[i];
-              const float ss_send = up ? su[i] : su[i + sft];
-              const float ss_keep = up ? su[i + sft] : su[i];
-              mx[i] = fmaxf(sm_keep, __shfl_xor_sync(0xffffffffu, sm_send, sft));
-              su[i] = ss_keep + __shfl_xor_sync(0xffffffffu, ss_send, sft);
+              for (int i = 0; i < sft; ++i) {
+                const float sm_send = up ? mx[i] : mx[i + sft];
+                const float sm_keep = up ? mx[i + sft] : mx[i];
+                const float ss_send = up ? su[i] : su[i + sft];
+                const float ss_keep = up ? su[i + sft] : su[i];
+                mx[i] = fmaxf(sm_keep, __shfl_xor_sync(0xffffffffu, sm_send, sft));
+                su[i] = ss_keep + __shfl_xor_sync(0xffffffffu, ss_send, sft);
+              }
             }
+            const int key = c * KC + half * 32 + lane;
+            float rc = 0.f;
+            if (key < g.own_img) {
+              if (sm.kreg[ib][key]) rc = su[0] * invH;
+              else atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(mx[0] * invH));
+            }
+            regacc += warp_sum_f(rc);
           }
-          const int key = half * PCOLS + pc * 32 + lane;
-          float rc = 0.f;
-          if (key < g.own_img) {
-            if (sm.kreg[ib][key]) rc = su[0] * invH;
-            else atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(mx[0] * invH));
-          }
-          regacc += warp_sum_f(rc);
         }
       }
       if (lane == 0) {
@@ -485,6 +559,13 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   __syncthreads();
   tc::fence_after();
   if (warp == MMA_WARP) tc::tmem_dealloc(tmem, TMEM_COLS);
+  if (sm.abort && tid == 0) {
+    // after an abort, peers' asynchronous exchange stores may still be in
+    // flight towards this CTA: give them time to land before it can exit
+    const uint64_t t0 = tc::globaltimer();
+    while (tc::globaltimer() - t0 < 100000ull) {
+    }
+  }
   // peers may still write into this CTA's exchange buffers until here
   tc::cluster_sync_all();
 }

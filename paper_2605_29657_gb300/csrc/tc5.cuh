@@ -217,6 +217,13 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// three-input maximum (sm_100+)
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
 // ---------------------------------------------------------------- distributed shared memory
 __device__ __forceinline__ void st_cluster_f2(const void* local_addr, uint32_t rank, float x, float y) {
   asm volatile(
@@ -224,6 +231,19 @@ __device__ __forceinline__ void st_cluster_f2(const void* local_addr, uint32_t r
       "mapa.shared::cluster.u32 ra, %0, %1;\n\t"
       "st.shared::cluster.v2.f32 [ra], {%2, %3};\n\t}" ::"r"(su32(local_addr)),
       "r"(rank), "f"(x), "f"(y)
+      : "memory");
+}
+// asynchronous 8-byte store into CTA `rank`'s copy of local_addr; its
+// completion is signalled as 8 transaction bytes on that CTA's copy of bar
+__device__ __forceinline__ void st_async_f2(const void* local_addr, const uint64_t* bar, uint32_t rank, float x,
+                                            float y) {
+  asm volatile(
+      "{\n\t.reg .b32 ra, rb;\n\t"
+      "mapa.shared::cluster.u32 ra, %0, %2;\n\t"
+      "mapa.shared::cluster.u32 rb, %1, %2;\n\t"
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [ra], {%3, %4}, [rb];\n\t}" ::"r"(
+          su32(local_addr)),
+      "r"(su32(bar)), "r"(rank), "f"(x), "f"(y)
       : "memory");
 }
 __device__ __forceinline__ uint32_t cluster_rank() {
