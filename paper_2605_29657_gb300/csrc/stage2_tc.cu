@@ -54,6 +54,12 @@ constexpr int EPI_WARP0 = NPROD + 1;
 constexpr int NEPI = kFusedEpiWarps;   // two per TMEM lane quadrant
 constexpr int THREADS = (NPROD + 1 + NEPI) * 32;
 constexpr int NXS = 4;                 // exchange slots (the exchange runs one head behind)
+// register split: warpgroup 0 (producers + MMA issuer) shrinks to REG_LOW per
+// thread, the two epilogue warpgroups grow to REG_HIGH; the sum must stay
+// within what the CTA was launched with (checked on the host before launch)
+constexpr int REG_LOW = 88, REG_HIGH = 208;
+constexpr int REG_NEEDED = 128 * REG_LOW + (THREADS - 128) * REG_HIGH;
+static_assert(NPROD + 1 == 4 && (THREADS - 128) % 128 == 0, "warpgroup 0 = producers + MMA warp");
 constexpr uint32_t IDESC = tc::idesc_bf16(128, KC);
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int S_COL = 0;               // two scratch buffers (text-key chunks), KC columns each
@@ -242,136 +248,142 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   const uint32_t tmem = sm.tmem_base;
   const int H = p.H;
 
-  if (warp < NPROD) {
-    // ------------------------------------------------------------ producers
-    // 96 threads; piece q = pt + 96 i (q < 1024) of a chunk is 16 bytes of key
-    // row (q >> 4), head slice bytes 16 * (q & 15); it lands at the row's
-    // 128-byte line of its K-block with the 16-byte chunk index XOR (row & 7).
-    const int pt = tid;
-    uint32_t qcnt = 0, kcnt = 0;
-    int ii = 0;
-    const int64_t HD = (int64_t)H * 128;
-    for (int item = cid; item < nF; item += ncl, ++ii) {
-      const ItemGeom g = item_geom<C>(p, p.items[item], rank);
-      const int ib = ii & 1;
-      if (*abort || !tc::bar_wait(&sm.idone[ib], ((ii >> 1) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-      for (int i = pt; i < g.own_img; i += NPROD * 32) {
-        const int row = p.dense[g.rbase + g.img0 + i];
-        sm.kidx[ib][i] = row;
-        sm.kreg[ib][i] = p.role[row];
-      }
-      for (int i = pt; i < g.own_txt; i += NPROD * 32) sm.kidx[ib][PMAX + i] = (int)(g.t0 + g.txt0 + i);
-      tc::bar_arrive(&sm.iready[ib]);
-      if (!tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-      const int nch = g.nic + g.ntc;
-      bool ok = true;
-      for (int h = 0; h < H && ok; ++h) {
-        if (pt == 0) {
-          const int qb = qcnt & 1;
-          if (!tc::bar_wait(&sm.qempty[qb], ((qcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
-            fail(sm, p.status);
-            ok = false;
-          } else {
-            tc::bar_expect_tx(&sm.qfull[qb], QBYTES);
-            tc::tma_load_2d(sm.q[qb], &mapQ, h * 128, (int)(g.t0 + g.j0), &sm.qfull[qb]);
-            tc::tma_load_2d(sm.q[qb] + QBYTES / 2, &mapQ, h * 128 + 64, (int)(g.t0 + g.j0), &sm.qfull[qb]);
-          }
-        }
-        ++qcnt;
-        for (int ci = 0; ci < nch && ok; ++ci) {
-          const int st = kcnt % NST;
-          if (!tc::bar_wait(&sm.kempty[st], ((kcnt / NST) & 1) ^ 1, abort, kLimitNs)) {
-            fail(sm, p.status);
-            ok = false;
-            break;
-          }
-          const bool is_txt = ci < g.ntc;  // text chunks first: they do not wait for an E buffer
-          const int c = is_txt ? ci : ci - g.ntc;
-          const int* rows = is_txt ? &sm.kidx[ib][PMAX + c * KC] : &sm.kidx[ib][c * KC];
-          const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
-          const __nv_bfloat16* base = is_txt ? p.Kt : p.K;
-          uint8_t* dst = sm.k[st];
-#pragma unroll
-          for (int i = 0; i < (KC * 16 + NPROD * 32 - 1) / (NPROD * 32); ++i) {
-            const int q = pt + NPROD * 32 * i;
-            if (q < KC * 16) {
-              const int key = q >> 4, c16 = q & 15;
-              const int kb = c16 >> 3, cc = c16 & 7;
-              const bool v = key < nv;
-              const __nv_bfloat16* src = base + (v ? (int64_t)rows[key] * HD + h * 128 + c16 * 8 : 0);
-              tc::cp_async16(dst + kb * (KBYTES / 2) + key * 128 + ((cc ^ (key & 7)) << 4), src, v ? 16 : 0);
-            }
-          }
-          tc::cp_async_arrive(&sm.kfull[st]);
-          ++kcnt;
-        }
-      }
-      if (!ok) break;
-    }
-    if (pt == 0) sm.issued_q = qcnt;
-    asm volatile("cp.async.wait_all;" ::: "memory");
-  } else if (warp == MMA_WARP) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      uint32_t qcnt = 0, kcnt = 0, tcnt = 0, hk = 0;
-      for (int item = cid; item < nF && !*abort; item += ncl) {
+  if (warp < 4) {
+    // warpgroup 0: producers and the MMA issuer give registers back
+    tc::setmaxnreg_dec<REG_LOW>();
+    if (warp < NPROD) {
+      // ------------------------------------------------------------ producers
+      // 96 threads; piece q = pt + 96 i (q < 1024) of a chunk is 16 bytes of key
+      // row (q >> 4), head slice bytes 16 * (q & 15); it lands at the row's
+      // 128-byte line of its K-block with the 16-byte chunk index XOR (row & 7).
+      const int pt = tid;
+      uint32_t qcnt = 0, kcnt = 0;
+      int ii = 0;
+      const int64_t HD = (int64_t)H * 128;
+      for (int item = cid; item < nF; item += ncl, ++ii) {
         const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+        const int ib = ii & 1;
+        if (*abort || !tc::bar_wait(&sm.idone[ib], ((ii >> 1) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
+        for (int i = pt; i < g.own_img; i += NPROD * 32) {
+          const int row = p.dense[g.rbase + g.img0 + i];
+          sm.kidx[ib][i] = row;
+          sm.kreg[ib][i] = p.role[row];
+        }
+        for (int i = pt; i < g.own_txt; i += NPROD * 32) sm.kidx[ib][PMAX + i] = (int)(g.t0 + g.txt0 + i);
+        tc::bar_arrive(&sm.iready[ib]);
+        if (!tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
         const int nch = g.nic + g.ntc;
-        for (int h = 0; h < H && !*abort; ++h, ++hk) {
-          const int qb = qcnt & 1;
-          if (!tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-          const int eb = hk & 1;
-          bool ok = true;
-          for (int ci = 0; ci < nch && ok; ++ci) {
-            const bool is_txt = ci < g.ntc;
-            const int st = kcnt % NST;
-            uint32_t d;
-            if (is_txt) {
-              const int sb = tcnt & 1;
-              ok = tc::bar_wait(&sm.sempty[sb], ((tcnt >> 1) & 1) ^ 1, abort, kLimitNs);
-              d = tmem + S_COL + sb * KC;
-            } else {
-              // E[eb] is free once the probabilities of head hk - 2 were read out of it
-              if (ci == g.ntc && hk >= 2) ok = tc::bar_wait(&sm.efree[eb], ((hk - 2) >> 1) & 1, abort, kLimitNs);
-              d = tmem + E_COL + eb * PMAX + (ci - g.ntc) * KC;
-            }
-            if (ok) ok = tc::bar_wait(&sm.kfull[st], (kcnt / NST) & 1, abort, kLimitNs);
-            if (!ok) {
+        bool ok = true;
+        for (int h = 0; h < H && ok; ++h) {
+          if (pt == 0) {
+            const int qb = qcnt & 1;
+            if (!tc::bar_wait(&sm.qempty[qb], ((qcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
               fail(sm, p.status);
+              ok = false;
+            } else {
+              tc::bar_expect_tx(&sm.qfull[qb], QBYTES);
+              tc::tma_load_2d(sm.q[qb], &mapQ, h * 128, (int)(g.t0 + g.j0), &sm.qfull[qb]);
+              tc::tma_load_2d(sm.q[qb] + QBYTES / 2, &mapQ, h * 128 + 64, (int)(g.t0 + g.j0), &sm.qfull[qb]);
+            }
+          }
+          ++qcnt;
+          for (int ci = 0; ci < nch && ok; ++ci) {
+            const int st = kcnt % NST;
+            if (!tc::bar_wait(&sm.kempty[st], ((kcnt / NST) & 1) ^ 1, abort, kLimitNs)) {
+              fail(sm, p.status);
+              ok = false;
               break;
             }
-            tc::fence_proxy_async();
-            tc::fence_after();
-            const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[st]);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const int kb = k >> 2, kk = k & 3;
-              tc::mma_bf16(d, tc::sdesc_sw128(qa + kb * (QBYTES / 2) + kk * 32),
-                           tc::sdesc_sw128(kbase + kb * (KBYTES / 2) + kk * 32), IDESC, k > 0 ? 1u : 0u);
+            const bool is_txt = ci < g.ntc;  // text chunks first: they do not wait for an E buffer
+            const int c = is_txt ? ci : ci - g.ntc;
+            const int* rows = is_txt ? &sm.kidx[ib][PMAX + c * KC] : &sm.kidx[ib][c * KC];
+            const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
+            const __nv_bfloat16* base = is_txt ? p.Kt : p.K;
+            uint8_t* dst = sm.k[st];
+  #pragma unroll
+            for (int i = 0; i < (KC * 16 + NPROD * 32 - 1) / (NPROD * 32); ++i) {
+              const int q = pt + NPROD * 32 * i;
+              if (q < KC * 16) {
+                const int key = q >> 4, c16 = q & 15;
+                const int kb = c16 >> 3, cc = c16 & 7;
+                const bool v = key < nv;
+                const __nv_bfloat16* src = base + (v ? (int64_t)rows[key] * HD + h * 128 + c16 * 8 : 0);
+                tc::cp_async16(dst + kb * (KBYTES / 2) + key * 128 + ((cc ^ (key & 7)) << 4), src, v ? 16 : 0);
+              }
             }
-            if (is_txt) {
-              tc::mma_commit(&sm.sfull[tcnt & 1]);
-              ++tcnt;
-            } else {
-              tc::mma_commit(&sm.efull[eb][ci - g.ntc]);
-            }
-            tc::mma_commit(&sm.kempty[st]);
+            tc::cp_async_arrive(&sm.kfull[st]);
             ++kcnt;
           }
-          if (!ok) break;
-          // the E-chunk barriers of chunks this item does not use still
-          // complete once per head, so every barrier's phase follows the head index
-          for (int c = g.nic; c < NIC_MAX; ++c) tc::mma_commit(&sm.efull[eb][c]);
-          tc::mma_commit(&sm.qempty[qb]);
-          ++qcnt;
         }
+        if (!ok) break;
       }
-      // every MMA issued by this thread has completed once this barrier flips
-      tc::mma_commit(&sm.mdone);
-      if (!tc::bar_wait(&sm.mdone, 0, nullptr, kLimitNs)) set_status(p.status, OCCAM_ERR_TIMEOUT);
+      if (pt == 0) sm.issued_q = qcnt;
+      asm volatile("cp.async.wait_all;" ::: "memory");
+    } else {
+      // ------------------------------------------------------------ MMA issuer
+      if (lane == 0) {
+        uint32_t qcnt = 0, kcnt = 0, tcnt = 0, hk = 0;
+        for (int item = cid; item < nF && !*abort; item += ncl) {
+          const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+          const int nch = g.nic + g.ntc;
+          for (int h = 0; h < H && !*abort; ++h, ++hk) {
+            const int qb = qcnt & 1;
+            if (!tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
+            const int eb = hk & 1;
+            bool ok = true;
+            for (int ci = 0; ci < nch && ok; ++ci) {
+              const bool is_txt = ci < g.ntc;
+              const int st = kcnt % NST;
+              uint32_t d;
+              if (is_txt) {
+                const int sb = tcnt & 1;
+                ok = tc::bar_wait(&sm.sempty[sb], ((tcnt >> 1) & 1) ^ 1, abort, kLimitNs);
+                d = tmem + S_COL + sb * KC;
+              } else {
+                // E[eb] is free once the probabilities of head hk - 2 were read out of it
+                if (ci == g.ntc && hk >= 2) ok = tc::bar_wait(&sm.efree[eb], ((hk - 2) >> 1) & 1, abort, kLimitNs);
+                d = tmem + E_COL + eb * PMAX + (ci - g.ntc) * KC;
+              }
+              if (ok) ok = tc::bar_wait(&sm.kfull[st], (kcnt / NST) & 1, abort, kLimitNs);
+              if (!ok) {
+                fail(sm, p.status);
+                break;
+              }
+              tc::fence_proxy_async();
+              tc::fence_after();
+              const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[st]);
+  #pragma unroll
+              for (int k = 0; k < 8; ++k) {
+                const int kb = k >> 2, kk = k & 3;
+                tc::mma_bf16(d, tc::sdesc_sw128(qa + kb * (QBYTES / 2) + kk * 32),
+                             tc::sdesc_sw128(kbase + kb * (KBYTES / 2) + kk * 32), IDESC, k > 0 ? 1u : 0u);
+              }
+              if (is_txt) {
+                tc::mma_commit(&sm.sfull[tcnt & 1]);
+                ++tcnt;
+              } else {
+                tc::mma_commit(&sm.efull[eb][ci - g.ntc]);
+              }
+              tc::mma_commit(&sm.kempty[st]);
+              ++kcnt;
+            }
+            if (!ok) break;
+            // the E-chunk barriers of chunks this item does not use still
+            // complete once per head, so every barrier's phase follows the head index
+            for (int c = g.nic; c < NIC_MAX; ++c) tc::mma_commit(&sm.efull[eb][c]);
+            tc::mma_commit(&sm.qempty[qb]);
+            ++qcnt;
+          }
+        }
+        // every MMA issued by this thread has completed once this barrier flips
+        tc::mma_commit(&sm.mdone);
+        if (!tc::bar_wait(&sm.mdone, 0, nullptr, kLimitNs)) set_status(p.status, OCCAM_ERR_TIMEOUT);
+      }
+      __syncwarp();
     }
-    __syncwarp();
   } else {
+    // warpgroups 1 and 2: the epilogue takes them
+    tc::setmaxnreg_inc<REG_HIGH>();
     // ------------------------------------------------------------ epilogue
     const int ew = warp - EPI_WARP0;    // 0..NEPI-1
     const int half = ew >> 2;           // the 32-column half of every chunk this warp owns
@@ -395,16 +407,19 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       for (int c = 0; c < NIC_MAX; ++c)
 #pragma unroll
         for (int b2 = 0; b2 < 32; ++b2) P[c][b2] = 0.f;
-      float cmc[NIC_MAX], cmp[NIC_MAX];  // half-chunk maxima of the current / previous head
+      float cmx[NIC_MAX];  // half-chunk maxima of the last head whose statistics were taken
 #pragma unroll
-      for (int c = 0; c < NIC_MAX; ++c) cmc[c] = cmp[c] = -INFINITY;
+      for (int c = 0; c < NIC_MAX; ++c) cmx[c] = -INFINITY;
       bool ok = true;
+      // Step s takes the text-key statistics of head s, then adds head s-1
+      // into P (which frees head s-1's E buffer for head s+1's MMAs while
+      // this step still works on head s), then the S1-key statistics of head
+      // s, and finally posts head s's (max, sum).
       for (int step = 0; step <= H && ok; ++step) {
         const uint32_t hcur = hk + step;  // global index of head `step` of this item
+        float m = -INFINITY, z = 0.f;
         if (step < H) {
-          // ---- statistics of head `step`: text-key chunks, then S1-key chunks
-          const int eb = hcur & 1;
-          float m = -INFINITY, z = 0.f;
+          // ---- text-key chunks of head `step` (scratch ring)
           for (int c = 0; c < g.ntc; ++c, ++tcnt) {
             const int sb = tcnt & 1;
             if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[sb], (tcnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
@@ -420,75 +435,81 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             __syncwarp();
             if (lane == 0) tc::bar_arrive(&sm.sempty[sb]);
           }
+        }
+        if (ok && step >= 1) {
+          // ---- probabilities of head step-1 over this warp's columns, added into P
+          const uint32_t hp = hcur - 1;
+          const int slot = hp & (NXS - 1);
+          const int eb = hp & 1;
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (hp / NXS) & 1, nullptr, kLimitNs, true))) {
+            ok = false;
+          } else {
+            if (wvalid) {
+              float Mx = -INFINITY;
+#pragma unroll
+              for (int r = 0; r < C; ++r) Mx = tc::fmax3(Mx, sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x);
+              float Z = 0.f;
+#pragma unroll
+              for (int r = 0; r < C; ++r)
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                  const float2 e = sm.xch[slot][r][hh][j];
+                  if (e.y > 0.f) Z += e.y * tc::ex2(e.x - Mx);
+                }
+              const float invZ = (vrow && Z > 0.f) ? 1.0f / Z : 0.f;
+              tc::fence_after();
+#pragma unroll
+              for (int c = 0; c < NIC_MAX; ++c) {
+                if (c < g.nic) {
+                  const float f = (invZ > 0.f && cmx[c] != -INFINITY) ? tc::ex2(cmx[c] - Mx) * invZ : 0.f;
+                  uint32_t v[32];
+                  tc::tmem_ld32(tmem + lane_base + E_COL + eb * PMAX + c * KC + half * 32, v);
+                  tc::tmem_wait_ld();
+                  const float2 ff = make_float2(f, f);
+#pragma unroll
+                  for (int i = 0; i < 16; ++i) {
+                    const float2 r2 = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])),
+                                                 ff, make_float2(P[c][2 * i], P[c][2 * i + 1]));
+                    P[c][2 * i] = r2.x;
+                    P[c][2 * i + 1] = r2.y;
+                  }
+                }
+              }
+            }
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) tc::bar_arrive(&sm.efree[eb]);
+            // the slot's phase for head hp is complete: arm it for head hp + NXS
+            if (armer) tc::bar_expect_tx(&sm.xbar[slot], Smem<C>::XBYTES);
+          }
+        }
+        if (ok && step < H) {
+          // ---- S1-key chunks of head `step` (E buffer), then the exchange
+          const int eb = hcur & 1;
 #pragma unroll
           for (int c = 0; c < NIC_MAX; ++c) {
-            cmc[c] = -INFINITY;
+            cmx[c] = -INFINITY;
             if (ok && c < g.nic) {
               if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.efull[eb][c], (hcur >> 1) & 1, nullptr, kLimitNs))) {
                 ok = false;
               } else if (wvalid) {
                 const int lim = vrow ? min(KC, g.own_img - c * KC) - half * 32 : 0;
                 float a;
-                half_stats<true>(tmem + lane_base + E_COL + eb * PMAX + c * KC + half * 32, lim, sl2, cmc[c], a);
-                online_merge(m, z, cmc[c], a);
+                half_stats<true>(tmem + lane_base + E_COL + eb * PMAX + c * KC + half * 32, lim, sl2, cmx[c], a);
+                online_merge(m, z, cmx[c], a);
               }
             }
           }
           if (wvalid) tc::tmem_wait_st();
           tc::fence_before();
-          if (!ok) break;
-          // ---- post this head's (max, sum) to every epilogue warp of the cluster
-          const int slot = hcur & (NXS - 1);
-#pragma unroll
-          for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][half][j], &sm.xbar[slot], (uint32_t)r, m, z);
-        }
-        if (step >= 1) {
-          // ---- probabilities of head step-1 over this warp's columns, added into P
-          const uint32_t hp = hcur - 1;
-          const int slot = hp & (NXS - 1);
-          const int eb = hp & 1;
-          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (hp / NXS) & 1, nullptr, kLimitNs, true))) { ok = false; break; }
-          if (wvalid) {
-            float Mx = -INFINITY;
+          if (ok) {
+            // ---- post this head's (max, sum) to every epilogue warp of the cluster
+            const int slot = hcur & (NXS - 1);
 #pragma unroll
             for (int r = 0; r < C; ++r)
-              Mx = tc::fmax3(Mx, sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x);
-            float Z = 0.f;
-#pragma unroll
-            for (int r = 0; r < C; ++r)
-#pragma unroll
-              for (int hh = 0; hh < 2; ++hh) {
-                const float2 e = sm.xch[slot][r][hh][j];
-                if (e.y > 0.f) Z += e.y * tc::ex2(e.x - Mx);
-              }
-            const float invZ = (vrow && Z > 0.f) ? 1.0f / Z : 0.f;
-            tc::fence_after();
-#pragma unroll
-            for (int c = 0; c < NIC_MAX; ++c) {
-              if (c < g.nic) {
-                const float f = (invZ > 0.f && cmp[c] != -INFINITY) ? tc::ex2(cmp[c] - Mx) * invZ : 0.f;
-                uint32_t v[32];
-                tc::tmem_ld32(tmem + lane_base + E_COL + eb * PMAX + c * KC + half * 32, v);
-                tc::tmem_wait_ld();
-                const float2 ff = make_float2(f, f);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                  const float2 r2 = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), ff,
-                                               make_float2(P[c][2 * i], P[c][2 * i + 1]));
-                  P[c][2 * i] = r2.x;
-                  P[c][2 * i + 1] = r2.y;
-                }
-              }
-            }
+              tc::st_async_f2(&sm.xch[slot][rank][half][j], &sm.xbar[slot], (uint32_t)r, m, z);
           }
-          tc::fence_before();
-          __syncwarp();
-          if (lane == 0) tc::bar_arrive(&sm.efree[eb]);
-          // the slot's phase for head hp is complete: arm it for head hp + NXS
-          if (armer) tc::bar_expect_tx(&sm.xbar[slot], Smem<C>::XBYTES);
         }
-#pragma unroll
-        for (int c = 0; c < NIC_MAX; ++c) cmp[c] = cmc[c];
       }
       hk += H;
       if (!ok) { fail(sm, p.status); break; }
@@ -500,28 +521,40 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         for (int c = 0; c < NIC_MAX; ++c) {
           if (c < g.nic) {
             // transpose-reduce over the 32 rows of this warp: afterwards lane l
-            // holds the max and the sum of this warp's column l of chunk c
-            float mx[32], su[32];
+            // holds the max (and, where a register key is among the columns,
+            // the sum) of this warp's column l of chunk c -- 31 shuffles each
+            const int key = c * KC + half * 32 + lane;
+            const bool live = key < g.own_img;
+            const bool is_reg = live && sm.kreg[ib][key];
+            float t[32];
 #pragma unroll
-            for (int col = 0; col < 32; ++col) mx[col] = su[col] = vrow ? P[c][col] : 0.f;
+            for (int col = 0; col < 32; ++col) t[col] = vrow ? P[c][col] : 0.f;
 #pragma unroll
             for (int sft = 16; sft >= 1; sft >>= 1) {
               const bool up = (lane & sft) != 0;
 #pragma unroll
               for (int i = 0; i < sft; ++i) {
-                const float sm_send = up ? mx[i] : mx[i + sft];
-                const float sm_keep = up ? mx[i + sft] : mx[i];
-                const float ss_send = up ? su[i] : su[i + sft];
-                const float ss_keep = up ? su[i + sft] : su[i];
-                mx[i] = fmaxf(sm_keep, __shfl_xor_sync(0xffffffffu, sm_send, sft));
-                su[i] = ss_keep + __shfl_xor_sync(0xffffffffu, ss_send, sft);
+                const float send = up ? t[i] : t[i + sft];
+                const float keep = up ? t[i + sft] : t[i];
+                t[i] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, sft));
               }
             }
-            const int key = c * KC + half * 32 + lane;
+            if (live && !is_reg) atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(t[0] * invH));
             float rc = 0.f;
-            if (key < g.own_img) {
-              if (sm.kreg[ib][key]) rc = su[0] * invH;
-              else atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(mx[0] * invH));
+            if (__any_sync(0xffffffffu, is_reg)) {
+#pragma unroll
+              for (int col = 0; col < 32; ++col) t[col] = vrow ? P[c][col] : 0.f;
+#pragma unroll
+              for (int sft = 16; sft >= 1; sft >>= 1) {
+                const bool up = (lane & sft) != 0;
+#pragma unroll
+                for (int i = 0; i < sft; ++i) {
+                  const float send = up ? t[i] : t[i + sft];
+                  const float keep = up ? t[i + sft] : t[i];
+                  t[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+                }
+              }
+              if (is_reg) rc = t[0] * invH;
             }
             regacc += warp_sum_f(rc);
           }
@@ -584,6 +617,14 @@ int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUte
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  // the register split inside the kernel needs the launch to reserve at least
+  // REG_NEEDED registers per CTA; refuse rather than launch a kernel whose
+  // setmaxnreg.inc could never be satisfied
+  cudaFuncAttributes fa;
+  if ((C == 8 ? cudaFuncGetAttributes(&fa, s2_fused_kernel<8>) : cudaFuncGetAttributes(&fa, s2_fused_kernel<4>)) !=
+      cudaSuccess)
+    return 1;
+  if (fa.numRegs * s2f::THREADS < s2f::REG_NEEDED) return 2;
   cudaError_t e;
   if (C == 8) {
     cudaFuncSetAttribute(s2_fused_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(8));

@@ -217,6 +217,16 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// per-warpgroup register budget (all four warps of the warpgroup execute it)
+template <int N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <int N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+
 // three-input maximum (sm_100+)
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float d;
