@@ -339,12 +339,10 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
   trace.mark(st);
   const int sms = num_sms();
   if (fused) {
-    CUtensorMap mq, mk, mkt;
+    CUtensorMap mq;
     const int64_t cols = (int64_t)a->H2 * 128;
     const void* kt = a->K_text ? a->K_text : a->Q_text;
-    if (!encode_map(&mq, a->Q_text, b->total_text, cols, 128) || !encode_map(&mk, a->K2, b->total_rows, cols, 1) ||
-        !encode_map(&mkt, kt, b->total_text, cols, 1))
-      return OCCAM_ERR_CUDA;
+    if (!encode_map(&mq, a->Q_text, b->total_text, cols, 128)) return OCCAM_ERR_CUDA;
     Stage2TcParams q;
     q.bt = p.bt;
     q.H = a->H2;
@@ -366,11 +364,10 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     q.lambda2 = lambda2;
     q.status = p.status;
     const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
-    if (launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
+    if (launch_fused(4, mq, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
     q.items = p.itemsF8;
     const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
-    if (launch_fused(8, mq, mk, mkt, q, ncl8, st) != 0) return OCCAM_ERR_CUDA;
-
+    if (launch_fused(8, mq, q, ncl8, st) != 0) return OCCAM_ERR_CUDA;
   }
   trace.mark(st);
   const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);

@@ -8,9 +8,20 @@
 namespace occam {
 
 constexpr int kFusedCluster = 4;        // CTAs per cluster of the fused tcgen05 Stage-II kernel (C = 8 variant for larger S1)
-constexpr int kFusedMaxOwnImg = 192;    // S1 keys one of its CTAs can hold (two TMEM buffers of this many columns)
-constexpr int kFusedMaxOwnTxt = 256;    // text keys one of its CTAs can take
+constexpr int kFusedMaxOwnImg = 192;    // S1 keys one of its CTAs can hold (P columns kept in registers)
+constexpr int kFusedKeyRows4 = 256;     // key rows per head one CTA of a 4-CTA cluster holds (= MMA N and TMEM columns)
+constexpr int kFusedKeyRows8 = 224;     // the same for an 8-CTA cluster (its exchange buffers take more shared memory)
 constexpr int kFusedEpiWarps = 8;       // epilogue warps per CTA of the fused kernel
+
+// Whether a sample with n1 S1 keys and M text tokens fits the fused kernel
+// with C CTAs per cluster: each CTA takes ceil(n1 / C) S1 keys (padded to 32)
+// and, for the last text tile, ceil(M / C) causal text keys (padded to 16).
+__host__ __device__ inline bool fused_fits(int C, int n1, int M) {
+  const int rows = C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;
+  const int ip = ((n1 + C - 1) / C + 31) & ~31;
+  const int tp = ((M + C - 1) / C + 15) & ~15;
+  return M > 0 && ip <= kFusedMaxOwnImg && ip + tp <= rows;
+}
 constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedEpiWarps;  // s2(r) partials per C=4 item (one per epilogue warp)
 constexpr int kFusedSlotsPerItem8 = 8 * kFusedEpiWarps;             // and per C=8 item
 constexpr int kMaxClsRowsPerCta = 512;  // rows of one segment handled by one CTA of a [CLS] cluster
@@ -169,8 +180,7 @@ int s2_scores_smem_bytes();
 int s2_stats_smem_bytes();
 
 // stage2_tc.cu
-int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt,
-                 const Stage2TcParams& q, int nclusters, cudaStream_t st);
+int launch_fused(int C, const CUtensorMap& mq, const Stage2TcParams& q, int nclusters, cudaStream_t st);
 int s2_fused_smem_bytes(int C);
 int s2_fused_threads();
 

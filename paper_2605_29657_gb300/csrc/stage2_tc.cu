@@ -1,5 +1,5 @@
 // stage2_tc.cu -- fused Stage-II scoring on the 5th-generation tensor cores
-// (tcgen05 + TMEM), for samples whose S1 fits a 4-CTA cluster.
+// (tcgen05 + TMEM), for samples whose S1 fits a 4- or 8-CTA cluster.
 //
 // What it computes (Sec. 3.5, Eq. 7; App. A, Eqs. 15-16): for sample b, text
 // token j and head h, A_{j,h} = softmax over {S1 rows of b} u {text keys 0..j}
@@ -9,27 +9,29 @@
 // Work item = (sample, tile of 128 text rows), processed by one cluster of C
 // CTAs (C = 4, or 8 for samples with more S1 keys). The text rows are the 128
 // TMEM lanes; each CTA owns 1/C of the sample's S1 keys and of the causal
-// text keys. Per head:
-//   1. three producer warps stream the CTA's key rows in 64-key chunks with
-//      16-byte cp.async into the 128-byte-swizzled operand layout (S1 rows
-//      are gathered by index straight from K2: pruned rows are never read,
-//      every key row is read once per text tile); the head's 128 x 128 query
-//      tile arrives by TMA;
-//   2. one thread issues S = Q K^T per chunk (tcgen05.mma, bf16 in, fp32 in
-//      TMEM): text-key chunks into a two-deep scratch ring, S1-key chunks
-//      into a per-head TMEM buffer E (two buffers, alternating by head);
+// text keys. Per head, a CTA's keys form one block of N <= 256 rows: its S1
+// keys (padded to a multiple of 32), then its text keys (padded to 16).
+//   1. seven producer warps gather the block's rows with 16-byte cp.async
+//      into the 128-byte-swizzled operand layout (S1 rows straight from K2 by
+//      index: pruned rows are never read); the head's 128 x 128 query tile
+//      arrives by TMA. Key blocks and query tiles are double-buffered by head;
+//   2. one thread issues S = Q K^T for the whole block as eight
+//      128 x N x 16 tcgen05.mma (bf16 in, fp32 accumulate) into a per-head
+//      TMEM buffer E (two buffers, alternating by head);
 //   3. eight epilogue warps (two per TMEM lane quadrant, one thread per text
-//      row) each own one 32-column half of every chunk. A warp turns its
-//      logits into exp2(l - cmax) (cmax: the row max of that half-chunk, kept
-//      in a register), writes them back over S1-key logits in E, and keeps
+//      row) each own every other 32-column piece of E. A warp turns its
+//      logits into exp2(l - cmax) (cmax: the row max of that piece, kept in a
+//      register), writes the S1-key ones back over the logits in E, and keeps
 //      the row's running softmax max / sum;
 //   4. the (max, sum) pairs go to every epilogue warp of the cluster with
 //      asynchronous distributed-shared-memory stores that complete on an
-//      mbarrier of the receiving CTA (no fences). The exchange of head h is
-//      awaited only after head h+1's statistics, so its latency is hidden;
-//   5. then every warp adds exp2(cmax - max) / sum * E over its own columns to
-//      the head-summed probabilities P, which live in registers for the
-//      whole item.
+//      mbarrier of the receiving CTA (no fences);
+//   5. every warp then adds exp2(cmax - max) / sum * E over its S1-key
+//      pieces to the head-summed probabilities P, which live in registers for
+//      the whole item.
+// Step s of the epilogue takes the text-key statistics of head s, adds head
+// s-1 into P (freeing head s-1's E buffer, so the MMAs of head s+1 overlap
+// the rest of step s), then the S1-key statistics of head s, and posts them.
 // After the last head every warp reduces its P columns over its 32 rows:
 // column max -> s2 (atomicMax on the fp32 bit pattern, exact and order-free
 // since P >= 0), register columns -> a partial of s2(r) reduced in fixed order.
@@ -41,43 +43,42 @@ namespace occam {
 
 namespace s2f {
 constexpr int QR = 128;                // text rows per item (TMEM lanes)
-constexpr int KC = 64;                 // keys per chunk (MMA N)
-constexpr int NST = 4;                 // key-chunk ring stages
 constexpr int PMAX = kFusedMaxOwnImg;  // max S1 keys per CTA
-constexpr int NIC_MAX = PMAX / KC;     // S1-key chunks per CTA
-constexpr int TMAX = kFusedMaxOwnTxt;  // max text keys per CTA
+constexpr int NPW = PMAX / 64;         // S1-key pieces per epilogue warp
 constexpr int QBYTES = QR * 256;       // one head's query tile: 2 K-blocks x 128 rows x 128 B
-constexpr int KBYTES = KC * 256;       // one chunk: 2 K-blocks x 64 rows x 128 B
-constexpr int NPROD = 3;               // producer warps (0-2); warp 3 issues MMAs; then the epilogue warps
+constexpr int NPROD = 7;               // producer warps (0-6); warp 7 issues MMAs; then the epilogue warps
 constexpr int MMA_WARP = NPROD;
 constexpr int EPI_WARP0 = NPROD + 1;
 constexpr int NEPI = kFusedEpiWarps;   // two per TMEM lane quadrant
 constexpr int THREADS = (NPROD + 1 + NEPI) * 32;
-constexpr int NXS = 4;                 // exchange slots (the exchange runs one head behind)
-// register split: warpgroup 0 (producers + MMA issuer) shrinks to REG_LOW per
-// thread, the two epilogue warpgroups grow to REG_HIGH; the sum must stay
+constexpr int NXS = 2;                 // exchange slots (a peer runs at most one head ahead of a slot's reader)
+// register split: warpgroups 0-1 (producers + MMA issuer) shrink to REG_LOW
+// per thread, the two epilogue warpgroups grow to REG_HIGH; the sum must stay
 // within what the CTA was launched with (checked on the host before launch)
-constexpr int REG_LOW = 88, REG_HIGH = 208;
-constexpr int REG_NEEDED = 128 * REG_LOW + (THREADS - 128) * REG_HIGH;
-static_assert(NPROD + 1 == 4 && (THREADS - 128) % 128 == 0, "warpgroup 0 = producers + MMA warp");
-constexpr uint32_t IDESC = tc::idesc_bf16(128, KC);
+constexpr int REG_LOW = 56, REG_HIGH = 200;
+constexpr int REG_NEEDED = EPI_WARP0 * 32 * REG_LOW + NEPI * 32 * REG_HIGH;
+static_assert(EPI_WARP0 % 4 == 0 && NEPI % 4 == 0, "roles split on warpgroup boundaries");
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int S_COL = 0;               // two scratch buffers (text-key chunks), KC columns each
-constexpr int E_COL = 2 * KC;          // two E buffers (by head parity), PMAX columns each
-static_assert(E_COL + 2 * PMAX <= (int)TMEM_COLS, "TMEM budget");
-static_assert(PMAX % KC == 0, "E buffers hold whole chunks");
+static_assert(2 * kFusedKeyRows4 <= (int)TMEM_COLS && 2 * kFusedKeyRows8 <= (int)TMEM_COLS, "two E buffers");
+static_assert(kFusedKeyRows4 % 32 == 0 && kFusedKeyRows8 % 32 == 0 && kFusedKeyRows4 <= 256, "MMA N <= 256");
+static_assert(PMAX % 64 == 0, "S1-key pieces split evenly between the two warps of a quadrant");
 constexpr uint64_t kLimitNs = 2000000000ull;
 
 template <int C>
+struct Geo {
+  static constexpr int KROWS = C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;  // key rows per head (max MMA N)
+  static constexpr int KBLK = KROWS * 128;                                  // bytes of one K-block of the key rows
+  static constexpr uint32_t XBYTES = C * NEPI * 32 * 8;                     // exchange bytes a CTA receives per head
+};
+
+template <int C>
 struct Smem {
-  static constexpr uint32_t XBYTES = C * NEPI * 32 * 8;  // exchange bytes one CTA receives per head
   uint8_t q[2][QBYTES];
-  uint8_t k[NST][KBYTES];
-  int32_t kidx[2][PMAX + TMAX];
-  float2 xch[NXS][C][2][QR];          // (max, sum) per (slot, CTA, epilogue half, row)
+  uint8_t k[2][2 * Geo<C>::KBLK];
+  float2 xch[NXS][C][2][QR];  // (max, sum) per (slot, CTA, epilogue half, row)
+  int32_t kidx[2][PMAX];
   uint8_t kreg[2][PMAX];
-  uint64_t kfull[NST], kempty[NST], qfull[2], qempty[2], sfull[2], sempty[2], efull[2][NIC_MAX], efree[2],
-      xbar[NXS], iready[2], idone[2], mdone;
+  uint64_t kfull[2], kempty[2], qfull[2], qempty[2], efull[2], efree[2], xbar[NXS], iready[2], idone[2], mdone;
   uint32_t tmem_base;
   int abort;
   uint32_t issued_q;
@@ -92,7 +93,8 @@ int s2_fused_threads() { return s2f::THREADS; }
 namespace {
 
 struct ItemGeom {
-  int b, j0, M, n, img0, own_img, txt0, own_txt, nic, ntc, slot;
+  int b, j0, M, n, img0, own_img, txt0, own_txt, ip, tp, N, slot;
+  bool fits;
   int64_t rbase, t0;
 };
 
@@ -114,8 +116,12 @@ __device__ __forceinline__ ItemGeom item_geom(const Stage2TcParams& p, int4 it, 
   const int per_t = (n_txt + C - 1) / C;
   g.txt0 = rank * per_t;
   g.own_txt = max(0, min(per_t, n_txt - g.txt0));
-  g.nic = (g.own_img + KC - 1) / KC;
-  g.ntc = (g.own_txt + KC - 1) / KC;
+  g.ip = (g.own_img + 31) & ~31;
+  g.tp = (g.own_txt + 15) & ~15;
+  g.N = g.ip + g.tp;
+  // the same on every CTA of the cluster (depends on the sample only)
+  const int ipmax = (per + 31) & ~31;
+  g.fits = ipmax <= PMAX && ipmax + ((per_t + 15) & ~15) <= Geo<C>::KROWS;
   return g;
 }
 
@@ -131,22 +137,30 @@ __device__ __forceinline__ float warp_sum_f(float v) {
   return v;
 }
 
-// Statistics of one thread's row over a 32-column half-chunk of logits at
-// TMEM address sa (warp-collective): cm = max of the first `lim` columns in
-// log2 units (-inf if none), a = sum over them of exp2(l * sl2 - cm). With
-// STORE the exponentials (0 past lim) are written back over the logits; the
-// caller waits for that store before the values are read again.
-template <bool STORE>
-__device__ __forceinline__ void half_stats(uint32_t sa, int lim, float sl2, float& cm, float& a) {
-  cm = -INFINITY;
-  a = 0.f;
-  if (__all_sync(0xffffffffu, lim <= 0)) return;
-  const bool full = __all_sync(0xffffffffu, lim >= 32);
-  uint32_t v[32];
-  tc::fence_after();
-  tc::tmem_ld32(sa, v);
+// Ties the 32 registers a tcgen05.ld wrote to the preceding wait::ld, so the
+// compiler cannot move their first use above it.
+__device__ __forceinline__ void reg_fence(uint32_t (&v)[32]) {
+  asm volatile(""
+               : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
+                 "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]), "+r"(v[12]), "+r"(v[13]), "+r"(v[14]), "+r"(v[15]),
+                 "+r"(v[16]), "+r"(v[17]), "+r"(v[18]), "+r"(v[19]), "+r"(v[20]), "+r"(v[21]), "+r"(v[22]), "+r"(v[23]),
+                 "+r"(v[24]), "+r"(v[25]), "+r"(v[26]), "+r"(v[27]), "+r"(v[28]), "+r"(v[29]), "+r"(v[30]), "+r"(v[31]));
+}
+
+__device__ __forceinline__ void ld_wait(uint32_t (&v)[32]) {
   tc::tmem_wait_ld();
-  if (full) {
+  reg_fence(v);
+}
+
+// Statistics of one thread's row over a 32-column piece of logits already
+// loaded into v (warp-collective): cm = max of the first `lim` columns in
+// log2 units (-inf if none), a = sum over them of exp2(l * sl2 - cm). v is
+// overwritten with the exponentials (0 past lim); with STORE they are also
+// written back to TMEM at sa (the caller waits for that store before the
+// values are read again).
+template <bool STORE>
+__device__ __forceinline__ void piece_stats(uint32_t (&v)[32], uint32_t sa, int lim, float sl2, float& cm, float& a) {
+  if (__all_sync(0xffffffffu, lim >= 32)) {
     float t[11];
 #pragma unroll
     for (int i = 0; i < 10; ++i)
@@ -156,18 +170,17 @@ __device__ __forceinline__ void half_stats(uint32_t sa, int lim, float sl2, floa
                            fmaxf(t[9], t[10]));
     cm = mx * sl2;
     const float2 sc = make_float2(sl2, sl2), off = make_float2(-cm, -cm);
-    float2 acc0 = make_float2(0.f, 0.f), acc1 = acc0;
+    float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), sc, off);
       x.x = tc::ex2(x.x);
       x.y = tc::ex2(x.y);
-      if (i & 1) acc1 = __fadd2_rn(acc1, x);
-      else acc0 = __fadd2_rn(acc0, x);
+      acc[i & 3] = __fadd2_rn(acc[i & 3], x);
       v[2 * i] = __float_as_uint(x.x);
       v[2 * i + 1] = __float_as_uint(x.y);
     }
-    a = (acc0.x + acc0.y) + (acc1.x + acc1.y);
+    a = ((acc[0].x + acc[0].y) + (acc[1].x + acc[1].y)) + ((acc[2].x + acc[2].y) + (acc[3].x + acc[3].y));
   } else {
     float c0 = -INFINITY, c1 = -INFINITY;
 #pragma unroll
@@ -191,7 +204,7 @@ __device__ __forceinline__ void half_stats(uint32_t sa, int lim, float sl2, floa
   if (STORE) tc::tmem_st32(sa, v);
 }
 
-// merges a half-chunk's (cm, a) into the row's running softmax (m, z), log2 units
+// merges a piece's (cm, a) into the row's running softmax (m, z), log2 units
 __device__ __forceinline__ void online_merge(float& m, float& z, float cm, float a) {
   if (cm != -INFINITY) {
     const float mn = fmaxf(m, cm);
@@ -200,13 +213,25 @@ __device__ __forceinline__ void online_merge(float& m, float& z, float cm, float
   }
 }
 
+// P[col] += f * v[col] over one 32-column piece
+__device__ __forceinline__ void p_accum(float (&P)[32], const uint32_t (&v)[32], float f) {
+  const float2 ff = make_float2(f, f);
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const float2 r2 = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), ff,
+                                 make_float2(P[2 * i], P[2 * i + 1]));
+    P[2 * i] = r2.x;
+    P[2 * i + 1] = r2.y;
+  }
+}
+
 }  // namespace
 
 template <int C>
 __global__ void __launch_bounds__(s2f::THREADS, 1)
-    s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
-                    const __grid_constant__ CUtensorMap mapKt, Stage2TcParams p) {
+    s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, Stage2TcParams p) {
   using namespace s2f;
+  using G = Geo<C>;
   extern __shared__ unsigned char smem_raw[];
   Smem<C>& sm = *reinterpret_cast<Smem<C>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -214,17 +239,14 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   const int nF = p.counters[C == 8 ? CNT_NF8 : CNT_NF];
   const int cid = (int)tc::cluster_id_x(), ncl = (int)tc::nclusters_x();
   volatile int* abort = &sm.abort;
-  (void)mapK;
-  (void)mapKt;
 
   if (tid == 0) {
-    for (int i = 0; i < NST; ++i) { tc::bar_init(&sm.kfull[i], NPROD * 32); tc::bar_init(&sm.kempty[i], 1); }
     for (int i = 0; i < 2; ++i) {
+      tc::bar_init(&sm.kfull[i], NPROD * 32);
+      tc::bar_init(&sm.kempty[i], 1);
       tc::bar_init(&sm.qfull[i], 1);
       tc::bar_init(&sm.qempty[i], 1);
-      tc::bar_init(&sm.sfull[i], 1);
-      tc::bar_init(&sm.sempty[i], NEPI);
-      for (int c = 0; c < NIC_MAX; ++c) tc::bar_init(&sm.efull[i][c], 1);
+      tc::bar_init(&sm.efull[i], 1);
       tc::bar_init(&sm.efree[i], NEPI);
       tc::bar_init(&sm.iready[i], NPROD * 32);
       tc::bar_init(&sm.idone[i], NEPI);
@@ -236,32 +258,33 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     sm.abort = 0;
     sm.issued_q = 0;
     tc::bar_fence_init();
-    for (int i = 0; i < NXS; ++i) tc::bar_expect_tx(&sm.xbar[i], Smem<C>::XBYTES);
+    for (int i = 0; i < NXS; ++i) tc::bar_expect_tx(&sm.xbar[i], G::XBYTES);
     tc::prefetch_map(&mapQ);
   }
   if (warp == MMA_WARP) tc::tmem_alloc(&sm.tmem_base, TMEM_COLS);
   tc::fence_before();
   __syncthreads();
   tc::fence_after();
-  // peers' barriers must be initialised before anyone arrives on them remotely
+  // peers' barriers must be initialised before anyone stores into them remotely
   tc::cluster_sync_all();
   const uint32_t tmem = sm.tmem_base;
   const int H = p.H;
 
-  if (warp < 4) {
-    // warpgroup 0: producers and the MMA issuer give registers back
+  if (warp < EPI_WARP0) {
+    // warpgroups 0-1: producers and the MMA issuer give registers back
     tc::setmaxnreg_dec<REG_LOW>();
     if (warp < NPROD) {
-      // ------------------------------------------------------------ producers
-      // 96 threads; piece q = pt + 96 i (q < 1024) of a chunk is 16 bytes of key
-      // row (q >> 4), head slice bytes 16 * (q & 15); it lands at the row's
-      // 128-byte line of its K-block with the 16-byte chunk index XOR (row & 7).
+      // ---------------------------------------------------------- producers
+      // NPROD * 32 threads; piece q (16 bytes) of the key block is row (q >> 4), head
+      // slice bytes 16 * (q & 15); it lands at the row's 128-byte line of its
+      // K-block with the 16-byte chunk index XOR (row & 7).
       const int pt = tid;
       uint32_t qcnt = 0, kcnt = 0;
       int ii = 0;
       const int64_t HD = (int64_t)H * 128;
       for (int item = cid; item < nF; item += ncl, ++ii) {
         const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+        if (!g.fits) continue;
         const int ib = ii & 1;
         if (*abort || !tc::bar_wait(&sm.idone[ib], ((ii >> 1) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
         for (int i = pt; i < g.own_img; i += NPROD * 32) {
@@ -269,12 +292,17 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
           sm.kidx[ib][i] = row;
           sm.kreg[ib][i] = p.role[row];
         }
-        for (int i = pt; i < g.own_txt; i += NPROD * 32) sm.kidx[ib][PMAX + i] = (int)(g.t0 + g.txt0 + i);
         tc::bar_arrive(&sm.iready[ib]);
         if (!tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-        const int nch = g.nic + g.ntc;
+        const int64_t tbase = g.t0 + g.txt0;
         bool ok = true;
         for (int h = 0; h < H && ok; ++h) {
+          const int kb = kcnt & 1;
+          if (!tc::bar_wait(&sm.kempty[kb], ((kcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
+            fail(sm, p.status);
+            ok = false;
+            break;
+          }
           if (pt == 0) {
             const int qb = qcnt & 1;
             if (!tc::bar_wait(&sm.qempty[qb], ((qcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
@@ -287,92 +315,64 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             }
           }
           ++qcnt;
-          for (int ci = 0; ci < nch && ok; ++ci) {
-            const int st = kcnt % NST;
-            if (!tc::bar_wait(&sm.kempty[st], ((kcnt / NST) & 1) ^ 1, abort, kLimitNs)) {
-              fail(sm, p.status);
-              ok = false;
-              break;
+          uint8_t* dst = sm.k[kb];
+          const int nq = g.N * 16;
+          for (int q = pt; q < nq; q += NPROD * 32) {
+            const int row = q >> 4, c16 = q & 15;
+            const int kblk = c16 >> 3, cc = c16 & 7;
+            const __nv_bfloat16* src = p.K;
+            int bytes = 0;
+            if (row < g.own_img) {
+              src = p.K + (int64_t)sm.kidx[ib][row] * HD + h * 128 + c16 * 8;
+              bytes = 16;
+            } else if (row >= g.ip && row - g.ip < g.own_txt) {
+              src = p.Kt + (tbase + (row - g.ip)) * HD + h * 128 + c16 * 8;
+              bytes = 16;
             }
-            const bool is_txt = ci < g.ntc;  // text chunks first: they do not wait for an E buffer
-            const int c = is_txt ? ci : ci - g.ntc;
-            const int* rows = is_txt ? &sm.kidx[ib][PMAX + c * KC] : &sm.kidx[ib][c * KC];
-            const int nv = is_txt ? min(KC, g.own_txt - c * KC) : min(KC, g.own_img - c * KC);
-            const __nv_bfloat16* base = is_txt ? p.Kt : p.K;
-            uint8_t* dst = sm.k[st];
-  #pragma unroll
-            for (int i = 0; i < (KC * 16 + NPROD * 32 - 1) / (NPROD * 32); ++i) {
-              const int q = pt + NPROD * 32 * i;
-              if (q < KC * 16) {
-                const int key = q >> 4, c16 = q & 15;
-                const int kb = c16 >> 3, cc = c16 & 7;
-                const bool v = key < nv;
-                const __nv_bfloat16* src = base + (v ? (int64_t)rows[key] * HD + h * 128 + c16 * 8 : 0);
-                tc::cp_async16(dst + kb * (KBYTES / 2) + key * 128 + ((cc ^ (key & 7)) << 4), src, v ? 16 : 0);
-              }
-            }
-            tc::cp_async_arrive(&sm.kfull[st]);
-            ++kcnt;
+            tc::cp_async16(dst + kblk * G::KBLK + row * 128 + ((cc ^ (row & 7)) << 4), src, bytes);
           }
+          tc::cp_async_arrive(&sm.kfull[kb]);
+          ++kcnt;
         }
         if (!ok) break;
       }
       if (pt == 0) sm.issued_q = qcnt;
       asm volatile("cp.async.wait_all;" ::: "memory");
     } else {
-      // ------------------------------------------------------------ MMA issuer
+      // ---------------------------------------------------------- MMA issuer
       if (lane == 0) {
-        uint32_t qcnt = 0, kcnt = 0, tcnt = 0, hk = 0;
+        uint32_t qcnt = 0, kcnt = 0, hk = 0;
         for (int item = cid; item < nF && !*abort; item += ncl) {
           const ItemGeom g = item_geom<C>(p, p.items[item], rank);
-          const int nch = g.nic + g.ntc;
-          for (int h = 0; h < H && !*abort; ++h, ++hk) {
-            const int qb = qcnt & 1;
-            if (!tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
-            const int eb = hk & 1;
-            bool ok = true;
-            for (int ci = 0; ci < nch && ok; ++ci) {
-              const bool is_txt = ci < g.ntc;
-              const int st = kcnt % NST;
-              uint32_t d;
-              if (is_txt) {
-                const int sb = tcnt & 1;
-                ok = tc::bar_wait(&sm.sempty[sb], ((tcnt >> 1) & 1) ^ 1, abort, kLimitNs);
-                d = tmem + S_COL + sb * KC;
-              } else {
-                // E[eb] is free once the probabilities of head hk - 2 were read out of it
-                if (ci == g.ntc && hk >= 2) ok = tc::bar_wait(&sm.efree[eb], ((hk - 2) >> 1) & 1, abort, kLimitNs);
-                d = tmem + E_COL + eb * PMAX + (ci - g.ntc) * KC;
-              }
-              if (ok) ok = tc::bar_wait(&sm.kfull[st], (kcnt / NST) & 1, abort, kLimitNs);
-              if (!ok) {
-                fail(sm, p.status);
-                break;
-              }
-              tc::fence_proxy_async();
-              tc::fence_after();
-              const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[st]);
-  #pragma unroll
-              for (int k = 0; k < 8; ++k) {
-                const int kb = k >> 2, kk = k & 3;
-                tc::mma_bf16(d, tc::sdesc_sw128(qa + kb * (QBYTES / 2) + kk * 32),
-                             tc::sdesc_sw128(kbase + kb * (KBYTES / 2) + kk * 32), IDESC, k > 0 ? 1u : 0u);
-              }
-              if (is_txt) {
-                tc::mma_commit(&sm.sfull[tcnt & 1]);
-                ++tcnt;
-              } else {
-                tc::mma_commit(&sm.efull[eb][ci - g.ntc]);
-              }
-              tc::mma_commit(&sm.kempty[st]);
-              ++kcnt;
+          if (!g.fits) continue;
+          const uint32_t idesc = tc::idesc_bf16(128, g.N > 0 ? g.N : 16);
+          bool ok = true;
+          for (int h = 0; h < H && ok; ++h, ++hk) {
+            const int qb = qcnt & 1, kb = kcnt & 1, eb = hk & 1;
+            // E[eb] is free once head hk - 2 was read out of it
+            ok = tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs);
+            if (ok && hk >= 2) ok = tc::bar_wait(&sm.efree[eb], ((hk - 2) >> 1) & 1, abort, kLimitNs);
+            if (ok) ok = tc::bar_wait(&sm.kfull[kb], (kcnt >> 1) & 1, abort, kLimitNs);
+            if (!ok) {
+              fail(sm, p.status);
+              break;
             }
-            if (!ok) break;
-            // the E-chunk barriers of chunks this item does not use still
-            // complete once per head, so every barrier's phase follows the head index
-            for (int c = g.nic; c < NIC_MAX; ++c) tc::mma_commit(&sm.efull[eb][c]);
+            tc::fence_proxy_async();
+            tc::fence_after();
+            if (g.N > 0) {
+              const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[kb]);
+#pragma unroll
+              for (int s = 0; s < 8; ++s) {
+                const int kblk = s >> 2, kk = s & 3;
+                tc::mma_bf16(tmem + eb * G::KROWS, tc::sdesc_sw128(qa + kblk * (QBYTES / 2) + kk * 32),
+                             tc::sdesc_sw128(kbase + kblk * G::KBLK + kk * 32), idesc, s > 0 ? 1u : 0u);
+              }
+            }
+            tc::mma_commit(&sm.efull[eb]);
+            tc::mma_commit(&sm.kempty[kb]);
             tc::mma_commit(&sm.qempty[qb]);
             ++qcnt;
+            ++kcnt;
           }
         }
         // every MMA issued by this thread has completed once this barrier flips
@@ -382,65 +382,73 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       __syncwarp();
     }
   } else {
-    // warpgroups 1 and 2: the epilogue takes them
+    // warpgroups 2-3: the epilogue takes them
     tc::setmaxnreg_inc<REG_HIGH>();
     // ------------------------------------------------------------ epilogue
     const int ew = warp - EPI_WARP0;    // 0..NEPI-1
-    const int half = ew >> 2;           // the 32-column half of every chunk this warp owns
+    const int half = ew >> 2;           // this warp owns the 32-column pieces of this parity
     const int quad = warp & 3;          // TMEM lane quadrant this warp may access
     const int j = quad * 32 + lane;     // text row of this thread inside the tile
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const float sl2 = p.scale_log2;
     const float invH = 1.0f / (float)H;
     const bool armer = ew == 0 && lane == 0;  // re-arms the exchange slots of this CTA
-    uint32_t tcnt = 0, hk = 0;
+    uint32_t hk = 0;
     int ii = 0;
     for (int item = cid; item < nF; item += ncl, ++ii) {
       const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+      if (!g.fits) {
+        if (tid == EPI_WARP0 * 32) set_status(p.status, OCCAM_ERR_UNSUPPORTED);
+        continue;
+      }
       const int ib = ii & 1;
       if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, nullptr, kLimitNs))) { fail(sm, p.status); break; }
       const bool vrow = g.j0 + j < g.M;
       const bool wvalid = __any_sync(0xffffffffu, vrow);  // warp-uniform: any real text row here
       const int jj = g.j0 + j;
-      float P[NIC_MAX][32];
+      const int npi = g.ip >> 5;                // S1-key pieces of this CTA
+      const int npc = (g.N + 31) >> 5;          // all pieces
+      bool own[NPW];                            // which of this warp's S1-key pieces exist
 #pragma unroll
-      for (int c = 0; c < NIC_MAX; ++c)
+      for (int q = 0; q < NPW; ++q) own[q] = 2 * q + half < npi;
+      float P[NPW][32];
 #pragma unroll
-        for (int b2 = 0; b2 < 32; ++b2) P[c][b2] = 0.f;
-      float cmx[NIC_MAX];  // half-chunk maxima of the last head whose statistics were taken
+      for (int q = 0; q < NPW; ++q)
 #pragma unroll
-      for (int c = 0; c < NIC_MAX; ++c) cmx[c] = -INFINITY;
+        for (int b2 = 0; b2 < 32; ++b2) P[q][b2] = 0.f;
+      float cmx[NPW];  // piece maxima of the last head whose statistics were taken
+#pragma unroll
+      for (int q = 0; q < NPW; ++q) cmx[q] = -INFINITY;
       bool ok = true;
-      // Step s takes the text-key statistics of head s, then adds head s-1
-      // into P (which frees head s-1's E buffer for head s+1's MMAs while
-      // this step still works on head s), then the S1-key statistics of head
-      // s, and finally posts head s's (max, sum).
       for (int step = 0; step <= H && ok; ++step) {
         const uint32_t hcur = hk + step;  // global index of head `step` of this item
+        const int eb = hcur & 1;
+        const uint32_t ebase = tmem + lane_base + eb * G::KROWS;
         float m = -INFINITY, z = 0.f;
         if (step < H) {
-          // ---- text-key chunks of head `step` (scratch ring)
-          for (int c = 0; c < g.ntc; ++c, ++tcnt) {
-            const int sb = tcnt & 1;
-            if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sfull[sb], (tcnt >> 1) & 1, nullptr, kLimitNs))) { ok = false; break; }
-            if (wvalid) {
-              const int nv = min(KC, g.own_txt - c * KC);
-              const int tbase = g.txt0 + c * KC + half * 32;  // sample-relative text index of this half's column 0
-              const int lim = vrow ? min(nv - half * 32, jj - tbase + 1) : 0;
+          // ---- text-key pieces of head `step`
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.efull[eb], (hcur >> 1) & 1, nullptr, kLimitNs))) {
+            ok = false;
+          } else if (wvalid) {
+            tc::fence_after();
+            for (int pc = npi + ((npi ^ half) & 1); pc < npc; pc += 2) {
+              const int tb = g.txt0 + pc * 32 - g.ip;  // sample-relative text index of the piece's column 0
+              const int lim = vrow ? min(g.own_txt - (pc * 32 - g.ip), jj - tb + 1) : 0;
+              if (__all_sync(0xffffffffu, lim <= 0)) continue;
+              uint32_t v[32];
+              tc::tmem_ld32(ebase + pc * 32, v);
+              ld_wait(v);
               float cm, a;
-              half_stats<false>(tmem + lane_base + S_COL + sb * KC + half * 32, lim, sl2, cm, a);
+              piece_stats<false>(v, 0, lim, sl2, cm, a);
               online_merge(m, z, cm, a);
             }
-            tc::fence_before();
-            __syncwarp();
-            if (lane == 0) tc::bar_arrive(&sm.sempty[sb]);
           }
         }
         if (ok && step >= 1) {
-          // ---- probabilities of head step-1 over this warp's columns, added into P
+          // ---- probabilities of head step-1 over this warp's S1-key pieces, added into P
           const uint32_t hp = hcur - 1;
           const int slot = hp & (NXS - 1);
-          const int eb = hp & 1;
+          const int pb = hp & 1;
           if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (hp / NXS) & 1, nullptr, kLimitNs, true))) {
             ok = false;
           } else {
@@ -457,58 +465,61 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
                   if (e.y > 0.f) Z += e.y * tc::ex2(e.x - Mx);
                 }
               const float invZ = (vrow && Z > 0.f) ? 1.0f / Z : 0.f;
+              float f[NPW];
+#pragma unroll
+              for (int q = 0; q < NPW; ++q) f[q] = (invZ > 0.f && cmx[q] != -INFINITY) ? tc::ex2(cmx[q] - Mx) * invZ : 0.f;
+              const uint32_t pbase = tmem + lane_base + pb * G::KROWS + half * 32;
               tc::fence_after();
 #pragma unroll
-              for (int c = 0; c < NIC_MAX; ++c) {
-                if (c < g.nic) {
-                  const float f = (invZ > 0.f && cmx[c] != -INFINITY) ? tc::ex2(cmx[c] - Mx) * invZ : 0.f;
+              for (int q = 0; q < NPW; ++q) {
+                if (own[q]) {
                   uint32_t v[32];
-                  tc::tmem_ld32(tmem + lane_base + E_COL + eb * PMAX + c * KC + half * 32, v);
-                  tc::tmem_wait_ld();
-                  const float2 ff = make_float2(f, f);
-#pragma unroll
-                  for (int i = 0; i < 16; ++i) {
-                    const float2 r2 = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])),
-                                                 ff, make_float2(P[c][2 * i], P[c][2 * i + 1]));
-                    P[c][2 * i] = r2.x;
-                    P[c][2 * i + 1] = r2.y;
-                  }
+                  tc::tmem_ld32(pbase + 64 * q, v);
+                  ld_wait(v);
+                  p_accum(P[q], v, f[q]);
                 }
               }
             }
             tc::fence_before();
             __syncwarp();
-            if (lane == 0) tc::bar_arrive(&sm.efree[eb]);
+            if (lane == 0) tc::bar_arrive(&sm.efree[pb]);
             // the slot's phase for head hp is complete: arm it for head hp + NXS
-            if (armer) tc::bar_expect_tx(&sm.xbar[slot], Smem<C>::XBYTES);
+            if (armer) tc::bar_expect_tx(&sm.xbar[slot], G::XBYTES);
           }
         }
         if (ok && step < H) {
-          // ---- S1-key chunks of head `step` (E buffer), then the exchange
-          const int eb = hcur & 1;
+          // ---- S1-key pieces of head `step` (written back as exponentials), then the exchange
+          if (wvalid) {
+            const uint32_t ibase = ebase + half * 32;
+            int lim[NPW];
+            bool live[NPW];
 #pragma unroll
-          for (int c = 0; c < NIC_MAX; ++c) {
-            cmx[c] = -INFINITY;
-            if (ok && c < g.nic) {
-              if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.efull[eb][c], (hcur >> 1) & 1, nullptr, kLimitNs))) {
-                ok = false;
-              } else if (wvalid) {
-                const int lim = vrow ? min(KC, g.own_img - c * KC) - half * 32 : 0;
-                float a;
-                half_stats<true>(tmem + lane_base + E_COL + eb * PMAX + c * KC + half * 32, lim, sl2, cmx[c], a);
-                online_merge(m, z, cmx[c], a);
+            for (int q = 0; q < NPW; ++q) {
+              lim[q] = vrow ? g.own_img - (2 * q + half) * 32 : 0;
+              live[q] = own[q] && !__all_sync(0xffffffffu, lim[q] <= 0);
+              cmx[q] = -INFINITY;
+            }
+            float a;
+#pragma unroll
+            for (int q = 0; q < NPW; ++q) {
+              if (live[q]) {
+                uint32_t v[32];
+                tc::tmem_ld32(ibase + 64 * q, v);
+                ld_wait(v);
+                piece_stats<true>(v, ibase + 64 * q, lim[q], sl2, cmx[q], a);
+                online_merge(m, z, cmx[q], a);
               }
             }
-          }
-          if (wvalid) tc::tmem_wait_st();
-          tc::fence_before();
-          if (ok) {
-            // ---- post this head's (max, sum) to every epilogue warp of the cluster
-            const int slot = hcur & (NXS - 1);
+            tc::tmem_wait_st();
+          } else {
 #pragma unroll
-            for (int r = 0; r < C; ++r)
-              tc::st_async_f2(&sm.xch[slot][rank][half][j], &sm.xbar[slot], (uint32_t)r, m, z);
+            for (int q = 0; q < NPW; ++q) cmx[q] = -INFINITY;
           }
+          tc::fence_before();
+          // ---- post this head's (max, sum) to every epilogue warp of the cluster
+          const int slot = hcur & (NXS - 1);
+#pragma unroll
+          for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][half][j], &sm.xbar[slot], (uint32_t)r, m, z);
         }
       }
       hk += H;
@@ -518,17 +529,17 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       float regacc = 0.f;
       if (wvalid) {
 #pragma unroll
-        for (int c = 0; c < NIC_MAX; ++c) {
-          if (c < g.nic) {
+        for (int q = 0; q < NPW; ++q) {
+          if (own[q]) {
             // transpose-reduce over the 32 rows of this warp: afterwards lane l
             // holds the max (and, where a register key is among the columns,
-            // the sum) of this warp's column l of chunk c -- 31 shuffles each
-            const int key = c * KC + half * 32 + lane;
+            // the sum) of this warp's column l of piece q -- 31 shuffles each
+            const int key = (2 * q + half) * 32 + lane;
             const bool live = key < g.own_img;
             const bool is_reg = live && sm.kreg[ib][key];
             float t[32];
 #pragma unroll
-            for (int col = 0; col < 32; ++col) t[col] = vrow ? P[c][col] : 0.f;
+            for (int col = 0; col < 32; ++col) t[col] = vrow ? P[q][col] : 0.f;
 #pragma unroll
             for (int sft = 16; sft >= 1; sft >>= 1) {
               const bool up = (lane & sft) != 0;
@@ -543,7 +554,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             float rc = 0.f;
             if (__any_sync(0xffffffffu, is_reg)) {
 #pragma unroll
-              for (int col = 0; col < 32; ++col) t[col] = vrow ? P[c][col] : 0.f;
+              for (int col = 0; col < 32; ++col) t[col] = vrow ? P[q][col] : 0.f;
 #pragma unroll
               for (int sft = 16; sft >= 1; sft >>= 1) {
                 const bool up = (lane & sft) != 0;
@@ -603,8 +614,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   tc::cluster_sync_all();
 }
 
-int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt,
-                 const Stage2TcParams& q, int nclusters, cudaStream_t st) {
+int launch_fused(int C, const CUtensorMap& mq, const Stage2TcParams& q, int nclusters, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(nclusters * C));
   cfg.blockDim = dim3(s2f::THREADS);
@@ -628,10 +638,10 @@ int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUte
   cudaError_t e;
   if (C == 8) {
     cudaFuncSetAttribute(s2_fused_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(8));
-    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<8>, mq, mk, mkt, q);
+    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<8>, mq, q);
   } else {
     cudaFuncSetAttribute(s2_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(4));
-    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<4>, mq, mk, mkt, q);
+    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<4>, mq, q);
   }
   return e == cudaSuccess ? 0 : 1;
 }
