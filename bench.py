@@ -366,8 +366,10 @@ def run_ours(args, rank, world, local):
         "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {
-            "workload": WORKLOAD, "B": meta["B"], "crops": meta["segs_per_sample"], "visual_per_crop": 576,
-            "registers_per_crop": meta["regs_per_seg"], "text_tokens": "16..256 (uniform)",
+            "workload": WORKLOAD, "B": meta["B"], "crops": meta["segs_per_sample"],
+            "visual_per_crop": (w.vis[1] if w.vis[0] == "fixed" else f"{w.vis[1]}..{w.vis[2]} (step {w.vis[3]})"),
+            "registers_per_crop": meta["regs_per_seg"],
+            "text_tokens": (str(w.M[1]) if w.M[0] == "fixed" else f"{w.M[1]}..{w.M[2]} (uniform)"),
             "H1xd1": f"{meta['H1']}x{meta['d1']}", "H2xd2": f"{meta['H2']}x{meta['d2']}", "hidden": meta["hidden"],
             "lambda1": w.lambda1, "lambda2": w.lambda2, "accumulate": "fp32",
             "parallelism": "replicas" if world > 1 else "single",
@@ -384,7 +386,10 @@ def run_ours(args, rank, world, local):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 8 * args.steps,
+        # kernels per occam_prune call: Stage I (1 [CLS] / 2 mutual), finalize,
+        # plan, fused Stage II with 4- and 8-CTA clusters, the two-pass Stage-II
+        # pair, scan, gather
+        "gpu_launches": (9 if w.stage1 == "cls" else 10) * args.steps,
         "clocks": clocks,
     }
     if world > 1:
