@@ -148,6 +148,30 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
+// A second stream (and fork / join events) per host thread and device, made
+// on first use and kept for the life of the thread; per-thread so that calls
+// from different host threads never share an event.
+struct SideStream {
+  cudaStream_t stream = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+  bool ok = false;
+};
+
+SideStream& side_stream() {
+  constexpr int kMaxDevices = 64;
+  thread_local SideStream per_dev[kMaxDevices];
+  static SideStream bad;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return bad;
+  SideStream& s = per_dev[dev];
+  if (!s.ok) {
+    s.ok = cudaStreamCreateWithFlags(&s.stream, cudaStreamNonBlocking) == cudaSuccess &&
+           cudaEventCreateWithFlags(&s.fork, cudaEventDisableTiming) == cudaSuccess &&
+           cudaEventCreateWithFlags(&s.join, cudaEventDisableTiming) == cudaSuccess;
+  }
+  return s;
+}
+
 // 2-D bf16 map over a [rows, cols] row-major tensor, 128-byte swizzle, box
 // of 64 columns x box_rows rows.
 bool encode_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, uint32_t box_rows) {
@@ -363,11 +387,24 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     q.tau2 = p.tau2;
     q.lambda2 = lambda2;
     q.status = p.status;
+    // The 8-CTA launch runs beside the 4-CTA one on a second stream (fork and
+    // join by events), so SMs one of them leaves idle serve the other. Both
+    // launch a cluster per SM group; clusters take items from a queue, so
+    // clusters that become resident late simply find less work.
+    SideStream& side = side_stream();
+    if (!side.ok) return OCCAM_ERR_CUDA;
+    OCCAM_CUDA(cudaEventRecord(side.fork, st));
+    OCCAM_CUDA(cudaStreamWaitEvent(side.stream, side.fork, 0));
+    Stage2TcParams q8 = q;
+    q8.items = p.itemsF8;
+    q8.queue = p.counters + CNT_QUEUE8;
+    const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
+    if (launch_fused(8, mq, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
+    q.queue = p.counters + CNT_QUEUE4;
     const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
     if (launch_fused(4, mq, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
-    q.items = p.itemsF8;
-    const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
-    if (launch_fused(8, mq, q, ncl8, st) != 0) return OCCAM_ERR_CUDA;
+    OCCAM_CUDA(cudaEventRecord(side.join, side.stream));
+    OCCAM_CUDA(cudaStreamWaitEvent(st, side.join, 0));
   }
   trace.mark(st);
   const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);

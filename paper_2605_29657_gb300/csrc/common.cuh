@@ -185,7 +185,17 @@ struct WsLayout {
 };
 
 // counters block (int32 slots)
-enum { CNT_DENSE_DONE = 0, CNT_SCAN_TICKET = 1, CNT_NA = 2, CNT_NB = 3, CNT_NF = 4, CNT_NF8 = 5, CNT_SLOTS = 6 };
+enum {
+  CNT_DENSE_DONE = 0,
+  CNT_SCAN_TICKET = 1,
+  CNT_NA = 2,
+  CNT_NB = 3,
+  CNT_NF = 4,
+  CNT_NF8 = 5,
+  CNT_QUEUE4 = 6,  // next fused Stage-II item (4-CTA clusters)
+  CNT_QUEUE8 = 7,  // next fused Stage-II item (8-CTA clusters)
+  CNT_SLOTS = 8
+};
 
 constexpr int kTextTile = 64;    // Stage-II text rows per item
 constexpr int kHeadGroup = 8;    // Stage-II heads per stats item

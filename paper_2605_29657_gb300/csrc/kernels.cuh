@@ -16,11 +16,12 @@ constexpr int kFusedEpiWarps = 8;       // epilogue warps per CTA of the fused k
 // Whether a sample with n1 S1 keys and M text tokens fits the fused kernel
 // with C CTAs per cluster: each CTA takes ceil(n1 / C) S1 keys (padded to 32)
 // and, for the last text tile, ceil(M / C) causal text keys (padded to 16).
-__host__ __device__ inline bool fused_fits(int C, int n1, int M) {
+// The kernel's item hand-off assumes at least 4 heads per item.
+__host__ __device__ inline bool fused_fits(int C, int n1, int M, int H) {
   const int rows = C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;
   const int ip = ((n1 + C - 1) / C + 31) & ~31;
   const int tp = ((M + C - 1) / C + 15) & ~15;
-  return M > 0 && ip <= kFusedMaxOwnImg && ip + tp <= rows;
+  return M > 0 && H >= 4 && ip <= kFusedMaxOwnImg && ip + tp <= rows;
 }
 constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedEpiWarps;  // s2(r) partials per C=4 item (one per epilogue warp)
 constexpr int kFusedSlotsPerItem8 = 8 * kFusedEpiWarps;             // and per C=8 item
@@ -153,6 +154,7 @@ struct Stage2TcParams {
   const uint8_t* role;
   const int4* items;
   const int32_t* counters;
+  int32_t* queue;  // item queue head, zero before the launch
   float* s2;
   float* refpart;
   const int32_t* slot_off;

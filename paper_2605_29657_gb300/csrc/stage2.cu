@@ -63,8 +63,8 @@ __global__ void __launch_bounds__(256) s2_dense_plan_kernel(Stage2Params p, int 
       const int n1 = *((volatile int32_t*)&p.n1[bb]);
       // the fused tensor-core kernel takes a sample when its S1 keys and its
       // causal text keys fit the cluster's TMEM / shared memory
-      const bool fused4 = p.use_fused && fused_fits(kFusedCluster, n1, M);
-      const bool fused8 = !fused4 && p.use_fused && fused_fits(8, n1, M);
+      const bool fused4 = p.use_fused && fused_fits(kFusedCluster, n1, M, p.H);
+      const bool fused8 = !fused4 && p.use_fused && fused_fits(8, n1, M, p.H);
       if (fused4) {
         tiles128 = (M + 127) / 128;
         nF = tiles128;

@@ -78,7 +78,9 @@ struct Smem {
   float2 xch[NXS][C][2][QR];  // (max, sum) per (slot, CTA, epilogue half, row)
   int32_t kidx[2][PMAX];
   uint8_t kreg[2][PMAX];
-  uint64_t kfull[2], kempty[2], qfull[2], qempty[2], efull[2], efree[2], xbar[NXS], iready[2], idone[2], mdone;
+  int32_t next_item[4];  // work item of the cluster's ii-th turn, by ii & 3
+  uint64_t kfull[2], kempty[2], qfull[2], qempty[2], efull[2], efree[2], xbar[NXS], iready[2], idone[2], inext[4],
+      mdone;
   uint32_t tmem_base;
   int abort;
   uint32_t issued_q;
@@ -129,6 +131,28 @@ template <class SM>
 __device__ __forceinline__ void fail(SM& sm, int* status) {
   sm.abort = 1;
   set_status(status, OCCAM_ERR_TIMEOUT);
+}
+
+// Rank 0 of the cluster takes the next work item from the queue and hands it
+// to every CTA of the cluster (the value, then a release arrival on the
+// CTA's inext barrier). Dynamic hand-out keeps the clusters busy although
+// items differ in cost and not every launched cluster is resident at once.
+template <int C, class SM>
+__device__ __forceinline__ void hand_out_item(SM& sm, int32_t* queue, int ii) {
+  const int idx = atomicAdd(queue, 1);
+#pragma unroll
+  for (int r = 0; r < C; ++r) tc::st_cluster_u32(&sm.next_item[ii & 3], (uint32_t)r, (uint32_t)idx);
+#pragma unroll
+  for (int r = 0; r < C; ++r) tc::bar_arrive_remote(&sm.inext[ii & 3], (uint32_t)r);
+}
+
+// The cluster's ii-th work item (a queue position; >= the item count ends
+// the loop). False if the hand-out did not arrive in time.
+template <class SM>
+__device__ __forceinline__ bool take_item(SM& sm, int ii, volatile int* abort, int& item) {
+  if (!tc::bar_wait(&sm.inext[ii & 3], (ii >> 2) & 1, abort, s2f::kLimitNs, true)) return false;
+  item = *reinterpret_cast<volatile int32_t*>(&sm.next_item[ii & 3]);
+  return true;
 }
 
 __device__ __forceinline__ float warp_sum_f(float v) {
@@ -237,7 +261,6 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rank = (int)tc::cluster_rank();
   const int nF = p.counters[C == 8 ? CNT_NF8 : CNT_NF];
-  const int cid = (int)tc::cluster_id_x(), ncl = (int)tc::nclusters_x();
   volatile int* abort = &sm.abort;
 
   if (tid == 0) {
@@ -254,6 +277,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     // one local arrival (with the expected byte count) plus the peers'
     // asynchronous stores complete each phase of an exchange slot
     for (int i = 0; i < NXS; ++i) tc::bar_init(&sm.xbar[i], 1);
+    for (int i = 0; i < 4; ++i) tc::bar_init(&sm.inext[i], 1);
     tc::bar_init(&sm.mdone, 1);
     sm.abort = 0;
     sm.issued_q = 0;
@@ -282,7 +306,11 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       uint32_t qcnt = 0, kcnt = 0;
       int ii = 0;
       const int64_t HD = (int64_t)H * 128;
-      for (int item = cid; item < nF; item += ncl, ++ii) {
+      for (;; ++ii) {
+        if (rank == 0 && pt == 0) hand_out_item<C>(sm, p.queue, ii);
+        int item;
+        if (!take_item(sm, ii, abort, item)) { fail(sm, p.status); break; }
+        if (item >= nF) break;
         const ItemGeom g = item_geom<C>(p, p.items[item], rank);
         if (!g.fits) continue;
         const int ib = ii & 1;
@@ -342,7 +370,10 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       // ---------------------------------------------------------- MMA issuer
       if (lane == 0) {
         uint32_t qcnt = 0, kcnt = 0, hk = 0;
-        for (int item = cid; item < nF && !*abort; item += ncl) {
+        for (int ii = 0; !*abort; ++ii) {
+          int item;
+          if (!take_item(sm, ii, abort, item)) { fail(sm, p.status); break; }
+          if (item >= nF) break;
           const ItemGeom g = item_geom<C>(p, p.items[item], rank);
           if (!g.fits) continue;
           const uint32_t idesc = tc::idesc_bf16(128, g.N > 0 ? g.N : 16);
@@ -394,8 +425,10 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     const float invH = 1.0f / (float)H;
     const bool armer = ew == 0 && lane == 0;  // re-arms the exchange slots of this CTA
     uint32_t hk = 0;
-    int ii = 0;
-    for (int item = cid; item < nF; item += ncl, ++ii) {
+    for (int ii = 0;; ++ii) {
+      int item = 0;
+      if (!__all_sync(0xffffffffu, take_item(sm, ii, nullptr, item))) { fail(sm, p.status); break; }
+      if (item >= nF) break;
       const ItemGeom g = item_geom<C>(p, p.items[item], rank);
       if (!g.fits) {
         if (tid == EPI_WARP0 * 32) set_status(p.status, OCCAM_ERR_UNSUPPORTED);

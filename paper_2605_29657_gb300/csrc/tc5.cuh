@@ -256,6 +256,14 @@ __device__ __forceinline__ void st_async_f2(const void* local_addr, const uint64
       "r"(su32(bar)), "r"(rank), "f"(x), "f"(y)
       : "memory");
 }
+__device__ __forceinline__ void st_cluster_u32(const void* local_addr, uint32_t rank, uint32_t x) {
+  asm volatile(
+      "{\n\t.reg .b32 ra;\n\t"
+      "mapa.shared::cluster.u32 ra, %0, %1;\n\t"
+      "st.shared::cluster.u32 [ra], %2;\n\t}" ::"r"(su32(local_addr)),
+      "r"(rank), "r"(x)
+      : "memory");
+}
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
