@@ -206,6 +206,13 @@ typedef struct occam_prune_out {
   int32_t* n1_vis;
 } occam_prune_out;
 
+/* The whole path in one call (Algorithm 1's pruning steps): Stage-I scores,
+ * S1 (threshold lambda1 per segment), Stage-II scores over S1, S2
+ * (threshold lambda2 per sample), compaction and gather. Part of Stage II
+ * runs on a second stream that the library owns (one per host thread and
+ * device, created on first use), forked from and joined back to `stream` with
+ * events, so the call stays ordered on `stream` and can be captured into a
+ * CUDA graph. */
 int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                 size_t workspace_bytes, occam_stream_t stream);
 
@@ -216,8 +223,10 @@ int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* 
  * fused tensor-core Stage II, two-pass Stage II (statistics and scores
  * kernels, for the samples the fused kernel does not take), compaction scan,
  * gather. Mutual scoring and the two-pass Stage II are two kernels each,
- * timed together. Extra events are left unrecorded; missing ones are
- * skipped. Results are identical to occam_prune. */
+ * timed together. When the fused kernel is enabled the two-pass kernels run
+ * on a second stream beside it, so the fused interval covers all of Stage II
+ * and the two-pass interval is empty. Extra events are left unrecorded;
+ * missing ones are skipped. Results are identical to occam_prune. */
 int occam_prune_traced(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                        size_t workspace_bytes, occam_stream_t stream, void* const* events, int32_t n_events);
 

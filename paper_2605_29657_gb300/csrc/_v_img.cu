@@ -1,0 +1,697 @@
+// stage2_tc.cu -- fused Stage-II scoring on the 5th-generation tensor cores
+// (tcgen05 + TMEM), for samples whose S1 fits a 4- or 8-CTA cluster.
+//
+// What it computes (Sec. 3.5, Eq. 7; App. A, Eqs. 15-16): for sample b, text
+// token j and head h, A_{j,h} = softmax over {S1 rows of b} u {text keys 0..j}
+// of q_{j,h} k^T / sqrt(d2); P[j, v] = sum_h A_{j,h}(v); s2(v) = max_j P[j, v] / H
+// for visual S1 rows and the registers' sum_j P[j, r] / H for s2(r).
+//
+// Work item = (sample, tile of 128 text rows), processed by one cluster of C
+// CTAs (C = 4, or 8 for samples with more S1 keys). The text rows are the 128
+// TMEM lanes; each CTA owns 1/C of the sample's S1 keys and of the causal
+// text keys. Per head, a CTA's keys form one block of N <= 256 rows: its S1
+// keys (padded to a multiple of 32), then its text keys (padded to 16).
+//   1. seven producer warps gather the block's rows with 16-byte cp.async
+//      into the 128-byte-swizzled operand layout (S1 rows straight from K2 by
+//      index: pruned rows are never read); the head's 128 x 128 query tile
+//      arrives by TMA. Key blocks and query tiles are double-buffered by head;
+//   2. one thread issues S = Q K^T for the whole block as eight
+//      128 x N x 16 tcgen05.mma (bf16 in, fp32 accumulate) into a per-head
+//      TMEM buffer E (two buffers, alternating by head);
+//   3. eight epilogue warps (two per TMEM lane quadrant, one thread per text
+//      row) each own every other 32-column piece of E. A warp turns its
+//      logits into exp2(l - cmax) (cmax: the row max of that piece, kept in a
+//      register), writes the S1-key ones back over the logits in E, and keeps
+//      the row's running softmax max / sum;
+//   4. the (max, sum) pairs go to every epilogue warp of the cluster with
+//      asynchronous distributed-shared-memory stores that complete on an
+//      mbarrier of the receiving CTA (no fences);
+//   5. every warp then adds exp2(cmax - max) / sum * E over its S1-key
+//      pieces to the head-summed probabilities P, which live in registers for
+//      the whole item.
+// Step s of the epilogue takes the text-key statistics of head s, adds head
+// s-1 into P (freeing head s-1's E buffer, so the MMAs of head s+1 overlap
+// the rest of step s), then the S1-key statistics of head s, and posts them.
+// After the last head every warp reduces its P columns over its 32 rows:
+// column max -> s2 (atomicMax on the fp32 bit pattern, exact and order-free
+// since P >= 0), register columns -> a partial of s2(r) reduced in fixed order.
+#include "common.cuh"
+#include "kernels.cuh"
+#include "tc5.cuh"
+
+namespace occam {
+
+namespace s2f {
+constexpr int QR = 128;                // text rows per item (TMEM lanes)
+constexpr int PMAX = kFusedMaxOwnImg;  // max S1 keys per CTA
+constexpr int NPW = PMAX / 64;         // S1-key pieces per epilogue warp
+constexpr int QBYTES = QR * 256;       // one head's query tile: 2 K-blocks x 128 rows x 128 B
+constexpr int NPROD = 7;               // producer warps (0-6); warp 7 issues MMAs; then the epilogue warps
+constexpr int MMA_WARP = NPROD;
+constexpr int EPI_WARP0 = NPROD + 1;
+constexpr int NEPI = kFusedEpiWarps;   // two per TMEM lane quadrant
+constexpr int THREADS = (NPROD + 1 + NEPI) * 32;
+constexpr int NXS = 2;                 // exchange slots (a peer runs at most one head ahead of a slot's reader)
+// register split: warpgroups 0-1 (producers + MMA issuer) shrink to REG_LOW
+// per thread, the two epilogue warpgroups grow to REG_HIGH; the sum must stay
+// within what the CTA was launched with (checked on the host before launch)
+constexpr int REG_LOW = 56, REG_HIGH = 200;
+constexpr int REG_NEEDED = EPI_WARP0 * 32 * REG_LOW + NEPI * 32 * REG_HIGH;
+static_assert(EPI_WARP0 % 4 == 0 && NEPI % 4 == 0, "roles split on warpgroup boundaries");
+constexpr uint32_t TMEM_COLS = 512;
+static_assert(2 * kFusedKeyRows4 <= (int)TMEM_COLS && 2 * kFusedKeyRows8 <= (int)TMEM_COLS, "two E buffers");
+static_assert(kFusedKeyRows4 % 32 == 0 && kFusedKeyRows8 % 32 == 0 && kFusedKeyRows4 <= 256, "MMA N <= 256");
+static_assert(PMAX % 64 == 0, "S1-key pieces split evenly between the two warps of a quadrant");
+constexpr uint64_t kLimitNs = 2000000000ull;
+
+template <int C>
+struct Geo {
+  static constexpr int KROWS = C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;  // key rows per head (max MMA N)
+  static constexpr int KBLK = KROWS * 128;                                  // bytes of one K-block of the key rows
+  static constexpr uint32_t XBYTES = C * NEPI * 32 * 8;                     // exchange bytes a CTA receives per head
+};
+
+template <int C>
+struct Smem {
+  uint8_t q[2][QBYTES];
+  uint8_t k[2][2 * Geo<C>::KBLK];
+  float2 xch[NXS][C][2][QR];  // (max, sum) per (slot, CTA, epilogue half, row)
+  int32_t kidx[2][PMAX];
+  uint8_t kreg[2][PMAX];
+  int32_t next_item[4];  // work item of the cluster's ii-th turn, by ii & 3
+  uint64_t kfull[2], kempty[2], qfull[2], qempty[2], efull[2], efree[2], xbar[NXS], iready[2], idone[2], inext[4],
+      mdone;
+  uint32_t tmem_base;
+  int abort;
+  uint32_t issued_q;
+};
+}  // namespace s2f
+
+int s2_fused_smem_bytes(int C) {
+  return (int)(C == 8 ? sizeof(s2f::Smem<8>) : sizeof(s2f::Smem<4>)) + 1024;
+}
+int s2_fused_threads() { return s2f::THREADS; }
+
+namespace {
+
+struct ItemGeom {
+  int b, j0, M, n, img0, own_img, txt0, own_txt, ip, tp, N, slot;
+  bool fits;
+  int64_t rbase, t0;
+};
+
+template <int C>
+__device__ __forceinline__ ItemGeom item_geom(const Stage2TcParams& p, int4 it, int rank) {
+  using namespace s2f;
+  ItemGeom g;
+  g.b = it.x;
+  g.j0 = it.y;
+  g.slot = it.z;
+  g.rbase = p.bt.row_off[g.b];
+  g.t0 = p.bt.text_off[g.b];
+  g.M = (int)(p.bt.text_off[g.b + 1] - g.t0);
+  g.n = p.n1[g.b];
+  const int per = (g.n + C - 1) / C;
+  g.img0 = rank * per;
+  g.own_img = max(0, min(per, g.n - g.img0));
+  const int n_txt = p.has_text ? min(g.j0 + QR, g.M) : 0;
+  const int per_t = (n_txt + C - 1) / C;
+  g.txt0 = rank * per_t;
+  g.own_txt = max(0, min(per_t, n_txt - g.txt0));
+  g.ip = (g.own_img + 31) & ~31;
+  g.tp = (g.own_txt + 15) & ~15;
+  g.N = g.ip + g.tp;
+  // the same on every CTA of the cluster (depends on the sample only)
+  const int ipmax = (per + 31) & ~31;
+  g.fits = ipmax <= PMAX && ipmax + ((per_t + 15) & ~15) <= Geo<C>::KROWS;
+  return g;
+}
+
+template <class SM>
+__device__ __forceinline__ void fail(SM& sm, int* status) {
+  sm.abort = 1;
+  set_status(status, OCCAM_ERR_TIMEOUT);
+}
+
+// Rank 0 of the cluster takes the next work item from the queue and hands it
+// to every CTA of the cluster (the value, then a release arrival on the
+// CTA's inext barrier). Dynamic hand-out keeps the clusters busy although
+// items differ in cost and not every launched cluster is resident at once.
+template <int C, class SM>
+__device__ __forceinline__ void hand_out_item(SM& sm, int32_t* queue, int ii) {
+  const int idx = atomicAdd(queue, 1);
+#pragma unroll
+  for (int r = 0; r < C; ++r) tc::st_cluster_u32(&sm.next_item[ii & 3], (uint32_t)r, (uint32_t)idx);
+#pragma unroll
+  for (int r = 0; r < C; ++r) tc::bar_arrive_remote(&sm.inext[ii & 3], (uint32_t)r);
+}
+
+// The cluster's ii-th work item (a queue position; >= the item count ends
+// the loop). False if the hand-out did not arrive in time.
+template <class SM>
+__device__ __forceinline__ bool take_item(SM& sm, int ii, volatile int* abort, int& item) {
+  if (!tc::bar_wait(&sm.inext[ii & 3], (ii >> 2) & 1, abort, s2f::kLimitNs, true)) return false;
+  item = *reinterpret_cast<volatile int32_t*>(&sm.next_item[ii & 3]);
+  return true;
+}
+
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Ties the 32 registers a tcgen05.ld wrote to the preceding wait::ld, so the
+// compiler cannot move their first use above it.
+__device__ __forceinline__ void reg_fence(uint32_t (&v)[32]) {
+  asm volatile(""
+               : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
+                 "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]), "+r"(v[12]), "+r"(v[13]), "+r"(v[14]), "+r"(v[15]),
+                 "+r"(v[16]), "+r"(v[17]), "+r"(v[18]), "+r"(v[19]), "+r"(v[20]), "+r"(v[21]), "+r"(v[22]), "+r"(v[23]),
+                 "+r"(v[24]), "+r"(v[25]), "+r"(v[26]), "+r"(v[27]), "+r"(v[28]), "+r"(v[29]), "+r"(v[30]), "+r"(v[31]));
+}
+
+__device__ __forceinline__ void ld_wait(uint32_t (&v)[32]) {
+  tc::tmem_wait_ld();
+  reg_fence(v);
+}
+
+// Statistics of one thread's row over a 32-column piece of logits already
+// loaded into v (warp-collective): cm = max of the first `lim` columns in
+// log2 units (-inf if none), a = sum over them of exp2(l * sl2 - cm). v is
+// overwritten with the exponentials (0 past lim); with STORE they are also
+// written back to TMEM at sa (the caller waits for that store before the
+// values are read again).
+template <bool STORE>
+__device__ __forceinline__ void piece_stats(uint32_t (&v)[32], uint32_t sa, int lim, float sl2, float& cm, float& a) {
+  if (__all_sync(0xffffffffu, lim >= 32)) {
+    float t[11];
+#pragma unroll
+    for (int i = 0; i < 10; ++i)
+      t[i] = tc::fmax3(__uint_as_float(v[3 * i]), __uint_as_float(v[3 * i + 1]), __uint_as_float(v[3 * i + 2]));
+    t[10] = fmaxf(__uint_as_float(v[30]), __uint_as_float(v[31]));
+    const float mx = fmaxf(tc::fmax3(tc::fmax3(t[0], t[1], t[2]), tc::fmax3(t[3], t[4], t[5]), tc::fmax3(t[6], t[7], t[8])),
+                           fmaxf(t[9], t[10]));
+    cm = mx * sl2;
+    const float2 sc = make_float2(sl2, sl2), off = make_float2(-cm, -cm);
+    float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), sc, off);
+      x.x = tc::ex2(x.x);
+      x.y = tc::ex2(x.y);
+      acc[i & 3] = __fadd2_rn(acc[i & 3], x);
+      v[2 * i] = __float_as_uint(x.x);
+      v[2 * i + 1] = __float_as_uint(x.y);
+    }
+    a = ((acc[0].x + acc[0].y) + (acc[1].x + acc[1].y)) + ((acc[2].x + acc[2].y) + (acc[3].x + acc[3].y));
+  } else {
+    float c0 = -INFINITY, c1 = -INFINITY;
+#pragma unroll
+    for (int col = 0; col < 32; col += 2) {
+      if (col < lim) c0 = fmaxf(c0, __uint_as_float(v[col]));
+      if (col + 1 < lim) c1 = fmaxf(c1, __uint_as_float(v[col + 1]));
+    }
+    cm = fmaxf(c0, c1) * sl2;
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int col = 0; col < 32; col += 2) {
+      const float e0 = (col < lim) ? tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -cm)) : 0.f;
+      const float e1 = (col + 1 < lim) ? tc::ex2(fmaf(__uint_as_float(v[col + 1]), sl2, -cm)) : 0.f;
+      a0 += e0;
+      a1 += e1;
+      v[col] = __float_as_uint(e0);
+      v[col + 1] = __float_as_uint(e1);
+    }
+    a = a0 + a1;
+  }
+  if (STORE) tc::tmem_st32(sa, v);
+}
+
+// merges a piece's (cm, a) into the row's running softmax (m, z), log2 units
+__device__ __forceinline__ void online_merge(float& m, float& z, float cm, float a) {
+  if (cm != -INFINITY) {
+    const float mn = fmaxf(m, cm);
+    z = (m == -INFINITY ? 0.f : z * tc::ex2(m - mn)) + a * tc::ex2(cm - mn);
+    m = mn;
+  }
+}
+
+// P[col] += f * v[col] over one 32-column piece
+__device__ __forceinline__ void p_accum(float (&P)[32], const uint32_t (&v)[32], float f) {
+  const float2 ff = make_float2(f, f);
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const float2 r2 = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), ff,
+                                 make_float2(P[2 * i], P[2 * i + 1]));
+    P[2 * i] = r2.x;
+    P[2 * i + 1] = r2.y;
+  }
+}
+
+}  // namespace
+
+template <int C>
+__global__ void __launch_bounds__(s2f::THREADS, 1)
+    s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, Stage2TcParams p) {
+  using namespace s2f;
+  using G = Geo<C>;
+  extern __shared__ unsigned char smem_raw[];
+  Smem<C>& sm = *reinterpret_cast<Smem<C>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rank = (int)tc::cluster_rank();
+  const int nF = p.counters[C == 8 ? CNT_NF8 : CNT_NF];
+  volatile int* abort = &sm.abort;
+
+  if (tid == 0) {
+    for (int i = 0; i < 2; ++i) {
+      tc::bar_init(&sm.kfull[i], NPROD * 32);
+      tc::bar_init(&sm.kempty[i], 1);
+      tc::bar_init(&sm.qfull[i], 1);
+      tc::bar_init(&sm.qempty[i], 1);
+      tc::bar_init(&sm.efull[i], 1);
+      tc::bar_init(&sm.efree[i], NEPI);
+      tc::bar_init(&sm.iready[i], NPROD * 32);
+      tc::bar_init(&sm.idone[i], NEPI);
+    }
+    // one local arrival (with the expected byte count) plus the peers'
+    // asynchronous stores complete each phase of an exchange slot
+    for (int i = 0; i < NXS; ++i) tc::bar_init(&sm.xbar[i], 1);
+    for (int i = 0; i < 4; ++i) tc::bar_init(&sm.inext[i], 1);
+    tc::bar_init(&sm.mdone, 1);
+    sm.abort = 0;
+    sm.issued_q = 0;
+    tc::bar_fence_init();
+    for (int i = 0; i < NXS; ++i) tc::bar_expect_tx(&sm.xbar[i], G::XBYTES);
+    tc::prefetch_map(&mapQ);
+  }
+  if (warp == MMA_WARP) tc::tmem_alloc(&sm.tmem_base, TMEM_COLS);
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  // peers' barriers must be initialised before anyone stores into them remotely
+  tc::cluster_sync_all();
+  const uint32_t tmem = sm.tmem_base;
+  const int H = p.H;
+
+  if (warp < EPI_WARP0) {
+    // warpgroups 0-1: producers and the MMA issuer give registers back
+    tc::setmaxnreg_dec<REG_LOW>();
+    if (warp < NPROD) {
+      // ---------------------------------------------------------- producers
+      // NPROD * 32 threads; piece q (16 bytes) of the key block is row (q >> 4), head
+      // slice bytes 16 * (q & 15); it lands at the row's 128-byte line of its
+      // K-block with the 16-byte chunk index XOR (row & 7).
+      const int pt = tid;
+      uint32_t qcnt = 0, kcnt = 0;
+      int ii = 0;
+      const int64_t HD = (int64_t)H * 128;
+      for (;; ++ii) {
+        if (rank == 0 && pt == 0) hand_out_item<C>(sm, p.queue, ii);
+        int item;
+        if (!take_item(sm, ii, abort, item)) { fail(sm, p.status); break; }
+        if (item >= nF) break;
+        const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+        if (!g.fits) continue;
+        const int ib = ii & 1;
+        if (*abort || !tc::bar_wait(&sm.idone[ib], ((ii >> 1) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
+        for (int i = pt; i < g.own_img; i += NPROD * 32) {
+          const int row = p.dense[g.rbase + g.img0 + i];
+          sm.kidx[ib][i] = row;
+          sm.kreg[ib][i] = p.role[row];
+        }
+        tc::bar_arrive(&sm.iready[ib]);
+        if (!tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
+        const int64_t tbase = g.t0 + g.txt0;
+        bool ok = true;
+        for (int h = 0; h < H && ok; ++h) {
+          const int kb = kcnt & 1;
+          if (!tc::bar_wait(&sm.kempty[kb], ((kcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
+            fail(sm, p.status);
+            ok = false;
+            break;
+          }
+          if (pt == 0) {
+            const int qb = qcnt & 1;
+            if (!tc::bar_wait(&sm.qempty[qb], ((qcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
+              fail(sm, p.status);
+              ok = false;
+            } else {
+              tc::bar_expect_tx(&sm.qfull[qb], QBYTES);
+              tc::tma_load_2d(sm.q[qb], &mapQ, h * 128, (int)(g.t0 + g.j0), &sm.qfull[qb]);
+              tc::tma_load_2d(sm.q[qb] + QBYTES / 2, &mapQ, h * 128 + 64, (int)(g.t0 + g.j0), &sm.qfull[qb]);
+            }
+          }
+          ++qcnt;
+          uint8_t* dst = sm.k[kb];
+          const int nq = g.N * 16;
+          for (int q = pt; q < nq; q += NPROD * 32) {
+            const int row = q >> 4, c16 = q & 15;
+            const int kblk = c16 >> 3, cc = c16 & 7;
+            const __nv_bfloat16* src = p.K;
+            int bytes = 0;
+            if (row < g.own_img) {
+              src = p.K + (int64_t)sm.kidx[ib][row] * HD + h * 128 + c16 * 8;
+              bytes = 16;
+            } else if (row >= g.ip && row - g.ip < g.own_txt) {
+              src = p.Kt + (tbase + (row - g.ip)) * HD + h * 128 + c16 * 8;
+              bytes = 16;
+            }
+            tc::cp_async16(dst + kblk * G::KBLK + row * 128 + ((cc ^ (row & 7)) << 4), src, bytes);
+          }
+          tc::cp_async_arrive(&sm.kfull[kb]);
+          ++kcnt;
+        }
+        if (!ok) break;
+      }
+      if (pt == 0) sm.issued_q = qcnt;
+      asm volatile("cp.async.wait_all;" ::: "memory");
+    } else {
+      // ---------------------------------------------------------- MMA issuer
+      if (lane == 0) {
+        uint32_t qcnt = 0, kcnt = 0, hk = 0;
+        for (int ii = 0; !*abort; ++ii) {
+          int item;
+          if (!take_item(sm, ii, abort, item)) { fail(sm, p.status); break; }
+          if (item >= nF) break;
+          const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+          if (!g.fits) continue;
+          const uint32_t idesc = tc::idesc_bf16(128, g.N > 0 ? g.N : 16);
+          bool ok = true;
+          for (int h = 0; h < H && ok; ++h, ++hk) {
+            const int qb = qcnt & 1, kb = kcnt & 1, eb = hk & 1;
+            // E[eb] is free once head hk - 2 was read out of it
+            ok = tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs);
+            if (ok && hk >= 2) ok = tc::bar_wait(&sm.efree[eb], ((hk - 2) >> 1) & 1, abort, kLimitNs);
+            if (ok) ok = tc::bar_wait(&sm.kfull[kb], (kcnt >> 1) & 1, abort, kLimitNs);
+            if (!ok) {
+              fail(sm, p.status);
+              break;
+            }
+            tc::fence_proxy_async();
+            tc::fence_after();
+            if (g.N > 0) {
+              const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[kb]);
+#pragma unroll
+              for (int s = 0; s < 8; ++s) {
+                const int kblk = s >> 2, kk = s & 3;
+                tc::mma_bf16(tmem + eb * G::KROWS, tc::sdesc_sw128(qa + kblk * (QBYTES / 2) + kk * 32),
+                             tc::sdesc_sw128(kbase + kblk * G::KBLK + kk * 32), idesc, s > 0 ? 1u : 0u);
+              }
+            }
+            tc::mma_commit(&sm.efull[eb]);
+            tc::mma_commit(&sm.kempty[kb]);
+            tc::mma_commit(&sm.qempty[qb]);
+            ++qcnt;
+            ++kcnt;
+          }
+        }
+        // every MMA issued by this thread has completed once this barrier flips
+        tc::mma_commit(&sm.mdone);
+        if (!tc::bar_wait(&sm.mdone, 0, nullptr, kLimitNs)) set_status(p.status, OCCAM_ERR_TIMEOUT);
+      }
+      __syncwarp();
+    }
+  } else {
+    // warpgroups 2-3: the epilogue takes them
+    tc::setmaxnreg_inc<REG_HIGH>();
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - EPI_WARP0;    // 0..NEPI-1
+    const int half = ew >> 2;           // this warp owns the 32-column pieces of this parity
+    const int quad = warp & 3;          // TMEM lane quadrant this warp may access
+    const int j = quad * 32 + lane;     // text row of this thread inside the tile
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    const float sl2 = p.scale_log2;
+    const float invH = 1.0f / (float)H;
+    const bool armer = ew == 0 && lane == 0;  // re-arms the exchange slots of this CTA
+    uint32_t hk = 0;
+    for (int ii = 0;; ++ii) {
+      int item = 0;
+      if (!__all_sync(0xffffffffu, take_item(sm, ii, nullptr, item))) { fail(sm, p.status); break; }
+      if (item >= nF) break;
+      const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+      if (!g.fits) {
+        if (tid == EPI_WARP0 * 32) set_status(p.status, OCCAM_ERR_UNSUPPORTED);
+        continue;
+      }
+      const int ib = ii & 1;
+      if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, nullptr, kLimitNs))) { fail(sm, p.status); break; }
+      const bool vrow = g.j0 + j < g.M;
+      const bool wvalid = __any_sync(0xffffffffu, vrow);  // warp-uniform: any real text row here
+      const int jj = g.j0 + j;
+      const int npi = g.ip >> 5;                // S1-key pieces of this CTA
+      const int npc = (g.N + 31) >> 5;          // all pieces
+      bool own[NPW];                            // which of this warp's S1-key pieces exist
+#pragma unroll
+      for (int q = 0; q < NPW; ++q) own[q] = 2 * q + half < npi;
+      float P[NPW][32];
+#pragma unroll
+      for (int q = 0; q < NPW; ++q)
+#pragma unroll
+        for (int b2 = 0; b2 < 32; ++b2) P[q][b2] = 0.f;
+      float cmx[NPW];  // piece maxima of the last head whose statistics were taken
+#pragma unroll
+      for (int q = 0; q < NPW; ++q) cmx[q] = -INFINITY;
+      bool ok = true;
+      for (int step = 0; step <= H && ok; ++step) {
+        const uint32_t hcur = hk + step;  // global index of head `step` of this item
+        const int eb = hcur & 1;
+        const uint32_t ebase = tmem + lane_base + eb * G::KROWS;
+        float m = -INFINITY, z = 0.f;
+        if (step < H) {
+          // ---- text-key pieces of head `step`
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.efull[eb], (hcur >> 1) & 1, nullptr, kLimitNs))) {
+            ok = false;
+          } else if (wvalid) {
+            tc::fence_after();
+            for (int pc = npi + ((npi ^ half) & 1); pc < npc; pc += 2) {
+              const int tb = g.txt0 + pc * 32 - g.ip;  // sample-relative text index of the piece's column 0
+              const int lim = vrow ? min(g.own_txt - (pc * 32 - g.ip), jj - tb + 1) : 0;
+              if (__all_sync(0xffffffffu, lim <= 0)) continue;
+              uint32_t v[32];
+              tc::tmem_ld32(ebase + pc * 32, v);
+              ld_wait(v);
+              float cm, a;
+              piece_stats<false>(v, 0, lim, sl2, cm, a);
+              online_merge(m, z, cm, a);
+            }
+          }
+        }
+        if (ok && step >= 1) {
+          // ---- probabilities of head step-1 over this warp's S1-key pieces, added into P
+          const uint32_t hp = hcur - 1;
+          const int slot = hp & (NXS - 1);
+          const int pb = hp & 1;
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (hp / NXS) & 1, nullptr, kLimitNs, true))) {
+            ok = false;
+          } else {
+            if (wvalid) {
+              float Mx = -INFINITY;
+#pragma unroll
+              for (int r = 0; r < C; ++r) Mx = tc::fmax3(Mx, sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x);
+              float Z = 0.f;
+#pragma unroll
+              for (int r = 0; r < C; ++r)
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                  const float2 e = sm.xch[slot][r][hh][j];
+                  if (e.y > 0.f) Z += e.y * tc::ex2(e.x - Mx);
+                }
+              const float invZ = (vrow && Z > 0.f) ? 1.0f / Z : 0.f;
+              float f[NPW];
+#pragma unroll
+              for (int q = 0; q < NPW; ++q) f[q] = (invZ > 0.f && cmx[q] != -INFINITY) ? tc::ex2(cmx[q] - Mx) * invZ : 0.f;
+              const uint32_t pbase = tmem + lane_base + pb * G::KROWS + half * 32;
+              tc::fence_after();
+#pragma unroll
+              for (int q = 0; q < NPW; ++q) {
+                if (own[q]) {
+                  uint32_t v[32];
+                  tc::tmem_ld32(pbase + 64 * q, v);
+                  ld_wait(v);
+                  p_accum(P[q], v, f[q]);
+                }
+              }
+            }
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) tc::bar_arrive(&sm.efree[pb]);
+            // the slot's phase for head hp is complete: arm it for head hp + NXS
+            if (armer) tc::bar_expect_tx(&sm.xbar[slot], G::XBYTES);
+          }
+        }
+        if (ok && step < H) {
+          // ---- S1-key pieces of head `step` (written back as exponentials), then the exchange
+          if (wvalid) {
+            const uint32_t ibase = ebase + half * 32;
+            int lim[NPW];
+            bool live[NPW];
+#pragma unroll
+            for (int q = 0; q < NPW; ++q) {
+              lim[q] = vrow ? g.own_img - (2 * q + half) * 32 : 0;
+              live[q] = own[q] && !__all_sync(0xffffffffu, lim[q] <= 0);
+              cmx[q] = -INFINITY;
+            }
+            float a;
+            // software-pipelined: the next piece's TMEM load is in flight
+            // while this piece is processed
+            uint32_t va[32], vb[32];
+            if (live[0]) tc::tmem_ld32(ibase, va);
+            if (live[0]) {
+              ld_wait(va);
+              if (live[1]) tc::tmem_ld32(ibase + 64, vb);
+              piece_stats<true>(va, ibase, lim[0], sl2, cmx[0], a);
+              online_merge(m, z, cmx[0], a);
+            } else if (live[1]) {
+              tc::tmem_ld32(ibase + 64, vb);
+            }
+            if (live[1]) {
+              ld_wait(vb);
+              if (live[2]) tc::tmem_ld32(ibase + 128, va);
+              piece_stats<true>(vb, ibase + 64, lim[1], sl2, cmx[1], a);
+              online_merge(m, z, cmx[1], a);
+            } else if (live[2]) {
+              tc::tmem_ld32(ibase + 128, va);
+            }
+            if (live[2]) {
+              ld_wait(va);
+              piece_stats<true>(va, ibase + 128, lim[2], sl2, cmx[2], a);
+              online_merge(m, z, cmx[2], a);
+            }
+            tc::tmem_wait_st();
+          } else {
+#pragma unroll
+            for (int q = 0; q < NPW; ++q) cmx[q] = -INFINITY;
+          }
+          tc::fence_before();
+          // ---- post this head's (max, sum) to every epilogue warp of the cluster
+          const int slot = hcur & (NXS - 1);
+#pragma unroll
+          for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][half][j], &sm.xbar[slot], (uint32_t)r, m, z);
+        }
+      }
+      hk += H;
+      if (!ok) { fail(sm, p.status); break; }
+      // ---- column reductions of P over this warp's 32 rows: column max ->
+      // s2 (atomicMax), register columns -> this warp's partial of s2(r)
+      float regacc = 0.f;
+      if (wvalid) {
+#pragma unroll
+        for (int q = 0; q < NPW; ++q) {
+          if (own[q]) {
+            // transpose-reduce over the 32 rows of this warp: afterwards lane l
+            // holds the max (and, where a register key is among the columns,
+            // the sum) of this warp's column l of piece q -- 31 shuffles each
+            const int key = (2 * q + half) * 32 + lane;
+            const bool live = key < g.own_img;
+            const bool is_reg = live && sm.kreg[ib][key];
+            float t[32];
+#pragma unroll
+            for (int col = 0; col < 32; ++col) t[col] = vrow ? P[q][col] : 0.f;
+#pragma unroll
+            for (int sft = 16; sft >= 1; sft >>= 1) {
+              const bool up = (lane & sft) != 0;
+#pragma unroll
+              for (int i = 0; i < sft; ++i) {
+                const float send = up ? t[i] : t[i + sft];
+                const float keep = up ? t[i + sft] : t[i];
+                t[i] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, sft));
+              }
+            }
+            if (live && !is_reg) atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(t[0] * invH));
+            float rc = 0.f;
+            if (__any_sync(0xffffffffu, is_reg)) {
+#pragma unroll
+              for (int col = 0; col < 32; ++col) t[col] = vrow ? P[q][col] : 0.f;
+#pragma unroll
+              for (int sft = 16; sft >= 1; sft >>= 1) {
+                const bool up = (lane & sft) != 0;
+#pragma unroll
+                for (int i = 0; i < sft; ++i) {
+                  const float send = up ? t[i] : t[i + sft];
+                  const float keep = up ? t[i + sft] : t[i];
+                  t[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+                }
+              }
+              if (is_reg) rc = t[0] * invH;
+            }
+            regacc += warp_sum_f(rc);
+          }
+        }
+      }
+      if (lane == 0) {
+        p.refpart[g.slot + rank * NEPI + ew] = regacc;  // C * NEPI slots per item
+        __threadfence();
+        const int nslots = p.slot_off[g.b + 1] - p.slot_off[g.b];
+        if (atomicAdd(&p.done[g.b], 1) == nslots - 1) {
+          __threadfence();
+          float acc = 0.f;
+          for (int i = p.slot_off[g.b]; i < p.slot_off[g.b + 1]; ++i) acc += *((volatile float*)&p.refpart[i]);
+          const int R = p.bt.reg_off[p.bt.seg_first[g.b + 1]] - p.bt.reg_off[p.bt.seg_first[g.b]];
+          const float r2 = (R > 0 && g.M > 0) ? acc / ((float)R * (float)g.M) : 0.f;
+          p.ref2[g.b] = r2;
+          p.tau2[g.b] = p.lambda2 * r2;
+        }
+      }
+      __syncwarp();
+      if (lane == 0) tc::bar_arrive(&sm.idone[ib]);
+    }
+  }
+
+  // ------------------------------------------------------------ teardown
+  tc::fence_before();
+  __syncthreads();
+  if (sm.abort && tid == 0) {
+    // drain the last query-tile copies (TMA) issued into each buffer; the
+    // producers' cp.async copies were drained by cp.async.wait_all
+    const uint32_t q1 = sm.issued_q;
+    for (uint32_t i = (q1 > 2 ? q1 - 2 : 0); i < q1; ++i)
+      tc::bar_wait(&sm.qfull[i & 1], (i >> 1) & 1, nullptr, kLimitNs / 8);
+  }
+  __syncthreads();
+  tc::fence_after();
+  if (warp == MMA_WARP) tc::tmem_dealloc(tmem, TMEM_COLS);
+  if (sm.abort && tid == 0) {
+    // after an abort, peers' asynchronous exchange stores may still be in
+    // flight towards this CTA: give them time to land before it can exit
+    const uint64_t t0 = tc::globaltimer();
+    while (tc::globaltimer() - t0 < 100000ull) {
+    }
+  }
+  // peers may still write into this CTA's exchange buffers until here
+  tc::cluster_sync_all();
+}
+
+int launch_fused(int C, const CUtensorMap& mq, const Stage2TcParams& q, int nclusters, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(nclusters * C));
+  cfg.blockDim = dim3(s2f::THREADS);
+  cfg.dynamicSmemBytes = s2_fused_smem_bytes(C);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // the register split inside the kernel needs the launch to reserve at least
+  // REG_NEEDED registers per CTA; refuse rather than launch a kernel whose
+  // setmaxnreg.inc could never be satisfied
+  cudaFuncAttributes fa;
+  if ((C == 8 ? cudaFuncGetAttributes(&fa, s2_fused_kernel<8>) : cudaFuncGetAttributes(&fa, s2_fused_kernel<4>)) !=
+      cudaSuccess)
+    return 1;
+  if (fa.numRegs * s2f::THREADS < s2f::REG_NEEDED) return 2;
+  cudaError_t e;
+  if (C == 8) {
+    cudaFuncSetAttribute(s2_fused_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(8));
+    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<8>, mq, q);
+  } else {
+    cudaFuncSetAttribute(s2_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(4));
+    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<4>, mq, q);
+  }
+  return e == cudaSuccess ? 0 : 1;
+}
+
+}  // namespace occam

@@ -123,11 +123,17 @@ int num_sms() {
   return n;
 }
 
+size_t finalize_smem_bytes(int rows, bool cls) {
+  return ((size_t)rows * ((cls ? 64 : 0) + 4 + 1) + 15) & ~(size_t)15;
+}
+
 void set_smem_attrs() {
   static std::once_flag once;
   std::call_once(once, [] {
-    cudaFuncSetAttribute(stage1_cls_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         stage1_cls_smem_bytes());
+    cudaFuncSetAttribute(stage1_logits_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         stage1_logits_smem_bytes());
+    cudaFuncSetAttribute(stage1_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)finalize_smem_bytes(16 * kFinalizeSmemRows, false));
     cudaFuncSetAttribute(s2_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_stats_smem_bytes());
     cudaFuncSetAttribute(s2_scores_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_scores_smem_bytes());
   });
@@ -215,7 +221,6 @@ int check_stage1(const occam_batch* b, const occam_stage1_args* a) {
   if (!aligned16(a->q) || !aligned16(a->K1) || (a->k_cls && !aligned16(a->k_cls))) return OCCAM_ERR_INVALID_ARG;
   if (a->mode == OCCAM_STAGE1_CLS) {
     if (a->H1 != 16 || a->d1 != 64) return OCCAM_ERR_UNSUPPORTED;
-    if (b->max_seg_rows > kMaxClusterCls * kMaxClsRowsPerCta) return OCCAM_ERR_UNSUPPORTED;
   } else if (a->mode == OCCAM_STAGE1_MUTUAL) {
     if (a->H1 < 1 || a->H1 > 64) return OCCAM_ERR_UNSUPPORTED;
     if (a->d1 != 64 && a->d1 != 72 && a->d1 != 80) return OCCAM_ERR_UNSUPPORTED;
@@ -262,31 +267,17 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
   const BatchDev bt = dev_batch(b);
   int* status = at<int>(ws, L.status);
   if (a->mode == OCCAM_STAGE1_CLS) {
+    // per-head logits only; the finalize kernel forms s1 from them
     Stage1ClsParams p;
     p.bt = bt;
     p.q_cls = static_cast<const __nv_bfloat16*>(a->q);
-    p.k_cls = static_cast<const __nv_bfloat16*>(a->k_cls);
     p.K1 = static_cast<const __nv_bfloat16*>(a->K1);
     p.scale = (float)(1.0 / std::sqrt((double)a->d1));
-    p.s1 = s1;
-    p.s2_zero = s2_zero;
+    p.logits = at<float>(ws, L.stats1);
     p.status = status;
-    int C = (int)cdiv(b->max_seg_rows, 160);
-    C = C < 1 ? 1 : (C > kMaxClusterCls ? kMaxClusterCls : C);
-    while (cdiv(b->max_seg_rows, C) > kMaxClsRowsPerCta && C < kMaxClusterCls) ++C;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(b->S_tot * C));
-    cfg.blockDim = dim3(256);
-    cfg.dynamicSmemBytes = stage1_cls_smem_bytes();
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = C;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    OCCAM_CUDA(cudaLaunchKernelEx(&cfg, stage1_cls_kernel, p));
+    const int64_t tiles = cdiv(b->total_rows, 16);
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(tiles, 2 * num_sms()));
+    stage1_logits_kernel<<<grid, 256, stage1_logits_smem_bytes(), st>>>(p);
     trace.mark(st);
   } else {
     MutualParams p;
@@ -304,11 +295,23 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
   return cuda_ok();
 }
 
-int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, const float* s1, const uint8_t* keep_in,
+// a1 (nullable): in [CLS] mode s1 is formed here from the logits of
+// launch_stage1_scores and written to s1; s2_zero (nullable) is zeroed.
+int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s1, const uint8_t* keep_in,
                      float lambda1, int do_threshold, float* ref1, uint8_t* keep1, int32_t* n1_vis,
-                     cudaStream_t st, Trace trace = Trace()) {
+                     const occam_stage1_args* a1, float* s2_zero, cudaStream_t st, Trace trace = Trace()) {
   Stage1FinalizeParams p;
   p.bt = dev_batch(b);
+  const bool cls = a1 && a1->mode == OCCAM_STAGE1_CLS;
+  p.logits = cls ? at<float>(ws, L.stats1) : nullptr;
+  p.q_cls = cls ? static_cast<const __nv_bfloat16*>(a1->q) : nullptr;
+  p.k_cls = cls ? static_cast<const __nv_bfloat16*>(a1->k_cls) : nullptr;
+  p.scale = cls ? (float)(1.0 / std::sqrt((double)a1->d1)) : 1.f;
+  p.s1_out = s1;
+  p.s2_zero = cls ? s2_zero : nullptr;
+  // a segment's logits ([CLS] mode, 64 B/row), s1 (4 B/row) and roles
+  // (1 B/row) are staged in shared memory when it fits (at most 96 KB)
+  p.smem_rows = s1 ? (int)std::min<int64_t>(b->max_seg_rows, cls ? kFinalizeSmemRows : 16 * kFinalizeSmemRows) : 0;
   p.s1 = s1;
   p.keep_in = keep_in;
   p.lambda1 = lambda1;
@@ -320,9 +323,18 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, const fl
   p.n1_seg = at<int32_t>(ws, L.n1_seg);
   p.n1_vis = n1_vis;
   p.status = at<int>(ws, L.status);
-  stage1_finalize_kernel<<<b->S_tot, 256, 0, st>>>(p);
+  stage1_finalize_kernel<<<b->S_tot, 256, finalize_smem_bytes(p.smem_rows, cls), st>>>(p);
   trace.mark(st);
   return cuda_ok();
+}
+
+// Stage II for the samples the plan routed to the two-pass kernels; both
+// loop over their item lists, which may be empty.
+void launch_twopass(const Stage2Params& p, const WsLayout& L, int sms, cudaStream_t st) {
+  const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);
+  const int gB = (int)std::min<int64_t>(L.maxB, sms);
+  if (gA > 0) s2_stats_kernel<<<gA, 128, s2_stats_smem_bytes(), st>>>(p);
+  if (gB > 0) s2_scores_kernel<<<gB, 256, s2_scores_smem_bytes(), st>>>(p);
 }
 
 int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayout& L, void* ws, float* s2,
@@ -400,17 +412,19 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     q8.queue = p.counters + CNT_QUEUE8;
     const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
     if (launch_fused(8, mq, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
+    // the two-pass kernels (samples the fused kernel cannot hold; often none)
+    // follow the 8-CTA launch on the second stream
+    launch_twopass(p, L, sms, side.stream);
     q.queue = p.counters + CNT_QUEUE4;
     const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
     if (launch_fused(4, mq, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
     OCCAM_CUDA(cudaEventRecord(side.join, side.stream));
     OCCAM_CUDA(cudaStreamWaitEvent(st, side.join, 0));
+    trace.mark(st);
+  } else {
+    trace.mark(st);
+    launch_twopass(p, L, sms, st);
   }
-  trace.mark(st);
-  const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);
-  const int gB = (int)std::min<int64_t>(L.maxB, sms);
-  if (gA > 0) s2_stats_kernel<<<gA, 128, s2_stats_smem_bytes(), st>>>(p);
-  if (gB > 0) s2_scores_kernel<<<gB, 256, s2_scores_smem_bytes(), st>>>(p);
   trace.mark(st);
   return cuda_ok();
 }
@@ -506,7 +520,7 @@ int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   set_smem_attrs();
   OCCAM_TRY(launch_stage1_scores(batch, args, L, workspace, s1, nullptr, st));
-  OCCAM_TRY(launch_finalize1(batch, L, workspace, s1, nullptr, 0.f, 0, ref1, nullptr, nullptr, st));
+  OCCAM_TRY(launch_finalize1(batch, L, workspace, s1, nullptr, 0.f, 0, ref1, nullptr, nullptr, args, nullptr, st));
   return OCCAM_OK;
 }
 
@@ -554,6 +568,13 @@ int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, 
   // S1 lists from the given mask (registers always in S1)
   Stage1FinalizeParams f;
   f.bt = dev_batch(batch);
+  f.logits = nullptr;
+  f.q_cls = nullptr;
+  f.k_cls = nullptr;
+  f.scale = 1.f;
+  f.s1_out = nullptr;
+  f.s2_zero = nullptr;
+  f.smem_rows = 0;
   f.s1 = nullptr;
   f.keep_in = keep1;
   f.lambda1 = 0.f;
@@ -616,7 +637,8 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   OCCAM_CUDA(cudaMemsetAsync(out->count_vis, 0, b->B * 4, st));
   trace.mark(st);
   OCCAM_TRY(launch_stage1_scores(b, &args->stage1, L, ws, s1, s2, st, trace));
-  OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, st, trace));
+  OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, &args->stage1, s2,
+                             st, trace));
   OCCAM_TRY(launch_stage2(b, &args->stage2, L, ws, s2, ref2, args->lambda2, st, trace));
   return launch_compact(b, L, ws, 1, nullptr, keep1, s2, args->keep_registers, out->keep2, args->n_tensors,
                         args->src, args->row_bytes, args->dst, args->capacity_rows, out->out_index,

@@ -12,6 +12,7 @@ constexpr int kFusedMaxOwnImg = 192;    // S1 keys one of its CTAs can hold (P c
 constexpr int kFusedKeyRows4 = 256;     // key rows per head one CTA of a 4-CTA cluster holds (= MMA N and TMEM columns)
 constexpr int kFusedKeyRows8 = 224;     // the same for an 8-CTA cluster (its exchange buffers take more shared memory)
 constexpr int kFusedEpiWarps = 8;       // epilogue warps per CTA of the fused kernel
+constexpr int kFinalizeSmemRows = 1400; // Stage-I finalize stages a [CLS] segment in shared memory up to this many rows
 
 // Whether a sample with n1 S1 keys and M text tokens fits the fused kernel
 // with C CTAs per cluster: each CTA takes ceil(n1 / C) S1 keys (padded to 32)
@@ -25,22 +26,27 @@ __host__ __device__ inline bool fused_fits(int C, int n1, int M, int H) {
 }
 constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedEpiWarps;  // s2(r) partials per C=4 item (one per epilogue warp)
 constexpr int kFusedSlotsPerItem8 = 8 * kFusedEpiWarps;             // and per C=8 item
-constexpr int kMaxClsRowsPerCta = 512;  // rows of one segment handled by one CTA of a [CLS] cluster
-constexpr int kMaxClusterCls = 8;       // portable cluster size
 
 struct Stage1ClsParams {
   BatchDev bt;
   const __nv_bfloat16* q_cls;
-  const __nv_bfloat16* k_cls;  // nullable
   const __nv_bfloat16* K1;
   float scale;
-  float* s1;
-  float* s2_zero;  // nullable: zeroed per row (Stage-II max accumulator)
+  float* logits;  // [rows, 16] per-head [CLS] logits
   int* status;
 };
 
 struct Stage1FinalizeParams {
   BatchDev bt;
+  // [CLS] mode: the segment's s1 is first formed from the per-head logits
+  // (softmax over the segment's rows and the [CLS] self key, head mean)
+  const float* logits;            // nullable: s1 is given instead
+  const __nv_bfloat16* q_cls;     // [CLS] mode
+  const __nv_bfloat16* k_cls;     // nullable
+  float scale;
+  float* s1_out;                  // [CLS] mode: where s1 is written
+  float* s2_zero;                 // nullable: zeroed per row (Stage-II max accumulator)
+  int smem_rows;                  // segments up to this many rows stage their logits in shared memory
   const float* s1;          // nullable when keep_in is given
   const uint8_t* keep_in;   // nullable: S1 membership of visual rows given instead of tested
   float lambda1;
@@ -166,8 +172,8 @@ struct Stage2TcParams {
 };
 
 // stage1.cu
-__global__ void stage1_cls_kernel(Stage1ClsParams p);
-int stage1_cls_smem_bytes();
+__global__ void stage1_logits_kernel(Stage1ClsParams p);
+int stage1_logits_smem_bytes();
 __global__ void stage1_finalize_kernel(Stage1FinalizeParams p);
 int mutual_colsum_smem_bytes(int DP);
 void launch_mutual(const MutualParams& p, int d1, int S_tot, int max_seg_rows, cudaStream_t st);

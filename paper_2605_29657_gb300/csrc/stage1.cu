@@ -2,25 +2,19 @@
 // scores of every visual and register row, the register reference of each
 // segment, and the image-adaptive threshold S1 = {v : s1(v) >= lambda1 s1(r)} u {r}
 // (Eqs. 4-6; App. A, Eqs. 10-13).
-#include <cooperative_groups.h>
-
 #include "common.cuh"
 #include "kernels.cuh"
-
-namespace cg = cooperative_groups;
 
 namespace occam {
 
 // ============================================================================
-// [CLS] scoring: one thread-block cluster per segment.
-//
-// The segment's K1 rows are contiguous in HBM (rows x H x D bf16). Each CTA of
-// the cluster streams its share of them through a ring of shared-memory
-// stages filled by 1-D bulk (TMA) copies, computes the H per-head logits of
-// every row against the segment's [CLS] query, and keeps them in shared
-// memory. The per-head softmax max / sum are combined across the cluster
-// through distributed shared memory, after which every CTA writes the
-// head-averaged probability s1 of its rows. HBM is read exactly once.
+// [CLS] logits (Sec. 3.4, Eq. 4): l[row][h] = q_cls[seg(row), h] . K1[row, h]
+// / sqrt(d1) for every visual and register row. The softmax over the
+// segment's rows and the head mean are taken by stage1_finalize_kernel from
+// these logits (64 bytes per row), so this kernel is a plain stream over K1:
+// persistent CTAs each take a contiguous range of 16-row tiles and pull them
+// through a ring of shared-memory stages filled by 1-D bulk (TMA) copies.
+// HBM is read exactly once.
 // ============================================================================
 namespace cls {
 constexpr int H = 16, D = 64;
@@ -28,85 +22,74 @@ constexpr int kThreads = 256;
 constexpr int kRowBytes = H * D * 2;            // 2048
 constexpr int kTileRows = 16;                   // rows per stage
 constexpr int kStageBytes = kTileRows * kRowBytes;
-constexpr int kStages = 2;
-constexpr int kLS = H + 1;                      // padded logit row stride (bank spread)
-constexpr int kSmem = kStages * kStageBytes + kMaxClsRowsPerCta * kLS * 4 + 1024;
+constexpr int kStages = 3;
+constexpr int kSmem = kStages * kStageBytes + 64;
 }  // namespace cls
 
-__global__ void __launch_bounds__(cls::kThreads) stage1_cls_kernel(Stage1ClsParams p) {
+__global__ void __launch_bounds__(cls::kThreads) stage1_logits_kernel(Stage1ClsParams p) {
   using namespace cls;
-  cg::cluster_group cluster = cg::this_cluster();
-  const int rank = (int)cluster.block_rank();
-  const int C = (int)cluster.num_blocks();
-  const int seg = blockIdx.x / C;
+  extern __shared__ __align__(128) unsigned char smem[];
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-
-  extern __shared__ __align__(1024) unsigned char smem[];
-  unsigned char* stage = smem;
-  float* logits = reinterpret_cast<float*>(smem + kStages * kStageBytes);
-  float* misc = logits + kMaxClsRowsPerCta * kLS;        // 1024 B
-  uint64_t* bar = reinterpret_cast<uint64_t*>(misc);     // kStages barriers
-  float2* stat = reinterpret_cast<float2*>(misc + 16);   // [H] local (max, sum)
-  float* gmax = misc + 16 + 2 * H;                       // [H]
-  float* ginv = gmax + H;                                // [H]
-  float* lcls = ginv + H;                                // [H]
-
-  const int64_t sb = p.bt.seg_off[seg], se = p.bt.seg_off[seg + 1];
-  const int n = (int)(se - sb);
-  const int chunk = (n + C - 1) / C;
-  const int64_t r0 = sb + (int64_t)rank * chunk;
-  int nloc = (se - r0 < (int64_t)chunk) ? (int)(se - r0) : chunk;
-  if (nloc < 0) nloc = 0;
-  if (nloc > kMaxClsRowsPerCta) {  // host validation prevents this
-    if (tid == 0) set_status(p.status, OCCAM_ERR_UNSUPPORTED);
-    nloc = 0;
-  }
-  const int ntiles = (nloc + kTileRows - 1) / kTileRows;
-
-  // lane layout for the dot products: 8 lanes share one (row, head); lane
-  // k = lane & 7 owns dims [8k, 8k+8) of that head.
-  const int slot = warp * 4 + (lane >> 3);   // 0..31
-  const int my_h = slot & (H - 1);
-  const int my_rr = slot >> 4;               // 0..1: row parity inside a step
-  const int kv = lane & 7;
-  float q[8];
-  {
-    const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + my_h) * D + kv * 8;
-    uint4 raw = *reinterpret_cast<const uint4*>(qp);
-    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) { q[2 * i] = bf16_lo(w[i]); q[2 * i + 1] = bf16_hi(w[i]); }
-  }
+  const int64_t R = p.bt.total_rows;
+  const int64_t nt_all = (R + kTileRows - 1) / kTileRows;
+  const int64_t t0 = nt_all * blockIdx.x / gridDim.x;
+  const int ntiles = (int)(nt_all * (blockIdx.x + 1) / gridDim.x - t0);
+  const unsigned char* gsrc = reinterpret_cast<const unsigned char*>(p.K1);
 
   if (tid == 0) {
     for (int i = 0; i < kStages; ++i) mbar_init(&bar[i], 1);
     fence_mbar_init();
-  }
-  __syncthreads();
-  const unsigned char* gsrc = reinterpret_cast<const unsigned char*>(p.K1) + r0 * kRowBytes;
-  if (tid == 0) {
     for (int i = 0; i < kStages && i < ntiles; ++i) {
-      const int rows = min(kTileRows, nloc - i * kTileRows);
+      const int64_t r0 = (t0 + i) * kTileRows;
+      const int rows = (int)min((int64_t)kTileRows, R - r0);
       mbar_arrive_expect_tx(&bar[i], rows * kRowBytes);
-      bulk_g2s(stage + i * kStageBytes, gsrc + (int64_t)i * kStageBytes, rows * kRowBytes, &bar[i]);
+      bulk_g2s(smem + i * kStageBytes, gsrc + r0 * kRowBytes, rows * kRowBytes, &bar[i]);
     }
   }
+  __syncthreads();
+
+  // lane layout for the dot products: 8 lanes share one (row, head); lane
+  // k = lane & 7 owns dims [8k, 8k+8) of that head. The four (row, head)
+  // slots of a warp share one row, so segment changes are warp-uniform.
+  const int slot = warp * 4 + (lane >> 3);   // 0..31
+  const int my_h = slot & (H - 1);
+  const int my_rr = slot >> 4;               // 0..1: row parity inside a step
+  const int kv = lane & 7;
+  int64_t seg_lo = 0, seg_hi = 0;            // rows of the segment q belongs to
+  float q[8];
 
   bool timed_out = false;
-  int fail_it = 0;
-  int issued = min(kStages, ntiles);
-  for (int it = 0; it < ntiles; ++it) {
+  int it = 0;
+  for (; it < ntiles; ++it) {
     const int st = it % kStages;
-    if (!mbar_wait(&bar[st], (it / kStages) & 1, kSpinLimit)) { timed_out = true; }
-    if (__syncthreads_or(timed_out)) { timed_out = true; fail_it = it; break; }
-    const unsigned char* buf = stage + st * kStageBytes;
-    const int rows = min(kTileRows, nloc - it * kTileRows);
+    if (!mbar_wait(&bar[st], (it / kStages) & 1, kSpinLimit)) timed_out = true;
+    if (__syncthreads_or(timed_out)) {
+      timed_out = true;
+      break;
+    }
+    const unsigned char* buf = smem + st * kStageBytes;
+    const int64_t r0 = (t0 + it) * kTileRows;
+    const int rows = (int)min((int64_t)kTileRows, R - r0);
 #pragma unroll
     for (int step = 0; step < kTileRows / 2; ++step) {
       const int rr = step * 2 + my_rr;
+      const int64_t row = r0 + rr;
       float acc = 0.f;
       if (rr < rows) {
-        uint4 raw = *reinterpret_cast<const uint4*>(buf + rr * kRowBytes + my_h * D * 2 + kv * 16);
+        if (row >= seg_hi || row < seg_lo) {
+          const int sg = upper_interval(p.bt.seg_off, p.bt.S_tot, row);
+          seg_lo = p.bt.seg_off[sg];
+          seg_hi = p.bt.seg_off[sg + 1];
+          const uint4 raw = *reinterpret_cast<const uint4*>(p.q_cls + ((int64_t)sg * H + my_h) * D + kv * 8);
+          const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            q[2 * i] = bf16_lo(w[i]);
+            q[2 * i + 1] = bf16_hi(w[i]);
+          }
+        }
+        const uint4 raw = *reinterpret_cast<const uint4*>(buf + rr * kRowBytes + my_h * D * 2 + kv * 16);
         const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -117,84 +100,25 @@ __global__ void __launch_bounds__(cls::kThreads) stage1_cls_kernel(Stage1ClsPara
       acc += __shfl_xor_sync(0xffffffffu, acc, 1);
       acc += __shfl_xor_sync(0xffffffffu, acc, 2);
       acc += __shfl_xor_sync(0xffffffffu, acc, 4);
-      if (kv == 0 && rr < rows) logits[(it * kTileRows + rr) * kLS + my_h] = acc * p.scale;
+      if (kv == 0 && rr < rows) p.logits[row * H + my_h] = acc * p.scale;
     }
     __syncthreads();
-    if (tid == 0 && issued < ntiles) {
-      const int rows_n = min(kTileRows, nloc - issued * kTileRows);
+    if (tid == 0 && it + kStages < ntiles) {
+      const int64_t rn = (t0 + it + kStages) * kTileRows;
+      const int rows_n = (int)min((int64_t)kTileRows, R - rn);
       mbar_arrive_expect_tx(&bar[st], rows_n * kRowBytes);
-      bulk_g2s(stage + st * kStageBytes, gsrc + (int64_t)issued * kStageBytes, rows_n * kRowBytes,
-               &bar[st]);
-      ++issued;
+      bulk_g2s(smem + st * kStageBytes, gsrc + rn * kRowBytes, rows_n * kRowBytes, &bar[st]);
     }
   }
-  if (timed_out) {
-    // Record the failure and drain every copy still in flight (bounded) before
-    // the shared memory goes away.
-    if (tid == 0) {
-      set_status(p.status, OCCAM_ERR_TIMEOUT);
-      for (int it = fail_it; it < issued; ++it) mbar_wait(&bar[it % kStages], (it / kStages) & 1, kSpinLimit);
-    }
-    __syncthreads();
-    nloc = 0;
+  if (timed_out && tid == 0) {
+    // record the failure and drain every copy still in flight (bounded)
+    // before the shared memory goes away
+    set_status(p.status, OCCAM_ERR_TIMEOUT);
+    for (int j = it; j < ntiles && j < it + kStages; ++j) mbar_wait(&bar[j % kStages], (j / kStages) & 1, kSpinLimit);
   }
-
-  // [CLS] self key (rank 0 only): l_cls,h = q_h . k_cls,h * scale
-  if (tid < H) {
-    float l = -INFINITY;
-    if (rank == 0 && p.k_cls != nullptr) {
-      const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + tid) * D;
-      const __nv_bfloat16* kp = p.k_cls + ((int64_t)seg * H + tid) * D;
-      float acc = 0.f;
-      for (int d = 0; d < D; ++d) acc = fmaf(__bfloat162float(qp[d]), __bfloat162float(kp[d]), acc);
-      l = acc * p.scale;
-    }
-    lcls[tid] = l;
-  }
-  __syncthreads();
-
-  // local per-head (max, sum of exp): warp w owns heads 2w and 2w+1
-  {
-    const int h = warp * 2 + (lane >> 4);
-    const int sub = lane & 15;
-    float m = (sub == 0) ? lcls[h] : -INFINITY;
-    for (int r = sub; r < nloc; r += 16) m = fmaxf(m, logits[r * kLS + h]);
-#pragma unroll
-    for (int o = 8; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-    float z = 0.f;
-    if (m != -INFINITY) {
-      if (sub == 0 && lcls[h] != -INFINITY) z = expf(lcls[h] - m);
-      for (int r = sub; r < nloc; r += 16) z += expf(logits[r * kLS + h] - m);
-    }
-#pragma unroll
-    for (int o = 8; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
-    if (sub == 0) stat[h] = make_float2(m, z);
-  }
-  cluster.sync();
-  if (tid < H) {
-    float M = -INFINITY;
-    for (int r = 0; r < C; ++r) M = fmaxf(M, cluster.map_shared_rank(stat, r)[tid].x);
-    float Z = 0.f;
-    for (int r = 0; r < C; ++r) {
-      const float2 v = cluster.map_shared_rank(stat, r)[tid];
-      if (v.y > 0.f) Z += v.y * expf(v.x - M);
-    }
-    gmax[tid] = M;
-    ginv[tid] = 1.0f / Z;
-  }
-  __syncthreads();
-  const float invH = 1.0f / H;
-  for (int r = tid; r < nloc; r += kThreads) {
-    float s = 0.f;
-#pragma unroll
-    for (int h = 0; h < H; ++h) s += expf(logits[r * kLS + h] - gmax[h]) * ginv[h];
-    p.s1[r0 + r] = s * invH;
-    if (p.s2_zero) p.s2_zero[r0 + r] = 0.f;
-  }
-  cluster.sync();  // peers may still read `stat` through DSMEM until here
 }
 
-int stage1_cls_smem_bytes() { return cls::kSmem; }
+int stage1_logits_smem_bytes() { return cls::kSmem; }
 
 // ============================================================================
 // Stage-I finalize: per segment, the register reference ref1 = mean of s1
@@ -202,7 +126,77 @@ int stage1_cls_smem_bytes() { return cls::kSmem; }
 // mask (registers always in), the row roles, and the order-preserving list
 // of the segment's S1 rows. One CTA per segment.
 // ============================================================================
+// [CLS] mode (Sec. 3.4, Eq. 4; App. A, Eq. 10): per head h the softmax of the
+// [CLS] row over {k_cls} u rows(segment) from the logits, s1 = mean over
+// heads. lg: the segment's logits [n][16] (shared or global memory); s1 is
+// written to s1_out (global) and, when given, to s1_loc (shared).
+__device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, int seg, int64_t sb, int n,
+                                               const float* lg, float* s1_loc) {
+  constexpr int H = 16, D = 64;
+  __shared__ float red[16][17];
+  __shared__ float gmax[16], ginv[16], lcls_s[16];
+  const int tid = threadIdx.x;
+  if (tid < 256) {
+    // l_cls,h: 16 threads per head, 4 dims each
+    const int h = tid >> 4, sub = tid & 15;
+    float acc = 0.f;
+    if (p.k_cls) {
+      const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + h) * D + sub * 4;
+      const __nv_bfloat16* kp = p.k_cls + ((int64_t)seg * H + h) * D + sub * 4;
+#pragma unroll
+      for (int d = 0; d < 4; ++d) acc = fmaf(__bfloat162float(qp[d]), __bfloat162float(kp[d]), acc);
+    }
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (sub == 0) lcls_s[h] = p.k_cls ? acc * p.scale : -INFINITY;
+  }
+  // thread t takes head (t & 15) of rows (t >> 4) + 16 k: a warp reads 32
+  // consecutive floats per step
+  const int h = tid & 15, j = tid >> 4;
+  float m = -INFINITY;
+  for (int r = j; r < n; r += 16) m = fmaxf(m, lg[r * H + h]);
+  red[j][h] = m;
+  __syncthreads();
+  if (tid < 16) {
+    float mm = lcls_s[tid];
+    for (int k = 0; k < 16; ++k) mm = fmaxf(mm, red[k][tid]);
+    gmax[tid] = mm;
+  }
+  __syncthreads();
+  const float mh = gmax[h];
+  float z = 0.f;
+  for (int r = j; r < n; r += 16) z += expf(lg[r * H + h] - mh);
+  red[j][h] = z;
+  __syncthreads();
+  if (tid < 16) {
+    float zz = lcls_s[tid] != -INFINITY ? expf(lcls_s[tid] - gmax[tid]) : 0.f;
+    for (int k = 0; k < 16; ++k) zz += red[k][tid];
+    ginv[tid] = 1.0f / zz;
+  }
+  __syncthreads();
+  for (int r = tid; r < n; r += blockDim.x) {
+    const float4* lp = reinterpret_cast<const float4*>(lg + r * H);
+    float acc = 0.f;
+#pragma unroll
+    for (int k = 0; k < H / 4; ++k) {
+      const float4 l = lp[k];
+      acc += expf(l.x - gmax[4 * k]) * ginv[4 * k] + expf(l.y - gmax[4 * k + 1]) * ginv[4 * k + 1] +
+             expf(l.z - gmax[4 * k + 2]) * ginv[4 * k + 2] + expf(l.w - gmax[4 * k + 3]) * ginv[4 * k + 3];
+    }
+    const float v = acc * (1.0f / H);
+    p.s1_out[sb + r] = v;
+    if (s1_loc) s1_loc[r] = v;
+    if (p.s2_zero) p.s2_zero[sb + r] = 0.f;
+  }
+  __syncthreads();
+}
+
+// 256 threads, one CTA per segment. With n <= smem_rows the segment's
+// logits ([CLS] mode), s1 and roles are staged in shared memory (one
+// coalesced pass over global memory each way); larger segments work from
+// global memory.
 __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizeParams p) {
+  extern __shared__ float4 fin_smem[];
   __shared__ int tmp[40];
   __shared__ float sref;
   const int seg = blockIdx.x;
@@ -210,36 +204,78 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   const int64_t sb = p.bt.seg_off[seg], se = p.bt.seg_off[seg + 1];
   const int n = (int)(se - sb);
   const int ra = p.bt.reg_off[seg], rb = p.bt.reg_off[seg + 1];
-  if (tid == 0) {
-    float acc = 0.f;
-    if (p.s1)
-      for (int i = ra; i < rb; ++i) acc += p.s1[p.bt.reg_idx[i]];
-    sref = (rb > ra) ? acc / (float)(rb - ra) : 0.f;
-    if (rb <= ra) set_status(p.status, OCCAM_ERR_INVALID_ARG);
-    if (p.ref1) p.ref1[seg] = sref;
+  const bool staged = n <= p.smem_rows;
+  // shared layout for a staged segment: [logits (CLS mode)][s1][role]
+  float* lg_loc = reinterpret_cast<float*>(fin_smem);
+  float* s1_loc = lg_loc + (p.logits ? (size_t)p.smem_rows * 16 : 0);
+  uint8_t* role_loc = reinterpret_cast<uint8_t*>(s1_loc + p.smem_rows);
+
+  const float* s1g = p.logits ? p.s1_out : p.s1;  // the segment's s1 in global memory
+  if (p.logits) {
+    const float* lg = p.logits + sb * 16;
+    if (staged) {
+      const float4* src = reinterpret_cast<const float4*>(lg);
+      float4* dst = reinterpret_cast<float4*>(lg_loc);
+      for (int i = tid; i < n * 4; i += blockDim.x) dst[i] = src[i];
+      __syncthreads();
+      lg = lg_loc;
+    }
+    cls_softmax_s1(p, seg, sb, n, lg, staged ? s1_loc : nullptr);
+  } else if (staged) {
+    for (int r = tid; r < n; r += blockDim.x) s1_loc[r] = s1g[sb + r];
   }
   // role bytes: 0 visual, 1 register
-  for (int r = tid; r < n; r += blockDim.x) p.role[sb + r] = 0;
-  __syncthreads();
-  for (int i = ra + tid; i < rb; i += blockDim.x) p.role[p.bt.reg_idx[i]] = 1;
-  __syncthreads();
+  if (staged) {
+    for (int r = tid; r < n; r += blockDim.x) role_loc[r] = 0;
+    __syncthreads();
+    for (int i = ra + tid; i < rb; i += blockDim.x) role_loc[p.bt.reg_idx[i] - sb] = 1;
+    __syncthreads();
+    for (int r = tid; r < n; r += blockDim.x) p.role[sb + r] = role_loc[r];
+  } else {
+    for (int r = tid; r < n; r += blockDim.x) p.role[sb + r] = 0;
+    __syncthreads();
+    for (int i = ra + tid; i < rb; i += blockDim.x) p.role[p.bt.reg_idx[i]] = 1;
+    __syncthreads();
+  }
+  // ref1 = mean of s1 over the segment's registers (parallel loads, fixed-order sum)
+  {
+    float v = 0.f;
+    if (s1g) {
+      for (int i = ra + tid; i < rb; i += blockDim.x) {
+        const int64_t row = p.bt.reg_idx[i];
+        v += staged ? s1_loc[row - sb] : s1g[row];
+      }
+    }
+    v = warp_sum(v);
+    if ((tid & 31) == 0) tmp[tid >> 5] = __float_as_int(v);
+    __syncthreads();
+    if (tid == 0) {
+      float acc = 0.f;
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) acc += __int_as_float(tmp[w]);
+      sref = (rb > ra) ? acc / (float)(rb - ra) : 0.f;
+      if (rb <= ra) set_status(p.status, OCCAM_ERR_INVALID_ARG);
+      if (p.ref1) p.ref1[seg] = sref;
+    }
+    __syncthreads();
+  }
   if (!p.do_threshold) return;
   const float tau = p.lambda1 * sref;
+  const uint8_t* role = staged ? role_loc : p.role + sb;
   // each thread owns a contiguous run of rows so the list stays in row order
   const int per = (n + blockDim.x - 1) / blockDim.x;
   const int a = min(n, tid * per), z = min(n, a + per);
   int cnt = 0, cvis = 0;
   for (int r = a; r < z; ++r) {
-    const bool reg = p.role[sb + r] != 0;
-    const bool k = reg || (p.keep_in ? p.keep_in[sb + r] != 0 : p.s1[sb + r] >= tau);
+    const bool reg = role[r] != 0;
+    const bool k = reg || (p.keep_in ? p.keep_in[sb + r] != 0 : (staged ? s1_loc[r] : s1g[sb + r]) >= tau);
     cnt += k;
     cvis += (k && !reg);
   }
   int total;
   int pos = block_exclusive_scan(cnt, tmp, &total);
   for (int r = a; r < z; ++r) {
-    const bool reg = p.role[sb + r] != 0;
-    const bool k = reg || (p.keep_in ? p.keep_in[sb + r] != 0 : p.s1[sb + r] >= tau);
+    const bool reg = role[r] != 0;
+    const bool k = reg || (p.keep_in ? p.keep_in[sb + r] != 0 : (staged ? s1_loc[r] : s1g[sb + r]) >= tau);
     if (p.keep1) p.keep1[sb + r] = k ? 1 : 0;
     if (k) p.s1_list[sb + pos++] = (int32_t)(sb + r);
   }
