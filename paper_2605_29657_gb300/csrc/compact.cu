@@ -5,10 +5,12 @@
 // scan_kernel: single pass over the batch's row space in tiles of 2048 rows.
 //   Each tile computes its keep flags (given, or the fused Stage-II test
 //   keep1 && s2 >= tau2), a block-wide scan, and its global offset by a
-//   decoupled look-back over its predecessors' published aggregates. Tile ids
-//   come from an atomic ticket, so every predecessor has already started and
-//   publishes without waiting: the look-back always ends. Its spin is bounded
-//   all the same and reports OCCAM_ERR_TIMEOUT instead of hanging.
+//   decoupled look-back over its predecessors' published aggregates, one warp
+//   reading a window of 32 predecessors at a time. Tile ids come from an
+//   atomic ticket, so every predecessor has already started and publishes
+//   without waiting: the look-back always ends. Its spin is bounded all the
+//   same and reports OCCAM_ERR_TIMEOUT instead of hanging. The sample
+//   offsets are staged in shared memory for the per-row sample lookups.
 // gather_kernel: persistent grid; one warp copies one kept row of one tensor
 //   with 16-byte loads / stores (exact bit copy).
 #include <mutex>
@@ -33,13 +35,20 @@ __device__ __forceinline__ unsigned long long ld_acquire(const unsigned long lon
 }
 }  // namespace
 
+constexpr int kScanSmemSamples = 2048;  // samples whose offsets fit the scan's shared copy
+
 __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   constexpr int PER = kScanTile / 256;  // 8 rows per thread
   __shared__ int tmp[40];
   __shared__ long long s_prefix;
   __shared__ int s_tile;
+  __shared__ int64_t s_ro[kScanSmemSamples + 1];
   const int tid = threadIdx.x;
   if (tid == 0) s_tile = atomicAdd(p.ticket, 1);
+  const bool ro_smem = p.bt.B <= kScanSmemSamples;
+  if (ro_smem)
+    for (int b = tid; b <= p.bt.B; b += blockDim.x) s_ro[b] = p.bt.row_off[b];
+  const int64_t* row_off = ro_smem ? s_ro : p.bt.row_off;
   __syncthreads();
   const int64_t tile = s_tile;
   const int64_t R = p.bt.total_rows;
@@ -49,14 +58,14 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   int samp = -1;
   int64_t samp_end = 0;
   if (r_first < R) {
-    samp = upper_interval(p.bt.row_off, p.bt.B, r_first);
-    samp_end = p.bt.row_off[samp + 1];
+    samp = upper_interval(row_off, p.bt.B, r_first);
+    samp_end = row_off[samp + 1];
   }
 #pragma unroll
   for (int i = 0; i < PER; ++i) {
     const int64_t r = r_first + i;
     if (r >= R) break;
-    while (r >= samp_end) { ++samp; samp_end = p.bt.row_off[samp + 1]; }
+    while (r >= samp_end) { ++samp; samp_end = row_off[samp + 1]; }
     bool k, vis;
     if (p.mode == 0) {
       k = p.keep_in[r] != 0;
@@ -79,32 +88,45 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   int tile_total;
   const int pos = block_exclusive_scan(cnt, tmp, &tile_total);
 
-  if (tid == 0) {
+  if (tid < 32) {
+    // warp-wide look-back: lane l reads predecessor (hi - l); the window
+    // moves back by 32 until it holds an inclusive prefix (tile "-1" counts
+    // as an inclusive prefix of 0)
+    const int lane = tid;
     long long excl = 0;
     if (tile == 0) {
-      st_release(&p.tile_state[0], kFlagPre | (unsigned long long)tile_total);
+      if (lane == 0) st_release(&p.tile_state[0], kFlagPre | (unsigned long long)tile_total);
     } else {
-      st_release(&p.tile_state[tile], kFlagAgg | (unsigned long long)tile_total);
-      int64_t q = tile - 1;
+      if (lane == 0) st_release(&p.tile_state[tile], kFlagAgg | (unsigned long long)tile_total);
+      int64_t hi = tile - 1;
       bool timed_out = false;
-      while (q >= 0) {
-        unsigned long long v = 0;
-        uint32_t spins = 0;
-        while (true) {
-          v = ld_acquire(&p.tile_state[q]);
-          if (v & (kFlagAgg | kFlagPre)) break;
-          if (++spins > kSpinLimit) { timed_out = true; break; }
-          __nanosleep(64);
+      uint32_t spins = 0;
+      while (true) {
+        const int64_t q = hi - lane;
+        const unsigned long long v = q >= 0 ? ld_acquire(&p.tile_state[q]) : kFlagPre;
+        if (!__all_sync(0xffffffffu, (v & (kFlagAgg | kFlagPre)) != 0)) {
+          if (++spins > kSpinLimit) {
+            timed_out = true;
+            break;
+          }
+          __nanosleep(32);
+          continue;
         }
-        if (timed_out) break;
-        excl += (long long)(v & kValMask);
-        if (v & kFlagPre) break;
-        --q;
+        const unsigned pre = __ballot_sync(0xffffffffu, (v & kFlagPre) != 0);
+        const int first = pre ? __ffs(pre) - 1 : 32;  // nearest predecessor with an inclusive prefix
+        long long val = lane <= first ? (long long)(v & kValMask) : 0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) val += __shfl_xor_sync(0xffffffffu, val, o);
+        excl += val;
+        if (pre) break;
+        hi -= 32;
       }
-      if (timed_out) set_status(p.status, OCCAM_ERR_TIMEOUT);
-      st_release(&p.tile_state[tile], kFlagPre | (unsigned long long)(excl + tile_total));
+      if (lane == 0) {
+        if (timed_out) set_status(p.status, OCCAM_ERR_TIMEOUT);
+        st_release(&p.tile_state[tile], kFlagPre | (unsigned long long)(excl + tile_total));
+      }
     }
-    s_prefix = excl;
+    if (lane == 0) s_prefix = excl;
   }
   __syncthreads();
   const int64_t base = s_prefix + pos;
@@ -123,8 +145,8 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   }
   // per-sample counts: a thread's rows may span several samples
   {
-    int s = (r_first < R) ? upper_interval(p.bt.row_off, p.bt.B, r_first) : -1;
-    int64_t send = (s >= 0) ? p.bt.row_off[s + 1] : 0;
+    int s = (r_first < R) ? upper_interval(row_off, p.bt.B, r_first) : -1;
+    int64_t send = (s >= 0) ? row_off[s + 1] : 0;
     int ck = 0, cv = 0;
     for (int i = 0; i < PER; ++i) {
       const int64_t r = r_first + i;
@@ -134,7 +156,7 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
         if (cv && p.count_vis) atomicAdd(&p.count_vis[s], cv);
         ck = cv = 0;
         ++s;
-        send = p.bt.row_off[s + 1];
+        send = row_off[s + 1];
       }
       ck += (kmask >> i) & 1;
       cv += (vmask >> i) & 1;
@@ -149,9 +171,9 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
     const int64_t r_end = min(r_first + PER, R);
     // empty samples share their start row with the next one: visit every b
     // whose first row lies in [r_first, r_end)
-    int bb = lower_bound_off(p.bt.row_off, p.bt.B, r_first);
-    for (; bb < p.bt.B && p.bt.row_off[bb] < r_end; ++bb) {
-      const int before = __popc(kmask & ((1u << (int)(p.bt.row_off[bb] - r_first)) - 1u));
+    int bb = lower_bound_off(row_off, p.bt.B, r_first);
+    for (; bb < p.bt.B && row_off[bb] < r_end; ++bb) {
+      const int before = __popc(kmask & ((1u << (int)(row_off[bb] - r_first)) - 1u));
       p.out_off[bb] = base + before;
     }
   }
@@ -159,7 +181,7 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   const int64_t ntiles = (R + kScanTile - 1) / kScanTile;
   if (tile == ntiles - 1 && tid == 0) {
     const long long total = s_prefix + tile_total;
-    for (int bb = p.bt.B; bb >= 0 && p.bt.row_off[bb] >= R; --bb) p.out_off[bb] = total;
+    for (int bb = p.bt.B; bb >= 0 && row_off[bb] >= R; --bb) p.out_off[bb] = total;
   }
 }
 

@@ -482,6 +482,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
           const uint32_t hp = hcur - 1;
           const int slot = hp & (NXS - 1);
           const int pb = hp & 1;
+          const uint32_t pbase = tmem + lane_base + pb * G::KROWS + half * 32;
           if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (hp / NXS) & 1, nullptr, kLimitNs, true))) {
             ok = false;
           } else {
@@ -495,13 +496,13 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
 #pragma unroll
                 for (int hh = 0; hh < 2; ++hh) {
                   const float2 e = sm.xch[slot][r][hh][j];
-                  if (e.y > 0.f) Z += e.y * tc::ex2(e.x - Mx);
+                  if (e.y > 0.f) Z = fmaf(e.y, tc::ex2(e.x - Mx), Z);
                 }
-              const float invZ = (vrow && Z > 0.f) ? 1.0f / Z : 0.f;
+              // Z >= 1 (the row max contributes exp2(0)); hardware reciprocal
+              const float invZ = (vrow && Z > 0.f) ? tc::rcp(Z) : 0.f;
               float f[NPW];
 #pragma unroll
               for (int q = 0; q < NPW; ++q) f[q] = (invZ > 0.f && cmx[q] != -INFINITY) ? tc::ex2(cmx[q] - Mx) * invZ : 0.f;
-              const uint32_t pbase = tmem + lane_base + pb * G::KROWS + half * 32;
               tc::fence_after();
 #pragma unroll
               for (int q = 0; q < NPW; ++q) {

@@ -227,6 +227,13 @@ __device__ __forceinline__ void setmaxnreg_inc() {
   asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
 }
 
+// hardware reciprocal (relative error within 1 ulp), flushing subnormals
+__device__ __forceinline__ float rcp(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // three-input maximum (sm_100+)
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float d;
