@@ -34,14 +34,19 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   };
   const int64_t rows = b->total_rows, S = b->S_tot, B = b->B, T = b->total_text;
   L.status = take(4);
+  // accumulators zeroed at the start of every prune call: one contiguous range
+  L.zero_begin = off;
   L.counters = take(CNT_SLOTS * 4);
+  L.done = take(B * 4);
+  L.scan_tiles = cdiv(rows, kScanTile);
+  L.scan_state = take(L.scan_tiles * 8);
+  L.seg_state = take(S * 8);
+  L.zero_end = off;
   L.role = take(rows);
   L.keep1 = take(rows);
   L.s1 = take(rows * 4);
   L.s2 = take(rows * 4);
   L.ref1 = take(S * 4);
-  L.s1_list = take(rows * 4);
-  L.n1_seg = take(S * 4);
   L.dense = take(rows * 4);
   L.n1 = take(B * 4);
   L.n1_vis = take(B * 4);
@@ -62,9 +67,6 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   L.refpart = take(L.maxSlots * 4);
   L.ref2 = take(B * 4);
   L.tau2 = take(B * 4);
-  L.done = take(B * 4);
-  L.scan_tiles = cdiv(rows, kScanTile);
-  L.scan_state = take(L.scan_tiles * 8);
   L.stats1_rows = rows;
   L.stats1 = take(rows * (H1 > 0 ? H1 : 1) * 8);
   L.total = off;
@@ -297,9 +299,12 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
 
 // a1 (nullable): in [CLS] mode s1 is formed here from the logits of
 // launch_stage1_scores and written to s1; s2_zero (nullable) is zeroed.
+// plan (nullable): the last CTA also builds the Stage-II work plan, and
+// zeroes the compaction counts count_out / count_vis (nullable).
 int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s1, const uint8_t* keep_in,
                      float lambda1, int do_threshold, float* ref1, uint8_t* keep1, int32_t* n1_vis,
-                     const occam_stage1_args* a1, float* s2_zero, cudaStream_t st, Trace trace = Trace()) {
+                     const occam_stage1_args* a1, float* s2_zero, const Stage2Params* plan, int32_t* count_out,
+                     int32_t* count_vis, cudaStream_t st, Trace trace = Trace()) {
   Stage1FinalizeParams p;
   p.bt = dev_batch(b);
   const bool cls = a1 && a1->mode == OCCAM_STAGE1_CLS;
@@ -319,10 +324,16 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   p.ref1 = ref1;
   p.role = at<uint8_t>(ws, L.role);
   p.keep1 = keep1;
-  p.s1_list = at<int32_t>(ws, L.s1_list);
-  p.n1_seg = at<int32_t>(ws, L.n1_seg);
-  p.n1_vis = n1_vis;
   p.status = at<int>(ws, L.status);
+  p.dense = at<int32_t>(ws, L.dense);
+  p.n1 = at<int32_t>(ws, L.n1);
+  p.n1_vis = n1_vis;
+  p.seg_state = at<unsigned long long>(ws, L.seg_state);
+  p.counters = at<int32_t>(ws, L.counters);
+  p.do_plan = plan ? 1 : 0;
+  if (plan) p.plan = *plan;
+  p.zero_count_out = count_out;
+  p.zero_count_vis = count_vis;
   stage1_finalize_kernel<<<b->S_tot, 256, finalize_smem_bytes(p.smem_rows, cls), st>>>(p);
   trace.mark(st);
   return cuda_ok();
@@ -337,8 +348,10 @@ void launch_twopass(const Stage2Params& p, const WsLayout& L, int sms, cudaStrea
   if (gB > 0) s2_scores_kernel<<<gB, 256, s2_scores_smem_bytes(), st>>>(p);
 }
 
-int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayout& L, void* ws, float* s2,
-                  float* ref2, float lambda2, cudaStream_t st, Trace trace = Trace()) {
+// Stage-II parameter block (the same for the plan, built by the Stage-I
+// finalize kernel, and for the Stage-II kernels).
+Stage2Params stage2_params(const occam_batch* b, const occam_stage2_args* a, const WsLayout& L, void* ws, float* s2,
+                           float* ref2, float lambda2) {
   Stage2Params p;
   p.bt = dev_batch(b);
   p.H = a->H2;
@@ -347,8 +360,6 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
   p.K = static_cast<const __nv_bfloat16*>(a->K2);
   p.scale = (float)(1.0 / std::sqrt((double)a->d2));
   p.role = at<uint8_t>(ws, L.role);
-  p.s1_list = at<int32_t>(ws, L.s1_list);
-  p.n1_seg = at<int32_t>(ws, L.n1_seg);
   p.dense = at<int32_t>(ws, L.dense);
   p.n1 = at<int32_t>(ws, L.n1);
   p.itemsA = at<int4>(ws, L.itemsA);
@@ -371,7 +382,14 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
   p.slot_off = at<int32_t>(ws, L.slot_off);
   p.maxF = L.maxF;
   p.use_fused = fused ? 1 : 0;
-  s2_dense_plan_kernel<<<b->B, 256, 0, st>>>(p, 1);
+  return p;
+}
+
+// Stage II after the Stage-I finalize kernel planned it (same arguments).
+int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayout& L, void* ws, float* s2,
+                  float* ref2, float lambda2, cudaStream_t st, Trace trace = Trace()) {
+  const Stage2Params p = stage2_params(b, a, L, ws, s2, ref2, lambda2);
+  const bool fused = p.use_fused != 0;
   trace.mark(st);
   const int sms = num_sms();
   if (fused) {
@@ -520,7 +538,8 @@ int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   set_smem_attrs();
   OCCAM_TRY(launch_stage1_scores(batch, args, L, workspace, s1, nullptr, st));
-  OCCAM_TRY(launch_finalize1(batch, L, workspace, s1, nullptr, 0.f, 0, ref1, nullptr, nullptr, args, nullptr, st));
+  OCCAM_TRY(launch_finalize1(batch, L, workspace, s1, nullptr, 0.f, 0, ref1, nullptr, nullptr, args, nullptr, nullptr,
+                             nullptr, nullptr, st));
   return OCCAM_OK;
 }
 
@@ -561,33 +580,12 @@ int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   set_smem_attrs();
   OCCAM_TRY(mark_roles(batch, L, workspace, st));
-  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(workspace, L.counters), 0, CNT_SLOTS * 4, st));
-  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(workspace, L.done), 0, batch->B * 4, st));
-  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(workspace, L.n1_vis), 0, batch->B * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(at<unsigned char>(workspace, L.zero_begin), 0, L.zero_end - L.zero_begin, st));
   OCCAM_CUDA(cudaMemsetAsync(s2, 0, batch->total_rows * 4, st));
-  // S1 lists from the given mask (registers always in S1)
-  Stage1FinalizeParams f;
-  f.bt = dev_batch(batch);
-  f.logits = nullptr;
-  f.q_cls = nullptr;
-  f.k_cls = nullptr;
-  f.scale = 1.f;
-  f.s1_out = nullptr;
-  f.s2_zero = nullptr;
-  f.smem_rows = 0;
-  f.s1 = nullptr;
-  f.keep_in = keep1;
-  f.lambda1 = 0.f;
-  f.do_threshold = 1;
-  f.ref1 = nullptr;
-  f.role = at<uint8_t>(workspace, L.role);
-  f.keep1 = nullptr;
-  f.s1_list = at<int32_t>(workspace, L.s1_list);
-  f.n1_seg = at<int32_t>(workspace, L.n1_seg);
-  f.n1_vis = at<int32_t>(workspace, L.n1_vis);
-  f.status = at<int>(workspace, L.status);
-  stage1_finalize_kernel<<<batch->S_tot, 256, 0, st>>>(f);
-  OCCAM_TRY(cuda_ok());
+  // S1 lists from the given mask (registers always in S1) and the Stage-II plan
+  const Stage2Params plan = stage2_params(batch, args, L, workspace, s2, ref2, 1.0f);
+  OCCAM_TRY(launch_finalize1(batch, L, workspace, nullptr, keep1, 0.f, 1, nullptr, nullptr,
+                             at<int32_t>(workspace, L.n1_vis), nullptr, nullptr, &plan, nullptr, nullptr, st));
   return launch_stage2(batch, args, L, workspace, s2, ref2, 1.0f, st);
 }
 
@@ -629,15 +627,12 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   int32_t* n1_vis = out->n1_vis ? out->n1_vis : at<int32_t>(ws, L.n1_vis);
   float* ref2 = out->ref2 ? out->ref2 : at<float>(ws, L.ref2);
   // every zero-initialised accumulator of the call, up front
-  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(ws, L.counters), 0, CNT_SLOTS * 4, st));
-  OCCAM_CUDA(cudaMemsetAsync(at<int32_t>(ws, L.done), 0, b->B * 4, st));
-  OCCAM_CUDA(cudaMemsetAsync(n1_vis, 0, b->B * 4, st));
-  OCCAM_CUDA(cudaMemsetAsync(at<unsigned long long>(ws, L.scan_state), 0, L.scan_tiles * 8, st));
-  OCCAM_CUDA(cudaMemsetAsync(out->count_out, 0, b->B * 4, st));
-  OCCAM_CUDA(cudaMemsetAsync(out->count_vis, 0, b->B * 4, st));
+  OCCAM_CUDA(cudaMemsetAsync(at<unsigned char>(ws, L.zero_begin), 0, L.zero_end - L.zero_begin, st));
   trace.mark(st);
   OCCAM_TRY(launch_stage1_scores(b, &args->stage1, L, ws, s1, s2, st, trace));
+  const Stage2Params plan = stage2_params(b, &args->stage2, L, ws, s2, ref2, args->lambda2);
   OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, &args->stage1, s2,
+                             &plan, out->count_out, out->count_vis,
                              st, trace));
   OCCAM_TRY(launch_stage2(b, &args->stage2, L, ws, s2, ref2, args->lambda2, st, trace));
   return launch_compact(b, L, ws, 1, nullptr, keep1, s2, args->keep_registers, out->keep2, args->n_tensors,

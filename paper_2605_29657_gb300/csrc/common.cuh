@@ -175,11 +175,23 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+// release store / acquire load of a 64-bit flag word (GPU scope)
+__device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
 // ---------------------------------------------------------------- internal parameter blocks
 // Workspace carve-up (byte offsets from the workspace base; see ws_layout()).
 struct WsLayout {
-  size_t status, counters, role, keep1, s1, s2, ref1, s1_list, n1_seg, dense, n1, n1_vis;
-  size_t itemsA, itemsB, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, stats1, itemsF, itemsF8, slot_off;
+  size_t status, counters, role, keep1, s1, s2, ref1, dense, n1, n1_vis;
+  size_t itemsA, itemsB, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, seg_state, stats1, itemsF, itemsF8,
+      slot_off;
+  size_t zero_begin, zero_end;  // the accumulators every prune call zeroes (one contiguous range)
   size_t total;
   int64_t maxA, maxB, maxF, maxSlots, scan_tiles, stats1_rows;
 };
@@ -194,7 +206,8 @@ enum {
   CNT_NF8 = 5,
   CNT_QUEUE4 = 6,  // next fused Stage-II item (4-CTA clusters)
   CNT_QUEUE8 = 7,  // next fused Stage-II item (8-CTA clusters)
-  CNT_SLOTS = 8
+  CNT_SEG_TICKET = 8,  // Stage-I finalize: segment order
+  CNT_SLOTS = 9
 };
 
 constexpr int kTextTile = 64;    // Stage-II text rows per item

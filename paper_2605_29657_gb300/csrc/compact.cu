@@ -25,14 +25,6 @@ constexpr unsigned long long kFlagAgg = 1ull << 62;
 constexpr unsigned long long kFlagPre = 2ull << 62;
 constexpr unsigned long long kValMask = (1ull << 62) - 1;
 
-__device__ __forceinline__ void st_release(unsigned long long* p, unsigned long long v) {
-  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
-}
-__device__ __forceinline__ unsigned long long ld_acquire(const unsigned long long* p) {
-  unsigned long long v;
-  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
-  return v;
-}
 }  // namespace
 
 constexpr int kScanSmemSamples = 2048;  // samples whose offsets fit the scan's shared copy
@@ -95,15 +87,15 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
     const int lane = tid;
     long long excl = 0;
     if (tile == 0) {
-      if (lane == 0) st_release(&p.tile_state[0], kFlagPre | (unsigned long long)tile_total);
+      if (lane == 0) st_release_u64(&p.tile_state[0], kFlagPre | (unsigned long long)tile_total);
     } else {
-      if (lane == 0) st_release(&p.tile_state[tile], kFlagAgg | (unsigned long long)tile_total);
+      if (lane == 0) st_release_u64(&p.tile_state[tile], kFlagAgg | (unsigned long long)tile_total);
       int64_t hi = tile - 1;
       bool timed_out = false;
       uint32_t spins = 0;
       while (true) {
         const int64_t q = hi - lane;
-        const unsigned long long v = q >= 0 ? ld_acquire(&p.tile_state[q]) : kFlagPre;
+        const unsigned long long v = q >= 0 ? ld_acquire_u64(&p.tile_state[q]) : kFlagPre;
         if (!__all_sync(0xffffffffu, (v & (kFlagAgg | kFlagPre)) != 0)) {
           if (++spins > kSpinLimit) {
             timed_out = true;
@@ -123,7 +115,7 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
       }
       if (lane == 0) {
         if (timed_out) set_status(p.status, OCCAM_ERR_TIMEOUT);
-        st_release(&p.tile_state[tile], kFlagPre | (unsigned long long)(excl + tile_total));
+        st_release_u64(&p.tile_state[tile], kFlagPre | (unsigned long long)(excl + tile_total));
       }
     }
     if (lane == 0) s_prefix = excl;

@@ -36,29 +36,6 @@ struct Stage1ClsParams {
   int* status;
 };
 
-struct Stage1FinalizeParams {
-  BatchDev bt;
-  // [CLS] mode: the segment's s1 is first formed from the per-head logits
-  // (softmax over the segment's rows and the [CLS] self key, head mean)
-  const float* logits;            // nullable: s1 is given instead
-  const __nv_bfloat16* q_cls;     // [CLS] mode
-  const __nv_bfloat16* k_cls;     // nullable
-  float scale;
-  float* s1_out;                  // [CLS] mode: where s1 is written
-  float* s2_zero;                 // nullable: zeroed per row (Stage-II max accumulator)
-  int smem_rows;                  // segments up to this many rows stage their logits in shared memory
-  const float* s1;          // nullable when keep_in is given
-  const uint8_t* keep_in;   // nullable: S1 membership of visual rows given instead of tested
-  float lambda1;
-  int do_threshold;
-  float* ref1;       // nullable
-  uint8_t* role;
-  uint8_t* keep1;
-  int32_t* s1_list;  // per segment, at seg_off[s]
-  int32_t* n1_seg;
-  int32_t* n1_vis;   // [B], accumulated
-  int* status;
-};
 
 struct MutualParams {
   BatchDev bt;
@@ -92,9 +69,7 @@ struct Stage2Params {
   const __nv_bfloat16* K;   // [rows, H, 128]
   float scale;
   const uint8_t* role;
-  const int32_t* s1_list;   // per segment lists
-  const int32_t* n1_seg;
-  int32_t* dense;           // per sample dense S1 list at row_off[b]
+  int32_t* dense;           // per sample S1 list at row_off[b]
   int32_t* n1;              // [B]
   int4* itemsA;             // (b, j0, head group, -)
   int4* itemsB;             // (b, j0, key chunk, item index within sample)
@@ -114,6 +89,40 @@ struct Stage2Params {
   float* tau2;              // [B]
   float lambda2;
   int* status;
+};
+
+struct Stage1FinalizeParams {
+  BatchDev bt;
+  // [CLS] mode: the segment's s1 is first formed from the per-head logits
+  // (softmax over the segment's rows and the [CLS] self key, head mean)
+  const float* logits;            // nullable: s1 is given instead
+  const __nv_bfloat16* q_cls;     // [CLS] mode
+  const __nv_bfloat16* k_cls;     // nullable
+  float scale;
+  float* s1_out;                  // [CLS] mode: where s1 is written
+  float* s2_zero;                 // nullable: zeroed per row (Stage-II max accumulator)
+  int smem_rows;                  // segments up to this many rows stage their logits in shared memory
+  const float* s1;          // nullable when keep_in is given
+  const uint8_t* keep_in;   // nullable: S1 membership of visual rows given instead of tested
+  float lambda1;
+  int do_threshold;
+  float* ref1;       // nullable
+  uint8_t* role;
+  uint8_t* keep1;
+  int* status;
+  // S1 lists (do_threshold): every sample's S1 rows in row order, at
+  // dense[row_off[b]]; segments take their place in the sample's list by a
+  // look-back over the sample's earlier segments
+  int32_t* dense;
+  int32_t* n1;               // [B] S1 keys of the sample (visual + registers)
+  int32_t* n1_vis;           // [B] visual S1 rows of the sample
+  unsigned long long* seg_state;  // [S_tot] look-back states, zero before the launch
+  int32_t* counters;         // CNT_SEG_TICKET, CNT_DENSE_DONE
+  // Stage-II work plan, built by the last CTA to finish (do_plan)
+  int do_plan;
+  Stage2Params plan;
+  int32_t* zero_count_out;   // nullable: [B] zeroed by the planning CTA (compaction accumulators)
+  int32_t* zero_count_vis;   // nullable
 };
 
 struct ScanParams {
@@ -181,7 +190,7 @@ __global__ void roles_scatter_kernel(BatchDev bt, uint8_t* role);
 __global__ void threshold_kernel(ThresholdParams p);
 
 // stage2.cu
-__global__ void s2_dense_plan_kernel(Stage2Params p, int build_dense);
+
 __global__ void s2_stats_kernel(Stage2Params p);
 __global__ void s2_scores_kernel(Stage2Params p);
 int s2_scores_smem_bytes();

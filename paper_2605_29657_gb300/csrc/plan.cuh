@@ -1,0 +1,83 @@
+// plan.cuh -- the Stage-II work plan (internal header): which Stage-II path
+// each sample takes and the item lists of those paths. Run by one CTA (the
+// last Stage-I finalize CTA to finish) once every sample's S1 size n1[b] is
+// known.
+#pragma once
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace occam {
+
+// Routes every sample (the fused tensor-core kernel with 4- or 8-CTA
+// clusters where its S1 keys and text keys fit, else the two-pass kernels)
+// and writes the item lists, the per-sample item and partial-slot offsets,
+// and the item counts. blockDim.x threads, tmp: >= 40 ints of shared memory.
+__device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
+  const int tid = threadIdx.x;
+  const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
+  int runA = 0, runB = 0, runF = 0, runF8 = 0, runS = 0;
+  for (int b0 = 0; b0 < p.bt.B; b0 += blockDim.x) {
+    const int bb = b0 + tid;
+    int nA = 0, nB = 0, nF = 0, nF8 = 0;
+    if (bb < p.bt.B) {
+      const int M = (int)(p.bt.text_off[bb + 1] - p.bt.text_off[bb]);
+      const int n1 = *((volatile int32_t*)&p.n1[bb]);
+      // the fused tensor-core kernel takes a sample when its S1 keys and its
+      // causal text keys fit the cluster's TMEM / shared memory
+      const bool fused4 = p.use_fused && fused_fits(kFusedCluster, n1, M, p.H);
+      const bool fused8 = !fused4 && p.use_fused && fused_fits(8, n1, M, p.H);
+      if (fused4) {
+        nF = (M + 127) / 128;
+      } else if (fused8) {
+        nF8 = (M + 127) / 128;
+      } else {
+        const int tiles = (M + kTextTile - 1) / kTextTile;
+        const int nch = (n1 + kKeyChunk - 1) / kKeyChunk;
+        nA = tiles * nhg;
+        nB = tiles * nch;
+      }
+      if (M == 0) {
+        set_status(p.status, OCCAM_ERR_INVALID_ARG);
+        p.ref2[bb] = 0.f;
+        p.tau2[bb] = 0.f;
+      }
+    }
+    const int nch = (bb < p.bt.B) ? (*((volatile int32_t*)&p.n1[bb]) + kKeyChunk - 1) / kKeyChunk : 0;
+    const int nS = nF * kFusedSlotsPerItem + nF8 * kFusedSlotsPerItem8 + nB;  // s2(r) partial slots of this sample
+    int totA, totB, totF, totF8, totS;
+    const int offA = runA + block_exclusive_scan(nA, tmp, &totA);
+    const int offB = runB + block_exclusive_scan(nB, tmp, &totB);
+    const int offF = runF + block_exclusive_scan(nF, tmp, &totF);
+    const int offF8 = runF8 + block_exclusive_scan(nF8, tmp, &totF8);
+    const int offS = runS + block_exclusive_scan(nS, tmp, &totS);
+    if (bb < p.bt.B) {
+      for (int i = 0; i < nA; ++i)
+        if (offA + i < p.maxA) p.itemsA[offA + i] = make_int4(bb, (i / nhg) * kTextTile, i % nhg, 0);
+      for (int i = 0; i < nB; ++i)
+        if (offB + i < p.maxB) p.itemsB[offB + i] = make_int4(bb, (i / nch) * kTextTile, i % nch, offS + i);
+      for (int i = 0; i < nF; ++i)
+        if (offF + i < p.maxF) p.itemsF[offF + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem, 0);
+      for (int i = 0; i < nF8; ++i)
+        if (offF8 + i < p.maxF) p.itemsF8[offF8 + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem8, 0);
+      p.itemB_off[bb] = offB;
+      p.slot_off[bb] = offS;
+    }
+    runA += totA;
+    runB += totB;
+    runF += totF;
+    runF8 += totF8;
+    runS += totS;
+  }
+  if (tid == 0) {
+    p.itemB_off[p.bt.B] = runB;
+    p.slot_off[p.bt.B] = runS;
+    if (runA > p.maxA || runB > p.maxB || runF > p.maxF || runF8 > p.maxF) set_status(p.status, OCCAM_ERR_CAPACITY);
+    p.counters[CNT_NA] = (int)(runA < p.maxA ? runA : p.maxA);
+    p.counters[CNT_NB] = (int)(runB < p.maxB ? runB : p.maxB);
+    p.counters[CNT_NF] = (int)(runF < p.maxF ? runF : p.maxF);
+    p.counters[CNT_NF8] = (int)(runF8 < p.maxF ? runF8 : p.maxF);
+  }
+}
+
+}  // namespace occam

@@ -4,6 +4,7 @@
 // (Eqs. 4-6; App. A, Eqs. 10-13).
 #include "common.cuh"
 #include "kernels.cuh"
+#include "plan.cuh"
 
 namespace occam {
 
@@ -199,8 +200,14 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   extern __shared__ float4 fin_smem[];
   __shared__ int tmp[40];
   __shared__ float sref;
-  const int seg = blockIdx.x;
+  __shared__ int s_seg, s_last;
+  __shared__ long long s_base;
   const int tid = threadIdx.x;
+  // with S1 lists, segments are taken in ticket order: every earlier segment
+  // of the sample has started, so the look-back below always ends
+  if (tid == 0) s_seg = p.do_threshold ? atomicAdd(&p.counters[CNT_SEG_TICKET], 1) : (int)blockIdx.x;
+  __syncthreads();
+  const int seg = s_seg;
   const int64_t sb = p.bt.seg_off[seg], se = p.bt.seg_off[seg + 1];
   const int n = (int)(se - sb);
   const int ra = p.bt.reg_off[seg], rb = p.bt.reg_off[seg + 1];
@@ -214,9 +221,22 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   if (p.logits) {
     const float* lg = p.logits + sb * 16;
     if (staged) {
-      const float4* src = reinterpret_cast<const float4*>(lg);
-      float4* dst = reinterpret_cast<float4*>(lg_loc);
-      for (int i = tid; i < n * 4; i += blockDim.x) dst[i] = src[i];
+      // eight independent 16-byte loads in flight per thread, then the stores
+      const float4* __restrict__ src = reinterpret_cast<const float4*>(lg);
+      const int nv = n * 4;
+      for (int base = 0; base < nv; base += 8 * 256) {
+        float4 t[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int i = base + u * 256 + tid;
+          if (i < nv) t[u] = __ldg(src + i);
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int i = base + u * 256 + tid;
+          if (i < nv) fin_smem[i] = t[u];
+        }
+      }
       __syncthreads();
       lg = lg_loc;
     }
@@ -271,19 +291,79 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
     cnt += k;
     cvis += (k && !reg);
   }
-  int total;
+  int total, vis_total;
   int pos = block_exclusive_scan(cnt, tmp, &total);
+  block_exclusive_scan(cvis, tmp, &vis_total);
+  // this segment's place in its sample's S1 list: a look-back over the
+  // sample's earlier segments (warp 0, a window of 32 at a time). A state
+  // packs the visual count (bits 31..61) and the key count (bits 0..30)
+  // with an "aggregate" or "inclusive prefix" flag.
+  const int b = p.bt.seg_sample[seg];
+  const int s0 = p.bt.seg_first[b];
+  constexpr unsigned long long kAgg = 1ull << 62, kPre = 2ull << 62, kLo = (1ull << 31) - 1;
+  if (tid < 32) {
+    const unsigned long long mine = ((unsigned long long)vis_total << 31) | (unsigned long long)total;
+    unsigned long long excl = 0;
+    if (seg == s0) {
+      if (tid == 0) st_release_u64(&p.seg_state[seg], kPre | mine);
+    } else {
+      if (tid == 0) st_release_u64(&p.seg_state[seg], kAgg | mine);
+      int hi = seg - 1;
+      bool timed_out = false;
+      uint32_t spins = 0;
+      while (true) {
+        const int q = hi - tid;
+        const unsigned long long v = q >= s0 ? ld_acquire_u64(&p.seg_state[q]) : kPre;
+        if (!__all_sync(0xffffffffu, (v & (kAgg | kPre)) != 0)) {
+          if (++spins > kSpinLimit) {
+            timed_out = true;
+            break;
+          }
+          __nanosleep(32);
+          continue;
+        }
+        const unsigned pre = __ballot_sync(0xffffffffu, (v & kPre) != 0);
+        const int first = pre ? __ffs(pre) - 1 : 32;
+        unsigned long long val = tid <= first ? (v & ~(kAgg | kPre)) : 0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) val += __shfl_xor_sync(0xffffffffu, val, o);
+        excl += val;
+        if (pre) break;
+        hi -= 32;
+      }
+      if (tid == 0) {
+        if (timed_out) set_status(p.status, OCCAM_ERR_TIMEOUT);
+        st_release_u64(&p.seg_state[seg], kPre | (excl + mine));
+      }
+    }
+    if (tid == 0) {
+      s_base = (long long)(excl & kLo);
+      if (seg + 1 == p.bt.seg_first[b + 1]) {  // the sample's last segment
+        p.n1[b] = (int)((excl & kLo) + (unsigned long long)total);
+        if (p.n1_vis) p.n1_vis[b] = (int)(((excl >> 31) & kLo) + (unsigned long long)vis_total);
+      }
+    }
+  }
+  __syncthreads();
+  int32_t* list = p.dense + p.bt.row_off[b] + s_base;
   for (int r = a; r < z; ++r) {
     const bool reg = role[r] != 0;
     const bool k = reg || (p.keep_in ? p.keep_in[sb + r] != 0 : (staged ? s1_loc[r] : s1g[sb + r]) >= tau);
     if (p.keep1) p.keep1[sb + r] = k ? 1 : 0;
-    if (k) p.s1_list[sb + pos++] = (int32_t)(sb + r);
+    if (k) list[pos++] = (int32_t)(sb + r);
   }
-  int vis_total;
-  block_exclusive_scan(cvis, tmp, &vis_total);
-  if (tid == 0) {
-    p.n1_seg[seg] = total;
-    atomicAdd(&p.n1_vis[p.bt.seg_sample[seg]], vis_total);
+  if (!p.do_plan) return;
+  // the last CTA to finish plans Stage II
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = atomicAdd(&p.counters[CNT_DENSE_DONE], 1) == (int)gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  plan_stage2(p.plan, tmp);
+  for (int i = tid; i < p.bt.B; i += blockDim.x) {
+    if (p.zero_count_out) p.zero_count_out[i] = 0;
+    if (p.zero_count_vis) p.zero_count_vis[i] = 0;
   }
 }
 

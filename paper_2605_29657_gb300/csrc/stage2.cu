@@ -27,98 +27,6 @@ constexpr int LD = D + 8;  // padded smem row (272 B): conflict-free ldmatrix
 constexpr int KT = 64;     // keys per stats chunk
 }  // namespace s2k
 
-// ---------------------------------------------------------------------------
-// Dense per-sample S1 lists + work plan. Grid: one CTA per sample; the last
-// CTA to finish builds the item lists of both passes.
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) s2_dense_plan_kernel(Stage2Params p, int build_dense) {
-  __shared__ int tmp[40];
-  __shared__ int is_last;
-  const int b = blockIdx.x, tid = threadIdx.x;
-  if (build_dense) {
-    const int sf = p.bt.seg_first[b], sl = p.bt.seg_first[b + 1];
-    const int64_t rbase = p.bt.row_off[b];
-    int base = 0;
-    for (int s = sf; s < sl; ++s) {
-      const int cnt = p.n1_seg[s];
-      const int64_t so = p.bt.seg_off[s];
-      for (int k = tid; k < cnt; k += blockDim.x) p.dense[rbase + base + k] = p.s1_list[so + k];
-      base += cnt;
-    }
-    if (tid == 0) p.n1[b] = base;
-  }
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) is_last = (atomicAdd(&p.counters[CNT_DENSE_DONE], 1) == (int)gridDim.x - 1);
-  __syncthreads();
-  if (!is_last) return;
-  __threadfence();
-  const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
-  int runA = 0, runB = 0, runF = 0, runF8 = 0, runS = 0;
-  for (int b0 = 0; b0 < p.bt.B; b0 += blockDim.x) {
-    const int bb = b0 + tid;
-    int nA = 0, nB = 0, nF = 0, nF8 = 0, tiles = 0, nch = 0, tiles128 = 0;
-    if (bb < p.bt.B) {
-      const int M = (int)(p.bt.text_off[bb + 1] - p.bt.text_off[bb]);
-      const int n1 = *((volatile int32_t*)&p.n1[bb]);
-      // the fused tensor-core kernel takes a sample when its S1 keys and its
-      // causal text keys fit the cluster's TMEM / shared memory
-      const bool fused4 = p.use_fused && fused_fits(kFusedCluster, n1, M, p.H);
-      const bool fused8 = !fused4 && p.use_fused && fused_fits(8, n1, M, p.H);
-      if (fused4) {
-        tiles128 = (M + 127) / 128;
-        nF = tiles128;
-      } else if (fused8) {
-        tiles128 = (M + 127) / 128;
-        nF8 = tiles128;
-      } else {
-        tiles = (M + kTextTile - 1) / kTextTile;
-        nch = (n1 + kKeyChunk - 1) / kKeyChunk;
-        nA = tiles * nhg;
-        nB = tiles * nch;
-      }
-      if (M == 0) {
-        set_status(p.status, OCCAM_ERR_INVALID_ARG);
-        p.ref2[bb] = 0.f;
-        p.tau2[bb] = 0.f;
-      }
-    }
-    const int nS = nF * kFusedSlotsPerItem + nF8 * kFusedSlotsPerItem8 + nB;  // s2(r) partial slots of this sample
-    int totA, totB, totF, totF8, totS;
-    const int offA = runA + block_exclusive_scan(nA, tmp, &totA);
-    const int offB = runB + block_exclusive_scan(nB, tmp, &totB);
-    const int offF = runF + block_exclusive_scan(nF, tmp, &totF);
-    const int offF8 = runF8 + block_exclusive_scan(nF8, tmp, &totF8);
-    const int offS = runS + block_exclusive_scan(nS, tmp, &totS);
-    if (bb < p.bt.B) {
-      for (int i = 0; i < nA; ++i)
-        if (offA + i < p.maxA) p.itemsA[offA + i] = make_int4(bb, (i / nhg) * kTextTile, i % nhg, 0);
-      for (int i = 0; i < nB; ++i)
-        if (offB + i < p.maxB) p.itemsB[offB + i] = make_int4(bb, (i / nch) * kTextTile, i % nch, offS + i);
-      for (int i = 0; i < nF; ++i)
-        if (offF + i < p.maxF) p.itemsF[offF + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem, 0);
-      for (int i = 0; i < nF8; ++i)
-        if (offF8 + i < p.maxF) p.itemsF8[offF8 + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem8, 0);
-      p.itemB_off[bb] = offB;
-      p.slot_off[bb] = offS;
-    }
-    runA += totA;
-    runB += totB;
-    runF += totF;
-    runF8 += totF8;
-    runS += totS;
-  }
-  if (tid == 0) {
-    p.itemB_off[p.bt.B] = runB;
-    p.slot_off[p.bt.B] = runS;
-    if (runA > p.maxA || runB > p.maxB || runF > p.maxF || runF8 > p.maxF) set_status(p.status, OCCAM_ERR_CAPACITY);
-    p.counters[CNT_NA] = (int)(runA < p.maxA ? runA : p.maxA);
-    p.counters[CNT_NB] = (int)(runB < p.maxB ? runB : p.maxB);
-    p.counters[CNT_NF] = (int)(runF < p.maxF ? runF : p.maxF);
-    p.counters[CNT_NF8] = (int)(runF8 < p.maxF ? runF8 : p.maxF);
-  }
-}
-
 // copy one 64- or 128-key chunk of head h into sdst[key][0..128) (stride LD)
 __device__ __forceinline__ void s2_load_keys(__nv_bfloat16* sdst, const Stage2Params& p, int b, int64_t t0,
                                              int n_img, int total, int k0, int nkeys_tile, int h, int tid,
