@@ -152,9 +152,9 @@ def algorithmic_bytes(meta: dict, n1_total: int, kept_total: int) -> dict:
     k2row = H2 * d2 * 2
     hrow = hid * 2                       # bytes of one hidden / V row (bf16)
     b = {}
-    b["stage1"] = rows * k1row + 2 * S * k1row + rows * 8            # K1 once, q/k_cls, s1 write, s2 zero
-    b["stage1_finalize"] = rows * (4 + 1 + 1 + 4)                    # s1 read, role, keep1, list
-    b["s1_list_plan"] = n1_total * 8                                 # list copy
+    b["stage1"] = rows * k1row + S * k1row + rows * H1 * 4           # K1 once, q_cls, logits write
+    b["stage1_finalize"] = rows * (H1 * 4 + 4 + 4 + 1 + 1 + 4) + S * k1row  # logits, s1 + s2 zero, role, keep1, list; q/k_cls
+    b["s1_list_plan"] = 0                                            # planned inside the finalize kernel
     b["stage2_fused"] = n1_total * k2row + 2 * T * k2row               # S1 keys once, Q + K_text
     b["stage2_twopass"] = 2 * n1_total * k2row + 3 * T * k2row + 2 * T * H2 * 8  # both passes
     b["scan"] = rows * (1 + 1 + 4 + 1) + kept_total * 4              # keep1, role, s2, keep2, out_index
@@ -386,10 +386,10 @@ def run_ours(args, rank, world, local):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        # kernels per occam_prune call: Stage I (1 [CLS] / 2 mutual), finalize,
-        # plan, fused Stage II with 4- and 8-CTA clusters, the two-pass Stage-II
-        # pair, scan, gather
-        "gpu_launches": (9 if w.stage1 == "cls" else 10) * args.steps,
+        # kernels per occam_prune call: Stage I (1 [CLS] / 2 mutual), finalize
+        # (with the Stage-II plan), fused Stage II with 4- and 8-CTA clusters,
+        # the two-pass Stage-II pair, scan, gather
+        "gpu_launches": (8 if w.stage1 == "cls" else 9) * args.steps,
         "clocks": clocks,
     }
     if world > 1:
