@@ -184,47 +184,34 @@ __device__ __forceinline__ void ld_wait(uint32_t (&v)[32]) {
 // values are read again).
 template <bool STORE>
 __device__ __forceinline__ void piece_stats(uint32_t (&v)[32], uint32_t sa, int lim, float sl2, float& cm, float& a) {
-  if (__all_sync(0xffffffffu, lim >= 32)) {
-    float t[11];
+  if (!__all_sync(0xffffffffu, lim >= 32)) {
+    // partial piece (causal text keys, the last S1 piece, padded rows):
+    // masked logits become -inf, whose exponential is exactly 0
 #pragma unroll
-    for (int i = 0; i < 10; ++i)
-      t[i] = tc::fmax3(__uint_as_float(v[3 * i]), __uint_as_float(v[3 * i + 1]), __uint_as_float(v[3 * i + 2]));
-    t[10] = fmaxf(__uint_as_float(v[30]), __uint_as_float(v[31]));
-    const float mx = fmaxf(tc::fmax3(tc::fmax3(t[0], t[1], t[2]), tc::fmax3(t[3], t[4], t[5]), tc::fmax3(t[6], t[7], t[8])),
-                           fmaxf(t[9], t[10]));
-    cm = mx * sl2;
-    const float2 sc = make_float2(sl2, sl2), off = make_float2(-cm, -cm);
-    float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), sc, off);
-      x.x = tc::ex2(x.x);
-      x.y = tc::ex2(x.y);
-      acc[i & 3] = __fadd2_rn(acc[i & 3], x);
-      v[2 * i] = __float_as_uint(x.x);
-      v[2 * i + 1] = __float_as_uint(x.y);
-    }
-    a = ((acc[0].x + acc[0].y) + (acc[1].x + acc[1].y)) + ((acc[2].x + acc[2].y) + (acc[3].x + acc[3].y));
-  } else {
-    float c0 = -INFINITY, c1 = -INFINITY;
-#pragma unroll
-    for (int col = 0; col < 32; col += 2) {
-      if (col < lim) c0 = fmaxf(c0, __uint_as_float(v[col]));
-      if (col + 1 < lim) c1 = fmaxf(c1, __uint_as_float(v[col + 1]));
-    }
-    cm = fmaxf(c0, c1) * sl2;
-    float a0 = 0.f, a1 = 0.f;
-#pragma unroll
-    for (int col = 0; col < 32; col += 2) {
-      const float e0 = (col < lim) ? tc::ex2(fmaf(__uint_as_float(v[col]), sl2, -cm)) : 0.f;
-      const float e1 = (col + 1 < lim) ? tc::ex2(fmaf(__uint_as_float(v[col + 1]), sl2, -cm)) : 0.f;
-      a0 += e0;
-      a1 += e1;
-      v[col] = __float_as_uint(e0);
-      v[col + 1] = __float_as_uint(e1);
-    }
-    a = a0 + a1;
+    for (int col = 0; col < 32; ++col) v[col] = col < lim ? v[col] : 0xff800000u;
   }
+  float t[11];
+#pragma unroll
+  for (int i = 0; i < 10; ++i)
+    t[i] = tc::fmax3(__uint_as_float(v[3 * i]), __uint_as_float(v[3 * i + 1]), __uint_as_float(v[3 * i + 2]));
+  t[10] = fmaxf(__uint_as_float(v[30]), __uint_as_float(v[31]));
+  const float mx = fmaxf(tc::fmax3(tc::fmax3(t[0], t[1], t[2]), tc::fmax3(t[3], t[4], t[5]), tc::fmax3(t[6], t[7], t[8])),
+                         fmaxf(t[9], t[10]));
+  cm = mx * sl2;  // -inf when no column is valid
+  const float2 sc = make_float2(sl2, sl2);
+  const float o = cm == -INFINITY ? 0.f : -cm;
+  const float2 off = make_float2(o, o);
+  float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), sc, off);
+    x.x = tc::ex2(x.x);
+    x.y = tc::ex2(x.y);
+    acc[i & 3] = __fadd2_rn(acc[i & 3], x);
+    v[2 * i] = __float_as_uint(x.x);
+    v[2 * i + 1] = __float_as_uint(x.y);
+  }
+  a = ((acc[0].x + acc[0].y) + (acc[1].x + acc[1].y)) + ((acc[2].x + acc[2].y) + (acc[3].x + acc[3].y));
   if (STORE) tc::tmem_st32(sa, v);
 }
 
