@@ -282,14 +282,19 @@ __global__ void __launch_bounds__(256, 1) s2_scores_kernel(Stage2Params p) {
       last_flag = (atomicAdd(&p.done[b], 1) == nslots - 1);
     }
     __syncthreads();
-    if (last_flag && tid == 0) {
+    if (last_flag && tid < 32) {
+      // the sample's last partial: lane l sums slots l, l + 32, ... in order,
+      // then a fixed tree over the lanes (deterministic)
       __threadfence();
       float acc = 0.f;
-      for (int i = p.slot_off[b]; i < p.slot_off[b + 1]; ++i) acc += *((volatile float*)&p.refpart[i]);
-      const int R = p.bt.reg_off[p.bt.seg_first[b + 1]] - p.bt.reg_off[p.bt.seg_first[b]];
-      const float r2 = (R > 0 && M > 0) ? acc / ((float)R * (float)M) : 0.f;
-      p.ref2[b] = r2;
-      p.tau2[b] = p.lambda2 * r2;
+      for (int i = p.slot_off[b] + tid; i < p.slot_off[b + 1]; i += 32) acc += __ldcg(&p.refpart[i]);
+      acc = warp_sum(acc);
+      if (tid == 0) {
+        const int R = p.bt.reg_off[p.bt.seg_first[b + 1]] - p.bt.reg_off[p.bt.seg_first[b]];
+        const float r2 = (R > 0 && M > 0) ? acc / ((float)R * (float)M) : 0.f;
+        p.ref2[b] = r2;
+        p.tau2[b] = p.lambda2 * r2;
+      }
     }
     __syncthreads();
   }

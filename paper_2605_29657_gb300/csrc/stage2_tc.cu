@@ -218,9 +218,11 @@ __device__ __forceinline__ void piece_stats(uint32_t (&v)[32], uint32_t sa, int 
 // merges a piece's (cm, a) into the row's running softmax (m, z), log2 units
 __device__ __forceinline__ void online_merge(float& m, float& z, float cm, float a) {
   if (cm != -INFINITY) {
-    const float mn = fmaxf(m, cm);
-    z = (m == -INFINITY ? 0.f : z * tc::ex2(m - mn)) + a * tc::ex2(cm - mn);
-    m = mn;
+    // one exponential: the smaller of the two maxima is rescaled to the larger
+    const bool up = cm > m;  // also when m is still -inf (then e = 0 and z = 0)
+    const float e = tc::ex2(up ? m - cm : cm - m);
+    z = up ? fmaf(z, e, a) : fmaf(a, e, z);
+    m = up ? cm : m;
   }
 }
 
@@ -592,14 +594,22 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
           }
         }
       }
+      int last = 0;
       if (lane == 0) {
         p.refpart[g.slot + rank * NEPI + ew] = regacc;  // C * NEPI slots per item
         __threadfence();
         const int nslots = p.slot_off[g.b + 1] - p.slot_off[g.b];
-        if (atomicAdd(&p.done[g.b], 1) == nslots - 1) {
-          __threadfence();
-          float acc = 0.f;
-          for (int i = p.slot_off[g.b]; i < p.slot_off[g.b + 1]; ++i) acc += *((volatile float*)&p.refpart[i]);
+        last = atomicAdd(&p.done[g.b], 1) == nslots - 1;
+      }
+      if (__shfl_sync(0xffffffffu, last, 0)) {
+        // the sample's last partial: ref2 = (sum of the partials) / (R M),
+        // lane l taking slots l, l + 32, ... in order, then a fixed tree
+        __threadfence();
+        const int s0 = p.slot_off[g.b], s1 = p.slot_off[g.b + 1];
+        float acc = 0.f;
+        for (int i = s0 + lane; i < s1; i += 32) acc += __ldcg(&p.refpart[i]);
+        acc = warp_sum_f(acc);
+        if (lane == 0) {
           const int R = p.bt.reg_off[p.bt.seg_first[g.b + 1]] - p.bt.reg_off[p.bt.seg_first[g.b]];
           const float r2 = (R > 0 && g.M > 0) ? acc / ((float)R * (float)g.M) : 0.f;
           p.ref2[g.b] = r2;
