@@ -11,7 +11,7 @@ constexpr int kFusedCluster = 4;        // CTAs per cluster of the fused tcgen05
 constexpr int kFusedMaxOwnImg = 192;    // S1 keys one of its CTAs can hold (P columns kept in registers)
 constexpr int kFusedKeyRows4 = 256;     // key rows per head one CTA of a 4-CTA cluster holds (= MMA N and TMEM columns)
 constexpr int kFusedKeyRows8 = 224;     // the same for an 8-CTA cluster (its exchange buffers take more shared memory)
-constexpr int kFusedEpiWarps = 8;       // epilogue warps per CTA of the fused kernel
+constexpr int kFusedPartialWarps = 4;   // warps per CTA of the fused kernel that write an s2(r) partial
 constexpr int kFinalizeSmemRows = 1400; // Stage-I finalize stages a [CLS] segment in shared memory up to this many rows
 
 // Whether a sample with n1 S1 keys and M text tokens fits the fused kernel
@@ -24,8 +24,8 @@ __host__ __device__ inline bool fused_fits(int C, int n1, int M, int H) {
   const int tp = ((M + C - 1) / C + 15) & ~15;
   return M > 0 && H >= 4 && ip <= kFusedMaxOwnImg && ip + tp <= rows;
 }
-constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedEpiWarps;  // s2(r) partials per C=4 item (one per epilogue warp)
-constexpr int kFusedSlotsPerItem8 = 8 * kFusedEpiWarps;             // and per C=8 item
+constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedPartialWarps;  // s2(r) partials per C=4 item
+constexpr int kFusedSlotsPerItem8 = 8 * kFusedPartialWarps;             // and per C=8 item
 
 struct Stage1ClsParams {
   BatchDev bt;

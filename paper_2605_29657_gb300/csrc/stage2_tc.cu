@@ -44,43 +44,49 @@ namespace occam {
 namespace s2f {
 constexpr int QR = 128;                // text rows per item (TMEM lanes)
 constexpr int PMAX = kFusedMaxOwnImg;  // max S1 keys per CTA
-constexpr int NPW = PMAX / 64;         // S1-key pieces per epilogue warp
+constexpr int NPC = PMAX / 32;         // S1-key pieces (32 columns each) per CTA
 constexpr int QBYTES = QR * 256;       // one head's query tile: 2 K-blocks x 128 rows x 128 B
-constexpr int NPROD = 7;               // producer warps (0-6); warp 7 issues MMAs; then the epilogue warps
+constexpr int NPROD = 7;               // producer warps (0-6); warp 7 issues MMAs
 constexpr int MMA_WARP = NPROD;
-constexpr int EPI_WARP0 = NPROD + 1;
-constexpr int NEPI = kFusedEpiWarps;   // two per TMEM lane quadrant
-constexpr int THREADS = (NPROD + 1 + NEPI) * 32;
-constexpr int NXS = 2;                 // exchange slots (a peer runs at most one head ahead of a slot's reader)
+constexpr int S_WARP0 = NPROD + 1;     // warpgroup 2: statistics warps, one per TMEM lane quadrant
+constexpr int P_WARP0 = S_WARP0 + 4;   // warpgroup 3: probability warps, one per TMEM lane quadrant
+constexpr int NPW = kFusedPartialWarps;
+constexpr int THREADS = (P_WARP0 + NPW) * 32;
+// exchange slots: a peer posts head h + 4 into a slot only after this CTA's
+// probability warps finished head h (the chain runs through both CTAs' E buffers)
+constexpr int NXS = 4;
 // register split: warpgroups 0-1 (producers + MMA issuer) shrink to REG_LOW
-// per thread, the two epilogue warpgroups grow to REG_HIGH; the sum must stay
-// within what the CTA was launched with (checked on the host before launch)
-constexpr int REG_LOW = 56, REG_HIGH = 200;
-constexpr int REG_NEEDED = EPI_WARP0 * 32 * REG_LOW + NEPI * 32 * REG_HIGH;
-static_assert(EPI_WARP0 % 4 == 0 && NEPI % 4 == 0, "roles split on warpgroup boundaries");
+// per thread, the statistics warps take REG_S, the probability warps (which
+// keep P in registers) REG_P; the sum must stay within what the CTA was
+// launched with (checked on the host before launch)
+constexpr int REG_LOW = 56, REG_S = 144, REG_P = 256;
+constexpr int REG_NEEDED = S_WARP0 * 32 * REG_LOW + 4 * 32 * REG_S + NPW * 32 * REG_P;
+static_assert(S_WARP0 % 4 == 0 && NPW == 4, "roles split on warpgroup boundaries");
+static_assert(REG_NEEDED <= 65536, "register split exceeds the register file");
 constexpr uint32_t TMEM_COLS = 512;
 static_assert(2 * kFusedKeyRows4 <= (int)TMEM_COLS && 2 * kFusedKeyRows8 <= (int)TMEM_COLS, "two E buffers");
 static_assert(kFusedKeyRows4 % 32 == 0 && kFusedKeyRows8 % 32 == 0 && kFusedKeyRows4 <= 256, "MMA N <= 256");
-static_assert(PMAX % 64 == 0, "S1-key pieces split evenly between the two warps of a quadrant");
+static_assert(PMAX % 32 == 0, "S1 keys in whole pieces");
 constexpr uint64_t kLimitNs = 2000000000ull;
 
 template <int C>
 struct Geo {
   static constexpr int KROWS = C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;  // key rows per head (max MMA N)
   static constexpr int KBLK = KROWS * 128;                                  // bytes of one K-block of the key rows
-  static constexpr uint32_t XBYTES = C * NEPI * 32 * 8;                     // exchange bytes a CTA receives per head
+  static constexpr uint32_t XBYTES = C * QR * 8;                            // exchange bytes a CTA receives per head
 };
 
 template <int C>
 struct Smem {
   uint8_t q[2][QBYTES];
   uint8_t k[2][2 * Geo<C>::KBLK];
-  float2 xch[NXS][C][2][QR];  // (max, sum) per (slot, CTA, epilogue half, row)
+  float2 xch[NXS][C][QR];    // (max, sum) per (slot, CTA, row)
+  float cmx[2][NPC][QR];     // per E buffer: the row max of each S1-key piece its exponentials are relative to
   int32_t kidx[2][PMAX];
   uint8_t kreg[2][PMAX];
   int32_t next_item[4];  // work item of the cluster's ii-th turn, by ii & 3
-  uint64_t kfull[2], kempty[2], qfull[2], qempty[2], efull[2], efree[2], xbar[NXS], iready[2], idone[2], inext[4],
-      mdone;
+  uint64_t kfull[2], kempty[2], qfull[2], qempty[2], efull[2], sdone[2], efree[2], xbar[NXS], iready[2], idone[2],
+      inext[4], mdone;
   uint32_t tmem_base;
   int abort;
   uint32_t issued_q;
@@ -176,14 +182,19 @@ __device__ __forceinline__ void ld_wait(uint32_t (&v)[32]) {
   reg_fence(v);
 }
 
+__device__ __forceinline__ void ld_wait64(uint32_t (&v)[64]) {
+  tc::tmem_wait_ld();
+  asm volatile("" : OCCAM_TC_RW64(v));
+}
+
 // Statistics of one thread's row over a 32-column piece of logits already
 // loaded into v (warp-collective): cm = max of the first `lim` columns in
 // log2 units (-inf if none), a = sum over them of exp2(l * sl2 - cm). v is
-// overwritten with the exponentials (0 past lim); with STORE they are also
-// written back to TMEM at sa (the caller waits for that store before the
-// values are read again).
-template <bool STORE>
-__device__ __forceinline__ void piece_stats(uint32_t (&v)[32], uint32_t sa, int lim, float sl2, float& cm, float& a) {
+// overwritten with the exponentials (0 past lim); with `store` (warp-uniform)
+// they are also written back to TMEM at sa (the caller waits for that store
+// before another thread reads them).
+__device__ __forceinline__ void piece_stats(uint32_t (&v)[32], uint32_t sa, int lim, float sl2, bool store, float& cm,
+                                            float& a) {
   if (!__all_sync(0xffffffffu, lim >= 32)) {
     // partial piece (causal text keys, the last S1 piece, padded rows):
     // masked logits become -inf, whose exponential is exactly 0
@@ -212,7 +223,52 @@ __device__ __forceinline__ void piece_stats(uint32_t (&v)[32], uint32_t sa, int 
     v[2 * i + 1] = __float_as_uint(x.y);
   }
   a = ((acc[0].x + acc[0].y) + (acc[1].x + acc[1].y)) + ((acc[2].x + acc[2].y) + (acc[3].x + acc[3].y));
-  if (STORE) tc::tmem_st32(sa, v);
+  if (store) tc::tmem_st32(sa, v);
+}
+
+// Statistics of one thread's row over 64 columns (two pieces) that are all
+// valid S1 keys: cm = their max in log2 units, a = sum of exp2(l * sl2 - cm);
+// the exponentials are written back to TMEM at sa. No masking and no
+// branches, so the two pieces' dependency chains interleave.
+__device__ __forceinline__ void group_stats(uint32_t (&v)[64], uint32_t sa, float sl2, float& cm, float& a) {
+  float t[22];
+#pragma unroll
+  for (int i = 0; i < 21; ++i)
+    t[i] = tc::fmax3(__uint_as_float(v[3 * i]), __uint_as_float(v[3 * i + 1]), __uint_as_float(v[3 * i + 2]));
+  t[21] = __uint_as_float(v[63]);
+  float u[8];
+#pragma unroll
+  for (int i = 0; i < 7; ++i) u[i] = tc::fmax3(t[3 * i], t[3 * i + 1], t[3 * i + 2]);
+  u[7] = t[21];
+  const float mx = fmaxf(tc::fmax3(u[0], u[1], u[2]), tc::fmax3(u[3], u[4], fmaxf(u[5], fmaxf(u[6], u[7]))));
+  cm = mx * sl2;
+  const float2 sc = make_float2(sl2, sl2);
+  const float2 off = make_float2(-cm, -cm);
+  float2 acc[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) acc[i] = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), sc, off);
+    x.x = tc::ex2(x.x);
+    x.y = tc::ex2(x.y);
+    acc[i & 7] = __fadd2_rn(acc[i & 7], x);
+    v[2 * i] = __float_as_uint(x.x);
+    v[2 * i + 1] = __float_as_uint(x.y);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) acc[i] = __fadd2_rn(acc[i], acc[i + 4]);
+  acc[0] = __fadd2_rn(__fadd2_rn(acc[0], acc[2]), __fadd2_rn(acc[1], acc[3]));
+  a = acc[0].x + acc[0].y;
+  tc::tmem_st64(sa, v);
+}
+
+// merges a finite piece maximum cm (with its sum a) into the running (m, z)
+__device__ __forceinline__ void merge_finite(float& m, float& z, float cm, float a) {
+  const bool up = cm > m;  // also when m is still -inf (then e = 0 and z = 0)
+  const float e = tc::ex2(up ? m - cm : cm - m);
+  z = up ? fmaf(z, e, a) : fmaf(a, e, z);
+  m = fmaxf(m, cm);
 }
 
 // merges a piece's (cm, a) into the row's running softmax (m, z), log2 units
@@ -259,9 +315,10 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       tc::bar_init(&sm.qfull[i], 1);
       tc::bar_init(&sm.qempty[i], 1);
       tc::bar_init(&sm.efull[i], 1);
-      tc::bar_init(&sm.efree[i], NEPI);
+      tc::bar_init(&sm.sdone[i], 4);
+      tc::bar_init(&sm.efree[i], NPW);
       tc::bar_init(&sm.iready[i], NPROD * 32);
-      tc::bar_init(&sm.idone[i], NEPI);
+      tc::bar_init(&sm.idone[i], NPW);
     }
     // one local arrival (with the expected byte count) plus the peers'
     // asynchronous stores complete each phase of an exchange slot
@@ -283,7 +340,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   const uint32_t tmem = sm.tmem_base;
   const int H = p.H;
 
-  if (warp < EPI_WARP0) {
+  if (warp < S_WARP0) {
     // warpgroups 0-1: producers and the MMA issuer give registers back
     tc::setmaxnreg_dec<REG_LOW>();
     if (warp < NPROD) {
@@ -401,18 +458,17 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       }
       __syncwarp();
     }
-  } else {
-    // warpgroups 2-3: the epilogue takes them
-    tc::setmaxnreg_inc<REG_HIGH>();
-    // ------------------------------------------------------------ epilogue
-    const int ew = warp - EPI_WARP0;    // 0..NEPI-1
-    const int half = ew >> 2;           // this warp owns the 32-column pieces of this parity
-    const int quad = warp & 3;          // TMEM lane quadrant this warp may access
-    const int j = quad * 32 + lane;     // text row of this thread inside the tile
+  } else if (warp < P_WARP0) {
+    // ------------------------------------------------------------ statistics warps
+    // warp (quad) owns text rows 32 quad .. 32 quad + 31 (its TMEM lane
+    // quadrant). Per head: every piece of E, S1 keys first, then the causal
+    // text keys; exponentials of the S1-key pieces go back into E with their
+    // piece maxima in cmx; the row's (max, sum) goes to the whole cluster.
+    tc::setmaxnreg_inc<REG_S>();
+    const int quad = warp & 3;
+    const int j = quad * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const float sl2 = p.scale_log2;
-    const float invH = 1.0f / (float)H;
-    const bool armer = ew == 0 && lane == 0;  // re-arms the exchange slots of this CTA
     uint32_t hk = 0;
     for (int ii = 0;; ++ii) {
       int item = 0;
@@ -420,183 +476,183 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       if (item >= nF) break;
       const ItemGeom g = item_geom<C>(p, p.items[item], rank);
       if (!g.fits) {
-        if (tid == EPI_WARP0 * 32) set_status(p.status, OCCAM_ERR_UNSUPPORTED);
+        if (tid == S_WARP0 * 32) set_status(p.status, OCCAM_ERR_UNSUPPORTED);
         continue;
       }
+      const bool vrow = g.j0 + j < g.M;
+      const int jj = g.j0 + j;
+      const int npi = g.ip >> 5;
+      // pieces this warp reads: all S1-key pieces, then the text-key pieces
+      // up to the causal limit of its last valid row
+      const int jl = min(g.j0 + quad * 32 + 31, g.M - 1);
+      const int ntc = max(0, min(g.own_txt, jl + 1 - g.txt0));
+      const int np = __any_sync(0xffffffffu, vrow) ? npi + ((ntc + 31) >> 5) : 0;
+      const int ngf = g.own_img >> 6;  // whole 64-column groups of S1 keys
+      bool ok = true;
+      for (int h = 0; h < H; ++h, ++hk) {
+        const int eb = hk & 1;
+        const uint32_t ebase = tmem + lane_base + eb * G::KROWS;
+        if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.efull[eb], (hk >> 1) & 1, nullptr, kLimitNs))) {
+          ok = false;
+          break;
+        }
+        tc::fence_after();
+        float m = -INFINITY, z = 0.f;
+        if (np > 0) {
+          // S1 keys in whole 64-column groups first (no masking), then the
+          // rest one 32-column piece at a time
+          for (int gi = 0; gi < ngf; ++gi) {
+            uint32_t v[64];
+            tc::tmem_ld64(ebase + gi * 64, v);
+            ld_wait64(v);
+            float cm, a;
+            group_stats(v, ebase + gi * 64, sl2, cm, a);
+            sm.cmx[eb][2 * gi][j] = cm;
+            sm.cmx[eb][2 * gi + 1][j] = cm;
+            merge_finite(m, z, cm, a);
+          }
+          for (int k = 2 * ngf; k < np; ++k) {
+            uint32_t v[32];
+            tc::tmem_ld32(ebase + k * 32, v);
+            ld_wait(v);
+            const bool img = k < npi;
+            const int lim = !vrow ? 0 : img ? g.own_img - k * 32 : min(g.own_txt - (k * 32 - g.ip), jj - (g.txt0 + k * 32 - g.ip) + 1);
+            float cm, a;
+            piece_stats(v, ebase + k * 32, lim, sl2, img, cm, a);
+            if (img) sm.cmx[eb][k][j] = cm;
+            online_merge(m, z, cm, a);
+          }
+          tc::tmem_wait_st();
+        }
+        tc::fence_before();
+        // post this head's (max, sum) to the probability warps of every CTA of the cluster
+        const int slot = hk & (NXS - 1);
+#pragma unroll
+        for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][j], &sm.xbar[slot], (uint32_t)r, m, z);
+        __syncwarp();
+        if (lane == 0) tc::bar_arrive(&sm.sdone[eb]);
+      }
+      if (!ok) { fail(sm, p.status); break; }
+    }
+  } else {
+    // ------------------------------------------------------------ probability warps
+    // warp (quad) keeps P for text rows 32 quad .. 32 quad + 31 over all of
+    // this CTA's S1 keys in registers. Per head, once the statistics warps
+    // are done with it and the cluster's (max, sum) pairs are in: P +=
+    // exp2(cmx - max) / sum * E over the S1-key pieces; then E is released.
+    tc::setmaxnreg_inc<REG_P>();
+    const int pw = warp - P_WARP0;
+    const int quad = warp & 3;
+    const int j = quad * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    const float invH = 1.0f / (float)H;
+    const bool armer = pw == 0 && lane == 0;  // re-arms the exchange slots of this CTA
+    uint32_t hk = 0;
+    for (int ii = 0;; ++ii) {
+      int item = 0;
+      if (!__all_sync(0xffffffffu, take_item(sm, ii, nullptr, item))) { fail(sm, p.status); break; }
+      if (item >= nF) break;
+      const ItemGeom g = item_geom<C>(p, p.items[item], rank);
+      if (!g.fits) continue;
       const int ib = ii & 1;
       if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, nullptr, kLimitNs))) { fail(sm, p.status); break; }
       const bool vrow = g.j0 + j < g.M;
       const bool wvalid = __any_sync(0xffffffffu, vrow);  // warp-uniform: any real text row here
-      const int jj = g.j0 + j;
-      const int npi = g.ip >> 5;                // S1-key pieces of this CTA
-      const int npc = (g.N + 31) >> 5;          // all pieces
-      bool own[NPW];                            // which of this warp's S1-key pieces exist
+      const int npi = g.ip >> 5;
+      float P[NPC][32];
 #pragma unroll
-      for (int q = 0; q < NPW; ++q) own[q] = 2 * q + half < npi;
-      float P[NPW][32];
-#pragma unroll
-      for (int q = 0; q < NPW; ++q)
+      for (int q = 0; q < NPC; ++q)
 #pragma unroll
         for (int b2 = 0; b2 < 32; ++b2) P[q][b2] = 0.f;
-      float cmx[NPW];  // piece maxima of the last head whose statistics were taken
-#pragma unroll
-      for (int q = 0; q < NPW; ++q) cmx[q] = -INFINITY;
       bool ok = true;
-      for (int step = 0; step <= H && ok; ++step) {
-        const uint32_t hcur = hk + step;  // global index of head `step` of this item
-        const int eb = hcur & 1;
-        const uint32_t ebase = tmem + lane_base + eb * G::KROWS;
-        float m = -INFINITY, z = 0.f;
-        if (step < H) {
-          // ---- text-key pieces of head `step`
-          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.efull[eb], (hcur >> 1) & 1, nullptr, kLimitNs))) {
-            ok = false;
-          } else if (wvalid) {
-            tc::fence_after();
-            for (int pc = npi + ((npi ^ half) & 1); pc < npc; pc += 2) {
-              const int tb = g.txt0 + pc * 32 - g.ip;  // sample-relative text index of the piece's column 0
-              const int lim = vrow ? min(g.own_txt - (pc * 32 - g.ip), jj - tb + 1) : 0;
-              if (__all_sync(0xffffffffu, lim <= 0)) continue;
+      for (int h = 0; h < H; ++h, ++hk) {
+        const int eb = hk & 1;
+        const int slot = hk & (NXS - 1);
+        if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sdone[eb], (hk >> 1) & 1, nullptr, kLimitNs))) {
+          ok = false;
+          break;
+        }
+        if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (hk / NXS) & 1, nullptr, kLimitNs, true))) {
+          ok = false;
+          break;
+        }
+        tc::fence_after();
+        if (wvalid) {
+          float Mx = -INFINITY;
+#pragma unroll
+          for (int r = 0; r < C; ++r) Mx = fmaxf(Mx, sm.xch[slot][r][j].x);
+          float Z = 0.f;
+#pragma unroll
+          for (int r = 0; r < C; ++r) {
+            const float2 e = sm.xch[slot][r][j];
+            if (e.y > 0.f) Z = fmaf(e.y, tc::ex2(e.x - Mx), Z);
+          }
+          // Z >= 1 (the row max contributes exp2(0)); hardware reciprocal
+          const float invZ = (vrow && Z > 0.f) ? tc::rcp(Z) : 0.f;
+          const uint32_t pbase = tmem + lane_base + eb * G::KROWS;
+#pragma unroll
+          for (int q = 0; q < NPC; ++q) {
+            if (q < npi) {
+              const float cm = sm.cmx[eb][q][j];
+              const float f = (invZ > 0.f && cm != -INFINITY) ? tc::ex2(cm - Mx) * invZ : 0.f;
               uint32_t v[32];
-              tc::tmem_ld32(ebase + pc * 32, v);
+              tc::tmem_ld32(pbase + 32 * q, v);
               ld_wait(v);
-              float cm, a;
-              piece_stats<false>(v, 0, lim, sl2, cm, a);
-              online_merge(m, z, cm, a);
+              p_accum(P[q], v, f);
             }
           }
         }
-        if (ok && step >= 1) {
-          // ---- probabilities of head step-1 over this warp's S1-key pieces, added into P
-          const uint32_t hp = hcur - 1;
-          const int slot = hp & (NXS - 1);
-          const int pb = hp & 1;
-          const uint32_t pbase = tmem + lane_base + pb * G::KROWS + half * 32;
-          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.xbar[slot], (hp / NXS) & 1, nullptr, kLimitNs, true))) {
-            ok = false;
-          } else {
-            if (wvalid) {
-              float Mx = -INFINITY;
-#pragma unroll
-              for (int r = 0; r < C; ++r) Mx = tc::fmax3(Mx, sm.xch[slot][r][0][j].x, sm.xch[slot][r][1][j].x);
-              float Z = 0.f;
-#pragma unroll
-              for (int r = 0; r < C; ++r)
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                  const float2 e = sm.xch[slot][r][hh][j];
-                  if (e.y > 0.f) Z = fmaf(e.y, tc::ex2(e.x - Mx), Z);
-                }
-              // Z >= 1 (the row max contributes exp2(0)); hardware reciprocal
-              const float invZ = (vrow && Z > 0.f) ? tc::rcp(Z) : 0.f;
-              float f[NPW];
-#pragma unroll
-              for (int q = 0; q < NPW; ++q) f[q] = (invZ > 0.f && cmx[q] != -INFINITY) ? tc::ex2(cmx[q] - Mx) * invZ : 0.f;
-              tc::fence_after();
-#pragma unroll
-              for (int q = 0; q < NPW; ++q) {
-                if (own[q]) {
-                  uint32_t v[32];
-                  tc::tmem_ld32(pbase + 64 * q, v);
-                  ld_wait(v);
-                  p_accum(P[q], v, f[q]);
-                }
-              }
-            }
-            tc::fence_before();
-            __syncwarp();
-            if (lane == 0) tc::bar_arrive(&sm.efree[pb]);
-            // the slot's phase for head hp is complete: arm it for head hp + NXS
-            if (armer) tc::bar_expect_tx(&sm.xbar[slot], G::XBYTES);
-          }
-        }
-        if (ok && step < H) {
-          // ---- S1-key pieces of head `step` (written back as exponentials), then the exchange
-          if (wvalid) {
-            const uint32_t ibase = ebase + half * 32;
-            int lim[NPW];
-            bool live[NPW];
-#pragma unroll
-            for (int q = 0; q < NPW; ++q) {
-              lim[q] = vrow ? g.own_img - (2 * q + half) * 32 : 0;
-              live[q] = own[q] && !__all_sync(0xffffffffu, lim[q] <= 0);
-              cmx[q] = -INFINITY;
-            }
-            float a;
-#pragma unroll
-            for (int q = 0; q < NPW; ++q) {
-              if (live[q]) {
-                uint32_t v[32];
-                tc::tmem_ld32(ibase + 64 * q, v);
-                ld_wait(v);
-                piece_stats<true>(v, ibase + 64 * q, lim[q], sl2, cmx[q], a);
-                online_merge(m, z, cmx[q], a);
-              }
-            }
-            tc::tmem_wait_st();
-          } else {
-#pragma unroll
-            for (int q = 0; q < NPW; ++q) cmx[q] = -INFINITY;
-          }
-          tc::fence_before();
-          // ---- post this head's (max, sum) to every epilogue warp of the cluster
-          const int slot = hcur & (NXS - 1);
-#pragma unroll
-          for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][half][j], &sm.xbar[slot], (uint32_t)r, m, z);
-        }
+        tc::fence_before();
+        __syncwarp();
+        if (lane == 0) tc::bar_arrive(&sm.efree[eb]);
+        // the slot's phase for head hk is complete: arm it for head hk + NXS
+        if (armer) tc::bar_expect_tx(&sm.xbar[slot], G::XBYTES);
       }
-      hk += H;
       if (!ok) { fail(sm, p.status); break; }
       // ---- column reductions of P over this warp's 32 rows: column max ->
       // s2 (atomicMax), register columns -> this warp's partial of s2(r)
       float regacc = 0.f;
       if (wvalid) {
 #pragma unroll
-        for (int q = 0; q < NPW; ++q) {
-          if (own[q]) {
-            // transpose-reduce over the 32 rows of this warp: afterwards lane l
-            // holds the max (and, where a register key is among the columns,
-            // the sum) of this warp's column l of piece q -- 31 shuffles each
-            const int key = (2 * q + half) * 32 + lane;
+        for (int q = 0; q < NPC; ++q) {
+          if (q < npi) {
+            const int key = q * 32 + lane;
             const bool live = key < g.own_img;
             const bool is_reg = live && sm.kreg[ib][key];
-            float t[32];
+            const uint32_t regmask = __ballot_sync(0xffffffffu, is_reg);
+            // register columns first (few): a warp sum over the rows of each
+            float rc = 0.f;
+            if (regmask) {
 #pragma unroll
-            for (int col = 0; col < 32; ++col) t[col] = vrow ? P[q][col] : 0.f;
+              for (int col = 0; col < 32; ++col) {
+                if (regmask & (1u << col)) {
+                  const float sum = warp_sum_f(vrow ? P[q][col] : 0.f);
+                  if (lane == col) rc = sum * invH;
+                }
+              }
+            }
+            regacc += warp_sum_f(rc);
+            // then the column max, transposed in place: afterwards lane l
+            // holds the max of this warp's column l of piece q (31 shuffles)
+#pragma unroll
+            for (int col = 0; col < 32; ++col) P[q][col] = vrow ? P[q][col] : 0.f;
 #pragma unroll
             for (int sft = 16; sft >= 1; sft >>= 1) {
               const bool up = (lane & sft) != 0;
 #pragma unroll
               for (int i = 0; i < sft; ++i) {
-                const float send = up ? t[i] : t[i + sft];
-                const float keep = up ? t[i + sft] : t[i];
-                t[i] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, sft));
+                const float send = up ? P[q][i] : P[q][i + sft];
+                const float keep = up ? P[q][i + sft] : P[q][i];
+                P[q][i] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, sft));
               }
             }
-            if (live && !is_reg) atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(t[0] * invH));
-            float rc = 0.f;
-            if (__any_sync(0xffffffffu, is_reg)) {
-#pragma unroll
-              for (int col = 0; col < 32; ++col) t[col] = vrow ? P[q][col] : 0.f;
-#pragma unroll
-              for (int sft = 16; sft >= 1; sft >>= 1) {
-                const bool up = (lane & sft) != 0;
-#pragma unroll
-                for (int i = 0; i < sft; ++i) {
-                  const float send = up ? t[i] : t[i + sft];
-                  const float keep = up ? t[i + sft] : t[i];
-                  t[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
-                }
-              }
-              if (is_reg) rc = t[0] * invH;
-            }
-            regacc += warp_sum_f(rc);
+            if (live && !is_reg) atomicMax(reinterpret_cast<int*>(&p.s2[sm.kidx[ib][key]]), __float_as_int(P[q][0] * invH));
           }
         }
       }
       int last = 0;
       if (lane == 0) {
-        p.refpart[g.slot + rank * NEPI + ew] = regacc;  // C * NEPI slots per item
+        p.refpart[g.slot + rank * NPW + pw] = regacc;  // C * NPW slots per item
         __threadfence();
         const int nslots = p.slot_off[g.b + 1] - p.slot_off[g.b];
         last = atomicAdd(&p.done[g.b], 1) == nslots - 1;
