@@ -397,6 +397,10 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     const int64_t cols = (int64_t)a->H2 * 128;
     const void* kt = a->K_text ? a->K_text : a->Q_text;
     if (!encode_map(&mq, a->Q_text, b->total_text, cols, 128)) return OCCAM_ERR_CUDA;
+    // key rows are gathered four at a time (TMA gather4: box one row high)
+    CUtensorMap mk, mkt;
+    if (!encode_map(&mk, a->K2, b->total_rows, cols, 1)) return OCCAM_ERR_CUDA;
+    if (!encode_map(&mkt, kt, b->total_text, cols, 1)) return OCCAM_ERR_CUDA;
     Stage2TcParams q;
     q.bt = p.bt;
     q.H = a->H2;
@@ -429,13 +433,13 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     q8.items = p.itemsF8;
     q8.queue = p.counters + CNT_QUEUE8;
     const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
-    if (launch_fused(8, mq, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
+    if (launch_fused(8, mq, mk, mkt, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
     // the two-pass kernels (samples the fused kernel cannot hold; often none)
     // follow the 8-CTA launch on the second stream
     launch_twopass(p, L, sms, side.stream);
     q.queue = p.counters + CNT_QUEUE4;
     const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
-    if (launch_fused(4, mq, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
+    if (launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
     OCCAM_CUDA(cudaEventRecord(side.join, side.stream));
     OCCAM_CUDA(cudaStreamWaitEvent(st, side.join, 0));
     trace.mark(st);

@@ -197,7 +197,8 @@ int s2_scores_smem_bytes();
 int s2_stats_smem_bytes();
 
 // stage2_tc.cu
-int launch_fused(int C, const CUtensorMap& mq, const Stage2TcParams& q, int nclusters, cudaStream_t st);
+int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt, const Stage2TcParams& q,
+                 int nclusters, cudaStream_t st);
 int s2_fused_smem_bytes(int C);
 int s2_fused_threads();
 

@@ -46,22 +46,22 @@ constexpr int QR = 128;                // text rows per item (TMEM lanes)
 constexpr int PMAX = kFusedMaxOwnImg;  // max S1 keys per CTA
 constexpr int NPC = PMAX / 32;         // S1-key pieces (32 columns each) per CTA
 constexpr int QBYTES = QR * 256;       // one head's query tile: 2 K-blocks x 128 rows x 128 B
-constexpr int NPROD = 7;               // producer warps (0-6); warp 7 issues MMAs
+constexpr int NPROD = 3;               // producer warps (0-2): TMA gathers; warp 3 issues MMAs
 constexpr int MMA_WARP = NPROD;
-constexpr int S_WARP0 = NPROD + 1;     // warpgroup 2: statistics warps, one per TMEM lane quadrant
-constexpr int P_WARP0 = S_WARP0 + 4;   // warpgroup 3: probability warps, one per TMEM lane quadrant
+constexpr int S_WARP0 = NPROD + 1;     // warpgroups 1-2: statistics warps, two per TMEM lane quadrant
+constexpr int P_WARP0 = S_WARP0 + 8;   // warpgroup 3: probability warps, one per TMEM lane quadrant
 constexpr int NPW = kFusedPartialWarps;
 constexpr int THREADS = (P_WARP0 + NPW) * 32;
 // exchange slots: a peer posts head h + 4 into a slot only after this CTA's
 // probability warps finished head h (the chain runs through both CTAs' E buffers)
 constexpr int NXS = 4;
-// register split: warpgroups 0-1 (producers + MMA issuer) shrink to REG_LOW
-// per thread, the statistics warps take REG_S, the probability warps (which
-// keep P in registers) REG_P; the sum must stay within what the CTA was
+// register split: warpgroup 0 (producers + MMA issuer) shrinks to REG_LOW per
+// thread, the statistics warps to REG_S, the probability warps (which keep P
+// in registers) grow to REG_P; the sum must stay within what the CTA was
 // launched with (checked on the host before launch)
-constexpr int REG_LOW = 56, REG_S = 144, REG_P = 256;
-constexpr int REG_NEEDED = S_WARP0 * 32 * REG_LOW + 4 * 32 * REG_S + NPW * 32 * REG_P;
-static_assert(S_WARP0 % 4 == 0 && NPW == 4, "roles split on warpgroup boundaries");
+constexpr int REG_LOW = 56, REG_S = 104, REG_P = 248;
+constexpr int REG_NEEDED = S_WARP0 * 32 * REG_LOW + 8 * 32 * REG_S + NPW * 32 * REG_P;
+static_assert(S_WARP0 % 4 == 0 && P_WARP0 % 4 == 0 && NPW == 4, "roles split on warpgroup boundaries");
 static_assert(REG_NEEDED <= 65536, "register split exceeds the register file");
 constexpr uint32_t TMEM_COLS = 512;
 static_assert(2 * kFusedKeyRows4 <= (int)TMEM_COLS && 2 * kFusedKeyRows8 <= (int)TMEM_COLS, "two E buffers");
@@ -82,11 +82,12 @@ struct Smem {
   uint8_t k[2][2 * Geo<C>::KBLK];
   float2 xch[NXS][C][QR];    // (max, sum) per (slot, CTA, row)
   float cmx[2][NPC][QR];     // per E buffer: the row max of each S1-key piece its exponentials are relative to
+  float2 spart[2][4][32];    // per E buffer and lane quadrant: the second statistics warp's (max, sum)
   int32_t kidx[2][PMAX];
   uint8_t kreg[2][PMAX];
   int32_t next_item[4];  // work item of the cluster's ii-th turn, by ii & 3
   uint64_t kfull[2], kempty[2], qfull[2], qempty[2], efull[2], sdone[2], efree[2], xbar[NXS], iready[2], idone[2],
-      inext[4], mdone;
+      inext[4], spb[2][4], mdone;
   uint32_t tmem_base;
   int abort;
   uint32_t issued_q;
@@ -298,7 +299,8 @@ __device__ __forceinline__ void p_accum(float (&P)[32], const uint32_t (&v)[32],
 
 template <int C>
 __global__ void __launch_bounds__(s2f::THREADS, 1)
-    s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, Stage2TcParams p) {
+    s2_fused_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
+                    const __grid_constant__ CUtensorMap mapKt, Stage2TcParams p) {
   using namespace s2f;
   using G = Geo<C>;
   extern __shared__ unsigned char smem_raw[];
@@ -315,7 +317,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       tc::bar_init(&sm.qfull[i], 1);
       tc::bar_init(&sm.qempty[i], 1);
       tc::bar_init(&sm.efull[i], 1);
-      tc::bar_init(&sm.sdone[i], 4);
+      tc::bar_init(&sm.sdone[i], 8);
       tc::bar_init(&sm.efree[i], NPW);
       tc::bar_init(&sm.iready[i], NPROD * 32);
       tc::bar_init(&sm.idone[i], NPW);
@@ -324,12 +326,15 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     // asynchronous stores complete each phase of an exchange slot
     for (int i = 0; i < NXS; ++i) tc::bar_init(&sm.xbar[i], 1);
     for (int i = 0; i < 4; ++i) tc::bar_init(&sm.inext[i], 1);
+    for (int i = 0; i < 8; ++i) tc::bar_init(&sm.spb[i >> 2][i & 3], 1);
     tc::bar_init(&sm.mdone, 1);
     sm.abort = 0;
     sm.issued_q = 0;
     tc::bar_fence_init();
     for (int i = 0; i < NXS; ++i) tc::bar_expect_tx(&sm.xbar[i], G::XBYTES);
     tc::prefetch_map(&mapQ);
+    tc::prefetch_map(&mapK);
+    tc::prefetch_map(&mapKt);
   }
   if (warp == MMA_WARP) tc::tmem_alloc(&sm.tmem_base, TMEM_COLS);
   tc::fence_before();
@@ -351,7 +356,6 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       const int pt = tid;
       uint32_t qcnt = 0, kcnt = 0;
       int ii = 0;
-      const int64_t HD = (int64_t)H * 128;
       for (;; ++ii) {
         if (rank == 0 && pt == 0) hand_out_item<C>(sm, p.queue, ii);
         int item;
@@ -389,29 +393,38 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             }
           }
           ++qcnt;
+          // TMA gathers of the key block: unit u is four rows (u >> 1) of
+          // one K-block (u & 1); every producer thread arrives once per head,
+          // announcing the bytes of its own units before it issues them
+          const int nu = (g.N >> 2) * 2;
+          const int mine = nu > pt ? (nu - pt + NPROD * 32 - 1) / (NPROD * 32) : 0;
+          tc::bar_expect_tx(&sm.kfull[kb], (uint32_t)mine * 512u);
           uint8_t* dst = sm.k[kb];
-          const int nq = g.N * 16;
-          for (int q = pt; q < nq; q += NPROD * 32) {
-            const int row = q >> 4, c16 = q & 15;
-            const int kblk = c16 >> 3, cc = c16 & 7;
-            const __nv_bfloat16* src = p.K;
-            int bytes = 0;
-            if (row < g.own_img) {
-              src = p.K + (int64_t)sm.kidx[ib][row] * HD + h * 128 + c16 * 8;
-              bytes = 16;
-            } else if (row >= g.ip && row - g.ip < g.own_txt) {
-              src = p.Kt + (tbase + (row - g.ip)) * HD + h * 128 + c16 * 8;
-              bytes = 16;
+          for (int u = pt; u < nu; u += NPROD * 32) {
+            const int r0 = (u >> 1) * 4, kblk = u & 1;
+            int y[4];
+            const CUtensorMap* map;
+            if (r0 < g.ip) {
+              // S1 rows straight from K2 by index; padding rows repeat the first
+              map = &mapK;
+#pragma unroll
+              for (int i = 0; i < 4; ++i) y[i] = sm.kidx[ib][r0 + i < g.own_img ? r0 + i : 0];
+            } else {
+              map = &mapKt;
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const int t = r0 + i - g.ip;
+                y[i] = (int)(tbase + (t < g.own_txt ? t : 0));
+              }
             }
-            tc::cp_async16(dst + kblk * G::KBLK + row * 128 + ((cc ^ (row & 7)) << 4), src, bytes);
+            tc::tma_gather4(dst + kblk * G::KBLK + r0 * 128, map, h * 128 + kblk * 64, y[0], y[1], y[2], y[3],
+                            &sm.kfull[kb]);
           }
-          tc::cp_async_arrive(&sm.kfull[kb]);
           ++kcnt;
         }
         if (!ok) break;
       }
       if (pt == 0) sm.issued_q = qcnt;
-      asm volatile("cp.async.wait_all;" ::: "memory");
     } else {
       // ---------------------------------------------------------- MMA issuer
       if (lane == 0) {
@@ -460,12 +473,15 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     }
   } else if (warp < P_WARP0) {
     // ------------------------------------------------------------ statistics warps
-    // warp (quad) owns text rows 32 quad .. 32 quad + 31 (its TMEM lane
-    // quadrant). Per head: every piece of E, S1 keys first, then the causal
-    // text keys; exponentials of the S1-key pieces go back into E with their
-    // piece maxima in cmx; the row's (max, sum) goes to the whole cluster.
-    tc::setmaxnreg_inc<REG_S>();
+    // two warps per TMEM lane quadrant (text rows 32 quad .. 32 quad + 31)
+    // share every head's pieces of E: whole 64-column groups of S1 keys
+    // alternate between them, then the remaining pieces (the partial S1 piece
+    // and the causal text keys). Exponentials of S1 keys go back into E with
+    // their maxima in cmx; the second warp hands its (max, sum) to the first,
+    // which posts the row's statistics to the whole cluster.
+    tc::setmaxnreg_dec<REG_S>();
     const int quad = warp & 3;
+    const int half = (warp - S_WARP0) >> 2;
     const int j = quad * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const float sl2 = p.scale_log2;
@@ -482,12 +498,14 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       const bool vrow = g.j0 + j < g.M;
       const int jj = g.j0 + j;
       const int npi = g.ip >> 5;
-      // pieces this warp reads: all S1-key pieces, then the text-key pieces
+      // pieces of the quadrant: all S1-key pieces, then the text-key pieces
       // up to the causal limit of its last valid row
       const int jl = min(g.j0 + quad * 32 + 31, g.M - 1);
       const int ntc = max(0, min(g.own_txt, jl + 1 - g.txt0));
       const int np = __any_sync(0xffffffffu, vrow) ? npi + ((ntc + 31) >> 5) : 0;
-      const int ngf = g.own_img >> 6;  // whole 64-column groups of S1 keys
+      const int ngf = np > 0 ? g.own_img >> 6 : 0;  // whole 64-column groups of S1 keys
+      // the remaining pieces start with the warp that took fewer groups
+      const int k0 = 2 * ngf + ((half + ngf) & 1);
       bool ok = true;
       for (int h = 0; h < H; ++h, ++hk) {
         const int eb = hk & 1;
@@ -498,39 +516,50 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         }
         tc::fence_after();
         float m = -INFINITY, z = 0.f;
-        if (np > 0) {
-          // S1 keys in whole 64-column groups first (no masking), then the
-          // rest one 32-column piece at a time
-          for (int gi = 0; gi < ngf; ++gi) {
-            uint32_t v[64];
-            tc::tmem_ld64(ebase + gi * 64, v);
-            ld_wait64(v);
-            float cm, a;
-            group_stats(v, ebase + gi * 64, sl2, cm, a);
-            sm.cmx[eb][2 * gi][j] = cm;
-            sm.cmx[eb][2 * gi + 1][j] = cm;
-            merge_finite(m, z, cm, a);
-          }
-          for (int k = 2 * ngf; k < np; ++k) {
-            uint32_t v[32];
-            tc::tmem_ld32(ebase + k * 32, v);
-            ld_wait(v);
-            const bool img = k < npi;
-            const int lim = !vrow ? 0 : img ? g.own_img - k * 32 : min(g.own_txt - (k * 32 - g.ip), jj - (g.txt0 + k * 32 - g.ip) + 1);
-            float cm, a;
-            piece_stats(v, ebase + k * 32, lim, sl2, img, cm, a);
-            if (img) sm.cmx[eb][k][j] = cm;
-            online_merge(m, z, cm, a);
-          }
-          tc::tmem_wait_st();
+        for (int gi = half; gi < ngf; gi += 2) {
+          uint32_t v[64];
+          tc::tmem_ld64(ebase + gi * 64, v);
+          ld_wait64(v);
+          float cm, a;
+          group_stats(v, ebase + gi * 64, sl2, cm, a);
+          sm.cmx[eb][2 * gi][j] = cm;
+          sm.cmx[eb][2 * gi + 1][j] = cm;
+          merge_finite(m, z, cm, a);
         }
+        for (int k = k0; k < np; k += 2) {
+          uint32_t v[32];
+          tc::tmem_ld32(ebase + k * 32, v);
+          ld_wait(v);
+          const bool img = k < npi;
+          const int lim = !vrow ? 0 : img ? g.own_img - k * 32 : min(g.own_txt - (k * 32 - g.ip), jj - (g.txt0 + k * 32 - g.ip) + 1);
+          float cm, a;
+          piece_stats(v, ebase + k * 32, lim, sl2, img, cm, a);
+          if (img) sm.cmx[eb][k][j] = cm;
+          online_merge(m, z, cm, a);
+        }
+        tc::tmem_wait_st();
         tc::fence_before();
-        // post this head's (max, sum) to the probability warps of every CTA of the cluster
-        const int slot = hk & (NXS - 1);
-#pragma unroll
-        for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][j], &sm.xbar[slot], (uint32_t)r, m, z);
         __syncwarp();
         if (lane == 0) tc::bar_arrive(&sm.sdone[eb]);
+        if (half == 1) {
+          // hand this warp's (max, sum) to the quadrant's first warp
+          // (one buffer per E buffer: this warp reaches head hk + 2 only
+          // after the first warp posted head hk)
+          sm.spart[eb][quad][lane] = make_float2(m, z);
+          __syncwarp();
+          if (lane == 0) tc::bar_arrive(&sm.spb[eb][quad]);
+        } else {
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.spb[eb][quad], (hk >> 1) & 1, nullptr, kLimitNs))) {
+            ok = false;
+            break;
+          }
+          const float2 o = sm.spart[eb][quad][lane];
+          online_merge(m, z, o.x, o.y);
+          // post the row's (max, sum) to the probability warps of every CTA of the cluster
+          const int slot = hk & (NXS - 1);
+#pragma unroll
+          for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][j], &sm.xbar[slot], (uint32_t)r, m, z);
+        }
       }
       if (!ok) { fail(sm, p.status); break; }
     }
@@ -701,7 +730,8 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   tc::cluster_sync_all();
 }
 
-int launch_fused(int C, const CUtensorMap& mq, const Stage2TcParams& q, int nclusters, cudaStream_t st) {
+int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt, const Stage2TcParams& q,
+                 int nclusters, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(nclusters * C));
   cfg.blockDim = dim3(s2f::THREADS);
@@ -725,10 +755,10 @@ int launch_fused(int C, const CUtensorMap& mq, const Stage2TcParams& q, int nclu
   cudaError_t e;
   if (C == 8) {
     cudaFuncSetAttribute(s2_fused_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(8));
-    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<8>, mq, q);
+    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<8>, mq, mk, mkt, q);
   } else {
     cudaFuncSetAttribute(s2_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(4));
-    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<4>, mq, q);
+    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<4>, mq, mk, mkt, q);
   }
   return e == cudaSuccess ? 0 : 1;
 }
