@@ -337,6 +337,14 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     tc::prefetch_map(&mapKt);
   }
   if (warp == MMA_WARP) tc::tmem_alloc(&sm.tmem_base, TMEM_COLS);
+  {
+    // key buffers start zeroed: rows past a CTA's keys, which are never
+    // loaded, then hold finite values, whose logits the epilogue masks out
+    uint4* z4 = reinterpret_cast<uint4*>(&sm.k[0][0]);
+    constexpr int n16 = (int)(sizeof(sm.k) / 16);
+    for (int i = tid; i < n16; i += THREADS) z4[i] = make_uint4(0u, 0u, 0u, 0u);
+    tc::fence_proxy_async();
+  }
   tc::fence_before();
   __syncthreads();
   tc::fence_after();
@@ -394,28 +402,31 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
           }
           ++qcnt;
           // TMA gathers of the key block: unit u is four rows (u >> 1) of
-          // one K-block (u & 1); every producer thread arrives once per head,
-          // announcing the bytes of its own units before it issues them
-          const int nu = (g.N >> 2) * 2;
+          // one K-block (u & 1), over the CTA's S1 rows and then its text
+          // rows (rows past them are not loaded); every producer thread
+          // arrives once per head, announcing the bytes of its own units
+          // before it issues them
+          const int gi4 = (g.own_img + 3) >> 2, gt4 = (g.own_txt + 3) >> 2;
+          const int nu = (gi4 + gt4) * 2;
           const int mine = nu > pt ? (nu - pt + NPROD * 32 - 1) / (NPROD * 32) : 0;
           tc::bar_expect_tx(&sm.kfull[kb], (uint32_t)mine * 512u);
           uint8_t* dst = sm.k[kb];
           for (int u = pt; u < nu; u += NPROD * 32) {
-            const int r0 = (u >> 1) * 4, kblk = u & 1;
-            int y[4];
+            const int g4 = u >> 1, kblk = u & 1;
+            int y[4], r0;
             const CUtensorMap* map;
-            if (r0 < g.ip) {
-              // S1 rows straight from K2 by index; padding rows repeat the first
+            if (g4 < gi4) {
+              // S1 rows straight from K2 by index; rows past the CTA's keys repeat its first
+              r0 = g4 * 4;
               map = &mapK;
 #pragma unroll
               for (int i = 0; i < 4; ++i) y[i] = sm.kidx[ib][r0 + i < g.own_img ? r0 + i : 0];
             } else {
+              const int t0 = (g4 - gi4) * 4;
+              r0 = g.ip + t0;
               map = &mapKt;
 #pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                const int t = r0 + i - g.ip;
-                y[i] = (int)(tbase + (t < g.own_txt ? t : 0));
-              }
+              for (int i = 0; i < 4; ++i) y[i] = (int)(tbase + (t0 + i < g.own_txt ? t0 + i : 0));
             }
             tc::tma_gather4(dst + kblk * G::KBLK + r0 * 128, map, h * 128 + kblk * 64, y[0], y[1], y[2], y[3],
                             &sm.kfull[kb]);
