@@ -397,10 +397,11 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     const int64_t cols = (int64_t)a->H2 * 128;
     const void* kt = a->K_text ? a->K_text : a->Q_text;
     if (!encode_map(&mq, a->Q_text, b->total_text, cols, 128)) return OCCAM_ERR_CUDA;
-    // key rows are gathered four at a time (TMA gather4: box one row high)
+    // S1 key rows are gathered four at a time (TMA gather4: box one row
+    // high); text key rows, which are consecutive, come in boxes of 16 rows
     CUtensorMap mk, mkt;
     if (!encode_map(&mk, a->K2, b->total_rows, cols, 1)) return OCCAM_ERR_CUDA;
-    if (!encode_map(&mkt, kt, b->total_text, cols, 1)) return OCCAM_ERR_CUDA;
+    if (!encode_map(&mkt, kt, b->total_text, cols, 16)) return OCCAM_ERR_CUDA;
     Stage2TcParams q;
     q.bt = p.bt;
     q.H = a->H2;

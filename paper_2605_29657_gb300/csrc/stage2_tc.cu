@@ -46,6 +46,7 @@ constexpr int QR = 128;                // text rows per item (TMEM lanes)
 constexpr int PMAX = kFusedMaxOwnImg;  // max S1 keys per CTA
 constexpr int NPC = PMAX / 32;         // S1-key pieces (32 columns each) per CTA
 constexpr int QBYTES = QR * 256;       // one head's query tile: 2 K-blocks x 128 rows x 128 B
+constexpr int TXT_BOX = 16;            // text key rows per TMA box (the text-key padding unit)
 constexpr int NPROD = 3;               // producer warps (0-2): TMA gathers; warp 3 issues MMAs
 constexpr int MMA_WARP = NPROD;
 constexpr int S_WARP0 = NPROD + 1;     // warpgroups 1-2: statistics warps, two per TMEM lane quadrant
@@ -401,35 +402,34 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
             }
           }
           ++qcnt;
-          // TMA gathers of the key block: unit u is four rows (u >> 1) of
-          // one K-block (u & 1), over the CTA's S1 rows and then its text
-          // rows (rows past them are not loaded); every producer thread
-          // arrives once per head, announcing the bytes of its own units
-          // before it issues them
-          const int gi4 = (g.own_img + 3) >> 2, gt4 = (g.own_txt + 3) >> 2;
-          const int nu = (gi4 + gt4) * 2;
-          const int mine = nu > pt ? (nu - pt + NPROD * 32 - 1) / (NPROD * 32) : 0;
-          tc::bar_expect_tx(&sm.kfull[kb], (uint32_t)mine * 512u);
+          // The key block by TMA: S1 rows four at a time (gather4: unit u <
+          // 2 * gi4 is rows 4 (u >> 1) .. + 3 of K-block u & 1), then the
+          // text rows, which are consecutive, in boxes of TXT_BOX rows (rows
+          // past a CTA's keys up to the next four / box are loaded but
+          // masked; no other padding row is loaded). Every producer thread
+          // arrives once per head, announcing the bytes of its own copies
+          // before it issues them.
+          const int gi4 = (g.own_img + 3) >> 2, nbt = (g.own_txt + TXT_BOX - 1) / TXT_BOX;
+          const int nu = (gi4 + nbt) * 2;
+          uint32_t mine = 0;
+          for (int u = pt; u < nu; u += NPROD * 32) mine += u < 2 * gi4 ? 512u : (uint32_t)(TXT_BOX * 128);
+          tc::bar_expect_tx(&sm.kfull[kb], mine);
           uint8_t* dst = sm.k[kb];
           for (int u = pt; u < nu; u += NPROD * 32) {
-            const int g4 = u >> 1, kblk = u & 1;
-            int y[4], r0;
-            const CUtensorMap* map;
-            if (g4 < gi4) {
+            const int kblk = u & 1;
+            if (u < 2 * gi4) {
               // S1 rows straight from K2 by index; rows past the CTA's keys repeat its first
-              r0 = g4 * 4;
-              map = &mapK;
+              const int r0 = (u >> 1) * 4;
+              int y[4];
 #pragma unroll
               for (int i = 0; i < 4; ++i) y[i] = sm.kidx[ib][r0 + i < g.own_img ? r0 + i : 0];
+              tc::tma_gather4(dst + kblk * G::KBLK + r0 * 128, &mapK, h * 128 + kblk * 64, y[0], y[1], y[2], y[3],
+                              &sm.kfull[kb]);
             } else {
-              const int t0 = (g4 - gi4) * 4;
-              r0 = g.ip + t0;
-              map = &mapKt;
-#pragma unroll
-              for (int i = 0; i < 4; ++i) y[i] = (int)(tbase + (t0 + i < g.own_txt ? t0 + i : 0));
+              const int t0 = ((u >> 1) - gi4) * TXT_BOX;
+              tc::tma_load_2d(dst + kblk * G::KBLK + (g.ip + t0) * 128, &mapKt, h * 128 + kblk * 64, (int)(tbase + t0),
+                              &sm.kfull[kb]);
             }
-            tc::tma_gather4(dst + kblk * G::KBLK + r0 * 128, map, h * 128 + kblk * 64, y[0], y[1], y[2], y[3],
-                            &sm.kfull[kb]);
           }
           ++kcnt;
         }
