@@ -215,6 +215,31 @@ typedef struct occam_prune_out {
  * CUDA graph. */
 int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                 size_t workspace_bytes, occam_stream_t stream);
+/* Memory kinds (occam_prune and occam_prune_traced): q, k_cls, K1, Q_text,
+ * K_text and K2 must be device (or managed) memory, since they are read by
+ * TMA copies; gather sources and destinations may also be pinned host
+ * memory. Anything else returns OCCAM_ERR_INVALID_ARG. */
+
+/* occam_prune for inputs that stay in host memory (a GB300 host's memory is
+ * reachable from the GPU). The paper has no counterpart: this is the
+ * deployment path for callers whose K2 and gather tensors live on the host.
+ * Arguments are those of occam_prune, with two differences:
+ *   - args->stage2.K2 and the gather sources args->src[t] (and destinations
+ *     args->dst[t]) may be pinned host memory (cudaHostAlloc /
+ *     cudaHostRegister); pageable host memory is refused with
+ *     OCCAM_ERR_INVALID_ARG. The scoring inputs (q, k_cls, K1, Q_text,
+ *     K_text) must be device memory, as for occam_prune.
+ *   - k2_stage: device memory of at least total_rows * H2 * d2 * 2 bytes,
+ *     16-byte aligned, owned by the caller. After Stage I the call copies
+ *     the S1 rows of K2, and only those, into k2_stage at their own row
+ *     positions; Stage II then reads k2_stage. Its other rows are left as
+ *     they are.
+ * So only the S1 rows of K2 and the kept rows of the gather sources cross
+ * the host link, not whole tensors. Results are identical to occam_prune on
+ * the same values. In occam_prune_traced's event order the copy falls in the
+ * interval after the Stage-I finalize. */
+int occam_prune_staged(const occam_prune_args* args, const occam_prune_out* out, void* k2_stage,
+                       size_t k2_stage_bytes, void* workspace, size_t workspace_bytes, occam_stream_t stream);
 
 /* occam_prune that also records caller-created CUDA events (cudaEvent_t,
  * passed as void*) on `stream` between its steps, for per-kernel timing:

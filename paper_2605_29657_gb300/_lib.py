@@ -102,9 +102,11 @@ def library() -> ctypes.CDLL:
         lib.occam_prune.argtypes = [P(CPruneArgs), P(CPruneOut), _p, ctypes.c_size_t, _p]
         lib.occam_compact_noalloc.argtypes = [P(CBatch), _p, _i32, P(_p), P(_i64), P(_p), _i64, _p, _p, _p, _p]
         lib.occam_prune_traced.argtypes = [P(CPruneArgs), P(CPruneOut), _p, ctypes.c_size_t, _p, P(_p), _i32]
+        lib.occam_prune_staged.argtypes = [P(CPruneArgs), P(CPruneOut), _p, ctypes.c_size_t, _p, ctypes.c_size_t,
+                                           _p]
         for name in ("occam_workspace_size", "occam_get_status", "occam_score_stage1", "occam_threshold",
                      "occam_score_stage2", "occam_compact", "occam_prune", "occam_prune_traced",
-                     "occam_compact_noalloc"):
+                     "occam_compact_noalloc", "occam_prune_staged"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -129,6 +131,17 @@ def _dev_tensor(t: torch.Tensor, dtype, name: str) -> torch.Tensor:
     if not t.is_contiguous():
         raise OccamError(OCCAM_ERR_INVALID_ARG, f"{name} must be contiguous")
     return t
+
+
+def _host_or_dev_tensor(t: torch.Tensor, dtype, name: str) -> torch.Tensor:
+    """A CUDA tensor, or a pinned host tensor the device can read in place."""
+    if isinstance(t, torch.Tensor) and not t.is_cuda:
+        if not t.is_pinned():
+            raise OccamError(OCCAM_ERR_INVALID_ARG, f"{name} must be a CUDA tensor or pinned host memory")
+        if t.dtype != dtype or not t.is_contiguous():
+            raise OccamError(OCCAM_ERR_INVALID_ARG, f"{name} must be contiguous {dtype}")
+        return t
+    return _dev_tensor(t, dtype, name)
 
 
 def _stream(stream) -> int | None:
@@ -331,7 +344,10 @@ class PruneCall:
 
     def __init__(self, layout: BatchLayout, stage1: dict, stage2: dict, lambda1: float, lambda2: float,
                  keep_registers: bool = True, gather=(), capacity_rows: int | None = None,
-                 want=OPTIONAL, ws=None):
+                 want=OPTIONAL, ws=None, host_inputs: bool = False):
+        """host_inputs: K2 and the gather tensors may be pinned host tensors,
+        read in place through occam_prune_staged (S1 rows of K2 and kept rows
+        only); a device staging tensor for K2 is allocated here."""
         bf = torch.bfloat16
         mode = OCCAM_STAGE1_CLS if stage1.get("mode", "cls") == "cls" else OCCAM_STAGE1_MUTUAL
         q = _dev_tensor(stage1["q"], bf, "q")
@@ -340,7 +356,7 @@ class PruneCall:
         if k_cls is not None:
             _dev_tensor(k_cls, bf, "k_cls")
         Q_text = _dev_tensor(stage2["Q_text"], bf, "Q_text")
-        K2 = _dev_tensor(stage2["K2"], bf, "K2")
+        K2 = (_host_or_dev_tensor if host_inputs else _dev_tensor)(stage2["K2"], bf, "K2")
         K_text = stage2.get("K_text")
         if K_text is not None:
             _dev_tensor(K_text, bf, "K_text")
@@ -350,7 +366,9 @@ class PruneCall:
         self.layout = layout
         self.keep_alive = [q, K1, k_cls, Q_text, K2, K_text]
         cap = layout.total_rows if capacity_rows is None else int(capacity_rows)
-        gather = [_dev_tensor(t, t.dtype, f"gather{i}") for i, t in enumerate(gather)]
+        check = _host_or_dev_tensor if host_inputs else _dev_tensor
+        gather = [check(t, t.dtype, f"gather{i}") for i, t in enumerate(gather)]
+        self.k2_stage = torch.empty(K2.shape, dtype=bf, device=dev) if host_inputs else None
         self.gathered = [torch.empty((cap,) + tuple(t.shape[1:]), dtype=t.dtype, device=dev) for t in gather]
         self.keep_alive += gather
         R, B = layout.total_rows, layout.B
@@ -389,6 +407,13 @@ class PruneCall:
         self.capacity = cap
 
     def __call__(self, stream=None) -> dict:
+        if self.k2_stage is not None:
+            _check(library().occam_prune_staged(ctypes.byref(self.args), ctypes.byref(self.cout),
+                                                _ptr(self.k2_stage),
+                                                self.k2_stage.numel() * self.k2_stage.element_size(),
+                                                _ptr(self.ws), self.ws.numel(), _stream(stream)),
+                   "occam_prune_staged")
+            return self.out
         _check(library().occam_prune(ctypes.byref(self.args), ctypes.byref(self.cout), _ptr(self.ws),
                                      self.ws.numel(), _stream(stream)), "occam_prune")
         return self.out
@@ -397,6 +422,8 @@ class PruneCall:
 
     def traced(self, events, stream=None) -> dict:
         """As __call__, recording ``events`` (torch.cuda.Event, enable_timing) between the kernels."""
+        if self.k2_stage is not None:
+            raise OccamError(OCCAM_ERR_UNSUPPORTED, "traced calls take device inputs")
         arr = (_p * len(events))(*[e.cuda_event for e in events])
         _check(library().occam_prune_traced(ctypes.byref(self.args), ctypes.byref(self.cout), _ptr(self.ws),
                                             self.ws.numel(), _stream(stream), arr, len(events)),
@@ -409,9 +436,12 @@ class PruneCall:
 
 def occam_prune(layout: BatchLayout, stage1: dict, stage2: dict, lambda1: float, lambda2: float,
                 keep_registers: bool = True, gather=(), capacity_rows: int | None = None,
-                want=PruneCall.OPTIONAL, ws=None, stream=None) -> dict:
-    """One fused prune call; returns the output tensors and the gathered rows."""
-    call = PruneCall(layout, stage1, stage2, lambda1, lambda2, keep_registers, gather, capacity_rows, want, ws)
+                want=PruneCall.OPTIONAL, ws=None, stream=None, host_inputs: bool = False) -> dict:
+    """One fused prune call; returns the output tensors and the gathered rows.
+    With host_inputs, K2 and the gather tensors may be pinned host tensors
+    (occam_prune_staged)."""
+    call = PruneCall(layout, stage1, stage2, lambda1, lambda2, keep_registers, gather, capacity_rows, want, ws,
+                     host_inputs)
     out = dict(call(stream))
     out["gathered"] = call.gathered
     out["ws"] = call.ws

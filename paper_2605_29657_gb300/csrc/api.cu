@@ -241,6 +241,39 @@ int check_stage2(const occam_stage2_args* a) {
   return OCCAM_OK;
 }
 
+// Memory kinds: the TMA-read inputs must live in device (or managed) memory;
+// the K2 of a staged call and gather sources / destinations may also be
+// pinned host memory, which kernels reach through its device-side address.
+// Pageable (unregistered) host memory is refused: a kernel cannot be sure
+// to reach it.
+int require_device(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return OCCAM_ERR_INVALID_ARG;
+  }
+  return (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) ? OCCAM_OK : OCCAM_ERR_INVALID_ARG;
+}
+
+int device_view(const void* p, const void** dev) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return OCCAM_ERR_INVALID_ARG;
+  }
+  if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) {
+    *dev = p;
+    return OCCAM_OK;
+  }
+  if (at.type == cudaMemoryTypeHost && at.devicePointer) {
+    // the same byte offset into the allocation, seen from the device
+    *dev = static_cast<const char*>(at.devicePointer) +
+           (static_cast<const char*>(p) - static_cast<const char*>(at.hostPointer));
+    return OCCAM_OK;
+  }
+  return OCCAM_ERR_INVALID_ARG;
+}
+
 int check_gather(int n, const void* const* src, const int64_t* rb, void* const* dst) {
   if (n < 0 || n > OCCAM_MAX_GATHER) return OCCAM_ERR_INVALID_ARG;
   for (int t = 0; t < n; ++t) {
@@ -610,7 +643,8 @@ int occam_compact(const occam_batch* batch, const uint8_t* keep, int32_t n_tenso
 }
 
 static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
-                      size_t workspace_bytes, occam_stream_t stream, Trace trace) {
+                      size_t workspace_bytes, occam_stream_t stream, Trace trace, void* k2_stage = nullptr,
+                      size_t k2_stage_bytes = 0) {
   if (!args || !out) return OCCAM_ERR_INVALID_ARG;
   const occam_batch* b = &args->batch;
   OCCAM_TRY(check_batch(b));
@@ -623,6 +657,31 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   if (!(args->lambda1 == args->lambda1) || !(args->lambda2 == args->lambda2)) return OCCAM_ERR_INVALID_ARG;
   WsLayout L;
   OCCAM_TRY(check_ws(b, args->stage1.H1, args->stage2.H2, workspace, workspace_bytes, &L));
+  // memory kinds (see device_view)
+  OCCAM_TRY(require_device(args->stage1.q));
+  OCCAM_TRY(require_device(args->stage1.K1));
+  if (args->stage1.mode == OCCAM_STAGE1_CLS) OCCAM_TRY(require_device(args->stage1.k_cls));
+  OCCAM_TRY(require_device(args->stage2.Q_text));
+  if (args->stage2.K_text) OCCAM_TRY(require_device(args->stage2.K_text));
+  occam_stage2_args a2 = args->stage2;
+  const void* k2_src = nullptr;
+  const int64_t k2_row = (int64_t)a2.H2 * a2.d2 * 2;
+  if (k2_stage) {
+    if (!aligned16(k2_stage) || k2_stage_bytes < (size_t)(b->total_rows * k2_row)) return OCCAM_ERR_INVALID_ARG;
+    OCCAM_TRY(require_device(k2_stage));
+    OCCAM_TRY(device_view(a2.K2, &k2_src));
+    a2.K2 = k2_stage;
+  } else {
+    OCCAM_TRY(require_device(a2.K2));
+  }
+  const void* src[OCCAM_MAX_GATHER];
+  void* dst[OCCAM_MAX_GATHER];
+  for (int t = 0; t < args->n_tensors; ++t) {
+    OCCAM_TRY(device_view(args->src[t], &src[t]));
+    const void* d = nullptr;
+    OCCAM_TRY(device_view(args->dst[t], &d));
+    dst[t] = const_cast<void*>(d);
+  }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   set_smem_attrs();
   void* ws = workspace;
@@ -635,19 +694,37 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   OCCAM_CUDA(cudaMemsetAsync(at<unsigned char>(ws, L.zero_begin), 0, L.zero_end - L.zero_begin, st));
   trace.mark(st);
   OCCAM_TRY(launch_stage1_scores(b, &args->stage1, L, ws, s1, s2, st, trace));
-  const Stage2Params plan = stage2_params(b, &args->stage2, L, ws, s2, ref2, args->lambda2);
+  const Stage2Params plan = stage2_params(b, &a2, L, ws, s2, ref2, args->lambda2);
   OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, &args->stage1, s2,
                              &plan, out->count_out, out->count_vis,
                              st, trace));
-  OCCAM_TRY(launch_stage2(b, &args->stage2, L, ws, s2, ref2, args->lambda2, st, trace));
+  if (k2_stage) {
+    // the S1 rows of K2 (only those) into the device staging tensor
+    StageRowsParams sp;
+    sp.bt = dev_batch(b);
+    sp.src = static_cast<const unsigned char*>(k2_src);
+    sp.dst = static_cast<unsigned char*>(k2_stage);
+    sp.row_bytes = k2_row;
+    sp.dense = at<int32_t>(ws, L.dense);
+    sp.n1 = at<int32_t>(ws, L.n1);
+    stage_rows_kernel<<<num_sms() * 4, 256, 0, st>>>(sp);
+    OCCAM_CUDA(cudaGetLastError());
+  }
+  OCCAM_TRY(launch_stage2(b, &a2, L, ws, s2, ref2, args->lambda2, st, trace));
   return launch_compact(b, L, ws, 1, nullptr, keep1, s2, args->keep_registers, out->keep2, args->n_tensors,
-                        args->src, args->row_bytes, args->dst, args->capacity_rows, out->out_index,
+                        src, args->row_bytes, dst, args->capacity_rows, out->out_index,
                         out->count_out, out->count_vis, out->out_off, st, false, trace);
 }
 
 int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                 size_t workspace_bytes, occam_stream_t stream) {
   return prune_impl(args, out, workspace, workspace_bytes, stream, Trace());
+}
+
+int occam_prune_staged(const occam_prune_args* args, const occam_prune_out* out, void* k2_stage,
+                       size_t k2_stage_bytes, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  if (!k2_stage) return OCCAM_ERR_INVALID_ARG;
+  return prune_impl(args, out, workspace, workspace_bytes, stream, Trace(), k2_stage, k2_stage_bytes);
 }
 
 int occam_prune_traced(const occam_prune_args* args, const occam_prune_out* out, void* workspace,

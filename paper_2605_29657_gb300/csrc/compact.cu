@@ -208,6 +208,34 @@ __global__ void __launch_bounds__(256) gather_kernel(GatherParams p) {
   }
 }
 
+// stage_rows_kernel: persistent grid; one warp per row position p of the
+// batch, copying row dense[p] (8 KB for H2 = 32) when p lies in its sample's
+// S1 list. With a host source the loads cross the host link, so each lane
+// keeps U 16-byte loads in flight.
+__global__ void __launch_bounds__(256) stage_rows_kernel(StageRowsParams p) {
+  constexpr int U = 8;
+  const int lane = threadIdx.x & 31;
+  const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int64_t rbytes = p.row_bytes;
+  for (int64_t pos = gw; pos < p.bt.total_rows; pos += nw) {
+    const int b = upper_interval(p.bt.row_off, p.bt.B, pos);
+    if (pos - p.bt.row_off[b] >= p.n1[b]) continue;
+    const int64_t row = p.dense[pos];
+    const unsigned char* src = p.src + row * rbytes;
+    unsigned char* dst = p.dst + row * rbytes;
+    int64_t off = (int64_t)lane * 16;
+    for (; off + (U - 1) * 512 < rbytes; off += U * 512) {
+      uint4 v[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) v[u] = ldg_stream(src + off + u * 512);
+#pragma unroll
+      for (int u = 0; u < U; ++u) *reinterpret_cast<uint4*>(dst + off + u * 512) = v[u];
+    }
+    for (; off < rbytes; off += 512) *reinterpret_cast<uint4*>(dst + off) = ldg_stream(src + off);
+  }
+}
+
 }  // namespace occam
 
 // ============================================================================

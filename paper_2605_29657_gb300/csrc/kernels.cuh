@@ -157,6 +157,18 @@ struct GatherParams {
   int64_t capacity;
 };
 
+// Copies the S1 rows of K2 into a staging tensor at the same row positions
+// (rows dense[row_off[b] + i], i < n1[b]); the source may be host memory
+// the device can read (pinned), the destination is device memory.
+struct StageRowsParams {
+  BatchDev bt;
+  const unsigned char* src;
+  unsigned char* dst;
+  int64_t row_bytes;
+  const int32_t* dense;
+  const int32_t* n1;
+};
+
 struct Stage2TcParams {
   BatchDev bt;
   int H;
@@ -204,6 +216,7 @@ int s2_fused_threads();
 
 // compact.cu
 __global__ void scan_kernel(ScanParams p);
+__global__ void stage_rows_kernel(StageRowsParams p);
 __global__ void gather_kernel(GatherParams p);
 __global__ void offsets_fix_kernel(ScanParams p);
 

@@ -29,13 +29,15 @@ def to_device(batch: dict, dev) -> dict:
 
 
 def run_prune(batch: dict, lam1: float, lam2: float, keep_registers: bool = True, dev="cuda",
-              capacity_rows=None, gather=True, text_keys: bool = True, g=None, path: str = "auto"):
-    """path: "auto" (fused tensor-core Stage II where it fits) or "twopass"."""
+              capacity_rows=None, gather=True, text_keys: bool = True, g=None, path: str = "auto",
+              host_inputs: bool = False):
+    """path: "auto" (fused tensor-core Stage II where it fits) or "twopass".
+    host_inputs: K2, hidden and V stay in pinned host memory (occam_prune_staged)."""
     import os
     old = os.environ.get("OCCAM_STAGE2_PATH")
     os.environ["OCCAM_STAGE2_PATH"] = path
     try:
-        return _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g)
+        return _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs)
     finally:
         if old is None:
             os.environ.pop("OCCAM_STAGE2_PATH", None)
@@ -43,11 +45,15 @@ def run_prune(batch: dict, lam1: float, lam2: float, keep_registers: bool = True
             os.environ["OCCAM_STAGE2_PATH"] = old
 
 
-def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g):
+def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs=False):
     import paper_2605_29657_gb300 as occ
 
     m = batch["meta"]
     g = to_device(batch, dev) if g is None else g
+    if host_inputs:
+        g = dict(g)
+        for k in ("K2", "hidden", "V"):
+            g[k] = g[k].cpu().pin_memory()
     layout = occ.BatchLayout.from_batch(batch, dev)
     if m["stage1"] == "cls":
         st1 = dict(mode="cls", q=g["q_cls"], k_cls=g.get("k_cls"), K1=g["K1"])
@@ -58,7 +64,7 @@ def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, te
     if gather:
         tensors = (g["hidden"], g["K2"].view(g["K2"].shape[0], -1), g["V"])
     out = occ.occam_prune(layout, st1, st2, lam1, lam2, keep_registers=keep_registers, gather=tensors,
-                          capacity_rows=capacity_rows)
+                          capacity_rows=capacity_rows, host_inputs=host_inputs)
     torch.cuda.synchronize()
     status = occ.occam_get_status(out["ws"])
     res = {k: v.cpu().numpy() for k, v in out.items() if isinstance(v, torch.Tensor) and k != "ws"}

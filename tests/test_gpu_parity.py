@@ -13,7 +13,7 @@ import torch
 
 from oracle import occam_oracle as O
 from synth import get_config, make_batch, tiny_batch
-from tests.gpu_helpers import check_prune, close, run_prune
+from tests.gpu_helpers import check_prune, close, run_prune, to_device
 
 pytestmark = pytest.mark.gpu
 
@@ -138,6 +138,52 @@ def test_deterministic_across_calls():
     c = run_prune(b, 0.2, 1.2)
     for k in ("s1", "ref1", "s2", "ref2", "keep1", "keep2", "out_index", "count_out", "out_off"):
         assert np.array_equal(a[k], c[k]), k
+
+
+@pytest.mark.parametrize("path", ["auto", "twopass"])
+def test_host_inputs_match_device_inputs(path):
+    # K2, hidden and V in pinned host memory (occam_prune_staged): only S1
+    # rows of K2 and the kept rows are read across the host link, and every
+    # output is bit-identical to the all-device call
+    b = _tiny(B=4, segs=2, P=(120, 57, 300, 9), R=3, M=(70, 5, 130, 1), seed=21)
+    dev = run_prune(b, 0.2, 1.2, path=path)
+    host = run_prune(b, 0.2, 1.2, path=path, host_inputs=True)
+    assert host["status"] == 0
+    for k in ("s1", "ref1", "s2", "ref2", "keep1", "keep2", "count_vis", "count_out", "out_off", "n1_vis"):
+        assert np.array_equal(host[k], dev[k]), k
+    kept = int(dev["out_off"][-1])
+    assert np.array_equal(host["out_index"][:kept], dev["out_index"][:kept])
+    for a, c in zip(host["gathered"], dev["gathered"]):
+        assert torch.equal(a[:kept], c[:kept])
+    check_prune(b, host, 0.2, 1.2)
+
+
+def test_host_inputs_refuse_pageable_memory():
+    import paper_2605_29657_gb300 as occ
+
+    b = _tiny(B=2, segs=1, P=(30, 40), R=2, M=(4, 6), seed=22)
+    g = to_device(b, "cuda")
+    layout = occ.BatchLayout.from_batch(b, "cuda")
+    st1 = dict(mode="cls", q=g["q_cls"], k_cls=g["k_cls"], K1=g["K1"])
+    # pageable host K2: refused by the binding before any launch
+    with pytest.raises(occ.OccamError):
+        occ.occam_prune(layout, st1, dict(Q_text=g["Q_text"], K_text=g["K_text"], K2=g["K2"].cpu()), 0.2, 1.0,
+                        host_inputs=True)
+    # ... and by the library itself when handed one through the C ABI
+    call = occ.PruneCall(layout, st1, dict(Q_text=g["Q_text"], K_text=g["K_text"], K2=g["K2"].cpu().pin_memory()),
+                         0.2, 1.0, host_inputs=True)
+    pageable = g["K2"].cpu()
+    call.args.stage2.K2 = pageable.data_ptr()
+    with pytest.raises(occ.OccamError) as e:
+        call()
+    assert e.value.code == occ._lib.OCCAM_ERR_INVALID_ARG
+    # a host tensor where the library requires device memory (a TMA-read input)
+    call2 = occ.PruneCall(layout, st1, dict(Q_text=g["Q_text"], K_text=g["K_text"], K2=g["K2"]), 0.2, 1.0)
+    pinned = g["K2"].cpu().pin_memory()
+    call2.args.stage2.K2 = pinned.data_ptr()
+    with pytest.raises(occ.OccamError) as e:
+        call2()
+    assert e.value.code == occ._lib.OCCAM_ERR_INVALID_ARG
 
 
 # ----------------------------------------------------------------------------- standalone entry points
