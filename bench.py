@@ -311,8 +311,9 @@ def run_ours(args, rank, world, local):
     # starts in pinned host memory each step. The scoring inputs (q/k_cls,
     # K1, Q_text, K_text) are copied to the device; K2, hidden and V stay on
     # the host and occam_prune_staged reads only what the method needs from
-    # them across the host link (the S1 rows of K2, the kept rows of all
-    # three). The results (counts, offsets, indices) are read back.
+    # them across the host link (the S1 rows of K2, the kept rows of hidden
+    # and V; the kept rows of K2 come from its staged S1 rows). The results
+    # (counts, offsets, indices) are read back.
     e2e = None
     if not args.no_e2e:
         copy_names = ["q_cls", "k_cls", "K1", "Q_text", "K_text"]
@@ -326,7 +327,8 @@ def run_ours(args, rank, world, local):
         res_host = {k: torch.empty_like(hcall.out[k], device="cpu").pin_memory() for k in res_names}
         copied = sum(host[k].numel() * host[k].element_size() for k in copy_names)
         k2row = meta["H2"] * meta["d2"] * 2
-        kept_row = sum(host[k][0].numel() * host[k].element_size() for k in ("hidden", "K2", "V"))
+        # the kept rows of K2 are read from the staged S1 rows on the device
+        kept_row = sum(host[k][0].numel() * host[k].element_size() for k in ("hidden", "V"))
         in_place = n1_total * k2row + kept_total * kept_row
         d2h = sum(t.numel() * t.element_size() for t in res_host.values())
 
@@ -363,7 +365,7 @@ def run_ours(args, rank, world, local):
                "h2d_bytes_per_step": int(copied + in_place), "d2h_bytes_per_step": int(d2h), "steps": e_steps,
                "h2d_copied_bytes_per_step": int(copied), "h2d_read_in_place_bytes_per_step": int(in_place),
                "inputs": "pinned host memory; q/k_cls, K1, Q_text, K_text copied each step; K2, hidden, V "
-                         "read in place (S1 rows of K2, kept rows of all three)"}
+                         "read in place (S1 rows of K2, kept rows of hidden and V)"}
 
     if rank != 0:
         if world > 1:

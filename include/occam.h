@@ -234,8 +234,10 @@ int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* 
  *     the S1 rows of K2, and only those, into k2_stage at their own row
  *     positions; Stage II then reads k2_stage. Its other rows are left as
  *     they are.
- * So only the S1 rows of K2 and the kept rows of the gather sources cross
- * the host link, not whole tensors. Results are identical to occam_prune on
+ * A gather source equal to K2 (same pointer, row_bytes = H2 * d2 * 2) is
+ * read from k2_stage, since every kept row is an S1 row. So only the S1
+ * rows of K2 and the kept rows of the other gather sources cross the host
+ * link, not whole tensors. Results are identical to occam_prune on
  * the same values. In occam_prune_traced's event order the copy falls in the
  * interval after the Stage-I finalize. */
 int occam_prune_staged(const occam_prune_args* args, const occam_prune_out* out, void* k2_stage,

@@ -677,7 +677,12 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   const void* src[OCCAM_MAX_GATHER];
   void* dst[OCCAM_MAX_GATHER];
   for (int t = 0; t < args->n_tensors; ++t) {
-    OCCAM_TRY(device_view(args->src[t], &src[t]));
+    if (k2_stage && args->src[t] == args->stage2.K2 && args->row_bytes[t] == k2_row) {
+      // the kept rows are S1 rows: a gather of K2 itself reads the staged copy
+      src[t] = k2_stage;
+    } else {
+      OCCAM_TRY(device_view(args->src[t], &src[t]));
+    }
     const void* d = nullptr;
     OCCAM_TRY(device_view(args->dst[t], &d));
     dst[t] = const_cast<void*>(d);
