@@ -168,6 +168,35 @@ int occam_compact(const occam_batch* batch, const uint8_t* keep, int32_t n_tenso
                   int64_t capacity_rows, int32_t* out_index, int32_t* count_out, int64_t* out_off,
                   void* workspace, size_t workspace_bytes, occam_stream_t stream);
 
+/* Test-time register construction (Algorithm 1, step 2; App. A, register
+ * redirection), the step before Stage I. h [total_rows, channels] bf16
+ * (device, in place) holds the activations of the layer that carries the
+ * register neurons; k_reg [n_k] int32 (device) lists those channels,
+ * distinct and each in [0, channels) (not checked on the device). For every segment s and k
+ * in k_reg: every register row r of s gets h[r][k] = max over the visual
+ * rows v of s of h[v][k], and then h[v][k] = 0 on those visual rows. Other
+ * channels and rows are unchanged; a segment without visual rows keeps its
+ * registers. Exact (the max is one of the inputs). */
+int occam_construct_registers(const occam_batch* batch, void* h, int64_t channels, const int32_t* k_reg,
+                              int32_t n_k, void* workspace, size_t workspace_bytes, occam_stream_t stream);
+
+/* Budget matching for lambda2 on the device (App. A, lambda2* of the
+ * average-budget equation). Over a calibration batch the Stage-II retained
+ * count at lambda2 is the number of visual S1 rows v (keep1[v] != 0, not a
+ * register) with s2[v] >= lambda2 * ref2[b(v)], so it steps down at each
+ * ratio s2[v] / ref2[b(v)]. lambda2_out (device, one fp32) receives the
+ * target_count-th largest such ratio, computed as an IEEE fp32 quotient:
+ * the largest lambda2 under which the ratio test keeps at least
+ * target_count rows (exactly target_count when the ratios are distinct).
+ * target_count = K_tar * |D| in total over the batch's samples. Samples with
+ * ref2 <= 0 contribute no candidates. target_count <= 0 gives +inf; a
+ * target above the candidate count gives 0 (keep all). n_candidates (device
+ * int32, nullable) receives the candidate count. s2 [total_rows] and ref2
+ * [B] are as written by occam_score_stage2 / occam_prune. */
+int occam_calibrate_lambda2(const occam_batch* batch, const float* s2, const float* ref2, const uint8_t* keep1,
+                            int64_t target_count, float* lambda2_out, int32_t* n_candidates, void* workspace,
+                            size_t workspace_bytes, occam_stream_t stream);
+
 /* The fused path: Stage-I scores -> Stage-I threshold (per segment,
  * lambda1; registers always in S1) -> Stage-II scores over S1 -> Stage-II
  * threshold (per sample, lambda2) -> compaction and gather. Per-sample
@@ -191,7 +220,11 @@ typedef struct occam_prune_args {
  * (kept visual rows = the sample's budget |S2 \ {r}|), count_out [B] int32,
  * out_off [B+1] int64. Optional (NULL to skip): keep1 [total_rows] u8 (S1,
  * registers = 1), s1 [total_rows], ref1 [S_tot], s2 [total_rows], ref2 [B]
- * (fp32), n1_vis [B] int32 (visual rows of S1). */
+ * (fp32), n1_vis [B] int32 (visual rows of S1), n_eff [S_tot, H1] fp32
+ * ([CLS] mode only, else OCCAM_ERR_UNSUPPORTED): per segment and head the
+ * effective number of attended keys of the Stage-I [CLS] attention,
+ * exp(H(a)) with H(a) = -sum_i a_i log a_i over the keys {[CLS]} u rows
+ * (Sec. 3.2, Observation 1). */
 typedef struct occam_prune_out {
   uint8_t* keep2;
   int32_t* out_index;
@@ -204,6 +237,7 @@ typedef struct occam_prune_out {
   float* s2;
   float* ref2;
   int32_t* n1_vis;
+  float* n_eff;
 } occam_prune_out;
 
 /* The whole path in one call (Algorithm 1's pruning steps): Stage-I scores,

@@ -11,11 +11,15 @@ Each function follows one equation of the paper:
 * relative comparison rule s_x(v) >= lambda s_x(r(x))            -- Sec. 3.2, Eq. 3
 * Stage I [CLS] scores s1(v) = A_{cls->v}, s1(r) = A_{cls->r},
   averaged over heads                                            -- Sec. 3.4, Eq. 4; App. A, Eq. 10
+* effective number of attended keys n_eff = exp(H(A)) of the
+  Stage-I [CLS] attention, per segment and head                 -- Sec. 3.2, Observation 1
 * Stage I mutual scores s1(v) = 1/(|V|+1) sum_u A_{u->v}         -- Sec. 3.4, Eq. 6; App. A, Eq. 13
 * Stage I set S1 = {v : s1(v) >= lambda1 s1(r)} u {r}            -- Eq. 5; App. A, Eqs. 11-12
 * Stage II scores s2(v) = max_j A_{t_j->v}, s2(r) = mean_j A_{t_j->r}
                                                                  -- Sec. 3.5, Eq. 7; App. A, Eqs. 15-16
 * Stage II set S2 = {v in S1\\{r} : s2(v) >= lambda2 s2(r)} u {r} -- Eq. 8; App. A, Eq. 17
+* lambda2 matching a retained budget over a calibration set      -- App. A, average-budget equation
+* test-time register construction h_r,k = max_v h_v,k, h_v,k = 0 -- Algorithm 1; App. A, register redirection
 * decoding continues on [S2; T]: order-preserving compaction of
   the kept rows (prefix and KV cache shrink with the kept count) -- Algorithm 1; App. A, Eq. 21
 
@@ -115,6 +119,40 @@ def stage1_cls(q_cls, k_cls, K1, seg_off, reg_idx, reg_off):
     return s1, ref1
 
 
+def effective_keys(a) -> float:
+    """n_eff = exp(H(a)) with H(a) = -sum_i a_i log a_i, the entropy of an
+    attention distribution a (Sec. 3.2, Observation 1): the support size of
+    the uniform distribution with the same entropy. Terms with a_i = 0 add 0."""
+    a = np.asarray(a, dtype=np.float64)
+    terms = np.where(a > 0, a * np.log(np.where(a > 0, a, 1.0)), 0.0)
+    return float(np.exp(-np.sum(terms)))
+
+
+def stage1_neff(q_cls, k_cls, K1, seg_off):
+    """n_eff of the Stage-I [CLS] attention (Sec. 3.2, Observation 1, on the
+    map of Sec. 3.4, Eq. 4): for each segment s and head h, the distribution
+    A = softmax(q k^T / sqrt(d1)) of the segment's [CLS] query over the keys
+    {k_cls[s]} u rows(s) (the [CLS] key included when given), and
+    n_eff = exp(-sum A log A). Returns [S_tot, H].
+    """
+    q = as_f64(q_cls)
+    kc = None if k_cls is None else as_f64(k_cls)
+    K = as_f64(K1)
+    seg_off = as_i64(seg_off)
+    S_tot = seg_off.shape[0] - 1
+    H, d = K.shape[1], K.shape[2]
+    scale = 1.0 / np.sqrt(d)
+    out = np.zeros((S_tot, H), dtype=np.float64)
+    for s in range(S_tot):
+        r0, r1 = seg_off[s], seg_off[s + 1]
+        for h in range(H):
+            logits = (K[r0:r1, h, :] @ q[s, h, :]) * scale
+            if kc is not None:
+                logits = np.concatenate([[np.dot(kc[s, h, :], q[s, h, :]) * scale], logits])
+            out[s, h] = effective_keys(softmax(logits))
+    return out
+
+
 def stage1_mutual(Q1, K1, seg_off, reg_idx, reg_off):
     """Stage-I mutual scores (Sec. 3.4, Eq. 6; App. A, Eq. 13).
 
@@ -166,6 +204,57 @@ def threshold(s, ref_of_row, lam: float, is_reg, prev_keep=None, keep_registers:
     if keep_registers:
         keep |= is_reg
     return keep
+
+
+def construct_registers(h, seg_off, reg_idx, reg_off, k_reg):
+    """Test-time register construction (Algorithm 1, step 2; App. A, register
+    redirection): for every segment and register channel k, each register
+    row takes the max of channel k over the segment's visual rows, and the
+    channel is then zeroed on those visual rows. A segment without visual
+    rows keeps its registers. Returns a new float64 array (the bf16 inputs
+    are exact in it; the results are inputs or 0, so exact in bf16 too).
+    """
+    h = as_f64(h).copy()
+    seg_off = as_i64(seg_off)
+    reg_idx = as_i64(reg_idx)
+    reg_off = as_i64(reg_off)
+    for s in range(len(seg_off) - 1):
+        rows = np.arange(seg_off[s], seg_off[s + 1])
+        regs = reg_idx[reg_off[s]:reg_off[s + 1]]
+        vis = np.setdiff1d(rows, regs)
+        for k in as_i64(k_reg):
+            if len(vis) > 0:
+                h[regs, k] = np.max(h[vis, k])
+                h[vis, k] = 0.0
+    return h
+
+
+def lambda2_for_budget(s2, ref2, keep1, is_reg, row_off, target_count: int):
+    """lambda2 matching a retained budget (App. A, the lambda2* that makes the
+    average |S2| over the calibration set D equal K_tar).
+
+    |S2(lambda2)| counts the visual S1 rows v with s2(v) >= lambda2 s2(r) of
+    their sample, so the total over D drops by one at each ratio
+    s2(v) / s2(r). The lambda2 whose total is K = target_count
+    (= K_tar |D|) is therefore the K-th largest ratio: at it the ratio test
+    keeps at least K rows, just above it fewer. The ratios are taken as fp32
+    quotients of the fp32 scores (the precision in which the scores are
+    given), and the K-th largest comes from a sort. Samples whose reference
+    is not positive contribute no candidates. K <= 0 gives +inf; K above the
+    candidate count gives 0 (keep all).
+    """
+    s2 = np.asarray(s2, dtype=np.float32)
+    ref2 = np.asarray(ref2, dtype=np.float32)
+    row_off = as_i64(row_off)
+    cand = np.asarray(keep1, dtype=bool) & ~np.asarray(is_reg, dtype=bool)
+    sample = np.repeat(np.arange(len(row_off) - 1), np.diff(row_off))
+    cand &= ref2[sample] > 0
+    ratios = np.sort(s2[cand] / ref2[sample][cand])[::-1]  # float32 / float32: IEEE quotient
+    if target_count <= 0:
+        return np.float32(np.inf), int(cand.sum())
+    if target_count > len(ratios):
+        return np.float32(0.0), int(cand.sum())
+    return np.float32(ratios[target_count - 1]), int(cand.sum())
 
 
 # --------------------------------------------------------------------------- Stage II

@@ -17,8 +17,10 @@ from ._lib import (  # noqa: F401
     PruneCall,
     alloc_workspace,
     library,
+    occam_calibrate_lambda2,
     occam_compact,
     occam_compact_noalloc,
+    occam_construct_registers,
     occam_get_status,
     occam_prune,
     occam_score_stage1,

@@ -74,7 +74,7 @@ class CPruneArgs(ctypes.Structure):
 class CPruneOut(ctypes.Structure):
     _fields_ = [
         ("keep2", _p), ("out_index", _p), ("count_vis", _p), ("count_out", _p), ("out_off", _p),
-        ("keep1", _p), ("s1", _p), ("ref1", _p), ("s2", _p), ("ref2", _p), ("n1_vis", _p),
+        ("keep1", _p), ("s1", _p), ("ref1", _p), ("s2", _p), ("ref2", _p), ("n1_vis", _p), ("n_eff", _p),
     ]
 
 
@@ -104,7 +104,10 @@ def library() -> ctypes.CDLL:
         lib.occam_prune_traced.argtypes = [P(CPruneArgs), P(CPruneOut), _p, ctypes.c_size_t, _p, P(_p), _i32]
         lib.occam_prune_staged.argtypes = [P(CPruneArgs), P(CPruneOut), _p, ctypes.c_size_t, _p, ctypes.c_size_t,
                                            _p]
-        for name in ("occam_workspace_size", "occam_get_status", "occam_score_stage1", "occam_threshold",
+        lib.occam_calibrate_lambda2.argtypes = [P(CBatch), _p, _p, _p, _i64, _p, _p, _p, ctypes.c_size_t, _p]
+        lib.occam_construct_registers.argtypes = [P(CBatch), _p, _i64, _p, _i32, _p, ctypes.c_size_t, _p]
+        for name in ("occam_construct_registers", "occam_calibrate_lambda2", "occam_workspace_size", "occam_get_status", "occam_score_stage1",
+                     "occam_threshold",
                      "occam_score_stage2", "occam_compact", "occam_prune", "occam_prune_traced",
                      "occam_compact_noalloc", "occam_prune_staged"):
             getattr(lib, name).restype = ctypes.c_int
@@ -284,6 +287,44 @@ def occam_score_stage2(layout: BatchLayout, Q_text, K2, keep1, K_text=None, s2=N
     return s2, ref2
 
 
+def occam_construct_registers(layout: BatchLayout, h, k_reg, ws=None, stream=None) -> torch.Tensor:
+    """Test-time register construction in place on h [total_rows, channels]
+    bf16 (Algorithm 1, step 2): per segment and channel in k_reg, the
+    registers take the visual rows' max, which is then zeroed on them."""
+    h = _dev_tensor(h, torch.bfloat16, "h")
+    k_reg = _dev_tensor(k_reg, torch.int32, "k_reg")
+    if h.dim() != 2 or h.shape[0] != layout.total_rows:
+        raise OccamError(OCCAM_ERR_INVALID_ARG, "h must be [total_rows, channels]")
+    if k_reg.numel() and (int(k_reg.min()) < 0 or int(k_reg.max()) >= h.shape[1]):
+        raise OccamError(OCCAM_ERR_INVALID_ARG, "k_reg channels out of range")
+    if k_reg.numel() != torch.unique(k_reg).numel():
+        raise OccamError(OCCAM_ERR_INVALID_ARG, "k_reg channels must be distinct")
+    ws = _ws(ws, layout, 1, 1)
+    cb = layout.c()
+    _check(library().occam_construct_registers(ctypes.byref(cb), _ptr(h), int(h.shape[1]), _ptr(k_reg),
+                                               int(k_reg.numel()), _ptr(ws), ws.numel(), _stream(stream)),
+           "occam_construct_registers")
+    return h
+
+
+def occam_calibrate_lambda2(layout: BatchLayout, s2, ref2, keep1, target_count: int, ws=None,
+                            stream=None) -> tuple[torch.Tensor, torch.Tensor]:
+    """lambda2 matching a total retained budget over the batch (App. A): the
+    target_count-th largest s2 / ref2 ratio of the visual S1 rows. Returns
+    (lambda2 [1] fp32, candidate count [1] int32), both on the device."""
+    s2 = _dev_tensor(s2, torch.float32, "s2")
+    ref2 = _dev_tensor(ref2, torch.float32, "ref2")
+    keep1 = _dev_tensor(keep1, torch.uint8, "keep1")
+    ws = _ws(ws, layout, 1, 1)
+    lam = torch.empty(1, dtype=torch.float32, device=layout.device)
+    n = torch.empty(1, dtype=torch.int32, device=layout.device)
+    cb = layout.c()
+    _check(library().occam_calibrate_lambda2(ctypes.byref(cb), _ptr(s2), _ptr(ref2), _ptr(keep1),
+                                             int(target_count), _ptr(lam), _ptr(n), _ptr(ws), ws.numel(),
+                                             _stream(stream)), "occam_calibrate_lambda2")
+    return lam, n
+
+
 def _gather_arrays(tensors, dsts):
     n = len(tensors)
     if n > OCCAM_MAX_GATHER:
@@ -340,7 +381,7 @@ class PruneCall:
     """A prepared occam_prune call: argument structs, outputs and workspace are
     built once and reused, so repeated calls marshal nothing."""
 
-    OPTIONAL = ("keep1", "s1", "ref1", "s2", "ref2", "n1_vis")
+    OPTIONAL = ("keep1", "s1", "ref1", "s2", "ref2", "n1_vis", "n_eff")  # n_eff: [CLS] mode only
 
     def __init__(self, layout: BatchLayout, stage1: dict, stage2: dict, lambda1: float, lambda2: float,
                  keep_registers: bool = True, gather=(), capacity_rows: int | None = None,
@@ -380,7 +421,10 @@ class PruneCall:
             out_off=torch.empty(B + 1, dtype=torch.int64, device=dev),
         )
         shapes = dict(keep1=(R, torch.uint8), s1=(R, torch.float32), ref1=(layout.S_tot, torch.float32),
-                      s2=(R, torch.float32), ref2=(B, torch.float32), n1_vis=(B, torch.int32))
+                      s2=(R, torch.float32), ref2=(B, torch.float32), n1_vis=(B, torch.int32),
+                      n_eff=((layout.S_tot, H1), torch.float32))
+        if mode != OCCAM_STAGE1_CLS:
+            want = tuple(k for k in want if k != "n_eff")
         for k in want:
             n, dt = shapes[k]
             o[k] = torch.empty(n, dtype=dt, device=dev)
@@ -403,7 +447,7 @@ class PruneCall:
         self.args = a
         self.cout = CPruneOut(*[_ptr(o.get(k)) for k in
                                 ("keep2", "out_index", "count_vis", "count_out", "out_off", "keep1", "s1", "ref1",
-                                 "s2", "ref2", "n1_vis")])
+                                 "s2", "ref2", "n1_vis", "n_eff")])
         self.capacity = cap
 
     def __call__(self, stream=None) -> dict:

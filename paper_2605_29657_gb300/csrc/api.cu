@@ -337,7 +337,7 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
 int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s1, const uint8_t* keep_in,
                      float lambda1, int do_threshold, float* ref1, uint8_t* keep1, int32_t* n1_vis,
                      const occam_stage1_args* a1, float* s2_zero, const Stage2Params* plan, int32_t* count_out,
-                     int32_t* count_vis, cudaStream_t st, Trace trace = Trace()) {
+                     int32_t* count_vis, cudaStream_t st, Trace trace = Trace(), float* n_eff = nullptr) {
   Stage1FinalizeParams p;
   p.bt = dev_batch(b);
   const bool cls = a1 && a1->mode == OCCAM_STAGE1_CLS;
@@ -346,6 +346,7 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   p.k_cls = cls ? static_cast<const __nv_bfloat16*>(a1->k_cls) : nullptr;
   p.scale = cls ? (float)(1.0 / std::sqrt((double)a1->d1)) : 1.f;
   p.s1_out = s1;
+  p.n_eff = cls ? n_eff : nullptr;
   p.s2_zero = cls ? s2_zero : nullptr;
   // a segment's logits ([CLS] mode, 64 B/row), s1 (4 B/row) and roles
   // (1 B/row) are staged in shared memory when it fits (at most 96 KB)
@@ -655,12 +656,13 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
       (args->capacity_rows > 0 && !out->out_index))
     return OCCAM_ERR_INVALID_ARG;
   if (!(args->lambda1 == args->lambda1) || !(args->lambda2 == args->lambda2)) return OCCAM_ERR_INVALID_ARG;
+  if (out->n_eff && args->stage1.mode != OCCAM_STAGE1_CLS) return OCCAM_ERR_UNSUPPORTED;
   WsLayout L;
   OCCAM_TRY(check_ws(b, args->stage1.H1, args->stage2.H2, workspace, workspace_bytes, &L));
   // memory kinds (see device_view)
   OCCAM_TRY(require_device(args->stage1.q));
   OCCAM_TRY(require_device(args->stage1.K1));
-  if (args->stage1.mode == OCCAM_STAGE1_CLS) OCCAM_TRY(require_device(args->stage1.k_cls));
+  if (args->stage1.mode == OCCAM_STAGE1_CLS && args->stage1.k_cls) OCCAM_TRY(require_device(args->stage1.k_cls));
   OCCAM_TRY(require_device(args->stage2.Q_text));
   if (args->stage2.K_text) OCCAM_TRY(require_device(args->stage2.K_text));
   occam_stage2_args a2 = args->stage2;
@@ -701,8 +703,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   OCCAM_TRY(launch_stage1_scores(b, &args->stage1, L, ws, s1, s2, st, trace));
   const Stage2Params plan = stage2_params(b, &a2, L, ws, s2, ref2, args->lambda2);
   OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, &args->stage1, s2,
-                             &plan, out->count_out, out->count_vis,
-                             st, trace));
+                             &plan, out->count_out, out->count_vis, st, trace, out->n_eff));
   if (k2_stage) {
     // the S1 rows of K2 (only those) into the device staging tensor
     StageRowsParams sp;
@@ -724,6 +725,52 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
 int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                 size_t workspace_bytes, occam_stream_t stream) {
   return prune_impl(args, out, workspace, workspace_bytes, stream, Trace());
+}
+
+int occam_construct_registers(const occam_batch* batch, void* h, int64_t channels, const int32_t* k_reg,
+                              int32_t n_k, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  OCCAM_TRY(check_batch(batch));
+  if (!h || channels <= 0 || n_k < 0 || (n_k > 0 && !k_reg)) return OCCAM_ERR_INVALID_ARG;
+  WsLayout L;
+  OCCAM_TRY(check_ws(batch, 1, 1, workspace, workspace_bytes, &L));
+  OCCAM_TRY(require_device(h));
+  if (n_k == 0 || batch->S_tot == 0) return OCCAM_OK;
+  OCCAM_TRY(require_device(k_reg));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  OCCAM_TRY(mark_roles(batch, L, workspace, st));
+  RegistersParams p;
+  p.bt = dev_batch(batch);
+  p.h = static_cast<__nv_bfloat16*>(h);
+  p.channels = channels;
+  p.k_reg = k_reg;
+  p.n_k = n_k;
+  p.role = at<uint8_t>(workspace, L.role);
+  registers_kernel<<<batch->S_tot, 256, 0, st>>>(p);
+  return cuda_ok();
+}
+
+int occam_calibrate_lambda2(const occam_batch* batch, const float* s2, const float* ref2, const uint8_t* keep1,
+                            int64_t target_count, float* lambda2_out, int32_t* n_candidates, void* workspace,
+                            size_t workspace_bytes, occam_stream_t stream) {
+  OCCAM_TRY(check_batch(batch));
+  if (!s2 || !ref2 || !keep1 || !lambda2_out) return OCCAM_ERR_INVALID_ARG;
+  if (batch->total_rows > (int64_t)0x7fffffff) return OCCAM_ERR_UNSUPPORTED;
+  WsLayout L;
+  OCCAM_TRY(check_ws(batch, 1, 1, workspace, workspace_bytes, &L));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  OCCAM_TRY(mark_roles(batch, L, workspace, st));
+  Lambda2Params p;
+  p.bt = dev_batch(batch);
+  p.s2 = s2;
+  p.ref2 = ref2;
+  p.keep1 = keep1;
+  p.role = at<uint8_t>(workspace, L.role);
+  p.target = target_count;
+  p.keys = reinterpret_cast<uint32_t*>(at<int32_t>(workspace, L.dense));
+  p.lambda2 = lambda2_out;
+  p.n_candidates = n_candidates;
+  lambda2_select_kernel<<<1, 1024, 0, st>>>(p);
+  return cuda_ok();
 }
 
 int occam_prune_staged(const occam_prune_args* args, const occam_prune_out* out, void* k2_stage,

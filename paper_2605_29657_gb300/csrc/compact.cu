@@ -236,6 +236,112 @@ __global__ void __launch_bounds__(256) stage_rows_kernel(StageRowsParams p) {
   }
 }
 
+// registers_kernel: one CTA per segment. For each register channel in turn,
+// the CTA takes the max over the segment's visual rows (a thread-strided
+// pass, then a block max), writes it into the channel of every register row
+// and zeroes the channel on the visual rows. Values are compared as floats;
+// the written max is one of the bf16 inputs, so results are exact.
+__global__ void __launch_bounds__(256) registers_kernel(RegistersParams p) {
+  __shared__ float wmax[8];
+  const int seg = blockIdx.x;
+  const int tid = threadIdx.x;
+  const int64_t r0 = p.bt.seg_off[seg], r1 = p.bt.seg_off[seg + 1];
+  const int32_t g0 = p.bt.reg_off[seg], g1 = p.bt.reg_off[seg + 1];
+  for (int j = 0; j < p.n_k; ++j) {
+    const int64_t k = p.k_reg[j];
+    float m = -INFINITY;
+    for (int64_t r = r0 + tid; r < r1; r += blockDim.x)
+      if (p.role[r] == 0) m = fmaxf(m, __bfloat162float(p.h[r * p.channels + k]));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if ((tid & 31) == 0) wmax[tid >> 5] = m;
+    __syncthreads();
+    float mx = wmax[0];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) mx = fmaxf(mx, wmax[w]);
+    // a segment without visual rows leaves its registers as they are
+    if (mx != -INFINITY)
+      for (int i = g0 + tid; i < g1; i += blockDim.x) p.h[(int64_t)p.bt.reg_idx[i] * p.channels + k] = __float2bfloat16_rn(mx);
+    for (int64_t r = r0 + tid; r < r1; r += blockDim.x)
+      if (p.role[r] == 0) p.h[r * p.channels + k] = __float2bfloat16_rn(0.f);
+    __syncthreads();
+  }
+}
+
+// lambda2_select_kernel: one CTA of 1,024 threads. Each candidate row (a
+// visual S1 row of a sample with ref2 > 0) gets the key bits(s2 / ref2), an
+// IEEE round-to-nearest fp32 quotient >= 0 whose bit pattern orders like its
+// value; every other row gets key 0, below or equal to every candidate. The
+// K-th largest key is then found most significant byte first: per byte, a
+// histogram of the keys that match the bytes chosen so far (one 256-bin
+// histogram per warp, then summed), and the bucket where the running count
+// from the top reaches K. With K <= the candidate count the result is the
+// K-th largest candidate ratio.
+__global__ void __launch_bounds__(1024) lambda2_select_kernel(Lambda2Params p) {
+  __shared__ uint32_t hist[32][256];
+  __shared__ uint32_t tot[256];
+  __shared__ uint32_t s_prefix, s_k;
+  __shared__ int s_cnt;
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int64_t R = p.bt.total_rows;
+  if (tid == 0) s_cnt = 0;
+  __syncthreads();
+  int cnt = 0;
+  for (int64_t r = tid; r < R; r += blockDim.x) {
+    const int b = upper_interval(p.bt.row_off, p.bt.B, r);
+    const float ref = p.ref2[b];
+    uint32_t key = 0;
+    if (p.keep1[r] && p.role[r] == 0 && ref > 0.f) {
+      key = __float_as_uint(__fdiv_rn(p.s2[r], ref));
+      ++cnt;
+    }
+    p.keys[r] = key;
+  }
+  atomicAdd(&s_cnt, cnt);
+  __syncthreads();
+  const int64_t n = s_cnt;
+  if (p.n_candidates && tid == 0) *p.n_candidates = (int32_t)n;
+  if (p.target <= 0 || p.target > n) {
+    // K <= 0: no lambda2 keeps nothing but +inf; K > n: 0 keeps every candidate
+    if (tid == 0) *p.lambda2 = p.target <= 0 ? __int_as_float(0x7f800000) : 0.f;
+    return;
+  }
+  if (tid == 0) {
+    s_prefix = 0;
+    s_k = (uint32_t)p.target;
+  }
+  uint32_t mask = 0;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = tid; i < 32 * 256; i += blockDim.x) (&hist[0][0])[i] = 0;
+    __syncthreads();
+    const uint32_t prefix = s_prefix;
+    for (int64_t r = tid; r < R; r += blockDim.x) {
+      const uint32_t key = p.keys[r];
+      if ((key & mask) == prefix) atomicAdd(&hist[warp][(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid < 256) {
+      uint32_t t = 0;
+      for (int w = 0; w < 32; ++w) t += hist[w][tid];
+      tot[tid] = t;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      // walk from the largest byte value down to the bucket holding the K-th key
+      uint32_t k = s_k, cum = 0;
+      int d = 255;
+      for (; d > 0; --d) {
+        if (cum + tot[d] >= k) break;
+        cum += tot[d];
+      }
+      s_k = k - cum;
+      s_prefix = prefix | ((uint32_t)d << shift);
+    }
+    mask |= 255u << shift;
+    __syncthreads();
+  }
+  if (tid == 0) *p.lambda2 = __uint_as_float(s_prefix);
+}
+
 }  // namespace occam
 
 // ============================================================================

@@ -100,6 +100,7 @@ struct Stage1FinalizeParams {
   const __nv_bfloat16* k_cls;     // nullable
   float scale;
   float* s1_out;                  // [CLS] mode: where s1 is written
+  float* n_eff;                   // nullable, [CLS] mode: [S_tot, 16] effective number of attended keys per head
   float* s2_zero;                 // nullable: zeroed per row (Stage-II max accumulator)
   int smem_rows;                  // segments up to this many rows stage their logits in shared memory
   const float* s1;          // nullable when keep_in is given
@@ -169,6 +170,32 @@ struct StageRowsParams {
   const int32_t* n1;
 };
 
+// Test-time register construction (Algorithm 1; App. A, register
+// redirection): per segment and register channel k, the register rows take
+// the max over the visual rows of h[., k], which is then zeroed on them
+struct RegistersParams {
+  BatchDev bt;
+  __nv_bfloat16* h;      // [total_rows, channels]
+  int64_t channels;
+  const int32_t* k_reg;  // [n_k] channel indices
+  int n_k;
+  const uint8_t* role;
+};
+
+// lambda2 budget matching (App. A): the K-th largest ratio s2[v] / ref2[b(v)]
+// over the visual S1 rows of a calibration batch
+struct Lambda2Params {
+  BatchDev bt;
+  const float* s2;
+  const float* ref2;
+  const uint8_t* keep1;
+  const uint8_t* role;
+  int64_t target;       // K
+  uint32_t* keys;       // [total_rows] scratch
+  float* lambda2;       // out
+  int32_t* n_candidates;  // out, nullable
+};
+
 struct Stage2TcParams {
   BatchDev bt;
   int H;
@@ -217,6 +244,8 @@ int s2_fused_threads();
 // compact.cu
 __global__ void scan_kernel(ScanParams p);
 __global__ void stage_rows_kernel(StageRowsParams p);
+__global__ void lambda2_select_kernel(Lambda2Params p);
+__global__ void registers_kernel(RegistersParams p);
 __global__ void gather_kernel(GatherParams p);
 __global__ void offsets_fix_kernel(ScanParams p);
 

@@ -134,7 +134,7 @@ int stage1_logits_smem_bytes() { return cls::kSmem; }
 __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, int seg, int64_t sb, int n,
                                                const float* lg, float* s1_loc) {
   constexpr int H = 16, D = 64;
-  __shared__ float red[16][17];
+  __shared__ float red[16][17], red2[16][17];
   __shared__ float gmax[16], ginv[16], lcls_s[16];
   const int tid = threadIdx.x;
   if (tid < 256) {
@@ -165,14 +165,29 @@ __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, in
   }
   __syncthreads();
   const float mh = gmax[h];
-  float z = 0.f;
-  for (int r = j; r < n; r += 16) z += expf(lg[r * H + h] - mh);
+  float z = 0.f, t = 0.f;  // t: sum of e (l - max), for the entropy
+  for (int r = j; r < n; r += 16) {
+    const float x = lg[r * H + h] - mh;
+    const float e = expf(x);
+    z += e;
+    t = fmaf(e, x, t);
+  }
   red[j][h] = z;
+  red2[j][h] = t;
   __syncthreads();
   if (tid < 16) {
-    float zz = lcls_s[tid] != -INFINITY ? expf(lcls_s[tid] - gmax[tid]) : 0.f;
-    for (int k = 0; k < 16; ++k) zz += red[k][tid];
+    const bool self = lcls_s[tid] != -INFINITY;
+    const float xc = self ? lcls_s[tid] - gmax[tid] : 0.f;
+    float zz = self ? expf(xc) : 0.f;
+    float tt = zz * xc;
+    for (int k = 0; k < 16; ++k) {
+      zz += red[k][tid];
+      tt += red2[k][tid];
+    }
     ginv[tid] = 1.0f / zz;
+    // entropy of the head's distribution a = e / Z over the keys:
+    // H = -sum a log a = log Z - (sum e (l - max)) / Z; n_eff = exp(H)
+    if (p.n_eff) p.n_eff[(int64_t)seg * H + tid] = expf(logf(zz) - tt / zz);
   }
   __syncthreads();
   for (int r = tid; r < n; r += blockDim.x) {

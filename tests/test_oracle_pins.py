@@ -406,3 +406,157 @@ def test_head_reduce_reading_differs_from_alternative():
     vis = ~a["is_reg"]
     assert (c["s2"][vis] >= a["s2"][vis] - 1e-15).all()
     assert (c["s2"][vis] > a["s2"][vis] * (1 + 1e-6)).any()
+
+
+# ----------------------------------------------------------------------------- n_eff (Sec. 3.2, Observation 1)
+
+def test_neff_uniform_attention_counts_every_key():
+    """q_cls = 0: the [CLS] attention is uniform over the N keys ({[CLS]} u rows), so n_eff = N."""
+    b = tiny_batch(B=2, segs=2, P=(5, 8), R=3, M=(2, 3), seed=6)
+    m = b["meta"]
+    ne = O.stage1_neff(_zero(b["q_cls"]), b["k_cls"], b["K1"], m["seg_off_host"])
+    n_keys = np.diff(m["seg_off_host"]) + 1
+    np.testing.assert_allclose(ne, np.repeat(n_keys[:, None], ne.shape[1], axis=1), rtol=1e-13)
+    # without the [CLS] key, the rows alone
+    ne2 = O.stage1_neff(_zero(b["q_cls"]), None, b["K1"], m["seg_off_host"])
+    np.testing.assert_allclose(ne2[:, 0], n_keys - 1, rtol=1e-13)
+
+
+@pytest.mark.parametrize("dl", [0, 1, 3, 40])
+def test_neff_two_keys_binary_entropy(dl):
+    """Two keys with an exact logit gap dl: a = (p, 1-p), p = 1/(1+e^-dl), n_eff = exp(h(p))."""
+    q = torch.tensor([[[2.0, 0, 0, 0]]]).to(torch.bfloat16)          # scale 1/2 -> logit = k[0]
+    K1 = torch.tensor([[[float(dl), 1, 2, 3]], [[0.0, -1, 5, 2]]]).to(torch.bfloat16)
+    ne = O.stage1_neff(q, None, K1, np.array([0, 2]))
+    p = 1.0 / (1.0 + math.exp(-dl))
+    h = -(p * math.log(p) + (1 - p) * math.log1p(-p)) if p < 1 else 0.0
+    assert abs(ne[0, 0] - math.exp(h)) <= 1e-12 * math.exp(h)
+    assert 1.0 <= ne[0, 0] <= 2.0 + 1e-15
+    if dl == 0:
+        assert abs(ne[0, 0] - 2.0) < 1e-14
+
+
+def test_neff_bounds_and_heads_independent():
+    """1 <= n_eff <= N on random inputs; identical heads give identical values."""
+    b = tiny_batch(B=2, segs=2, P=(9, 14), R=2, M=(2, 2), seed=31)
+    m = b["meta"]
+    ne = O.stage1_neff(b["q_cls"], b["k_cls"], b["K1"], m["seg_off_host"])
+    n_keys = np.diff(m["seg_off_host"]) + 1
+    assert (ne >= 1.0 - 1e-12).all() and (ne <= n_keys[:, None] + 1e-9).all()
+    q = b["q_cls"].clone()
+    K = b["K1"].clone()
+    q[:] = q[:, :1]
+    K[:] = K[:, :1]
+    ne_same = O.stage1_neff(q, b["k_cls"][:, :1].expand_as(b["k_cls"]).contiguous(), K, m["seg_off_host"])
+    assert np.all(ne_same == ne_same[:, :1])
+
+
+def test_neff_brute_force_decimal_tiny():
+    """exp(-sum a log a) at 50 digits from the exact bf16 values."""
+    getcontext().prec = 50
+    b = tiny_batch(B=1, segs=2, P=(3,), R=1, M=(2,), H1=2, d1=4, seed=33)
+    m = b["meta"]
+    ne = O.stage1_neff(b["q_cls"], b["k_cls"], b["K1"], m["seg_off_host"])
+    q = O.as_f64(b["q_cls"])
+    kc = O.as_f64(b["k_cls"])
+    K = O.as_f64(b["K1"])
+    sc = Decimal(1) / Decimal(4).sqrt()
+    dot = lambda a, c: sum(Decimal(float(x)) * Decimal(float(y)) for x, y in zip(a, c))  # noqa: E731
+    so = m["seg_off_host"]
+    for s in range(len(so) - 1):
+        for h in range(2):
+            lg = [dot(kc[s, h], q[s, h]) * sc] + [dot(K[r, h], q[s, h]) * sc for r in range(so[s], so[s + 1])]
+            mx = max(lg)
+            e = [(x - mx).exp() for x in lg]
+            z = sum(e)
+            a = [x / z for x in e]
+            want = (-sum(x * x.ln() for x in a)).exp()
+            assert abs(Decimal(ne[s, h]) - want) <= Decimal("1e-12") * want
+
+
+# ----------------------------------------------------------------------------- lambda2 budget matching (App. A)
+
+def _ratio_count(s2, ref2, keep1, is_reg, row_off, lam):
+    """Rows the Stage-II ratio test keeps at lam (visual S1 rows, positive reference)."""
+    s2 = np.asarray(s2, np.float32)
+    ref2 = np.asarray(ref2, np.float32)
+    sample = np.repeat(np.arange(len(row_off) - 1), np.diff(row_off))
+    cand = keep1.astype(bool) & ~is_reg & (ref2[sample] > 0)
+    return int(np.sum(s2[cand] / ref2[sample][cand] >= np.float32(lam)))
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_lambda2_budget_is_the_count_step(seed):
+    """At lambda2* the ratio test keeps >= K rows, just above it < K; every K of a small set, brute force."""
+    rng = np.random.default_rng(seed)
+    row_off = np.array([0, 7, 7, 19, 30])
+    R = row_off[-1]
+    s2 = rng.random(R).astype(np.float32) * rng.choice([1e-3, 1.0], R).astype(np.float32)
+    ref2 = np.array([0.2, 0.5, 0.01, 0.0], np.float32)       # the last sample has no positive reference
+    keep1 = rng.random(R) < 0.7
+    is_reg = np.zeros(R, bool)
+    is_reg[[6, 18]] = True
+    n = _ratio_count(s2, ref2, keep1, is_reg, row_off, 0.0)
+    for K in range(0, n + 2):
+        lam, cnt = O.lambda2_for_budget(s2, ref2, keep1, is_reg, row_off, K)
+        assert cnt == n
+        if K == 0:
+            assert np.isinf(lam)
+            continue
+        if K > n:
+            assert lam == 0.0
+            continue
+        assert _ratio_count(s2, ref2, keep1, is_reg, row_off, lam) >= K
+        assert _ratio_count(s2, ref2, keep1, is_reg, row_off, np.nextafter(lam, np.float32(np.inf))) < K
+        # distinct ratios here: exactly K
+        assert _ratio_count(s2, ref2, keep1, is_reg, row_off, lam) == K
+
+
+def test_lambda2_budget_on_oracle_scores_matches_the_threshold_rule():
+    """On oracle Stage-II scores, lambda2* of a budget gives that budget through O.threshold."""
+    b = tiny_batch(B=3, segs=2, P=(20, 13, 31), R=2, M=(5, 9, 2), seed=10)
+    out = O.prune(b, 0.9, 1.2)
+    m = b["meta"]
+    row_off = m["row_off_host"]
+    n_vis1 = int(np.sum(out["keep1"] & ~out["is_reg"]))
+    sample = np.repeat(np.arange(m["B"]), np.diff(row_off))
+    s2f = np.asarray(out["s2"], np.float32)
+    r2f = np.asarray(out["ref2"], np.float32)
+    for K in (1, n_vis1 // 3, n_vis1 - 1):
+        lam, _ = O.lambda2_for_budget(s2f, r2f, out["keep1"], out["is_reg"], row_off, K)
+        keep = O.threshold(s2f.astype(np.float64) / r2f[sample].astype(np.float64), np.ones(len(s2f)),
+                           float(lam), out["is_reg"], prev_keep=out["keep1"], keep_registers=False)
+        assert int(keep.sum()) == K
+
+
+# ----------------------------------------------------------------------------- register construction (Algorithm 1)
+
+def test_register_construction_properties():
+    """Per segment and register channel: the registers hold a value that bounds every visual entry and
+    equals one of them; the visual entries are 0; every other entry is untouched; the result does not
+    depend on the order of the visual rows."""
+    b = tiny_batch(B=2, segs=3, P=(9, 14), R=2, M=(2, 2), hidden=32, seed=61)
+    m = b["meta"]
+    h = b["hidden"].clone()
+    h[3, 5] = 40.0                                           # a sink-like activation
+    k_reg = np.array([5, 17, 30])
+    out = O.construct_registers(h, m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"], k_reg)
+    before = O.as_f64(h)
+    so, ri, ro = m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"]
+    other = np.setdiff1d(np.arange(before.shape[1]), k_reg)
+    assert np.array_equal(out[:, other], before[:, other])
+    for s in range(m["S_tot"]):
+        regs = ri[ro[s]:ro[s + 1]]
+        vis = np.setdiff1d(np.arange(so[s], so[s + 1]), regs)
+        for k in k_reg:
+            v = before[vis, k]
+            for r in regs:
+                assert all(out[r, k] >= x for x in v) and any(out[r, k] == x for x in v)
+            assert np.all(out[vis, k] == 0.0)
+    assert out[ri[ro[0]], 5] == 40.0 or 3 not in range(so[0], so[1])
+    # permuting the visual rows of a segment changes nothing at the registers
+    perm = before.copy()
+    vis0 = np.setdiff1d(np.arange(so[0], so[1]), ri[ro[0]:ro[1]])
+    perm[vis0] = perm[vis0[::-1]]
+    out2 = O.construct_registers(torch.from_numpy(perm), so, ri, ro, k_reg)
+    assert np.array_equal(out2[ri[ro[0]:ro[1]]][:, k_reg], out[ri[ro[0]:ro[1]]][:, k_reg])
