@@ -388,6 +388,40 @@ def run_ours(args, rank, world, local):
                          "input sets, the next step's copies overlapping the current step); K2, hidden, V "
                          "read in place (S1 rows of K2, kept rows of hidden and V)"}
 
+    # ---- the rows beyond the pruning path, timed on this workload's tensors
+    # (outside the step; not part of `value`)
+    next_rows = None
+    if not args.no_next:
+        def timed(fn, reps=20):
+            for _ in range(3):
+                fn()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(reps):
+                fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            return e0.elapsed_time(e1) / reps
+
+        K_tar = int(round(float(out["count_vis"].float().mean().item()) * meta["B"]))
+        lam_ms = timed(lambda: occ.occam_calibrate_lambda2(layout, out["s2"], out["ref2"], out["keep1"], K_tar,
+                                                             ws=call.ws))
+        lam, ncand = occ.occam_calibrate_lambda2(layout, out["s2"], out["ref2"], out["keep1"], K_tar, ws=call.ws)
+        k_reg = torch.tensor([7, 100, 511, 1000, 2047, 2048, 3000, 3333, 4000, 4095], dtype=torch.int32,
+                             device=dev)
+        h_copy = batch["hidden"].clone()
+        reg_ms = timed(lambda: occ.occam_construct_registers(layout, h_copy, k_reg, ws=call.ws))
+        del h_copy
+        next_rows = {
+            "lambda2_budget": {"ms": lam_ms, "target_rows": K_tar, "candidates": int(ncand.item()),
+                               "lambda2": float(lam.item()), "calibrated_lambda2": w.lambda2,
+                               "how": "radix select of the K-th largest s2/ref2 over the step's S1 rows"},
+            "register_construction": {"ms": reg_ms, "rows": meta["total_rows"], "channels": 10,
+                                      "how": "in place on hidden [rows, 4096] bf16, per segment"},
+            "n_eff": "computed in the Stage-I finalize of every timed step ([CLS] mode, optional output)",
+        }
+
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
@@ -438,6 +472,7 @@ def run_ours(args, rank, world, local):
         # the two-pass Stage-II pair, scan, gather
         "gpu_launches": (8 if w.stage1 == "cls" else 9) * args.steps,
         "clocks": clocks,
+        "next_rows": next_rows,
     }
     if world > 1:
         dist.destroy_process_group()
@@ -484,6 +519,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-next", action="store_true", help="skip timing the rows beyond the pruning path")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="synthetic workload to time (default: the LLaVA-NeXT batch-64 throughput workload)")
     args = ap.parse_args()
