@@ -151,9 +151,14 @@ def algorithmic_bytes(meta: dict, n1_total: int, kept_total: int) -> dict:
     k1row = H1 * d1 * 2
     k2row = H2 * d2 * 2
     hrow = hid * 2                       # bytes of one hidden / V row (bf16)
+    cls = meta["stage1"] == "cls"
     b = {}
-    b["stage1"] = rows * k1row + S * k1row + rows * H1 * 4           # K1 once, q_cls, logits write
-    b["stage1_finalize"] = rows * (H1 * 4 + 4 + 4 + 1 + 1 + 4) + S * k1row  # logits, s1 + s2 zero, role, keep1, list; q/k_cls
+    if cls:
+        b["stage1"] = rows * k1row + S * k1row + rows * H1 * 4           # K1 once, q_cls, logits write
+        b["stage1_finalize"] = rows * (H1 * 4 + 4 + 4 + 1 + 1 + 4) + S * k1row  # logits, s1 + s2 zero, role, keep1, list; q/k_cls
+    else:
+        b["stage1"] = 2 * rows * 2 * k1row                               # Q1 and K1 in each of the two passes
+        b["stage1_finalize"] = rows * (4 + 1 + 1 + 4)                   # s1, role, keep1, list
     b["s1_list_plan"] = 0                                            # planned inside the finalize kernel
     b["stage2_fused"] = n1_total * k2row + 2 * T * k2row               # S1 keys once, Q + K_text
     b["stage2_twopass"] = 2 * n1_total * k2row + 3 * T * k2row + 2 * T * H2 * 8  # both passes
@@ -161,7 +166,8 @@ def algorithmic_bytes(meta: dict, n1_total: int, kept_total: int) -> dict:
     b["gather"] = kept_total * 2 * (2 * hrow + k2row)                # read + write hidden, K, V rows
     # whole step, each byte once: K1, S1 keys, text Q/K, hidden+V of kept rows
     # (their K rows were read for scoring), writes of the 3 gathered rows
-    step = (rows * k1row + 2 * S * k1row + n1_total * k2row + 2 * T * k2row
+    stage1_in = rows * k1row + 2 * S * k1row if cls else 2 * rows * k1row   # K1 (+ q/k_cls) or Q1 + K1, once
+    step = (stage1_in + n1_total * k2row + 2 * T * k2row
             + kept_total * (2 * hrow) + kept_total * (2 * hrow + k2row) + rows + kept_total * 4)
     b["step"] = step
     return b
@@ -249,7 +255,10 @@ def run_ours(args, rank, world, local):
     layout = occ.BatchLayout.from_batch(batch, dev)
     K2flat = batch["K2"].view(batch["K2"].shape[0], -1)
     gather = (batch["hidden"], K2flat, batch["V"])
-    call = occ.PruneCall(layout, dict(mode="cls", q=batch["q_cls"], k_cls=batch["k_cls"], K1=batch["K1"]),
+    cls = w.stage1 == "cls"
+    stage1_of = ((lambda t: dict(mode="cls", q=t["q_cls"], k_cls=t["k_cls"], K1=t["K1"])) if cls else
+                 (lambda t: dict(mode="mutual", q=t["Q1"], K1=t["K1"])))
+    call = occ.PruneCall(layout, stage1_of(batch),
                          dict(Q_text=batch["Q_text"], K_text=batch["K_text"], K2=batch["K2"]),
                          w.lambda1, w.lambda2, keep_registers=True, gather=gather)
     stream = torch.cuda.current_stream()
@@ -262,7 +271,7 @@ def run_ours(args, rank, world, local):
     if st != 0:
         raise RuntimeError(f"device status {st} after warm-up")
     out = call.out
-    n1_total = int(out["n1_vis"].sum().item()) + int(meta["regs_per_seg"] * meta["S_tot"])
+    n1_total = int(out["n1_vis"].sum().item()) + int(meta["regs_per_seg"] * meta["S_tot"])  # registers are in S1
     kept_total = int(out["out_off"][-1].item())
     bytes_ = algorithmic_bytes(meta, n1_total, kept_total)
 
@@ -316,7 +325,7 @@ def run_ours(args, rank, world, local):
     # (counts, offsets, indices) are read back.
     e2e = None
     if not args.no_e2e:
-        copy_names = ["q_cls", "k_cls", "K1", "Q_text", "K_text"]
+        copy_names = (["q_cls", "k_cls"] if cls else ["Q1"]) + ["K1", "Q_text", "K_text"]
         host = {k: batch[k].cpu().pin_memory() for k in copy_names + ["K2", "hidden", "V"]}
         K2h = host["K2"]
         res_names = ["count_vis", "count_out", "out_off", "out_index"]
@@ -327,7 +336,7 @@ def run_ours(args, rank, world, local):
         for _ in range(nset):
             d = {k: torch.empty_like(batch[k]) for k in copy_names}
             dins.append(d)
-            hcalls.append(occ.PruneCall(layout, dict(mode="cls", q=d["q_cls"], k_cls=d["k_cls"], K1=d["K1"]),
+            hcalls.append(occ.PruneCall(layout, stage1_of(d),
                                         dict(Q_text=d["Q_text"], K_text=d["K_text"], K2=K2h),
                                         w.lambda1, w.lambda2, keep_registers=True,
                                         gather=(host["hidden"], K2h.view(K2h.shape[0], -1), host["V"]),
@@ -384,7 +393,7 @@ def run_ours(args, rank, world, local):
                "h2d_bytes_per_step": int(copied_bytes + in_place), "d2h_bytes_per_step": int(d2h),
                "steps": e_steps, "h2d_copied_bytes_per_step": int(copied_bytes),
                "h2d_read_in_place_bytes_per_step": int(in_place),
-               "inputs": "pinned host memory; q/k_cls, K1, Q_text, K_text copied each step (two device "
+               "inputs": f"pinned host memory; {', '.join(copy_names)} copied each step (two device "
                          "input sets, the next step's copies overlapping the current step); K2, hidden, V "
                          "read in place (S1 rows of K2, kept rows of hidden and V)"}
 

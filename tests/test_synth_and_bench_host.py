@@ -54,9 +54,14 @@ def _agg_worker(rank, world, port, out):
 
 def test_algorithmic_bytes_accounting():
     import bench
-    meta = dict(total_rows=1000, S_tot=5, total_text=100, H1=16, d1=64, H2=32, d2=128, hidden=4096)
+    meta = dict(total_rows=1000, S_tot=5, total_text=100, H1=16, d1=64, H2=32, d2=128, hidden=4096, stage1="cls")
     b = bench.algorithmic_bytes(meta, n1_total=200, kept_total=50)
     # K1 once, the [CLS] queries, 16 fp32 logits per row
     assert b["stage1"] == 1000 * 2048 + 5 * 2048 + 1000 * 16 * 4
     assert b["gather"] == 50 * 2 * 3 * 8192
     assert b["step"] > b["stage1"]
+    # mutual mode: Q1 and K1 in each of the two passes
+    mm = dict(meta, stage1="mutual", d1=72)
+    bm = bench.algorithmic_bytes(mm, n1_total=200, kept_total=50)
+    assert bm["stage1"] == 2 * 1000 * 2 * 16 * 72 * 2
+    assert bm["step"] > 2 * 1000 * 16 * 72 * 2
