@@ -11,30 +11,34 @@
 // TMEM lanes; each CTA owns 1/C of the sample's S1 keys and of the causal
 // text keys. Per head, a CTA's keys form one block of N <= 256 rows: its S1
 // keys (padded to a multiple of 32), then its text keys (padded to 16).
-//   1. seven producer warps gather the block's rows with 16-byte cp.async
-//      into the 128-byte-swizzled operand layout (S1 rows straight from K2 by
-//      index: pruned rows are never read); the head's 128 x 128 query tile
-//      arrives by TMA. Key blocks and query tiles are double-buffered by head;
-//   2. one thread issues S = Q K^T for the whole block as eight
+// Warp roles (512 threads):
+//   producers (warps 0-2): the block's S1 rows by TMA gather4 (four rows of
+//      one 128-byte K-block per copy, straight from K2 by index: pruned rows
+//      are never read), its text rows by 16-row TMA boxes, and the head's
+//      128 x 128 query tile by TMA, all into the 128-byte-swizzled operand
+//      layout; key blocks and query tiles are double-buffered by head;
+//   MMA issuer (warp 3): S = Q K^T for the whole block as eight
 //      128 x N x 16 tcgen05.mma (bf16 in, fp32 accumulate) into a per-head
 //      TMEM buffer E (two buffers, alternating by head);
-//   3. eight epilogue warps (two per TMEM lane quadrant, one thread per text
-//      row) each own every other 32-column piece of E. A warp turns its
-//      logits into exp2(l - cmax) (cmax: the row max of that piece, kept in a
-//      register), writes the S1-key ones back over the logits in E, and keeps
-//      the row's running softmax max / sum;
-//   4. the (max, sum) pairs go to every epilogue warp of the cluster with
-//      asynchronous distributed-shared-memory stores that complete on an
-//      mbarrier of the receiving CTA (no fences);
-//   5. every warp then adds exp2(cmax - max) / sum * E over its S1-key
-//      pieces to the head-summed probabilities P, which live in registers for
-//      the whole item.
-// Step s of the epilogue takes the text-key statistics of head s, adds head
-// s-1 into P (freeing head s-1's E buffer, so the MMAs of head s+1 overlap
-// the rest of step s), then the S1-key statistics of head s, and posts them.
-// After the last head every warp reduces its P columns over its 32 rows:
-// column max -> s2 (atomicMax on the fp32 bit pattern, exact and order-free
-// since P >= 0), register columns -> a partial of s2(r) reduced in fixed order.
+//   statistics warps (8, two per TMEM lane quadrant, one thread per text
+//      row): they split E's pieces (whole 64-column groups of S1 keys without
+//      masking, then the partial S1 piece and the causal text keys), turn
+//      the S1-key logits into exp2(l - group max) written back over E, keep
+//      the maxima in shared memory, and reduce the row's softmax max / sum;
+//      the quadrant's two warps merge theirs and post the row's log-sum
+//      L = max + log2(sum) to every CTA of the cluster with asynchronous
+//      distributed-shared-memory stores that complete on an mbarrier of the
+//      receiving CTA (no fences);
+//   probability warps (4, one per quadrant): once a head's statistics are
+//      done in this CTA and the cluster's log-sums are in, they add
+//      exp2(group max - M) / Z * E over the S1-key pieces to the head-summed
+//      probabilities P (registers, all of the CTA's S1 keys, the whole item),
+//      with sum_r exp2(L_r) = exp2(M) Z, and release E for the MMAs of the
+//      head after next.
+// After the last head the probability warps reduce their P columns over
+// their 32 rows: column max -> s2 (atomicMax on the fp32 bit pattern, exact
+// and order-free since P >= 0), register columns -> a partial of s2(r)
+// reduced in fixed order.
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc5.cuh"
@@ -74,14 +78,14 @@ template <int C>
 struct Geo {
   static constexpr int KROWS = C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;  // key rows per head (max MMA N)
   static constexpr int KBLK = KROWS * 128;                                  // bytes of one K-block of the key rows
-  static constexpr uint32_t XBYTES = C * QR * 8;                            // exchange bytes a CTA receives per head
+  static constexpr uint32_t XBYTES = C * QR * 4;                            // exchange bytes a CTA receives per head
 };
 
 template <int C>
 struct Smem {
   uint8_t q[2][QBYTES];
   uint8_t k[2][2 * Geo<C>::KBLK];
-  float2 xch[NXS][C][QR];    // (max, sum) per (slot, CTA, row)
+  float xch[NXS][C][QR];     // log2 of the row's exp2-sum over the CTA's keys, per (slot, CTA, row)
   float cmx[2][NPC][QR];     // per E buffer: the row max of each S1-key piece its exponentials are relative to
   float2 spart[2][4][32];    // per E buffer and lane quadrant: the second statistics warp's (max, sum)
   int32_t kidx[2][PMAX];
@@ -566,10 +570,13 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
           }
           const float2 o = sm.spart[eb][quad][lane];
           online_merge(m, z, o.x, o.y);
-          // post the row's (max, sum) to the probability warps of every CTA of the cluster
+          // post the row's log-sum L = m + log2(z) (log2 of the sum of exp2
+          // of its logits over this CTA's keys; -inf without keys) to the
+          // probability warps of every CTA of the cluster
+          const float L = z > 0.f ? m + tc::lg2(z) : -INFINITY;
           const int slot = hk & (NXS - 1);
 #pragma unroll
-          for (int r = 0; r < C; ++r) tc::st_async_f2(&sm.xch[slot][rank][j], &sm.xbar[slot], (uint32_t)r, m, z);
+          for (int r = 0; r < C; ++r) tc::st_async_f32(&sm.xch[slot][rank][j], &sm.xbar[slot], (uint32_t)r, L);
         }
       }
       if (!ok) { fail(sm, p.status); break; }
@@ -578,7 +585,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
     // ------------------------------------------------------------ probability warps
     // warp (quad) keeps P for text rows 32 quad .. 32 quad + 31 over all of
     // this CTA's S1 keys in registers. Per head, once the statistics warps
-    // are done with it and the cluster's (max, sum) pairs are in: P +=
+    // are done with it and the cluster's log-sums are in: P +=
     // exp2(cmx - max) / sum * E over the S1-key pieces; then E is released.
     tc::setmaxnreg_inc<REG_P>();
     const int pw = warp - P_WARP0;
@@ -618,16 +625,18 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         }
         tc::fence_after();
         if (wvalid) {
+          // the row's softmax denominator over the whole cluster:
+          // sum_r exp2(L_r) = exp2(Mx) * Z
           float Mx = -INFINITY;
 #pragma unroll
-          for (int r = 0; r < C; ++r) Mx = fmaxf(Mx, sm.xch[slot][r][j].x);
+          for (int r = 0; r < C; ++r) Mx = fmaxf(Mx, sm.xch[slot][r][j]);
           float Z = 0.f;
 #pragma unroll
           for (int r = 0; r < C; ++r) {
-            const float2 e = sm.xch[slot][r][j];
-            if (e.y > 0.f) Z = fmaf(e.y, tc::ex2(e.x - Mx), Z);
+            const float L = sm.xch[slot][r][j];
+            if (L != -INFINITY) Z += tc::ex2(L - Mx);
           }
-          // Z >= 1 (the row max contributes exp2(0)); hardware reciprocal
+          // Z >= 1 (the largest term is exp2(0)); hardware reciprocal
           const float invZ = (vrow && Z > 0.f) ? tc::rcp(Z) : 0.f;
           const uint32_t pbase = tmem + lane_base + eb * G::KROWS;
 #pragma unroll

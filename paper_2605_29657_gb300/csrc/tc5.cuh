@@ -236,6 +236,13 @@ __device__ __forceinline__ void setmaxnreg_inc() {
   asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
 }
 
+// log2(x) with the hardware approximation (absolute error about 2^-22 near 1)
+__device__ __forceinline__ float lg2(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // hardware reciprocal (relative error within 1 ulp), flushing subnormals
 __device__ __forceinline__ float rcp(float x) {
   float y;
@@ -270,6 +277,15 @@ __device__ __forceinline__ void st_async_f2(const void* local_addr, const uint64
       "st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [ra], {%3, %4}, [rb];\n\t}" ::"r"(
           su32(local_addr)),
       "r"(su32(bar)), "r"(rank), "f"(x), "f"(y)
+      : "memory");
+}
+__device__ __forceinline__ void st_async_f32(const void* local_addr, const uint64_t* bar, uint32_t rank, float x) {
+  asm volatile(
+      "{\n\t.reg .b32 ra, rb;\n\t"
+      "mapa.shared::cluster.u32 ra, %0, %2;\n\t"
+      "mapa.shared::cluster.u32 rb, %1, %2;\n\t"
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [ra], %3, [rb];\n\t}" ::"r"(su32(local_addr)),
+      "r"(su32(bar)), "r"(rank), "r"(__float_as_uint(x))
       : "memory");
 }
 __device__ __forceinline__ void st_cluster_u32(const void* local_addr, uint32_t rank, uint32_t x) {
