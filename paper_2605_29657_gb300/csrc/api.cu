@@ -56,11 +56,12 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   L.maxA = B * tps * nhg;
   L.maxB = B * tps * chmax;
   L.maxF = B * cdiv(b->max_text, 128);
-  L.maxSlots = L.maxB + L.maxF * kFusedSlotsPerItem8;
+  L.maxSlots = L.maxB + L.maxF * kFusedSlotsPerItem16;
   L.itemsA = take(L.maxA * 16);
   L.itemsB = take(L.maxB * 16);
   L.itemsF = take(L.maxF * 16);
   L.itemsF8 = take(L.maxF * 16);
+  L.itemsF16 = take(L.maxF * 16);
   L.itemB_off = take((B + 1) * 4);
   L.slot_off = take((B + 1) * 4);
   L.stats2 = take(T * (H2 > 0 ? H2 : 1) * 8);
@@ -413,6 +414,7 @@ Stage2Params stage2_params(const occam_batch* b, const occam_stage2_args* a, con
   const bool fused = fused_enabled() && L.maxF > 0 && b->total_text > 0;
   p.itemsF = at<int4>(ws, L.itemsF);
   p.itemsF8 = at<int4>(ws, L.itemsF8);
+  p.itemsF16 = at<int4>(ws, L.itemsF16);
   p.slot_off = at<int32_t>(ws, L.slot_off);
   p.maxF = L.maxF;
   p.use_fused = fused ? 1 : 0;
@@ -472,6 +474,15 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     // the two-pass kernels (samples the fused kernel cannot hold; often none)
     // follow the 8-CTA launch on the second stream
     launch_twopass(p, L, sms, side.stream);
+    // samples too large for 8 CTAs: 16-CTA clusters, on this stream ahead of
+    // the 4-CTA launch. A launch without items returns at once; it also
+    // lets the 8-CTA clusters (larger items) take their SMs first, which
+    // measured faster than starting the 4-CTA launch first.
+    Stage2TcParams q16 = q;
+    q16.items = p.itemsF16;
+    q16.queue = p.counters + CNT_QUEUE16;
+    const int ncl16 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 16));
+    if (launch_fused(16, mq, mk, mkt, q16, ncl16, st) != 0) return OCCAM_ERR_CUDA;
     q.queue = p.counters + CNT_QUEUE4;
     const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
     if (launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;

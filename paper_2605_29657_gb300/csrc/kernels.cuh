@@ -11,6 +11,7 @@ constexpr int kFusedCluster = 4;        // CTAs per cluster of the fused tcgen05
 constexpr int kFusedMaxOwnImg = 192;    // S1 keys one of its CTAs can hold (P columns kept in registers)
 constexpr int kFusedKeyRows4 = 256;     // key rows per head one CTA of a 4-CTA cluster holds (= MMA N and TMEM columns)
 constexpr int kFusedKeyRows8 = 224;     // the same for an 8-CTA cluster (its exchange buffers take more shared memory)
+constexpr int kFusedKeyRows16 = 224;    // and for a 16-CTA cluster (non-portable cluster size)
 constexpr int kFusedPartialWarps = 4;   // warps per CTA of the fused kernel that write an s2(r) partial
 constexpr int kFinalizeSmemRows = 1400; // Stage-I finalize stages a [CLS] segment in shared memory up to this many rows
 
@@ -19,13 +20,14 @@ constexpr int kFinalizeSmemRows = 1400; // Stage-I finalize stages a [CLS] segme
 // and, for the last text tile, ceil(M / C) causal text keys (padded to 16).
 // The kernel's item hand-off assumes at least 4 heads per item.
 __host__ __device__ inline bool fused_fits(int C, int n1, int M, int H) {
-  const int rows = C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;
+  const int rows = C == 16 ? kFusedKeyRows16 : C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;
   const int ip = ((n1 + C - 1) / C + 31) & ~31;
   const int tp = ((M + C - 1) / C + 15) & ~15;
   return M > 0 && H >= 4 && ip <= kFusedMaxOwnImg && ip + tp <= rows;
 }
 constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedPartialWarps;  // s2(r) partials per C=4 item
 constexpr int kFusedSlotsPerItem8 = 8 * kFusedPartialWarps;             // and per C=8 item
+constexpr int kFusedSlotsPerItem16 = 16 * kFusedPartialWarps;           // and per C=16 item
 
 struct Stage1ClsParams {
   BatchDev bt;
@@ -82,6 +84,7 @@ struct Stage2Params {
   int32_t* done;            // [B] finished score items per sample (zeroed)
   int4* itemsF;             // fused items for 4-CTA clusters (b, j0, slot, -)
   int4* itemsF8;            // fused items for 8-CTA clusters
+  int4* itemsF16;           // fused items for 16-CTA clusters
   int use_fused;            // route eligible samples to the fused tensor-core kernel
   int32_t* slot_off;        // [B+1] partial-slot range of each sample
   int64_t maxF;

@@ -9,17 +9,17 @@
 
 namespace occam {
 
-// Routes every sample (the fused tensor-core kernel with 4- or 8-CTA
+// Routes every sample (the fused tensor-core kernel with 4-, 8- or 16-CTA
 // clusters where its S1 keys and text keys fit, else the two-pass kernels)
 // and writes the item lists, the per-sample item and partial-slot offsets,
 // and the item counts. blockDim.x threads, tmp: >= 40 ints of shared memory.
 __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
   const int tid = threadIdx.x;
   const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
-  int runA = 0, runB = 0, runF = 0, runF8 = 0, runS = 0;
+  int runA = 0, runB = 0, runF = 0, runF8 = 0, runF16 = 0, runS = 0;
   for (int b0 = 0; b0 < p.bt.B; b0 += blockDim.x) {
     const int bb = b0 + tid;
-    int nA = 0, nB = 0, nF = 0, nF8 = 0;
+    int nA = 0, nB = 0, nF = 0, nF8 = 0, nF16 = 0;
     if (bb < p.bt.B) {
       const int M = (int)(p.bt.text_off[bb + 1] - p.bt.text_off[bb]);
       const int n1 = *((volatile int32_t*)&p.n1[bb]);
@@ -27,10 +27,13 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
       // causal text keys fit the cluster's TMEM / shared memory
       const bool fused4 = p.use_fused && fused_fits(kFusedCluster, n1, M, p.H);
       const bool fused8 = !fused4 && p.use_fused && fused_fits(8, n1, M, p.H);
+      const bool fused16 = !fused4 && !fused8 && p.use_fused && fused_fits(16, n1, M, p.H);
       if (fused4) {
         nF = (M + 127) / 128;
       } else if (fused8) {
         nF8 = (M + 127) / 128;
+      } else if (fused16) {
+        nF16 = (M + 127) / 128;
       } else {
         const int tiles = (M + kTextTile - 1) / kTextTile;
         const int nch = (n1 + kKeyChunk - 1) / kKeyChunk;
@@ -44,12 +47,14 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
       }
     }
     const int nch = (bb < p.bt.B) ? (*((volatile int32_t*)&p.n1[bb]) + kKeyChunk - 1) / kKeyChunk : 0;
-    const int nS = nF * kFusedSlotsPerItem + nF8 * kFusedSlotsPerItem8 + nB;  // s2(r) partial slots of this sample
-    int totA, totB, totF, totF8, totS;
+    const int nS = nF * kFusedSlotsPerItem + nF8 * kFusedSlotsPerItem8 + nF16 * kFusedSlotsPerItem16 +
+                   nB;  // s2(r) partial slots of this sample
+    int totA, totB, totF, totF8, totF16, totS;
     const int offA = runA + block_exclusive_scan(nA, tmp, &totA);
     const int offB = runB + block_exclusive_scan(nB, tmp, &totB);
     const int offF = runF + block_exclusive_scan(nF, tmp, &totF);
     const int offF8 = runF8 + block_exclusive_scan(nF8, tmp, &totF8);
+    const int offF16 = runF16 + block_exclusive_scan(nF16, tmp, &totF16);
     const int offS = runS + block_exclusive_scan(nS, tmp, &totS);
     if (bb < p.bt.B) {
       for (int i = 0; i < nA; ++i)
@@ -60,6 +65,8 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
         if (offF + i < p.maxF) p.itemsF[offF + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem, 0);
       for (int i = 0; i < nF8; ++i)
         if (offF8 + i < p.maxF) p.itemsF8[offF8 + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem8, 0);
+      for (int i = 0; i < nF16; ++i)
+        if (offF16 + i < p.maxF) p.itemsF16[offF16 + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem16, 0);
       p.itemB_off[bb] = offB;
       p.slot_off[bb] = offS;
     }
@@ -67,16 +74,19 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
     runB += totB;
     runF += totF;
     runF8 += totF8;
+    runF16 += totF16;
     runS += totS;
   }
   if (tid == 0) {
     p.itemB_off[p.bt.B] = runB;
     p.slot_off[p.bt.B] = runS;
-    if (runA > p.maxA || runB > p.maxB || runF > p.maxF || runF8 > p.maxF) set_status(p.status, OCCAM_ERR_CAPACITY);
+    if (runA > p.maxA || runB > p.maxB || runF > p.maxF || runF8 > p.maxF || runF16 > p.maxF)
+      set_status(p.status, OCCAM_ERR_CAPACITY);
     p.counters[CNT_NA] = (int)(runA < p.maxA ? runA : p.maxA);
     p.counters[CNT_NB] = (int)(runB < p.maxB ? runB : p.maxB);
     p.counters[CNT_NF] = (int)(runF < p.maxF ? runF : p.maxF);
     p.counters[CNT_NF8] = (int)(runF8 < p.maxF ? runF8 : p.maxF);
+    p.counters[CNT_NF16] = (int)(runF16 < p.maxF ? runF16 : p.maxF);
   }
 }
 

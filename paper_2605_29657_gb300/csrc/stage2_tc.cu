@@ -1,5 +1,5 @@
 // stage2_tc.cu -- fused Stage-II scoring on the 5th-generation tensor cores
-// (tcgen05 + TMEM), for samples whose S1 fits a 4- or 8-CTA cluster.
+// (tcgen05 + TMEM), for samples whose S1 fits a 4-, 8- or 16-CTA cluster.
 //
 // What it computes (Sec. 3.5, Eq. 7; App. A, Eqs. 15-16): for sample b, text
 // token j and head h, A_{j,h} = softmax over {S1 rows of b} u {text keys 0..j}
@@ -7,7 +7,7 @@
 // for visual S1 rows and the registers' sum_j P[j, r] / H for s2(r).
 //
 // Work item = (sample, tile of 128 text rows), processed by one cluster of C
-// CTAs (C = 4, or 8 for samples with more S1 keys). The text rows are the 128
+// CTAs (C = 4; 8 or 16 for samples with more S1 keys). The text rows are the 128
 // TMEM lanes; each CTA owns 1/C of the sample's S1 keys and of the causal
 // text keys. Per head, a CTA's keys form one block of N <= 256 rows: its S1
 // keys (padded to a multiple of 32), then its text keys (padded to 16).
@@ -69,14 +69,18 @@ constexpr int REG_NEEDED = S_WARP0 * 32 * REG_LOW + 8 * 32 * REG_S + NPW * 32 * 
 static_assert(S_WARP0 % 4 == 0 && P_WARP0 % 4 == 0 && NPW == 4, "roles split on warpgroup boundaries");
 static_assert(REG_NEEDED <= 65536, "register split exceeds the register file");
 constexpr uint32_t TMEM_COLS = 512;
-static_assert(2 * kFusedKeyRows4 <= (int)TMEM_COLS && 2 * kFusedKeyRows8 <= (int)TMEM_COLS, "two E buffers");
-static_assert(kFusedKeyRows4 % 32 == 0 && kFusedKeyRows8 % 32 == 0 && kFusedKeyRows4 <= 256, "MMA N <= 256");
+static_assert(2 * kFusedKeyRows4 <= (int)TMEM_COLS && 2 * kFusedKeyRows8 <= (int)TMEM_COLS &&
+                  2 * kFusedKeyRows16 <= (int)TMEM_COLS,
+              "two E buffers");
+static_assert(kFusedKeyRows4 % 32 == 0 && kFusedKeyRows8 % 32 == 0 && kFusedKeyRows16 % 32 == 0 &&
+                  kFusedKeyRows4 <= 256,
+              "MMA N <= 256");
 static_assert(PMAX % 32 == 0, "S1 keys in whole pieces");
 constexpr uint64_t kLimitNs = 2000000000ull;
 
 template <int C>
 struct Geo {
-  static constexpr int KROWS = C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;  // key rows per head (max MMA N)
+  static constexpr int KROWS = C == 16 ? kFusedKeyRows16 : C == 8 ? kFusedKeyRows8 : kFusedKeyRows4;  // max MMA N
   static constexpr int KBLK = KROWS * 128;                                  // bytes of one K-block of the key rows
   static constexpr uint32_t XBYTES = C * QR * 4;                            // exchange bytes a CTA receives per head
 };
@@ -99,8 +103,12 @@ struct Smem {
 };
 }  // namespace s2f
 
+static_assert(sizeof(s2f::Smem<16>) + 1024 <= 227 * 1024 && sizeof(s2f::Smem<8>) + 1024 <= 227 * 1024 &&
+                  sizeof(s2f::Smem<4>) + 1024 <= 227 * 1024,
+              "shared memory per CTA");
+
 int s2_fused_smem_bytes(int C) {
-  return (int)(C == 8 ? sizeof(s2f::Smem<8>) : sizeof(s2f::Smem<4>)) + 1024;
+  return (int)(C == 16 ? sizeof(s2f::Smem<16>) : C == 8 ? sizeof(s2f::Smem<8>) : sizeof(s2f::Smem<4>)) + 1024;
 }
 int s2_fused_threads() { return s2f::THREADS; }
 
@@ -312,7 +320,10 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   Smem<C>& sm = *reinterpret_cast<Smem<C>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rank = (int)tc::cluster_rank();
-  const int nF = p.counters[C == 8 ? CNT_NF8 : CNT_NF];
+  const int nF = p.counters[C == 16 ? CNT_NF16 : C == 8 ? CNT_NF8 : CNT_NF];
+  // no work for this cluster size (every CTA of every cluster reads the same
+  // count): leave before touching shared memory, TMEM or the cluster
+  if (nF == 0) return;
   volatile int* abort = &sm.abort;
 
   if (tid == 0) {
@@ -767,19 +778,14 @@ int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUte
   // the register split inside the kernel needs the launch to reserve at least
   // REG_NEEDED registers per CTA; refuse rather than launch a kernel whose
   // setmaxnreg.inc could never be satisfied
+  auto kern = C == 16 ? s2_fused_kernel<16> : C == 8 ? s2_fused_kernel<8> : s2_fused_kernel<4>;
   cudaFuncAttributes fa;
-  if ((C == 8 ? cudaFuncGetAttributes(&fa, s2_fused_kernel<8>) : cudaFuncGetAttributes(&fa, s2_fused_kernel<4>)) !=
-      cudaSuccess)
-    return 1;
+  if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) return 1;
   if (fa.numRegs * s2f::THREADS < s2f::REG_NEEDED) return 2;
-  cudaError_t e;
-  if (C == 8) {
-    cudaFuncSetAttribute(s2_fused_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(8));
-    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<8>, mq, mk, mkt, q);
-  } else {
-    cudaFuncSetAttribute(s2_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(4));
-    e = cudaLaunchKernelEx(&cfg, s2_fused_kernel<4>, mq, mk, mkt, q);
-  }
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(C));
+  // 16-CTA clusters exceed the portable limit of 8
+  if (C == 16) cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mq, mk, mkt, q);
   return e == cudaSuccess ? 0 : 1;
 }
 
