@@ -477,9 +477,9 @@ def run_ours(args, rank, world, local):
         "cpu_baseline": cpu,
         "e2e": e2e,
         # kernels per occam_prune call: Stage I (1 [CLS] / 2 mutual), finalize
-        # (with the Stage-II plan), fused Stage II with 4- and 8-CTA clusters,
-        # the two-pass Stage-II pair, scan, gather
-        "gpu_launches": (8 if w.stage1 == "cls" else 9) * args.steps,
+        # (with the Stage-II plan), fused Stage II with 16-, 8- and 4-CTA
+        # clusters, the two-pass Stage-II pair, scan, gather
+        "gpu_launches": (9 if w.stage1 == "cls" else 10) * args.steps,
         "clocks": clocks,
         "next_rows": next_rows,
     }
