@@ -195,6 +195,20 @@ bool encode_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, ui
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D bf16 map over a [rows, heads, dims] tensor, 128-byte swizzle, box of
+// 64 dims x 1 head x 128 rows; dims past `dims` read as zero.
+bool encode_map3(CUtensorMap* m, const void* base, int64_t rows, int heads, int dims) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t gdim[3] = {(cuuint64_t)dims, (cuuint64_t)heads, (cuuint64_t)rows};
+  cuuint64_t gstride[2] = {(cuuint64_t)dims * 2, (cuuint64_t)heads * dims * 2};
+  cuuint32_t box[3] = {64, 1, 128};
+  cuuint32_t es[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), gdim, gstride, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Stage-II path selection: the fused tensor-core kernel for every sample that
 // fits it (default), or the two-pass kernels for all samples when
 // OCCAM_STAGE2_PATH=twopass (used to test both paths on the same inputs).
@@ -227,7 +241,7 @@ int check_stage1(const occam_batch* b, const occam_stage1_args* a) {
   } else if (a->mode == OCCAM_STAGE1_MUTUAL) {
     if (a->H1 < 1 || a->H1 > 64) return OCCAM_ERR_UNSUPPORTED;
     if (a->d1 != 64 && a->d1 != 72 && a->d1 != 80) return OCCAM_ERR_UNSUPPORTED;
-    if (b->max_seg_rows > 65535 * kMutQTile) return OCCAM_ERR_UNSUPPORTED;
+    if (b->max_seg_rows > 65535 * 128 || b->S_tot > 65535) return OCCAM_ERR_UNSUPPORTED;
   } else {
     return OCCAM_ERR_INVALID_ARG;
   }
@@ -316,16 +330,21 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
     stage1_logits_kernel<<<grid, 256, stage1_logits_smem_bytes(), st>>>(p);
     trace.mark(st);
   } else {
-    MutualParams p;
+    MutualTcParams p;
     p.bt = bt;
     p.H = a->H1;
-    p.Q = static_cast<const __nv_bfloat16*>(a->q);
-    p.K = static_cast<const __nv_bfloat16*>(a->K1);
-    p.scale = (float)(1.0 / std::sqrt((double)a->d1));
-    p.stats = at<float2>(ws, L.stats1);
+    p.d1 = a->d1;
+    p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)a->d1));
+    p.inv_h = 1.0f / (float)a->H1;
+    p.lsum = at<float>(ws, L.stats1);
     p.s1 = s1;
     p.s2_zero = s2_zero;
-    launch_mutual(p, a->d1, b->S_tot, b->max_seg_rows, st);
+    p.status = status;
+    // Q1 and K1 as [rows, H1, d1]: boxes of 64 dims x 1 head x 128 rows
+    CUtensorMap mq, mk;
+    if (!encode_map3(&mq, a->q, b->total_rows, a->H1, a->d1) || !encode_map3(&mk, a->K1, b->total_rows, a->H1, a->d1))
+      return OCCAM_ERR_CUDA;
+    launch_mutual_tc(p, mq, mk, b->S_tot, b->max_seg_rows, st);
     trace.mark(st);
   }
   return cuda_ok();

@@ -216,8 +216,6 @@ constexpr int kTextTile = 64;    // Stage-II text rows per item
 constexpr int kHeadGroup = 8;    // Stage-II heads per stats item
 constexpr int kKeyChunk = 128;   // Stage-II image keys per score item
 constexpr int kScanTile = 2048;  // compaction rows per scan tile (256 threads x 8)
-constexpr int kMutQTile = 64;    // mutual-mode query rows per stats item
-constexpr int kMutKChunk = 128;  // mutual-mode keys per column-sum item
 constexpr uint32_t kSpinLimit = 1u << 22;
 
 struct BatchDev {

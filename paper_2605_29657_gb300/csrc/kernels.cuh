@@ -39,16 +39,19 @@ struct Stage1ClsParams {
 };
 
 
-struct MutualParams {
+// Mutual Stage I on the tensor cores (stage1_tc.cu)
+struct MutualTcParams {
   BatchDev bt;
   int H;
-  const __nv_bfloat16* Q;
-  const __nv_bfloat16* K;
-  float scale;
-  float2* stats;  // [rows, H] (max in log2 units, 1/sum)
+  int d1;
+  float scale_log2;  // log2(e) / sqrt(d1)
+  float inv_h;       // 1 / H
+  float* lsum;       // [H, total_rows] per query row and head: log2 of its softmax denominator (log2 domain)
   float* s1;
-  float* s2_zero;
+  float* s2_zero;    // nullable
+  int* status;
 };
+
 
 struct ThresholdParams {
   BatchDev bt;
@@ -226,8 +229,8 @@ struct Stage2TcParams {
 __global__ void stage1_logits_kernel(Stage1ClsParams p);
 int stage1_logits_smem_bytes();
 __global__ void stage1_finalize_kernel(Stage1FinalizeParams p);
-int mutual_colsum_smem_bytes(int DP);
-void launch_mutual(const MutualParams& p, int d1, int S_tot, int max_seg_rows, cudaStream_t st);
+void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, int S_tot,
+                      int max_seg_rows, cudaStream_t st);
 __global__ void roles_scatter_kernel(BatchDev bt, uint8_t* role);
 __global__ void threshold_kernel(ThresholdParams p);
 

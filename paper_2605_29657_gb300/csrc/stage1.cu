@@ -382,232 +382,6 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   }
 }
 
-// ============================================================================
-// Mutual scoring (Sec. 3.4, Eq. 6): every row u of a segment attends to every
-// row v of the segment, per head. Two passes over the keys:
-//   pass 1 (mutual_stats_kernel): per query row and head the softmax max and
-//          sum over the segment's keys (online, flash-style);
-//   pass 2 (mutual_colsum_kernel): per key chunk, sum over all query rows and
-//          heads of exp(l - m)/Z, i.e. the attention each key receives.
-// Both passes run QK^T on the tensor cores (mma.sync m16n8k16, bf16 in, fp32
-// accumulate). d1 is zero-padded to DP (a multiple of 16).
-// ============================================================================
-namespace mut {
-constexpr int kThreads = 128;  // 4 warps x 16 query rows
-}
-
-template <int D, int DP>
-__device__ __forceinline__ void load_rows_tile(__nv_bfloat16* sdst, const __nv_bfloat16* base,
-                                               int64_t row0, int nrows_valid, int nrows_tile,
-                                               int row_stride_elems, int head, int tid, int nthreads) {
-  // copies rows [row0, row0+nrows_tile) of head `head` into sdst[r][0..DP) (row
-  // stride DP+8); rows past nrows_valid and dims past D are zero.
-  constexpr int LD = DP + 8;
-  constexpr int VPR = DP / 8;  // 16-byte vectors per row
-  for (int i = tid; i < nrows_tile * VPR; i += nthreads) {
-    const int r = i / VPR, v = i % VPR;
-    __nv_bfloat16* dst = sdst + r * LD + v * 8;
-    const bool ok = (r < nrows_valid) && (v * 8 < D);
-    const __nv_bfloat16* src =
-        ok ? base + (row0 + r) * (int64_t)row_stride_elems + (int64_t)head * D + v * 8 : base;
-    cp_async16_zfill(dst, src, ok ? 16 : 0);
-  }
-}
-
-template <int DP, int NT>
-__device__ __forceinline__ void warp_qk(float (&S)[NT][4], const __nv_bfloat16* sQ, int q_row0,
-                                        const __nv_bfloat16* sK, int k_row0, int lane) {
-  constexpr int LD = DP + 8;
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) S[nt][0] = S[nt][1] = S[nt][2] = S[nt][3] = 0.f;
-#pragma unroll
-  for (int kk = 0; kk < DP / 16; ++kk) {
-    uint32_t a[4];
-    ldmatrix_x4(a, sQ + (q_row0 + (lane & 7) + ((lane >> 3) & 1) * 8) * LD + kk * 16 + ((lane >> 4) & 1) * 8);
-#pragma unroll
-    for (int nt = 0; nt < NT; nt += 2) {
-      uint32_t b[4];
-      ldmatrix_x4(b, sK + (k_row0 + nt * 8 + (lane & 7) + ((lane >> 4) & 1) * 8) * LD + kk * 16 +
-                         ((lane >> 3) & 1) * 8);
-      mma_bf16_16816(S[nt], a, b[0], b[1]);
-      mma_bf16_16816(S[nt + 1], a, b[2], b[3]);
-    }
-  }
-}
-
-template <int D, int DP>
-__global__ void __launch_bounds__(mut::kThreads) mutual_stats_kernel(MutualParams p) {
-  constexpr int LD = DP + 8;
-  constexpr int KT = 64;  // keys per chunk
-  __shared__ __align__(128) __nv_bfloat16 sQ[kMutQTile * LD];
-  __shared__ __align__(128) __nv_bfloat16 sK[2][KT * LD];
-  const int seg = blockIdx.x;
-  const int qt = blockIdx.y;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t sb = p.bt.seg_off[seg], se = p.bt.seg_off[seg + 1];
-  const int n = (int)(se - sb);
-  const int q0 = qt * kMutQTile;
-  if (q0 >= n) return;
-  const int nq = min(kMutQTile, n - q0);
-  const int HD = p.H * D;
-  const float c = p.scale * 1.4426950408889634f;  // log2(e) folded into the scale
-  const int nchunks = (n + KT - 1) / KT;
-  for (int h = blockIdx.z; h < p.H; h += gridDim.z) {
-    load_rows_tile<D, DP>(sQ, p.Q, sb + q0, nq, kMutQTile, HD, h, tid, mut::kThreads);
-    load_rows_tile<D, DP>(sK[0], p.K, sb, min(KT, n), KT, HD, h, tid, mut::kThreads);
-    cp_async_commit();
-    float m[2] = {-INFINITY, -INFINITY}, z[2] = {0.f, 0.f};  // rows g and g+8 (log2 domain max)
-    for (int kc = 0; kc < nchunks; ++kc) {
-      if (kc + 1 < nchunks) {
-        load_rows_tile<D, DP>(sK[(kc + 1) & 1], p.K, sb + (kc + 1) * KT, min(KT, n - (kc + 1) * KT), KT, HD,
-                              h, tid, mut::kThreads);
-      }
-      cp_async_commit();
-      cp_async_wait<1>();
-      __syncthreads();
-      float S[8][4];
-      warp_qk<DP, 8>(S, sQ, warp * 16, sK[kc & 1], 0, lane);
-      const int kbase = kc * KT;
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        float cm = -INFINITY;
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const int key = kbase + nt * 8 + (lane & 3) * 2 + e;
-            const float x = (key < n) ? S[nt][half * 2 + e] * c : -INFINITY;
-            S[nt][half * 2 + e] = x;
-            cm = fmaxf(cm, x);
-          }
-        cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 1));
-        cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 2));
-        const float mn = fmaxf(m[half], cm);
-        float acc = 0.f;
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-          for (int e = 0; e < 2; ++e) acc += exp2f(S[nt][half * 2 + e] - mn);
-        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
-        z[half] = (m[half] == -INFINITY ? 0.f : z[half] * exp2f(m[half] - mn)) + acc;
-        m[half] = mn;
-      }
-      __syncthreads();
-    }
-    if ((lane & 3) == 0) {
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const int r = warp * 16 + (lane >> 2) + half * 8;
-        if (r < nq) p.stats[(sb + q0 + r) * p.H + h] = make_float2(m[half], 1.0f / z[half]);
-      }
-    }
-    __syncthreads();
-  }
-}
-
-template <int D, int DP>
-__global__ void __launch_bounds__(256) mutual_colsum_kernel(MutualParams p) {
-  constexpr int LD = DP + 8;
-  constexpr int KC = kMutKChunk;  // 128 keys: warp w -> rows (w&3)*16, keys (w>>2)*64
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  __nv_bfloat16* sK = reinterpret_cast<__nv_bfloat16*>(smem_raw);            // [2][KC][LD] (by head parity)
-  __nv_bfloat16* sQ = sK + 2 * KC * LD;                                      // [2][64][LD]
-  float2* sst = reinterpret_cast<float2*>(sQ + 2 * kMutQTile * LD);          // [2][64]
-  float* colsum = reinterpret_cast<float*>(sst + 2 * kMutQTile);             // [4][KC]
-  const int seg = blockIdx.x;
-  const int kc = blockIdx.y;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int rb = warp & 3, kh = warp >> 2;
-  const int64_t sb = p.bt.seg_off[seg], se = p.bt.seg_off[seg + 1];
-  const int n = (int)(se - sb);
-  const int k0 = kc * KC;
-  if (k0 >= n) return;
-  const int nk = min(KC, n - k0);
-  const int HD = p.H * D;
-  const float c = p.scale * 1.4426950408889634f;
-  const int nqt = (n + kMutQTile - 1) / kMutQTile;
-  float P[8][4];
-#pragma unroll
-  for (int nt = 0; nt < 8; ++nt) P[nt][0] = P[nt][1] = P[nt][2] = P[nt][3] = 0.f;
-  const int njobs = p.H * nqt;  // (head, query tile) pairs, head-major
-  auto issue = [&](int job, int buf) {
-    const int h = job / nqt, qt = job % nqt;
-    if (qt == 0) load_rows_tile<D, DP>(sK + (h & 1) * KC * LD, p.K, sb + k0, nk, KC, HD, h, tid, 256);
-    load_rows_tile<D, DP>(sQ + buf * kMutQTile * LD, p.Q, sb + qt * kMutQTile, min(kMutQTile, n - qt * kMutQTile),
-                          kMutQTile, HD, h, tid, 256);
-    for (int i = tid; i < kMutQTile; i += 256) {
-      const int r = qt * kMutQTile + i;
-      sst[buf * kMutQTile + i] = (r < n) ? p.stats[(sb + r) * p.H + h] : make_float2(0.f, 0.f);
-    }
-  };
-  issue(0, 0);
-  cp_async_commit();
-  for (int job = 0; job < njobs; ++job) {
-    const int buf = job & 1;
-    const int qt = job % nqt;
-    const int h = job / nqt;
-    if (job + 1 < njobs) issue(job + 1, buf ^ 1);
-    cp_async_commit();
-    cp_async_wait<1>();
-    __syncthreads();
-    float S[8][4];
-    warp_qk<DP, 8>(S, sQ + buf * kMutQTile * LD, rb * 16, sK + (h & 1) * KC * LD, kh * 64, lane);
-    const int rowA = rb * 16 + (lane >> 2);
-    const float2 stA = sst[buf * kMutQTile + rowA];
-    const float2 stB = sst[buf * kMutQTile + rowA + 8];
-    const bool vA = qt * kMutQTile + rowA < n, vB = qt * kMutQTile + rowA + 8 < n;
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        if (vA) P[nt][e] += exp2f(fmaf(S[nt][e], c, -stA.x)) * stA.y;
-        if (vB) P[nt][2 + e] += exp2f(fmaf(S[nt][2 + e], c, -stB.x)) * stB.y;
-      }
-    }
-    __syncthreads();  // buffers of this job are reused by the loads issued next iteration
-  }
-  // column sums over the 16 row slots of each warp, then over the 4 row blocks
-#pragma unroll
-  for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      float v = P[nt][e] + P[nt][2 + e];
-      v += __shfl_xor_sync(0xffffffffu, v, 4);
-      v += __shfl_xor_sync(0xffffffffu, v, 8);
-      v += __shfl_xor_sync(0xffffffffu, v, 16);
-      if ((lane >> 2) == 0) colsum[rb * KC + kh * 64 + nt * 8 + (lane & 3) * 2 + e] = v;
-    }
-  }
-  __syncthreads();
-  const float norm = 1.0f / ((float)p.H * (float)n);
-  for (int k = tid; k < nk; k += 256) {
-    const float v = (colsum[k] + colsum[KC + k]) + (colsum[2 * KC + k] + colsum[3 * KC + k]);
-    p.s1[sb + k0 + k] = v * norm;
-    if (p.s2_zero) p.s2_zero[sb + k0 + k] = 0.f;
-  }
-}
-
-int mutual_colsum_smem_bytes(int DP) {
-  const int LD = DP + 8;
-  return (2 * kMutKChunk * LD + 2 * kMutQTile * LD) * 2 + 2 * kMutQTile * 8 + 4 * kMutKChunk * 4;
-}
-
-template <int D, int DP>
-static void launch_mutual_t(const MutualParams& p, int S_tot, int max_seg_rows, cudaStream_t st) {
-  const int qtiles = (max_seg_rows + kMutQTile - 1) / kMutQTile;
-  const int kchunks = (max_seg_rows + kMutKChunk - 1) / kMutKChunk;
-  const int smem = mutual_colsum_smem_bytes(DP);
-  cudaFuncSetAttribute(mutual_colsum_kernel<D, DP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  mutual_stats_kernel<D, DP><<<dim3(S_tot, qtiles, p.H), mut::kThreads, 0, st>>>(p);
-  mutual_colsum_kernel<D, DP><<<dim3(S_tot, kchunks), 256, smem, st>>>(p);
-}
-
-void launch_mutual(const MutualParams& p, int d1, int S_tot, int max_seg_rows, cudaStream_t st) {
-  if (d1 == 64) launch_mutual_t<64, 64>(p, S_tot, max_seg_rows, st);
-  else if (d1 == 72) launch_mutual_t<72, 80>(p, S_tot, max_seg_rows, st);
-  else launch_mutual_t<80, 80>(p, S_tot, max_seg_rows, st);
-}
 
 // ============================================================================
 // Row roles (0 visual, 1 register) from the register lists; the role array

@@ -1,0 +1,307 @@
+// stage1_tc.cu -- mutual Stage-I scoring on the 5th-generation tensor cores
+// (tcgen05 + TMEM + TMA).
+//
+// What it computes (Sec. 3.4, Eq. 6; App. A, Eq. 13): in segment s with n
+// rows, every row u attends to every row v per head h with
+// A_h(u -> v) = softmax_v(q_{u,h} k_{v,h} / sqrt(d1)), and
+// s1[v] = 1/n sum_u 1/H sum_h A_h(u -> v).
+// Two launches of one kernel template:
+//   pass 1: per (segment, tile of 128 query rows, head) the query rows'
+//           softmax log-sums L[h][u] = log2 sum_v exp2(c q_u k_v), with
+//           c = log2(e) / sqrt(d1), over all the segment's keys;
+//   pass 2: per (segment, tile of 128 key rows) the attention each key
+//           receives, sum_h sum_u exp2(c q_u k_v - L[h][u]), over all heads
+//           and query rows.
+// In both, the CTA's 128 tile rows are the TMEM lanes (the MMA's A operand)
+// and the other side streams in blocks of 256 rows (the B operand):
+// S = A B^T is 128 x 256 fp32 in TMEM, from 4-5 tcgen05.mma of K = 16.
+// Q1 and K1 are read as 3-D TMA boxes {64 dims, 1 head, 128 rows} with the
+// 128-byte swizzle; dims past d1 (72 -> 80) come zero-filled by the box, so
+// the padded K-steps add nothing.
+// Roles (384 threads): warp 0 issues the TMA loads, warp 1 the MMAs, warps
+// 4-11 (two per TMEM lane quadrant, each taking 128 of the 256 columns) the
+// softmax arithmetic. A tiles, B blocks and the TMEM accumulator are double
+// buffered. Every wait is bounded; on a timeout the CTA records
+// OCCAM_ERR_TIMEOUT, lets its copies land, frees TMEM and returns.
+#include "common.cuh"
+#include "kernels.cuh"
+#include "tc5.cuh"
+
+namespace occam {
+
+namespace m1 {
+constexpr int AR = 128;                   // tile rows (TMEM lanes)
+constexpr int BR = 256;                   // block rows (MMA N)
+constexpr int ABYTES = AR * 128;          // one K-block of an A tile
+constexpr int BBYTES = BR * 128;          // one K-block of a B block
+constexpr int THREADS = 384;
+constexpr int EPI0 = 4;                   // first epilogue warp
+constexpr uint64_t kLimitNs = 2000000000ull;
+
+struct Smem {
+  uint8_t a[2][2][ABYTES];  // [buffer][K-block]
+  uint8_t b[2][2][BBYTES];
+  float lsm[8][128];        // pass 2: log-sums of each epilogue warp's 128 columns
+  float2 part[2][4][32];    // second-half partials per (item parity, quadrant, lane)
+  uint64_t afull[2], aempty[2], bfull[2], bempty[2], dfull[2], dfree[2], hb[4], mdone;
+  uint32_t tmem_base;
+  int abort;
+};
+}  // namespace m1
+
+int mutual_tc_smem_bytes() { return (int)sizeof(m1::Smem) + 1024; }
+
+namespace {
+
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+      "[%5];" ::"r"(tc::su32(dst)),
+      "l"(map), "r"(x), "r"(y), "r"(z), "r"(tc::su32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void wait_ld64(uint32_t (&v)[64]) {
+  tc::tmem_wait_ld();
+  asm volatile("" : OCCAM_TC_RW64(v));
+}
+
+}  // namespace
+
+// PASS 1: A = query tiles, B = key blocks, one head per CTA (blockIdx.y).
+// PASS 2: A = key tiles, B = query blocks, all heads.
+template <int PASS>
+__global__ void __launch_bounds__(m1::THREADS, 1)
+    mutual_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+                     MutualTcParams p) {
+  using namespace m1;
+  extern __shared__ unsigned char smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int seg = blockIdx.z;
+  const int64_t sb = p.bt.seg_off[seg];
+  const int n = (int)(p.bt.seg_off[seg + 1] - sb);
+  const int a0 = blockIdx.x * AR;
+  if (a0 >= n) return;  // uniform over the CTA, before any shared state
+  const int H = p.H;
+  const int nb = (n + BR - 1) / BR;
+  const int nheads = PASS == 1 ? 1 : H;
+  const int steps = nheads * nb;
+  const int nkb = p.d1 > 64 ? 2 : 1;         // K-blocks of 64 dims
+  const int nks = (p.d1 + 15) / 16;          // K-steps of 16 dims
+  volatile int* abort = &sm.abort;
+
+  if (tid == 0) {
+    for (int i = 0; i < 2; ++i) {
+      tc::bar_init(&sm.afull[i], 1);
+      tc::bar_init(&sm.aempty[i], 1);
+      tc::bar_init(&sm.bfull[i], 1);
+      tc::bar_init(&sm.bempty[i], 1);
+      tc::bar_init(&sm.dfull[i], 1);
+      tc::bar_init(&sm.dfree[i], 8);
+    }
+    for (int i = 0; i < 4; ++i) tc::bar_init(&sm.hb[i], 1);
+    tc::bar_init(&sm.mdone, 1);
+    sm.abort = 0;
+    tc::bar_fence_init();
+    tc::prefetch_map(&mapA);
+    tc::prefetch_map(&mapB);
+  }
+  if (warp == 1) tc::tmem_alloc(&sm.tmem_base, 512);
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem = sm.tmem_base;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      uint32_t na = 0, nbk = 0;
+      for (int s = 0; s < steps && !*abort; ++s) {
+        const int h = PASS == 1 ? (int)blockIdx.y : s / nb;
+        const int jb = s % nb;
+        if (jb == 0) {
+          const int ab = na & 1;
+          if (!tc::bar_wait(&sm.aempty[ab], ((na >> 1) & 1) ^ 1, abort, kLimitNs)) {
+            sm.abort = 1;
+            set_status(p.status, OCCAM_ERR_TIMEOUT);
+            break;
+          }
+          tc::bar_expect_tx(&sm.afull[ab], (uint32_t)(nkb * ABYTES));
+          for (int kb = 0; kb < nkb; ++kb)
+            tma_load_3d(sm.a[ab][kb], &mapA, kb * 64, h, (int)(sb + a0), &sm.afull[ab]);
+          ++na;
+        }
+        const int bb = nbk & 1;
+        if (!tc::bar_wait(&sm.bempty[bb], ((nbk >> 1) & 1) ^ 1, abort, kLimitNs)) {
+          sm.abort = 1;
+          set_status(p.status, OCCAM_ERR_TIMEOUT);
+          break;
+        }
+        tc::bar_expect_tx(&sm.bfull[bb], (uint32_t)(nkb * BBYTES));
+        for (int kb = 0; kb < nkb; ++kb)
+          for (int hh = 0; hh < BR / AR; ++hh)
+            tma_load_3d(sm.b[bb][kb] + hh * ABYTES, &mapB, kb * 64, h, (int)(sb + jb * BR + hh * AR), &sm.bfull[bb]);
+        ++nbk;
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = tc::idesc_bf16(AR, BR);
+      uint32_t na = 0;
+      for (int s = 0; s < steps; ++s) {
+        const int jb = s % nb;
+        const int ab = na & 1, bb = s & 1, db = s & 1;
+        bool ok = true;
+        if (jb == 0) ok = tc::bar_wait(&sm.afull[ab], (na >> 1) & 1, abort, kLimitNs);
+        if (ok) ok = tc::bar_wait(&sm.bfull[bb], (s >> 1) & 1, abort, kLimitNs);
+        if (ok && s >= 2) ok = tc::bar_wait(&sm.dfree[db], ((s - 2) >> 1) & 1, abort, kLimitNs);
+        if (!ok) {
+          sm.abort = 1;
+          set_status(p.status, OCCAM_ERR_TIMEOUT);
+          break;
+        }
+        tc::fence_after();
+        const uint32_t abase = tc::su32(sm.a[ab][0]), bbase = tc::su32(sm.b[bb][0]);
+        for (int ks = 0; ks < nks; ++ks) {
+          const int kb = ks >> 2, kk = ks & 3;
+          tc::mma_bf16(tmem + db * BR, tc::sdesc_sw128(abase + kb * ABYTES + kk * 32),
+                       tc::sdesc_sw128(bbase + kb * BBYTES + kk * 32), idesc, ks > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(&sm.dfull[db]);
+        tc::mma_commit(&sm.bempty[bb]);
+        if (jb == nb - 1) {
+          tc::mma_commit(&sm.aempty[ab]);
+          ++na;
+        }
+      }
+      tc::mma_commit(&sm.mdone);
+      if (!tc::bar_wait(&sm.mdone, 0, nullptr, kLimitNs)) set_status(p.status, OCCAM_ERR_TIMEOUT);
+    }
+    __syncwarp();
+  } else if (warp >= EPI0) {
+    // ------------------------------------------------------------ softmax warps
+    const int ew = warp - EPI0;
+    const int quad = warp & 3, half = ew >> 2;
+    const int row = quad * 32 + lane;                   // tile row = TMEM lane
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    const float c = p.scale_log2;
+    const bool vrow = a0 + row < n;
+    const int64_t R = p.bt.total_rows;
+    float m = -INFINITY, z = 0.f;  // pass 1: running max / sum (log2 domain)
+    float acc = 0.f;               // pass 2: attention received by this key row
+    bool ok = true;
+    for (int s = 0; s < steps && ok; ++s) {
+      const int h = PASS == 1 ? (int)blockIdx.y : s / nb;
+      const int jb = s % nb;
+      const int col0 = jb * BR + half * 128;            // segment-relative index of this warp's column 0
+      if (PASS == 2) {
+        // log-sums of this warp's 128 query columns; past the segment: +inf (contributes 0)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int qq = col0 + lane * 4 + i;
+          sm.lsm[ew][lane * 4 + i] = qq < n ? __ldcg(&p.lsum[(int64_t)h * R + sb + qq]) : INFINITY;
+        }
+        __syncwarp();
+      }
+      const int db = s & 1;
+      if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.dfull[db], (s >> 1) & 1, nullptr, kLimitNs))) {
+        ok = false;
+        break;
+      }
+      tc::fence_after();
+#pragma unroll
+      for (int g = 0; g < 2; ++g) {
+        uint32_t v[64];
+        tc::tmem_ld64(tmem + lane_base + db * BR + half * 128 + g * 64, v);
+        wait_ld64(v);
+        if (PASS == 1) {
+          // keys past the segment are masked out of this row's softmax
+          const int lim = n - (col0 + g * 64);
+          float mx = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < 64; ++i) {
+            const float x = i < lim ? __uint_as_float(v[i]) * c : -INFINITY;
+            v[i] = __float_as_uint(x);
+            mx = fmaxf(mx, x);
+          }
+          if (mx != -INFINITY) {
+            float ap[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int i = 0; i < 64; ++i) ap[i & 7] += tc::ex2(__uint_as_float(v[i]) - mx);
+            const float a = ((ap[0] + ap[1]) + (ap[2] + ap[3])) + ((ap[4] + ap[5]) + (ap[6] + ap[7]));
+            const bool up = mx > m;
+            const float e = tc::ex2(up ? m - mx : mx - m);
+            z = up ? fmaf(z, e, a) : fmaf(a, e, z);
+            m = fmaxf(m, mx);
+          }
+        } else {
+          const float* L = sm.lsm[ew] + g * 64;
+          float ap[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int i = 0; i < 64; ++i) ap[i & 7] += tc::ex2(fmaf(__uint_as_float(v[i]), c, -L[i]));
+          acc += ((ap[0] + ap[1]) + (ap[2] + ap[3])) + ((ap[4] + ap[5]) + (ap[6] + ap[7]));
+        }
+      }
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) tc::bar_arrive(&sm.dfree[db]);
+    }
+    if (!ok) {
+      sm.abort = 1;
+      set_status(p.status, OCCAM_ERR_TIMEOUT);
+    } else {
+      // the two halves of each row: the second hands its partial to the first
+      if (half == 1) {
+        sm.part[0][quad][lane] = make_float2(PASS == 1 ? m : acc, z);
+        __syncwarp();
+        if (lane == 0) tc::bar_arrive(&sm.hb[quad]);
+      } else if (__all_sync(0xffffffffu, tc::bar_wait(&sm.hb[quad], 0, nullptr, kLimitNs))) {
+        const float2 o = sm.part[0][quad][lane];
+        if (PASS == 1) {
+          if (o.x != -INFINITY) {
+            const bool up = o.x > m;
+            const float e = tc::ex2(up ? m - o.x : o.x - m);
+            z = up ? fmaf(z, e, o.y) : fmaf(o.y, e, z);
+            m = fmaxf(m, o.x);
+          }
+          // L = log2 of the row's sum of exp2(c q k) over the segment's keys
+          if (vrow) p.lsum[(int64_t)blockIdx.y * R + sb + a0 + row] = m + log2f(z);
+        } else if (vrow) {
+          p.s1[sb + a0 + row] = (acc + o.x) * p.inv_h / (float)n;
+          if (p.s2_zero) p.s2_zero[sb + a0 + row] = 0.f;
+        }
+      } else {
+        sm.abort = 1;
+        set_status(p.status, OCCAM_ERR_TIMEOUT);
+      }
+    }
+  }
+
+  // ------------------------------------------------------------ teardown
+  tc::fence_before();
+  __syncthreads();
+  if (sm.abort && tid == 0) {
+    // let the TMA copies still in flight land before the CTA's shared memory goes away
+    const uint64_t t0 = tc::globaltimer();
+    while (tc::globaltimer() - t0 < 100000ull) {
+    }
+  }
+  __syncthreads();
+  tc::fence_after();
+  if (warp == 1) tc::tmem_dealloc(tmem, 512);
+}
+
+void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, int S_tot,
+                      int max_seg_rows, cudaStream_t st) {
+  const int tiles = (max_seg_rows + m1::AR - 1) / m1::AR;
+  const int smem = mutual_tc_smem_bytes();
+  cudaFuncSetAttribute(mutual_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaFuncSetAttribute(mutual_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  mutual_tc_kernel<1><<<dim3(tiles, p.H, S_tot), m1::THREADS, smem, st>>>(mq, mk, p);
+  mutual_tc_kernel<2><<<dim3(tiles, 1, S_tot), m1::THREADS, smem, st>>>(mk, mq, p);
+}
+
+}  // namespace occam
