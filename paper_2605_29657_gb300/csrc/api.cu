@@ -195,18 +195,19 @@ bool encode_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, ui
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// 3-D bf16 map over a [rows, heads, dims] tensor, 128-byte swizzle, box of
-// 64 dims x 1 head x 128 rows; dims past `dims` read as zero.
-bool encode_map3(CUtensorMap* m, const void* base, int64_t rows, int heads, int dims) {
+// 3-D bf16 map over a [rows, heads, dims] tensor, box of box_dims dims x 1
+// head x 128 rows: 64 dims with the 128-byte swizzle, or 16 dims with the
+// 32-byte swizzle; dims past `dims` read as zero.
+bool encode_map3(CUtensorMap* m, const void* base, int64_t rows, int heads, int dims, uint32_t box_dims = 64) {
   auto enc = tensor_map_encoder();
   if (!enc) return false;
   cuuint64_t gdim[3] = {(cuuint64_t)dims, (cuuint64_t)heads, (cuuint64_t)rows};
   cuuint64_t gstride[2] = {(cuuint64_t)dims * 2, (cuuint64_t)heads * dims * 2};
-  cuuint32_t box[3] = {64, 1, 128};
+  cuuint32_t box[3] = {box_dims, 1, 128};
   cuuint32_t es[3] = {1, 1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), gdim, gstride, box, es,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+             CU_TENSOR_MAP_INTERLEAVE_NONE, box_dims == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_32B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // Stage-II path selection: the fused tensor-core kernel for every sample that
@@ -241,7 +242,8 @@ int check_stage1(const occam_batch* b, const occam_stage1_args* a) {
   } else if (a->mode == OCCAM_STAGE1_MUTUAL) {
     if (a->H1 < 1 || a->H1 > 64) return OCCAM_ERR_UNSUPPORTED;
     if (a->d1 != 64 && a->d1 != 72 && a->d1 != 80) return OCCAM_ERR_UNSUPPORTED;
-    if (b->max_seg_rows > 65535 * 128 || b->S_tot > 65535) return OCCAM_ERR_UNSUPPORTED;
+    // work items of the first pass, S_tot * tiles * H1, are int32
+    if ((int64_t)b->S_tot * cdiv(b->max_seg_rows, 128) * a->H1 > 0x7fffff00) return OCCAM_ERR_UNSUPPORTED;
   } else {
     return OCCAM_ERR_INVALID_ARG;
   }
@@ -341,10 +343,15 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
     p.s2_zero = s2_zero;
     p.status = status;
     // Q1 and K1 as [rows, H1, d1]: boxes of 64 dims x 1 head x 128 rows
-    CUtensorMap mq, mk;
-    if (!encode_map3(&mq, a->q, b->total_rows, a->H1, a->d1) || !encode_map3(&mk, a->K1, b->total_rows, a->H1, a->d1))
+    CUtensorMap mq, mk, mq1, mk1;
+    if (!encode_map3(&mq, a->q, b->total_rows, a->H1, a->d1) || !encode_map3(&mk, a->K1, b->total_rows, a->H1, a->d1) ||
+        !encode_map3(&mq1, a->q, b->total_rows, a->H1, a->d1, 16) ||
+        !encode_map3(&mk1, a->K1, b->total_rows, a->H1, a->d1, 16))
       return OCCAM_ERR_CUDA;
-    launch_mutual_tc(p, mq, mk, b->S_tot, b->max_seg_rows, st);
+    p.tiles = (int)cdiv(b->max_seg_rows, 128);
+    p.queue = at<int32_t>(ws, L.counters) + CNT_MUT;
+    OCCAM_CUDA(cudaMemsetAsync(p.queue, 0, 2 * sizeof(int32_t), st));
+    launch_mutual_tc(p, mq, mk, mq1, mk1, num_sms(), st);
     trace.mark(st);
   }
   return cuda_ok();

@@ -209,7 +209,8 @@ enum {
   CNT_SEG_TICKET = 8,  // Stage-I finalize: segment order
   CNT_NF16 = 9,
   CNT_QUEUE16 = 10,    // next fused Stage-II item (16-CTA clusters)
-  CNT_SLOTS = 11
+  CNT_MUT = 11,        // [2] next mutual Stage-I item of each pass
+  CNT_SLOTS = 13
 };
 
 constexpr int kTextTile = 64;    // Stage-II text rows per item

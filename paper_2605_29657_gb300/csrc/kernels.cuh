@@ -50,6 +50,8 @@ struct MutualTcParams {
   float* s1;
   float* s2_zero;    // nullable
   int* status;
+  int tiles;         // 128-row tiles of the longest segment
+  int32_t* queue;    // [2] work-queue heads of the two passes, zero before the launch
 };
 
 
@@ -229,8 +231,8 @@ struct Stage2TcParams {
 __global__ void stage1_logits_kernel(Stage1ClsParams p);
 int stage1_logits_smem_bytes();
 __global__ void stage1_finalize_kernel(Stage1FinalizeParams p);
-void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, int S_tot,
-                      int max_seg_rows, cudaStream_t st);
+void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mq1,
+                      const CUtensorMap& mk1, int sms, cudaStream_t st);
 __global__ void roles_scatter_kernel(BatchDev bt, uint8_t* role);
 __global__ void threshold_kernel(ThresholdParams p);
 

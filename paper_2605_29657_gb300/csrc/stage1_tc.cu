@@ -16,8 +16,9 @@
 // and the other side streams in blocks of 256 rows (the B operand):
 // S = A B^T is 128 x 256 fp32 in TMEM, from 4-5 tcgen05.mma of K = 16.
 // Q1 and K1 are read as 3-D TMA boxes {64 dims, 1 head, 128 rows} with the
-// 128-byte swizzle; dims past d1 (72 -> 80) come zero-filled by the box, so
-// the padded K-steps add nothing.
+// 128-byte swizzle, plus {16 dims, 1 head, 128 rows} with the 32-byte swizzle
+// for dims 64-79; dims past d1 (72 -> 80) come zero-filled by the box, so the
+// padded K-step adds nothing.
 // Roles (384 threads): warp 0 issues the TMA loads, warp 1 the MMAs, warps
 // 4-11 (two per TMEM lane quadrant, each taking 128 of the 256 columns) the
 // softmax arithmetic. A tiles, B blocks and the TMEM accumulator are double
@@ -32,18 +33,23 @@ namespace occam {
 namespace m1 {
 constexpr int AR = 128;                   // tile rows (TMEM lanes)
 constexpr int BR = 256;                   // block rows (MMA N)
-constexpr int ABYTES = AR * 128;          // one K-block of an A tile
-constexpr int BBYTES = BR * 128;          // one K-block of a B block
+constexpr int ABYTES = AR * 128;          // K-block 0 (dims 0-63) of an A tile
+constexpr int BBYTES = BR * 128;          // K-block 0 of a B block
+constexpr int ABYTES1 = AR * 32;          // K-block 1 (dims 64-79, 32-byte rows) of an A tile
+constexpr int BBYTES1 = BR * 32;
 constexpr int THREADS = 384;
 constexpr int EPI0 = 4;                   // first epilogue warp
 constexpr uint64_t kLimitNs = 2000000000ull;
 
 struct Smem {
-  uint8_t a[2][2][ABYTES];  // [buffer][K-block]
-  uint8_t b[2][2][BBYTES];
+  uint8_t a[2][ABYTES];     // K-block 0 per buffer
+  uint8_t b[2][BBYTES];
+  uint8_t a1[2][ABYTES1];   // K-block 1 per buffer
+  uint8_t b1[2][BBYTES1];
   float lsm[8][128];        // pass 2: log-sums of each epilogue warp's 128 columns
   float2 part[2][4][32];    // second-half partials per (item parity, quadrant, lane)
-  uint64_t afull[2], aempty[2], bfull[2], bempty[2], dfull[2], dfree[2], hb[4], mdone;
+  int32_t item[8];          // the ii-th work item, by ii & 7 (-1: no more)
+  uint64_t afull[2], aempty[2], bfull[2], bempty[2], dfull[2], dfree[2], hb[2][4], inext[8], mdone;
   uint32_t tmem_base;
   int abort;
 };
@@ -68,27 +74,47 @@ __device__ __forceinline__ void wait_ld64(uint32_t (&v)[64]) {
 
 }  // namespace
 
-// PASS 1: A = query tiles, B = key blocks, one head per CTA (blockIdx.y).
-// PASS 2: A = key tiles, B = query blocks, all heads.
+// Work items, taken from a queue by a persistent grid (one CTA per SM):
+// PASS 1: (segment, tile of 128 query rows, head), A = query tile, B = key
+//         blocks of that head;
+// PASS 2: (segment, tile of 128 key rows), A = key tile, B = query blocks,
+//         for every head in turn.
+// The producer thread draws items (skipping tiles past a segment's rows) and
+// hands each to the MMA and softmax warps through an 8-deep ring in shared
+// memory (the producer runs at most a few steps ahead, so a slot is read
+// before it comes round again); buffer and phase counters run on across
+// items, so the next item's loads overlap the current item's tail.
+struct MutItem {
+  int seg, a0, h, n;
+};
+
+template <int PASS>
+__device__ __forceinline__ bool mut_item(const MutualTcParams& p, int it, MutItem& w) {
+  const int per_seg = p.tiles * (PASS == 1 ? p.H : 1);
+  w.seg = it / per_seg;
+  const int rem = it - w.seg * per_seg;
+  const int tile = PASS == 1 ? rem / p.H : rem;
+  w.h = PASS == 1 ? rem - tile * p.H : 0;
+  w.a0 = tile * m1::AR;
+  w.n = (int)(p.bt.seg_off[w.seg + 1] - p.bt.seg_off[w.seg]);
+  return w.a0 < w.n;
+}
+
 template <int PASS>
 __global__ void __launch_bounds__(m1::THREADS, 1)
     mutual_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+                     const __grid_constant__ CUtensorMap mapA1, const __grid_constant__ CUtensorMap mapB1,
                      MutualTcParams p) {
   using namespace m1;
   extern __shared__ unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int seg = blockIdx.z;
-  const int64_t sb = p.bt.seg_off[seg];
-  const int n = (int)(p.bt.seg_off[seg + 1] - sb);
-  const int a0 = blockIdx.x * AR;
-  if (a0 >= n) return;  // uniform over the CTA, before any shared state
   const int H = p.H;
-  const int nb = (n + BR - 1) / BR;
+  const int total = p.bt.S_tot * p.tiles * (PASS == 1 ? H : 1);
   const int nheads = PASS == 1 ? 1 : H;
-  const int steps = nheads * nb;
   const int nkb = p.d1 > 64 ? 2 : 1;         // K-blocks of 64 dims
   const int nks = (p.d1 + 15) / 16;          // K-steps of 16 dims
+  int* queue = p.queue + (PASS - 1);
   volatile int* abort = &sm.abort;
 
   if (tid == 0) {
@@ -100,12 +126,15 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       tc::bar_init(&sm.dfull[i], 1);
       tc::bar_init(&sm.dfree[i], 8);
     }
-    for (int i = 0; i < 4; ++i) tc::bar_init(&sm.hb[i], 1);
+    for (int i = 0; i < 8; ++i) tc::bar_init(&sm.hb[i >> 2][i & 3], 1);
+    for (int i = 0; i < 8; ++i) tc::bar_init(&sm.inext[i], 1);
     tc::bar_init(&sm.mdone, 1);
     sm.abort = 0;
     tc::bar_fence_init();
     tc::prefetch_map(&mapA);
     tc::prefetch_map(&mapB);
+    tc::prefetch_map(&mapA1);
+    tc::prefetch_map(&mapB1);
   }
   if (warp == 1) tc::tmem_alloc(&sm.tmem_base, 512);
   tc::fence_before();
@@ -117,32 +146,53 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       uint32_t na = 0, nbk = 0;
-      for (int s = 0; s < steps && !*abort; ++s) {
-        const int h = PASS == 1 ? (int)blockIdx.y : s / nb;
-        const int jb = s % nb;
-        if (jb == 0) {
-          const int ab = na & 1;
-          if (!tc::bar_wait(&sm.aempty[ab], ((na >> 1) & 1) ^ 1, abort, kLimitNs)) {
-            sm.abort = 1;
-            set_status(p.status, OCCAM_ERR_TIMEOUT);
+      for (int ii = 0;; ++ii) {
+        int it;
+        MutItem w;
+        do {
+          it = atomicAdd(queue, 1);
+        } while (it < total && !mut_item<PASS>(p, it, w));
+        sm.item[ii & 7] = it < total && !*abort ? it : -1;
+        tc::bar_arrive(&sm.inext[ii & 7]);
+        if (it >= total || *abort) break;
+        const int64_t sb = p.bt.seg_off[w.seg];
+        const int nb = (w.n + BR - 1) / BR;
+        bool ok = true;
+        for (int s = 0; s < nheads * nb && ok; ++s) {
+          const int h = PASS == 1 ? w.h : s / nb;
+          const int jb = s % nb;
+          if (jb == 0) {
+            const int ab = na & 1;
+            if (!tc::bar_wait(&sm.aempty[ab], ((na >> 1) & 1) ^ 1, abort, kLimitNs)) {
+              ok = false;
+              break;
+            }
+            tc::bar_expect_tx(&sm.afull[ab], (uint32_t)(ABYTES + (nkb > 1 ? ABYTES1 : 0)));
+            tma_load_3d(sm.a[ab], &mapA, 0, h, (int)(sb + w.a0), &sm.afull[ab]);
+            if (nkb > 1) tma_load_3d(sm.a1[ab], &mapA1, 64, h, (int)(sb + w.a0), &sm.afull[ab]);
+            ++na;
+          }
+          const int bb = nbk & 1;
+          if (!tc::bar_wait(&sm.bempty[bb], ((nbk >> 1) & 1) ^ 1, abort, kLimitNs)) {
+            ok = false;
             break;
           }
-          tc::bar_expect_tx(&sm.afull[ab], (uint32_t)(nkb * ABYTES));
-          for (int kb = 0; kb < nkb; ++kb)
-            tma_load_3d(sm.a[ab][kb], &mapA, kb * 64, h, (int)(sb + a0), &sm.afull[ab]);
-          ++na;
+          tc::bar_expect_tx(&sm.bfull[bb], (uint32_t)(BBYTES + (nkb > 1 ? BBYTES1 : 0)));
+          for (int hh = 0; hh < BR / AR; ++hh) {
+            const int y = (int)(sb + jb * BR + hh * AR);
+            tma_load_3d(sm.b[bb] + hh * ABYTES, &mapB, 0, h, y, &sm.bfull[bb]);
+            if (nkb > 1) tma_load_3d(sm.b1[bb] + hh * ABYTES1, &mapB1, 64, h, y, &sm.bfull[bb]);
+          }
+          ++nbk;
         }
-        const int bb = nbk & 1;
-        if (!tc::bar_wait(&sm.bempty[bb], ((nbk >> 1) & 1) ^ 1, abort, kLimitNs)) {
+        if (!ok) {
           sm.abort = 1;
           set_status(p.status, OCCAM_ERR_TIMEOUT);
+          // tell the other roles to stop at the next hand-out
+          sm.item[(ii + 1) & 7] = -1;
+          tc::bar_arrive(&sm.inext[(ii + 1) & 7]);
           break;
         }
-        tc::bar_expect_tx(&sm.bfull[bb], (uint32_t)(nkb * BBYTES));
-        for (int kb = 0; kb < nkb; ++kb)
-          for (int hh = 0; hh < BR / AR; ++hh)
-            tma_load_3d(sm.b[bb][kb] + hh * ABYTES, &mapB, kb * 64, h, (int)(sb + jb * BR + hh * AR), &sm.bfull[bb]);
-        ++nbk;
       }
     }
     __syncwarp();
@@ -150,31 +200,46 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc = tc::idesc_bf16(AR, BR);
-      uint32_t na = 0;
-      for (int s = 0; s < steps; ++s) {
-        const int jb = s % nb;
-        const int ab = na & 1, bb = s & 1, db = s & 1;
-        bool ok = true;
-        if (jb == 0) ok = tc::bar_wait(&sm.afull[ab], (na >> 1) & 1, abort, kLimitNs);
-        if (ok) ok = tc::bar_wait(&sm.bfull[bb], (s >> 1) & 1, abort, kLimitNs);
-        if (ok && s >= 2) ok = tc::bar_wait(&sm.dfree[db], ((s - 2) >> 1) & 1, abort, kLimitNs);
-        if (!ok) {
+      uint32_t na = 0, sg = 0;
+      for (int ii = 0;; ++ii) {
+        if (!tc::bar_wait(&sm.inext[ii & 7], (ii >> 3) & 1, abort, kLimitNs)) {
           sm.abort = 1;
           set_status(p.status, OCCAM_ERR_TIMEOUT);
           break;
         }
-        tc::fence_after();
-        const uint32_t abase = tc::su32(sm.a[ab][0]), bbase = tc::su32(sm.b[bb][0]);
-        for (int ks = 0; ks < nks; ++ks) {
-          const int kb = ks >> 2, kk = ks & 3;
-          tc::mma_bf16(tmem + db * BR, tc::sdesc_sw128(abase + kb * ABYTES + kk * 32),
-                       tc::sdesc_sw128(bbase + kb * BBYTES + kk * 32), idesc, ks > 0 ? 1u : 0u);
+        const int it = *reinterpret_cast<volatile int*>(&sm.item[ii & 7]);
+        if (it < 0) break;
+        MutItem w;
+        mut_item<PASS>(p, it, w);
+        const int nb = (w.n + BR - 1) / BR;
+        bool ok = true;
+        for (int s = 0; s < nheads * nb; ++s, ++sg) {
+          const int jb = s % nb;
+          const int ab = na & 1, bb = sg & 1, db = sg & 1;
+          if (jb == 0) ok = tc::bar_wait(&sm.afull[ab], (na >> 1) & 1, abort, kLimitNs);
+          if (ok) ok = tc::bar_wait(&sm.bfull[bb], (sg >> 1) & 1, abort, kLimitNs);
+          if (ok && sg >= 2) ok = tc::bar_wait(&sm.dfree[db], ((sg - 2) >> 1) & 1, abort, kLimitNs);
+          if (!ok) break;
+          tc::fence_after();
+          const uint32_t abase = tc::su32(sm.a[ab]), bbase = tc::su32(sm.b[bb]);
+          for (int ks = 0; ks < nks && ks < 4; ++ks)
+            tc::mma_bf16(tmem + db * BR, tc::sdesc_sw128(abase + ks * 32), tc::sdesc_sw128(bbase + ks * 32), idesc,
+                         ks > 0 ? 1u : 0u);
+          // dims 64-79: one K-step over the 32-byte rows
+          if (nks > 4)
+            tc::mma_bf16(tmem + db * BR, tc::sdesc_sw32(tc::su32(sm.a1[ab])), tc::sdesc_sw32(tc::su32(sm.b1[bb])),
+                         idesc, 1u);
+          tc::mma_commit(&sm.dfull[db]);
+          tc::mma_commit(&sm.bempty[bb]);
+          if (jb == nb - 1) {
+            tc::mma_commit(&sm.aempty[ab]);
+            ++na;
+          }
         }
-        tc::mma_commit(&sm.dfull[db]);
-        tc::mma_commit(&sm.bempty[bb]);
-        if (jb == nb - 1) {
-          tc::mma_commit(&sm.aempty[ab]);
-          ++na;
+        if (!ok) {
+          sm.abort = 1;
+          set_status(p.status, OCCAM_ERR_TIMEOUT);
+          break;
         }
       }
       tc::mma_commit(&sm.mdone);
@@ -188,94 +253,127 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
     const int row = quad * 32 + lane;                   // tile row = TMEM lane
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const float c = p.scale_log2;
-    const bool vrow = a0 + row < n;
     const int64_t R = p.bt.total_rows;
-    float m = -INFINITY, z = 0.f;  // pass 1: running max / sum (log2 domain)
-    float acc = 0.f;               // pass 2: attention received by this key row
-    bool ok = true;
-    for (int s = 0; s < steps && ok; ++s) {
-      const int h = PASS == 1 ? (int)blockIdx.y : s / nb;
-      const int jb = s % nb;
-      const int col0 = jb * BR + half * 128;            // segment-relative index of this warp's column 0
-      if (PASS == 2) {
-        // log-sums of this warp's 128 query columns; past the segment: +inf (contributes 0)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int qq = col0 + lane * 4 + i;
-          sm.lsm[ew][lane * 4 + i] = qq < n ? __ldcg(&p.lsum[(int64_t)h * R + sb + qq]) : INFINITY;
-        }
-        __syncwarp();
-      }
-      const int db = s & 1;
-      if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.dfull[db], (s >> 1) & 1, nullptr, kLimitNs))) {
-        ok = false;
-        break;
-      }
-      tc::fence_after();
-#pragma unroll
-      for (int g = 0; g < 2; ++g) {
-        uint32_t v[64];
-        tc::tmem_ld64(tmem + lane_base + db * BR + half * 128 + g * 64, v);
-        wait_ld64(v);
-        if (PASS == 1) {
-          // keys past the segment are masked out of this row's softmax
-          const int lim = n - (col0 + g * 64);
-          float mx = -INFINITY;
-#pragma unroll
-          for (int i = 0; i < 64; ++i) {
-            const float x = i < lim ? __uint_as_float(v[i]) * c : -INFINITY;
-            v[i] = __float_as_uint(x);
-            mx = fmaxf(mx, x);
-          }
-          if (mx != -INFINITY) {
-            float ap[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int i = 0; i < 64; ++i) ap[i & 7] += tc::ex2(__uint_as_float(v[i]) - mx);
-            const float a = ((ap[0] + ap[1]) + (ap[2] + ap[3])) + ((ap[4] + ap[5]) + (ap[6] + ap[7]));
-            const bool up = mx > m;
-            const float e = tc::ex2(up ? m - mx : mx - m);
-            z = up ? fmaf(z, e, a) : fmaf(a, e, z);
-            m = fmaxf(m, mx);
-          }
-        } else {
-          const float* L = sm.lsm[ew] + g * 64;
-          float ap[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-          for (int i = 0; i < 64; ++i) ap[i & 7] += tc::ex2(fmaf(__uint_as_float(v[i]), c, -L[i]));
-          acc += ((ap[0] + ap[1]) + (ap[2] + ap[3])) + ((ap[4] + ap[5]) + (ap[6] + ap[7]));
-        }
-      }
-      tc::fence_before();
-      __syncwarp();
-      if (lane == 0) tc::bar_arrive(&sm.dfree[db]);
-    }
-    if (!ok) {
-      sm.abort = 1;
-      set_status(p.status, OCCAM_ERR_TIMEOUT);
-    } else {
-      // the two halves of each row: the second hands its partial to the first
-      if (half == 1) {
-        sm.part[0][quad][lane] = make_float2(PASS == 1 ? m : acc, z);
-        __syncwarp();
-        if (lane == 0) tc::bar_arrive(&sm.hb[quad]);
-      } else if (__all_sync(0xffffffffu, tc::bar_wait(&sm.hb[quad], 0, nullptr, kLimitNs))) {
-        const float2 o = sm.part[0][quad][lane];
-        if (PASS == 1) {
-          if (o.x != -INFINITY) {
-            const bool up = o.x > m;
-            const float e = tc::ex2(up ? m - o.x : o.x - m);
-            z = up ? fmaf(z, e, o.y) : fmaf(o.y, e, z);
-            m = fmaxf(m, o.x);
-          }
-          // L = log2 of the row's sum of exp2(c q k) over the segment's keys
-          if (vrow) p.lsum[(int64_t)blockIdx.y * R + sb + a0 + row] = m + log2f(z);
-        } else if (vrow) {
-          p.s1[sb + a0 + row] = (acc + o.x) * p.inv_h / (float)n;
-          if (p.s2_zero) p.s2_zero[sb + a0 + row] = 0.f;
-        }
-      } else {
+    uint32_t sg = 0;
+    for (int ii = 0;; ++ii) {
+      if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.inext[ii & 7], (ii >> 3) & 1, nullptr, kLimitNs))) {
         sm.abort = 1;
         set_status(p.status, OCCAM_ERR_TIMEOUT);
+        break;
+      }
+      const int it = *reinterpret_cast<volatile int*>(&sm.item[ii & 7]);
+      if (it < 0) break;
+      MutItem w;
+      mut_item<PASS>(p, it, w);
+      const int n = w.n;
+      const int64_t sb = p.bt.seg_off[w.seg];
+      const int nb = (n + BR - 1) / BR;
+      const int steps = nheads * nb;
+      const bool vrow = w.a0 + row < n;
+      const int pp = ii & 1;
+      float m = -INFINITY, z = 0.f;  // pass 1: running max / sum (log2 domain)
+      float acc = 0.f;               // pass 2: attention received by this key row
+      bool ok = true;
+      for (int s = 0; s < steps; ++s, ++sg) {
+        const int h = PASS == 1 ? w.h : s / nb;
+        const int jb = s % nb;
+        const int col0 = jb * BR + half * 128;          // segment-relative index of this warp's column 0
+        if (PASS == 2) {
+          // log-sums of this warp's 128 query columns; past the segment: +inf (contributes 0)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int qq = col0 + lane * 4 + i;
+            sm.lsm[ew][lane * 4 + i] = qq < n ? __ldcg(&p.lsum[(int64_t)h * R + sb + qq]) : INFINITY;
+          }
+          __syncwarp();
+        }
+        const int db = sg & 1;
+        if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.dfull[db], (sg >> 1) & 1, nullptr, kLimitNs))) {
+          ok = false;
+          break;
+        }
+        tc::fence_after();
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+          uint32_t v[64];
+          tc::tmem_ld64(tmem + lane_base + db * BR + half * 128 + g * 64, v);
+          wait_ld64(v);
+          if (PASS == 1) {
+            // keys past the segment are masked out of this row's softmax
+            const int lim = n - (col0 + g * 64);
+            if (lim < 64) {
+#pragma unroll
+              for (int i = 0; i < 64; ++i) v[i] = i < lim ? v[i] : 0xff800000u;  // -inf
+            }
+            // max as a tree of three-input maxima (short dependency chains)
+            float t[22];
+#pragma unroll
+            for (int i = 0; i < 21; ++i)
+              t[i] = tc::fmax3(__uint_as_float(v[3 * i]), __uint_as_float(v[3 * i + 1]), __uint_as_float(v[3 * i + 2]));
+            t[21] = __uint_as_float(v[63]);
+            float u[8];
+#pragma unroll
+            for (int i = 0; i < 7; ++i) u[i] = tc::fmax3(t[3 * i], t[3 * i + 1], t[3 * i + 2]);
+            u[7] = t[21];
+            // c > 0: the max of c l is c times the max of l
+            const float mx =
+                fmaxf(tc::fmax3(u[0], u[1], u[2]), tc::fmax3(u[3], u[4], fmaxf(u[5], fmaxf(u[6], u[7])))) * c;
+            if (mx != -INFINITY) {
+              float ap[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+              for (int i = 0; i < 64; ++i) ap[i & 7] += tc::ex2(fmaf(__uint_as_float(v[i]), c, -mx));
+              const float a = ((ap[0] + ap[1]) + (ap[2] + ap[3])) + ((ap[4] + ap[5]) + (ap[6] + ap[7]));
+              const bool up = mx > m;
+              const float e = tc::ex2(up ? m - mx : mx - m);
+              z = up ? fmaf(z, e, a) : fmaf(a, e, z);
+              m = fmaxf(m, mx);
+            }
+          } else {
+            const float* L = sm.lsm[ew] + g * 64;
+            float ap[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int i = 0; i < 64; ++i) ap[i & 7] += tc::ex2(fmaf(__uint_as_float(v[i]), c, -L[i]));
+            acc += ((ap[0] + ap[1]) + (ap[2] + ap[3])) + ((ap[4] + ap[5]) + (ap[6] + ap[7]));
+          }
+        }
+        tc::fence_before();
+        __syncwarp();
+        const bool last = s == steps - 1;
+        if (half == 1 && last) {
+          // the second half hands its partial to the first
+          sm.part[pp][quad][lane] = make_float2(PASS == 1 ? m : acc, z);
+          __syncwarp();
+          if (lane == 0) tc::bar_arrive(&sm.hb[pp][quad]);
+        }
+        if (half == 0 && last) {
+          // read the partner's partial before releasing this step's
+          // accumulator: its next write to the slot waits on that release
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.hb[pp][quad], (ii >> 1) & 1, nullptr, kLimitNs))) {
+            ok = false;
+            break;
+          }
+          const float2 o = sm.part[pp][quad][lane];
+          if (PASS == 1) {
+            if (o.x != -INFINITY) {
+              const bool up = o.x > m;
+              const float e = tc::ex2(up ? m - o.x : o.x - m);
+              z = up ? fmaf(z, e, o.y) : fmaf(o.y, e, z);
+              m = fmaxf(m, o.x);
+            }
+            // L = log2 of the row's sum of exp2(c q k) over the segment's keys
+            if (vrow) p.lsum[(int64_t)w.h * R + sb + w.a0 + row] = m + log2f(z);
+          } else if (vrow) {
+            p.s1[sb + w.a0 + row] = (acc + o.x) * p.inv_h / (float)n;
+            if (p.s2_zero) p.s2_zero[sb + w.a0 + row] = 0.f;
+          }
+          __syncwarp();
+        }
+        if (lane == 0) tc::bar_arrive(&sm.dfree[db]);
+      }
+      if (!ok) {
+        sm.abort = 1;
+        set_status(p.status, OCCAM_ERR_TIMEOUT);
+        break;
       }
     }
   }
@@ -294,14 +392,13 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
   if (warp == 1) tc::tmem_dealloc(tmem, 512);
 }
 
-void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, int S_tot,
-                      int max_seg_rows, cudaStream_t st) {
-  const int tiles = (max_seg_rows + m1::AR - 1) / m1::AR;
+void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mq1,
+                      const CUtensorMap& mk1, int sms, cudaStream_t st) {
   const int smem = mutual_tc_smem_bytes();
   cudaFuncSetAttribute(mutual_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   cudaFuncSetAttribute(mutual_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  mutual_tc_kernel<1><<<dim3(tiles, p.H, S_tot), m1::THREADS, smem, st>>>(mq, mk, p);
-  mutual_tc_kernel<2><<<dim3(tiles, 1, S_tot), m1::THREADS, smem, st>>>(mk, mq, p);
+  mutual_tc_kernel<1><<<sms, m1::THREADS, smem, st>>>(mq, mk, mq1, mk1, p);
+  mutual_tc_kernel<2><<<sms, m1::THREADS, smem, st>>>(mk, mq, mk1, mq1, p);
 }
 
 }  // namespace occam
