@@ -46,7 +46,7 @@ struct Smem {
   uint8_t b[2][BBYTES];
   uint8_t a1[2][ABYTES1];   // K-block 1 per buffer
   uint8_t b1[2][BBYTES1];
-  float lsm[8][128];        // pass 2: log-sums of each epilogue warp's 128 columns
+  float lsm[8][128];        // pass 2: minus the log-sums of each epilogue warp's 128 columns
   float2 part[2][4][32];    // second-half partials per (item parity, quadrant, lane)
   int32_t item[8];          // the ii-th work item, by ii & 7 (-1: no more)
   uint64_t afull[2], aempty[2], bfull[2], bempty[2], dfull[2], dfree[2], hb[2][4], inext[8], mdone;
@@ -273,19 +273,34 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       const int pp = ii & 1;
       float m = -INFINITY, z = 0.f;  // pass 1: running max / sum (log2 domain)
       float acc = 0.f;               // pass 2: attention received by this key row
+      float lnext[4];                // pass 2: the next step's minus log-sums of 4 columns
       bool ok = true;
       for (int s = 0; s < steps; ++s, ++sg) {
         const int h = PASS == 1 ? w.h : s / nb;
         const int jb = s % nb;
         const int col0 = jb * BR + half * 128;          // segment-relative index of this warp's column 0
         if (PASS == 2) {
-          // log-sums of this warp's 128 query columns; past the segment: +inf (contributes 0)
+          // minus the log-sums of this warp's 128 query columns (past the
+          // segment: -inf, which contributes 0); those of the item's first
+          // step are loaded here, the others one step ahead (below)
+          if (s == 0) {
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int qq = col0 + lane * 4 + i;
-            sm.lsm[ew][lane * 4 + i] = qq < n ? __ldcg(&p.lsum[(int64_t)h * R + sb + qq]) : INFINITY;
+            for (int i = 0; i < 4; ++i) {
+              const int qq = col0 + lane * 4 + i;
+              lnext[i] = qq < n ? -__ldcg(&p.lsum[(int64_t)h * R + sb + qq]) : -INFINITY;
+            }
           }
           __syncwarp();
+          *reinterpret_cast<float4*>(&sm.lsm[ew][lane * 4]) = make_float4(lnext[0], lnext[1], lnext[2], lnext[3]);
+          __syncwarp();
+          if (s + 1 < steps) {
+            const int h1 = (s + 1) / nb, c1 = ((s + 1) % nb) * BR + half * 128;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int qq = c1 + lane * 4 + i;
+              lnext[i] = qq < n ? -__ldcg(&p.lsum[(int64_t)h1 * R + sb + qq]) : -INFINITY;
+            }
+          }
         }
         const int db = sg & 1;
         if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.dfull[db], (sg >> 1) & 1, nullptr, kLimitNs))) {
@@ -319,21 +334,35 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
             const float mx =
                 fmaxf(tc::fmax3(u[0], u[1], u[2]), tc::fmax3(u[3], u[4], fmaxf(u[5], fmaxf(u[6], u[7])))) * c;
             if (mx != -INFINITY) {
-              float ap[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+              const float2 cc = make_float2(c, c), om = make_float2(-mx, -mx);
+              float2 ap[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
-              for (int i = 0; i < 64; ++i) ap[i & 7] += tc::ex2(fmaf(__uint_as_float(v[i]), c, -mx));
-              const float a = ((ap[0] + ap[1]) + (ap[2] + ap[3])) + ((ap[4] + ap[5]) + (ap[6] + ap[7]));
+              for (int i = 0; i < 32; ++i) {
+                float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), cc, om);
+                x.x = tc::ex2(x.x);
+                x.y = tc::ex2(x.y);
+                ap[i & 3] = __fadd2_rn(ap[i & 3], x);
+              }
+              const float2 a2 = __fadd2_rn(__fadd2_rn(ap[0], ap[1]), __fadd2_rn(ap[2], ap[3]));
+              const float a = a2.x + a2.y;
               const bool up = mx > m;
               const float e = tc::ex2(up ? m - mx : mx - m);
               z = up ? fmaf(z, e, a) : fmaf(a, e, z);
               m = fmaxf(m, mx);
             }
           } else {
-            const float* L = sm.lsm[ew] + g * 64;
-            float ap[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            const float2* nl = reinterpret_cast<const float2*>(sm.lsm[ew] + g * 64);
+            const float2 cc = make_float2(c, c);
+            float2 ap[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
-            for (int i = 0; i < 64; ++i) ap[i & 7] += tc::ex2(fmaf(__uint_as_float(v[i]), c, -L[i]));
-            acc += ((ap[0] + ap[1]) + (ap[2] + ap[3])) + ((ap[4] + ap[5]) + (ap[6] + ap[7]));
+            for (int i = 0; i < 32; ++i) {
+              float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), cc, nl[i]);
+              x.x = tc::ex2(x.x);
+              x.y = tc::ex2(x.y);
+              ap[i & 3] = __fadd2_rn(ap[i & 3], x);
+            }
+            const float2 a2 = __fadd2_rn(__fadd2_rn(ap[0], ap[1]), __fadd2_rn(ap[2], ap[3]));
+            acc += a2.x + a2.y;
           }
         }
         tc::fence_before();
