@@ -349,6 +349,8 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
         !encode_map3(&mk1, a->K1, b->total_rows, a->H1, a->d1, 16))
       return OCCAM_ERR_CUDA;
     p.tiles = (int)cdiv(b->max_seg_rows, 128);
+    p.hgroups = (int)cdiv(a->H1, kMutHeadGroup);
+    p.part = p.lsum + (int64_t)a->H1 * b->total_rows;  // stats1 holds 2 * H1 floats per row
     p.queue = at<int32_t>(ws, L.counters) + CNT_MUT;
     OCCAM_CUDA(cudaMemsetAsync(p.queue, 0, 2 * sizeof(int32_t), st));
     launch_mutual_tc(p, mq, mk, mq1, mk1, num_sms(), st);

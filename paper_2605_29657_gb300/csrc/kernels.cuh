@@ -52,7 +52,10 @@ struct MutualTcParams {
   int* status;
   int tiles;         // 128-row tiles of the longest segment
   int32_t* queue;    // [2] work-queue heads of the two passes, zero before the launch
+  int hgroups;       // head groups of kMutHeadGroup heads (second pass)
+  float* part;       // [hgroups, total_rows] each head group's share of s1
 };
+constexpr int kMutHeadGroup = 4;
 
 
 struct ThresholdParams {

@@ -9,9 +9,10 @@
 //   pass 1: per (segment, tile of 128 query rows, head) the query rows'
 //           softmax log-sums L[h][u] = log2 sum_v exp2(c q_u k_v), with
 //           c = log2(e) / sqrt(d1), over all the segment's keys;
-//   pass 2: per (segment, tile of 128 key rows) the attention each key
-//           receives, sum_h sum_u exp2(c q_u k_v - L[h][u]), over all heads
-//           and query rows.
+//   pass 2: per (segment, tile of 128 key rows, group of 4 heads) the
+//           attention each key receives, sum_h sum_u exp2(c q_u k_v - L[h][u]),
+//           over the group's heads and all query rows; a small third kernel
+//           sums the groups' shares in order into s1.
 // In both, the CTA's 128 tile rows are the TMEM lanes (the MMA's A operand)
 // and the other side streams in blocks of 256 rows (the B operand):
 // S = A B^T is 128 x 256 fp32 in TMEM, from 4-5 tcgen05.mma of K = 16.
@@ -77,8 +78,8 @@ __device__ __forceinline__ void wait_ld64(uint32_t (&v)[64]) {
 // Work items, taken from a queue by a persistent grid (one CTA per SM):
 // PASS 1: (segment, tile of 128 query rows, head), A = query tile, B = key
 //         blocks of that head;
-// PASS 2: (segment, tile of 128 key rows), A = key tile, B = query blocks,
-//         for every head in turn.
+// PASS 2: (segment, tile of 128 key rows, group of 4 heads), A = key tile,
+//         B = query blocks, for the group's heads in turn.
 // The producer thread draws items (skipping tiles past a segment's rows) and
 // hands each to the MMA and softmax warps through an 8-deep ring in shared
 // memory (the producer runs at most a few steps ahead, so a slot is read
@@ -90,11 +91,12 @@ struct MutItem {
 
 template <int PASS>
 __device__ __forceinline__ bool mut_item(const MutualTcParams& p, int it, MutItem& w) {
-  const int per_seg = p.tiles * (PASS == 1 ? p.H : 1);
+  const int sub_n = PASS == 1 ? p.H : p.hgroups;  // heads (pass 1) or head groups (pass 2) per tile
+  const int per_seg = p.tiles * sub_n;
   w.seg = it / per_seg;
   const int rem = it - w.seg * per_seg;
-  const int tile = PASS == 1 ? rem / p.H : rem;
-  w.h = PASS == 1 ? rem - tile * p.H : 0;
+  const int tile = rem / sub_n;
+  w.h = (rem - tile * sub_n) * (PASS == 1 ? 1 : kMutHeadGroup);  // first head of the item
   w.a0 = tile * m1::AR;
   w.n = (int)(p.bt.seg_off[w.seg + 1] - p.bt.seg_off[w.seg]);
   return w.a0 < w.n;
@@ -110,8 +112,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
   Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int H = p.H;
-  const int total = p.bt.S_tot * p.tiles * (PASS == 1 ? H : 1);
-  const int nheads = PASS == 1 ? 1 : H;
+  const int total = p.bt.S_tot * p.tiles * (PASS == 1 ? H : p.hgroups);
   const int nkb = p.d1 > 64 ? 2 : 1;         // K-blocks of 64 dims
   const int nks = (p.d1 + 15) / 16;          // K-steps of 16 dims
   int* queue = p.queue + (PASS - 1);
@@ -157,9 +158,10 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         if (it >= total || *abort) break;
         const int64_t sb = p.bt.seg_off[w.seg];
         const int nb = (w.n + BR - 1) / BR;
+        const int nheads = PASS == 1 ? 1 : min(kMutHeadGroup, H - w.h);
         bool ok = true;
         for (int s = 0; s < nheads * nb && ok; ++s) {
-          const int h = PASS == 1 ? w.h : s / nb;
+          const int h = w.h + s / nb;
           const int jb = s % nb;
           if (jb == 0) {
             const int ab = na & 1;
@@ -212,6 +214,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         MutItem w;
         mut_item<PASS>(p, it, w);
         const int nb = (w.n + BR - 1) / BR;
+        const int nheads = PASS == 1 ? 1 : min(kMutHeadGroup, H - w.h);
         bool ok = true;
         for (int s = 0; s < nheads * nb; ++s, ++sg) {
           const int jb = s % nb;
@@ -268,7 +271,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       const int n = w.n;
       const int64_t sb = p.bt.seg_off[w.seg];
       const int nb = (n + BR - 1) / BR;
-      const int steps = nheads * nb;
+      const int steps = (PASS == 1 ? 1 : min(kMutHeadGroup, H - w.h)) * nb;
       const bool vrow = w.a0 + row < n;
       const int pp = ii & 1;
       float m = -INFINITY, z = 0.f;  // pass 1: running max / sum (log2 domain)
@@ -276,7 +279,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       float lnext[4];                // pass 2: the next step's minus log-sums of 4 columns
       bool ok = true;
       for (int s = 0; s < steps; ++s, ++sg) {
-        const int h = PASS == 1 ? w.h : s / nb;
+        const int h = w.h + s / nb;
         const int jb = s % nb;
         const int col0 = jb * BR + half * 128;          // segment-relative index of this warp's column 0
         if (PASS == 2) {
@@ -294,7 +297,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
           *reinterpret_cast<float4*>(&sm.lsm[ew][lane * 4]) = make_float4(lnext[0], lnext[1], lnext[2], lnext[3]);
           __syncwarp();
           if (s + 1 < steps) {
-            const int h1 = (s + 1) / nb, c1 = ((s + 1) % nb) * BR + half * 128;
+            const int h1 = w.h + (s + 1) / nb, c1 = ((s + 1) % nb) * BR + half * 128;
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
               const int qq = c1 + lane * 4 + i;
@@ -392,8 +395,8 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
             // L = log2 of the row's sum of exp2(c q k) over the segment's keys
             if (vrow) p.lsum[(int64_t)w.h * R + sb + w.a0 + row] = m + log2f(z);
           } else if (vrow) {
-            p.s1[sb + w.a0 + row] = (acc + o.x) * p.inv_h / (float)n;
-            if (p.s2_zero) p.s2_zero[sb + w.a0 + row] = 0.f;
+            // this head group's share of s1 (summed over the groups in order afterwards)
+            p.part[(int64_t)(w.h / kMutHeadGroup) * R + sb + w.a0 + row] = (acc + o.x) * p.inv_h / (float)n;
           }
           __syncwarp();
         }
@@ -421,6 +424,17 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
   if (warp == 1) tc::tmem_dealloc(tmem, 512);
 }
 
+// s1 = the sum of the head groups' shares, in group order (deterministic)
+__global__ void __launch_bounds__(256) mutual_reduce_kernel(MutualTcParams p) {
+  const int64_t R = p.bt.total_rows;
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < R; r += (int64_t)gridDim.x * blockDim.x) {
+    float v = 0.f;
+    for (int g = 0; g < p.hgroups; ++g) v += __ldcg(&p.part[(int64_t)g * R + r]);
+    p.s1[r] = v;
+    if (p.s2_zero) p.s2_zero[r] = 0.f;
+  }
+}
+
 void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mq1,
                       const CUtensorMap& mk1, int sms, cudaStream_t st) {
   const int smem = mutual_tc_smem_bytes();
@@ -428,6 +442,7 @@ void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUte
   cudaFuncSetAttribute(mutual_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   mutual_tc_kernel<1><<<sms, m1::THREADS, smem, st>>>(mq, mk, mq1, mk1, p);
   mutual_tc_kernel<2><<<sms, m1::THREADS, smem, st>>>(mk, mq, mk1, mq1, p);
+  mutual_reduce_kernel<<<sms * 2, 256, 0, st>>>(p);
 }
 
 }  // namespace occam
