@@ -53,18 +53,17 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   const int64_t tps = cdiv(b->max_text, kTextTile);
   const int64_t nhg = cdiv(H2 > 0 ? H2 : 1, kHeadGroup);
   const int64_t chmax = cdiv(b->max_sample_rows, kKeyChunk);
-  L.maxA = B * tps * nhg;
+  L.maxA = B * tps * nhg * kStatSplits;
   L.maxB = B * tps * chmax;
   L.maxF = B * cdiv(b->max_text, 128);
   L.maxSlots = L.maxB + L.maxF * kFusedSlotsPerItem16;
-  L.itemsA = take(L.maxA * 16);
-  L.itemsB = take(L.maxB * 16);
   L.itemsF = take(L.maxF * 16);
   L.itemsF8 = take(L.maxF * 16);
   L.itemsF16 = take(L.maxF * 16);
+  L.itemA_off = take((B + 1) * 4);
   L.itemB_off = take((B + 1) * 4);
   L.slot_off = take((B + 1) * 4);
-  L.stats2 = take(T * (H2 > 0 ? H2 : 1) * 8);
+  L.stats2 = take(T * (H2 > 0 ? H2 : 1) * kStatSplits * 8);
   L.refpart = take(L.maxSlots * 4);
   L.ref2 = take(B * 4);
   L.tau2 = take(B * 4);
@@ -425,8 +424,7 @@ Stage2Params stage2_params(const occam_batch* b, const occam_stage2_args* a, con
   p.role = at<uint8_t>(ws, L.role);
   p.dense = at<int32_t>(ws, L.dense);
   p.n1 = at<int32_t>(ws, L.n1);
-  p.itemsA = at<int4>(ws, L.itemsA);
-  p.itemsB = at<int4>(ws, L.itemsB);
+  p.itemA_off = at<int32_t>(ws, L.itemA_off);
   p.itemB_off = at<int32_t>(ws, L.itemB_off);
   p.counters = at<int32_t>(ws, L.counters);
   p.maxA = L.maxA;

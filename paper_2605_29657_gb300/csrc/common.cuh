@@ -189,7 +189,7 @@ __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long
 // Workspace carve-up (byte offsets from the workspace base; see ws_layout()).
 struct WsLayout {
   size_t status, counters, role, keep1, s1, s2, ref1, dense, n1, n1_vis;
-  size_t itemsA, itemsB, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, seg_state, stats1, itemsF, itemsF8, itemsF16,
+  size_t itemA_off, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, seg_state, stats1, itemsF, itemsF8, itemsF16,
       slot_off;
   size_t zero_begin, zero_end;  // the accumulators every prune call zeroes (one contiguous range)
   size_t total;
@@ -214,7 +214,8 @@ enum {
 };
 
 constexpr int kTextTile = 64;    // Stage-II text rows per item
-constexpr int kHeadGroup = 8;    // Stage-II heads per stats item
+constexpr int kHeadGroup = 4;    // Stage-II heads per stats item
+constexpr int kStatSplits = 16;  // at most this many key ranges per (text tile, head group) in the stats pass
 constexpr int kKeyChunk = 128;   // Stage-II image keys per score item
 constexpr int kScanTile = 2048;  // compaction rows per scan tile (256 threads x 8)
 constexpr uint32_t kSpinLimit = 1u << 22;

@@ -25,6 +25,14 @@ __host__ __device__ inline bool fused_fits(int C, int n1, int M, int H) {
   const int tp = ((M + C - 1) / C + 15) & ~15;
   return M > 0 && H >= 4 && ip <= kFusedMaxOwnImg && ip + tp <= rows;
 }
+// Key ranges of the two-pass statistics pass for a sample with n1 S1 keys and
+// M text tokens: about four 64-key chunks per range, at most kStatSplits.
+// The scores pass merges the ranges' partial statistics, so both passes take
+// the count from this one function.
+__host__ __device__ inline int s2_stat_splits(int n1, int M) {
+  const int s = ((n1 + M + 63) / 64 + 3) / 4;
+  return s < 1 ? 1 : s > kStatSplits ? kStatSplits : s;
+}
 constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedPartialWarps;  // s2(r) partials per C=4 item
 constexpr int kFusedSlotsPerItem8 = 8 * kFusedPartialWarps;             // and per C=8 item
 constexpr int kFusedSlotsPerItem16 = 16 * kFusedPartialWarps;           // and per C=16 item
@@ -81,12 +89,17 @@ struct Stage2Params {
   const uint8_t* role;
   int32_t* dense;           // per sample S1 list at row_off[b]
   int32_t* n1;              // [B]
-  int4* itemsA;             // (b, j0, head group, -)
-  int4* itemsB;             // (b, j0, key chunk, item index within sample)
+  // two-pass items of sample b are [item*_off[b], item*_off[b + 1]); a
+  // kernel finds the sample of its item by binary search and decodes the rest:
+  //   stats item i of b:  text tile i / (head groups * key ranges), head group
+  //                       (i / key ranges) % head groups, key range i % key ranges
+  //   scores item i of b: text tile i / key chunks, key chunk i % key chunks,
+  //                       partial slot slot_off[b] + i
+  int32_t* itemA_off;       // [B+1]
   int32_t* itemB_off;       // [B+1]
   int32_t* counters;
   int64_t maxA, maxB;
-  float2* stats;            // [total_text, H] (max in log2 units, 1/sum)
+  float2* stats;            // [total_text, H, kStatSplits] partial (max in log2 units, sum) per key range
   float* s2;                // atomicMax accumulator, zeroed beforehand
   float* refpart;           // [maxB]
   int32_t* done;            // [B] finished score items per sample (zeroed)

@@ -13,6 +13,7 @@ namespace occam {
 // clusters where its S1 keys and text keys fit, else the two-pass kernels)
 // and writes the item lists, the per-sample item and partial-slot offsets,
 // and the item counts. blockDim.x threads, tmp: >= 40 ints of shared memory.
+// The two-pass kernels get per-sample item offsets, not item lists.
 __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
   const int tid = threadIdx.x;
   const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
@@ -37,7 +38,7 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
       } else {
         const int tiles = (M + kTextTile - 1) / kTextTile;
         const int nch = (n1 + kKeyChunk - 1) / kKeyChunk;
-        nA = tiles * nhg;
+        nA = tiles * nhg * s2_stat_splits(n1, M);
         nB = tiles * nch;
       }
       if (M == 0) {
@@ -46,7 +47,6 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
         p.tau2[bb] = 0.f;
       }
     }
-    const int nch = (bb < p.bt.B) ? (*((volatile int32_t*)&p.n1[bb]) + kKeyChunk - 1) / kKeyChunk : 0;
     const int nS = nF * kFusedSlotsPerItem + nF8 * kFusedSlotsPerItem8 + nF16 * kFusedSlotsPerItem16 +
                    nB;  // s2(r) partial slots of this sample
     int totA, totB, totF, totF8, totF16, totS;
@@ -57,16 +57,13 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
     const int offF16 = runF16 + block_exclusive_scan(nF16, tmp, &totF16);
     const int offS = runS + block_exclusive_scan(nS, tmp, &totS);
     if (bb < p.bt.B) {
-      for (int i = 0; i < nA; ++i)
-        if (offA + i < p.maxA) p.itemsA[offA + i] = make_int4(bb, (i / nhg) * kTextTile, i % nhg, 0);
-      for (int i = 0; i < nB; ++i)
-        if (offB + i < p.maxB) p.itemsB[offB + i] = make_int4(bb, (i / nch) * kTextTile, i % nch, offS + i);
       for (int i = 0; i < nF; ++i)
         if (offF + i < p.maxF) p.itemsF[offF + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem, 0);
       for (int i = 0; i < nF8; ++i)
         if (offF8 + i < p.maxF) p.itemsF8[offF8 + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem8, 0);
       for (int i = 0; i < nF16; ++i)
         if (offF16 + i < p.maxF) p.itemsF16[offF16 + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem16, 0);
+      p.itemA_off[bb] = offA;
       p.itemB_off[bb] = offB;
       p.slot_off[bb] = offS;
     }
@@ -78,6 +75,7 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
     runS += totS;
   }
   if (tid == 0) {
+    p.itemA_off[p.bt.B] = runA;
     p.itemB_off[p.bt.B] = runB;
     p.slot_off[p.bt.B] = runS;
     if (runA > p.maxA || runB > p.maxB || runF > p.maxF || runF8 > p.maxF || runF16 > p.maxF)

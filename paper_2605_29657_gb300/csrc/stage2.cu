@@ -6,10 +6,14 @@
 // App. A, Eqs. 15-16), and tau2 = lambda2 * s2(r) (Eq. 8).
 //
 // Work is split in two passes so that any S1 size and any text length fit:
-//   stats  (item = sample, 64 text rows, 8 heads): per (j, h) the softmax
-//          max and sum over all keys, online over 64-key chunks;
+//   stats  (item = sample, 64 text rows, 4 heads, key range): per (j, h)
+//          the softmax max and sum over the range's keys, online over
+//          64-key chunks; a sample's keys are split into up to 16 ranges so
+//          that samples too large for the fused kernel still spread over
+//          the SMs;
 //   scores (item = sample, 64 text rows, 128 S1 keys): for every head the
-//          probabilities of the chunk's keys, accumulated over heads in
+//          probabilities of the chunk's keys (the ranges' statistics merged
+//          on load), accumulated over heads in
 //          registers, then the column max over j (atomicMax on the fp32 bit
 //          pattern -- exact and order-free because p >= 0) and the
 //          registers' column sums (written per item and reduced in a fixed
@@ -62,6 +66,16 @@ __device__ __forceinline__ void s2_load_queries(__nv_bfloat16* sdst, const Stage
   }
 }
 
+// The sample whose items [off[b], off[b + 1]) hold item it (off ascending).
+__device__ __forceinline__ int item_sample(const int32_t* off, int B, int it) {
+  int lo = 0, hi = B - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (off[mid] <= it) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
 template <int NT>
 __device__ __forceinline__ void warp_qk128(float (&S)[NT][4], const __nv_bfloat16* sQ, int q_row0,
                                            const __nv_bfloat16* sK, int k_row0, int lane) {
@@ -95,29 +109,44 @@ __global__ void __launch_bounds__(128) s2_stats_kernel(Stage2Params p) {
   const int nA = p.counters[CNT_NA];
   const float c = p.scale * 1.4426950408889634f;
   for (int it = blockIdx.x; it < nA; it += gridDim.x) {
-    const int4 item = p.itemsA[it];
-    const int b = item.x, j0 = item.y, hg = item.z;
+    const int b = item_sample(p.itemA_off, p.bt.B, it);
     const int64_t t0 = p.bt.text_off[b];
     const int M = (int)(p.bt.text_off[b + 1] - t0);
-    const int nq = min(kTextTile, M - j0);
     const int n_img = p.n1[b];
+    const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
+    const int nsp = s2_stat_splits(n_img, M);
+    const int i = it - p.itemA_off[b];
+    const int j0 = (i / (nhg * nsp)) * kTextTile, hg = (i / nsp) % nhg, sp = i % nsp;
+    const int nq = min(kTextTile, M - j0);
     const int n_txt = p.Kt ? min(j0 + kTextTile, M) : 0;
     const int total = n_img + n_txt;
+    // this item's chunks [c0, c1) of the tile's key list (may be empty)
     const int nchunks = (total + KT - 1) / KT;
+    const int per = (nchunks + nsp - 1) / nsp;
+    const int c0 = min(nchunks, sp * per), c1 = min(nchunks, c0 + per);
     const int jA = j0 + warp * 16 + (lane >> 2), jB = jA + 8;
     const int hend = min(p.H, (hg + 1) * kHeadGroup);
+    if (c0 >= c1) {  // an empty key range: neutral partials
+      if ((lane & 3) == 0)
+        for (int h = hg * kHeadGroup; h < hend; ++h) {
+          if (jA < M) p.stats[((t0 + jA) * p.H + h) * kStatSplits + sp] = make_float2(-INFINITY, 0.f);
+          if (jB < M) p.stats[((t0 + jB) * p.H + h) * kStatSplits + sp] = make_float2(-INFINITY, 0.f);
+        }
+      continue;
+    }
     for (int h = hg * kHeadGroup; h < hend; ++h) {
       s2_load_queries(sQ, p, t0 + j0, nq, h, tid, 128);
-      s2_load_keys(sK, p, b, t0, n_img, total, 0, KT, h, tid, 128);
+      s2_load_keys(sK, p, b, t0, n_img, total, c0 * KT, KT, h, tid, 128);
       cp_async_commit();
       float m[2] = {-INFINITY, -INFINITY}, z[2] = {0.f, 0.f};
-      for (int kc = 0; kc < nchunks; ++kc) {
-        if (kc + 1 < nchunks) s2_load_keys(sK + ((kc + 1) & 1) * KT * LD, p, b, t0, n_img, total, (kc + 1) * KT, KT, h, tid, 128);
+      for (int kc = c0; kc < c1; ++kc) {
+        const int lb = (kc - c0) & 1;
+        if (kc + 1 < c1) s2_load_keys(sK + (lb ^ 1) * KT * LD, p, b, t0, n_img, total, (kc + 1) * KT, KT, h, tid, 128);
         cp_async_commit();
         cp_async_wait<1>();
         __syncthreads();
         float S[8][4];
-        warp_qk128<8>(S, sQ, warp * 16, sK + (kc & 1) * KT * LD, 0, lane);
+        warp_qk128<8>(S, sQ, warp * 16, sK + lb * KT * LD, 0, lane);
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
           const int j = half ? jB : jA;
@@ -150,8 +179,8 @@ __global__ void __launch_bounds__(128) s2_stats_kernel(Stage2Params p) {
         __syncthreads();
       }
       if ((lane & 3) == 0) {
-        if (jA < M) p.stats[(t0 + jA) * p.H + h] = make_float2(m[0], 1.0f / z[0]);
-        if (jB < M) p.stats[(t0 + jB) * p.H + h] = make_float2(m[1], 1.0f / z[1]);
+        if (jA < M) p.stats[((t0 + jA) * p.H + h) * kStatSplits + sp] = make_float2(m[0], z[0]);
+        if (jB < M) p.stats[((t0 + jB) * p.H + h) * kStatSplits + sp] = make_float2(m[1], z[1]);
       }
     }
   }
@@ -191,18 +220,32 @@ __global__ void __launch_bounds__(256, 1) s2_scores_kernel(Stage2Params p) {
   const float c = p.scale * 1.4426950408889634f;
   const float invH = 1.0f / (float)p.H;
   for (int it = blockIdx.x; it < nB; it += gridDim.x) {
-    const int4 item = p.itemsB[it];
-    const int b = item.x, j0 = item.y, kc = item.z, slot = item.w;
+    const int b = item_sample(p.itemB_off, p.bt.B, it);
     const int64_t t0 = p.bt.text_off[b];
     const int M = (int)(p.bt.text_off[b + 1] - t0);
-    const int nq = min(kTextTile, M - j0);
     const int n_img = p.n1[b];
+    const int nch = (n_img + kKeyChunk - 1) / kKeyChunk;
+    const int i = it - p.itemB_off[b];
+    const int j0 = (i / nch) * kTextTile, kc = i % nch, slot = p.slot_off[b] + i;
+    const int nq = min(kTextTile, M - j0);
     const int k0 = kc * kKeyChunk;
     const int nk = min(kKeyChunk, n_img - k0);
     const int64_t rbase = p.bt.row_off[b];
+    // merge the key ranges' partial statistics: max, then the sums rescaled to it
+    const int nsp = s2_stat_splits(n_img, M);
     for (int i = tid; i < kTextTile * p.H; i += 256) {
       const int r = i / p.H, h = i - r * p.H;
-      sst[r * p.H + h] = (r < nq) ? p.stats[(t0 + j0 + r) * p.H + h] : make_float2(0.f, 0.f);
+      float2 st = make_float2(0.f, 0.f);
+      if (r < nq) {
+        const float2* ps = p.stats + ((t0 + j0 + r) * p.H + h) * kStatSplits;
+        float mx = -INFINITY;
+        for (int s = 0; s < nsp; ++s) mx = fmaxf(mx, ps[s].x);
+        float z = 0.f;
+        for (int s = 0; s < nsp; ++s)
+          if (ps[s].x != -INFINITY) z += ps[s].y * exp2f(ps[s].x - mx);
+        st = make_float2(mx, 1.0f / z);
+      }
+      sst[r * p.H + h] = st;
     }
     for (int i = tid; i < kKeyChunk; i += 256) {
       const int row = (i < nk) ? p.dense[rbase + k0 + i] : -1;
