@@ -20,6 +20,10 @@ Each function follows one equation of the paper:
 * Stage II set S2 = {v in S1\\{r} : s2(v) >= lambda2 s2(r)} u {r} -- Eq. 8; App. A, Eq. 17
 * lambda2 matching a retained budget over a calibration set      -- App. A, average-budget equation
 * test-time register construction h_r,k = max_v h_v,k, h_v,k = 0 -- Algorithm 1; App. A, register redirection
+* rule variants of the component ablation (App., "compact component
+  ablation"): a mean-based reference instead of the register's score, and a
+  fixed per-sample budget (the top-K rule of Sec. 2) instead of the
+  Stage-II threshold                                             -- Sec. 2, top-K rule; ablation table
 * decoding continues on [S2; T]: order-preserving compaction of
   the kept rows (prefix and KV cache shrink with the kept count) -- Algorithm 1; App. A, Eq. 21
 
@@ -42,6 +46,12 @@ Readings where the paper is silent (each one is also a keyword flag here):
   (causal); ``text_keys="none"`` drops the text keys;
 * the mutual-mode average divides by the segment's row count P+R;
 * ties keep (the test is >=); lambda <= 0 keeps every visual row;
+* the mean threshold takes, per stage, the mean score of that stage's
+  candidates (Stage I: the segment's visual rows; Stage II: the sample's
+  visual S1 rows) as the reference, in both stages;
+* the fixed budget keeps Stage I as in the method and, per sample, the
+  budget[b] visual S1 rows with the largest s2 (all of them when there are
+  fewer); equal scores keep the lower row first;
 * kept rows are emitted in ascending row order, samples in batch order.
 
 Parity pins live in tests/test_oracle_pins.py; no function here is
@@ -257,6 +267,48 @@ def lambda2_for_budget(s2, ref2, keep1, is_reg, row_off, target_count: int):
     return np.float32(ratios[target_count - 1]), int(cand.sum())
 
 
+def mean_reference(s, unit_off, cand):
+    """Mean-threshold reference (component ablation, "Mean threshold"): for
+    each unit [unit_off[u], unit_off[u+1]) the mean of s over its candidate
+    rows (``cand``: visual rows, restricted to S1 in Stage II); 0 for a unit
+    without candidates. The threshold is then s(v) >= lambda * mean.
+    """
+    s = np.asarray(s, dtype=np.float64)
+    cand = np.asarray(cand, dtype=bool)
+    unit_off = as_i64(unit_off)
+    ref = np.zeros(len(unit_off) - 1, dtype=np.float64)
+    for u in range(len(unit_off) - 1):
+        c = cand[unit_off[u]:unit_off[u + 1]]
+        if c.any():
+            ref[u] = np.mean(s[unit_off[u]:unit_off[u + 1]][c])
+    return ref
+
+
+def budget_keep(s, row_off, cand, budget, is_reg, keep_registers: bool = True):
+    """Fixed-budget selection (Sec. 2, S = top-K(V, s); component ablation,
+    "Fixed budget"): in sample b the min(budget[b], #candidates) candidate rows
+    with the largest s. Candidates are ranked by score, high first, and equal
+    scores by row id, low first; the first budget[b] of that order are kept.
+    Register rows are kept iff ``keep_registers``. Returns (keep, count_vis).
+    """
+    s = np.asarray(s, dtype=np.float64)
+    cand = np.asarray(cand, dtype=bool) & ~is_reg
+    row_off = as_i64(row_off)
+    keep = np.zeros(s.shape[0], dtype=bool)
+    B = len(row_off) - 1
+    count = np.zeros(B, dtype=np.int64)
+    for b in range(B):
+        rows = np.arange(row_off[b], row_off[b + 1])[cand[row_off[b]:row_off[b + 1]]]
+        k = max(0, int(budget[b]))
+        order = sorted(rows.tolist(), key=lambda r: (-s[r], r))
+        chosen = order[:k]
+        keep[chosen] = True
+        count[b] = len(chosen)
+    if keep_registers:
+        keep |= is_reg
+    return keep, count
+
+
 # --------------------------------------------------------------------------- Stage II
 
 def stage2_scores(Q_text, K_text, K2, keep1, is_reg, row_off, text_off,
@@ -345,12 +397,16 @@ def near_threshold(s, tau, rel: float = 1e-5) -> np.ndarray:
 
 def prune(batch: dict, lambda1: float, lambda2: float, keep_registers: bool = True,
           text_keys: str = "causal", head_reduce: str = "mean", keep1_override=None,
-          gather=("hidden", "K2", "V"), stage1: str | None = None) -> dict:
+          gather=("hidden", "K2", "V"), stage1: str | None = None, rule: str = "register",
+          budget=None) -> dict:
     """Two-stage OccamToken pruning of one batch (Algorithm 1: Stage I, then Stage II).
 
     ``batch`` holds the synthetic tensors (any array type convertible to
     numpy) and its ``meta`` dict. ``keep1_override`` replaces the Stage-I
     decision (used to re-run Stage II on another Stage-I mask).
+    ``rule``: "register" (the method, Eqs. 5 and 8), "mean" (both references
+    replaced by mean_reference) or "budget" (Stage II replaced by
+    budget_keep with the per-sample ``budget``).
     """
     meta = batch["meta"]
     rows = int(meta["total_rows"])
@@ -366,6 +422,10 @@ def prune(batch: dict, lambda1: float, lambda2: float, keep_registers: bool = Tr
     else:
         s1, ref1 = stage1_mutual(batch["Q1"], batch["K1"], seg_off, reg_idx, reg_off)
     seg_of_row = np.repeat(np.arange(len(seg_off) - 1), np.diff(seg_off))
+    if rule == "mean":
+        ref1 = mean_reference(s1, seg_off, ~is_reg)
+    elif rule not in ("register", "budget"):
+        raise ValueError(rule)
     tau1 = lambda1 * ref1[seg_of_row]
     # S1 = {v : s1(v) >= lambda1 s1(r)} u {r}: the registers are always in S1 (Eq. 5)
     keep1 = threshold(s1, ref1[seg_of_row], lambda1, is_reg, keep_registers=True)
@@ -374,9 +434,14 @@ def prune(batch: dict, lambda1: float, lambda2: float, keep_registers: bool = Tr
     s2, ref2 = stage2_scores(batch["Q_text"], batch.get("K_text"), batch["K2"], keep1, is_reg,
                              row_off, text_off, text_keys=text_keys, head_reduce=head_reduce)
     sample_of_row = np.repeat(np.arange(len(row_off) - 1), np.diff(row_off))
+    if rule == "mean":
+        ref2 = mean_reference(s2, row_off, keep1 & ~is_reg)
     tau2 = lambda2 * ref2[sample_of_row]
-    keep2 = threshold(s2, ref2[sample_of_row], lambda2, is_reg, prev_keep=keep1,
-                      keep_registers=keep_registers)
+    if rule == "budget":
+        keep2, _ = budget_keep(s2, row_off, keep1, budget, is_reg, keep_registers=keep_registers)
+    else:
+        keep2 = threshold(s2, ref2[sample_of_row], lambda2, is_reg, prev_keep=keep1,
+                          keep_registers=keep_registers)
     B = len(row_off) - 1
     count_vis = np.array([int((keep2 & ~is_reg)[row_off[b]:row_off[b + 1]].sum()) for b in range(B)])
     n1_vis = np.array([int((keep1 & ~is_reg)[row_off[b]:row_off[b + 1]].sum()) for b in range(B)])

@@ -560,3 +560,88 @@ def test_register_construction_properties():
     perm[vis0] = perm[vis0[::-1]]
     out2 = O.construct_registers(torch.from_numpy(perm), so, ri, ro, k_reg)
     assert np.array_equal(out2[ri[ro[0]:ro[1]]][:, k_reg], out[ri[ro[0]:ro[1]]][:, k_reg])
+
+
+# ----------------------------------------------------------------------------- rule variants (component ablation)
+
+def test_mean_reference_hand_values():
+    """Mean over the unit's candidates only (registers and rows outside prev_keep excluded); 0 without any."""
+    s = np.array([1.0, 2.0, 6.0, 100.0, 5.0, 7.0, 3.0])
+    is_reg = np.array([False, False, False, True, False, False, True])
+    prev = np.array([True, True, True, True, False, True, True])
+    ref = O.mean_reference(s, np.array([0, 4, 7]), ~is_reg)
+    assert ref.tolist() == [3.0, 6.0]
+    ref = O.mean_reference(s, np.array([0, 4, 7]), ~is_reg & prev)
+    assert ref.tolist() == [3.0, 7.0]
+    ref = O.mean_reference(s, np.array([0, 3, 4, 7]), ~is_reg & prev)
+    assert ref.tolist() == [3.0, 0.0, 7.0]                   # the middle unit holds only a register
+
+
+def _budget_brute(s, rows, k):
+    """The unique k-subset of `rows` whose every member precedes every non-member in the
+    order (score high first, row low first), by enumeration."""
+    import itertools
+    found = []
+    for sub in itertools.combinations(rows, k):
+        rest = [r for r in rows if r not in sub]
+        if all((s[a] > s[d]) or (s[a] == s[d] and a < d) for a in sub for d in rest):
+            found.append(set(sub))
+    assert len(found) == 1
+    return found[0]
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2, 3])
+def test_budget_keep_brute_force(seed):
+    """Fixed budget = the top-K rule of Sec. 2 with ties taken lower row first; brute force over subsets."""
+    rng = np.random.default_rng(seed)
+    row_off = np.array([0, 8, 8, 15, 22])
+    R = row_off[-1]
+    s = rng.choice([0.0, 0.1, 0.2, 0.3, 0.5], R)             # many ties
+    is_reg = np.zeros(R, bool)
+    is_reg[[7, 14]] = True
+    cand = rng.random(R) < 0.8
+    budget = np.array([3, 2, 9, 0])
+    keep, count = O.budget_keep(s, row_off, cand, budget, is_reg, keep_registers=True)
+    for b in range(4):
+        rows = [r for r in range(row_off[b], row_off[b + 1]) if cand[r] and not is_reg[r]]
+        k = min(budget[b], len(rows))
+        assert count[b] == k
+        want = _budget_brute(s, rows, k) if rows else set()
+        got = {r for r in range(row_off[b], row_off[b + 1]) if keep[r] and not is_reg[r]}
+        assert got == want
+    assert keep[is_reg].all()
+    keep0, _ = O.budget_keep(s, row_off, cand, budget, is_reg, keep_registers=False)
+    assert not keep0[is_reg].any()
+
+
+def test_budget_rule_equals_the_method_at_its_own_counts():
+    """With budget[b] = the method's count_vis the fixed-budget rule keeps the same rows (the threshold
+    keeps the top count_vis of s2 per sample; no ties at the threshold in these inputs)."""
+    b = tiny_batch(B=3, segs=2, P=(20, 13, 31), R=2, M=(5, 9, 2), seed=10)
+    ref = O.prune(b, 0.9, 1.2)
+    bud = O.prune(b, 0.9, 1.2, rule="budget", budget=ref["count_vis"])
+    assert np.array_equal(bud["keep1"], ref["keep1"])
+    assert np.array_equal(bud["keep2"], ref["keep2"])
+    half = O.prune(b, 0.9, 1.2, rule="budget", budget=ref["count_vis"] // 2)
+    assert np.array_equal(half["count_vis"], ref["count_vis"] // 2)
+    assert not (half["keep2"] & ~ref["keep2"]).any()           # a smaller budget keeps a subset
+
+
+def test_mean_rule_equals_the_method_at_a_matched_lambda():
+    """One segment, one sample: the mean rule at lambda * s(r) / mean gives the method's threshold, so the
+    same sets (rows within 1e-9 of either threshold are avoided)."""
+    b = tiny_batch(B=1, segs=1, P=(40,), R=2, M=(6,), seed=21)
+    lam1, lam2 = 0.9, 1.1
+    ref = O.prune(b, lam1, lam2)
+    is_reg = ref["is_reg"]
+    m1 = O.mean_reference(ref["s1"], b["meta"]["seg_off_host"], ~is_reg)[0]
+    m2 = O.mean_reference(ref["s2"], b["meta"]["row_off_host"], ref["keep1"] & ~is_reg)[0]
+    mean = O.prune(b, lam1 * ref["ref1"][0] / m1, lam2 * ref["ref2"][0] / m2, rule="mean")
+    assert np.isclose(mean["ref1"][0], m1) and np.isclose(mean["ref2"][0], m2)
+    assert np.allclose(mean["tau1"], ref["tau1"], rtol=1e-12)
+    assert np.allclose(mean["tau2"], ref["tau2"], rtol=1e-12)
+    assert np.min(np.abs(ref["s1"] - ref["tau1"])[~is_reg]) > 1e-9 * ref["tau1"][0]
+    assert np.array_equal(mean["keep1"], ref["keep1"])
+    assert np.array_equal(mean["keep2"], ref["keep2"])
+    # the mean of the visual scores differs from the register reference: the rule is not a no-op
+    assert abs(m1 - ref["ref1"][0]) > 1e-3 * m1
