@@ -67,6 +67,12 @@ enum {
 enum { OCCAM_STAGE1_CLS = 0, OCCAM_STAGE1_MUTUAL = 1 };
 enum { OCCAM_REF_SEGMENT = 0, OCCAM_REF_SAMPLE = 1 };
 enum { OCCAM_TEXT_KEYS_CAUSAL = 0, OCCAM_TEXT_KEYS_NONE = 1 };
+/* Selection rules of occam_prune. REGISTER is the method (Eqs. 5 and 8).
+ * MEAN and BUDGET are the variants of the paper's component ablation:
+ * MEAN replaces the register score by the mean score of the stage's
+ * candidates in both stages; BUDGET keeps Stage I and replaces the Stage-II
+ * threshold by a fixed per-sample budget (the top-K rule of Sec. 2). */
+enum { OCCAM_RULE_REGISTER = 0, OCCAM_RULE_MEAN = 1, OCCAM_RULE_BUDGET = 2 };
 
 #define OCCAM_MAX_GATHER 8
 
@@ -148,6 +154,29 @@ int occam_threshold(const occam_batch* batch, const float* s, const float* ref, 
  * over heads. s2 [total_rows] fp32 = max over j for visual S1 rows, 0 for
  * every other row; ref2 [B] fp32 = the mean over the sample's registers of
  * the mean over j. */
+/* Mean-threshold reference (component ablation, "Mean threshold"). ref[u]
+ * = the mean of s over the candidate rows of unit u: an fp64 sum in a fixed
+ * order, divided by the count and rounded to fp32; 0 for a unit without
+ * candidates. Candidates are the visual rows with prev_keep[row] != 0
+ * (prev_keep NULL: every visual row). unit = segment (ref_scope =
+ * OCCAM_REF_SEGMENT, ref [S_tot]) or sample (OCCAM_REF_SAMPLE, ref [B]).
+ * occam_threshold with this ref applies the mean-threshold rule. */
+int occam_mean_reference(const occam_batch* batch, const float* s, int32_t ref_scope, const uint8_t* prev_keep,
+                         float* ref, void* workspace, size_t workspace_bytes, occam_stream_t stream);
+
+/* Fixed-budget selection (Sec. 2, S = top-K(V, s); component ablation,
+ * "Fixed budget"). Candidates are the visual rows with prev_keep[row] != 0
+ * (prev_keep NULL: every visual row); n_b is sample b's candidate count.
+ * In sample b, keep[row] = 1 for the first min(budget[b], n_b) candidates
+ * in the order "s high first, then row id low first", so equal scores keep
+ * the lower row. budget [B] int32 (device; a negative entry counts as 0).
+ * Register rows get keep_registers, every other row 0. count_vis [B]
+ * (int32, nullable) receives min(budget[b], n_b). Exact: the decision uses
+ * the fp32 values of s. */
+int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* prev_keep, const int32_t* budget,
+                      int32_t keep_registers, uint8_t* keep, int32_t* count_vis, void* workspace,
+                      size_t workspace_bytes, occam_stream_t stream);
+
 int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, const uint8_t* keep1,
                        float* s2, float* ref2, void* workspace, size_t workspace_bytes,
                        occam_stream_t stream);
@@ -199,8 +228,9 @@ int occam_calibrate_lambda2(const occam_batch* batch, const float* s2, const flo
 
 /* The fused path: Stage-I scores -> Stage-I threshold (per segment,
  * lambda1; registers always in S1) -> Stage-II scores over S1 -> Stage-II
- * threshold (per sample, lambda2) -> compaction and gather. Per-sample
- * budgets are outputs, never inputs (App. A: no hard token budget). */
+ * threshold (per sample, lambda2) -> compaction and gather. Under the
+ * method's rule per-sample budgets are outputs, never inputs (App. A: no
+ * hard token budget); only the fixed-budget variant takes them as input. */
 typedef struct occam_prune_args {
   occam_batch batch;
   occam_stage1_args stage1;
@@ -213,6 +243,14 @@ typedef struct occam_prune_args {
   int64_t row_bytes[OCCAM_MAX_GATHER];
   void* dst[OCCAM_MAX_GATHER];
   int64_t capacity_rows;
+  /* OCCAM_RULE_REGISTER (0, the method), OCCAM_RULE_MEAN (ref1 and ref2
+   * become the mean scores of the segment's visual rows and of the sample's
+   * visual S1 rows, as occam_mean_reference computes them; the outputs ref1
+   * and ref2 hold those means) or OCCAM_RULE_BUDGET (Stage I unchanged; S2 =
+   * occam_budget_keep of s2 over the visual S1 rows with `budget`; lambda2
+   * is unused and ref2 keeps the register reference). */
+  int32_t rule;
+  const int32_t* budget; /* [B] int32 device, OCCAM_RULE_BUDGET only (else unused) */
 } occam_prune_args;
 
 /* Outputs of occam_prune. Required: keep2 [total_rows] u8 (S2, registers =

@@ -10,6 +10,9 @@ kept rows -- all in the CUDA kernels of liboccam.so, reached through its C ABI
 from ._lib import (  # noqa: F401
     OCCAM_REF_SAMPLE,
     OCCAM_REF_SEGMENT,
+    OCCAM_RULE_BUDGET,
+    OCCAM_RULE_MEAN,
+    OCCAM_RULE_REGISTER,
     OCCAM_STAGE1_CLS,
     OCCAM_STAGE1_MUTUAL,
     BatchLayout,
@@ -17,11 +20,13 @@ from ._lib import (  # noqa: F401
     PruneCall,
     alloc_workspace,
     library,
+    occam_budget_keep,
     occam_calibrate_lambda2,
     occam_compact,
     occam_compact_noalloc,
     occam_construct_registers,
     occam_get_status,
+    occam_mean_reference,
     occam_prune,
     occam_score_stage1,
     occam_score_stage2,

@@ -32,6 +32,10 @@ OCCAM_STAGE1_MUTUAL = 1
 OCCAM_REF_SEGMENT = 0
 OCCAM_REF_SAMPLE = 1
 OCCAM_MAX_GATHER = 8
+OCCAM_RULE_REGISTER = 0
+OCCAM_RULE_MEAN = 1
+OCCAM_RULE_BUDGET = 2
+RULES = {"register": OCCAM_RULE_REGISTER, "mean": OCCAM_RULE_MEAN, "budget": OCCAM_RULE_BUDGET}
 
 _p = ctypes.c_void_p
 _i32 = ctypes.c_int32
@@ -67,7 +71,7 @@ class CPruneArgs(ctypes.Structure):
         ("lambda1", ctypes.c_float), ("lambda2", ctypes.c_float),
         ("keep_registers", _i32), ("n_tensors", _i32),
         ("src", _p * OCCAM_MAX_GATHER), ("row_bytes", _i64 * OCCAM_MAX_GATHER), ("dst", _p * OCCAM_MAX_GATHER),
-        ("capacity_rows", _i64),
+        ("capacity_rows", _i64), ("rule", _i32), ("budget", _p),
     ]
 
 
@@ -106,7 +110,9 @@ def library() -> ctypes.CDLL:
                                            _p]
         lib.occam_calibrate_lambda2.argtypes = [P(CBatch), _p, _p, _p, _i64, _p, _p, _p, ctypes.c_size_t, _p]
         lib.occam_construct_registers.argtypes = [P(CBatch), _p, _i64, _p, _i32, _p, ctypes.c_size_t, _p]
-        for name in ("occam_construct_registers", "occam_calibrate_lambda2", "occam_workspace_size", "occam_get_status", "occam_score_stage1",
+        lib.occam_mean_reference.argtypes = [P(CBatch), _p, _i32, _p, _p, _p, ctypes.c_size_t, _p]
+        lib.occam_budget_keep.argtypes = [P(CBatch), _p, _p, _p, _i32, _p, _p, _p, ctypes.c_size_t, _p]
+        for name in ("occam_mean_reference", "occam_budget_keep", "occam_construct_registers", "occam_calibrate_lambda2", "occam_workspace_size", "occam_get_status", "occam_score_stage1",
                      "occam_threshold",
                      "occam_score_stage2", "occam_compact", "occam_prune", "occam_prune_traced",
                      "occam_compact_noalloc", "occam_prune_staged"):
@@ -269,6 +275,42 @@ def occam_threshold(layout: BatchLayout, s, ref, ref_scope: int, lam: float, pre
     return keep, count_vis
 
 
+def occam_mean_reference(layout: BatchLayout, s, ref_scope: int, prev_keep=None, ref=None, ws=None, stream=None):
+    """Mean-threshold reference: per segment (OCCAM_REF_SEGMENT) or sample
+    (OCCAM_REF_SAMPLE) the mean of s over the visual rows with prev_keep."""
+    _dev_tensor(s, torch.float32, "s")
+    if prev_keep is not None:
+        _dev_tensor(prev_keep, torch.uint8, "prev_keep")
+    n = layout.S_tot if ref_scope == OCCAM_REF_SEGMENT else layout.B
+    ref = torch.empty(n, dtype=torch.float32, device=layout.device) if ref is None else ref
+    ws = _ws(ws, layout, 1, 1)
+    cb = layout.c()
+    _check(library().occam_mean_reference(ctypes.byref(cb), _ptr(s), int(ref_scope), _ptr(prev_keep), _ptr(ref),
+                                          _ptr(ws), ws.numel(), _stream(stream)), "occam_mean_reference")
+    return ref
+
+
+def occam_budget_keep(layout: BatchLayout, s, budget, prev_keep=None, keep_registers: bool = True, keep=None,
+                      count_vis=None, ws=None, stream=None):
+    """Fixed-budget rule: per sample the budget[b] candidates (visual rows with
+    prev_keep) with the largest s, equal scores lower row first."""
+    _dev_tensor(s, torch.float32, "s")
+    _dev_tensor(budget, torch.int32, "budget")
+    if prev_keep is not None:
+        _dev_tensor(prev_keep, torch.uint8, "prev_keep")
+    if budget.numel() != layout.B:
+        raise OccamError(OCCAM_ERR_INVALID_ARG, "budget must have one entry per sample")
+    dev = layout.device
+    keep = torch.empty(layout.total_rows, dtype=torch.uint8, device=dev) if keep is None else keep
+    count_vis = torch.empty(layout.B, dtype=torch.int32, device=dev) if count_vis is None else count_vis
+    ws = _ws(ws, layout, 1, 1)
+    cb = layout.c()
+    _check(library().occam_budget_keep(ctypes.byref(cb), _ptr(s), _ptr(prev_keep), _ptr(budget),
+                                       int(bool(keep_registers)), _ptr(keep), _ptr(count_vis), _ptr(ws),
+                                       ws.numel(), _stream(stream)), "occam_budget_keep")
+    return keep, count_vis
+
+
 def occam_score_stage2(layout: BatchLayout, Q_text, K2, keep1, K_text=None, s2=None, ref2=None, ws=None,
                        stream=None):
     bf = torch.bfloat16
@@ -385,10 +427,12 @@ class PruneCall:
 
     def __init__(self, layout: BatchLayout, stage1: dict, stage2: dict, lambda1: float, lambda2: float,
                  keep_registers: bool = True, gather=(), capacity_rows: int | None = None,
-                 want=OPTIONAL, ws=None, host_inputs: bool = False):
+                 want=OPTIONAL, ws=None, host_inputs: bool = False, rule: str = "register", budget=None):
         """host_inputs: K2 and the gather tensors may be pinned host tensors,
         read in place through occam_prune_staged (S1 rows of K2 and kept rows
-        only); a device staging tensor for K2 is allocated here."""
+        only); a device staging tensor for K2 is allocated here.
+        rule: "register" (the method), "mean" or "budget" (the component
+        ablation's variants); budget: [B] int32 CUDA tensor for "budget"."""
         bf = torch.bfloat16
         mode = OCCAM_STAGE1_CLS if stage1.get("mode", "cls") == "cls" else OCCAM_STAGE1_MUTUAL
         q = _dev_tensor(stage1["q"], bf, "q")
@@ -444,6 +488,17 @@ class PruneCall:
             a.dst[i] = dst_a[i]
             a.row_bytes[i] = rb_a[i]
         a.capacity_rows = cap
+        if rule not in RULES:
+            raise OccamError(OCCAM_ERR_INVALID_ARG, f"rule must be one of {sorted(RULES)}")
+        a.rule = RULES[rule]
+        if rule == "budget":
+            if budget is None:
+                raise OccamError(OCCAM_ERR_INVALID_ARG, "rule 'budget' needs a budget tensor")
+            budget = _dev_tensor(budget, torch.int32, "budget")
+            if budget.numel() != B:
+                raise OccamError(OCCAM_ERR_INVALID_ARG, "budget must have one entry per sample")
+            self.keep_alive.append(budget)
+            a.budget = _ptr(budget)
         self.args = a
         self.cout = CPruneOut(*[_ptr(o.get(k)) for k in
                                 ("keep2", "out_index", "count_vis", "count_out", "out_off", "keep1", "s1", "ref1",
@@ -480,12 +535,13 @@ class PruneCall:
 
 def occam_prune(layout: BatchLayout, stage1: dict, stage2: dict, lambda1: float, lambda2: float,
                 keep_registers: bool = True, gather=(), capacity_rows: int | None = None,
-                want=PruneCall.OPTIONAL, ws=None, stream=None, host_inputs: bool = False) -> dict:
+                want=PruneCall.OPTIONAL, ws=None, stream=None, host_inputs: bool = False,
+                rule: str = "register", budget=None) -> dict:
     """One fused prune call; returns the output tensors and the gathered rows.
     With host_inputs, K2 and the gather tensors may be pinned host tensors
-    (occam_prune_staged)."""
+    (occam_prune_staged). rule / budget select the rule variant (PruneCall)."""
     call = PruneCall(layout, stage1, stage2, lambda1, lambda2, keep_registers, gather, capacity_rows, want, ws,
-                     host_inputs)
+                     host_inputs, rule, budget)
     out = dict(call(stream))
     out["gathered"] = call.gathered
     out["ws"] = call.ws

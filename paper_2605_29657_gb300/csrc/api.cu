@@ -365,7 +365,8 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
 int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s1, const uint8_t* keep_in,
                      float lambda1, int do_threshold, float* ref1, uint8_t* keep1, int32_t* n1_vis,
                      const occam_stage1_args* a1, float* s2_zero, const Stage2Params* plan, int32_t* count_out,
-                     int32_t* count_vis, cudaStream_t st, Trace trace = Trace(), float* n_eff = nullptr) {
+                     int32_t* count_vis, cudaStream_t st, Trace trace = Trace(), float* n_eff = nullptr,
+                     int ref_mean = 0) {
   Stage1FinalizeParams p;
   p.bt = dev_batch(b);
   const bool cls = a1 && a1->mode == OCCAM_STAGE1_CLS;
@@ -382,6 +383,7 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   p.s1 = s1;
   p.keep_in = keep_in;
   p.lambda1 = lambda1;
+  p.ref_mean = ref_mean;
   p.do_threshold = do_threshold;
   p.ref1 = ref1;
   p.role = at<uint8_t>(ws, L.role);
@@ -527,12 +529,12 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
                    const uint8_t* keep1, const float* s2, int keep_registers, uint8_t* keep_out, int n_tensors,
                    const void* const* src, const int64_t* row_bytes, void* const* dst, int64_t capacity,
                    int32_t* out_index, int32_t* count_out, int32_t* count_vis, int64_t* out_off,
-                   cudaStream_t st, bool do_memsets = true, Trace trace = Trace()) {
+                   cudaStream_t st, bool do_memsets = true, Trace trace = Trace(), bool use_role = false) {
   ScanParams p;
   p.bt = dev_batch(b);
   p.mode = mode;
   p.keep_in = keep_in;
-  p.role = (mode == 1) ? at<uint8_t>(ws, L.role) : nullptr;
+  p.role = (mode == 1 || use_role) ? at<uint8_t>(ws, L.role) : nullptr;
   p.keep1 = keep1;
   p.s2 = s2;
   p.tau2 = at<float>(ws, L.tau2);
@@ -646,6 +648,50 @@ int occam_threshold(const occam_batch* batch, const float* s, const float* ref, 
   return cuda_ok();
 }
 
+int occam_mean_reference(const occam_batch* batch, const float* s, int32_t ref_scope, const uint8_t* prev_keep,
+                         float* ref, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  OCCAM_TRY(check_batch(batch));
+  if (!s || !ref) return OCCAM_ERR_INVALID_ARG;
+  if (ref_scope != OCCAM_REF_SEGMENT && ref_scope != OCCAM_REF_SAMPLE) return OCCAM_ERR_INVALID_ARG;
+  WsLayout L;
+  OCCAM_TRY(check_ws(batch, 1, 1, workspace, workspace_bytes, &L));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  OCCAM_TRY(mark_roles(batch, L, workspace, st));
+  MeanRefParams p;
+  p.bt = dev_batch(batch);
+  p.s = s;
+  p.role = at<uint8_t>(workspace, L.role);
+  p.prev_keep = prev_keep;
+  p.scope = ref_scope;
+  p.ref = ref;
+  p.lambda = 0.f;
+  p.tau = nullptr;
+  mean_ref_kernel<<<ref_scope == OCCAM_REF_SEGMENT ? batch->S_tot : batch->B, 256, 0, st>>>(p);
+  return cuda_ok();
+}
+
+int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* prev_keep, const int32_t* budget,
+                      int32_t keep_registers, uint8_t* keep, int32_t* count_vis, void* workspace,
+                      size_t workspace_bytes, occam_stream_t stream) {
+  OCCAM_TRY(check_batch(batch));
+  if (!s || !budget || !keep) return OCCAM_ERR_INVALID_ARG;
+  WsLayout L;
+  OCCAM_TRY(check_ws(batch, 1, 1, workspace, workspace_bytes, &L));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  OCCAM_TRY(mark_roles(batch, L, workspace, st));
+  BudgetParams p;
+  p.bt = dev_batch(batch);
+  p.s = s;
+  p.role = at<uint8_t>(workspace, L.role);
+  p.prev_keep = prev_keep;
+  p.budget = budget;
+  p.keep_registers = keep_registers;
+  p.keep = keep;
+  p.count_vis = count_vis;
+  budget_keep_kernel<<<batch->B, 1024, 0, st>>>(p);
+  return cuda_ok();
+}
+
 int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, const uint8_t* keep1, float* s2,
                        float* ref2, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
   OCCAM_TRY(check_batch(batch));
@@ -693,6 +739,12 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
       (args->capacity_rows > 0 && !out->out_index))
     return OCCAM_ERR_INVALID_ARG;
   if (!(args->lambda1 == args->lambda1) || !(args->lambda2 == args->lambda2)) return OCCAM_ERR_INVALID_ARG;
+  if (args->rule != OCCAM_RULE_REGISTER && args->rule != OCCAM_RULE_MEAN && args->rule != OCCAM_RULE_BUDGET)
+    return OCCAM_ERR_INVALID_ARG;
+  if (args->rule == OCCAM_RULE_BUDGET) {
+    if (!args->budget) return OCCAM_ERR_INVALID_ARG;
+    OCCAM_TRY(require_device(args->budget));
+  }
   if (out->n_eff && args->stage1.mode != OCCAM_STAGE1_CLS) return OCCAM_ERR_UNSUPPORTED;
   WsLayout L;
   OCCAM_TRY(check_ws(b, args->stage1.H1, args->stage2.H2, workspace, workspace_bytes, &L));
@@ -740,7 +792,8 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   OCCAM_TRY(launch_stage1_scores(b, &args->stage1, L, ws, s1, s2, st, trace));
   const Stage2Params plan = stage2_params(b, &a2, L, ws, s2, ref2, args->lambda2);
   OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, &args->stage1, s2,
-                             &plan, out->count_out, out->count_vis, st, trace, out->n_eff));
+                             &plan, out->count_out, out->count_vis, st, trace, out->n_eff,
+                             args->rule == OCCAM_RULE_MEAN ? 1 : 0));
   if (k2_stage) {
     // the S1 rows of K2 (only those) into the device staging tensor
     StageRowsParams sp;
@@ -754,6 +807,38 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
     OCCAM_CUDA(cudaGetLastError());
   }
   OCCAM_TRY(launch_stage2(b, &a2, L, ws, s2, ref2, args->lambda2, st, trace));
+  if (args->rule == OCCAM_RULE_BUDGET) {
+    // S2 = the budget[b] visual S1 rows with the largest s2 per sample, then
+    // the compaction of that mask
+    BudgetParams bp;
+    bp.bt = dev_batch(b);
+    bp.s = s2;
+    bp.role = at<uint8_t>(ws, L.role);
+    bp.prev_keep = keep1;
+    bp.budget = args->budget;
+    bp.keep_registers = args->keep_registers;
+    bp.keep = out->keep2;
+    bp.count_vis = nullptr;
+    budget_keep_kernel<<<b->B, 1024, 0, st>>>(bp);
+    OCCAM_CUDA(cudaGetLastError());
+    return launch_compact(b, L, ws, 0, out->keep2, nullptr, nullptr, args->keep_registers, nullptr, args->n_tensors,
+                          src, args->row_bytes, dst, args->capacity_rows, out->out_index, out->count_out,
+                          out->count_vis, out->out_off, st, false, trace, true);
+  }
+  if (args->rule == OCCAM_RULE_MEAN) {
+    // the sample's reference becomes the mean s2 of its visual S1 rows
+    MeanRefParams mp;
+    mp.bt = dev_batch(b);
+    mp.s = s2;
+    mp.role = at<uint8_t>(ws, L.role);
+    mp.prev_keep = keep1;
+    mp.scope = OCCAM_REF_SAMPLE;
+    mp.ref = ref2;
+    mp.lambda = args->lambda2;
+    mp.tau = at<float>(ws, L.tau2);
+    mean_ref_kernel<<<b->B, 256, 0, st>>>(mp);
+    OCCAM_CUDA(cudaGetLastError());
+  }
   return launch_compact(b, L, ws, 1, nullptr, keep1, s2, args->keep_registers, out->keep2, args->n_tensors,
                         src, args->row_bytes, dst, args->capacity_rows, out->out_index,
                         out->count_out, out->count_vis, out->out_off, st, false, trace);

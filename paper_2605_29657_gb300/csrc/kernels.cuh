@@ -130,6 +130,7 @@ struct Stage1FinalizeParams {
   const float* s1;          // nullable when keep_in is given
   const uint8_t* keep_in;   // nullable: S1 membership of visual rows given instead of tested
   float lambda1;
+  int ref_mean;      // 1: ref1 = mean of s1 over the segment's visual rows (mean-threshold rule)
   int do_threshold;
   float* ref1;       // nullable
   uint8_t* role;
@@ -220,6 +221,32 @@ struct Lambda2Params {
   int32_t* n_candidates;  // out, nullable
 };
 
+// mean-threshold reference (component ablation): ref[u] = mean of s over the
+// unit's candidate rows (role 0, and prev_keep where given)
+struct MeanRefParams {
+  BatchDev bt;
+  const float* s;
+  const uint8_t* role;
+  const uint8_t* prev_keep;  // nullable
+  int scope;                 // OCCAM_REF_SEGMENT or OCCAM_REF_SAMPLE
+  float* ref;                // [units]
+  float lambda;
+  float* tau;                // nullable: tau[u] = lambda * ref[u]
+};
+
+// fixed-budget rule (Sec. 2 top-K; component ablation): per sample the
+// budget[b] candidates with the largest s, ties lower row first
+struct BudgetParams {
+  BatchDev bt;
+  const float* s;
+  const uint8_t* role;
+  const uint8_t* prev_keep;  // nullable
+  const int32_t* budget;     // [B]
+  int keep_registers;
+  uint8_t* keep;             // [total_rows]
+  int32_t* count_vis;        // nullable, [B]
+};
+
 struct Stage2TcParams {
   BatchDev bt;
   int H;
@@ -270,6 +297,10 @@ __global__ void scan_kernel(ScanParams p);
 __global__ void stage_rows_kernel(StageRowsParams p);
 __global__ void lambda2_select_kernel(Lambda2Params p);
 __global__ void registers_kernel(RegistersParams p);
+
+// rules.cu
+__global__ void mean_ref_kernel(MeanRefParams p);
+__global__ void budget_keep_kernel(BudgetParams p);
 __global__ void gather_kernel(GatherParams p);
 __global__ void offsets_fix_kernel(ScanParams p);
 

@@ -272,8 +272,28 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
     for (int i = ra + tid; i < rb; i += blockDim.x) p.role[p.bt.reg_idx[i]] = 1;
     __syncthreads();
   }
-  // ref1 = mean of s1 over the segment's registers (parallel loads, fixed-order sum)
-  {
+  // ref1 = mean of s1 over the segment's registers (parallel loads, fixed-order
+  // sum); under the mean-threshold rule the mean over its visual rows (fp64)
+  if (p.ref_mean) {
+    const uint8_t* role = staged ? role_loc : p.role + sb;
+    double v = 0.0;
+    if (s1g)
+      for (int r = tid; r < n; r += blockDim.x)
+        if (role[r] == 0) v += (double)(staged ? s1_loc[r] : s1g[sb + r]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __shared__ double dsum[8];
+    if ((tid & 31) == 0) dsum[tid >> 5] = v;
+    __syncthreads();
+    if (tid == 0) {
+      double acc = 0.0;
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) acc += dsum[w];
+      const int nv = n - (rb - ra);
+      sref = nv > 0 ? (float)(acc / (double)nv) : 0.f;
+      if (p.ref1) p.ref1[seg] = sref;
+    }
+    __syncthreads();
+  } else {
     float v = 0.f;
     if (s1g) {
       for (int i = ra + tid; i < rb; i += blockDim.x) {

@@ -98,3 +98,20 @@ def test_no_cpu_fallback_without_device():
     x = torch.zeros(10, 16, 64, dtype=torch.bfloat16)
     with pytest.raises(occ.OccamError):
         occ.occam_score_stage1(lay, occ.OCCAM_STAGE1_CLS, x[:1], x)
+
+
+def test_rule_argument_checked_on_host(lib):
+    import paper_2605_29657_gb300 as occ
+    a = occ._lib.CPruneArgs()
+    a.batch = _host_batch()
+    a.stage1 = occ._lib.CStage1(0, 16, 64, 0x1000, None, 0x1000)
+    a.stage2 = occ._lib.CStage2(32, 128, 0x1000, 0x1000, 0x1000)
+    a.capacity_rows = 0
+    o = occ._lib.CPruneOut()
+    o.keep2 = o.count_vis = o.count_out = o.out_off = 0x1000
+    a.rule = 7
+    assert lib.occam_prune(ctypes.byref(a), ctypes.byref(o), None, 0, None) == occ._lib.OCCAM_ERR_INVALID_ARG
+    a.rule = occ.OCCAM_RULE_BUDGET                               # a budget rule needs the budget array
+    assert lib.occam_prune(ctypes.byref(a), ctypes.byref(o), None, 0, None) == occ._lib.OCCAM_ERR_INVALID_ARG
+    a.rule = occ.OCCAM_RULE_MEAN                                 # valid: fails later, on the workspace
+    assert lib.occam_prune(ctypes.byref(a), ctypes.byref(o), None, 0, None) == occ._lib.OCCAM_ERR_WORKSPACE
