@@ -30,14 +30,17 @@ def to_device(batch: dict, dev) -> dict:
 
 def run_prune(batch: dict, lam1: float, lam2: float, keep_registers: bool = True, dev="cuda",
               capacity_rows=None, gather=True, text_keys: bool = True, g=None, path: str = "auto",
-              host_inputs: bool = False):
+              host_inputs: bool = False, rule: str = "register", budget=None):
     """path: "auto" (fused tensor-core Stage II where it fits) or "twopass".
-    host_inputs: K2, hidden and V stay in pinned host memory (occam_prune_staged)."""
+    host_inputs: K2, hidden and V stay in pinned host memory (occam_prune_staged).
+    rule / budget: the selection rule ("register", "mean", "budget") and the
+    per-sample budget array (host ints) of the "budget" rule."""
     import os
     old = os.environ.get("OCCAM_STAGE2_PATH")
     os.environ["OCCAM_STAGE2_PATH"] = path
     try:
-        return _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs)
+        return _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs,
+                          rule, budget)
     finally:
         if old is None:
             os.environ.pop("OCCAM_STAGE2_PATH", None)
@@ -45,7 +48,8 @@ def run_prune(batch: dict, lam1: float, lam2: float, keep_registers: bool = True
             os.environ["OCCAM_STAGE2_PATH"] = old
 
 
-def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs=False):
+def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs=False,
+               rule="register", budget=None):
     import paper_2605_29657_gb300 as occ
 
     m = batch["meta"]
@@ -63,8 +67,9 @@ def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, te
     tensors = ()
     if gather:
         tensors = (g["hidden"], g["K2"].view(g["K2"].shape[0], -1), g["V"])
+    bud = None if budget is None else torch.as_tensor(np.asarray(budget, np.int32)).to(dev)
     out = occ.occam_prune(layout, st1, st2, lam1, lam2, keep_registers=keep_registers, gather=tensors,
-                          capacity_rows=capacity_rows, host_inputs=host_inputs)
+                          capacity_rows=capacity_rows, host_inputs=host_inputs, rule=rule, budget=bud)
     torch.cuda.synchronize()
     status = occ.occam_get_status(out["ws"])
     res = {k: v.cpu().numpy() for k, v in out.items() if isinstance(v, torch.Tensor) and k != "ws"}
@@ -85,10 +90,17 @@ def close(name, got, want, rtol=RTOL, atol=ATOL):
 
 
 def check_prune(batch: dict, gpu: dict, lam1: float, lam2: float, keep_registers: bool = True,
-                text_keys: str = "causal", gather=True, capacity_rows=None) -> dict:
-    """Compares a GPU prune result with the oracle; returns a small report."""
+                text_keys: str = "causal", gather=True, capacity_rows=None, rule: str = "register",
+                budget=None) -> dict:
+    """Compares a GPU prune result with the oracle; returns a small report.
+
+    Under the "budget" rule the Stage-II selection is an integer decision
+    taken from fp32 scores: the GPU's keep2 must equal the oracle's
+    budget_keep applied to the GPU's own s2 exactly, and where it differs
+    from the oracle's keep2 the row's oracle s2 must lie within 1e-5
+    (relative) of its sample's budget-th largest score."""
     ref = O.prune(batch, lam1, lam2, keep_registers=keep_registers, text_keys=text_keys,
-                  gather=("hidden", "K2", "V") if gather else ())
+                  gather=("hidden", "K2", "V") if gather else (), rule=rule, budget=budget)
     meta = batch["meta"]
     row_off = meta["row_off_host"]
     B = meta["B"]
@@ -104,12 +116,27 @@ def check_prune(batch: dict, gpu: dict, lam1: float, lam2: float, keep_registers
     if d1.any():
         rep["cascade"] = True
         ref = O.prune(batch, lam1, lam2, keep_registers=keep_registers, text_keys=text_keys,
-                      keep1_override=k1, gather=("hidden", "K2", "V") if gather else ())
+                      keep1_override=k1, gather=("hidden", "K2", "V") if gather else (), rule=rule,
+                      budget=budget)
     close("s2", gpu["s2"], ref["s2"])
     close("ref2", gpu["ref2"], ref["ref2"])
     k2 = gpu["keep2"].astype(bool)
     d2 = k2 != ref["keep2"]
-    assert not (d2 & ~ref["near2"]).any(), f"keep2 differs outside the band at rows {np.nonzero(d2 & ~ref['near2'])[0][:10]}"
+    if rule == "budget":
+        own, _ = O.budget_keep(gpu["s2"].astype(np.float64), row_off, k1, budget, is_reg,
+                               keep_registers=keep_registers)
+        assert np.array_equal(k2, own), "keep2 is not the budget selection of the GPU's own s2"
+        near = np.zeros_like(d2)
+        for b in range(B):
+            a, z = row_off[b], row_off[b + 1]
+            c = np.nonzero(k1[a:z] & ~is_reg[a:z])[0] + a
+            k = min(max(int(budget[b]), 0), len(c))
+            if 0 < k < len(c):
+                kth = np.sort(ref["s2"][c])[::-1][k - 1]
+                near[c] = np.abs(ref["s2"][c] - kth) <= 1e-5 * kth
+        assert not (d2 & ~near).any(), f"keep2 differs away from the budget boundary at {np.nonzero(d2 & ~near)[0][:10]}"
+    else:
+        assert not (d2 & ~ref["near2"]).any(), f"keep2 differs outside the band at rows {np.nonzero(d2 & ~ref['near2'])[0][:10]}"
     rep["band2"] = int(d2.sum())
     assert (k2[is_reg] == keep_registers).all(), "register rows in keep2 must equal keep_registers"
     # compaction must be exact for the GPU's own mask
