@@ -318,6 +318,8 @@ def stage2_scores(Q_text, K_text, K2, keep1, is_reg, row_off, text_off,
     For sample b the keys are the S1 rows (visual rows with keep1 and all
     registers, in row order) followed, for text token j, by the text keys
     0..j. Per head A = softmax(q_j k^T / sqrt(d2)); p[j, row] = mean_h A_h.
+    K2 / K_text may hold fewer heads than Q_text (grouped-query attention);
+    query head h then uses key head h // (H / H_kv).
     s2[v] = max_j p[j, v] for visual S1 rows (0 elsewhere) and
     ref2[b] = mean over the sample's registers of mean_j p[j, reg].
     Returns (s2 [rows], ref2 [B]).
@@ -329,7 +331,10 @@ def stage2_scores(Q_text, K_text, K2, keep1, is_reg, row_off, text_off,
     text_off = as_i64(text_off)
     keep1 = np.asarray(keep1, dtype=bool)
     B = row_off.shape[0] - 1
-    H, d = K.shape[1], K.shape[2]
+    # grouped-query attention: H query heads share H_kv key heads, query head h reading key head h // (H / H_kv)
+    H, Hkv, d = Q.shape[1], K.shape[1], K.shape[2]
+    assert H % Hkv == 0
+    grp = H // Hkv
     scale = 1.0 / np.sqrt(d)
     s2 = np.zeros(K.shape[0], dtype=np.float64)
     ref2 = np.zeros(B, dtype=np.float64)
@@ -344,9 +349,9 @@ def stage2_scores(Q_text, K_text, K2, keep1, is_reg, row_off, text_off,
         pmax = np.zeros((M, n), dtype=np.float64)
         for h in range(H):
             q = Q[t0:t1, h, :]                                # [M, d]
-            li = (q @ K[s1_rows, h, :].T) * scale             # [M, n]
+            li = (q @ K[s1_rows, h // grp, :].T) * scale      # [M, n]
             if Kt is not None:
-                lt = (q @ Kt[t0:t1, h, :].T) * scale          # [M, M]
+                lt = (q @ Kt[t0:t1, h // grp, :].T) * scale   # [M, M]
                 causal = np.tril(np.ones((M, M), dtype=bool))
                 lt = np.where(causal, lt, -np.inf)
                 A = softmax(np.concatenate([li, lt], axis=1), axis=1)[:, :n]

@@ -40,6 +40,7 @@ class Workload:
     seed: int
     H2: int = 32
     d2: int = 128
+    H2kv: int = 0               # key / value heads of K2, K_text (0: H2; fewer: grouped-query attention)
     hidden: int = 4096
     query_bias: float = 0.0     # mutual mode: per-segment shared query component (fraction of sqrt(d1))
     lambda1: float = 0.045

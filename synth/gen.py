@@ -144,10 +144,10 @@ def _apply_dups(x: torch.Tensor, steps, rho: float) -> torch.Tensor:
     return x
 
 
-def _stage2(out, gen, T, rows, H2, d2, device, dups, rho, sink_rows):
+def _stage2(out, gen, T, rows, H2, H2kv, d2, device, dups, rho, sink_rows):
     out["Q_text"] = _randn(gen, (T, H2, d2), device).to(BF16)
-    out["K_text"] = _randn(gen, (T, H2, d2), device).to(BF16)
-    K2 = _randn(gen, (rows, H2, d2), device)
+    out["K_text"] = _randn(gen, (T, H2kv, d2), device).to(BF16)
+    K2 = _randn(gen, (rows, H2kv, d2), device)
     K2 = _apply_dups(K2, dups, rho)
     K2[sink_rows] *= 8.0
     out["K2"] = K2.to(BF16)
@@ -220,7 +220,7 @@ def make_batch(w: Workload | str, device: str | torch.device = "cpu", seed: int 
     if not with_stage2:
         with_gather = False
     else:
-        _stage2(out, gen, T, rows, H2, d2, device, dups, rho, sink_rows)
+        _stage2(out, gen, T, rows, H2, w.H2kv or H2, d2, device, dups, rho, sink_rows)
 
     # ---- rows gathered after pruning (hidden states and values of layer l)
     if with_gather:
@@ -238,7 +238,7 @@ def make_batch(w: Workload | str, device: str | torch.device = "cpu", seed: int 
         max_sample_rows=int(np.diff(lay["row_off"]).max()),
         max_text=int(M.max()), min_text=int(M.min()),
         regs_per_seg=w.regs, segs_per_sample=w.segs,
-        H1=H1, d1=d1, H2=H2, d2=d2, hidden=w.hidden, stage1=w.stage1,
+        H1=H1, d1=d1, H2=H2, d2=d2, H2kv=w.H2kv or H2, hidden=w.hidden, stage1=w.stage1,
         lambda1=w.lambda1, lambda2=w.lambda2, beta1=w.beta1,
         P=P, M=M, sinks=sinks, seed=seed,
         **{k + "_host": lay[k] for k in lay},
@@ -247,7 +247,7 @@ def make_batch(w: Workload | str, device: str | torch.device = "cpu", seed: int 
     return out
 
 
-def tiny_batch(B=2, segs=2, P=(5, 7), R=2, M=(3, 4), H1=2, d1=8, H2=2, d2=8, hidden=16,
+def tiny_batch(B=2, segs=2, P=(5, 7), R=2, M=(3, 4), H1=2, d1=8, H2=2, d2=8, hidden=16, H2kv=0,
                stage1="cls", seed=0, beta1=1.5, query_bias=0.5, sinks=("count", 1),
                dup=None, lambda1=0.5, lambda2=1.0) -> dict:
     """A small batch with explicit sizes (for oracle pins and ragged parity cases).
@@ -260,7 +260,7 @@ def tiny_batch(B=2, segs=2, P=(5, 7), R=2, M=(3, 4), H1=2, d1=8, H2=2, d2=8, hid
     w = Workload(
         name="tiny", description="explicit small sizes", B=B, segs=segs, vis=("fixed", 0),
         regs=R, stage1=stage1, H1=H1, d1=d1, sinks=sinks, dup=dup, M=("fixed", 0), seed=seed,
-        H2=H2, d2=d2, hidden=hidden, query_bias=query_bias, beta1=beta1,
+        H2=H2, d2=d2, H2kv=H2kv, hidden=hidden, query_bias=query_bias, beta1=beta1,
         lambda1=lambda1, lambda2=lambda2,
     )
     return make_batch(w, "cpu", P=P, M=M)

@@ -645,3 +645,26 @@ def test_mean_rule_equals_the_method_at_a_matched_lambda():
     assert np.array_equal(mean["keep2"], ref["keep2"])
     # the mean of the visual scores differs from the register reference: the rule is not a no-op
     assert abs(m1 - ref["ref1"][0]) > 1e-3 * m1
+
+
+# ----------------------------------------------------------------------------- grouped-query Stage II
+
+@pytest.mark.parametrize("text_keys", ["causal", "none"])
+def test_grouped_query_heads_equal_expanded_keys(text_keys):
+    """H_kv key heads shared by groups of H / H_kv query heads = H separate heads whose keys are copies
+    (query head h reading key head h // group). A wrong group index (h % H_kv) fails this."""
+    b = tiny_batch(B=2, segs=2, P=(9, 14), R=2, M=(5, 7), H2=8, H2kv=2, d2=16, seed=91)
+    assert b["K2"].shape[1] == 2 and b["Q_text"].shape[1] == 8
+    full = dict(b)
+    idx = torch.arange(8) // 4
+    full["K2"] = b["K2"][:, idx, :].contiguous()
+    full["K_text"] = b["K_text"][:, idx, :].contiguous()
+    g = O.prune(b, 0.6, 1.1, text_keys=text_keys)
+    e = O.prune(full, 0.6, 1.1, text_keys=text_keys)
+    assert np.array_equal(g["s2"], e["s2"]) and np.array_equal(g["ref2"], e["ref2"])
+    assert np.array_equal(g["keep2"], e["keep2"])
+    # and the grouping matters: pairing query head h with key head h % H_kv gives other scores
+    wrong = dict(b)
+    wrong["K2"] = b["K2"][:, torch.arange(8) % 2, :].contiguous()
+    wrong["K_text"] = b["K_text"][:, torch.arange(8) % 2, :].contiguous()
+    assert not np.allclose(O.prune(wrong, 0.6, 1.1, text_keys=text_keys)["s2"], g["s2"])
