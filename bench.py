@@ -149,7 +149,9 @@ def algorithmic_bytes(meta: dict, n1_total: int, kept_total: int) -> dict:
     rows, S, T = meta["total_rows"], meta["S_tot"], meta["total_text"]
     H1, d1, H2, d2, hid = meta["H1"], meta["d1"], meta["H2"], meta["d2"], meta["hidden"]
     k1row = H1 * d1 * 2
-    k2row = H2 * d2 * 2
+    H2kv = meta.get("H2kv", H2)          # key heads (fewer than H2 under grouped-query attention)
+    k2row = H2kv * d2 * 2                # one K2 / K_text row
+    qrow = H2 * d2 * 2                   # one Q_text row
     hrow = hid * 2                       # bytes of one hidden / V row (bf16)
     cls = meta["stage1"] == "cls"
     b = {}
@@ -160,14 +162,14 @@ def algorithmic_bytes(meta: dict, n1_total: int, kept_total: int) -> dict:
         b["stage1"] = 2 * rows * 2 * k1row                               # Q1 and K1 in each of the two passes
         b["stage1_finalize"] = rows * (4 + 1 + 1 + 4)                   # s1, role, keep1, list
     b["s1_list_plan"] = 0                                            # planned inside the finalize kernel
-    b["stage2_fused"] = n1_total * k2row + 2 * T * k2row               # S1 keys once, Q + K_text
-    b["stage2_twopass"] = 2 * n1_total * k2row + 3 * T * k2row + 2 * T * H2 * 8  # both passes
+    b["stage2_fused"] = n1_total * k2row + T * (qrow + k2row)          # S1 keys once, Q + K_text
+    b["stage2_twopass"] = 2 * n1_total * k2row + T * (2 * qrow + k2row) + 2 * T * H2 * 8  # both passes
     b["scan"] = rows * (1 + 1 + 4 + 1) + kept_total * 4              # keep1, role, s2, keep2, out_index
     b["gather"] = kept_total * 2 * (2 * hrow + k2row)                # read + write hidden, K, V rows
     # whole step, each byte once: K1, S1 keys, text Q/K, hidden+V of kept rows
     # (their K rows were read for scoring), writes of the 3 gathered rows
     stage1_in = rows * k1row + 2 * S * k1row if cls else 2 * rows * k1row   # K1 (+ q/k_cls) or Q1 + K1, once
-    step = (stage1_in + n1_total * k2row + 2 * T * k2row
+    step = (stage1_in + n1_total * k2row + T * (qrow + k2row)
             + kept_total * (2 * hrow) + kept_total * (2 * hrow + k2row) + rows + kept_total * 4)
     b["step"] = step
     return b
@@ -346,7 +348,7 @@ def run_ours(args, rank, world, local):
         copied = [torch.cuda.Event() for _ in range(nset)]
         done = [torch.cuda.Event() for _ in range(nset)]
         copied_bytes = sum(host[k].numel() * host[k].element_size() for k in copy_names)
-        k2row = meta["H2"] * meta["d2"] * 2
+        k2row = meta.get("H2kv", meta["H2"]) * meta["d2"] * 2
         # the kept rows of K2 are read from the staged S1 rows on the device
         kept_row = sum(host[k][0].numel() * host[k].element_size() for k in ("hidden", "V"))
         in_place = n1_total * k2row + kept_total * kept_row
@@ -430,6 +432,32 @@ def run_ours(args, rank, world, local):
                                       "how": "in place on hidden [rows, 4096] bf16, per segment"},
             "n_eff": "computed in the Stage-I finalize of every timed step ([CLS] mode, optional output)",
         }
+        # the component ablation's rule variants as whole prune steps on the
+        # same tensors. Mean threshold: lambdas scaled by the step's average
+        # register / mean reference ratio (thresholds matched on average).
+        # Fixed budget: every sample keeps the step's average count_vis.
+        ref1m = occ.occam_mean_reference(layout, out["s1"], occ.OCCAM_REF_SEGMENT)
+        ref2m = occ.occam_mean_reference(layout, out["s2"], occ.OCCAM_REF_SAMPLE, prev_keep=out["keep1"])
+        r1 = float((out["ref1"] / ref1m.clamp_min(1e-30)).mean().item())
+        r2 = float((out["ref2"] / ref2m.clamp_min(1e-30)).mean().item())
+        avg_budget = int(round(float(out["count_vis"].float().mean().item())))
+        budget = torch.full((meta["B"],), avg_budget, dtype=torch.int32, device=dev)
+        variants = {}
+        for rule, l1, l2, bud in (("mean", w.lambda1 * r1, w.lambda2 * r2, None),
+                                  ("budget", w.lambda1, w.lambda2, budget)):
+            vcall = occ.PruneCall(layout, stage1_of(batch),
+                                  dict(Q_text=batch["Q_text"], K_text=batch["K_text"], K2=batch["K2"]),
+                                  l1, l2, keep_registers=True, gather=gather, rule=rule, budget=bud,
+                                  ws=call.ws)
+            v_ms = timed(lambda: vcall())
+            if vcall.status() != 0:
+                raise RuntimeError(f"device status after the {rule} rule")
+            variants[rule] = {"ms_per_step": v_ms, "images_per_s": meta["B"] / (v_ms / 1e3),
+                              "kept_rows": int(vcall.out["out_off"][-1].item()),
+                              "lambda1": l1, "lambda2": l2 if rule == "mean" else None,
+                              "budget_per_sample": avg_budget if rule == "budget" else None}
+            del vcall
+        next_rows["rule_variants"] = variants
 
     if rank != 0:
         if world > 1:

@@ -110,15 +110,20 @@ typedef struct occam_stage1_args {
 } occam_stage1_args;
 
 /* Stage-II inputs (Sec. 3.5): layer-l queries and keys. Q_text [total_text,H2,d2];
- * K_text [total_text,H2,d2] or NULL (= OCCAM_TEXT_KEYS_NONE: the text keys are
- * left out of the softmax); K2 [rows,H2,d2], read only at S1 rows. Built for
- * d2 = 128 and 1 <= H2 <= 64. */
+ * K_text [total_text,H2_kv,d2] or NULL (= OCCAM_TEXT_KEYS_NONE: the text keys
+ * are left out of the softmax); K2 [rows,H2_kv,d2], read only at S1 rows.
+ * Built for d2 = 128 and 1 <= H2 <= 64. */
 typedef struct occam_stage2_args {
   int32_t H2;
   int32_t d2;
   const void* Q_text;
   const void* K_text;
   const void* K2;
+  /* key / value heads of K2 and K_text: 0 (or H2) for one per query head;
+   * a divisor of H2 for grouped-query attention, where query head h reads
+   * key head h / (H2 / H2_kv). Rows of K2 and K_text then hold H2_kv * d2
+   * values, rows of Q_text H2 * d2. */
+  int32_t H2_kv;
 } occam_stage2_args;
 
 /* Size of the scratch workspace every entry point needs for this batch and

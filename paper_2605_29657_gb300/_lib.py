@@ -62,7 +62,7 @@ class CStage1(ctypes.Structure):
 
 
 class CStage2(ctypes.Structure):
-    _fields_ = [("H2", _i32), ("d2", _i32), ("Q_text", _p), ("K_text", _p), ("K2", _p)]
+    _fields_ = [("H2", _i32), ("d2", _i32), ("Q_text", _p), ("K_text", _p), ("K2", _p), ("H2_kv", _i32)]
 
 
 class CPruneArgs(ctypes.Structure):
@@ -317,13 +317,14 @@ def occam_score_stage2(layout: BatchLayout, Q_text, K2, keep1, K_text=None, s2=N
     _dev_tensor(Q_text, bf, "Q_text"); _dev_tensor(K2, bf, "K2"); _dev_tensor(keep1, torch.uint8, "keep1")
     if K_text is not None:
         _dev_tensor(K_text, bf, "K_text")
-    H2, d2 = int(K2.shape[1]), int(K2.shape[2])
+    # query heads from Q_text, key heads from K2 (fewer under grouped-query attention)
+    H2, d2, H2kv = int(Q_text.shape[1]), int(K2.shape[2]), int(K2.shape[1])
     dev = layout.device
     s2 = torch.empty(layout.total_rows, dtype=torch.float32, device=dev) if s2 is None else s2
     ref2 = torch.empty(layout.B, dtype=torch.float32, device=dev) if ref2 is None else ref2
     ws = _ws(ws, layout, 1, H2)
     cb = layout.c()
-    a = CStage2(H2, d2, _ptr(Q_text), _ptr(K_text), _ptr(K2))
+    a = CStage2(H2, d2, _ptr(Q_text), _ptr(K_text), _ptr(K2), H2kv)
     _check(library().occam_score_stage2(ctypes.byref(cb), ctypes.byref(a), _ptr(keep1), _ptr(s2), _ptr(ref2),
                                         _ptr(ws), ws.numel(), _stream(stream)), "occam_score_stage2")
     return s2, ref2
@@ -446,7 +447,8 @@ class PruneCall:
         if K_text is not None:
             _dev_tensor(K_text, bf, "K_text")
         H1, d1 = int(K1.shape[1]), int(K1.shape[2])
-        H2, d2 = int(K2.shape[1]), int(K2.shape[2])
+        # query heads from Q_text, key heads from K2 (fewer under grouped-query attention)
+        H2, d2, H2kv = int(Q_text.shape[1]), int(K2.shape[2]), int(K2.shape[1])
         dev = layout.device
         self.layout = layout
         self.keep_alive = [q, K1, k_cls, Q_text, K2, K_text]
@@ -478,7 +480,7 @@ class PruneCall:
         a = CPruneArgs()
         a.batch = layout.c()
         a.stage1 = CStage1(mode, H1, d1, _ptr(q), _ptr(k_cls), _ptr(K1))
-        a.stage2 = CStage2(H2, d2, _ptr(Q_text), _ptr(K_text), _ptr(K2))
+        a.stage2 = CStage2(H2, d2, _ptr(Q_text), _ptr(K_text), _ptr(K2), H2kv)
         a.lambda1 = float(lambda1)
         a.lambda2 = float(lambda2)
         a.keep_registers = int(bool(keep_registers))

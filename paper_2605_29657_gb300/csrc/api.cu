@@ -249,9 +249,13 @@ int check_stage1(const occam_batch* b, const occam_stage1_args* a) {
   return OCCAM_OK;
 }
 
+// Key / value heads of Stage II: H2_kv, where 0 stands for H2.
+int kv_heads(const occam_stage2_args* a) { return a->H2_kv > 0 ? a->H2_kv : a->H2; }
+
 int check_stage2(const occam_stage2_args* a) {
   if (!a || !a->Q_text || !a->K2) return OCCAM_ERR_INVALID_ARG;
   if (a->d2 != 128 || a->H2 < 1 || a->H2 > 64) return OCCAM_ERR_UNSUPPORTED;
+  if (a->H2_kv < 0 || a->H2 % kv_heads(a) != 0) return OCCAM_ERR_INVALID_ARG;
   if (!aligned16(a->Q_text) || !aligned16(a->K2) || (a->K_text && !aligned16(a->K_text)))
     return OCCAM_ERR_INVALID_ARG;
   return OCCAM_OK;
@@ -419,6 +423,7 @@ Stage2Params stage2_params(const occam_batch* b, const occam_stage2_args* a, con
   Stage2Params p;
   p.bt = dev_batch(b);
   p.H = a->H2;
+  p.Hkv = kv_heads(a);
   p.Q = static_cast<const __nv_bfloat16*>(a->Q_text);
   p.Kt = static_cast<const __nv_bfloat16*>(a->K_text);
   p.K = static_cast<const __nv_bfloat16*>(a->K2);
@@ -464,11 +469,14 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     // S1 key rows are gathered four at a time (TMA gather4: box one row
     // high); text key rows, which are consecutive, come in boxes of 16 rows
     CUtensorMap mk, mkt;
-    if (!encode_map(&mk, a->K2, b->total_rows, cols, 1)) return OCCAM_ERR_CUDA;
-    if (!encode_map(&mkt, kt, b->total_text, cols, 16)) return OCCAM_ERR_CUDA;
+    // keys: H2_kv heads per row (grouped-query attention), queries H2
+    const int64_t cols_kv = (int64_t)kv_heads(a) * 128;
+    if (!encode_map(&mk, a->K2, b->total_rows, cols_kv, 1)) return OCCAM_ERR_CUDA;
+    if (!encode_map(&mkt, kt, b->total_text, a->K_text ? cols_kv : cols, 16)) return OCCAM_ERR_CUDA;
     Stage2TcParams q;
     q.bt = p.bt;
     q.H = a->H2;
+    q.kv_group = a->H2 / kv_heads(a);
     q.K = static_cast<const __nv_bfloat16*>(a->K2);
     q.Kt = static_cast<const __nv_bfloat16*>(kt);
     q.scale_log2 = p.scale * 1.4426950408889634f;
@@ -756,7 +764,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   if (args->stage2.K_text) OCCAM_TRY(require_device(args->stage2.K_text));
   occam_stage2_args a2 = args->stage2;
   const void* k2_src = nullptr;
-  const int64_t k2_row = (int64_t)a2.H2 * a2.d2 * 2;
+  const int64_t k2_row = (int64_t)kv_heads(&a2) * a2.d2 * 2;
   if (k2_stage) {
     if (!aligned16(k2_stage) || k2_stage_bytes < (size_t)(b->total_rows * k2_row)) return OCCAM_ERR_INVALID_ARG;
     OCCAM_TRY(require_device(k2_stage));

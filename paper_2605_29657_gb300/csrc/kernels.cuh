@@ -82,9 +82,10 @@ struct ThresholdParams {
 struct Stage2Params {
   BatchDev bt;
   int H;  // H2, d2 = 128
+  int Hkv;  // key / value heads: H, or a divisor of H (grouped-query attention)
   const __nv_bfloat16* Q;   // [total_text, H, 128]
-  const __nv_bfloat16* Kt;  // nullable
-  const __nv_bfloat16* K;   // [rows, H, 128]
+  const __nv_bfloat16* Kt;  // nullable, [total_text, Hkv, 128]
+  const __nv_bfloat16* K;   // [rows, Hkv, 128]
   float scale;
   const uint8_t* role;
   int32_t* dense;           // per sample S1 list at row_off[b]
@@ -250,8 +251,9 @@ struct BudgetParams {
 struct Stage2TcParams {
   BatchDev bt;
   int H;
-  const __nv_bfloat16* K;   // [rows, H, 128]
-  const __nv_bfloat16* Kt;  // [total_text, H, 128] (any valid pointer when has_text == 0)
+  int kv_group;             // query heads per key / value head (1 unless grouped-query attention)
+  const __nv_bfloat16* K;   // [rows, H / kv_group, 128]
+  const __nv_bfloat16* Kt;  // [total_text, H / kv_group, 128] (any valid pointer when has_text == 0)
   float scale_log2;
   int has_text;
   const int32_t* dense;

@@ -31,23 +31,25 @@ constexpr int LD = D + 8;  // padded smem row (272 B): conflict-free ldmatrix
 constexpr int KT = 64;     // keys per stats chunk
 }  // namespace s2k
 
-// copy one 64- or 128-key chunk of head h into sdst[key][0..128) (stride LD)
+// copy one 64- or 128-key chunk of query head h's keys into sdst[key][0..128) (stride LD)
 __device__ __forceinline__ void s2_load_keys(__nv_bfloat16* sdst, const Stage2Params& p, int b, int64_t t0,
                                              int n_img, int total, int k0, int nkeys_tile, int h, int tid,
                                              int nthreads) {
   using namespace s2k;
   const int64_t rbase = p.bt.row_off[b];
-  const int64_t HD = (int64_t)p.H * D;
+  // grouped-query attention: query head h reads key head h / (H / Hkv)
+  const int64_t HD = (int64_t)p.Hkv * D;
+  const int64_t hoff = (int64_t)(h / (p.H / p.Hkv)) * D;
   for (int i = tid; i < nkeys_tile * 16; i += nthreads) {
     const int kr = i >> 4, v = i & 15;
     const int kk = k0 + kr;
     const __nv_bfloat16* src = p.K;
     int bytes = 0;
     if (kk < n_img) {
-      src = p.K + (int64_t)p.dense[rbase + kk] * HD + (int64_t)h * D + v * 8;
+      src = p.K + (int64_t)p.dense[rbase + kk] * HD + hoff + v * 8;
       bytes = 16;
     } else if (kk < total) {
-      src = p.Kt + (t0 + (kk - n_img)) * HD + (int64_t)h * D + v * 8;
+      src = p.Kt + (t0 + (kk - n_img)) * HD + hoff + v * 8;
       bytes = 16;
     }
     cp_async16_zfill(sdst + kr * LD + v * 8, src, bytes);

@@ -400,6 +400,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         bool ok = true;
         for (int h = 0; h < H && ok; ++h) {
           const int kb = kcnt & 1;
+          const int hkv = h / p.kv_group;  // the key / value head query head h reads
           if (!tc::bar_wait(&sm.kempty[kb], ((kcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
             fail(sm, p.status);
             ok = false;
@@ -438,12 +439,12 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
               int y[4];
 #pragma unroll
               for (int i = 0; i < 4; ++i) y[i] = sm.kidx[ib][r0 + i < g.own_img ? r0 + i : 0];
-              tc::tma_gather4(dst + kblk * G::KBLK + r0 * 128, &mapK, h * 128 + kblk * 64, y[0], y[1], y[2], y[3],
+              tc::tma_gather4(dst + kblk * G::KBLK + r0 * 128, &mapK, hkv * 128 + kblk * 64, y[0], y[1], y[2], y[3],
                               &sm.kfull[kb]);
             } else {
               const int t0 = ((u >> 1) - gi4) * TXT_BOX;
-              tc::tma_load_2d(dst + kblk * G::KBLK + (g.ip + t0) * 128, &mapKt, h * 128 + kblk * 64, (int)(tbase + t0),
-                              &sm.kfull[kb]);
+              tc::tma_load_2d(dst + kblk * G::KBLK + (g.ip + t0) * 128, &mapKt, hkv * 128 + kblk * 64,
+                              (int)(tbase + t0), &sm.kfull[kb]);
             }
           }
           ++kcnt;

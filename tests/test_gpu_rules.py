@@ -144,3 +144,52 @@ def test_prune_rule_small_workloads(name, rule):
         n1 = gpu["n1_vis"]
         assert gpu["count_vis"].tolist() == np.minimum(budget, n1).tolist()
     print(name, rule, rep)
+
+
+# ----------------------------------------------------------------------------- grouped-query Stage II
+
+GQA_CASES = [
+    ("gqa_ragged", dict(B=3, segs=2, P=(5, 37, 130), R=2, M=(1, 7, 70), seed=31, H2kv=8), 0.4, 1.1),
+    ("gqa_c8", dict(B=2, segs=1, P=(1000, 1532), R=4, M=(130, 33), seed=32, H2kv=8), 0.0, 1.15),
+    ("gqa_mixed", dict(B=2, segs=1, P=(1700, 200), R=3, M=(70, 90), seed=33, H2kv=4), 0.0, 1.1),
+    ("gqa_one_kv_head", dict(B=2, segs=2, P=(200, 90), R=4, M=(64, 129), seed=34, H2kv=1), 0.3, 1.3),
+]
+
+
+@pytest.mark.parametrize("path", ["auto", "twopass"])
+@pytest.mark.parametrize("name,kw,l1,l2", GQA_CASES, ids=[c[0] for c in GQA_CASES])
+def test_prune_grouped_query_matches_oracle(name, kw, l1, l2, path):
+    b = _tiny(**kw)
+    assert b["K2"].shape[1] == kw["H2kv"] and b["Q_text"].shape[1] == 32
+    gpu = run_prune(b, l1, l2, path=path)
+    assert gpu["status"] == 0
+    rep = check_prune(b, gpu, l1, l2)
+    assert rep["kept"] > 0
+
+
+def test_grouped_query_text_keys_none():
+    b = _tiny(B=2, segs=1, P=(40, 70), R=2, M=(12, 3), seed=35, H2kv=8)
+    gpu = run_prune(b, 0.3, 1.0, text_keys=False)
+    check_prune(b, gpu, 0.3, 1.0, text_keys="none")
+
+
+def test_grouped_query_workload_shape():
+    """LLaVA-NeXT-shaped batch of 8 with 8 key heads (a grouped-query LLM layer)."""
+    from dataclasses import replace
+    w = replace(get_config("llavanext_b8"), H2kv=8)
+    b = make_batch(w)
+    gpu = run_prune(b, w.lambda1, w.lambda2)
+    assert gpu["status"] == 0
+    check_prune(b, gpu, w.lambda1, w.lambda2)
+
+
+def test_kv_heads_must_divide_query_heads():
+    import paper_2605_29657_gb300 as occ
+
+    b = _tiny(B=1, segs=1, P=(20,), R=2, M=(4,), seed=36)
+    g = {k: v.cuda() for k, v in b.items() if isinstance(v, torch.Tensor) and v.dtype == torch.bfloat16}
+    layout = occ.BatchLayout.from_batch(b, "cuda")
+    keep1 = torch.ones(b["meta"]["total_rows"], dtype=torch.uint8, device="cuda")
+    bad = g["K2"][:, :12].contiguous()                       # 12 key heads for 32 query heads
+    with pytest.raises(occ.OccamError):
+        occ.occam_score_stage2(layout, g["Q_text"], bad, keep1, K_text=g["K_text"][:, :12].contiguous())
