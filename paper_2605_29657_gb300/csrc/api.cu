@@ -212,9 +212,16 @@ bool encode_map3(CUtensorMap* m, const void* base, int64_t rows, int heads, int 
 // Stage-II path selection: the fused tensor-core kernel for every sample that
 // fits it (default), or the two-pass kernels for all samples when
 // OCCAM_STAGE2_PATH=twopass (used to test both paths on the same inputs).
+// OCCAM_STAGE2_PATH: unset or "auto" (default routing), "twopass" (every
+// sample on the two-pass kernels) or "narrow" (no widening of clusters for
+// small batches); the last two exist so that tests reach every path.
 bool fused_enabled() {
   const char* e = std::getenv("OCCAM_STAGE2_PATH");
   return !(e && std::strcmp(e, "twopass") == 0);
+}
+bool widening_enabled() {
+  const char* e = std::getenv("OCCAM_STAGE2_PATH");
+  return !(e && std::strcmp(e, "narrow") == 0);
 }
 
 int cuda_ok() {
@@ -451,6 +458,8 @@ Stage2Params stage2_params(const occam_batch* b, const occam_stage2_args* a, con
   p.slot_off = at<int32_t>(ws, L.slot_off);
   p.maxF = L.maxF;
   p.use_fused = fused ? 1 : 0;
+  p.res16 = widening_enabled() ? fused_resident_clusters(16) : 0;
+  p.res8 = widening_enabled() ? fused_resident_clusters(8) : 0;
   return p;
 }
 

@@ -108,6 +108,7 @@ struct Stage2Params {
   int4* itemsF8;            // fused items for 8-CTA clusters
   int4* itemsF16;           // fused items for 16-CTA clusters
   int use_fused;            // route eligible samples to the fused tensor-core kernel
+  int res16, res8;          // resident 16- and 8-CTA fused clusters (0: no widening for small batches)
   int32_t* slot_off;        // [B+1] partial-slot range of each sample
   int64_t maxF;
   float* ref2;              // [B]
@@ -289,6 +290,7 @@ int s2_scores_smem_bytes();
 int s2_stats_smem_bytes();
 
 // stage2_tc.cu
+int fused_resident_clusters(int C);
 int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt, const Stage2TcParams& q,
                  int nclusters, cudaStream_t st);
 int s2_fused_smem_bytes(int C);

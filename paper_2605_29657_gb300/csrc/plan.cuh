@@ -18,6 +18,18 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
   const int tid = threadIdx.x;
   const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
   int runA = 0, runB = 0, runF = 0, runF8 = 0, runF16 = 0, runS = 0;
+  // A small batch leaves most SMs idle with 4-CTA clusters: when every text
+  // tile of the batch can run at once as a resident 16- (or 8-) CTA cluster,
+  // samples take the wider cluster, whose CTAs hold fewer keys and finish
+  // each head sooner.
+  int wide = 0;
+  if (p.use_fused) {
+    int tiles = 0;
+    for (int b = tid; b < p.bt.B; b += blockDim.x) tiles += (int)((p.bt.text_off[b + 1] - p.bt.text_off[b] + 127) / 128);
+    int total_tiles;
+    block_exclusive_scan(tiles, tmp, &total_tiles);
+    wide = total_tiles <= p.res16 ? 16 : total_tiles <= p.res8 ? 8 : 0;
+  }
   for (int b0 = 0; b0 < p.bt.B; b0 += blockDim.x) {
     const int bb = b0 + tid;
     int nA = 0, nB = 0, nF = 0, nF8 = 0, nF16 = 0;
@@ -26,9 +38,11 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
       const int n1 = *((volatile int32_t*)&p.n1[bb]);
       // the fused tensor-core kernel takes a sample when its S1 keys and its
       // causal text keys fit the cluster's TMEM / shared memory
-      const bool fused4 = p.use_fused && fused_fits(kFusedCluster, n1, M, p.H);
-      const bool fused8 = !fused4 && p.use_fused && fused_fits(8, n1, M, p.H);
-      const bool fused16 = !fused4 && !fused8 && p.use_fused && fused_fits(16, n1, M, p.H);
+      const bool w16 = wide == 16 && fused_fits(16, n1, M, p.H);
+      const bool w8 = !w16 && wide >= 8 && fused_fits(8, n1, M, p.H);
+      const bool fused4 = !w16 && !w8 && p.use_fused && fused_fits(kFusedCluster, n1, M, p.H);
+      const bool fused8 = w8 || (!w16 && !fused4 && p.use_fused && fused_fits(8, n1, M, p.H));
+      const bool fused16 = w16 || (!fused4 && !fused8 && p.use_fused && fused_fits(16, n1, M, p.H));
       if (fused4) {
         nF = (M + 127) / 128;
       } else if (fused8) {

@@ -39,6 +39,8 @@
 // their 32 rows: column max -> s2 (atomicMax on the fp32 bit pattern, exact
 // and order-free since P >= 0), register columns -> a partial of s2(r)
 // reduced in fixed order.
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc5.cuh"
@@ -760,6 +762,40 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   }
   // peers may still write into this CTA's exchange buffers until here
   tc::cluster_sync_all();
+}
+
+// How many C-CTA clusters of the fused kernel the current device holds at
+// once (a cluster must fit in one GPC, so this is below SMs / C), from the
+// occupancy API; looked up once per device and cluster size.
+int fused_resident_clusters(int C) {
+  static std::mutex mu;
+  static int cache[64][3] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  const int ci = C == 16 ? 2 : C == 8 ? 1 : 0;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache[dev][ci] != 0) return cache[dev][ci] > 0 ? cache[dev][ci] : 0;
+  auto kern = C == 16 ? s2_fused_kernel<16> : C == 8 ? s2_fused_kernel<8> : s2_fused_kernel<4>;
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_fused_smem_bytes(C));
+  if (C == 16) cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)C);
+  cfg.blockDim = dim3(s2f::THREADS);
+  cfg.dynamicSmemBytes = s2_fused_smem_bytes(C);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  cache[dev][ci] = n > 0 ? n : -1;
+  return n > 0 ? n : 0;
 }
 
 int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt, const Stage2TcParams& q,

@@ -31,7 +31,8 @@ def to_device(batch: dict, dev) -> dict:
 def run_prune(batch: dict, lam1: float, lam2: float, keep_registers: bool = True, dev="cuda",
               capacity_rows=None, gather=True, text_keys: bool = True, g=None, path: str = "auto",
               host_inputs: bool = False, rule: str = "register", budget=None):
-    """path: "auto" (fused tensor-core Stage II where it fits) or "twopass".
+    """path: "auto" (fused tensor-core Stage II where it fits, wider clusters
+    for small batches), "narrow" (the same without the widening) or "twopass".
     host_inputs: K2, hidden and V stay in pinned host memory (occam_prune_staged).
     rule / budget: the selection rule ("register", "mean", "budget") and the
     per-sample budget array (host ints) of the "budget" rule."""

@@ -50,7 +50,7 @@ CASES = [
 ]
 
 
-@pytest.mark.parametrize("path", ["auto", "twopass"])
+@pytest.mark.parametrize("path", ["auto", "narrow", "twopass"])
 @pytest.mark.parametrize("name,kw,l1,l2", CASES, ids=[c[0] for c in CASES])
 def test_prune_cls_matches_oracle(name, kw, l1, l2, path):
     b = _tiny(**kw)

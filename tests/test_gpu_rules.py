@@ -156,7 +156,7 @@ GQA_CASES = [
 ]
 
 
-@pytest.mark.parametrize("path", ["auto", "twopass"])
+@pytest.mark.parametrize("path", ["auto", "narrow", "twopass"])
 @pytest.mark.parametrize("name,kw,l1,l2", GQA_CASES, ids=[c[0] for c in GQA_CASES])
 def test_prune_grouped_query_matches_oracle(name, kw, l1, l2, path):
     b = _tiny(**kw)
