@@ -221,10 +221,10 @@ def oracle_throughput(n_workers: int, samples_per_worker: int, seed0: int, pool=
     n = sum(k for _, k in res)
     del mp
     return {"value": n / wall, "unit": UNIT, "cores": n_workers, "kind": "oracle",
-            "sample": f"{n} samples of the {WORKLOAD} workload (each: 5 crops x 580 rows, text 16..256), "
+            "sample": f"{n} samples of the {WORKLOAD} workload (batch of one each), "
                       f"{samples_per_worker} per worker on {n_workers} single-threaded workers; "
                       f"value = samples / slowest worker's oracle time",
-            "seconds": wall}
+            "seconds": wall, "cpu_seconds": sum(t for t, _ in res)}
 
 
 def _make_pool(n):
@@ -277,8 +277,36 @@ def run_ours(args, rank, world, local):
     kept_total = int(out["out_off"][-1].item())
     bytes_ = algorithmic_bytes(meta, n1_total, kept_total)
 
-    # traced steps: a spread of the timed steps record per-kernel events
-    n_traced = min(args.steps, 400)
+    # one prune call captured as a CUDA graph: the timed steps replay it (one
+    # replay = one whole occam_prune call, every kernel), which removes the
+    # host's per-call launch work; its outputs must equal the eager call's
+    graph = None
+    if not args.no_graph:
+        want = {k: v.clone() for k, v in call.out.items()}
+        cap_stream = torch.cuda.Stream(device=dev)
+        cap_stream.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(cap_stream):
+            call(cap_stream)
+        torch.cuda.current_stream().wait_stream(cap_stream)
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            call()
+        graph.replay()
+        torch.cuda.synchronize()
+        for k, v in want.items():
+            if k == "out_index":
+                same = torch.equal(v[:kept_total], call.out[k][:kept_total])
+            else:
+                same = torch.equal(v, call.out[k])
+            if not same:
+                raise RuntimeError(f"graph replay differs from the eager call in {k}")
+        step = graph.replay
+    else:
+        step = call
+
+    # traced steps: a spread of the timed steps record per-kernel events (eager calls)
+    n_traced = max(1, min(args.steps // 5 if graph is not None else args.steps, 400))
     traced_at = set(np.linspace(0, args.steps - 1, n_traced).astype(int).tolist())
     events = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(n_traced)]
     for evs in events:
@@ -301,7 +329,7 @@ def run_ours(args, rank, world, local):
             call.traced(events[ti])
             ti += 1
         else:
-            call()
+            step()
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -476,7 +504,7 @@ def run_ours(args, rank, world, local):
     step_gbs = bytes_["step"] / (step_ms / 1e3) / 1e9
     cpu = None
     if pool is not None:
-        cpu = oracle_throughput(n_workers, 4, 0, pool=pool)
+        cpu = oracle_throughput(n_workers, 12, 0, pool=pool)
         pool.close()
         pool.join()
     line = {
@@ -492,6 +520,9 @@ def run_ours(args, rank, world, local):
             "lambda1": w.lambda1, "lambda2": w.lambda2, "accumulate": "fp32",
             "parallelism": "replicas" if world > 1 else "single",
             "l2": "inputs larger than L2 (about 5 GB resident per step); no flush",
+            "launch": ("CUDA graph of one occam_prune call, replayed per step; "
+                       f"{n_traced} of the steps are eager calls recording per-kernel events")
+                      if graph is not None else f"eager occam_prune calls ({n_traced} recording per-kernel events)",
             "mean_n1_vis": float(out["n1_vis"].float().mean().item()),
             "mean_count_vis": float(out["count_vis"].float().mean().item()),
             "kept_rows_per_step": kept_total,
@@ -555,6 +586,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-graph", action="store_true", help="time eager calls instead of a captured CUDA graph")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next", action="store_true", help="skip timing the rows beyond the pruning path")
     ap.add_argument("--workload", default=WORKLOAD,
