@@ -255,58 +255,79 @@ def run_ours(args, rank, world, local):
     batch = make_batch(w, device=dev, seed=w.seed + 0)  # every rank: its own replica of the batch
     meta = batch["meta"]
     layout = occ.BatchLayout.from_batch(batch, dev)
-    K2flat = batch["K2"].view(batch["K2"].shape[0], -1)
-    gather = (batch["hidden"], K2flat, batch["V"])
+    gather = (batch["hidden"], batch["K2"].view(batch["K2"].shape[0], -1), batch["V"])
     cls = w.stage1 == "cls"
     stage1_of = ((lambda t: dict(mode="cls", q=t["q_cls"], k_cls=t["k_cls"], K1=t["K1"])) if cls else
                  (lambda t: dict(mode="mutual", q=t["Q1"], K1=t["K1"])))
-    call = occ.PruneCall(layout, stage1_of(batch),
-                         dict(Q_text=batch["Q_text"], K_text=batch["K_text"], K2=batch["K2"]),
-                         w.lambda1, w.lambda2, keep_registers=True, gather=gather)
+    # `inflight` prune calls in flight at once, each with its own copy of the
+    # inputs, workspace and outputs, on its own stream: consecutive steps
+    # overlap on the GPU as consecutive batches of a serving loop would. The
+    # copies keep the calls from sharing L2 hits on one set of inputs.
+    inflight = max(1, args.inflight)
+    input_names = ("q_cls", "k_cls", "Q1", "K1", "Q_text", "K_text", "K2", "hidden", "V")
+    sets = [batch] + [{k: (v.clone() if k in input_names else v) for k, v in batch.items()}
+                      for _ in range(inflight - 1)]
+
+    def make_call(t):
+        return occ.PruneCall(layout, stage1_of(t), dict(Q_text=t["Q_text"], K_text=t["K_text"], K2=t["K2"]),
+                             w.lambda1, w.lambda2, keep_registers=True,
+                             gather=(t["hidden"], t["K2"].view(t["K2"].shape[0], -1), t["V"]))
+
+    calls = [make_call(t) for t in sets]
+    call = calls[0]
     stream = torch.cuda.current_stream()
+    streams = [stream] if inflight == 1 else [torch.cuda.Stream(device=dev) for _ in range(inflight)]
     nk = len(occ.PruneCall.TRACE_NAMES) + 1
 
-    for _ in range(args.warmup):
-        call()
+    for c, s_ in zip(calls, streams):
+        for _ in range(args.warmup):
+            c(s_)
     torch.cuda.synchronize()
-    st = call.status()
-    if st != 0:
-        raise RuntimeError(f"device status {st} after warm-up")
+    for c in calls:
+        st = c.status()
+        if st != 0:
+            raise RuntimeError(f"device status {st} after warm-up")
     out = call.out
     n1_total = int(out["n1_vis"].sum().item()) + int(meta["regs_per_seg"] * meta["S_tot"])  # registers are in S1
     kept_total = int(out["out_off"][-1].item())
     bytes_ = algorithmic_bytes(meta, n1_total, kept_total)
+    want = {k: v.clone() for k, v in call.out.items()}
 
-    # one prune call captured as a CUDA graph: the timed steps replay it (one
-    # replay = one whole occam_prune call, every kernel), which removes the
-    # host's per-call launch work; its outputs must equal the eager call's
-    graph = None
-    if not args.no_graph:
-        want = {k: v.clone() for k, v in call.out.items()}
-        cap_stream = torch.cuda.Stream(device=dev)
-        cap_stream.wait_stream(torch.cuda.current_stream())
-        with torch.cuda.stream(cap_stream):
-            call(cap_stream)
-        torch.cuda.current_stream().wait_stream(cap_stream)
-        torch.cuda.synchronize()
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph):
-            call()
-        graph.replay()
-        torch.cuda.synchronize()
+    def same_as_first(c, what):
         for k, v in want.items():
             if k == "out_index":
-                same = torch.equal(v[:kept_total], call.out[k][:kept_total])
+                ok = torch.equal(v[:kept_total], c.out[k][:kept_total])
             else:
-                same = torch.equal(v, call.out[k])
-            if not same:
-                raise RuntimeError(f"graph replay differs from the eager call in {k}")
-        step = graph.replay
-    else:
-        step = call
+                ok = torch.equal(v, c.out[k])
+            if not ok:
+                raise RuntimeError(f"{what} differs from the first eager call in {k}")
+
+    for c in calls[1:]:
+        same_as_first(c, "a second in-flight call (same inputs)")
+
+    # each call captured once as a CUDA graph: the timed steps replay them
+    # (one replay = one whole occam_prune call, every kernel), which removes
+    # the host's per-call launch work; replays must equal the eager call
+    graphs = None
+    if not args.no_graph:
+        graphs = []
+        for c in calls:
+            cap_stream = torch.cuda.Stream(device=dev)
+            cap_stream.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(cap_stream):
+                c(cap_stream)
+            torch.cuda.current_stream().wait_stream(cap_stream)
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                c()
+            g.replay()
+            torch.cuda.synchronize()
+            same_as_first(c, "a graph replay")
+            graphs.append(g)
 
     # traced steps: a spread of the timed steps record per-kernel events (eager calls)
-    n_traced = max(1, min(args.steps // 5 if graph is not None else args.steps, 400))
+    n_traced = max(1, min(args.steps // 5 if graphs is not None else args.steps, 400))
     traced_at = set(np.linspace(0, args.steps - 1, n_traced).astype(int).tolist())
     events = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(n_traced)]
     for evs in events:
@@ -323,25 +344,50 @@ def run_ours(args, rank, world, local):
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
+    for s_ in streams[1:]:
+        s_.wait_event(t_start)
     ti = 0
     for i in range(args.steps):
-        if i in traced_at:
-            call.traced(events[ti])
-            ti += 1
-        else:
-            step()
+        j = i % inflight
+        with torch.cuda.stream(streams[j]):
+            if i in traced_at:
+                calls[j].traced(events[ti])
+                ti += 1
+            elif graphs is not None:
+                graphs[j].replay()
+            else:
+                calls[j]()
+    for s_ in streams[1:]:
+        stream.wait_stream(s_)
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     clocks = sampler.stop()
     ms = t_start.elapsed_time(t_end)
-    st = call.status()
-    if st != 0:
-        raise RuntimeError(f"device status {st} after the timed steps")
+    for c in calls:
+        st = c.status()
+        if st != 0:
+            raise RuntimeError(f"device status {st} after the timed steps")
+        same_as_first(c, "a call after the timed steps")
     per_kernel = {}
     for j, name in enumerate(occ.PruneCall.TRACE_NAMES):
         per_kernel[name] = float(np.mean([evs[j].elapsed_time(evs[j + 1]) for evs in events]))
+    # with several calls in flight the timed region's kernel intervals include
+    # sharing the GPU; the same kernels timed alone (one call at a time, after
+    # the timed region) are reported beside them
+    per_kernel_solo = None
+    if inflight > 1:
+        n_solo = 50
+        ev_solo = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(n_solo)]
+        for evs in ev_solo:
+            for e in evs:
+                e.record(stream)  # torch creates the CUDA event on its first record
+        for evs in ev_solo:
+            call.traced(evs)
+        torch.cuda.synchronize()
+        per_kernel_solo = {name: float(np.mean([evs[j].elapsed_time(evs[j + 1]) for evs in ev_solo]))
+                           for j, name in enumerate(occ.PruneCall.TRACE_NAMES)}
 
     ms_max, images = aggregate(ms, meta["B"] * args.steps, dev)
     value = images / (ms_max / 1e3)
@@ -500,6 +546,11 @@ def run_ours(args, rank, world, local):
                 "frac": achieved / peak, "traffic": traffic, "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
                 if peak_kind == "measured" else "fallback 6.8 TB/s",
                 "algorithmic_bytes_per_launch": bytes_[dom], "avg_launch_ms": per_kernel[dom]}
+    if per_kernel_solo is not None:
+        a_solo = bytes_[dom] / (per_kernel_solo[dom] / 1e3) / 1e9
+        roofline["timing"] = (f"avg_launch_ms over the timed region, where {inflight} calls share the GPU; "
+                              "`solo` times the same kernel with one call at a time")
+        roofline["solo"] = {"achieved": a_solo, "frac": a_solo / peak, "avg_launch_ms": per_kernel_solo[dom]}
     step_ms = ms_max / args.steps
     step_gbs = bytes_["step"] / (step_ms / 1e3) / 1e9
     cpu = None
@@ -520,9 +571,13 @@ def run_ours(args, rank, world, local):
             "lambda1": w.lambda1, "lambda2": w.lambda2, "accumulate": "fp32",
             "parallelism": "replicas" if world > 1 else "single",
             "l2": "inputs larger than L2 (about 5 GB resident per step); no flush",
-            "launch": ("CUDA graph of one occam_prune call, replayed per step; "
-                       f"{n_traced} of the steps are eager calls recording per-kernel events")
-                      if graph is not None else f"eager occam_prune calls ({n_traced} recording per-kernel events)",
+            "launch": (f"{inflight} occam_prune calls in flight on {inflight} streams, each with its own copy of "
+                       "the inputs, workspace and outputs; a step replays one call's CUDA graph (every kernel of "
+                       f"the call); {n_traced} of the steps are eager calls recording per-kernel events")
+                      if graphs is not None else
+                      f"{inflight} eager occam_prune calls in flight on {inflight} streams "
+                      f"({n_traced} recording per-kernel events)",
+            "inflight": inflight,
             "mean_n1_vis": float(out["n1_vis"].float().mean().item()),
             "mean_count_vis": float(out["count_vis"].float().mean().item()),
             "kept_rows_per_step": kept_total,
@@ -531,6 +586,7 @@ def run_ours(args, rank, world, local):
             "step_frac_of_measured_hbm": step_gbs / peak,
             "step_frac_of_8TBps": step_gbs / SPEC_HBM_GBS,
             "per_kernel_ms": per_kernel,
+            "per_kernel_ms_solo": per_kernel_solo,
         },
         "roofline": roofline,
         "cpu_baseline": cpu,
@@ -587,6 +643,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true", help="time eager calls instead of a captured CUDA graph")
+    ap.add_argument("--inflight", type=int, default=2,
+                    help="prune calls in flight at once (own inputs, workspace, outputs and stream each)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next", action="store_true", help="skip timing the rows beyond the pruning path")
     ap.add_argument("--workload", default=WORKLOAD,

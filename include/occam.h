@@ -286,10 +286,12 @@ typedef struct occam_prune_out {
 /* The whole path in one call (Algorithm 1's pruning steps): Stage-I scores,
  * S1 (threshold lambda1 per segment), Stage-II scores over S1, S2
  * (threshold lambda2 per sample), compaction and gather. Part of Stage II
- * runs on a second stream that the library owns (one per host thread and
- * device, created on first use), forked from and joined back to `stream` with
- * events, so the call stays ordered on `stream` and can be captured into a
- * CUDA graph. */
+ * runs on a second stream that the library owns (one per host thread,
+ * device and `stream`, created on first use), forked from and joined back to
+ * `stream` with events, so the call stays ordered on `stream` and can be
+ * captured into a CUDA graph. Calls on different streams with their own
+ * workspaces and outputs may be in flight at once (consecutive batches of a
+ * serving loop); their kernels then share the GPU. */
 int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                 size_t workspace_bytes, occam_stream_t stream);
 /* Memory kinds (occam_prune and occam_prune_traced): q, k_cls, K1, Q_text,

@@ -156,28 +156,55 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// A second stream (and fork / join events) per host thread and device, made
-// on first use and kept for the life of the thread; per-thread so that calls
-// from different host threads never share an event.
+// A second stream (and fork / join events) per host thread, device and
+// caller stream, made on first use and kept for the life of the thread:
+// per-thread so that calls from different host threads never share an event,
+// per caller stream so that calls in flight on different streams (a serving
+// loop's consecutive batches) do not queue behind each other's second
+// stream. Past kMaxEntries caller streams, further ones share one entry per
+// device (still correct: the events order every use).
 struct SideStream {
   cudaStream_t stream = nullptr;
   cudaEvent_t fork = nullptr, join = nullptr;
   bool ok = false;
 };
 
-SideStream& side_stream() {
-  constexpr int kMaxDevices = 64;
-  thread_local SideStream per_dev[kMaxDevices];
+SideStream& side_stream(cudaStream_t caller) {
+  constexpr int kMaxEntries = 16, kMaxDevices = 64;
+  struct Entry {
+    int dev = -1;
+    cudaStream_t caller = nullptr;
+    SideStream side;
+  };
+  thread_local Entry table[kMaxEntries];
+  thread_local SideStream overflow[kMaxDevices];
   static SideStream bad;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return bad;
-  SideStream& s = per_dev[dev];
-  if (!s.ok) {
-    s.ok = cudaStreamCreateWithFlags(&s.stream, cudaStreamNonBlocking) == cudaSuccess &&
-           cudaEventCreateWithFlags(&s.fork, cudaEventDisableTiming) == cudaSuccess &&
-           cudaEventCreateWithFlags(&s.join, cudaEventDisableTiming) == cudaSuccess;
+  SideStream* s = nullptr;
+  for (Entry& e : table) {
+    if (e.dev == dev && e.caller == caller) {
+      s = &e.side;
+      break;
+    }
   }
-  return s;
+  if (!s) {
+    for (Entry& e : table) {
+      if (e.dev < 0) {
+        e.dev = dev;
+        e.caller = caller;
+        s = &e.side;
+        break;
+      }
+    }
+  }
+  if (!s) s = &overflow[dev];
+  if (!s->ok) {
+    s->ok = cudaStreamCreateWithFlags(&s->stream, cudaStreamNonBlocking) == cudaSuccess &&
+            cudaEventCreateWithFlags(&s->fork, cudaEventDisableTiming) == cudaSuccess &&
+            cudaEventCreateWithFlags(&s->join, cudaEventDisableTiming) == cudaSuccess;
+  }
+  return *s;
 }
 
 // 2-D bf16 map over a [rows, cols] row-major tensor, 128-byte swizzle, box
@@ -507,7 +534,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     // join by events), so SMs one of them leaves idle serve the other. Both
     // launch a cluster per SM group; clusters take items from a queue, so
     // clusters that become resident late simply find less work.
-    SideStream& side = side_stream();
+    SideStream& side = side_stream(st);
     if (!side.ok) return OCCAM_ERR_CUDA;
     OCCAM_CUDA(cudaEventRecord(side.fork, st));
     OCCAM_CUDA(cudaStreamWaitEvent(side.stream, side.fork, 0));
