@@ -20,9 +20,10 @@
 // 128-byte swizzle, plus {16 dims, 1 head, 128 rows} with the 32-byte swizzle
 // for dims 64-79; dims past d1 (72 -> 80) come zero-filled by the box, so the
 // padded K-step adds nothing.
-// Roles (384 threads): warp 0 issues the TMA loads, warp 1 the MMAs, warps
-// 4-11 (two per TMEM lane quadrant, each taking 128 of the 256 columns) the
-// softmax arithmetic. A tiles, B blocks and the TMEM accumulator are double
+// Roles (640 threads): warp 0 issues the TMA loads, warp 1 the MMAs, warps
+// 4-19 (four per TMEM lane quadrant, each taking 64 of the 256 columns) the
+// softmax arithmetic; four warps per SM sub-partition keep the exponential
+// unit fed through the load -> max -> exp2 latency chains. A tiles, B blocks and the TMEM accumulator are double
 // buffered. Every wait is bounded; on a timeout the CTA records
 // OCCAM_ERR_TIMEOUT, lets its copies land, frees TMEM and returns.
 #include "common.cuh"
@@ -38,23 +39,30 @@ constexpr int ABYTES = AR * 128;          // K-block 0 (dims 0-63) of an A tile
 constexpr int BBYTES = BR * 128;          // K-block 0 of a B block
 constexpr int ABYTES1 = AR * 32;          // K-block 1 (dims 64-79, 32-byte rows) of an A tile
 constexpr int BBYTES1 = BR * 32;
-constexpr int THREADS = 384;
-constexpr int EPI0 = 4;                   // first epilogue warp
+constexpr int NEPI = 16;                  // softmax warps: NEPI / 4 per TMEM lane quadrant
+constexpr int QW = NEPI / 4;              // softmax warps per quadrant
+constexpr int COLS = BR / QW;             // accumulator columns per softmax warp (64)
+constexpr int EPI0 = 4;                   // first softmax warp
+constexpr int THREADS = (EPI0 + NEPI) * 32;
+constexpr int NBB = 4;                    // B blocks in flight (a ring; A tiles and accumulators: 2 each)
+static_assert(COLS == 64, "one 64-column TMEM load per softmax warp and block");
 constexpr uint64_t kLimitNs = 2000000000ull;
 
 struct Smem {
   uint8_t a[2][ABYTES];     // K-block 0 per buffer
-  uint8_t b[2][BBYTES];
+  uint8_t b[NBB][BBYTES];
   uint8_t a1[2][ABYTES1];   // K-block 1 per buffer
-  uint8_t b1[2][BBYTES1];
-  float lsm[8][128];        // pass 2: minus the log-sums of each epilogue warp's 128 columns
-  float2 part[2][4][32];    // second-half partials per (item parity, quadrant, lane)
+  uint8_t b1[NBB][BBYTES1];
+  float lsm[NEPI][COLS];    // pass 2: minus the log-sums of each softmax warp's columns
+  float2 part[2][QW - 1][4][32];  // partials of quarters 1.. per (item parity, quarter, quadrant, lane)
   int32_t item[8];          // the ii-th work item, by ii & 7 (-1: no more)
-  uint64_t afull[2], aempty[2], bfull[2], bempty[2], dfull[2], dfree[2], hb[2][4], inext[8], mdone;
+  uint64_t afull[2], aempty[2], bfull[NBB], bempty[NBB], dfull[2], dfree[2], hb[2][4], inext[8], mdone;
   uint32_t tmem_base;
   int abort;
 };
 }  // namespace m1
+
+static_assert(sizeof(m1::Smem) + 1024 <= 227 * 1024, "shared memory per CTA");
 
 int mutual_tc_smem_bytes() { return (int)sizeof(m1::Smem) + 1024; }
 
@@ -122,12 +130,15 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
     for (int i = 0; i < 2; ++i) {
       tc::bar_init(&sm.afull[i], 1);
       tc::bar_init(&sm.aempty[i], 1);
+
+      tc::bar_init(&sm.dfull[i], 1);
+      tc::bar_init(&sm.dfree[i], NEPI);
+    }
+    for (int i = 0; i < NBB; ++i) {
       tc::bar_init(&sm.bfull[i], 1);
       tc::bar_init(&sm.bempty[i], 1);
-      tc::bar_init(&sm.dfull[i], 1);
-      tc::bar_init(&sm.dfree[i], 8);
     }
-    for (int i = 0; i < 8; ++i) tc::bar_init(&sm.hb[i >> 2][i & 3], 1);
+    for (int i = 0; i < 8; ++i) tc::bar_init(&sm.hb[i >> 2][i & 3], QW - 1);
     for (int i = 0; i < 8; ++i) tc::bar_init(&sm.inext[i], 1);
     tc::bar_init(&sm.mdone, 1);
     sm.abort = 0;
@@ -174,8 +185,8 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
             if (nkb > 1) tma_load_3d(sm.a1[ab], &mapA1, 64, h, (int)(sb + w.a0), &sm.afull[ab]);
             ++na;
           }
-          const int bb = nbk & 1;
-          if (!tc::bar_wait(&sm.bempty[bb], ((nbk >> 1) & 1) ^ 1, abort, kLimitNs)) {
+          const int bb = nbk % NBB;
+          if (!tc::bar_wait(&sm.bempty[bb], ((nbk / NBB) & 1) ^ 1, abort, kLimitNs)) {
             ok = false;
             break;
           }
@@ -218,9 +229,9 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         bool ok = true;
         for (int s = 0; s < nheads * nb; ++s, ++sg) {
           const int jb = s % nb;
-          const int ab = na & 1, bb = sg & 1, db = sg & 1;
+          const int ab = na & 1, bb = sg % NBB, db = sg & 1;
           if (jb == 0) ok = tc::bar_wait(&sm.afull[ab], (na >> 1) & 1, abort, kLimitNs);
-          if (ok) ok = tc::bar_wait(&sm.bfull[bb], (sg >> 1) & 1, abort, kLimitNs);
+          if (ok) ok = tc::bar_wait(&sm.bfull[bb], (sg / NBB) & 1, abort, kLimitNs);
           if (ok && sg >= 2) ok = tc::bar_wait(&sm.dfree[db], ((sg - 2) >> 1) & 1, abort, kLimitNs);
           if (!ok) break;
           tc::fence_after();
@@ -252,7 +263,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
   } else if (warp >= EPI0) {
     // ------------------------------------------------------------ softmax warps
     const int ew = warp - EPI0;
-    const int quad = warp & 3, half = ew >> 2;
+    const int quad = warp & 3, qtr = ew >> 2;           // TMEM lane quadrant; which 64 of the 256 columns
     const int row = quad * 32 + lane;                   // tile row = TMEM lane
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     const float c = p.scale_log2;
@@ -276,31 +287,31 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       const int pp = ii & 1;
       float m = -INFINITY, z = 0.f;  // pass 1: running max / sum (log2 domain)
       float acc = 0.f;               // pass 2: attention received by this key row
-      float lnext[4];                // pass 2: the next step's minus log-sums of 4 columns
+      float lnext[2];                // pass 2: the next step's minus log-sums of 2 columns
       bool ok = true;
       for (int s = 0; s < steps; ++s, ++sg) {
         const int h = w.h + s / nb;
         const int jb = s % nb;
-        const int col0 = jb * BR + half * 128;          // segment-relative index of this warp's column 0
+        const int col0 = jb * BR + qtr * COLS;          // segment-relative index of this warp's column 0
         if (PASS == 2) {
-          // minus the log-sums of this warp's 128 query columns (past the
+          // minus the log-sums of this warp's 64 query columns (past the
           // segment: -inf, which contributes 0); those of the item's first
           // step are loaded here, the others one step ahead (below)
           if (s == 0) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const int qq = col0 + lane * 4 + i;
+            for (int i = 0; i < 2; ++i) {
+              const int qq = col0 + lane * 2 + i;
               lnext[i] = qq < n ? -__ldcg(&p.lsum[(int64_t)h * R + sb + qq]) : -INFINITY;
             }
           }
           __syncwarp();
-          *reinterpret_cast<float4*>(&sm.lsm[ew][lane * 4]) = make_float4(lnext[0], lnext[1], lnext[2], lnext[3]);
+          *reinterpret_cast<float2*>(&sm.lsm[ew][lane * 2]) = make_float2(lnext[0], lnext[1]);
           __syncwarp();
           if (s + 1 < steps) {
-            const int h1 = w.h + (s + 1) / nb, c1 = ((s + 1) % nb) * BR + half * 128;
+            const int h1 = w.h + (s + 1) / nb, c1 = ((s + 1) % nb) * BR + qtr * COLS;
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const int qq = c1 + lane * 4 + i;
+            for (int i = 0; i < 2; ++i) {
+              const int qq = c1 + lane * 2 + i;
               lnext[i] = qq < n ? -__ldcg(&p.lsum[(int64_t)h1 * R + sb + qq]) : -INFINITY;
             }
           }
@@ -311,31 +322,30 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
           break;
         }
         tc::fence_after();
-#pragma unroll
-        for (int g = 0; g < 2; ++g) {
+        {
           uint32_t v[64];
-          tc::tmem_ld64(tmem + lane_base + db * BR + half * 128 + g * 64, v);
+          tc::tmem_ld64(tmem + lane_base + db * BR + qtr * COLS, v);
           wait_ld64(v);
           if (PASS == 1) {
             // keys past the segment are masked out of this row's softmax
-            const int lim = n - (col0 + g * 64);
+            const int lim = n - col0;
             if (lim < 64) {
 #pragma unroll
               for (int i = 0; i < 64; ++i) v[i] = i < lim ? v[i] : 0xff800000u;  // -inf
             }
-            // max as a tree of three-input maxima (short dependency chains)
-            float t[22];
+            // max as a tree of three-input maxima (short dependency chains,
+            // few values live beside v)
+            float t[16];
 #pragma unroll
-            for (int i = 0; i < 21; ++i)
-              t[i] = tc::fmax3(__uint_as_float(v[3 * i]), __uint_as_float(v[3 * i + 1]), __uint_as_float(v[3 * i + 2]));
-            t[21] = __uint_as_float(v[63]);
-            float u[8];
+            for (int i = 0; i < 16; ++i)
+              t[i] = fmaxf(tc::fmax3(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]), __uint_as_float(v[4 * i + 2])),
+                           __uint_as_float(v[4 * i + 3]));
+            float u[6];
 #pragma unroll
-            for (int i = 0; i < 7; ++i) u[i] = tc::fmax3(t[3 * i], t[3 * i + 1], t[3 * i + 2]);
-            u[7] = t[21];
+            for (int i = 0; i < 5; ++i) u[i] = tc::fmax3(t[3 * i], t[3 * i + 1], t[3 * i + 2]);
+            u[5] = t[15];
             // c > 0: the max of c l is c times the max of l
-            const float mx =
-                fmaxf(tc::fmax3(u[0], u[1], u[2]), tc::fmax3(u[3], u[4], fmaxf(u[5], fmaxf(u[6], u[7])))) * c;
+            const float mx = fmaxf(tc::fmax3(u[0], u[1], u[2]), tc::fmax3(u[3], u[4], u[5])) * c;
             if (mx != -INFINITY) {
               const float2 cc = make_float2(c, c), om = make_float2(-mx, -mx);
               float2 ap[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
@@ -354,7 +364,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
               m = fmaxf(m, mx);
             }
           } else {
-            const float2* nl = reinterpret_cast<const float2*>(sm.lsm[ew] + g * 64);
+            const float2* nl = reinterpret_cast<const float2*>(sm.lsm[ew]);
             const float2 cc = make_float2(c, c);
             float2 ap[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
@@ -371,32 +381,38 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         tc::fence_before();
         __syncwarp();
         const bool last = s == steps - 1;
-        if (half == 1 && last) {
-          // the second half hands its partial to the first
-          sm.part[pp][quad][lane] = make_float2(PASS == 1 ? m : acc, z);
+        if (qtr > 0 && last) {
+          // quarters 1.. hand their partials to quarter 0
+          sm.part[pp][qtr - 1][quad][lane] = make_float2(PASS == 1 ? m : acc, z);
           __syncwarp();
           if (lane == 0) tc::bar_arrive(&sm.hb[pp][quad]);
         }
-        if (half == 0 && last) {
-          // read the partner's partial before releasing this step's
-          // accumulator: its next write to the slot waits on that release
+        if (qtr == 0 && last) {
+          // read the partners' partials before releasing this step's
+          // accumulator: their next writes to the slots wait on that release
           if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.hb[pp][quad], (ii >> 1) & 1, nullptr, kLimitNs))) {
             ok = false;
             break;
           }
-          const float2 o = sm.part[pp][quad][lane];
           if (PASS == 1) {
-            if (o.x != -INFINITY) {
-              const bool up = o.x > m;
-              const float e = tc::ex2(up ? m - o.x : o.x - m);
-              z = up ? fmaf(z, e, o.y) : fmaf(o.y, e, z);
-              m = fmaxf(m, o.x);
+#pragma unroll
+            for (int q = 0; q < QW - 1; ++q) {
+              const float2 o = sm.part[pp][q][quad][lane];
+              if (o.x != -INFINITY) {
+                const bool up = o.x > m;
+                const float e = tc::ex2(up ? m - o.x : o.x - m);
+                z = up ? fmaf(z, e, o.y) : fmaf(o.y, e, z);
+                m = fmaxf(m, o.x);
+              }
             }
             // L = log2 of the row's sum of exp2(c q k) over the segment's keys
             if (vrow) p.lsum[(int64_t)w.h * R + sb + w.a0 + row] = m + log2f(z);
-          } else if (vrow) {
+          } else {
+            float tot = acc;
+#pragma unroll
+            for (int q = 0; q < QW - 1; ++q) tot += sm.part[pp][q][quad][lane].x;
             // this head group's share of s1 (summed over the groups in order afterwards)
-            p.part[(int64_t)(w.h / kMutHeadGroup) * R + sb + w.a0 + row] = (acc + o.x) * p.inv_h / (float)n;
+            if (vrow) p.part[(int64_t)(w.h / kMutHeadGroup) * R + sb + w.a0 + row] = tot * p.inv_h / (float)n;
           }
           __syncwarp();
         }
