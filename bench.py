@@ -252,6 +252,9 @@ def run_ours(args, rank, world, local):
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
     w = get_config(WORKLOAD)
+    if args.kv_heads:
+        from dataclasses import replace
+        w = replace(w, H2kv=args.kv_heads)   # a grouped-query LLM layer of the same shape
     batch = make_batch(w, device=dev, seed=w.seed + 0)  # every rank: its own replica of the batch
     meta = batch["meta"]
     layout = occ.BatchLayout.from_batch(batch, dev)
@@ -568,6 +571,7 @@ def run_ours(args, rank, world, local):
             "registers_per_crop": meta["regs_per_seg"],
             "text_tokens": (str(w.M[1]) if w.M[0] == "fixed" else f"{w.M[1]}..{w.M[2]} (uniform)"),
             "H1xd1": f"{meta['H1']}x{meta['d1']}", "H2xd2": f"{meta['H2']}x{meta['d2']}", "hidden": meta["hidden"],
+            "kv_heads": meta.get("H2kv", meta["H2"]),
             "lambda1": w.lambda1, "lambda2": w.lambda2, "accumulate": "fp32",
             "parallelism": "replicas" if world > 1 else "single",
             "l2": "inputs larger than L2 (about 5 GB resident per step); no flush",
@@ -643,6 +647,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true", help="time eager calls instead of a captured CUDA graph")
+    ap.add_argument("--kv-heads", type=int, default=0,
+                    help="key / value heads of the LLM layer (grouped-query variant; 0: one per query head)")
     ap.add_argument("--inflight", type=int, default=2,
                     help="prune calls in flight at once (own inputs, workspace, outputs and stream each)")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -400,10 +400,13 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         if (!tc::bar_wait(&sm.iready[ib], (ii >> 1) & 1, abort, kLimitNs)) { fail(sm, p.status); break; }
         const int64_t tbase = g.t0 + g.txt0;
         bool ok = true;
-        for (int h = 0; h < H && ok; ++h) {
+        // grouped-query attention: the group's query heads share one key
+        // block, loaded for the group's first head (the ring advances per key
+        // head); gi = h's index in its group, hkv = the key head it reads
+        for (int h = 0, gi = 0, hkv = 0; h < H && ok; ++h, gi = gi + 1 == p.kv_group ? 0 : gi + 1, hkv += gi == 0) {
           const int kb = kcnt & 1;
-          const int hkv = h / p.kv_group;  // the key / value head query head h reads
-          if (!tc::bar_wait(&sm.kempty[kb], ((kcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
+          const bool load_keys = gi == 0;
+          if (load_keys && !tc::bar_wait(&sm.kempty[kb], ((kcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
             fail(sm, p.status);
             ok = false;
             break;
@@ -427,6 +430,10 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
           // masked; no other padding row is loaded). Every producer thread
           // arrives once per head, announcing the bytes of its own copies
           // before it issues them.
+          if (!load_keys) {
+            if (gi == p.kv_group - 1) ++kcnt;
+            continue;
+          }
           const int gi4 = (g.own_img + 3) >> 2, nbt = (g.own_txt + TXT_BOX - 1) / TXT_BOX;
           const int nu = (gi4 + nbt) * 2;
           uint32_t mine = 0;
@@ -449,7 +456,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
                               (int)(tbase + t0), &sm.kfull[kb]);
             }
           }
-          ++kcnt;
+          if (gi == p.kv_group - 1) ++kcnt;
         }
         if (!ok) break;
       }
@@ -466,12 +473,13 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
           if (!g.fits) continue;
           const uint32_t idesc = tc::idesc_bf16(128, g.N > 0 ? g.N : 16);
           bool ok = true;
-          for (int h = 0; h < H && ok; ++h, ++hk) {
+          for (int h = 0, gi = 0; h < H && ok; ++h, ++hk, gi = gi + 1 == p.kv_group ? 0 : gi + 1) {
             const int qb = qcnt & 1, kb = kcnt & 1, eb = hk & 1;
             // E[eb] is free once head hk - 2 was read out of it
             ok = tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs);
             if (ok && hk >= 2) ok = tc::bar_wait(&sm.efree[eb], ((hk - 2) >> 1) & 1, abort, kLimitNs);
-            if (ok) ok = tc::bar_wait(&sm.kfull[kb], (kcnt >> 1) & 1, abort, kLimitNs);
+            // the key block of a group of query heads lands once, before its first head
+            if (ok && gi == 0) ok = tc::bar_wait(&sm.kfull[kb], (kcnt >> 1) & 1, abort, kLimitNs);
             if (!ok) {
               fail(sm, p.status);
               break;
@@ -488,10 +496,13 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
               }
             }
             tc::mma_commit(&sm.efull[eb]);
-            tc::mma_commit(&sm.kempty[kb]);
             tc::mma_commit(&sm.qempty[qb]);
+            if (gi == p.kv_group - 1) {
+              // the group's last query head frees the key block
+              tc::mma_commit(&sm.kempty[kb]);
+              ++kcnt;
+            }
             ++qcnt;
-            ++kcnt;
           }
         }
         // every MMA issued by this thread has completed once this barrier flips

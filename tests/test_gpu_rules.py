@@ -193,3 +193,66 @@ def test_kv_heads_must_divide_query_heads():
     bad = g["K2"][:, :12].contiguous()                       # 12 key heads for 32 query heads
     with pytest.raises(occ.OccamError):
         occ.occam_score_stage2(layout, g["Q_text"], bad, keep1, K_text=g["K_text"][:, :12].contiguous())
+
+
+# ----------------------------------------------------------------------------- combinations with host inputs
+
+@pytest.mark.parametrize("variant", ["gqa", "budget", "mean"])
+def test_host_inputs_with_variants(variant):
+    """occam_prune_staged (K2, hidden, V in pinned host memory) under grouped-query keys and under both
+    rule variants: bit-identical to the all-device call, and under the parity rule against the oracle."""
+    kw = dict(B=3, segs=2, P=(120, 57, 300), R=3, M=(70, 5, 130), seed=41)
+    if variant == "gqa":
+        kw["H2kv"] = 8
+    b = _tiny(**kw)
+    rule = "register" if variant == "gqa" else variant
+    budget = _budget_for(b, 0.15, 2) if variant == "budget" else None
+    l1, l2 = (0.1, 0.6) if variant == "mean" else (0.2, 1.2)
+    dev = run_prune(b, l1, l2, rule=rule, budget=budget)
+    host = run_prune(b, l1, l2, rule=rule, budget=budget, host_inputs=True)
+    assert host["status"] == 0 and dev["status"] == 0
+    for k in ("s1", "ref1", "s2", "ref2", "keep1", "keep2", "count_vis", "count_out", "out_off", "n1_vis"):
+        assert np.array_equal(host[k], dev[k]), k
+    kept = int(dev["out_off"][-1])
+    assert np.array_equal(host["out_index"][:kept], dev["out_index"][:kept])
+    for a, c in zip(host["gathered"], dev["gathered"]):
+        assert torch.equal(a[:kept], c[:kept])
+    check_prune(b, host, l1, l2, rule=rule, budget=budget)
+
+
+def test_rules_capture_into_a_graph_and_replay_identically():
+    """occam_prune under each rule inside a CUDA graph: a replay reproduces the eager outputs."""
+    import paper_2605_29657_gb300 as occ
+
+    b = _tiny(B=3, segs=2, P=(100, 57, 220), R=3, M=(70, 5, 130), seed=42)
+    g = {k: v.cuda() for k, v in b.items() if isinstance(v, torch.Tensor) and v.dtype == torch.bfloat16}
+    layout = occ.BatchLayout.from_batch(b, "cuda")
+    st1 = dict(mode="cls", q=g["q_cls"], k_cls=g["k_cls"], K1=g["K1"])
+    st2 = dict(Q_text=g["Q_text"], K_text=g["K_text"], K2=g["K2"])
+    budget = torch.tensor(_budget_for(b, 0.1, 3), dtype=torch.int32, device="cuda")
+    for rule in ("register", "mean", "budget"):
+        call = occ.PruneCall(layout, st1, st2, 0.2, 1.2, gather=(g["hidden"],), rule=rule,
+                             budget=budget if rule == "budget" else None)
+        call()
+        torch.cuda.synchronize()
+        want = {k: v.clone() for k, v in call.out.items()}
+        cs = torch.cuda.Stream()
+        cs.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(cs):
+            call(cs)
+        torch.cuda.current_stream().wait_stream(cs)
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            call()
+        for k in call.out:
+            call.out[k].zero_()
+        graph.replay()
+        torch.cuda.synchronize()
+        assert call.status() == 0
+        kept = int(want["out_off"][-1])
+        for k, v in want.items():
+            if k == "out_index":
+                assert torch.equal(v[:kept], call.out[k][:kept]), (rule, k)
+            else:
+                assert torch.equal(v, call.out[k]), (rule, k)
