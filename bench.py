@@ -649,7 +649,7 @@ def main():
     ap.add_argument("--no-graph", action="store_true", help="time eager calls instead of a captured CUDA graph")
     ap.add_argument("--kv-heads", type=int, default=0,
                     help="key / value heads of the LLM layer (grouped-query variant; 0: one per query head)")
-    ap.add_argument("--inflight", type=int, default=2,
+    ap.add_argument("--inflight", type=int, default=3,
                     help="prune calls in flight at once (own inputs, workspace, outputs and stream each)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next", action="store_true", help="skip timing the rows beyond the pruning path")
