@@ -20,6 +20,8 @@ Each function follows one equation of the paper:
 * Stage II set S2 = {v in S1\\{r} : s2(v) >= lambda2 s2(r)} u {r} -- Eq. 8; App. A, Eq. 17
 * lambda2 matching a retained budget over a calibration set      -- App. A, average-budget equation
 * test-time register construction h_r,k = max_v h_v,k, h_v,k = 0 -- Algorithm 1; App. A, register redirection
+* pooling of patch scores onto merged tokens (Qwen3-VL's 2x2 patch merger
+  puts each merged token's four patches on consecutive rows)   -- Sec. 4 setup; reading below
 * rule variants of the component ablation (App., "compact component
   ablation"): a mean-based reference instead of the register's score, and a
   fixed per-sample budget (the top-K rule of Sec. 2) instead of the
@@ -49,6 +51,10 @@ Readings where the paper is silent (each one is also a keyword flag here):
 * the mean threshold takes, per stage, the mean score of that stage's
   candidates (Stage I: the segment's visual rows; Stage II: the sample's
   visual S1 rows) as the reference, in both stages;
+* merged tokens (the paper is silent on how patch scores become merged-token
+  scores): the score of a group of consecutive patch rows is the sum of its
+  patches' scores (the attention mass the merged token receives); the mean
+  and the max are flags;
 * the fixed budget keeps Stage I as in the method and, per sample, the
   budget[b] visual S1 rows with the largest s2 (all of them when there are
   fewer); equal scores keep the lower row first;
@@ -282,6 +288,24 @@ def mean_reference(s, unit_off, cand):
         if c.any():
             ref[u] = np.mean(s[unit_off[u]:unit_off[u + 1]][c])
     return ref
+
+
+def pool_scores(s, group: int, mode: str = "sum"):
+    """Scores of merged tokens from the scores of their patches: rows
+    [group i, group i + group) of ``s`` form merged row i, reduced by "sum"
+    (the attention mass of the group), "mean" or "max". The row count must
+    be a multiple of ``group``.
+    """
+    s = np.asarray(s, dtype=np.float64)
+    assert group >= 1 and s.shape[0] % group == 0
+    g = s.reshape(-1, group)
+    if mode == "sum":
+        return g.sum(axis=1)
+    if mode == "mean":
+        return g.mean(axis=1)
+    if mode == "max":
+        return g.max(axis=1)
+    raise ValueError(mode)
 
 
 def budget_keep(s, row_off, cand, budget, is_reg, keep_registers: bool = True):

@@ -668,3 +668,20 @@ def test_grouped_query_heads_equal_expanded_keys(text_keys):
     wrong["K2"] = b["K2"][:, torch.arange(8) % 2, :].contiguous()
     wrong["K_text"] = b["K_text"][:, torch.arange(8) % 2, :].contiguous()
     assert not np.allclose(O.prune(wrong, 0.6, 1.1, text_keys=text_keys)["s2"], g["s2"])
+
+
+# ----------------------------------------------------------------------------- merged-token pooling (Qwen 2x2 merger)
+
+def test_pool_scores_hand_values_and_mass():
+    s = np.array([0.1, 0.2, 0.3, 0.4, 1.0, 0.0, 0.0, 3.0])
+    assert np.allclose(O.pool_scores(s, 4, "sum"), [1.0, 4.0])
+    assert np.allclose(O.pool_scores(s, 4, "mean"), [0.25, 1.0])
+    assert O.pool_scores(s, 4, "max").tolist() == [0.4, 3.0]
+    assert O.pool_scores(s, 1, "sum").tolist() == s.tolist()
+    # sum pooling keeps the total attention mass of a segment's [CLS] row
+    b = tiny_batch(B=1, segs=1, P=(38,), R=2, M=(2,), seed=5, H1=4, d1=16)
+    s1, _ = O.stage1_cls(b["q_cls"], None, b["K1"], b["meta"]["seg_off_host"], b["meta"]["reg_idx_host"],
+                         b["meta"]["reg_off_host"])
+    assert abs(O.pool_scores(s1, 4, "sum").sum() - 1.0) < 1e-12
+    with pytest.raises(AssertionError):
+        O.pool_scores(np.zeros(6), 4)
