@@ -73,6 +73,8 @@ enum { OCCAM_TEXT_KEYS_CAUSAL = 0, OCCAM_TEXT_KEYS_NONE = 1 };
  * candidates in both stages; BUDGET keeps Stage I and replaces the Stage-II
  * threshold by a fixed per-sample budget (the top-K rule of Sec. 2). */
 enum { OCCAM_RULE_REGISTER = 0, OCCAM_RULE_MEAN = 1, OCCAM_RULE_BUDGET = 2 };
+/* Reductions of occam_pool_scores. */
+enum { OCCAM_POOL_SUM = 0, OCCAM_POOL_MEAN = 1, OCCAM_POOL_MAX = 2 };
 
 #define OCCAM_MAX_GATHER 8
 
@@ -181,6 +183,17 @@ int occam_mean_reference(const occam_batch* batch, const float* s, int32_t ref_s
 int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* prev_keep, const int32_t* budget,
                       int32_t keep_registers, uint8_t* keep, int32_t* count_vis, void* workspace,
                       size_t workspace_bytes, occam_stream_t stream);
+
+/* Merged-token scores from patch scores. A 2x2 patch merger (Qwen3-VL's)
+ * turns every group of `group` consecutive patch rows into one token; the
+ * paper does not say how patch scores become token scores. s_out[i] = the
+ * sum (OCCAM_POOL_SUM, the attention mass the group receives), mean
+ * (OCCAM_POOL_MEAN) or max (OCCAM_POOL_MAX) of s_in[group i .. group i +
+ * group - 1], added in row order. s_in [rows_in], s_out [rows_in / group]
+ * fp32, device; rows_in must be a multiple of group (>= 1), else
+ * OCCAM_ERR_INVALID_ARG. */
+int occam_pool_scores(const float* s_in, int64_t rows_in, int32_t group, int32_t mode, float* s_out,
+                      occam_stream_t stream);
 
 int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, const uint8_t* keep1,
                        float* s2, float* ref2, void* workspace, size_t workspace_bytes,

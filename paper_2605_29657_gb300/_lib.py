@@ -36,6 +36,7 @@ OCCAM_RULE_REGISTER = 0
 OCCAM_RULE_MEAN = 1
 OCCAM_RULE_BUDGET = 2
 RULES = {"register": OCCAM_RULE_REGISTER, "mean": OCCAM_RULE_MEAN, "budget": OCCAM_RULE_BUDGET}
+POOLS = {"sum": 0, "mean": 1, "max": 2}
 
 _p = ctypes.c_void_p
 _i32 = ctypes.c_int32
@@ -112,7 +113,8 @@ def library() -> ctypes.CDLL:
         lib.occam_construct_registers.argtypes = [P(CBatch), _p, _i64, _p, _i32, _p, ctypes.c_size_t, _p]
         lib.occam_mean_reference.argtypes = [P(CBatch), _p, _i32, _p, _p, _p, ctypes.c_size_t, _p]
         lib.occam_budget_keep.argtypes = [P(CBatch), _p, _p, _p, _i32, _p, _p, _p, ctypes.c_size_t, _p]
-        for name in ("occam_mean_reference", "occam_budget_keep", "occam_construct_registers", "occam_calibrate_lambda2", "occam_workspace_size", "occam_get_status", "occam_score_stage1",
+        lib.occam_pool_scores.argtypes = [_p, _i64, _i32, _i32, _p, _p]
+        for name in ("occam_pool_scores", "occam_mean_reference", "occam_budget_keep", "occam_construct_registers", "occam_calibrate_lambda2", "occam_workspace_size", "occam_get_status", "occam_score_stage1",
                      "occam_threshold",
                      "occam_score_stage2", "occam_compact", "occam_prune", "occam_prune_traced",
                      "occam_compact_noalloc", "occam_prune_staged"):
@@ -288,6 +290,20 @@ def occam_mean_reference(layout: BatchLayout, s, ref_scope: int, prev_keep=None,
     _check(library().occam_mean_reference(ctypes.byref(cb), _ptr(s), int(ref_scope), _ptr(prev_keep), _ptr(ref),
                                           _ptr(ws), ws.numel(), _stream(stream)), "occam_mean_reference")
     return ref
+
+
+def occam_pool_scores(s, group: int, mode: str = "sum", out=None, stream=None) -> torch.Tensor:
+    """Merged-token scores: the sum (default), mean or max of every group of
+    `group` consecutive rows of s (a 2x2 patch merger's four patches)."""
+    _dev_tensor(s, torch.float32, "s")
+    if mode not in POOLS:
+        raise OccamError(OCCAM_ERR_INVALID_ARG, f"mode must be one of {sorted(POOLS)}")
+    if group < 1 or s.numel() % group:
+        raise OccamError(OCCAM_ERR_INVALID_ARG, "the row count must be a multiple of group")
+    out = torch.empty(s.numel() // group, dtype=torch.float32, device=s.device) if out is None else out
+    _check(library().occam_pool_scores(_ptr(s), s.numel(), int(group), POOLS[mode], _ptr(out), _stream(stream)),
+           "occam_pool_scores")
+    return out
 
 
 def occam_budget_keep(layout: BatchLayout, s, budget, prev_keep=None, keep_registers: bool = True, keep=None,

@@ -714,6 +714,20 @@ int occam_mean_reference(const occam_batch* batch, const float* s, int32_t ref_s
   return cuda_ok();
 }
 
+int occam_pool_scores(const float* s_in, int64_t rows_in, int32_t group, int32_t mode, float* s_out,
+                      occam_stream_t stream) {
+  if (!s_in || !s_out || group < 1 || rows_in < 0 || rows_in % group != 0) return OCCAM_ERR_INVALID_ARG;
+  if (mode != OCCAM_POOL_SUM && mode != OCCAM_POOL_MEAN && mode != OCCAM_POOL_MAX) return OCCAM_ERR_INVALID_ARG;
+  const int64_t rows_out = rows_in / group;
+  if (rows_out == 0) return OCCAM_OK;
+  OCCAM_TRY(require_device(s_in));
+  OCCAM_TRY(require_device(s_out));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const unsigned blocks = (unsigned)std::min<int64_t>(cdiv(rows_out, 256), (int64_t)num_sms() * 8);
+  pool_scores_kernel<<<blocks, 256, 0, st>>>(s_in, rows_out, group, mode, s_out);
+  return cuda_ok();
+}
+
 int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* prev_keep, const int32_t* budget,
                       int32_t keep_registers, uint8_t* keep, int32_t* count_vis, void* workspace,
                       size_t workspace_bytes, occam_stream_t stream) {

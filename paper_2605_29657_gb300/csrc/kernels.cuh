@@ -305,6 +305,7 @@ __global__ void registers_kernel(RegistersParams p);
 // rules.cu
 __global__ void mean_ref_kernel(MeanRefParams p);
 __global__ void budget_keep_kernel(BudgetParams p);
+__global__ void pool_scores_kernel(const float* s_in, int64_t rows_out, int group, int mode, float* s_out);
 __global__ void gather_kernel(GatherParams p);
 __global__ void offsets_fix_kernel(ScanParams p);
 

@@ -8,7 +8,11 @@
 //                       Sec. 2, S = top-K(V, s): per sample the budget[b]
 //                       candidate rows with the largest score, equal scores
 //                       taken lower row first.
-// Both are deterministic: fixed-order sums, and a selection whose result
+//   pool_scores_kernel  scores of merged tokens from their patches' scores
+//                       (a 2x2 patch merger puts a merged token's patches on
+//                       consecutive rows): the sum, mean or max of each
+//                       group of consecutive rows.
+// All are deterministic: fixed-order sums, and a selection whose result
 // does not depend on thread timing.
 #include "common.cuh"
 #include "kernels.cuh"
@@ -164,6 +168,17 @@ __global__ void __launch_bounds__(1024) budget_keep_kernel(BudgetParams p) {
     p.keep[r] = k ? 1 : 0;
   }
   if (tid == 0 && p.count_vis) p.count_vis[b] = K;
+}
+
+// One thread per merged row; the group's values are added in row order.
+__global__ void __launch_bounds__(256) pool_scores_kernel(const float* __restrict__ s_in, int64_t rows_out, int group,
+                                                          int mode, float* __restrict__ s_out) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < rows_out; i += (int64_t)gridDim.x * blockDim.x) {
+    const float* g = s_in + i * group;
+    float acc = g[0];
+    for (int k = 1; k < group; ++k) acc = mode == OCCAM_POOL_MAX ? fmaxf(acc, g[k]) : acc + g[k];
+    s_out[i] = mode == OCCAM_POOL_MEAN ? acc / (float)group : acc;
+  }
 }
 
 }  // namespace occam

@@ -256,3 +256,41 @@ def test_rules_capture_into_a_graph_and_replay_identically():
                 assert torch.equal(v[:kept], call.out[k][:kept]), (rule, k)
             else:
                 assert torch.equal(v, call.out[k]), (rule, k)
+
+
+# ----------------------------------------------------------------------------- merged-token pooling
+
+@pytest.mark.parametrize("mode", ["sum", "mean", "max"])
+@pytest.mark.parametrize("group", [1, 4, 16])
+def test_pool_scores_matches_oracle(mode, group):
+    import paper_2605_29657_gb300 as occ
+
+    rng = np.random.default_rng(group)
+    s = (rng.random(4 * 16 * 777) * rng.choice([1e-5, 1e-2, 1.0], 4 * 16 * 777)).astype(np.float32)
+    got = occ.occam_pool_scores(torch.from_numpy(s).cuda(), group, mode).cpu().numpy()
+    want = O.pool_scores(s.astype(np.float64), group, mode)
+    if mode == "max":
+        assert np.array_equal(got.astype(np.float64), want)
+    else:
+        # fp32 additions of `group` values in row order
+        np.testing.assert_allclose(got, want, rtol=group * 2 ** -23, atol=0)
+
+
+def test_pool_scores_of_mutual_stage1():
+    """Stage-I mutual scores of patch rows pooled 4 to 1 (a 2x2 merger) match the oracle's pooled scores."""
+    import paper_2605_29657_gb300 as occ
+
+    b = _tiny(B=2, segs=1, P=(60, 124), R=4, M=(3, 3), stage1="mutual", d1=72, seed=43, query_bias=0.5)
+    m = b["meta"]
+    layout = occ.BatchLayout.from_batch(b, "cuda")
+    s1, _ = occ.occam_score_stage1(layout, occ.OCCAM_STAGE1_MUTUAL, b["Q1"].cuda(), b["K1"].cuda())
+    pooled = occ.occam_pool_scores(s1, 4, "sum").cpu().numpy()
+    ref1, _ = O.stage1_mutual(b["Q1"], b["K1"], m["seg_off_host"], m["reg_idx_host"], m["reg_off_host"])
+    np.testing.assert_allclose(pooled, O.pool_scores(ref1, 4, "sum"), rtol=1e-3, atol=1e-5)
+
+
+def test_pool_scores_rejects_ragged_groups():
+    import paper_2605_29657_gb300 as occ
+
+    with pytest.raises(occ.OccamError):
+        occ.occam_pool_scores(torch.zeros(10, device="cuda"), 4)
