@@ -242,3 +242,37 @@ def test_invalid_arguments_raise():
         occ.occam_score_stage1(layout, occ.OCCAM_STAGE1_CLS, g["q_cls"], g["K1"][:, :8].contiguous())
     with pytest.raises(occ.OccamError):
         occ.occam_score_stage1(layout, occ.OCCAM_STAGE1_CLS, g["q_cls"].float(), g["K1"])
+
+
+# ----------------------------------------------------------------------------- shapes beyond the workloads
+
+@pytest.mark.parametrize("H2", [2, 8, 64])
+def test_other_llm_head_counts(H2):
+    """H2 = 2 takes the two-pass path (the fused kernel needs at least 4 heads); 8 and 64 the fused one."""
+    b = tiny_batch(B=2, segs=2, P=(90, 41), R=2, M=(70, 9), H1=16, d1=64, H2=H2, d2=128, hidden=64, seed=61,
+                   beta1=2.0)
+    for path in ("auto", "twopass"):
+        gpu = run_prune(b, 0.3, 1.1, path=path)
+        assert gpu["status"] == 0
+        check_prune(b, gpu, 0.3, 1.1)
+
+
+def test_many_small_samples():
+    """More samples than one planning block holds (257 > 256 threads), one-token texts, tiny segments."""
+    B = 257
+    rng = np.random.default_rng(62)
+    P = tuple(int(x) for x in rng.integers(1, 12, B))
+    M = tuple(int(x) for x in rng.integers(1, 4, B))
+    b = tiny_batch(B=B, segs=1, P=P, R=1, M=M, H1=16, d1=64, H2=32, d2=128, hidden=32, seed=62, beta1=2.0)
+    gpu = run_prune(b, 0.4, 1.0)
+    assert gpu["status"] == 0
+    check_prune(b, gpu, 0.4, 1.0)
+
+
+def test_long_text_many_fused_items():
+    """Text of 600 tokens: five 128-row fused items (and ten 64-row two-pass tiles) for one sample."""
+    b = _tiny(B=2, segs=1, P=(300, 40), R=4, M=(600, 3), seed=63)
+    for path in ("auto", "narrow", "twopass"):
+        gpu = run_prune(b, 0.2, 1.2, path=path)
+        assert gpu["status"] == 0
+        check_prune(b, gpu, 0.2, 1.2)
