@@ -378,6 +378,16 @@ int occam_compact_noalloc(const occam_batch* batch, const uint8_t* keep, int32_t
                           occam_stream_t stream);
 
 /* Library version string (static storage). */
+/* Diagnostic of the bounded device-side waits (no fault, trap or hang). One
+ * warp waits, each time for about limit_ns (1 .. 1e9), on an mbarrier that
+ * nothing completes (the tensor-core kernels' timer-bounded wait and the
+ * streaming kernels' iteration-bounded wait) and on a flag that nothing sets
+ * (the look-backs' spin). scratch: 4 int32, device. It is zeroed first; on
+ * completion scratch[0] = a bitmask of the waits that gave up (7 when all
+ * three did) and scratch[1] = OCCAM_ERR_TIMEOUT if any did, else 0; scratch[2..3] is the
+ * flag. The context stays usable afterwards. */
+int occam_selftest_wait(uint64_t limit_ns, int32_t* scratch, occam_stream_t stream);
+
 const char* occam_version(void);
 
 #ifdef __cplusplus

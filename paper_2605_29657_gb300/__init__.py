@@ -28,6 +28,7 @@ from ._lib import (  # noqa: F401
     occam_get_status,
     occam_mean_reference,
     occam_pool_scores,
+    occam_selftest_wait,
     occam_prune,
     occam_score_stage1,
     occam_score_stage2,

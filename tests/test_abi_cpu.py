@@ -115,3 +115,10 @@ def test_rule_argument_checked_on_host(lib):
     assert lib.occam_prune(ctypes.byref(a), ctypes.byref(o), None, 0, None) == occ._lib.OCCAM_ERR_INVALID_ARG
     a.rule = occ.OCCAM_RULE_MEAN                                 # valid: fails later, on the workspace
     assert lib.occam_prune(ctypes.byref(a), ctypes.byref(o), None, 0, None) == occ._lib.OCCAM_ERR_WORKSPACE
+
+
+def test_selftest_arguments_checked_on_host(lib):
+    import paper_2605_29657_gb300 as occ
+    assert lib.occam_selftest_wait(0, None, None) == occ._lib.OCCAM_ERR_INVALID_ARG
+    assert lib.occam_selftest_wait(10 ** 6, None, None) == occ._lib.OCCAM_ERR_INVALID_ARG
+    assert lib.occam_selftest_wait(2 * 10 ** 9, 0x1000, None) == occ._lib.OCCAM_ERR_INVALID_ARG
