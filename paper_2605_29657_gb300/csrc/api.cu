@@ -55,11 +55,17 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   const int64_t chmax = cdiv(b->max_sample_rows, kKeyChunk);
   L.maxA = B * tps * nhg * kStatSplits;
   L.maxB = B * tps * chmax;
-  L.maxF = B * cdiv(b->max_text, 128);
+  // fused items: one per text tile, or kHsGroups per tile of a head-split batch
+  L.maxF = std::max<int64_t>(B * cdiv(b->max_text, 128), kHsMaxTiles * kHsGroups);
   L.maxSlots = L.maxB + L.maxF * kFusedSlotsPerItem16;
   L.itemsF = take(L.maxF * 16);
   L.itemsF8 = take(L.maxF * 16);
   L.itemsF16 = take(L.maxF * 16);
+  L.itemsHS = take(kHsMaxTiles * 16);
+  // head-split scratch only for batches with at most kHsMaxTiles text tiles
+  L.ppart = (B * cdiv(b->max_text, kHsRows) <= kHsMaxTiles)
+                ? take((size_t)kHsMaxTiles * kHsGroups * 16 * kHsRows * kFusedMaxOwnImg * 4)
+                : 0;
   L.itemA_off = take((B + 1) * 4);
   L.itemB_off = take((B + 1) * 4);
   L.slot_off = take((B + 1) * 4);
@@ -486,6 +492,8 @@ Stage2Params stage2_params(const occam_batch* b, const occam_stage2_args* a, con
   p.maxF = L.maxF;
   p.use_fused = fused ? 1 : 0;
   p.res16 = widening_enabled() ? fused_resident_clusters(16) : 0;
+  p.itemsHS = at<int4>(ws, L.itemsHS);
+  p.has_ppart = L.ppart != 0 ? 1 : 0;
   p.res8 = widening_enabled() ? fused_resident_clusters(8) : 0;
   return p;
 }
@@ -512,6 +520,8 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     Stage2TcParams q;
     q.bt = p.bt;
     q.H = a->H2;
+    q.ppart = L.ppart != 0 ? at<float>(ws, L.ppart) : nullptr;
+    q.itemsHS = p.itemsHS;
     q.kv_group = a->H2 / kv_heads(a);
     q.K = static_cast<const __nv_bfloat16*>(a->K2);
     q.Kt = static_cast<const __nv_bfloat16*>(kt);
@@ -560,6 +570,9 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     if (launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
     OCCAM_CUDA(cudaEventRecord(side.join, side.stream));
     OCCAM_CUDA(cudaStreamWaitEvent(st, side.join, 0));
+    // head-split tiles (small batches) meet here
+    launch_s2_merge(q16, st);
+    OCCAM_CUDA(cudaGetLastError());
     trace.mark(st);
   } else {
     trace.mark(st);

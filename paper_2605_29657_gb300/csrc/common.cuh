@@ -189,7 +189,7 @@ __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long
 // Workspace carve-up (byte offsets from the workspace base; see ws_layout()).
 struct WsLayout {
   size_t status, counters, role, keep1, s1, s2, ref1, dense, n1, n1_vis;
-  size_t itemA_off, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, seg_state, stats1, itemsF, itemsF8, itemsF16,
+  size_t itemsHS, ppart, itemA_off, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, seg_state, stats1, itemsF, itemsF8, itemsF16,
       slot_off;
   size_t zero_begin, zero_end;  // the accumulators every prune call zeroes (one contiguous range)
   size_t total;
@@ -210,7 +210,8 @@ enum {
   CNT_NF16 = 9,
   CNT_QUEUE16 = 10,    // next fused Stage-II item (16-CTA clusters)
   CNT_MUT = 11,        // [2] next mutual Stage-I item of each pass
-  CNT_SLOTS = 13
+  CNT_NHS = 13,        // Stage-II text tiles split over head groups (merge items)
+  CNT_SLOTS = 14
 };
 
 constexpr int kTextTile = 64;    // Stage-II text rows per item

@@ -33,6 +33,17 @@ __host__ __device__ inline int s2_stat_splits(int n1, int M) {
   const int s = ((n1 + M + 63) / 64 + 3) / 4;
   return s < 1 ? 1 : s > kStatSplits ? kStatSplits : s;
 }
+// Head split of small batches: when every text tile of the batch fits as
+// kHsGroups resident 16-CTA clusters, each tile's heads are split over that
+// many items; their partial head sums meet in a scratch area of kHsMaxTiles
+// tiles (allocated only when the batch can have no more tiles than that).
+constexpr int kHsMaxTiles = 2;
+constexpr int kHsGroups = 8;
+constexpr int kHsRows = 128;  // text rows of a fused item
+// the fused item's w field: (tile index in the scratch << 8) | (head group << 4) | head groups (0 = 1)
+__host__ __device__ inline int hs_groups(int w) { return (w & 15) ? (w & 15) : 1; }
+__host__ __device__ inline int hs_group(int w) { return (w >> 4) & 15; }
+__host__ __device__ inline int hs_tile(int w) { return w >> 8; }
 constexpr int kFusedSlotsPerItem = kFusedCluster * kFusedPartialWarps;  // s2(r) partials per C=4 item
 constexpr int kFusedSlotsPerItem8 = 8 * kFusedPartialWarps;             // and per C=8 item
 constexpr int kFusedSlotsPerItem16 = 16 * kFusedPartialWarps;           // and per C=16 item
@@ -109,6 +120,8 @@ struct Stage2Params {
   int4* itemsF16;           // fused items for 16-CTA clusters
   int use_fused;            // route eligible samples to the fused tensor-core kernel
   int res16, res8;          // resident 16- and 8-CTA fused clusters (0: no widening for small batches)
+  int4* itemsHS;            // head-split text tiles (b, j0, slot, head groups), for the merge kernel
+  int has_ppart;            // the head-split scratch exists
   int32_t* slot_off;        // [B+1] partial-slot range of each sample
   int64_t maxF;
   float* ref2;              // [B]
@@ -252,6 +265,8 @@ struct BudgetParams {
 struct Stage2TcParams {
   BatchDev bt;
   int H;
+  float* ppart;             // head-split scratch [kHsMaxTiles][kHsGroups][16][128][kFusedMaxOwnImg]
+  const int4* itemsHS;      // head-split tiles (merge kernel)
   int kv_group;             // query heads per key / value head (1 unless grouped-query attention)
   const __nv_bfloat16* K;   // [rows, H / kv_group, 128]
   const __nv_bfloat16* Kt;  // [total_text, H / kv_group, 128] (any valid pointer when has_text == 0)
@@ -291,6 +306,7 @@ int s2_stats_smem_bytes();
 
 // stage2_tc.cu
 int fused_resident_clusters(int C);
+void launch_s2_merge(const Stage2TcParams& q, cudaStream_t st);
 int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt, const Stage2TcParams& q,
                  int nclusters, cudaStream_t st);
 int s2_fused_smem_bytes(int C);

@@ -17,18 +17,30 @@ namespace occam {
 __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
   const int tid = threadIdx.x;
   const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
-  int runA = 0, runB = 0, runF = 0, runF8 = 0, runF16 = 0, runS = 0;
+  int runA = 0, runB = 0, runF = 0, runF8 = 0, runF16 = 0, runS = 0, runHS = 0;
   // A small batch leaves most SMs idle with 4-CTA clusters: when every text
   // tile of the batch can run at once as a resident 16- (or 8-) CTA cluster,
   // samples take the wider cluster, whose CTAs hold fewer keys and finish
   // each head sooner.
-  int wide = 0;
+  int wide = 0, hsg = 1;  // hsg: head groups of a split tile (1: no split)
   if (p.use_fused) {
     int tiles = 0;
     for (int b = tid; b < p.bt.B; b += blockDim.x) tiles += (int)((p.bt.text_off[b + 1] - p.bt.text_off[b] + 127) / 128);
     int total_tiles;
     block_exclusive_scan(tiles, tmp, &total_tiles);
     wide = total_tiles <= p.res16 ? 16 : total_tiles <= p.res8 ? 8 : 0;
+    // head split: a batch of at most kHsMaxTiles tiles whose tiles fit hsg
+    // times over as resident 16-CTA clusters splits each 16-CTA tile's heads
+    // into hsg groups (whole key groups, at least 4 heads each)
+    if (wide == 16 && p.has_ppart && total_tiles <= kHsMaxTiles) {
+      const int grp = p.H / p.Hkv;
+      for (int g = kHsGroups; g >= 2; g >>= 1) {
+        if (total_tiles * g <= p.res16 && p.H % g == 0 && p.H / g >= 4 && (p.H / g) % grp == 0) {
+          hsg = g;
+          break;
+        }
+      }
+    }
   }
   for (int b0 = 0; b0 < p.bt.B; b0 += blockDim.x) {
     const int bb = b0 + tid;
@@ -48,7 +60,7 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
       } else if (fused8) {
         nF8 = (M + 127) / 128;
       } else if (fused16) {
-        nF16 = (M + 127) / 128;
+        nF16 = (M + 127) / 128 * hsg;
       } else {
         const int tiles = (M + kTextTile - 1) / kTextTile;
         const int nch = (n1 + kKeyChunk - 1) / kKeyChunk;
@@ -61,22 +73,31 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
         p.tau2[bb] = 0.f;
       }
     }
-    const int nS = nF * kFusedSlotsPerItem + nF8 * kFusedSlotsPerItem8 + nF16 * kFusedSlotsPerItem16 +
-                   nB;  // s2(r) partial slots of this sample
-    int totA, totB, totF, totF8, totF16, totS;
+    const int nS = nF * kFusedSlotsPerItem + nF8 * kFusedSlotsPerItem8 + nF16 / hsg * kFusedSlotsPerItem16 +
+                   nB;  // s2(r) partial slots of this sample (a split tile's items share its slots)
+    const int nHS = hsg > 1 ? nF16 / hsg : 0;  // this sample's head-split tiles
+    int totA, totB, totF, totF8, totF16, totS, totHS;
     const int offA = runA + block_exclusive_scan(nA, tmp, &totA);
     const int offB = runB + block_exclusive_scan(nB, tmp, &totB);
     const int offF = runF + block_exclusive_scan(nF, tmp, &totF);
     const int offF8 = runF8 + block_exclusive_scan(nF8, tmp, &totF8);
     const int offF16 = runF16 + block_exclusive_scan(nF16, tmp, &totF16);
     const int offS = runS + block_exclusive_scan(nS, tmp, &totS);
+    const int offHS = runHS + block_exclusive_scan(nHS, tmp, &totHS);
     if (bb < p.bt.B) {
       for (int i = 0; i < nF; ++i)
         if (offF + i < p.maxF) p.itemsF[offF + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem, 0);
       for (int i = 0; i < nF8; ++i)
         if (offF8 + i < p.maxF) p.itemsF8[offF8 + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem8, 0);
-      for (int i = 0; i < nF16; ++i)
-        if (offF16 + i < p.maxF) p.itemsF16[offF16 + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem16, 0);
+      for (int i = 0; i < nF16; ++i) {
+        const int tile = i / hsg, hg = i % hsg;
+        const int w = hsg > 1 ? ((offHS + tile) << 8) | (hg << 4) | hsg : 0;
+        if (offF16 + i < p.maxF)
+          p.itemsF16[offF16 + i] = make_int4(bb, tile * 128, offS + tile * kFusedSlotsPerItem16, w);
+      }
+      for (int t = 0; t < nHS; ++t)
+        if (offHS + t < kHsMaxTiles)
+          p.itemsHS[offHS + t] = make_int4(bb, t * 128, offS + t * kFusedSlotsPerItem16, hsg);
       p.itemA_off[bb] = offA;
       p.itemB_off[bb] = offB;
       p.slot_off[bb] = offS;
@@ -87,6 +108,7 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
     runF8 += totF8;
     runF16 += totF16;
     runS += totS;
+    runHS += totHS;
   }
   if (tid == 0) {
     p.itemA_off[p.bt.B] = runA;
@@ -99,6 +121,7 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
     p.counters[CNT_NF] = (int)(runF < p.maxF ? runF : p.maxF);
     p.counters[CNT_NF8] = (int)(runF8 < p.maxF ? runF8 : p.maxF);
     p.counters[CNT_NF16] = (int)(runF16 < p.maxF ? runF16 : p.maxF);
+    p.counters[CNT_NHS] = runHS < kHsMaxTiles ? runHS : kHsMaxTiles;
   }
 }
 

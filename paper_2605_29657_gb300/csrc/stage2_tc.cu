@@ -118,6 +118,7 @@ namespace {
 
 struct ItemGeom {
   int b, j0, M, n, img0, own_img, txt0, own_txt, ip, tp, N, slot;
+  int h0, h1, nhg, hs_tile;  // heads [h0, h1) of this item; head groups of its tile (1: no split)
   bool fits;
   int64_t rbase, t0;
 };
@@ -146,6 +147,10 @@ __device__ __forceinline__ ItemGeom item_geom(const Stage2TcParams& p, int4 it, 
   // the same on every CTA of the cluster (depends on the sample only)
   const int ipmax = (per + 31) & ~31;
   g.fits = ipmax <= PMAX && ipmax + ((per_t + 15) & ~15) <= Geo<C>::KROWS;
+  g.nhg = hs_groups(it.w);
+  g.h0 = hs_group(it.w) * p.H / g.nhg;
+  g.h1 = (hs_group(it.w) + 1) * p.H / g.nhg;
+  g.hs_tile = hs_tile(it.w);
   return g;
 }
 
@@ -403,7 +408,8 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         // grouped-query attention: the group's query heads share one key
         // block, loaded for the group's first head (the ring advances per key
         // head); gi = h's index in its group, hkv = the key head it reads
-        for (int h = 0, gi = 0, hkv = 0; h < H && ok; ++h, gi = gi + 1 == p.kv_group ? 0 : gi + 1, hkv += gi == 0) {
+        for (int h = g.h0, gi = 0, hkv = g.h0 / p.kv_group; h < g.h1 && ok;
+             ++h, gi = gi + 1 == p.kv_group ? 0 : gi + 1, hkv += gi == 0) {
           const int kb = kcnt & 1;
           const bool load_keys = gi == 0;
           if (load_keys && !tc::bar_wait(&sm.kempty[kb], ((kcnt >> 1) & 1) ^ 1, abort, kLimitNs)) {
@@ -473,7 +479,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
           if (!g.fits) continue;
           const uint32_t idesc = tc::idesc_bf16(128, g.N > 0 ? g.N : 16);
           bool ok = true;
-          for (int h = 0, gi = 0; h < H && ok; ++h, ++hk, gi = gi + 1 == p.kv_group ? 0 : gi + 1) {
+          for (int h = g.h0, gi = 0; h < g.h1 && ok; ++h, ++hk, gi = gi + 1 == p.kv_group ? 0 : gi + 1) {
             const int qb = qcnt & 1, kb = kcnt & 1, eb = hk & 1;
             // E[eb] is free once head hk - 2 was read out of it
             ok = tc::bar_wait(&sm.qfull[qb], (qcnt >> 1) & 1, abort, kLimitNs);
@@ -547,7 +553,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       // the remaining pieces start with the warp that took fewer groups
       const int k0 = 2 * ngf + ((half + ngf) & 1);
       bool ok = true;
-      for (int h = 0; h < H; ++h, ++hk) {
+      for (int h = g.h0; h < g.h1; ++h, ++hk) {
         const int eb = hk & 1;
         const uint32_t ebase = tmem + lane_base + eb * G::KROWS;
         if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.efull[eb], (hk >> 1) & 1, nullptr, kLimitNs))) {
@@ -637,7 +643,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
 #pragma unroll
         for (int b2 = 0; b2 < 32; ++b2) P[q][b2] = 0.f;
       bool ok = true;
-      for (int h = 0; h < H; ++h, ++hk) {
+      for (int h = g.h0; h < g.h1; ++h, ++hk) {
         const int eb = hk & 1;
         const int slot = hk & (NXS - 1);
         if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.sdone[eb], (hk >> 1) & 1, nullptr, kLimitNs))) {
@@ -683,6 +689,25 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         if (armer) tc::bar_expect_tx(&sm.xbar[slot], G::XBYTES);
       }
       if (!ok) { fail(sm, p.status); break; }
+      if (g.nhg > 1) {
+        // a head group of a split tile: its partial head sums go to the
+        // scratch, rows of zeros past the text; the merge kernel reduces them
+        float* dst = p.ppart + ((((int64_t)g.hs_tile * kHsGroups + hs_group(p.items[item].w)) * 16 + rank) * kHsRows + j) *
+                                   PMAX;
+#pragma unroll
+        for (int q = 0; q < NPC; ++q) {
+          if (q < npi) {
+#pragma unroll
+            for (int c4 = 0; c4 < 8; ++c4)
+              *reinterpret_cast<float4*>(dst + q * 32 + 4 * c4) =
+                  vrow && wvalid ? make_float4(P[q][4 * c4], P[q][4 * c4 + 1], P[q][4 * c4 + 2], P[q][4 * c4 + 3])
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) tc::bar_arrive(&sm.idone[ib]);
+        continue;
+      }
       // ---- column reductions of P over this warp's 32 rows: column max ->
       // s2 (atomicMax), register columns -> this warp's partial of s2(r)
       float regacc = 0.f;
@@ -773,6 +798,93 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   }
   // peers may still write into this CTA's exchange buffers until here
   tc::cluster_sync_all();
+}
+
+// Merge of head-split tiles. CTA (t, rank) of a kHsMaxTiles x 16 grid takes
+// tile t's S1 keys of cluster rank `rank`, one key column per thread: it sums
+// the head groups' partials (in group order) row by row, takes the column
+// max over the tile's text rows into s2, and sums the register columns over
+// rows. The register sums of the CTA's columns, added in a fixed order, fill
+// the tile's partial slots of that rank. The sample's last slot writer turns
+// the slots into ref2 and tau2 as the fused kernel does.
+__global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParams p) {
+  using namespace s2f;
+  constexpr int NW = kFusedMaxOwnImg / 32;
+  __shared__ float wsum[NW];
+  __shared__ int s_last;
+  const int t = blockIdx.x / 16, rank = blockIdx.x % 16;
+  if (t >= p.counters[CNT_NHS]) return;
+  const int4 it = p.itemsHS[t];
+  const int nhg = it.w;
+  const ItemGeom g = item_geom<16>(p, make_int4(it.x, it.y, it.z, 0), rank);
+  const int k = threadIdx.x, lane = k & 31;
+  const int rows = min(kHsRows, g.M - g.j0);
+  const float invH = 1.0f / (float)p.H;
+  float rc = 0.f;
+  if (k < g.own_img) {
+    const int row_id = p.dense[g.rbase + g.img0 + k];
+    const bool is_reg = p.role[row_id] != 0;
+    const float* src = p.ppart + (((int64_t)t * kHsGroups * 16 + rank) * kHsRows) * PMAX + k;
+    float cmax = 0.f, rsum = 0.f;
+    // eight rows at a time, every group's load issued before any add (up to
+    // 32 loads in flight); the sums still run in group order, then row order
+    for (int r0 = 0; r0 < rows; r0 += 8) {
+      float v[8][kHsGroups];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+#pragma unroll
+        for (int hg = 0; hg < kHsGroups; ++hg)
+          v[u][hg] = (r0 + u < rows && hg < nhg) ? __ldcg(src + ((int64_t)hg * 16 * kHsRows + r0 + u) * PMAX) : 0.f;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (r0 + u < rows) {
+          float x = v[u][0];
+#pragma unroll
+          for (int hg = 1; hg < kHsGroups; ++hg) x += v[u][hg];
+          cmax = fmaxf(cmax, x);
+          rsum += x;
+        }
+      }
+    }
+    if (is_reg) {
+      rc = rsum * invH;
+    } else {
+      atomicMax(reinterpret_cast<int*>(&p.s2[row_id]), __float_as_int(cmax * invH));
+    }
+  }
+  rc = warp_sum_f(rc);
+  if (lane == 0) wsum[k >> 5] = rc;
+  __syncthreads();
+  if (k == 0) {
+    float acc = 0.f;
+    for (int w = 0; w < NW; ++w) acc += wsum[w];
+    // the tile's NPW slots of this rank: the sum in the first, zeros after
+    p.refpart[g.slot + rank * NPW] = acc;
+    for (int i = 1; i < NPW; ++i) p.refpart[g.slot + rank * NPW + i] = 0.f;
+    __threadfence();
+    const int nslots = p.slot_off[g.b + 1] - p.slot_off[g.b];
+    s_last = atomicAdd(&p.done[g.b], NPW) == nslots - NPW;
+  }
+  __syncthreads();
+  if (s_last && k < 32) {
+    // the sample's last partials: ref2 = (sum of the partials) / (R M),
+    // lane l taking slots l, l + 32, ... in order, then a fixed tree
+    __threadfence();
+    const int s0 = p.slot_off[g.b], s1 = p.slot_off[g.b + 1];
+    float acc = 0.f;
+    for (int i = s0 + lane; i < s1; i += 32) acc += __ldcg(&p.refpart[i]);
+    acc = warp_sum_f(acc);
+    if (lane == 0) {
+      const int R = p.bt.reg_off[p.bt.seg_first[g.b + 1]] - p.bt.reg_off[p.bt.seg_first[g.b]];
+      const float r2 = (R > 0 && g.M > 0) ? acc / ((float)R * (float)g.M) : 0.f;
+      p.ref2[g.b] = r2;
+      p.tau2[g.b] = p.lambda2 * r2;
+    }
+  }
+}
+
+void launch_s2_merge(const Stage2TcParams& q, cudaStream_t st) {
+  if (q.ppart) s2_merge_kernel<<<kHsMaxTiles * 16, kFusedMaxOwnImg, 0, st>>>(q);
 }
 
 // How many C-CTA clusters of the fused kernel the current device holds at
