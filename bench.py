@@ -291,6 +291,9 @@ def run_ours(args, rank, world, local):
         if st != 0:
             raise RuntimeError(f"device status {st} after warm-up")
     out = call.out
+    call()                                         # an eager call, to count the kernels it launches
+    torch.cuda.synchronize()
+    kernels_per_step = occ.occam_last_call_kernels()
     n1_total = int(out["n1_vis"].sum().item()) + int(meta["regs_per_seg"] * meta["S_tot"])  # registers are in S1
     kept_total = int(out["out_off"][-1].item())
     bytes_ = algorithmic_bytes(meta, n1_total, kept_total)
@@ -598,7 +601,7 @@ def run_ours(args, rank, world, local):
         # kernels per occam_prune call: Stage I (1 [CLS] / 2 mutual), finalize
         # (with the Stage-II plan), fused Stage II with 16-, 8- and 4-CTA
         # clusters, the two-pass Stage-II pair, scan, gather
-        "gpu_launches": (9 if w.stage1 == "cls" else 10) * args.steps,
+        "gpu_launches": kernels_per_step * args.steps,
         "clocks": clocks,
         "next_rows": next_rows,
     }

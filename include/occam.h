@@ -388,6 +388,12 @@ int occam_compact_noalloc(const occam_batch* batch, const uint8_t* keep, int32_t
  * flag. The context stays usable afterwards. */
 int occam_selftest_wait(uint64_t limit_ns, int32_t* scratch, occam_stream_t stream);
 
+/* How many kernels the last entry point called on this host thread launched
+ * (host-side count; an entry point that returned an error may have launched
+ * fewer than a full call). A launch whose work list turns out empty on the
+ * device still counts. */
+int occam_last_call_kernels(void);
+
 const char* occam_version(void);
 
 #ifdef __cplusplus

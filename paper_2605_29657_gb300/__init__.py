@@ -26,6 +26,7 @@ from ._lib import (  # noqa: F401
     occam_compact_noalloc,
     occam_construct_registers,
     occam_get_status,
+    occam_last_call_kernels,
     occam_mean_reference,
     occam_pool_scores,
     occam_selftest_wait,

@@ -115,7 +115,8 @@ def library() -> ctypes.CDLL:
         lib.occam_budget_keep.argtypes = [P(CBatch), _p, _p, _p, _i32, _p, _p, _p, ctypes.c_size_t, _p]
         lib.occam_pool_scores.argtypes = [_p, _i64, _i32, _i32, _p, _p]
         lib.occam_selftest_wait.argtypes = [ctypes.c_uint64, _p, _p]
-        for name in ("occam_selftest_wait", "occam_pool_scores", "occam_mean_reference", "occam_budget_keep", "occam_construct_registers", "occam_calibrate_lambda2", "occam_workspace_size", "occam_get_status", "occam_score_stage1",
+        lib.occam_last_call_kernels.argtypes = []
+        for name in ("occam_last_call_kernels", "occam_selftest_wait", "occam_pool_scores", "occam_mean_reference", "occam_budget_keep", "occam_construct_registers", "occam_calibrate_lambda2", "occam_workspace_size", "occam_get_status", "occam_score_stage1",
                      "occam_threshold",
                      "occam_score_stage2", "occam_compact", "occam_prune", "occam_prune_traced",
                      "occam_compact_noalloc", "occam_prune_staged"):
@@ -291,6 +292,11 @@ def occam_mean_reference(layout: BatchLayout, s, ref_scope: int, prev_keep=None,
     _check(library().occam_mean_reference(ctypes.byref(cb), _ptr(s), int(ref_scope), _ptr(prev_keep), _ptr(ref),
                                           _ptr(ws), ws.numel(), _stream(stream)), "occam_mean_reference")
     return ref
+
+
+def occam_last_call_kernels() -> int:
+    """Kernels the last entry point called on this thread launched."""
+    return int(library().occam_last_call_kernels())
 
 
 def occam_selftest_wait(limit_ns: int = 20_000_000, device="cuda", stream=None) -> tuple[int, int]:

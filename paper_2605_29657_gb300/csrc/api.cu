@@ -14,6 +14,11 @@
 
 using namespace occam;
 
+int& occam::launch_counter() {
+  thread_local int n = 0;
+  return n;
+}
+
 namespace {
 
 constexpr size_t kAlign = 256;
@@ -373,6 +378,7 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
     const int64_t tiles = cdiv(b->total_rows, 16);
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(tiles, 2 * num_sms()));
     stage1_logits_kernel<<<grid, 256, stage1_logits_smem_bytes(), st>>>(p);
+    count_launch();
     trace.mark(st);
   } else {
     MutualTcParams p;
@@ -443,6 +449,7 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   p.zero_count_out = count_out;
   p.zero_count_vis = count_vis;
   stage1_finalize_kernel<<<b->S_tot, 256, finalize_smem_bytes(p.smem_rows, cls), st>>>(p);
+  count_launch();
   trace.mark(st);
   return cuda_ok();
 }
@@ -454,6 +461,7 @@ void launch_twopass(const Stage2Params& p, const WsLayout& L, int sms, cudaStrea
   const int gB = (int)std::min<int64_t>(L.maxB, sms);
   if (gA > 0) s2_stats_kernel<<<gA, 128, s2_stats_smem_bytes(), st>>>(p);
   if (gB > 0) s2_scores_kernel<<<gB, 256, s2_scores_smem_bytes(), st>>>(p);
+  count_launch((gA > 0) + (gB > 0));
 }
 
 // Stage-II parameter block (the same for the plan, built by the Stage-I
@@ -548,11 +556,16 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     if (!side.ok) return OCCAM_ERR_CUDA;
     OCCAM_CUDA(cudaEventRecord(side.fork, st));
     OCCAM_CUDA(cudaStreamWaitEvent(side.stream, side.fork, 0));
+    // A batch whose every text tile fits as a resident 16-CTA cluster gets
+    // the 16-CTA routing for all of its fused samples (the plan's widening;
+    // a sample that a 16-CTA cluster cannot hold fits no smaller one): its
+    // 8- and 4-CTA launches would have no items, so they are not made.
+    const bool only16 = p.res16 > 0 && (int64_t)b->B * cdiv(b->max_text, 128) <= p.res16;
     Stage2TcParams q8 = q;
     q8.items = p.itemsF8;
     q8.queue = p.counters + CNT_QUEUE8;
     const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
-    if (launch_fused(8, mq, mk, mkt, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
+    if (!only16 && launch_fused(8, mq, mk, mkt, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
     // the two-pass kernels (samples the fused kernel cannot hold; often none)
     // follow the 8-CTA launch on the second stream
     launch_twopass(p, L, sms, side.stream);
@@ -567,7 +580,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     if (launch_fused(16, mq, mk, mkt, q16, ncl16, st) != 0) return OCCAM_ERR_CUDA;
     q.queue = p.counters + CNT_QUEUE4;
     const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
-    if (launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
+    if (!only16 && launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
     OCCAM_CUDA(cudaEventRecord(side.join, side.stream));
     OCCAM_CUDA(cudaStreamWaitEvent(st, side.join, 0));
     // head-split tiles (small batches) meet here
@@ -613,6 +626,7 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
     if (count_vis) OCCAM_CUDA(cudaMemsetAsync(count_vis, 0, b->B * 4, st));
   }
   scan_kernel<<<(unsigned)L.scan_tiles, 256, 0, st>>>(p);
+  count_launch();
   trace.mark(st);
   if (n_tensors > 0) {
     GatherParams g;
@@ -627,6 +641,7 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
     g.B = b->B;
     g.capacity = capacity;
     gather_kernel<<<num_sms() * 4, 256, 0, st>>>(g);
+    count_launch();
   }
   trace.mark(st);
   return cuda_ok();
@@ -636,12 +651,15 @@ int mark_roles(const occam_batch* b, const WsLayout& L, void* ws, cudaStream_t s
   uint8_t* role = at<uint8_t>(ws, L.role);
   OCCAM_CUDA(cudaMemsetAsync(role, 0, b->total_rows, st));
   roles_scatter_kernel<<<64, 256, 0, st>>>(dev_batch(b), role);
+  count_launch();
   return cuda_ok();
 }
 
 }  // namespace
 
 extern "C" {
+
+int occam_last_call_kernels(void) { return launch_counter(); }
 
 const char* occam_version(void) { return "occam-gb300 0.1 (sm_103a)"; }
 
@@ -665,6 +683,7 @@ int occam_get_status(void* workspace, int32_t* status, occam_stream_t stream) {
 
 int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, float* s1, float* ref1,
                        void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   OCCAM_TRY(check_stage1(batch, args));
   if (!s1) return OCCAM_ERR_INVALID_ARG;
@@ -681,6 +700,7 @@ int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, 
 int occam_threshold(const occam_batch* batch, const float* s, const float* ref, int32_t ref_scope, float lambda,
                     const uint8_t* prev_keep, int32_t keep_registers, uint8_t* keep, int32_t* count_vis,
                     void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!s || !ref || !keep) return OCCAM_ERR_INVALID_ARG;
   if (ref_scope != OCCAM_REF_SEGMENT && ref_scope != OCCAM_REF_SAMPLE) return OCCAM_ERR_INVALID_ARG;
@@ -702,11 +722,13 @@ int occam_threshold(const occam_batch* batch, const float* s, const float* ref, 
   p.keep = keep;
   p.count_vis = count_vis;
   threshold_kernel<<<(unsigned)cdiv(batch->total_rows, 256), 256, 0, st>>>(p);
+  count_launch();
   return cuda_ok();
 }
 
 int occam_mean_reference(const occam_batch* batch, const float* s, int32_t ref_scope, const uint8_t* prev_keep,
                          float* ref, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!s || !ref) return OCCAM_ERR_INVALID_ARG;
   if (ref_scope != OCCAM_REF_SEGMENT && ref_scope != OCCAM_REF_SAMPLE) return OCCAM_ERR_INVALID_ARG;
@@ -724,11 +746,13 @@ int occam_mean_reference(const occam_batch* batch, const float* s, int32_t ref_s
   p.lambda = 0.f;
   p.tau = nullptr;
   mean_ref_kernel<<<ref_scope == OCCAM_REF_SEGMENT ? batch->S_tot : batch->B, 256, 0, st>>>(p);
+  count_launch();
   return cuda_ok();
 }
 
 int occam_pool_scores(const float* s_in, int64_t rows_in, int32_t group, int32_t mode, float* s_out,
                       occam_stream_t stream) {
+  launch_counter() = 0;
   if (!s_in || !s_out || group < 1 || rows_in < 0 || rows_in % group != 0) return OCCAM_ERR_INVALID_ARG;
   if (mode != OCCAM_POOL_SUM && mode != OCCAM_POOL_MEAN && mode != OCCAM_POOL_MAX) return OCCAM_ERR_INVALID_ARG;
   const int64_t rows_out = rows_in / group;
@@ -738,12 +762,14 @@ int occam_pool_scores(const float* s_in, int64_t rows_in, int32_t group, int32_t
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const unsigned blocks = (unsigned)std::min<int64_t>(cdiv(rows_out, 256), (int64_t)num_sms() * 8);
   pool_scores_kernel<<<blocks, 256, 0, st>>>(s_in, rows_out, group, mode, s_out);
+  count_launch();
   return cuda_ok();
 }
 
 int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* prev_keep, const int32_t* budget,
                       int32_t keep_registers, uint8_t* keep, int32_t* count_vis, void* workspace,
                       size_t workspace_bytes, occam_stream_t stream) {
+  launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!s || !budget || !keep) return OCCAM_ERR_INVALID_ARG;
   WsLayout L;
@@ -760,11 +786,13 @@ int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* p
   p.keep = keep;
   p.count_vis = count_vis;
   budget_keep_kernel<<<batch->B, 1024, 0, st>>>(p);
+  count_launch();
   return cuda_ok();
 }
 
 int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, const uint8_t* keep1, float* s2,
                        float* ref2, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   OCCAM_TRY(check_stage2(args));
   if (!keep1 || !s2 || !ref2) return OCCAM_ERR_INVALID_ARG;
@@ -786,6 +814,7 @@ int occam_compact(const occam_batch* batch, const uint8_t* keep, int32_t n_tenso
                   const int64_t* row_bytes, void* const* dst, int64_t capacity_rows, int32_t* out_index,
                   int32_t* count_out, int64_t* out_off, void* workspace, size_t workspace_bytes,
                   occam_stream_t stream) {
+  launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!keep || !count_out || !out_off || capacity_rows < 0 || (capacity_rows > 0 && !out_index))
     return OCCAM_ERR_INVALID_ARG;
@@ -800,6 +829,7 @@ int occam_compact(const occam_batch* batch, const uint8_t* keep, int32_t n_tenso
 static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                       size_t workspace_bytes, occam_stream_t stream, Trace trace, void* k2_stage = nullptr,
                       size_t k2_stage_bytes = 0) {
+  launch_counter() = 0;
   if (!args || !out) return OCCAM_ERR_INVALID_ARG;
   const occam_batch* b = &args->batch;
   OCCAM_TRY(check_batch(b));
@@ -875,6 +905,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
     sp.dense = at<int32_t>(ws, L.dense);
     sp.n1 = at<int32_t>(ws, L.n1);
     stage_rows_kernel<<<num_sms() * 4, 256, 0, st>>>(sp);
+    count_launch();
     OCCAM_CUDA(cudaGetLastError());
   }
   OCCAM_TRY(launch_stage2(b, &a2, L, ws, s2, ref2, args->lambda2, st, trace));
@@ -891,6 +922,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
     bp.keep = out->keep2;
     bp.count_vis = nullptr;
     budget_keep_kernel<<<b->B, 1024, 0, st>>>(bp);
+    count_launch();
     OCCAM_CUDA(cudaGetLastError());
     return launch_compact(b, L, ws, 0, out->keep2, nullptr, nullptr, args->keep_registers, nullptr, args->n_tensors,
                           src, args->row_bytes, dst, args->capacity_rows, out->out_index, out->count_out,
@@ -908,6 +940,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
     mp.lambda = args->lambda2;
     mp.tau = at<float>(ws, L.tau2);
     mean_ref_kernel<<<b->B, 256, 0, st>>>(mp);
+    count_launch();
     OCCAM_CUDA(cudaGetLastError());
   }
   return launch_compact(b, L, ws, 1, nullptr, keep1, s2, args->keep_registers, out->keep2, args->n_tensors,
@@ -922,6 +955,7 @@ int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* 
 
 int occam_construct_registers(const occam_batch* batch, void* h, int64_t channels, const int32_t* k_reg,
                               int32_t n_k, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!h || channels <= 0 || n_k < 0 || (n_k > 0 && !k_reg)) return OCCAM_ERR_INVALID_ARG;
   WsLayout L;
@@ -939,12 +973,14 @@ int occam_construct_registers(const occam_batch* batch, void* h, int64_t channel
   p.n_k = n_k;
   p.role = at<uint8_t>(workspace, L.role);
   registers_kernel<<<batch->S_tot, 256, 0, st>>>(p);
+  count_launch();
   return cuda_ok();
 }
 
 int occam_calibrate_lambda2(const occam_batch* batch, const float* s2, const float* ref2, const uint8_t* keep1,
                             int64_t target_count, float* lambda2_out, int32_t* n_candidates, void* workspace,
                             size_t workspace_bytes, occam_stream_t stream) {
+  launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!s2 || !ref2 || !keep1 || !lambda2_out) return OCCAM_ERR_INVALID_ARG;
   if (batch->total_rows > (int64_t)0x7fffffff) return OCCAM_ERR_UNSUPPORTED;
@@ -963,6 +999,7 @@ int occam_calibrate_lambda2(const occam_batch* batch, const float* s2, const flo
   p.lambda2 = lambda2_out;
   p.n_candidates = n_candidates;
   lambda2_select_kernel<<<1, 1024, 0, st>>>(p);
+  count_launch();
   return cuda_ok();
 }
 

@@ -10,6 +10,11 @@
 
 namespace occam {
 
+// Kernels launched by the current host thread since the entry point it is in
+// began (each entry point resets it; occam_last_call_kernels reports it).
+int& launch_counter();
+inline void count_launch(int n = 1) { launch_counter() += n; }
+
 constexpr int kWarp = 32;
 
 // ---------------------------------------------------------------- status word

@@ -390,6 +390,7 @@ extern "C" int occam_compact_noalloc(const occam_batch* b, const uint8_t* keep, 
                                      const void* const* src, const int64_t* row_bytes, void* const* dst,
                                      int64_t capacity_rows, int32_t* out_index, int32_t* count_out,
                                      int64_t* out_off, occam_stream_t stream) {
+  occam::launch_counter() = 0;
   using namespace occam;
   if (!b || b->B < 1 || b->S_tot < b->B || b->total_rows < 1 || !b->row_off || !b->seg_off ||
       !b->reg_idx || !b->reg_off)
@@ -446,6 +447,7 @@ extern "C" int occam_compact_noalloc(const occam_batch* b, const uint8_t* keep, 
   p.ntiles = ntiles;
   p.status = status;
   scan_kernel<<<(unsigned)ntiles, 256, 0, st>>>(p);
+  count_launch();
   if (n_tensors > 0) {
     GatherParams g;
     g.n_tensors = n_tensors;
@@ -459,6 +461,7 @@ extern "C" int occam_compact_noalloc(const occam_batch* b, const uint8_t* keep, 
     g.B = b->B;
     g.capacity = capacity_rows;
     gather_kernel<<<sms * 4, 256, 0, st>>>(g);
+    count_launch();
   }
   return cudaGetLastError() == cudaSuccess ? OCCAM_OK : OCCAM_ERR_CUDA;
 }

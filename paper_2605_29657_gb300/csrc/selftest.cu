@@ -46,6 +46,8 @@ extern "C" int occam_selftest_wait(uint64_t limit_ns, int32_t* scratch, occam_st
   if (cudaMemsetAsync(scratch, 0, 16, st) != cudaSuccess) return OCCAM_ERR_CUDA;
   // about one try per 32 ns sleep: the iteration limit spans a similar time
   const uint32_t max_iter = (uint32_t)std::min<uint64_t>(limit_ns / 32, 1u << 24);
+  launch_counter() = 0;
   selftest_wait_kernel<<<1, 32, 0, st>>>(limit_ns, max_iter < 16 ? 16 : max_iter, scratch);
+  count_launch();
   return cudaGetLastError() == cudaSuccess ? OCCAM_OK : OCCAM_ERR_CUDA;
 }

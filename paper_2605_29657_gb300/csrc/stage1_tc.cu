@@ -459,6 +459,7 @@ void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUte
   mutual_tc_kernel<1><<<sms, m1::THREADS, smem, st>>>(mq, mk, mq1, mk1, p);
   mutual_tc_kernel<2><<<sms, m1::THREADS, smem, st>>>(mk, mq, mk1, mq1, p);
   mutual_reduce_kernel<<<sms * 2, 256, 0, st>>>(p);
+  count_launch(3);
 }
 
 }  // namespace occam

@@ -884,7 +884,10 @@ __global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParam
 }
 
 void launch_s2_merge(const Stage2TcParams& q, cudaStream_t st) {
-  if (q.ppart) s2_merge_kernel<<<kHsMaxTiles * 16, kFusedMaxOwnImg, 0, st>>>(q);
+  if (q.ppart) {
+    s2_merge_kernel<<<kHsMaxTiles * 16, kFusedMaxOwnImg, 0, st>>>(q);
+    count_launch();
+  }
 }
 
 // How many C-CTA clusters of the fused kernel the current device holds at
@@ -946,6 +949,7 @@ int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUte
   // 16-CTA clusters exceed the portable limit of 8
   if (C == 16) cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mq, mk, mkt, q);
+  count_launch();
   return e == cudaSuccess ? 0 : 1;
 }
 

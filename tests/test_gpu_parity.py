@@ -276,3 +276,28 @@ def test_long_text_many_fused_items():
         gpu = run_prune(b, 0.2, 1.2, path=path)
         assert gpu["status"] == 0
         check_prune(b, gpu, 0.2, 1.2)
+
+
+@pytest.mark.parametrize("name", ["llava15_b1", "llavanext_b8", "llavanext_b64"])
+def test_kernel_count_matches_profiler(name):
+    """occam_last_call_kernels agrees with the kernels a profiler sees for one prune call."""
+    import paper_2605_29657_gb300 as occ
+    from torch.profiler import ProfilerActivity, profile
+
+    w = get_config(name)
+    b = make_batch(w, "cuda", with_gather=True)
+    layout = occ.BatchLayout.from_batch(b, "cuda")
+    call = occ.PruneCall(layout, dict(mode="cls", q=b["q_cls"], k_cls=b["k_cls"], K1=b["K1"]),
+                         dict(Q_text=b["Q_text"], K_text=b["K_text"], K2=b["K2"]), w.lambda1, w.lambda2,
+                         gather=(b["hidden"],))
+    call()
+    torch.cuda.synchronize()
+    with profile(activities=[ProfilerActivity.CUDA]) as prof:
+        call()
+        torch.cuda.synchronize()
+    claimed = occ.occam_last_call_kernels()
+    ours = [e for e in prof.events() if e.device_type == torch.autograd.DeviceType.CUDA and "occam" in e.name]
+    if not ours:
+        pytest.skip("the profiler sees no device activity here")
+    assert len(ours) == claimed, (claimed, sorted(e.name for e in ours))
+    assert call.status() == 0
