@@ -292,9 +292,10 @@ def test_kernel_count_matches_profiler(name):
                          gather=(b["hidden"],))
     call()
     torch.cuda.synchronize()
-    with profile(activities=[ProfilerActivity.CUDA]) as prof:
-        call()
-        torch.cuda.synchronize()
+    for _ in range(2):  # a process's first profiling session may miss device activity
+        with profile(activities=[ProfilerActivity.CUDA]) as prof:
+            call()
+            torch.cuda.synchronize()
     claimed = occ.occam_last_call_kernels()
     ours = [e for e in prof.events() if e.device_type == torch.autograd.DeviceType.CUDA and "occam" in e.name]
     if not ours:
