@@ -42,12 +42,6 @@ __device__ __forceinline__ void stg_stream(void* p, uint4 v) {
                : "memory");
 }
 
-// ---------------------------------------------------------------- warp reductions
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

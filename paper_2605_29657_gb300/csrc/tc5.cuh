@@ -102,9 +102,6 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_b
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(dst)), "l"(src), "r"(src_bytes)
                : "memory");
 }
-__device__ __forceinline__ void cp_async_arrive(uint64_t* bar) {
-  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(su32(bar)) : "memory");
-}
 // makes shared-memory data written through the generic proxy visible to
 // subsequent tensor-core (async proxy) reads by this thread
 __device__ __forceinline__ void fence_proxy_async() {
@@ -269,27 +266,8 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 }
 
 // ---------------------------------------------------------------- distributed shared memory
-__device__ __forceinline__ void st_cluster_f2(const void* local_addr, uint32_t rank, float x, float y) {
-  asm volatile(
-      "{\n\t.reg .b32 ra;\n\t"
-      "mapa.shared::cluster.u32 ra, %0, %1;\n\t"
-      "st.shared::cluster.v2.f32 [ra], {%2, %3};\n\t}" ::"r"(su32(local_addr)),
-      "r"(rank), "f"(x), "f"(y)
-      : "memory");
-}
-// asynchronous 8-byte store into CTA `rank`'s copy of local_addr; its
-// completion is signalled as 8 transaction bytes on that CTA's copy of bar
-__device__ __forceinline__ void st_async_f2(const void* local_addr, const uint64_t* bar, uint32_t rank, float x,
-                                            float y) {
-  asm volatile(
-      "{\n\t.reg .b32 ra, rb;\n\t"
-      "mapa.shared::cluster.u32 ra, %0, %2;\n\t"
-      "mapa.shared::cluster.u32 rb, %1, %2;\n\t"
-      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [ra], {%3, %4}, [rb];\n\t}" ::"r"(
-          su32(local_addr)),
-      "r"(su32(bar)), "r"(rank), "f"(x), "f"(y)
-      : "memory");
-}
+// asynchronous 4-byte store into CTA `rank`'s copy of local_addr; its
+// completion is signalled as 4 transaction bytes on that CTA's copy of bar
 __device__ __forceinline__ void st_async_f32(const void* local_addr, const uint64_t* bar, uint32_t rank, float x) {
   asm volatile(
       "{\n\t.reg .b32 ra, rb;\n\t"
@@ -312,21 +290,8 @@ __device__ __forceinline__ uint32_t cluster_rank() {
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
   return r;
 }
-__device__ __forceinline__ uint32_t cluster_id_x() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ uint32_t nclusters_x() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
-  return r;
-}
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void named_bar_sync(int id, int count) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
 }  // namespace tc
