@@ -332,9 +332,16 @@ def run_ours(args, rank, world, local):
             same_as_first(c, "a graph replay")
             graphs.append(g)
 
-    # traced steps: a spread of the timed steps record per-kernel events (eager calls)
-    n_traced = max(1, min(args.steps // 5 if graphs is not None else args.steps, 400))
-    traced_at = set(np.linspace(0, args.steps - 1, n_traced).astype(int).tolist())
+    # traced steps record per-kernel events (eager calls). With one call in
+    # flight they are spread over the timed steps; with several, they are the
+    # last steps of the timed region, made one call at a time on one stream,
+    # so that a kernel's interval is its own and not shared with other calls
+    if inflight > 1:
+        n_traced = max(1, min(args.steps // 20, 100))
+        traced_at = set(range(args.steps - n_traced, args.steps))
+    else:
+        n_traced = max(1, min(args.steps // 5 if graphs is not None else args.steps, 400))
+        traced_at = set(np.linspace(0, args.steps - 1, n_traced).astype(int).tolist())
     events = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(n_traced)]
     for evs in events:
         for e in evs:
@@ -353,7 +360,16 @@ def run_ours(args, rank, world, local):
     for s_ in streams[1:]:
         s_.wait_event(t_start)
     ti = 0
+    joined = False
     for i in range(args.steps):
+        if inflight > 1 and i in traced_at:
+            if not joined:  # the in-flight steps end here; the traced ones follow on one stream
+                for s_ in streams:
+                    stream.wait_stream(s_)
+                joined = True
+            calls[0].traced(events[ti], stream)
+            ti += 1
+            continue
         j = i % inflight
         with torch.cuda.stream(streams[j]):
             if i in traced_at:
@@ -379,21 +395,6 @@ def run_ours(args, rank, world, local):
     per_kernel = {}
     for j, name in enumerate(occ.PruneCall.TRACE_NAMES):
         per_kernel[name] = float(np.mean([evs[j].elapsed_time(evs[j + 1]) for evs in events]))
-    # with several calls in flight the timed region's kernel intervals include
-    # sharing the GPU; the same kernels timed alone (one call at a time, after
-    # the timed region) are reported beside them
-    per_kernel_solo = None
-    if inflight > 1:
-        n_solo = 50
-        ev_solo = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(n_solo)]
-        for evs in ev_solo:
-            for e in evs:
-                e.record(stream)  # torch creates the CUDA event on its first record
-        for evs in ev_solo:
-            call.traced(evs)
-        torch.cuda.synchronize()
-        per_kernel_solo = {name: float(np.mean([evs[j].elapsed_time(evs[j + 1]) for evs in ev_solo]))
-                           for j, name in enumerate(occ.PruneCall.TRACE_NAMES)}
 
     ms_max, images = aggregate(ms, meta["B"] * args.steps, dev)
     value = images / (ms_max / 1e3)
@@ -552,11 +553,9 @@ def run_ours(args, rank, world, local):
                 "frac": achieved / peak, "traffic": traffic, "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
                 if peak_kind == "measured" else "fallback 6.8 TB/s",
                 "algorithmic_bytes_per_launch": bytes_[dom], "avg_launch_ms": per_kernel[dom]}
-    if per_kernel_solo is not None:
-        a_solo = bytes_[dom] / (per_kernel_solo[dom] / 1e3) / 1e9
-        roofline["timing"] = (f"avg_launch_ms over the timed region, where {inflight} calls share the GPU; "
-                              "`solo` times the same kernel with one call at a time")
-        roofline["solo"] = {"achieved": a_solo, "frac": a_solo / peak, "avg_launch_ms": per_kernel_solo[dom]}
+    roofline["timing"] = (f"avg_launch_ms from CUDA events around the kernel in {n_traced} of the {args.steps} "
+                          "timed steps" + (f", made one call at a time at the end of the timed region (the other "
+                                           f"steps keep {inflight} calls in flight)" if inflight > 1 else ""))
     step_ms = ms_max / args.steps
     step_gbs = bytes_["step"] / (step_ms / 1e3) / 1e9
     cpu = None
@@ -580,7 +579,8 @@ def run_ours(args, rank, world, local):
             "l2": "inputs larger than L2 (about 5 GB resident per step); no flush",
             "launch": (f"{inflight} occam_prune calls in flight on {inflight} streams, each with its own copy of "
                        "the inputs, workspace and outputs; a step replays one call's CUDA graph (every kernel of "
-                       f"the call); {n_traced} of the steps are eager calls recording per-kernel events")
+                       f"the call); the last {n_traced} steps are eager calls, one at a time, recording "
+                       "per-kernel events")
                       if graphs is not None else
                       f"{inflight} eager occam_prune calls in flight on {inflight} streams "
                       f"({n_traced} recording per-kernel events)",
@@ -593,7 +593,6 @@ def run_ours(args, rank, world, local):
             "step_frac_of_measured_hbm": step_gbs / peak,
             "step_frac_of_8TBps": step_gbs / SPEC_HBM_GBS,
             "per_kernel_ms": per_kernel,
-            "per_kernel_ms_solo": per_kernel_solo,
         },
         "roofline": roofline,
         "cpu_baseline": cpu,
