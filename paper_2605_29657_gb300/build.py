@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "liboccam.so")
-SOURCES = ["stage1.cu", "stage1_tc.cu", "stage2.cu", "stage2_tc.cu", "compact.cu", "rules.cu", "selftest.cu", "api.cu"]
+SOURCES = ["stage1.cu", "stage1_tc.cu", "stage2.cu", "stage2_tc.cu", "stage2_scores_tc.cu", "compact.cu", "rules.cu", "selftest.cu", "api.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

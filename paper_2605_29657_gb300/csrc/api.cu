@@ -148,7 +148,6 @@ void set_smem_attrs() {
     cudaFuncSetAttribute(stage1_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)finalize_smem_bytes(16 * kFinalizeSmemRows, false));
     cudaFuncSetAttribute(s2_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_stats_smem_bytes());
-    cudaFuncSetAttribute(s2_scores_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_scores_smem_bytes());
   });
 }
 
@@ -456,12 +455,23 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
 
 // Stage II for the samples the plan routed to the two-pass kernels; both
 // loop over their item lists, which may be empty.
-void launch_twopass(const Stage2Params& p, const WsLayout& L, int sms, cudaStream_t st) {
+int launch_twopass(const Stage2Params& p, const WsLayout& L, int sms, const occam_batch* b,
+                   const occam_stage2_args* a, cudaStream_t st) {
   const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);
   const int gB = (int)std::min<int64_t>(L.maxB, sms);
-  if (gA > 0) s2_stats_kernel<<<gA, 128, s2_stats_smem_bytes(), st>>>(p);
-  if (gB > 0) s2_scores_kernel<<<gB, 256, s2_scores_smem_bytes(), st>>>(p);
-  count_launch((gA > 0) + (gB > 0));
+  if (gA > 0) {
+    s2_stats_kernel<<<gA, 128, s2_stats_smem_bytes(), st>>>(p);
+    count_launch();
+  }
+  if (gB > 0) {
+    // the score pass on the tensor cores: S1 keys gathered from K2 by row
+    // (box one row high), the text queries in boxes of 64 rows
+    CUtensorMap mk, mq64;
+    if (!encode_map(&mk, a->K2, b->total_rows, (int64_t)kv_heads(a) * 128, 1)) return OCCAM_ERR_CUDA;
+    if (!encode_map(&mq64, a->Q_text, b->total_text, (int64_t)a->H2 * 128, kTextTile)) return OCCAM_ERR_CUDA;
+    if (launch_scores_tc(p, mq64, mk, gB, st) != 0) return OCCAM_ERR_CUDA;
+  }
+  return OCCAM_OK;
 }
 
 // Stage-II parameter block (the same for the plan, built by the Stage-I
@@ -568,7 +578,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     if (!only16 && launch_fused(8, mq, mk, mkt, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
     // the two-pass kernels (samples the fused kernel cannot hold; often none)
     // follow the 8-CTA launch on the second stream
-    launch_twopass(p, L, sms, side.stream);
+    OCCAM_TRY(launch_twopass(p, L, sms, b, a, side.stream));
     // samples too large for 8 CTAs: 16-CTA clusters, on this stream ahead of
     // the 4-CTA launch. A launch without items returns at once; it also
     // lets the 8-CTA clusters (larger items) take their SMs first, which
@@ -589,7 +599,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     trace.mark(st);
   } else {
     trace.mark(st);
-    launch_twopass(p, L, sms, st);
+    OCCAM_TRY(launch_twopass(p, L, sms, b, a, st));
   }
   trace.mark(st);
   return cuda_ok();

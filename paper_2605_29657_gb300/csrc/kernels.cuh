@@ -300,13 +300,13 @@ __global__ void threshold_kernel(ThresholdParams p);
 // stage2.cu
 
 __global__ void s2_stats_kernel(Stage2Params p);
-__global__ void s2_scores_kernel(Stage2Params p);
-int s2_scores_smem_bytes();
 int s2_stats_smem_bytes();
 
 // stage2_tc.cu
 int fused_resident_clusters(int C);
 void launch_s2_merge(const Stage2TcParams& q, cudaStream_t st);
+int launch_scores_tc(const Stage2Params& p, const CUtensorMap& mq64, const CUtensorMap& mk, int grid,
+                     cudaStream_t st);
 int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt, const Stage2TcParams& q,
                  int nclusters, cudaStream_t st);
 int s2_fused_smem_bytes(int C);

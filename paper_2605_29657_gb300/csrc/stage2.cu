@@ -11,15 +11,11 @@
 //          64-key chunks; a sample's keys are split into up to 16 ranges so
 //          that samples too large for the fused kernel still spread over
 //          the SMs;
-//   scores (item = sample, 64 text rows, 128 S1 keys): for every head the
-//          probabilities of the chunk's keys (the ranges' statistics merged
-//          on load), accumulated over heads in
-//          registers, then the column max over j (atomicMax on the fp32 bit
-//          pattern -- exact and order-free because p >= 0) and the
-//          registers' column sums (written per item and reduced in a fixed
-//          order by the sample's last item, so ref2 is deterministic).
-// QK^T runs on the tensor cores (mma.sync m16n8k16, bf16 in, fp32
-// accumulate); operands are staged in shared memory by cp.async.
+//   scores (item = sample, 64 text rows, 128 S1 keys): on the 5th-generation
+//          tensor cores, in stage2_scores_tc.cu.
+// The statistics pass runs QK^T on the tensor cores with mma.sync
+// m16n8k16 (bf16 in, fp32 accumulate); its operands are staged in shared
+// memory by cp.async.
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -189,160 +185,5 @@ __global__ void __launch_bounds__(128) s2_stats_kernel(Stage2Params p) {
 }
 
 int s2_stats_smem_bytes() { return (kTextTile + 2 * s2k::KT) * s2k::LD * 2; }
-
-// ---------------------------------------------------------------------------
-// pass 2: head-averaged probabilities of 128 S1 keys for 64 text rows
-// ---------------------------------------------------------------------------
-namespace s2s {
-constexpr int kQBytes = kTextTile * s2k::LD * 2;      // 17408
-constexpr int kKBytes = kKeyChunk * s2k::LD * 2;      // 34816
-constexpr int kMaxH = 64;
-constexpr int kSmem = 2 * kQBytes + 2 * kKBytes + kTextTile * kMaxH * 8 + 2 * 4 * kKeyChunk * 4 +
-                      kKeyChunk * 8 + 64;
-}  // namespace s2s
-
-int s2_scores_smem_bytes() { return s2s::kSmem; }
-
-__global__ void __launch_bounds__(256, 1) s2_scores_kernel(Stage2Params p) {
-  using namespace s2k;
-  using namespace s2s;
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem_raw);                       // [2][64][LD]
-  __nv_bfloat16* sK = reinterpret_cast<__nv_bfloat16*>(smem_raw + 2 * kQBytes);         // [2][128][LD]
-  float2* sst = reinterpret_cast<float2*>(smem_raw + 2 * kQBytes + 2 * kKBytes);        // [64][H]
-  float* cmax = reinterpret_cast<float*>(sst + kTextTile * kMaxH);                      // [4][128]
-  float* csum = cmax + 4 * kKeyChunk;                                                   // [4][128]
-  int* krow = reinterpret_cast<int*>(csum + 4 * kKeyChunk);                             // [128]
-  int* kreg = krow + kKeyChunk;                                                         // [128]
-  __shared__ float red[kKeyChunk];
-  __shared__ int last_flag;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int rb = warp & 3, kh = warp >> 2;
-  const int nB = p.counters[CNT_NB];
-  const float c = p.scale * 1.4426950408889634f;
-  const float invH = 1.0f / (float)p.H;
-  for (int it = blockIdx.x; it < nB; it += gridDim.x) {
-    const int b = item_sample(p.itemB_off, p.bt.B, it);
-    const int64_t t0 = p.bt.text_off[b];
-    const int M = (int)(p.bt.text_off[b + 1] - t0);
-    const int n_img = p.n1[b];
-    const int nch = (n_img + kKeyChunk - 1) / kKeyChunk;
-    const int i = it - p.itemB_off[b];
-    const int j0 = (i / nch) * kTextTile, kc = i % nch, slot = p.slot_off[b] + i;
-    const int nq = min(kTextTile, M - j0);
-    const int k0 = kc * kKeyChunk;
-    const int nk = min(kKeyChunk, n_img - k0);
-    const int64_t rbase = p.bt.row_off[b];
-    // merge the key ranges' partial statistics: max, then the sums rescaled to it
-    const int nsp = s2_stat_splits(n_img, M);
-    for (int i = tid; i < kTextTile * p.H; i += 256) {
-      const int r = i / p.H, h = i - r * p.H;
-      float2 st = make_float2(0.f, 0.f);
-      if (r < nq) {
-        const float2* ps = p.stats + ((t0 + j0 + r) * p.H + h) * kStatSplits;
-        float mx = -INFINITY;
-        for (int s = 0; s < nsp; ++s) mx = fmaxf(mx, ps[s].x);
-        float z = 0.f;
-        for (int s = 0; s < nsp; ++s)
-          if (ps[s].x != -INFINITY) z += ps[s].y * exp2f(ps[s].x - mx);
-        st = make_float2(mx, 1.0f / z);
-      }
-      sst[r * p.H + h] = st;
-    }
-    for (int i = tid; i < kKeyChunk; i += 256) {
-      const int row = (i < nk) ? p.dense[rbase + k0 + i] : -1;
-      krow[i] = row;
-      kreg[i] = (row >= 0) ? (int)p.role[row] : 0;
-    }
-    // operands of head 0
-    s2_load_queries(sQ, p, t0 + j0, nq, 0, tid, 256);
-    s2_load_keys(sK, p, b, t0, n_img, n_img, k0, kKeyChunk, 0, tid, 256);
-    cp_async_commit();
-    float P[8][4];
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) P[nt][0] = P[nt][1] = P[nt][2] = P[nt][3] = 0.f;
-    const int rowA = rb * 16 + (lane >> 2), rowB = rowA + 8;
-    const bool vA = rowA < nq, vB = rowB < nq;
-    for (int h = 0; h < p.H; ++h) {
-      const int buf = h & 1;
-      if (h + 1 < p.H) {
-        s2_load_queries(sQ + (buf ^ 1) * kTextTile * LD, p, t0 + j0, nq, h + 1, tid, 256);
-        s2_load_keys(sK + (buf ^ 1) * kKeyChunk * LD, p, b, t0, n_img, n_img, k0, kKeyChunk, h + 1, tid, 256);
-      }
-      cp_async_commit();
-      cp_async_wait<1>();
-      __syncthreads();
-      float S[8][4];
-      warp_qk128<8>(S, sQ + buf * kTextTile * LD, rb * 16, sK + buf * kKeyChunk * LD, kh * 64, lane);
-      const float2 sa = sst[rowA * p.H + h], sb = sst[rowB * p.H + h];
-#pragma unroll
-      for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          if (vA) P[nt][e] += exp2f(fmaf(S[nt][e], c, -sa.x)) * sa.y;
-          if (vB) P[nt][2 + e] += exp2f(fmaf(S[nt][2 + e], c, -sb.x)) * sb.y;
-        }
-      __syncthreads();
-    }
-    // column max / sum over this item's text rows
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        float mx = fmaxf(vA ? P[nt][e] : 0.f, vB ? P[nt][2 + e] : 0.f);
-        float sm = (vA ? P[nt][e] : 0.f) + (vB ? P[nt][2 + e] : 0.f);
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-        sm += __shfl_xor_sync(0xffffffffu, sm, 4);
-        sm += __shfl_xor_sync(0xffffffffu, sm, 8);
-        sm += __shfl_xor_sync(0xffffffffu, sm, 16);
-        if ((lane >> 2) == 0) {
-          const int col = kh * 64 + nt * 8 + (lane & 3) * 2 + e;
-          cmax[rb * kKeyChunk + col] = mx;
-          csum[rb * kKeyChunk + col] = sm;
-        }
-      }
-    __syncthreads();
-    if (tid < kKeyChunk) {
-      float rs = 0.f;
-      if (tid < nk) {
-        const float mx = fmaxf(fmaxf(cmax[tid], cmax[kKeyChunk + tid]),
-                               fmaxf(cmax[2 * kKeyChunk + tid], cmax[3 * kKeyChunk + tid])) * invH;
-        if (kreg[tid]) {
-          rs = ((csum[tid] + csum[kKeyChunk + tid]) + (csum[2 * kKeyChunk + tid] + csum[3 * kKeyChunk + tid])) * invH;
-        } else {
-          atomicMax(reinterpret_cast<int*>(&p.s2[krow[tid]]), __float_as_int(mx));
-        }
-      }
-      red[tid] = rs;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      float acc = 0.f;
-      for (int i = 0; i < kKeyChunk; ++i) acc += red[i];
-      p.refpart[slot] = acc;
-      __threadfence();
-      const int nslots = p.slot_off[b + 1] - p.slot_off[b];
-      last_flag = (atomicAdd(&p.done[b], 1) == nslots - 1);
-    }
-    __syncthreads();
-    if (last_flag && tid < 32) {
-      // the sample's last partial: lane l sums slots l, l + 32, ... in order,
-      // then a fixed tree over the lanes (deterministic)
-      __threadfence();
-      float acc = 0.f;
-      for (int i = p.slot_off[b] + tid; i < p.slot_off[b + 1]; i += 32) acc += __ldcg(&p.refpart[i]);
-      acc = warp_sum(acc);
-      if (tid == 0) {
-        const int R = p.bt.reg_off[p.bt.seg_first[b + 1]] - p.bt.reg_off[p.bt.seg_first[b]];
-        const float r2 = (R > 0 && M > 0) ? acc / ((float)R * (float)M) : 0.f;
-        p.ref2[b] = r2;
-        p.tau2[b] = p.lambda2 * r2;
-      }
-    }
-    __syncthreads();
-  }
-}
 
 }  // namespace occam
