@@ -41,7 +41,8 @@ FALLBACK_HBM_GBS = 6800.0
 SPEC_HBM_GBS = 8000.0
 KERNEL_SOURCES = {
     "stage1": "stage1.cu", "stage1_finalize": "stage1.cu", "s1_list_plan": "stage2.cu",
-    "stage2_fused": "stage2_tc.cu", "stage2_twopass": "stage2.cu", "scan": "compact.cu", "gather": "compact.cu",
+    "stage2_fused": "stage2_tc.cu", "stage2_twopass": ("stage2.cu", "stage2_scores_tc.cu"), "scan": "compact.cu",
+    "gather": "compact.cu",
 }
 
 
@@ -136,8 +137,12 @@ def _traffic_from_profiles(kernel: str):
             vals[k.strip()] = v.strip()
     if "dram_bytes_per_launch" not in vals or "source_sha" not in vals:
         return None
-    src = os.path.join(ROOT, "paper_2605_29657_gb300", "csrc", KERNEL_SOURCES[kernel])
-    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    files = KERNEL_SOURCES[kernel]
+    files = (files,) if isinstance(files, str) else files
+    h = hashlib.sha256()
+    for f in files:  # a kernel built from several sources hashes their concatenation
+        h.update(open(os.path.join(ROOT, "paper_2605_29657_gb300", "csrc", f), "rb").read())
+    sha = h.hexdigest()[:16]
     if sha != vals["source_sha"]:
         return None
     return float(vals["dram_bytes_per_launch"])
