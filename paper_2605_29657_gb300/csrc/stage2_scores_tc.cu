@@ -138,17 +138,29 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
     }
     // the statistics pass's partials of every key range, merged: max, then
     // the sums rescaled to it
+    // An entry's kStatSplits slots are 128 contiguous, 128-byte aligned
+    // bytes: all are loaded at once (independent 16-byte loads, one L2 round
+    // trip), slots past the sample's nsp ranges taken as empty.
     const int nsp = s2_stat_splits(n_img, M);
     for (int i = tid; i < TR * H; i += THREADS) {
       const int r = i / H, h = i - r * H;
       float2 st = make_float2(INFINITY, 0.f);
       if (r < nq) {
-        const float2* ps = p.stats + ((t0 + j0 + r) * H + h) * kStatSplits;
+        const float4* ps = reinterpret_cast<const float4*>(p.stats + ((t0 + j0 + r) * H + h) * kStatSplits);
+        float2 v[kStatSplits];
+#pragma unroll
+        for (int q = 0; q < kStatSplits / 2; ++q) {
+          const float4 w = 2 * q < nsp ? __ldcg(ps + q) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+          v[2 * q] = make_float2(w.x, w.y);
+          v[2 * q + 1] = 2 * q + 1 < nsp ? make_float2(w.z, w.w) : make_float2(-INFINITY, 0.f);
+        }
         float mx = -INFINITY;
-        for (int s = 0; s < nsp; ++s) mx = fmaxf(mx, ps[s].x);
+#pragma unroll
+        for (int s = 0; s < kStatSplits; ++s) mx = fmaxf(mx, v[s].x);
         float z = 0.f;
-        for (int s = 0; s < nsp; ++s)
-          if (ps[s].x != -INFINITY) z += ps[s].y * exp2f(ps[s].x - mx);
+#pragma unroll
+        for (int s = 0; s < kStatSplits; ++s)
+          if (v[s].x != -INFINITY) z += v[s].y * exp2f(v[s].x - mx);
         st = make_float2(mx, 1.0f / z);
       }
       sm.sst[r][h] = st;
