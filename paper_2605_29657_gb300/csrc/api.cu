@@ -464,12 +464,11 @@ int launch_twopass(const Stage2Params& p, const WsLayout& L, int sms, const occa
     count_launch();
   }
   if (gB > 0) {
-    // the score pass on the tensor cores: S1 keys gathered from K2 by row
-    // (box one row high), the text queries in boxes of 64 rows
-    CUtensorMap mk, mq64;
-    if (!encode_map(&mk, a->K2, b->total_rows, (int64_t)kv_heads(a) * 128, 1)) return OCCAM_ERR_CUDA;
+    // the score pass on the tensor cores: S1 keys copied from K2 by row
+    // (cp.async), the text queries in TMA boxes of 64 rows
+    CUtensorMap mq64;
     if (!encode_map(&mq64, a->Q_text, b->total_text, (int64_t)a->H2 * 128, kTextTile)) return OCCAM_ERR_CUDA;
-    if (launch_scores_tc(p, mq64, mk, gB, st) != 0) return OCCAM_ERR_CUDA;
+    if (launch_scores_tc(p, mq64, gB, st) != 0) return OCCAM_ERR_CUDA;
   }
   return OCCAM_OK;
 }

@@ -305,8 +305,8 @@ int s2_stats_smem_bytes();
 // stage2_tc.cu
 int fused_resident_clusters(int C);
 void launch_s2_merge(const Stage2TcParams& q, cudaStream_t st);
-int launch_scores_tc(const Stage2Params& p, const CUtensorMap& mq64, const CUtensorMap& mk, int grid,
-                     cudaStream_t st);
+// stage2_scores_tc.cu
+int launch_scores_tc(const Stage2Params& p, const CUtensorMap& mq64, int grid, cudaStream_t st);
 int launch_fused(int C, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mkt, const Stage2TcParams& q,
                  int nclusters, cudaStream_t st);
 int s2_fused_smem_bytes(int C);

@@ -13,14 +13,20 @@
 // sample's last slot writer reduces the slots in order into ref2 and tau2).
 //
 // Per head: the 128 keys are the MMA's A operand (one per TMEM lane, fetched
-// from K2 through the S1 list by TMA tile::gather4, four rows a copy), the
-// 64 text queries its B operand (one TMA box per 64-dim K-block), and
-// D = K Q^T (128 x 64 fp32) lands in one of two TMEM buffers.
-// Roles (384 threads): warp 0 issues the TMA copies, warp 1 the MMAs, warps
-// 4-11 (two per TMEM lane quadrant, 32 text rows each) add each head into
-// register accumulators. Operand stages and accumulators are double
-// buffered. Every wait is bounded; on a timeout the CTA records
-// OCCAM_ERR_TIMEOUT, lets its copies land, frees TMEM and returns.
+// from K2 through the S1 list by 16-byte cp.async copies into the 128-byte
+// swizzled K-major layout), the 64 text queries its B operand (one TMA box
+// per 64-dim K-block), and D = K Q^T (128 x 64 fp32) lands in one of two
+// TMEM buffers. The key rows are scattered: per-copy TMA gathers (four rows
+// a copy) left this pass bound by the copy rate, while 96 threads' cp.async
+// keep two heads' key tiles in flight.
+// Roles (384 threads): warps 0, 2 and 3 load the keys (warp 0 also issues
+// the query TMA boxes), warp 1 issues the MMAs, warps 4-11 (two per TMEM
+// lane quadrant, 32 text rows each) add each head into register
+// accumulators. Operands have three stages, accumulators two. A loader
+// signals a stage once its own copies landed and, through a proxy fence,
+// are visible to the tensor cores. Every wait is bounded; on a timeout the
+// CTA records OCCAM_ERR_TIMEOUT, lets its copies land, frees TMEM and
+// returns.
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc5.cuh"
@@ -32,7 +38,8 @@ constexpr int KR = 128;                   // keys per item (MMA M, TMEM lanes)
 constexpr int TR = kTextTile;             // text rows per item (MMA N)
 constexpr int ABYTES = KR * 128;          // one 64-dim K-block of the key tile
 constexpr int BBYTES = TR * 128;          // one 64-dim K-block of the query tile
-constexpr int NST = 2;                    // operand stages
+constexpr int NST = 3;                    // operand stages
+constexpr int NLOAD = 96;                 // key loader threads (warps 0, 2, 3)
 constexpr int EPI0 = 4;                   // first softmax warp
 constexpr int NEPI = 8;
 constexpr int THREADS = (EPI0 + NEPI) * 32;
@@ -84,8 +91,7 @@ __device__ __forceinline__ void ld_wait32(uint32_t (&v)[32]) {
 }  // namespace
 
 __global__ void __launch_bounds__(s2t::THREADS, 1)
-    s2_scores_tc_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
-                        Stage2Params p) {
+    s2_scores_tc_kernel(const __grid_constant__ CUtensorMap mapQ, Stage2Params p) {
   using namespace s2t;
   extern __shared__ unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -100,7 +106,7 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
 
   if (tid == 0) {
     for (int i = 0; i < NST; ++i) {
-      tc::bar_init(&sm.full[i], 1);
+      tc::bar_init(&sm.full[i], NLOAD + 1);  // every loader, plus the query boxes' expect_tx
       tc::bar_init(&sm.empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -110,7 +116,6 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
     sm.abort = 0;
     tc::bar_fence_init();
     tc::prefetch_map(&mapQ);
-    tc::prefetch_map(&mapK);
   }
   if (warp == 1) tc::tmem_alloc(&sm.tmem_base, 2 * TR);
   tc::fence_before();
@@ -170,11 +175,15 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
     tc::fence_after();
     if (*abort) break;  // uniform: read after the barrier
 
-    if (warp == 0) {
-      // ---------------------------------------------------------- TMA producer
-      // per head: 2 x 32 gather4 copies of the key tile (lane l: units l and
-      // l + 32; unit u = rows 4 (u >> 1) .. + 3 of K-block u & 1), then the
-      // query tile's two K-blocks (lane 0)
+    if (warp == 0 || warp == 2 || warp == 3) {
+      // ---------------------------------------------------------- loaders
+      // per head: the key tile's 2 x 128 rows of 128 bytes as 2,048 16-byte
+      // copies, copy i = (key i >> 4, K-block (i >> 3) & 1, chunk i & 7),
+      // written where the 128-byte swizzle puts it (chunk ^ (row & 7)); then
+      // stage g - 1 is signalled once this thread's copies for it landed.
+      // Lane 0 of warp 0 also issues the query tile's two TMA boxes.
+      const int lt = (warp == 0 ? 0 : warp - 1) * 32 + lane;
+      const int64_t HD = (int64_t)p.Hkv * 128;
       bool ok = true;
       for (int h = 0; h < H && ok; ++h) {
         const uint32_t g = sg + h, s = g % NST;
@@ -182,20 +191,27 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
           ok = false;
           break;
         }
-        if (lane == 0) tc::bar_expect_tx(&sm.full[s], 2 * ABYTES + 2 * BBYTES);
-        __syncwarp();
-        const int hk = h / kv_group;
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-          const int u = lane + 32 * k;
-          const int r0 = (u >> 1) * 4, kb = u & 1;
-          tc::tma_gather4(sm.a[s][kb] + r0 * 128, &mapK, hk * 128 + kb * 64, sm.kidx[r0], sm.kidx[r0 + 1],
-                          sm.kidx[r0 + 2], sm.kidx[r0 + 3], &sm.full[s]);
-        }
-        if (lane == 0) {
+        if (warp == 0 && lane == 0) {
+          tc::bar_expect_tx(&sm.full[s], 2 * BBYTES);
           tc::tma_load_2d(sm.b[s][0], &mapQ, h * 128, (int)(t0 + j0), &sm.full[s]);
           tc::tma_load_2d(sm.b[s][1], &mapQ, h * 128 + 64, (int)(t0 + j0), &sm.full[s]);
         }
+        const __nv_bfloat16* kh = p.K + (int64_t)(h / kv_group) * 128;
+        for (int i = lt; i < 2 * KR * 8; i += NLOAD) {
+          const int r = i >> 4, kb = (i >> 3) & 1, ch = i & 7;
+          tc::cp_async16(sm.a[s][kb] + r * 128 + ((ch ^ (r & 7)) << 4), kh + sm.kidx[r] * HD + kb * 64 + ch * 8, 16);
+        }
+        cp_async_commit();
+        if (h > 0) {
+          cp_async_wait<1>();
+          tc::fence_proxy_async();
+          tc::bar_arrive(&sm.full[(g - 1) % NST]);
+        }
+      }
+      cp_async_wait<0>();  // on a timeout too: no copy may land after the CTA ends
+      if (ok) {
+        tc::fence_proxy_async();
+        tc::bar_arrive(&sm.full[(sg + H - 1) % NST]);
       }
       if (!ok && lane == 0) {
         sm.abort = 1;
@@ -211,6 +227,7 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
           ok = tc::bar_wait(&sm.full[s], (g / NST) & 1, abort, kLimitNs);
           if (ok && g >= 2) ok = tc::bar_wait(&sm.dfree[db], ((g - 2) >> 1) & 1, abort, kLimitNs);
           if (!ok) break;
+          tc::fence_proxy_async();
           tc::fence_after();
 #pragma unroll
           for (int kb = 0; kb < 2; ++kb)
@@ -325,11 +342,10 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
   if (warp == 1) tc::tmem_dealloc(tmem, 2 * TR);
 }
 
-int launch_scores_tc(const Stage2Params& p, const CUtensorMap& mq64, const CUtensorMap& mk, int grid,
-                     cudaStream_t st) {
+int launch_scores_tc(const Stage2Params& p, const CUtensorMap& mq64, int grid, cudaStream_t st) {
   const int smem = s2_scores_tc_smem_bytes();
   cudaFuncSetAttribute(s2_scores_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  s2_scores_tc_kernel<<<grid, s2t::THREADS, smem, st>>>(mq64, mk, p);
+  s2_scores_tc_kernel<<<grid, s2t::THREADS, smem, st>>>(mq64, p);
   count_launch();
   return cudaGetLastError() == cudaSuccess ? 0 : 1;
 }
