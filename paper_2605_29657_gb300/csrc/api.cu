@@ -147,7 +147,6 @@ void set_smem_attrs() {
                          stage1_logits_smem_bytes());
     cudaFuncSetAttribute(stage1_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)finalize_smem_bytes(16 * kFinalizeSmemRows, false));
-    cudaFuncSetAttribute(s2_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_stats_smem_bytes());
   });
 }
 
@@ -457,19 +456,15 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
 // loop over their item lists, which may be empty.
 int launch_twopass(const Stage2Params& p, const WsLayout& L, int sms, const occam_batch* b,
                    const occam_stage2_args* a, cudaStream_t st) {
-  const int gA = (int)std::min<int64_t>(L.maxA, 4 * sms);
+  const int gA = (int)std::min<int64_t>(L.maxA, sms);
   const int gB = (int)std::min<int64_t>(L.maxB, sms);
-  if (gA > 0) {
-    s2_stats_kernel<<<gA, 128, s2_stats_smem_bytes(), st>>>(p);
-    count_launch();
-  }
-  if (gB > 0) {
-    // the score pass on the tensor cores: S1 keys copied from K2 by row
-    // (cp.async), the text queries in TMA boxes of 64 rows
-    CUtensorMap mq64;
-    if (!encode_map(&mq64, a->Q_text, b->total_text, (int64_t)a->H2 * 128, kTextTile)) return OCCAM_ERR_CUDA;
-    if (launch_scores_tc(p, mq64, gB, st) != 0) return OCCAM_ERR_CUDA;
-  }
+  if (gA <= 0 && gB <= 0) return OCCAM_OK;
+  // both passes on the tensor cores: keys copied from K2 (and the text keys)
+  // by row with cp.async, the text queries in TMA boxes of 64 rows
+  CUtensorMap mq64;
+  if (!encode_map(&mq64, a->Q_text, b->total_text, (int64_t)a->H2 * 128, kTextTile)) return OCCAM_ERR_CUDA;
+  if (gA > 0 && launch_stats_tc(p, mq64, gA, st) != 0) return OCCAM_ERR_CUDA;
+  if (gB > 0 && launch_scores_tc(p, mq64, gB, st) != 0) return OCCAM_ERR_CUDA;
   return OCCAM_OK;
 }
 

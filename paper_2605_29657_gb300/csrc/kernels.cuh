@@ -299,8 +299,8 @@ __global__ void threshold_kernel(ThresholdParams p);
 
 // stage2.cu
 
-__global__ void s2_stats_kernel(Stage2Params p);
 int s2_stats_smem_bytes();
+int launch_stats_tc(const Stage2Params& p, const CUtensorMap& mq64, int grid, cudaStream_t st);
 
 // stage2_tc.cu
 int fused_resident_clusters(int C);

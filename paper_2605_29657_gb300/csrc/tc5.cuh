@@ -96,8 +96,7 @@ __device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }
 
-// cp.async (16 bytes, zero-filled when src_bytes == 0) and an mbarrier
-// arrival that fires once all of this thread's prior cp.async copies landed
+// cp.async of 16 bytes; copies src_bytes (0 or 16) and zero-fills the rest
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(dst)), "l"(src), "r"(src_bytes)
                : "memory");
