@@ -154,13 +154,6 @@ int occam_threshold(const occam_batch* batch, const float* s, const float* ref, 
                     float lambda, const uint8_t* prev_keep, int32_t keep_registers, uint8_t* keep,
                     int32_t* count_vis, void* workspace, size_t workspace_bytes, occam_stream_t stream);
 
-/* Stage-II scores (Sec. 3.5, Eq. 7; App. A, Eqs. 15-16). keep1 [total_rows]
- * u8 marks the visual rows of S1 (register rows are always in S1). For
- * sample b and text token j, per head, the softmax runs over the S1 rows of
- * b and the text keys 0..j (causal); the per-head probabilities are averaged
- * over heads. s2 [total_rows] fp32 = max over j for visual S1 rows, 0 for
- * every other row; ref2 [B] fp32 = the mean over the sample's registers of
- * the mean over j. */
 /* Mean-threshold reference (component ablation, "Mean threshold"). ref[u]
  * = the mean of s over the candidate rows of unit u: an fp64 sum in a fixed
  * order, divided by the count and rounded to fp32; 0 for a unit without
@@ -195,6 +188,13 @@ int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* p
 int occam_pool_scores(const float* s_in, int64_t rows_in, int32_t group, int32_t mode, float* s_out,
                       occam_stream_t stream);
 
+/* Stage-II scores (Sec. 3.5, Eq. 7; App. A, Eqs. 15-16). keep1 [total_rows]
+ * u8 marks the visual rows of S1 (register rows are always in S1). For
+ * sample b and text token j, per head, the softmax runs over the S1 rows of
+ * b and the text keys 0..j (causal); the per-head probabilities are averaged
+ * over heads. s2 [total_rows] fp32 = max over j for visual S1 rows, 0 for
+ * every other row; ref2 [B] fp32 = the mean over the sample's registers of
+ * the mean over j. */
 int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, const uint8_t* keep1,
                        float* s2, float* ref2, void* workspace, size_t workspace_bytes,
                        occam_stream_t stream);
@@ -232,9 +232,11 @@ int occam_construct_registers(const occam_batch* batch, void* h, int64_t channel
  * count at lambda2 is the number of visual S1 rows v (keep1[v] != 0, not a
  * register) with s2[v] >= lambda2 * ref2[b(v)], so it steps down at each
  * ratio s2[v] / ref2[b(v)]. lambda2_out (device, one fp32) receives the
- * target_count-th largest such ratio, computed as an IEEE fp32 quotient:
- * the largest lambda2 under which the ratio test keeps at least
- * target_count rows (exactly target_count when the ratios are distinct).
+ * largest fp32 lambda2 under which the test as this library applies it,
+ * s2[v] >= fl(lambda2 * ref2[b(v)]) in fp32, keeps at least target_count
+ * rows: the target_count-th largest IEEE fp32 quotient s2 / ref2, moved by
+ * single fp32 steps where the product's rounding disagrees with the
+ * quotient's. Just above it the test keeps fewer rows.
  * target_count = K_tar * |D| in total over the batch's samples. Samples with
  * ref2 <= 0 contribute no candidates. target_count <= 0 gives +inf; a
  * target above the candidate count gives 0 (keep all). n_candidates (device
@@ -362,22 +364,26 @@ int occam_prune_traced(const occam_prune_args* args, const occam_prune_out* out,
  * library routine. Limits and behaviour:
  * - total_rows <= 16,777,216 (8,192 scan tiles of 2,048 rows); larger batches
  *   are rejected with OCCAM_ERR_UNSUPPORTED and nothing is launched.
- * - The first call on a device, made with that device current, looks up the
- *   array's device address (cudaGetSymbolAddress) and caches it; make that
- *   first call before any stream capture.
+ * - The first call in a CUDA context (normally a device's primary context),
+ *   made with that device current, looks up the array's device address
+ *   (cudaGetSymbolAddress) and caches it under the context's unique id; make
+ *   that first call before any stream capture. A context created later on
+ *   the same device (after cudaDeviceReset, say) gets a fresh lookup.
+ * - Arguments are checked exactly as occam_compact checks them.
  * - All calls on a device share the one array. Each call clears the parts it
  *   needs before use, but calls that overlap on the GPU (different streams
  *   without ordering, or different host threads) race on it and produce
  *   wrong results: order them.
  * - Device-side errors are not reported (there is no workspace status word to
  *   read): a capacity overflow shows as out_off[B] > capacity_rows, with
- *   counts and offsets still exact. */
+ *   counts and offsets still exact. The scan's bounded look-back wait, a
+ *   guard against a fault that correct operation never reaches, is not
+ *   reported either: if it ran out, the outputs would be undefined. */
 int occam_compact_noalloc(const occam_batch* batch, const uint8_t* keep, int32_t n_tensors,
                           const void* const* src, const int64_t* row_bytes, void* const* dst,
                           int64_t capacity_rows, int32_t* out_index, int32_t* count_out, int64_t* out_off,
                           occam_stream_t stream);
 
-/* Library version string (static storage). */
 /* Diagnostic of the bounded device-side waits (no fault, trap or hang). One
  * warp waits, each time for about limit_ns (1 .. 1e9), on an mbarrier that
  * nothing completes (the tensor-core kernels' timer-bounded wait and the
@@ -394,7 +400,23 @@ int occam_selftest_wait(uint64_t limit_ns, int32_t* scratch, occam_stream_t stre
  * device still counts. */
 int occam_last_call_kernels(void);
 
+/* Library version string (static storage). */
 const char* occam_version(void);
+
+/* Stage-II routing, for tests and diagnostics only (the paper has no
+ * counterpart). OCCAM_ROUTE_AUTO (the default, and what a deployment uses):
+ * each sample takes the fused tensor-core kernel where its S1 fits, small
+ * batches on wider clusters; OCCAM_ROUTE_TWOPASS: every sample takes the
+ * two-pass kernels; OCCAM_ROUTE_NARROW: AUTO without the wider clusters.
+ * Results agree across routes within the scores' tolerance; the switch lets
+ * tests reach every path on the same inputs. Process-wide; it applies to
+ * calls made after it returns. previous (host, nullable) receives the route
+ * in force before the call. An unknown route returns OCCAM_ERR_INVALID_ARG
+ * and changes nothing. */
+#define OCCAM_ROUTE_AUTO 0
+#define OCCAM_ROUTE_TWOPASS 1
+#define OCCAM_ROUTE_NARROW 2
+int occam_set_stage2_route(int32_t route, int32_t* previous);
 
 #ifdef __cplusplus
 }

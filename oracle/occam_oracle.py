@@ -252,12 +252,15 @@ def lambda2_for_budget(s2, ref2, keep1, is_reg, row_off, target_count: int):
     |S2(lambda2)| counts the visual S1 rows v with s2(v) >= lambda2 s2(r) of
     their sample, so the total over D drops by one at each ratio
     s2(v) / s2(r). The lambda2 whose total is K = target_count
-    (= K_tar |D|) is therefore the K-th largest ratio: at it the ratio test
-    keeps at least K rows, just above it fewer. The ratios are taken as fp32
-    quotients of the fp32 scores (the precision in which the scores are
-    given), and the K-th largest comes from a sort. Samples whose reference
-    is not positive contribute no candidates. K <= 0 gives +inf; K above the
-    candidate count gives 0 (keep all).
+    (= K_tar |D|) is therefore the K-th largest ratio. The scores are fp32,
+    and the rule applies lambda2 as one fp32 product (s2(v) >= fl(lambda2
+    s2(r))), so lambda2* is taken as the largest fp32 value under which that
+    product test keeps at least K rows: the K-th largest fp32 quotient
+    s2(v) / s2(r) (from a sort), moved by single fp32 steps while the
+    product's rounding disagrees with the quotient's (a few ulps at most).
+    Just above lambda2* the test keeps fewer than K rows. Samples whose
+    reference is not positive contribute no candidates. K <= 0 gives +inf;
+    K above the candidate count gives 0 (keep all).
     """
     s2 = np.asarray(s2, dtype=np.float32)
     ref2 = np.asarray(ref2, dtype=np.float32)
@@ -265,12 +268,25 @@ def lambda2_for_budget(s2, ref2, keep1, is_reg, row_off, target_count: int):
     cand = np.asarray(keep1, dtype=bool) & ~np.asarray(is_reg, dtype=bool)
     sample = np.repeat(np.arange(len(row_off) - 1), np.diff(row_off))
     cand &= ref2[sample] > 0
-    ratios = np.sort(s2[cand] / ref2[sample][cand])[::-1]  # float32 / float32: IEEE quotient
+    s2c, refc = s2[cand], ref2[sample][cand]
+    ratios = np.sort(s2c / refc)[::-1]  # float32 / float32: IEEE quotient
     if target_count <= 0:
         return np.float32(np.inf), int(cand.sum())
     if target_count > len(ratios):
         return np.float32(0.0), int(cand.sum())
-    return np.float32(ratios[target_count - 1]), int(cand.sum())
+
+    def kept(lam):  # the product test in fp32: s2 >= fl(lam * ref)
+        return int(np.sum(s2c >= np.float32(lam) * refc))
+
+    lam = np.float32(ratios[target_count - 1])
+    while kept(lam) < target_count:  # kept(0) counts every candidate (s2 >= 0)
+        lam = np.nextafter(lam, np.float32(0.0))
+    while True:                      # kept(+inf) is 0
+        up = np.nextafter(lam, np.float32(np.inf))
+        if kept(up) < target_count:
+            break
+        lam = up
+    return np.float32(lam), int(cand.sum())
 
 
 def mean_reference(s, unit_off, cand):

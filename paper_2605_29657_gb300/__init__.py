@@ -10,6 +10,9 @@ kept rows -- all in the CUDA kernels of liboccam.so, reached through its C ABI
 from ._lib import (  # noqa: F401
     OCCAM_REF_SAMPLE,
     OCCAM_REF_SEGMENT,
+    OCCAM_ROUTE_AUTO,
+    OCCAM_ROUTE_NARROW,
+    OCCAM_ROUTE_TWOPASS,
     OCCAM_RULE_BUDGET,
     OCCAM_RULE_MEAN,
     OCCAM_RULE_REGISTER,
@@ -30,6 +33,7 @@ from ._lib import (  # noqa: F401
     occam_mean_reference,
     occam_pool_scores,
     occam_selftest_wait,
+    occam_set_stage2_route,
     occam_prune,
     occam_score_stage1,
     occam_score_stage2,

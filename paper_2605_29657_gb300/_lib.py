@@ -31,6 +31,7 @@ OCCAM_STAGE1_CLS = 0
 OCCAM_STAGE1_MUTUAL = 1
 OCCAM_REF_SEGMENT = 0
 OCCAM_REF_SAMPLE = 1
+OCCAM_ROUTE_AUTO, OCCAM_ROUTE_TWOPASS, OCCAM_ROUTE_NARROW = 0, 1, 2
 OCCAM_MAX_GATHER = 8
 OCCAM_RULE_REGISTER = 0
 OCCAM_RULE_MEAN = 1
@@ -116,10 +117,11 @@ def library() -> ctypes.CDLL:
         lib.occam_pool_scores.argtypes = [_p, _i64, _i32, _i32, _p, _p]
         lib.occam_selftest_wait.argtypes = [ctypes.c_uint64, _p, _p]
         lib.occam_last_call_kernels.argtypes = []
+        lib.occam_set_stage2_route.argtypes = [_i32, P(_i32)]
         for name in ("occam_last_call_kernels", "occam_selftest_wait", "occam_pool_scores", "occam_mean_reference", "occam_budget_keep", "occam_construct_registers", "occam_calibrate_lambda2", "occam_workspace_size", "occam_get_status", "occam_score_stage1",
                      "occam_threshold",
                      "occam_score_stage2", "occam_compact", "occam_prune", "occam_prune_traced",
-                     "occam_compact_noalloc", "occam_prune_staged"):
+                     "occam_compact_noalloc", "occam_prune_staged", "occam_set_stage2_route"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -297,6 +299,14 @@ def occam_mean_reference(layout: BatchLayout, s, ref_scope: int, prev_keep=None,
 def occam_last_call_kernels() -> int:
     """Kernels the last entry point called on this thread launched."""
     return int(library().occam_last_call_kernels())
+
+
+def occam_set_stage2_route(route: int) -> int:
+    """Stage-II routing for tests and diagnostics (OCCAM_ROUTE_AUTO is the
+    default). Returns the route in force before the call."""
+    prev = _i32(0)
+    _check(library().occam_set_stage2_route(int(route), ctypes.byref(prev)), "occam_set_stage2_route")
+    return int(prev.value)
 
 
 def occam_selftest_wait(limit_ns: int = 20_000_000, device="cuda", stream=None) -> tuple[int, int]:

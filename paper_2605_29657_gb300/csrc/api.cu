@@ -4,6 +4,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -11,6 +12,7 @@
 
 #include "common.cuh"
 #include "kernels.cuh"
+#include "validate.cuh"
 
 using namespace occam;
 
@@ -27,7 +29,6 @@ size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   WsLayout L{};
@@ -87,18 +88,6 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
 template <typename T>
 T* at(void* ws, size_t off) {
   return reinterpret_cast<T*>(static_cast<unsigned char*>(ws) + off);
-}
-
-int check_batch(const occam_batch* b) {
-  if (!b) return OCCAM_ERR_INVALID_ARG;
-  if (b->B < 1 || b->S_tot < b->B || b->total_rows < 1 || b->total_rows >= (int64_t(1) << 31) ||
-      b->total_text < 0 || b->total_text >= (int64_t(1) << 31) || b->max_seg_rows < 1 ||
-      b->max_sample_rows < b->max_seg_rows || b->max_text < 0 || b->max_regs < 1)
-    return OCCAM_ERR_INVALID_ARG;
-  if (!b->row_off || !b->seg_off || !b->seg_first || !b->seg_sample || !b->reg_idx || !b->reg_off ||
-      !b->text_off)
-    return OCCAM_ERR_INVALID_ARG;
-  return OCCAM_OK;
 }
 
 int check_ws(const occam_batch* b, int H1, int H2, void* ws, size_t bytes, WsLayout* L) {
@@ -245,20 +234,13 @@ bool encode_map3(CUtensorMap* m, const void* base, int64_t rows, int heads, int 
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Stage-II path selection: the fused tensor-core kernel for every sample that
-// fits it (default), or the two-pass kernels for all samples when
-// OCCAM_STAGE2_PATH=twopass (used to test both paths on the same inputs).
-// OCCAM_STAGE2_PATH: unset or "auto" (default routing), "twopass" (every
-// sample on the two-pass kernels) or "narrow" (no widening of clusters for
-// small batches); the last two exist so that tests reach every path.
-bool fused_enabled() {
-  const char* e = std::getenv("OCCAM_STAGE2_PATH");
-  return !(e && std::strcmp(e, "twopass") == 0);
-}
-bool widening_enabled() {
-  const char* e = std::getenv("OCCAM_STAGE2_PATH");
-  return !(e && std::strcmp(e, "narrow") == 0);
-}
+// Stage-II path selection (occam_set_stage2_route): the fused tensor-core
+// kernel for every sample that fits it (AUTO, the default), the two-pass
+// kernels for all samples (TWOPASS), or AUTO without widening the clusters of
+// small batches (NARROW); the last two let tests reach every path.
+std::atomic<int> g_route{OCCAM_ROUTE_AUTO};
+bool fused_enabled() { return g_route.load(std::memory_order_relaxed) != OCCAM_ROUTE_TWOPASS; }
+bool widening_enabled() { return g_route.load(std::memory_order_relaxed) != OCCAM_ROUTE_NARROW; }
 
 int cuda_ok() {
   cudaError_t e = cudaGetLastError();
@@ -335,16 +317,6 @@ int device_view(const void* p, const void** dev) {
     return OCCAM_OK;
   }
   return OCCAM_ERR_INVALID_ARG;
-}
-
-int check_gather(int n, const void* const* src, const int64_t* rb, void* const* dst) {
-  if (n < 0 || n > OCCAM_MAX_GATHER) return OCCAM_ERR_INVALID_ARG;
-  for (int t = 0; t < n; ++t) {
-    if (!src || !dst || !rb || !src[t] || !dst[t] || rb[t] <= 0 || (rb[t] & 15) || !aligned16(src[t]) ||
-        !aligned16(dst[t]))
-      return OCCAM_ERR_INVALID_ARG;
-  }
-  return OCCAM_OK;
 }
 
 // Optional CUDA events recorded between the kernels of one call (for live
@@ -664,6 +636,14 @@ int mark_roles(const occam_batch* b, const WsLayout& L, void* ws, cudaStream_t s
 extern "C" {
 
 int occam_last_call_kernels(void) { return launch_counter(); }
+
+int occam_set_stage2_route(int32_t route, int32_t* previous) {
+  if (route != OCCAM_ROUTE_AUTO && route != OCCAM_ROUTE_TWOPASS && route != OCCAM_ROUTE_NARROW)
+    return OCCAM_ERR_INVALID_ARG;
+  const int old = g_route.exchange(route);
+  if (previous) *previous = old;
+  return OCCAM_OK;
+}
 
 const char* occam_version(void) { return "occam-gb300 0.1 (sm_103a)"; }
 

@@ -13,10 +13,13 @@
 //   offsets are staged in shared memory for the per-row sample lookups.
 // gather_kernel: persistent grid; one warp copies one kept row of one tensor
 //   with 16-byte loads / stores (exact bit copy).
+#include <cuda.h>
+
 #include <mutex>
 
 #include "common.cuh"
 #include "kernels.cuh"
+#include "validate.cuh"
 
 namespace occam {
 
@@ -267,15 +270,39 @@ __global__ void __launch_bounds__(256) registers_kernel(RegistersParams p) {
   }
 }
 
+// Rows the Stage-II test keeps at lam, as the library applies it: candidates
+// (key bit 31) with s2 >= fl(lam * ref2) in fp32. Block-wide; every thread
+// of the CTA calls it and gets the total.
+__device__ int lambda2_kept(const Lambda2Params& p, float lam, int* s_cnt) {
+  if (threadIdx.x == 0) *s_cnt = 0;
+  __syncthreads();
+  int c = 0;
+  for (int64_t r = threadIdx.x; r < p.bt.total_rows; r += blockDim.x) {
+    if (p.keys[r] >> 31) {
+      const int b = upper_interval(p.bt.row_off, p.bt.B, r);
+      c += p.s2[r] >= __fmul_rn(lam, p.ref2[b]) ? 1 : 0;
+    }
+  }
+  c = __reduce_add_sync(0xffffffffu, c);
+  if ((threadIdx.x & 31) == 0) atomicAdd(s_cnt, c);
+  __syncthreads();
+  const int tot = *s_cnt;
+  __syncthreads();
+  return tot;
+}
+
 // lambda2_select_kernel: one CTA of 1,024 threads. Each candidate row (a
-// visual S1 row of a sample with ref2 > 0) gets the key bits(s2 / ref2), an
-// IEEE round-to-nearest fp32 quotient >= 0 whose bit pattern orders like its
-// value; every other row gets key 0, below or equal to every candidate. The
-// K-th largest key is then found most significant byte first: per byte, a
-// histogram of the keys that match the bytes chosen so far (one 256-bin
+// visual S1 row of a sample with ref2 > 0) gets the key 2^31 | bits(s2 /
+// ref2), with an IEEE round-to-nearest fp32 quotient >= 0 whose bit pattern
+// orders like its value; every other row gets key 0, below every candidate.
+// The K-th largest key is then found most significant byte first: per byte,
+// a histogram of the keys that match the bytes chosen so far (one 256-bin
 // histogram per warp, then summed), and the bucket where the running count
 // from the top reaches K. With K <= the candidate count the result is the
-// K-th largest candidate ratio.
+// K-th largest candidate ratio. The rule applies lambda2 as one fp32 product
+// (s2 >= fl(lambda2 * ref2)), whose rounding can disagree with the
+// quotient's by an ulp or two: the ratio is then moved by single fp32 steps
+// to the largest value under which that test keeps at least K rows.
 __global__ void __launch_bounds__(1024) lambda2_select_kernel(Lambda2Params p) {
   __shared__ uint32_t hist[32][256];
   __shared__ uint32_t tot[256];
@@ -291,7 +318,7 @@ __global__ void __launch_bounds__(1024) lambda2_select_kernel(Lambda2Params p) {
     const float ref = p.ref2[b];
     uint32_t key = 0;
     if (p.keep1[r] && p.role[r] == 0 && ref > 0.f) {
-      key = __float_as_uint(__fdiv_rn(p.s2[r], ref));
+      key = 0x80000000u | __float_as_uint(__fdiv_rn(p.s2[r], ref));
       ++cnt;
     }
     p.keys[r] = key;
@@ -339,7 +366,28 @@ __global__ void __launch_bounds__(1024) lambda2_select_kernel(Lambda2Params p) {
     mask |= 255u << shift;
     __syncthreads();
   }
-  if (tid == 0) *p.lambda2 = __uint_as_float(s_prefix);
+  // from the K-th largest quotient to the largest fp32 lambda2 whose product
+  // test keeps >= K rows: down while it keeps fewer (kept(0) counts every
+  // candidate), then up while the next value still keeps K (a few steps;
+  // bounded)
+  __shared__ float s_lam;
+  __shared__ int s_kept;
+  if (tid == 0) s_lam = __uint_as_float(s_prefix & 0x7fffffffu);
+  __syncthreads();
+  const int K = p.target;
+  for (int it = 0; it < 64; ++it) {
+    const float lam = s_lam;
+    if (lambda2_kept(p, lam, &s_kept) >= K) break;
+    if (tid == 0) s_lam = nextafterf(lam, 0.f);
+    __syncthreads();
+  }
+  for (int it = 0; it < 64; ++it) {
+    const float up = nextafterf(s_lam, __int_as_float(0x7f800000));
+    if (lambda2_kept(p, up, &s_kept) < K) break;
+    if (tid == 0) s_lam = up;
+    __syncthreads();
+  }
+  if (tid == 0) *p.lambda2 = s_lam;
 }
 
 }  // namespace occam
@@ -359,30 +407,81 @@ constexpr int kNoAllocMaxDevices = 64;
 // [0, kNoAllocMaxTiles): tile states; then one int32 ticket and one int32 status
 static __device__ __align__(256) unsigned long long g_noalloc_scratch[kNoAllocMaxTiles + 32];
 
+// The array's device address belongs to the CUDA context that loaded this
+// module: it is looked up once per context (with its device current) and
+// cached under the context's unique id, so a context created later on the
+// same device (after cudaDeviceReset, or a driver-API context) gets its own
+// lookup instead of a stale address.
+struct NoAllocEntry {
+  unsigned long long ctx_id = 0;
+  void* ptr = nullptr;
+  int sms = 0;
+};
 std::mutex g_noalloc_mu;
-void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
-int g_noalloc_sms[kNoAllocMaxDevices] = {};
+NoAllocEntry g_noalloc[kNoAllocMaxDevices];
+int g_noalloc_next = 0;
 
-// Device address of the static scratch on the current device (looked up once
-// per device, with that device current).
-int noalloc_scratch(void** ptr, int* sms) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices) return OCCAM_ERR_CUDA;
-  std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (g_noalloc_ptr[dev] == nullptr) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return OCCAM_ERR_CUDA;
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
-    g_noalloc_ptr[dev] = p;
-    g_noalloc_sms[dev] = n;
-  }
-  *ptr = g_noalloc_ptr[dev];
-  *sms = g_noalloc_sms[dev];
-  return OCCAM_OK;
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+// The unique id of the current context (0 if there is none or the driver
+// cannot say).
+unsigned long long current_ctx_id() {
+  static CtxGetCurrentFn get_cur = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_cur = reinterpret_cast<CtxGetCurrentFn>(f);
+    f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(f);
+  });
+  CUcontext c = nullptr;
+  unsigned long long id = 0;
+  if (!get_cur || !get_id || get_cur(&c) != CUDA_SUCCESS || c == nullptr || get_id(c, &id) != CUDA_SUCCESS) return 0;
+  return id;
 }
 
-bool aligned16_na(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+// Device address of the static scratch in the current context, and the
+// device's SM count.
+int noalloc_scratch(void** ptr, int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return OCCAM_ERR_CUDA;
+  // the runtime creates the device's context on its first use: look the
+  // address up first, then read the id of the context it belongs to
+  void* p = nullptr;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  unsigned long long id = current_ctx_id();
+  if (id != 0) {
+    for (const NoAllocEntry& e : g_noalloc) {
+      if (e.ctx_id == id) {
+        *ptr = e.ptr;
+        *sms = e.sms;
+        return OCCAM_OK;
+      }
+    }
+  }
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return OCCAM_ERR_CUDA;
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+  if (id == 0) id = current_ctx_id();
+  if (id != 0) {
+    // a new context: one cache slot (round robin once all are taken)
+    NoAllocEntry& e = g_noalloc[g_noalloc_next];
+    g_noalloc_next = (g_noalloc_next + 1) % kNoAllocMaxDevices;
+    e.ctx_id = id;
+    e.ptr = p;
+    e.sms = n;
+  }
+  *ptr = p;
+  *sms = n;
+  return OCCAM_OK;
+}
 
 }  // namespace
 
@@ -392,17 +491,13 @@ extern "C" int occam_compact_noalloc(const occam_batch* b, const uint8_t* keep, 
                                      int64_t* out_off, occam_stream_t stream) {
   occam::launch_counter() = 0;
   using namespace occam;
-  if (!b || b->B < 1 || b->S_tot < b->B || b->total_rows < 1 || !b->row_off || !b->seg_off ||
-      !b->reg_idx || !b->reg_off)
-    return OCCAM_ERR_INVALID_ARG;
+  // the same checks as occam_compact's, then the limit of the fixed scratch
+  const int rc_batch = check_batch(b);
+  if (rc_batch != OCCAM_OK) return rc_batch;
+  const int rc_gather = check_gather(n_tensors, src, row_bytes, dst);
+  if (rc_gather != OCCAM_OK) return rc_gather;
   if (!keep || !count_out || !out_off || capacity_rows < 0 || (capacity_rows > 0 && !out_index))
     return OCCAM_ERR_INVALID_ARG;
-  if (n_tensors < 0 || n_tensors > OCCAM_MAX_GATHER) return OCCAM_ERR_INVALID_ARG;
-  for (int t = 0; t < n_tensors; ++t) {
-    if (!src || !dst || !row_bytes || !src[t] || !dst[t] || row_bytes[t] <= 0 || (row_bytes[t] & 15) ||
-        !aligned16_na(src[t]) || !aligned16_na(dst[t]))
-      return OCCAM_ERR_INVALID_ARG;
-  }
   const int64_t ntiles = (b->total_rows + kScanTile - 1) / kScanTile;
   if (ntiles > kNoAllocMaxTiles) return OCCAM_ERR_UNSUPPORTED;  // more rows than the static scratch covers
   void* scratch = nullptr;

@@ -36,17 +36,14 @@ def run_prune(batch: dict, lam1: float, lam2: float, keep_registers: bool = True
     host_inputs: K2, hidden and V stay in pinned host memory (occam_prune_staged).
     rule / budget: the selection rule ("register", "mean", "budget") and the
     per-sample budget array (host ints) of the "budget" rule."""
-    import os
-    old = os.environ.get("OCCAM_STAGE2_PATH")
-    os.environ["OCCAM_STAGE2_PATH"] = path
+    import paper_2605_29657_gb300 as occ
+    route = {"auto": occ.OCCAM_ROUTE_AUTO, "twopass": occ.OCCAM_ROUTE_TWOPASS, "narrow": occ.OCCAM_ROUTE_NARROW}[path]
+    old = occ.occam_set_stage2_route(route)
     try:
         return _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs,
                           rule, budget)
     finally:
-        if old is None:
-            os.environ.pop("OCCAM_STAGE2_PATH", None)
-        else:
-            os.environ["OCCAM_STAGE2_PATH"] = old
+        occ.occam_set_stage2_route(old)
 
 
 def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs=False,

@@ -58,7 +58,21 @@ def _lambda2_case(b, s2, ref2, keep1, K):
     want, n_want = O.lambda2_for_budget(s2, ref2, keep1, is_reg, m["row_off_host"], K)
     got = lam.cpu().numpy()[0]
     assert int(n.cpu()[0]) == n_want
-    assert got.tobytes() == np.float32(want).tobytes(), (K, got, want)   # bit-exact: same fp32 quotients
+    assert got.tobytes() == np.float32(want).tobytes(), (K, got, want)   # bit-exact: same fp32 arithmetic
+    if 0 < K <= n_want:
+        # the library's own threshold at lambda2* keeps at least K rows over the samples with a
+        # positive reference, and fewer one fp32 step above it
+        pos = torch.from_numpy(ref2 > 0).cuda()
+        k1 = torch.from_numpy(keep1.astype(np.uint8)).cuda()
+        r2 = torch.from_numpy(ref2).cuda()
+        s2d = torch.from_numpy(s2).cuda()
+        kept = []
+        for lam_try in (got, np.nextafter(got, np.float32(np.inf))):
+            _, cnt = occ.occam_threshold(layout, s2d, r2, occ.OCCAM_REF_SAMPLE, float(lam_try),
+                                         prev_keep=k1, keep_registers=False)
+            torch.cuda.synchronize()
+            kept.append(int(cnt[pos].sum().item()))
+        assert kept[0] >= K > kept[1], (K, kept)
 
 
 @pytest.mark.parametrize("seed", [0, 1])

@@ -1,8 +1,9 @@
 """occam_compact_noalloc: the compaction entry point for callers that cannot
 allocate device memory (it uses the library's fixed scratch array instead of
-a workspace). Its output must equal occam_compact's on the same inputs, on
-two calls in a row (the second call reuses the array the first one left
-behind). This file is collected last on purpose."""
+a workspace). Its output must equal the oracle's compaction and
+occam_compact's on the same inputs, on two calls in a row (the second call
+reuses the array the first one left behind). This file is collected last on
+purpose."""
 
 from __future__ import annotations
 
@@ -24,6 +25,7 @@ def test_noalloc_matches_workspace_entry_two_calls():
     import __graft_entry__ as g
     g.build()
     import paper_2605_29657_gb300 as occ
+    from oracle import occam_oracle as O
 
     assert torch.cuda.is_available()
     b = _batch()
@@ -39,6 +41,15 @@ def test_noalloc_matches_workspace_entry_two_calls():
         torch.cuda.synchronize()
         n = int(want["out_off"][-1])
         assert n == int(mask.sum())
+        # against the oracle's compaction of the same mask and tensors (bit-exact)
+        r_index, r_count, r_off, r_rows = O.compact(mask.cpu().numpy().astype(bool), b["meta"]["row_off_host"],
+                                                    tensors=[t.cpu().view(torch.int16).numpy() for t in tensors])
+        assert np.array_equal(got["out_off"].cpu().numpy(), r_off), f"call {call}: oracle out_off"
+        assert np.array_equal(got["count_out"].cpu().numpy(), r_count), f"call {call}: oracle counts"
+        assert np.array_equal(got["out_index"][:n].cpu().numpy(), r_index), f"call {call}: oracle index"
+        for t in range(len(tensors)):
+            assert np.array_equal(got["gathered"][t][:n].cpu().view(torch.int16).numpy(), r_rows[t]), \
+                f"call {call}: oracle gathered {t}"
         assert torch.equal(got["out_off"], want["out_off"]), f"call {call}: out_off"
         assert torch.equal(got["count_out"], want["count_out"]), f"call {call}: count_out"
         assert torch.equal(got["out_index"][:n], want["out_index"][:n]), f"call {call}: out_index"
