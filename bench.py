@@ -64,6 +64,14 @@ def _peaks():
     return FALLBACK_HBM_GBS, "fallback"
 
 
+def _peak_tflops_sustained():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return float(json.load(f).get("bf16_tflops_sustained", 1700.0))
+    return 1700.0
+
+
 class ClockSampler:
     """Samples SM clocks / throttle reasons with nvidia-smi while running."""
 
@@ -180,6 +188,130 @@ def algorithmic_bytes(meta: dict, n1_total: int, kept_total: int) -> dict:
     return b
 
 
+def _kernel_stats(occ, events):
+    """Per-kernel interval means (ms) and, per kernel, the spread over the
+    traced calls (min, max, standard deviation)."""
+    mean, spread = {}, {}
+    for j, name in enumerate(occ.PruneCall.TRACE_NAMES):
+        xs = [evs[j].elapsed_time(evs[j + 1]) for evs in events]
+        mean[name] = float(np.mean(xs))
+        spread[name] = {"min": float(np.min(xs)), "max": float(np.max(xs)), "std": float(np.std(xs)), "n": len(xs)}
+    return mean, spread
+
+
+def mutual_stage1_flops(meta: dict) -> float:
+    """Multiply-add FLOPs of the mutual Stage I (Sec. 3.4, Eq. 6): per
+    segment of n rows, two passes of n x n logits per head over d1 dims."""
+    seg = np.diff(np.asarray(meta["seg_off_host"], dtype=np.int64)).astype(np.float64)
+    return float(2 * np.sum(2.0 * seg * seg * meta["H1"] * meta["d1"]))
+
+
+def measure_workload(occ, name: str, dev, steps: int, warmup: int, l2_flush: bool = False, n_traced: int = 20,
+                     peak_gbs: float = FALLBACK_HBM_GBS, peak_tflops: float = 0.0) -> dict:
+    """One workload, one occam_prune call at a time: `steps` replays of the
+    call's CUDA graph timed with CUDA events (with l2_flush, a 256 MB buffer
+    is written before every step and each step is timed alone), then
+    `n_traced` eager calls recording per-kernel events."""
+    import torch
+    from synth import get_config, make_batch
+
+    w = get_config(name)
+    batch = make_batch(w, device=dev, seed=w.seed)
+    meta = batch["meta"]
+    layout = occ.BatchLayout.from_batch(batch, dev)
+    cls = w.stage1 == "cls"
+    st1 = (dict(mode="cls", q=batch["q_cls"], k_cls=batch["k_cls"], K1=batch["K1"]) if cls else
+           dict(mode="mutual", q=batch["Q1"], K1=batch["K1"]))
+    call = occ.PruneCall(layout, st1, dict(Q_text=batch["Q_text"], K_text=batch["K_text"], K2=batch["K2"]),
+                         w.lambda1, w.lambda2, keep_registers=True,
+                         gather=(batch["hidden"], batch["K2"].view(batch["K2"].shape[0], -1), batch["V"]))
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        call()
+    call()
+    torch.cuda.synchronize()
+    if call.status() != 0:
+        raise RuntimeError(f"device status {call.status()} on {name}")
+    kernels = occ.occam_last_call_kernels()
+    out = call.out
+    n1_total = int(out["n1_vis"].sum().item()) + int(meta["regs_per_seg"] * meta["S_tot"])
+    kept_total = int(out["out_off"][-1].item())
+    bytes_ = algorithmic_bytes(meta, n1_total, kept_total)
+    want = {k: v.clone() for k, v in out.items()}
+    cap = torch.cuda.Stream(device=dev)
+    cap.wait_stream(stream)
+    with torch.cuda.stream(cap):
+        call(cap)
+    stream.wait_stream(cap)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        call()
+    g.replay()
+    torch.cuda.synchronize()
+    for k, v in want.items():
+        same = torch.equal(v[:kept_total], out[k][:kept_total]) if k == "out_index" else torch.equal(v, out[k])
+        if not same:
+            raise RuntimeError(f"{name}: a graph replay differs from the eager call in {k}")
+    if l2_flush:
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for i, (a, b) in enumerate(ev):
+            flush.fill_(i & 255)
+            a.record(stream)
+            g.replay()
+            b.record(stream)
+        torch.cuda.synchronize()
+        ms = float(sum(a.elapsed_time(b) for a, b in ev))
+        del flush
+    else:
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(steps):
+            g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b)
+    nk = len(occ.PruneCall.TRACE_NAMES) + 1
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(n_traced)]
+    for evs in events:  # torch creates an event's CUDA handle on its first record
+        for e in evs:
+            e.record(stream)
+    torch.cuda.synchronize()
+    for evs in events:
+        call.traced(evs, stream)
+    torch.cuda.synchronize()
+    if call.status() != 0:
+        raise RuntimeError(f"device status {call.status()} on {name} after timing")
+    per_kernel, spread = _kernel_stats(occ, events)
+    dom = max(per_kernel, key=per_kernel.get)
+    step_ms = ms / steps
+    res = {
+        "ms_per_step": step_ms, "images_per_s": meta["B"] / (step_ms / 1e3), "steps": steps,
+        "l2": "a 256 MB buffer written before every step (L2 flushed)" if l2_flush else
+              ("no flush: inputs " + ("larger" if bytes_["step"] > (128 << 20) else "smaller") + " than L2"),
+        "mean_n1_vis": float(out["n1_vis"].float().mean().item()),
+        "mean_count_vis": float(out["count_vis"].float().mean().item()),
+        "algorithmic_bytes_per_step": bytes_["step"],
+        "step_frac_of_measured_hbm": bytes_["step"] / (step_ms / 1e3) / 1e9 / peak_gbs,
+        "dominant_interval": dom, "dominant_ms": per_kernel[dom], "dominant_ms_spread": spread[dom],
+        "kernels_per_step": kernels, "per_kernel_ms": per_kernel,
+    }
+    if cls or dom != "stage1":
+        res["dominant_frac_of_measured_hbm"] = bytes_[dom] / (per_kernel[dom] / 1e3) / 1e9 / peak_gbs
+    if not cls:
+        fl = mutual_stage1_flops(meta)
+        tf = fl / (per_kernel["stage1"] / 1e3) / 1e12
+        res["stage1_mutual"] = {"flops": fl, "achieved_tflops": tf, "peak_tflops": peak_tflops,
+                                "frac": tf / peak_tflops if peak_tflops else None,
+                                "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained",
+                                "note": "multiply-add FLOPs of both passes (2 n^2 H1 d1 each per segment)"}
+    del call, g, batch, out, want
+    torch.cuda.empty_cache()
+    return res
+
+
 def aggregate(ms_local: float, images_local: int, device=None):
     """Max of the timed milliseconds and sum of the images over all ranks
     (replicas: nothing else is exchanged)."""
@@ -248,10 +380,13 @@ def run_ours(args, rank, world, local):
     import paper_2605_29657_gb300 as occ
     from synth import get_config, make_batch
 
-    # host-core oracle pool first: spawn, before the first GPU call
-    n_workers = min(16, os.cpu_count() or 1)
+    # host-core oracle pool first: spawn, before the first GPU call; one
+    # single-threaded worker per host core
+    n_workers = os.cpu_count() or 1
     pool = _make_pool(n_workers) if (rank == 0 and not args.no_cpu_baseline) else None
 
+    occ.occam_set_stage2_route({"auto": occ.OCCAM_ROUTE_AUTO, "narrow": occ.OCCAM_ROUTE_NARROW,
+                                "twopass": occ.OCCAM_ROUTE_TWOPASS}[args.route])
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     if world > 1:
@@ -337,18 +472,12 @@ def run_ours(args, rank, world, local):
             same_as_first(c, "a graph replay")
             graphs.append(g)
 
-    # traced steps record per-kernel events (eager calls). With one call in
-    # flight they are spread over the timed steps; with several, they are the
-    # last steps of the timed region, made one call at a time on one stream,
-    # so that a kernel's interval is its own and not shared with other calls
-    if inflight > 1:
-        n_traced = max(1, min(args.steps // 20, 100))
-        traced_at = set(range(args.steps - n_traced, args.steps))
-    else:
-        n_traced = max(1, min(args.steps // 5 if graphs is not None else args.steps, 400))
-        traced_at = set(np.linspace(0, args.steps - 1, n_traced).astype(int).tolist())
+    # per-kernel events come from eager calls made one at a time on one
+    # stream after the timed region (so a kernel's interval is its own, not
+    # shared with another call's kernels, and `value` is untouched)
+    n_traced = max(20, min(args.steps // 5, 200))
     events = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(n_traced)]
-    for evs in events:
+    for evs in events:  # torch creates an event's CUDA handle on its first record
         for e in evs:
             e.record(stream)
     torch.cuda.synchronize()
@@ -364,23 +493,10 @@ def run_ours(args, rank, world, local):
     t_start.record(stream)
     for s_ in streams[1:]:
         s_.wait_event(t_start)
-    ti = 0
-    joined = False
     for i in range(args.steps):
-        if inflight > 1 and i in traced_at:
-            if not joined:  # the in-flight steps end here; the traced ones follow on one stream
-                for s_ in streams:
-                    stream.wait_stream(s_)
-                joined = True
-            calls[0].traced(events[ti], stream)
-            ti += 1
-            continue
         j = i % inflight
         with torch.cuda.stream(streams[j]):
-            if i in traced_at:
-                calls[j].traced(events[ti])
-                ti += 1
-            elif graphs is not None:
+            if graphs is not None:
                 graphs[j].replay()
             else:
                 calls[j]()
@@ -397,9 +513,10 @@ def run_ours(args, rank, world, local):
         if st != 0:
             raise RuntimeError(f"device status {st} after the timed steps")
         same_as_first(c, "a call after the timed steps")
-    per_kernel = {}
-    for j, name in enumerate(occ.PruneCall.TRACE_NAMES):
-        per_kernel[name] = float(np.mean([evs[j].elapsed_time(evs[j + 1]) for evs in events]))
+    for evs in events:
+        calls[0].traced(evs, stream)
+    torch.cuda.synchronize()
+    per_kernel, per_kernel_spread = _kernel_stats(occ, events)
 
     ms_max, images = aggregate(ms, meta["B"] * args.steps, dev)
     value = images / (ms_max / 1e3)
@@ -465,7 +582,7 @@ def run_ours(args, rank, world, local):
                     raise RuntimeError(f"host-input call differs from the device-input call in {k}")
             if not torch.equal(rh["out_index"][:kept_total], call.out["out_index"][:kept_total].cpu()):
                 raise RuntimeError("host-input call differs from the device-input call in out_index")
-        e_steps = max(4, min(12, args.steps // 100))
+        e_steps = max(20, min(50, args.steps // 20))
         if world > 1:
             dist.barrier()
         a = torch.cuda.Event(enable_timing=True)
@@ -551,6 +668,20 @@ def run_ours(args, rank, world, local):
         return None
 
     peak, peak_kind = _peaks()
+    # the other workloads of the configuration list, one call at a time
+    # (parity-test shapes, reported beside the headline; not part of `value`)
+    workloads = None
+    used_graph = graphs is not None
+    if not args.no_workloads:
+        del sets, calls, graphs
+        torch.cuda.empty_cache()
+        wsteps = max(50, min(300, args.steps // 4))
+        workloads = {}
+        for nm in ("llava15_b1", "llavanext_b8", "qwen3vl_b32", "video_b4"):
+            workloads[nm] = measure_workload(occ, nm, dev, wsteps, 5, peak_gbs=peak,
+                                             peak_tflops=_peak_tflops_sustained())
+        for nm in ("llava15_b1", "llavanext_b8"):
+            workloads[nm + "_l2flush"] = measure_workload(occ, nm, dev, wsteps, 5, l2_flush=True, peak_gbs=peak)
     dom = max(per_kernel, key=per_kernel.get)
     achieved = bytes_[dom] / (per_kernel[dom] / 1e3) / 1e9
     traffic = _traffic_from_profiles(dom)
@@ -558,16 +689,18 @@ def run_ours(args, rank, world, local):
                 "frac": achieved / peak, "traffic": traffic, "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
                 if peak_kind == "measured" else "fallback 6.8 TB/s",
                 "algorithmic_bytes_per_launch": bytes_[dom], "avg_launch_ms": per_kernel[dom]}
-    roofline["timing"] = (f"avg_launch_ms from CUDA events around the kernel in {n_traced} of the {args.steps} "
-                          "timed steps" + (f", made one call at a time at the end of the timed region (the other "
-                                           f"steps keep {inflight} calls in flight)" if inflight > 1 else ""))
+    roofline["timing"] = (f"avg_launch_ms from CUDA events around the kernel in {n_traced} eager calls made one at "
+                          "a time after the timed region (outside `value`)")
+    roofline["launch_ms_spread"] = per_kernel_spread[dom]
     step_ms = ms_max / args.steps
     step_gbs = bytes_["step"] / (step_ms / 1e3) / 1e9
     cpu = None
     if pool is not None:
-        cpu = oracle_throughput(n_workers, 12, 0, pool=pool)
+        cpu = oracle_throughput(n_workers, 10, 0, pool=pool)
         pool.close()
         pool.join()
+        one = oracle_throughput(1, 8, 50_000)   # the same oracle on one core, alone
+        cpu["single_thread"] = {"value": one["value"], "unit": UNIT, "cores": 1, "sample": one["sample"]}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
@@ -584,11 +717,10 @@ def run_ours(args, rank, world, local):
             "l2": "inputs larger than L2 (about 5 GB resident per step); no flush",
             "launch": (f"{inflight} occam_prune calls in flight on {inflight} streams, each with its own copy of "
                        "the inputs, workspace and outputs; a step replays one call's CUDA graph (every kernel of "
-                       f"the call); the last {n_traced} steps are eager calls, one at a time, recording "
-                       "per-kernel events")
-                      if graphs is not None else
+                       f"the call); per-kernel events from {n_traced} eager calls after the timed region")
+                      if used_graph else
                       f"{inflight} eager occam_prune calls in flight on {inflight} streams "
-                      f"({n_traced} recording per-kernel events)",
+                      f"(per-kernel events from {n_traced} eager calls after the timed region)",
             "inflight": inflight,
             "mean_n1_vis": float(out["n1_vis"].float().mean().item()),
             "mean_count_vis": float(out["count_vis"].float().mean().item()),
@@ -598,6 +730,7 @@ def run_ours(args, rank, world, local):
             "step_frac_of_measured_hbm": step_gbs / peak,
             "step_frac_of_8TBps": step_gbs / SPEC_HBM_GBS,
             "per_kernel_ms": per_kernel,
+            "per_kernel_ms_spread": per_kernel_spread,
         },
         "roofline": roofline,
         "cpu_baseline": cpu,
@@ -608,6 +741,7 @@ def run_ours(args, rank, world, local):
         "gpu_launches": kernels_per_step * args.steps,
         "clocks": clocks,
         "next_rows": next_rows,
+        "workloads": workloads,
     }
     if world > 1:
         dist.destroy_process_group()
@@ -619,7 +753,7 @@ def run_ours(args, rank, world, local):
 def run_reference(args, rank, world):
     if rank != 0:
         return None
-    n_workers = min(16, os.cpu_count() or 1)
+    n_workers = os.cpu_count() or 1
     pool = _make_pool(n_workers)
     for i in range(args.warmup):
         oracle_throughput(n_workers, 1, 10_000 + i, pool=pool)
@@ -660,6 +794,9 @@ def main():
                     help="prune calls in flight at once (own inputs, workspace, outputs and stream each)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next", action="store_true", help="skip timing the rows beyond the pruning path")
+    ap.add_argument("--no-workloads", action="store_true", help="skip timing the other four workloads")
+    ap.add_argument("--route", default="auto", choices=["auto", "narrow", "twopass"],
+                    help="Stage-II routing (diagnostics; auto is the library default)")
     ap.add_argument("--workload", default=WORKLOAD,
                     help="synthetic workload to time (default: the LLaVA-NeXT batch-64 throughput workload)")
     args = ap.parse_args()
