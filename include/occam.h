@@ -61,7 +61,9 @@ enum {
   OCCAM_ERR_CUDA = 3,        /* a CUDA launch failed (cudaGetLastError) */
   OCCAM_ERR_TIMEOUT = 4,     /* a bounded device-side wait gave up */
   OCCAM_ERR_UNSUPPORTED = 5, /* head count / head dim / size outside what the kernels are built for */
-  OCCAM_ERR_WORKSPACE = 6    /* workspace null, too small or not 256-byte aligned */
+  OCCAM_ERR_WORKSPACE = 6,   /* workspace null, too small or not 256-byte aligned */
+  OCCAM_ERR_BOUNDS = 7       /* checked builds (OCCAM_CHECKED=1) only: a computed index fell outside the
+                                buffer it addresses; the access was skipped (see occam_get_status) */
 };
 
 enum { OCCAM_STAGE1_CLS = 0, OCCAM_STAGE1_MUTUAL = 1 };
@@ -134,7 +136,11 @@ int occam_workspace_size(const occam_batch* batch, int32_t H1, int32_t H2, size_
 
 /* Reads and clears the device status word of `workspace` (synchronises
  * `stream`). *status receives OCCAM_OK or the first device-side error code
- * recorded since the last call. */
+ * recorded since the last call. In a checked build of the library
+ * (compiled with OCCAM_CHECKED=1, every computed index of the kernels'
+ * gathers, lists and scans tested against its buffer) a violation records
+ * OCCAM_ERR_BOUNDS, and the int32 after the status word (workspace bytes
+ * 4..7) names the check site that failed first; both are cleared here. */
 int occam_get_status(void* workspace, int32_t* status, occam_stream_t stream);
 
 /* Stage-I scores (Sec. 3.4, Eqs. 4 and 6; App. A, Eqs. 10 and 13).

@@ -87,6 +87,16 @@ class CPruneOut(ctypes.Structure):
 _lib = None
 
 
+def use_library(path: str) -> None:
+    """Selects the shared library the binding loads (for example the
+    bounds-checked build, liboccam_checked.so). Must come before the first
+    call into the library."""
+    global LIB_PATH
+    if _lib is not None and os.path.abspath(path) != os.path.abspath(LIB_PATH):
+        raise OccamError(OCCAM_ERR_INVALID_ARG, f"the library is already loaded from {LIB_PATH}")
+    LIB_PATH = path
+
+
 def library() -> ctypes.CDLL:
     """Loads liboccam.so once; raises OccamError when it is missing."""
     global _lib

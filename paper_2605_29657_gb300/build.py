@@ -2,7 +2,10 @@
 
 The translation units are compiled in parallel into ``_build/`` next to this
 file and linked into ``liboccam.so`` in this package directory (both are
-git-ignored build products).
+git-ignored build products). ``build(checked=True)`` makes the bounds-checked
+variant instead (``-DOCCAM_CHECKED=1``: every computed gather, list and scan
+index is tested in-kernel and a violation is recorded in the status word):
+``liboccam_checked.so``, from ``_build_checked/``.
 """
 
 from __future__ import annotations
@@ -17,6 +20,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "liboccam.so")
+LIB_CHECKED = os.path.join(HERE, "liboccam_checked.so")
 SOURCES = ["stage1.cu", "stage1_tc.cu", "stage2.cu", "stage2_tc.cu", "stage2_scores_tc.cu", "compact.cu", "rules.cu", "selftest.cu", "api.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
@@ -32,33 +36,38 @@ def _flags():
     return ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", os.path.join(ROOT, "include")]
 
 
-def build(verbose: bool = False, force: bool = False) -> str:
-    """Builds liboccam.so unless it is newer than every source. Concurrent
-    callers (one per rank) serialise on a lock file."""
+def build(verbose: bool = False, force: bool = False, checked: bool = False) -> str:
+    """Builds liboccam.so (or, with checked, liboccam_checked.so) unless it
+    is newer than every source. Concurrent callers (one per rank) serialise
+    on a lock file."""
     import fcntl
 
-    os.makedirs(BUILD, exist_ok=True)
-    with open(os.path.join(BUILD, ".lock"), "w") as lk:
+    bdir = BUILD + ("_checked" if checked else "")
+    os.makedirs(bdir, exist_ok=True)
+    with open(os.path.join(bdir, ".lock"), "w") as lk:
         fcntl.flock(lk, fcntl.LOCK_EX)
         try:
-            return _build(verbose, force)
+            return _build(verbose, force, checked)
         finally:
             fcntl.flock(lk, fcntl.LOCK_UN)
 
 
-def _build(verbose: bool, force: bool) -> str:
+def _build(verbose: bool, force: bool, checked: bool = False) -> str:
+    BUILD_DIR = BUILD + ("_checked" if checked else "")
+    LIB_OUT = LIB_CHECKED if checked else LIB
+    extra = ["-DOCCAM_CHECKED=1"] if checked else []
     nv = nvcc()
     deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC)] + [os.path.join(ROOT, "include", "occam.h")]
     newest = max(os.path.getmtime(d) for d in deps)
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= newest and os.path.getmtime(LIB) >= os.path.getmtime(__file__):
-        return LIB
+    if not force and os.path.exists(LIB_OUT) and os.path.getmtime(LIB_OUT) >= newest and os.path.getmtime(LIB_OUT) >= os.path.getmtime(__file__):
+        return LIB_OUT
     procs = []
     objs = []
     for src in SOURCES:
-        obj = os.path.join(BUILD, src.replace(".cu", ".o"))
+        obj = os.path.join(BUILD_DIR, src.replace(".cu", ".o"))
         objs.append(obj)
-        cmd = [nv] + _flags() + ["-Xptxas", "-v", "-c", os.path.join(CSRC, src), "-o", obj]
-        log = open(os.path.join(BUILD, src.replace(".cu", ".log")), "w")
+        cmd = [nv] + _flags() + extra + ["-Xptxas", "-v", "-c", os.path.join(CSRC, src), "-o", obj]
+        log = open(os.path.join(BUILD_DIR, src.replace(".cu", ".log")), "w")
         procs.append((src, subprocess.Popen(cmd, stdout=log, stderr=subprocess.STDOUT), log))
     failed = []
     for src, p, log in procs:
@@ -67,16 +76,16 @@ def _build(verbose: bool, force: bool) -> str:
         if rc != 0:
             failed.append(src)
     if failed:
-        msgs = "".join(open(os.path.join(BUILD, s.replace(".cu", ".log"))).read()[-3000:] for s in failed)
+        msgs = "".join(open(os.path.join(BUILD_DIR, s.replace(".cu", ".log"))).read()[-3000:] for s in failed)
         raise RuntimeError(f"nvcc failed for {failed}:\n{msgs}")
-    tmp = LIB + ".tmp"
+    tmp = LIB_OUT + ".tmp"
     cmd = [nv] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs
     subprocess.run(cmd, check=True, capture_output=not verbose)
-    os.replace(tmp, LIB)
+    os.replace(tmp, LIB_OUT)
     if verbose:
-        print("built", LIB, file=sys.stderr)
-    return LIB
+        print("built", LIB_OUT, file=sys.stderr)
+    return LIB_OUT
 
 
 if __name__ == "__main__":
-    build(verbose=True, force="--force" in sys.argv)
+    build(verbose=True, force="--force" in sys.argv, checked="--checked" in sys.argv)

@@ -616,6 +616,8 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
     g.out_off = out_off;
     g.B = b->B;
     g.capacity = capacity;
+    g.src_rows = b->total_rows;
+    g.status = at<int>(ws, L.status);
     gather_kernel<<<num_sms() * 4, 256, 0, st>>>(g);
     count_launch();
   }
@@ -659,7 +661,8 @@ int occam_get_status(void* workspace, int32_t* status, occam_stream_t stream) {
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   int32_t v = 0;
   OCCAM_CUDA(cudaMemcpyAsync(&v, workspace, 4, cudaMemcpyDeviceToHost, st));
-  OCCAM_CUDA(cudaMemsetAsync(workspace, 0, 4, st));
+  // the status word and, after it, the check site of a checked build
+  OCCAM_CUDA(cudaMemsetAsync(workspace, 0, 8, st));
   OCCAM_CUDA(cudaStreamSynchronize(st));
   *status = v;
   return OCCAM_OK;
@@ -888,6 +891,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
     sp.row_bytes = k2_row;
     sp.dense = at<int32_t>(ws, L.dense);
     sp.n1 = at<int32_t>(ws, L.n1);
+    sp.status = at<int>(ws, L.status);
     stage_rows_kernel<<<num_sms() * 4, 256, 0, st>>>(sp);
     count_launch();
     OCCAM_CUDA(cudaGetLastError());

@@ -23,6 +23,12 @@ __device__ __forceinline__ void set_status(int* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }
 
+}  // namespace occam
+
+#include "check.cuh"
+
+namespace occam {
+
 // ---------------------------------------------------------------- bf16 helpers
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }

@@ -54,6 +54,7 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   int64_t samp_end = 0;
   if (r_first < R) {
     samp = upper_interval(row_off, p.bt.B, r_first);
+    if (!in_bounds(samp >= 0 && samp < p.bt.B, p.status, kSiteScanSample)) samp = 0;
     samp_end = row_off[samp + 1];
   }
 #pragma unroll
@@ -141,6 +142,7 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   // per-sample counts: a thread's rows may span several samples
   {
     int s = (r_first < R) ? upper_interval(row_off, p.bt.B, r_first) : -1;
+    if (s >= 0 && !in_bounds(s < p.bt.B, p.status, kSiteScanSample)) s = 0;
     int64_t send = (s >= 0) ? row_off[s + 1] : 0;
     int ck = 0, cv = 0;
     for (int i = 0; i < PER; ++i) {
@@ -197,6 +199,7 @@ __global__ void __launch_bounds__(256) gather_kernel(GatherParams p) {
     const int t = (int)(w - k * p.n_tensors);
     const int64_t rbytes = p.row_bytes[t];
     const int64_t row = p.out_index[k];
+    if (!in_bounds(row >= 0 && row < p.src_rows, p.status, kSiteGatherRow)) continue;
     const unsigned char* src = p.src[t] + row * rbytes;
     unsigned char* dst = p.dst[t] + k * rbytes;
     int64_t off = (int64_t)lane * 16;
@@ -225,6 +228,7 @@ __global__ void __launch_bounds__(256) stage_rows_kernel(StageRowsParams p) {
     const int b = upper_interval(p.bt.row_off, p.bt.B, pos);
     if (pos - p.bt.row_off[b] >= p.n1[b]) continue;
     const int64_t row = p.dense[pos];
+    if (!in_bounds(row >= 0 && row < p.bt.total_rows, p.status, kSiteStageRow)) continue;
     const unsigned char* src = p.src + row * rbytes;
     unsigned char* dst = p.dst + row * rbytes;
     int64_t off = (int64_t)lane * 16;
@@ -555,6 +559,8 @@ extern "C" int occam_compact_noalloc(const occam_batch* b, const uint8_t* keep, 
     g.out_off = out_off;
     g.B = b->B;
     g.capacity = capacity_rows;
+    g.src_rows = b->total_rows;
+    g.status = status;
     gather_kernel<<<sms * 4, 256, 0, st>>>(g);
     count_launch();
   }

@@ -196,6 +196,8 @@ struct GatherParams {
   const int64_t* out_off;    // total kept = out_off[B]
   int B;
   int64_t capacity;
+  int64_t src_rows;          // rows of every source tensor (checked builds)
+  int* status;               // nullable
 };
 
 // Copies the S1 rows of K2 into a staging tensor at the same row positions
@@ -208,6 +210,7 @@ struct StageRowsParams {
   int64_t row_bytes;
   const int32_t* dense;
   const int32_t* n1;
+  int* status;               // nullable
 };
 
 // Test-time register construction (Algorithm 1; App. A, register

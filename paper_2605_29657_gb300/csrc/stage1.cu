@@ -79,7 +79,8 @@ __global__ void __launch_bounds__(cls::kThreads) stage1_logits_kernel(Stage1ClsP
       float acc = 0.f;
       if (rr < rows) {
         if (row >= seg_hi || row < seg_lo) {
-          const int sg = upper_interval(p.bt.seg_off, p.bt.S_tot, row);
+          int sg = upper_interval(p.bt.seg_off, p.bt.S_tot, row);
+          if (!in_bounds(sg >= 0 && sg < p.bt.S_tot, p.status, kSiteLogitsSegment)) sg = 0;
           seg_lo = p.bt.seg_off[sg];
           seg_hi = p.bt.seg_off[sg + 1];
           const uint4 raw = *reinterpret_cast<const uint4*>(p.q_cls + ((int64_t)sg * H + my_h) * D + kv * 8);
@@ -263,13 +264,19 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   if (staged) {
     for (int r = tid; r < n; r += blockDim.x) role_loc[r] = 0;
     __syncthreads();
-    for (int i = ra + tid; i < rb; i += blockDim.x) role_loc[p.bt.reg_idx[i] - sb] = 1;
+    for (int i = ra + tid; i < rb; i += blockDim.x) {
+      const int64_t reg = p.bt.reg_idx[i];
+      if (in_bounds(reg >= sb && reg < se, p.status, kSiteRegisterRow)) role_loc[reg - sb] = 1;
+    }
     __syncthreads();
     for (int r = tid; r < n; r += blockDim.x) p.role[sb + r] = role_loc[r];
   } else {
     for (int r = tid; r < n; r += blockDim.x) p.role[sb + r] = 0;
     __syncthreads();
-    for (int i = ra + tid; i < rb; i += blockDim.x) p.role[p.bt.reg_idx[i]] = 1;
+    for (int i = ra + tid; i < rb; i += blockDim.x) {
+      const int64_t reg = p.bt.reg_idx[i];
+      if (in_bounds(reg >= sb && reg < se, p.status, kSiteRegisterRow)) p.role[reg] = 1;
+    }
     __syncthreads();
   }
   // ref1 = mean of s1 over the segment's registers (parallel loads, fixed-order
@@ -381,11 +388,15 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   }
   __syncthreads();
   int32_t* list = p.dense + p.bt.row_off[b] + s_base;
+  const int64_t list_len = p.bt.row_off[b + 1] - p.bt.row_off[b] - s_base;  // room left in the sample's list
   for (int r = a; r < z; ++r) {
     const bool reg = role[r] != 0;
     const bool k = reg || (p.keep_in ? p.keep_in[sb + r] != 0 : (staged ? s1_loc[r] : s1g[sb + r]) >= tau);
     if (p.keep1) p.keep1[sb + r] = k ? 1 : 0;
-    if (k) list[pos++] = (int32_t)(sb + r);
+    if (k) {
+      if (in_bounds(pos >= 0 && pos < list_len, p.status, kSiteListPos)) list[pos] = (int32_t)(sb + r);
+      ++pos;
+    }
   }
   if (!p.do_plan) return;
   // the last CTA to finish plans Stage II

@@ -406,13 +406,15 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
               }
             }
             // L = log2 of the row's sum of exp2(c q k) over the segment's keys
-            if (vrow) p.lsum[(int64_t)w.h * R + sb + w.a0 + row] = m + log2f(z);
+            if (vrow && in_bounds(sb + w.a0 + row < R, p.status, kSiteMutualRow))
+              p.lsum[(int64_t)w.h * R + sb + w.a0 + row] = m + log2f(z);
           } else {
             float tot = acc;
 #pragma unroll
             for (int q = 0; q < QW - 1; ++q) tot += sm.part[pp][q][quad][lane].x;
             // this head group's share of s1 (summed over the groups in order afterwards)
-            if (vrow) p.part[(int64_t)(w.h / kMutHeadGroup) * R + sb + w.a0 + row] = tot * p.inv_h / (float)n;
+            if (vrow && in_bounds(sb + w.a0 + row < R, p.status, kSiteMutualRow))
+              p.part[(int64_t)(w.h / kMutHeadGroup) * R + sb + w.a0 + row] = tot * p.inv_h / (float)n;
           }
           __syncwarp();
         }

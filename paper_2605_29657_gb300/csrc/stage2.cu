@@ -217,8 +217,12 @@ __global__ void __launch_bounds__(s2s::THREADS, 1)
             int bytes = 0;
             if (kk < s.k_hi) {
               bytes = 16;
-              src = kk < s.n_img ? p.K + (int64_t)p.dense[s.rbase + kk] * HD
-                                 : p.Kt + (s.t0 + (kk - s.n_img)) * HD;
+              if (kk < s.n_img) {
+                const int64_t row = p.dense[s.rbase + kk];
+                src = p.K + (in_bounds(row >= 0 && row < p.bt.total_rows, p.status, kSiteTwoPassKeyRow) ? row : 0) * HD;
+              } else {
+                src = p.Kt + (s.t0 + (kk - s.n_img)) * HD;
+              }
               src += hoff + kb * 64 + ch * 8;
             }
             tc::cp_async16(sm.k[st][kb] + r * 128 + ((ch ^ (r & 7)) << 4), src, bytes);

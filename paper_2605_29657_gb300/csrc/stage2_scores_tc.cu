@@ -137,7 +137,8 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
     const int nk = min(KR, n_img - k0);
     const int64_t rbase = p.bt.row_off[b];
     for (int i = tid; i < KR; i += THREADS) {
-      const int row = p.dense[rbase + k0 + (i < nk ? i : 0)];
+      int row = p.dense[rbase + k0 + (i < nk ? i : 0)];
+      if (!in_bounds(row >= 0 && row < p.bt.total_rows, p.status, kSiteTwoPassKeyRow)) row = 0;
       sm.kidx[i] = row;
       sm.kreg[i] = (i < nk) ? p.role[row] : 0;
     }

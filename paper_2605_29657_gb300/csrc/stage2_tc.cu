@@ -130,6 +130,8 @@ __device__ __forceinline__ ItemGeom item_geom(const Stage2TcParams& p, int4 it, 
   g.b = it.x;
   g.j0 = it.y;
   g.slot = it.z;
+  const bool item_ok = in_bounds(g.b >= 0 && g.b < p.bt.B, p.status, kSiteFusedItem);
+  if (!item_ok) g.b = 0;
   g.rbase = p.bt.row_off[g.b];
   g.t0 = p.bt.text_off[g.b];
   g.M = (int)(p.bt.text_off[g.b + 1] - g.t0);
@@ -147,6 +149,8 @@ __device__ __forceinline__ ItemGeom item_geom(const Stage2TcParams& p, int4 it, 
   // the same on every CTA of the cluster (depends on the sample only)
   const int ipmax = (per + 31) & ~31;
   g.fits = ipmax <= PMAX && ipmax + ((per_t + 15) & ~15) <= Geo<C>::KROWS;
+  // a bad item (checked builds) is skipped by every role of every CTA alike
+  g.fits = g.fits && item_ok && in_bounds(g.j0 >= 0 && g.j0 < g.M, p.status, kSiteFusedItem);
   g.nhg = hs_groups(it.w);
   g.h0 = hs_group(it.w) * p.H / g.nhg;
   g.h1 = (hs_group(it.w) + 1) * p.H / g.nhg;
@@ -397,7 +401,8 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
         const int ib = ii & 1;
         if (*abort || !tc::bar_wait(&sm.idone[ib], ((ii >> 1) & 1) ^ 1, abort, kLimitNs)) { fail(sm, p.status); break; }
         for (int i = pt; i < g.own_img; i += NPROD * 32) {
-          const int row = p.dense[g.rbase + g.img0 + i];
+          int row = p.dense[g.rbase + g.img0 + i];
+          if (!in_bounds(row >= 0 && row < p.bt.total_rows, p.status, kSiteFusedKeyRow)) row = 0;
           sm.kidx[ib][i] = row;
           sm.kreg[ib][i] = p.role[row];
         }
@@ -751,7 +756,8 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
       }
       int last = 0;
       if (lane == 0) {
-        p.refpart[g.slot + rank * NPW + pw] = regacc;  // C * NPW slots per item
+        const int slot = g.slot + rank * NPW + pw;  // C * NPW slots per item
+        if (in_bounds(slot >= 0 && slot < p.slot_off[p.bt.B], p.status, kSiteFusedSlot)) p.refpart[slot] = regacc;
         __threadfence();
         const int nslots = p.slot_off[g.b + 1] - p.slot_off[g.b];
         last = atomicAdd(&p.done[g.b], 1) == nslots - 1;
@@ -822,7 +828,8 @@ __global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParam
   const float invH = 1.0f / (float)p.H;
   float rc = 0.f;
   if (k < g.own_img) {
-    const int row_id = p.dense[g.rbase + g.img0 + k];
+    int row_id = p.dense[g.rbase + g.img0 + k];
+    if (!in_bounds(row_id >= 0 && row_id < p.bt.total_rows, p.status, kSiteFusedKeyRow)) row_id = 0;
     const bool is_reg = p.role[row_id] != 0;
     const float* src = p.ppart + (((int64_t)t * kHsGroups * 16 + rank) * kHsRows) * PMAX + k;
     float cmax = 0.f, rsum = 0.f;
