@@ -62,7 +62,7 @@ def _slice_gpu(gpu, batch, samples):
 
 @pytest.mark.parametrize("name,samples", [
     ("llavanext_b64", [0, 21, 42, 63]),
-    ("video_b4", [0, 3]),
+    ("video_b4", [0, 1, 2, 3]),
     ("qwen3vl_b32", None),
 ])
 def test_fullsize_sampled(name, samples):
