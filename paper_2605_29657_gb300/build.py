@@ -79,7 +79,7 @@ def _build(verbose: bool, force: bool, checked: bool = False) -> str:
         msgs = "".join(open(os.path.join(BUILD_DIR, s.replace(".cu", ".log"))).read()[-3000:] for s in failed)
         raise RuntimeError(f"nvcc failed for {failed}:\n{msgs}")
     tmp = LIB_OUT + ".tmp"
-    cmd = [nv] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs
+    cmd = [nv] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs + ["-ldl"]
     subprocess.run(cmd, check=True, capture_output=not verbose)
     os.replace(tmp, LIB_OUT)
     if verbose:

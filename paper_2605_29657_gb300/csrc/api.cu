@@ -12,6 +12,7 @@
 
 #include "common.cuh"
 #include "kernels.cuh"
+#include "nvtx.cuh"
 #include "validate.cuh"
 
 using namespace occam;
@@ -334,6 +335,7 @@ struct Trace {
 
 int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const WsLayout& L, void* ws,
                          float* s1, float* s2_zero, cudaStream_t st, Trace trace = Trace()) {
+  const NvtxRange nvtx(a->mode == OCCAM_STAGE1_CLS ? "stage1_cls_scores" : "stage1_mutual_scores");
   const BatchDev bt = dev_batch(b);
   int* status = at<int>(ws, L.status);
   if (a->mode == OCCAM_STAGE1_CLS) {
@@ -387,6 +389,7 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
                      const occam_stage1_args* a1, float* s2_zero, const Stage2Params* plan, int32_t* count_out,
                      int32_t* count_vis, cudaStream_t st, Trace trace = Trace(), float* n_eff = nullptr,
                      int ref_mean = 0) {
+  const NvtxRange nvtx("stage1_finalize");
   Stage1FinalizeParams p;
   p.bt = dev_batch(b);
   const bool cls = a1 && a1->mode == OCCAM_STAGE1_CLS;
@@ -485,6 +488,7 @@ Stage2Params stage2_params(const occam_batch* b, const occam_stage2_args* a, con
 // Stage II after the Stage-I finalize kernel planned it (same arguments).
 int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayout& L, void* ws, float* s2,
                   float* ref2, float lambda2, cudaStream_t st, Trace trace = Trace()) {
+  const NvtxRange nvtx("stage2_scores");
   const Stage2Params p = stage2_params(b, a, L, ws, s2, ref2, lambda2);
   const bool fused = p.use_fused != 0;
   trace.mark(st);
@@ -576,6 +580,7 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
                    const void* const* src, const int64_t* row_bytes, void* const* dst, int64_t capacity,
                    int32_t* out_index, int32_t* count_out, int32_t* count_vis, int64_t* out_off,
                    cudaStream_t st, bool do_memsets = true, Trace trace = Trace(), bool use_role = false) {
+  const NvtxRange nvtx(mode == 1 ? "stage2_threshold_compact" : "compact");
   ScanParams p;
   p.bt = dev_batch(b);
   p.mode = mode;
@@ -670,6 +675,7 @@ int occam_get_status(void* workspace, int32_t* status, occam_stream_t stream) {
 
 int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, float* s1, float* ref1,
                        void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_score_stage1");
   launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   OCCAM_TRY(check_stage1(batch, args));
@@ -687,6 +693,7 @@ int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, 
 int occam_threshold(const occam_batch* batch, const float* s, const float* ref, int32_t ref_scope, float lambda,
                     const uint8_t* prev_keep, int32_t keep_registers, uint8_t* keep, int32_t* count_vis,
                     void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_threshold");
   launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!s || !ref || !keep) return OCCAM_ERR_INVALID_ARG;
@@ -715,6 +722,7 @@ int occam_threshold(const occam_batch* batch, const float* s, const float* ref, 
 
 int occam_mean_reference(const occam_batch* batch, const float* s, int32_t ref_scope, const uint8_t* prev_keep,
                          float* ref, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_mean_reference");
   launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!s || !ref) return OCCAM_ERR_INVALID_ARG;
@@ -739,6 +747,7 @@ int occam_mean_reference(const occam_batch* batch, const float* s, int32_t ref_s
 
 int occam_pool_scores(const float* s_in, int64_t rows_in, int32_t group, int32_t mode, float* s_out,
                       occam_stream_t stream) {
+  const NvtxRange nvtx("occam_pool_scores");
   launch_counter() = 0;
   if (!s_in || !s_out || group < 1 || rows_in < 0 || rows_in % group != 0) return OCCAM_ERR_INVALID_ARG;
   if (mode != OCCAM_POOL_SUM && mode != OCCAM_POOL_MEAN && mode != OCCAM_POOL_MAX) return OCCAM_ERR_INVALID_ARG;
@@ -756,6 +765,7 @@ int occam_pool_scores(const float* s_in, int64_t rows_in, int32_t group, int32_t
 int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* prev_keep, const int32_t* budget,
                       int32_t keep_registers, uint8_t* keep, int32_t* count_vis, void* workspace,
                       size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_budget_keep");
   launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!s || !budget || !keep) return OCCAM_ERR_INVALID_ARG;
@@ -779,6 +789,7 @@ int occam_budget_keep(const occam_batch* batch, const float* s, const uint8_t* p
 
 int occam_score_stage2(const occam_batch* batch, const occam_stage2_args* args, const uint8_t* keep1, float* s2,
                        float* ref2, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_score_stage2");
   launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   OCCAM_TRY(check_stage2(args));
@@ -801,6 +812,7 @@ int occam_compact(const occam_batch* batch, const uint8_t* keep, int32_t n_tenso
                   const int64_t* row_bytes, void* const* dst, int64_t capacity_rows, int32_t* out_index,
                   int32_t* count_out, int64_t* out_off, void* workspace, size_t workspace_bytes,
                   occam_stream_t stream) {
+  const NvtxRange nvtx("occam_compact");
   launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!keep || !count_out || !out_off || capacity_rows < 0 || (capacity_rows > 0 && !out_index))
@@ -884,6 +896,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
                              args->rule == OCCAM_RULE_MEAN ? 1 : 0));
   if (k2_stage) {
     // the S1 rows of K2 (only those) into the device staging tensor
+    const NvtxRange nvtx("stage_k2_rows");
     StageRowsParams sp;
     sp.bt = dev_batch(b);
     sp.src = static_cast<const unsigned char*>(k2_src);
@@ -900,6 +913,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   if (args->rule == OCCAM_RULE_BUDGET) {
     // S2 = the budget[b] visual S1 rows with the largest s2 per sample, then
     // the compaction of that mask
+    const NvtxRange nvtx("stage2_budget");
     BudgetParams bp;
     bp.bt = dev_batch(b);
     bp.s = s2;
@@ -918,6 +932,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   }
   if (args->rule == OCCAM_RULE_MEAN) {
     // the sample's reference becomes the mean s2 of its visual S1 rows
+    const NvtxRange nvtx("stage2_mean_reference");
     MeanRefParams mp;
     mp.bt = dev_batch(b);
     mp.s = s2;
@@ -938,11 +953,13 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
 
 int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                 size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_prune");
   return prune_impl(args, out, workspace, workspace_bytes, stream, Trace());
 }
 
 int occam_construct_registers(const occam_batch* batch, void* h, int64_t channels, const int32_t* k_reg,
                               int32_t n_k, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_construct_registers");
   launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!h || channels <= 0 || n_k < 0 || (n_k > 0 && !k_reg)) return OCCAM_ERR_INVALID_ARG;
@@ -968,6 +985,7 @@ int occam_construct_registers(const occam_batch* batch, void* h, int64_t channel
 int occam_calibrate_lambda2(const occam_batch* batch, const float* s2, const float* ref2, const uint8_t* keep1,
                             int64_t target_count, float* lambda2_out, int32_t* n_candidates, void* workspace,
                             size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_calibrate_lambda2");
   launch_counter() = 0;
   OCCAM_TRY(check_batch(batch));
   if (!s2 || !ref2 || !keep1 || !lambda2_out) return OCCAM_ERR_INVALID_ARG;
@@ -993,12 +1011,14 @@ int occam_calibrate_lambda2(const occam_batch* batch, const float* s2, const flo
 
 int occam_prune_staged(const occam_prune_args* args, const occam_prune_out* out, void* k2_stage,
                        size_t k2_stage_bytes, void* workspace, size_t workspace_bytes, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_prune_staged");
   if (!k2_stage) return OCCAM_ERR_INVALID_ARG;
   return prune_impl(args, out, workspace, workspace_bytes, stream, Trace(), k2_stage, k2_stage_bytes);
 }
 
 int occam_prune_traced(const occam_prune_args* args, const occam_prune_out* out, void* workspace,
                        size_t workspace_bytes, occam_stream_t stream, void* const* events, int32_t n_events) {
+  const NvtxRange nvtx("occam_prune_traced");
   if (n_events < 0 || (n_events > 0 && !events)) return OCCAM_ERR_INVALID_ARG;
   int next = 0;
   Trace t;

@@ -19,6 +19,7 @@
 
 #include "common.cuh"
 #include "kernels.cuh"
+#include "nvtx.cuh"
 #include "validate.cuh"
 
 namespace occam {
@@ -493,6 +494,7 @@ extern "C" int occam_compact_noalloc(const occam_batch* b, const uint8_t* keep, 
                                      const void* const* src, const int64_t* row_bytes, void* const* dst,
                                      int64_t capacity_rows, int32_t* out_index, int32_t* count_out,
                                      int64_t* out_off, occam_stream_t stream) {
+  const NvtxRange nvtx("occam_compact_noalloc");
   occam::launch_counter() = 0;
   using namespace occam;
   // the same checks as occam_compact's, then the limit of the fixed scratch

@@ -65,7 +65,7 @@ struct MutualTcParams {
   int d1;
   float scale_log2;  // log2(e) / sqrt(d1)
   float inv_h;       // 1 / H
-  float* lsum;       // [H, total_rows] per query row and head: log2 of its softmax denominator (log2 domain)
+  float* lsum;       // [H, total_rows] per query row and head: minus log2 of its softmax denominator (log2 domain)
   float* s1;
   float* s2_zero;    // nullable
   int* status;

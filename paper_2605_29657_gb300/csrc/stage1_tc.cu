@@ -8,7 +8,8 @@
 // Two launches of one kernel template:
 //   pass 1: per (segment, tile of 128 query rows, head) the query rows'
 //           softmax log-sums L[h][u] = log2 sum_v exp2(c q_u k_v), with
-//           c = log2(e) / sqrt(d1), over all the segment's keys;
+//           c = log2(e) / sqrt(d1), over all the segment's keys (stored
+//           negated, as the second pass adds them);
 //   pass 2: per (segment, tile of 128 key rows, group of 4 heads) the
 //           attention each key receives, sum_h sum_u exp2(c q_u k_v - L[h][u]),
 //           over the group's heads and all query rows; a small third kernel
@@ -53,7 +54,7 @@ struct Smem {
   uint8_t b[NBB][BBYTES];
   uint8_t a1[2][ABYTES1];   // K-block 1 per buffer
   uint8_t b1[NBB][BBYTES1];
-  float lsm[NEPI][COLS];    // pass 2: minus the log-sums of each softmax warp's columns
+  float lsm[2][NEPI][COLS];  // pass 2: minus the log-sums of each softmax warp's columns (a ring of 2 steps)
   float2 part[2][QW - 1][4][32];  // partials of quarters 1.. per (item parity, quarter, quadrant, lane)
   int32_t item[8];          // the ii-th work item, by ii & 7 (-1: no more)
   uint64_t afull[2], aempty[2], bfull[NBB], bempty[NBB], dfull[2], dfree[2], hb[2][4], inext[8], mdone;
@@ -74,6 +75,10 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, i
       "[%5];" ::"r"(tc::su32(dst)),
       "l"(map), "r"(x), "r"(y), "r"(z), "r"(tc::su32(bar))
       : "memory");
+}
+
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(tc::su32(dst)), "l"(src) : "memory");
 }
 
 __device__ __forceinline__ void wait_ld64(uint32_t (&v)[64]) {
@@ -287,7 +292,6 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       const int pp = ii & 1;
       float m = -INFINITY, z = 0.f;  // pass 1: running max / sum (log2 domain)
       float acc = 0.f;               // pass 2: attention received by this key row
-      float lnext[2];                // pass 2: the next step's minus log-sums of 2 columns
       bool ok = true;
       for (int s = 0; s < steps; ++s, ++sg) {
         const int h = w.h + s / nb;
@@ -295,26 +299,27 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         const int col0 = jb * BR + qtr * COLS;          // segment-relative index of this warp's column 0
         if (PASS == 2) {
           // minus the log-sums of this warp's 64 query columns (past the
-          // segment: -inf, which contributes 0); those of the item's first
-          // step are loaded here, the others one step ahead (below)
-          if (s == 0) {
+          // segment: -inf, which contributes 0) come by cp.async into a ring
+          // of two step slots, one step ahead; the item's first step's are
+          // fetched here. The slot refilled below was last read in the
+          // previous step, which every lane of the warp has finished.
+          auto fetch = [&](int t) {
+            const int ht = w.h + t / nb, ct = (t % nb) * BR + qtr * COLS;
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
-              const int qq = col0 + lane * 2 + i;
-              lnext[i] = qq < n ? -__ldcg(&p.lsum[(int64_t)h * R + sb + qq]) : -INFINITY;
+              const int qq = ct + lane * 2 + i;
+              float* dst = &sm.lsm[t & 1][ew][lane * 2 + i];
+              if (qq < n)
+                cp_async4(dst, &p.lsum[(int64_t)ht * R + sb + qq]);
+              else
+                *dst = -INFINITY;
             }
-          }
+            cp_async_commit();
+          };
+          if (s == 0) fetch(0);
+          cp_async_wait<0>();
           __syncwarp();
-          *reinterpret_cast<float2*>(&sm.lsm[ew][lane * 2]) = make_float2(lnext[0], lnext[1]);
-          __syncwarp();
-          if (s + 1 < steps) {
-            const int h1 = w.h + (s + 1) / nb, c1 = ((s + 1) % nb) * BR + qtr * COLS;
-#pragma unroll
-            for (int i = 0; i < 2; ++i) {
-              const int qq = c1 + lane * 2 + i;
-              lnext[i] = qq < n ? -__ldcg(&p.lsum[(int64_t)h1 * R + sb + qq]) : -INFINITY;
-            }
-          }
+          if (s + 1 < steps) fetch(s + 1);
         }
         const int db = sg & 1;
         if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.dfull[db], (sg >> 1) & 1, nullptr, kLimitNs))) {
@@ -364,7 +369,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
               m = fmaxf(m, mx);
             }
           } else {
-            const float2* nl = reinterpret_cast<const float2*>(sm.lsm[ew]);
+            const float2* nl = reinterpret_cast<const float2*>(sm.lsm[s & 1][ew]);
             const float2 cc = make_float2(c, c);
             float2 ap[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
@@ -405,9 +410,9 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
                 m = fmaxf(m, o.x);
               }
             }
-            // L = log2 of the row's sum of exp2(c q k) over the segment's keys
+            // -L, L = log2 of the row's sum of exp2(c q k) over the segment's keys
             if (vrow && in_bounds(sb + w.a0 + row < R, p.status, kSiteMutualRow))
-              p.lsum[(int64_t)w.h * R + sb + w.a0 + row] = m + log2f(z);
+              p.lsum[(int64_t)w.h * R + sb + w.a0 + row] = -(m + log2f(z));
           } else {
             float tot = acc;
 #pragma unroll
