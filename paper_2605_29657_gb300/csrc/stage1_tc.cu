@@ -58,6 +58,7 @@ struct Smem {
   float2 part[2][QW - 1][4][32];  // partials of quarters 1.. per (item parity, quarter, quadrant, lane)
   int32_t item[8];          // the ii-th work item, by ii & 7 (-1: no more)
   uint64_t afull[2], aempty[2], bfull[NBB], bempty[NBB], dfull[2], dfree[2], hb[2][4], inext[8], mdone;
+  uint64_t aready[2], bready[NBB];  // pass 2 with the log-sums folded into the MMA: tiles completed for it
   uint32_t tmem_base;
   int abort;
 };
@@ -115,7 +116,7 @@ __device__ __forceinline__ bool mut_item(const MutualTcParams& p, int it, MutIte
   return w.a0 < w.n;
 }
 
-template <int PASS>
+template <int PASS, bool FOLD>
 __global__ void __launch_bounds__(m1::THREADS, 1)
     mutual_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
                      const __grid_constant__ CUtensorMap mapA1, const __grid_constant__ CUtensorMap mapB1,
@@ -142,7 +143,9 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
     for (int i = 0; i < NBB; ++i) {
       tc::bar_init(&sm.bfull[i], 1);
       tc::bar_init(&sm.bempty[i], 1);
+      tc::bar_init(&sm.bready[i], 2);
     }
+    for (int i = 0; i < 2; ++i) tc::bar_init(&sm.aready[i], 2);
     for (int i = 0; i < 8; ++i) tc::bar_init(&sm.hb[i >> 2][i & 3], QW - 1);
     for (int i = 0; i < 8; ++i) tc::bar_init(&sm.inext[i], 1);
     tc::bar_init(&sm.mdone, 1);
@@ -235,8 +238,8 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         for (int s = 0; s < nheads * nb; ++s, ++sg) {
           const int jb = s % nb;
           const int ab = na & 1, bb = sg % NBB, db = sg & 1;
-          if (jb == 0) ok = tc::bar_wait(&sm.afull[ab], (na >> 1) & 1, abort, kLimitNs);
-          if (ok) ok = tc::bar_wait(&sm.bfull[bb], (sg / NBB) & 1, abort, kLimitNs);
+          if (jb == 0) ok = tc::bar_wait(FOLD ? &sm.aready[ab] : &sm.afull[ab], (na >> 1) & 1, abort, kLimitNs);
+          if (ok) ok = tc::bar_wait(FOLD ? &sm.bready[bb] : &sm.bfull[bb], (sg / NBB) & 1, abort, kLimitNs);
           if (ok && sg >= 2) ok = tc::bar_wait(&sm.dfree[db], ((sg - 2) >> 1) & 1, abort, kLimitNs);
           if (!ok) break;
           tc::fence_after();
@@ -265,6 +268,99 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       if (!tc::bar_wait(&sm.mdone, 0, nullptr, kLimitNs)) set_status(p.status, OCCAM_ERR_TIMEOUT);
     }
     __syncwarp();
+  } else if (FOLD && (warp == 2 || warp == 3)) {
+    // ------------------------------------------------------------ fold warps
+    // Pass 2 with d1 = 72: dims 72-79 of the last K-step arrive zero-filled
+    // by the TMA box. Into dims 72-74 go 1.0 on the key side (A) and, on the
+    // query side (B), a three-term bf16 split of -L_u / c (each term the
+    // rounding of what the previous ones leave, so the three hold 24
+    // significant bits), so the MMA yields S - L_u / c and the softmax warps
+    // need only c times it. A query row past the segment gets -1e30, whose
+    // exponential is 0. In the 32-byte-swizzled rows, dims 72-79 (16-byte
+    // chunk 1 of row r) sit in chunk 1 ^ ((r >> 2) & 1). Warp 2 takes the
+    // first half of each tile's rows, warp 3 the second.
+    const float inv_c = 1.0f / p.scale_log2;
+    const int half = warp - 2;
+    const int64_t R = p.bt.total_rows;
+    uint32_t na = 0, nbk = 0;
+    for (int ii = 0;; ++ii) {
+      if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.inext[ii & 7], (ii >> 3) & 1, nullptr, kLimitNs))) {
+        sm.abort = 1;
+        set_status(p.status, OCCAM_ERR_TIMEOUT);
+        break;
+      }
+      const int it = *reinterpret_cast<volatile int*>(&sm.item[ii & 7]);
+      if (it < 0) break;
+      MutItem w;
+      mut_item<PASS>(p, it, w);
+      const int n = w.n;
+      const int64_t sb = p.bt.seg_off[w.seg];
+      const int nb = (n + BR - 1) / BR;
+      const int steps = min(kMutHeadGroup, H - w.h) * nb;
+      // -L of the block's query rows lane + 32 k, loaded a step ahead
+      // (clamped to the segment; rows past it are replaced below)
+      constexpr int KR = BR / 64;  // B rows per lane and step
+      float lpre[KR];
+      auto load_l = [&](int t) {
+        const int ht = w.h + t / nb, base = (t % nb) * BR + half * (BR / 2);
+#pragma unroll
+        for (int k = 0; k < KR; ++k)
+          lpre[k] = __ldcg(&p.lsum[(int64_t)ht * R + sb + min(base + lane + 32 * k, n - 1)]);
+      };
+      load_l(0);
+      bool ok = true;
+      for (int s = 0; s < steps; ++s) {
+        const int jb = s % nb;
+        if (jb == 0) {
+          const int ab = na & 1;
+          if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.afull[ab], (na >> 1) & 1, nullptr, kLimitNs))) {
+            ok = false;
+            break;
+          }
+          for (int r = half * (AR / 2) + lane; r < (half + 1) * (AR / 2); r += 32)
+            *reinterpret_cast<uint4*>(sm.a1[ab] + r * 32 + 16 * (1 ^ ((r >> 2) & 1))) =
+                make_uint4(0x3F803F80u, 0x00003F80u, 0u, 0u);  // bf16 1.0 in dims 72, 73, 74
+          tc::fence_proxy_async();
+          __syncwarp();
+          if (lane == 0) tc::bar_arrive(&sm.aready[ab]);
+          ++na;
+        }
+        const int bb = nbk % NBB;
+        if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.bfull[bb], (nbk / NBB) & 1, nullptr, kLimitNs))) {
+          ok = false;
+          break;
+        }
+        float cur[KR];
+#pragma unroll
+        for (int k = 0; k < KR; ++k) cur[k] = lpre[k];
+        if (s + 1 < steps) load_l(s + 1);
+#pragma unroll
+        for (int k = 0; k < KR; ++k) {
+          const int r = half * (BR / 2) + lane + 32 * k;
+          uint4 t4 = make_uint4(__bfloat16_as_ushort(__float2bfloat16_rn(-1e30f)), 0u, 0u, 0u);
+          if (jb * BR + r < n) {
+            const float y = cur[k] * inv_c;  // -L / c
+            const __nv_bfloat16 h1 = __float2bfloat16_rn(y);
+            const float r1 = y - __bfloat162float(h1);
+            const __nv_bfloat16 h2 = __float2bfloat16_rn(r1);
+            const float r2 = r1 - __bfloat162float(h2);
+            const __nv_bfloat16 h3 = __float2bfloat16_rn(r2);
+            t4.x = (uint32_t)__bfloat16_as_ushort(h1) | ((uint32_t)__bfloat16_as_ushort(h2) << 16);
+            t4.y = (uint32_t)__bfloat16_as_ushort(h3);
+          }
+          *reinterpret_cast<uint4*>(sm.b1[bb] + r * 32 + 16 * (1 ^ ((r >> 2) & 1))) = t4;
+        }
+        tc::fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) tc::bar_arrive(&sm.bready[bb]);
+        ++nbk;
+      }
+      if (!ok) {
+        sm.abort = 1;
+        set_status(p.status, OCCAM_ERR_TIMEOUT);
+        break;
+      }
+    }
   } else if (warp >= EPI0) {
     // ------------------------------------------------------------ softmax warps
     const int ew = warp - EPI0;
@@ -297,7 +393,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         const int h = w.h + s / nb;
         const int jb = s % nb;
         const int col0 = jb * BR + qtr * COLS;          // segment-relative index of this warp's column 0
-        if (PASS == 2) {
+        if (PASS == 2 && !FOLD) {
           // minus the log-sums of this warp's 64 query columns (past the
           // segment: -inf, which contributes 0) come by cp.async into a ring
           // of two step slots, one step ahead; the item's first step's are
@@ -374,7 +470,9 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
             float2 ap[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              float2 x = __ffma2_rn(make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), cc, nl[i]);
+              // FOLD: the accumulator already holds S - L / c
+              const float2 sv = make_float2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+              float2 x = FOLD ? __fmul2_rn(sv, cc) : __ffma2_rn(sv, cc, nl[i]);
               x.x = tc::ex2(x.x);
               x.y = tc::ex2(x.y);
               ap[i & 3] = __fadd2_rn(ap[i & 3], x);
@@ -461,10 +559,15 @@ __global__ void __launch_bounds__(256) mutual_reduce_kernel(MutualTcParams p) {
 void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mq1,
                       const CUtensorMap& mk1, int sms, cudaStream_t st) {
   const int smem = mutual_tc_smem_bytes();
-  cudaFuncSetAttribute(mutual_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  cudaFuncSetAttribute(mutual_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  mutual_tc_kernel<1><<<sms, m1::THREADS, smem, st>>>(mq, mk, mq1, mk1, p);
-  mutual_tc_kernel<2><<<sms, m1::THREADS, smem, st>>>(mk, mq, mk1, mq1, p);
+  cudaFuncSetAttribute(mutual_tc_kernel<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaFuncSetAttribute(mutual_tc_kernel<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaFuncSetAttribute(mutual_tc_kernel<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  mutual_tc_kernel<1, false><<<sms, m1::THREADS, smem, st>>>(mq, mk, mq1, mk1, p);
+  // with d1 = 72 the last K-step has free dims for the log-sums (see the fold warp)
+  if (p.d1 == 72)
+    mutual_tc_kernel<2, true><<<sms, m1::THREADS, smem, st>>>(mk, mq, mk1, mq1, p);
+  else
+    mutual_tc_kernel<2, false><<<sms, m1::THREADS, smem, st>>>(mk, mq, mk1, mq1, p);
   mutual_reduce_kernel<<<sms * 2, 256, 0, st>>>(p);
   count_launch(3);
 }

@@ -79,6 +79,13 @@ _BASE = [
         lambda1=0.5, beta1=3.0, targets={"n1_frac": 0.5, "count_frac": 0.222},
     ),
     Workload(
+        name="qwen3vl_b16",
+        description="Qwen3-VL-shaped, ragged batch 16 (the small case for kernel profiling): as qwen3vl_b32",
+        B=16, segs=1, vis=("uniform_step", 256, 4096, 4), regs=4, stage1="mutual", H1=16, d1=72,
+        sinks=("frac", 0.01), dup=None, M=("uniform", 32, 512), seed=5, query_bias=0.5,
+        lambda1=0.5, beta1=3.0, targets={"n1_frac": 0.5, "count_frac": 0.222},
+    ),
+    Workload(
         name="video_b4",
         description="video-shaped, batch 4: 16 frames x (1024 + 4 registers), 50% inter-frame duplicates, 1% sinks, 128 text tokens",
         B=4, segs=16, vis=("fixed", 1024), regs=4, stage1="cls", H1=16, d1=64,
