@@ -77,6 +77,23 @@ def test_prune_mutual_matches_oracle(d1):
     check_prune(b, gpu, 0.5, 1.1)
 
 
+@pytest.mark.parametrize("d1", [72, 64])
+def test_prune_mutual_late_large_logits(d1):
+    """Keys past the first 256 of a segment with logits far above the first
+    block's (their K1 rows scaled by 64, exactly in bf16; about 340 in log2
+    units above it): the first mutual pass's online softmax rescales its
+    running sums by 2^-340 and below, and the scores still match the oracle."""
+    b = _tiny(B=2, segs=1, P=(700, 300), R=4, M=(20, 50), stage1="mutual", d1=d1, seed=31, query_bias=0.5,
+              beta1=2.0)
+    m = b["meta"]
+    a, z = int(m["seg_off_host"][0]), int(m["seg_off_host"][1])
+    K1 = b["K1"]
+    K1[a + 256:z] = (K1[a + 256:z].float() * 64).to(K1.dtype)
+    gpu = run_prune(b, 0.5, 1.1)
+    assert gpu["status"] == 0
+    check_prune(b, gpu, 0.5, 1.1)
+
+
 @pytest.mark.parametrize("name", ["llava15_b1", "llavanext_b8"])
 def test_small_workloads(name):
     w = get_config(name)
