@@ -126,9 +126,8 @@ int num_sms() {
   return n;
 }
 
-size_t finalize_smem_bytes(int rows, bool cls) {
-  return ((size_t)rows * ((cls ? 64 : 0) + 4 + 1) + 15) & ~(size_t)15;
-}
+// the finalize kernel's shared copy of a segment: s1 (4 B) and role (1 B) per row
+size_t finalize_smem_bytes(int rows) { return ((size_t)rows * (4 + 1) + 15) & ~(size_t)15; }
 
 void set_smem_attrs() {
   static std::once_flag once;
@@ -136,7 +135,7 @@ void set_smem_attrs() {
     cudaFuncSetAttribute(stage1_logits_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          stage1_logits_smem_bytes());
     cudaFuncSetAttribute(stage1_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)finalize_smem_bytes(16 * kFinalizeSmemRows, false));
+                         (int)finalize_smem_bytes(kFinalizeSmemRows));
   });
 }
 
@@ -344,7 +343,7 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
     p.bt = bt;
     p.q_cls = static_cast<const __nv_bfloat16*>(a->q);
     p.K1 = static_cast<const __nv_bfloat16*>(a->K1);
-    p.scale = (float)(1.0 / std::sqrt((double)a->d1));
+    p.scale = (float)(1.4426950408889634 / std::sqrt((double)a->d1));  // logits in log2 units
     p.logits = at<float>(ws, L.stats1);
     p.status = status;
     const int64_t tiles = cdiv(b->total_rows, 16);
@@ -396,13 +395,13 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   p.logits = cls ? at<float>(ws, L.stats1) : nullptr;
   p.q_cls = cls ? static_cast<const __nv_bfloat16*>(a1->q) : nullptr;
   p.k_cls = cls ? static_cast<const __nv_bfloat16*>(a1->k_cls) : nullptr;
-  p.scale = cls ? (float)(1.0 / std::sqrt((double)a1->d1)) : 1.f;
+  p.scale = cls ? (float)(1.4426950408889634 / std::sqrt((double)a1->d1)) : 1.f;  // log2 units, as the logits
   p.s1_out = s1;
   p.n_eff = cls ? n_eff : nullptr;
   p.s2_zero = cls ? s2_zero : nullptr;
-  // a segment's logits ([CLS] mode, 64 B/row), s1 (4 B/row) and roles
-  // (1 B/row) are staged in shared memory when it fits (at most 96 KB)
-  p.smem_rows = s1 ? (int)std::min<int64_t>(b->max_seg_rows, cls ? kFinalizeSmemRows : 16 * kFinalizeSmemRows) : 0;
+  // a segment's s1 (4 B/row) and roles (1 B/row) are staged in shared
+  // memory when it fits (at most 110 KB)
+  p.smem_rows = s1 ? (int)std::min<int64_t>(b->max_seg_rows, kFinalizeSmemRows) : 0;
   p.s1 = s1;
   p.keep_in = keep_in;
   p.lambda1 = lambda1;
@@ -421,7 +420,7 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   if (plan) p.plan = *plan;
   p.zero_count_out = count_out;
   p.zero_count_vis = count_vis;
-  stage1_finalize_kernel<<<b->S_tot, 256, finalize_smem_bytes(p.smem_rows, cls), st>>>(p);
+  stage1_finalize_kernel<<<b->S_tot, 256, finalize_smem_bytes(p.smem_rows), st>>>(p);
   count_launch();
   trace.mark(st);
   return cuda_ok();

@@ -90,6 +90,55 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* tmp, int* total)
   return res;
 }
 
+// 2^x with the hardware approximation (relative error about 2^-22),
+// flushing subnormal results to zero; 2^-inf = 0
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// N exclusive prefix sums over the block at once (three barriers in all, as
+// for one): excl[k] = sum of v[k] over the threads before this one, total[k]
+// = the block's sum. tmp: N * 33 ints of shared memory.
+template <int N>
+__device__ __forceinline__ void block_exclusive_scan_n(const int (&v)[N], int (&excl)[N], int (&total)[N], int* tmp) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  int incl[N];
+#pragma unroll
+  for (int k = 0; k < N; ++k) {
+    incl[k] = v[k];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, incl[k], o);
+      if (lane >= o) incl[k] += n;
+    }
+    if (lane == 31) tmp[k * 33 + warp] = incl[k];
+  }
+  __syncthreads();
+  if (warp == 0) {
+#pragma unroll
+    for (int k = 0; k < N; ++k) {
+      const int w = lane < nw ? tmp[k * 33 + lane] : 0;
+      int wi = w;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(0xffffffffu, wi, o);
+        if (lane >= o) wi += n;
+      }
+      if (lane < nw) tmp[k * 33 + lane] = wi - w;
+      if (lane == nw - 1) tmp[k * 33 + 32] = wi;
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < N; ++k) {
+    excl[k] = tmp[k * 33 + warp] + incl[k] - v[k];
+    total[k] = tmp[k * 33 + 32];
+  }
+  __syncthreads();
+}
+
 // Index of the interval of `off` ([n+1] ascending) that holds x: off[i] <= x < off[i+1].
 template <typename T>
 __device__ __forceinline__ int upper_interval(const T* off, int n, int64_t x) {

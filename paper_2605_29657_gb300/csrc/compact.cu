@@ -39,12 +39,19 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   __shared__ long long s_prefix;
   __shared__ int s_tile;
   __shared__ int64_t s_ro[kScanSmemSamples + 1];
+  __shared__ float s_tau[kScanSmemSamples];
   const int tid = threadIdx.x;
   if (tid == 0) s_tile = atomicAdd(p.ticket, 1);
+  // the row offsets and (Stage-II threshold mode) the samples' thresholds,
+  // loaded while the ticket is drawn
   const bool ro_smem = p.bt.B <= kScanSmemSamples;
-  if (ro_smem)
+  if (ro_smem) {
     for (int b = tid; b <= p.bt.B; b += blockDim.x) s_ro[b] = p.bt.row_off[b];
+    if (p.mode != 0)
+      for (int b = tid; b < p.bt.B; b += blockDim.x) s_tau[b] = p.tau2[b];
+  }
   const int64_t* row_off = ro_smem ? s_ro : p.bt.row_off;
+  const float* tau2 = ro_smem ? s_tau : p.tau2;
   __syncthreads();
   const int64_t tile = s_tile;
   const int64_t R = p.bt.total_rows;
@@ -73,7 +80,7 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
         k = p.keep_registers != 0;
         vis = false;
       } else {
-        k = (p.keep1[r] != 0) && (p.s2[r] >= p.tau2[samp]);
+        k = (p.keep1[r] != 0) && (p.s2[r] >= tau2[samp]);
         vis = k;
       }
       if (p.keep_out) p.keep_out[r] = k ? 1 : 0;

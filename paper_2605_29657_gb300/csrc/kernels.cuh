@@ -13,7 +13,7 @@ constexpr int kFusedKeyRows4 = 256;     // key rows per head one CTA of a 4-CTA 
 constexpr int kFusedKeyRows8 = 224;     // the same for an 8-CTA cluster (its exchange buffers take more shared memory)
 constexpr int kFusedKeyRows16 = 224;    // and for a 16-CTA cluster (non-portable cluster size)
 constexpr int kFusedPartialWarps = 4;   // warps per CTA of the fused kernel that write an s2(r) partial
-constexpr int kFinalizeSmemRows = 1400; // Stage-I finalize stages a [CLS] segment in shared memory up to this many rows
+constexpr int kFinalizeSmemRows = 22400; // Stage-I finalize stages a segment's s1 and roles in shared memory up to this many rows
 
 // Whether a sample with n1 S1 keys and M text tokens fits the fused kernel
 // with C CTAs per cluster: each CTA takes ceil(n1 / C) S1 keys (padded to 32)
@@ -52,8 +52,8 @@ struct Stage1ClsParams {
   BatchDev bt;
   const __nv_bfloat16* q_cls;
   const __nv_bfloat16* K1;
-  float scale;
-  float* logits;  // [rows, 16] per-head [CLS] logits
+  float scale;  // log2(e) / sqrt(d1): [CLS] logits in log2 units
+  float* logits;  // [rows, 16] per-head [CLS] logits in log2 units
   int* status;
 };
 
@@ -137,11 +137,11 @@ struct Stage1FinalizeParams {
   const float* logits;            // nullable: s1 is given instead
   const __nv_bfloat16* q_cls;     // [CLS] mode
   const __nv_bfloat16* k_cls;     // nullable
-  float scale;
+  float scale;  // log2(e) / sqrt(d1): [CLS] logits in log2 units
   float* s1_out;                  // [CLS] mode: where s1 is written
   float* n_eff;                   // nullable, [CLS] mode: [S_tot, 16] effective number of attended keys per head
   float* s2_zero;                 // nullable: zeroed per row (Stage-II max accumulator)
-  int smem_rows;                  // segments up to this many rows stage their logits in shared memory
+  int smem_rows;                  // segments up to this many rows stage their s1 and roles in shared memory
   const float* s1;          // nullable when keep_in is given
   const uint8_t* keep_in;   // nullable: S1 membership of visual rows given instead of tested
   float lambda1;

@@ -23,9 +23,17 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
   // samples take the wider cluster, whose CTAs hold fewer keys and finish
   // each head sooner.
   int wide = 0, hsg = 1;  // hsg: head groups of a split tile (1: no split)
+  // the first blockDim.x samples' text lengths and S1 sizes, loaded together
+  // up front (one memory round trip instead of two in a row)
+  int M0 = 0, n10 = 0;
+  if (tid < p.bt.B) {
+    M0 = (int)(p.bt.text_off[tid + 1] - p.bt.text_off[tid]);
+    n10 = *((volatile int32_t*)&p.n1[tid]);
+  }
   if (p.use_fused) {
     int tiles = 0;
-    for (int b = tid; b < p.bt.B; b += blockDim.x) tiles += (int)((p.bt.text_off[b + 1] - p.bt.text_off[b] + 127) / 128);
+    for (int b = tid; b < p.bt.B; b += blockDim.x)
+      tiles += b == tid ? (M0 + 127) / 128 : (int)((p.bt.text_off[b + 1] - p.bt.text_off[b] + 127) / 128);
     int total_tiles;
     block_exclusive_scan(tiles, tmp, &total_tiles);
     wide = total_tiles <= p.res16 ? 16 : total_tiles <= p.res8 ? 8 : 0;
@@ -46,8 +54,8 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
     const int bb = b0 + tid;
     int nA = 0, nB = 0, nF = 0, nF8 = 0, nF16 = 0;
     if (bb < p.bt.B) {
-      const int M = (int)(p.bt.text_off[bb + 1] - p.bt.text_off[bb]);
-      const int n1 = *((volatile int32_t*)&p.n1[bb]);
+      const int M = b0 == 0 ? M0 : (int)(p.bt.text_off[bb + 1] - p.bt.text_off[bb]);
+      const int n1 = b0 == 0 ? n10 : *((volatile int32_t*)&p.n1[bb]);
       // the fused tensor-core kernel takes a sample when its S1 keys and its
       // causal text keys fit the cluster's TMEM / shared memory
       const bool w16 = wide == 16 && fused_fits(16, n1, M, p.H);
@@ -76,14 +84,15 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
     const int nS = nF * kFusedSlotsPerItem + nF8 * kFusedSlotsPerItem8 + nF16 / hsg * kFusedSlotsPerItem16 +
                    nB;  // s2(r) partial slots of this sample (a split tile's items share its slots)
     const int nHS = hsg > 1 ? nF16 / hsg : 0;  // this sample's head-split tiles
-    int totA, totB, totF, totF8, totF16, totS, totHS;
-    const int offA = runA + block_exclusive_scan(nA, tmp, &totA);
-    const int offB = runB + block_exclusive_scan(nB, tmp, &totB);
-    const int offF = runF + block_exclusive_scan(nF, tmp, &totF);
-    const int offF8 = runF8 + block_exclusive_scan(nF8, tmp, &totF8);
-    const int offF16 = runF16 + block_exclusive_scan(nF16, tmp, &totF16);
-    const int offS = runS + block_exclusive_scan(nS, tmp, &totS);
-    const int offHS = runHS + block_exclusive_scan(nHS, tmp, &totHS);
+    // the seven item and slot counts, scanned together
+    __shared__ int mtmp[7 * 33];
+    const int cnt[7] = {nA, nB, nF, nF8, nF16, nS, nHS};
+    int ex[7], tot[7];
+    block_exclusive_scan_n<7>(cnt, ex, tot, mtmp);
+    const int totA = tot[0], totB = tot[1], totF = tot[2], totF8 = tot[3], totF16 = tot[4], totS = tot[5],
+              totHS = tot[6];
+    const int offA = runA + ex[0], offB = runB + ex[1], offF = runF + ex[2], offF8 = runF8 + ex[3],
+              offF16 = runF16 + ex[4], offS = runS + ex[5], offHS = runHS + ex[6];
     if (bb < p.bt.B) {
       for (int i = 0; i < nF; ++i)
         if (offF + i < p.maxF) p.itemsF[offF + i] = make_int4(bb, i * 128, offS + i * kFusedSlotsPerItem, 0);

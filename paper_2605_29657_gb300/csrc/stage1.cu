@@ -10,7 +10,8 @@ namespace occam {
 
 // ============================================================================
 // [CLS] logits (Sec. 3.4, Eq. 4): l[row][h] = q_cls[seg(row), h] . K1[row, h]
-// / sqrt(d1) for every visual and register row. The softmax over the
+// / sqrt(d1) for every visual and register row, stored in log2 units (times
+// log2(e)), so that the finalize kernel's exponentials are plain exp2. The softmax over the
 // segment's rows and the head mean are taken by stage1_finalize_kernel from
 // these logits (64 bytes per row), so this kernel is a plain stream over K1:
 // persistent CTAs each take a contiguous range of 16-row tiles and pull them
@@ -102,7 +103,7 @@ __global__ void __launch_bounds__(cls::kThreads) stage1_logits_kernel(Stage1ClsP
       acc += __shfl_xor_sync(0xffffffffu, acc, 1);
       acc += __shfl_xor_sync(0xffffffffu, acc, 2);
       acc += __shfl_xor_sync(0xffffffffu, acc, 4);
-      if (kv == 0 && rr < rows) p.logits[row * H + my_h] = acc * p.scale;
+      if (kv == 0 && rr < rows) p.logits[row * H + my_h] = acc * p.scale;  // log2 units
     }
     __syncthreads();
     if (tid == 0 && it + kStages < ntiles) {
@@ -128,77 +129,122 @@ int stage1_logits_smem_bytes() { return cls::kSmem; }
 // mask (registers always in), the row roles, and the order-preserving list
 // of the segment's S1 rows. One CTA per segment.
 // ============================================================================
+// Merges the softmax statistics of a part into (M, Z, T), all in log2 units:
+// M the part's max, Z = sum 2^(x - M), T = sum 2^(x - M) (x - M). A part
+// with max -inf is empty.
+__device__ __forceinline__ void merge_softmax_stats(float& M, float& Z, float& T, float m2, float z2, float t2) {
+  if (m2 == -INFINITY) return;
+  if (M == -INFINITY) {
+    M = m2;
+    Z = z2;
+    T = t2;
+  } else if (m2 > M) {
+    const float d = M - m2, f = fast_exp2(d);
+    T = fmaf(f, fmaf(d, Z, T), t2);
+    Z = fmaf(Z, f, z2);
+    M = m2;
+  } else {
+    const float d = m2 - M, f = fast_exp2(d);
+    T = fmaf(f, fmaf(d, z2, t2), T);
+    Z = fmaf(z2, f, Z);
+  }
+}
+
 // [CLS] mode (Sec. 3.4, Eq. 4; App. A, Eq. 10): per head h the softmax of the
-// [CLS] row over {k_cls} u rows(segment) from the logits, s1 = mean over
-// heads. lg: the segment's logits [n][16] (shared or global memory); s1 is
-// written to s1_out (global) and, when given, to s1_loc (shared).
+// [CLS] row over {k_cls} u rows(segment), s1 = mean over heads. The logits
+// come in log2 units (the logits kernel scales by log2(e) / sqrt(d1)), so
+// 2^(x - max) is each exponential. One pass keeps per thread and head the
+// running max, the sum of exponentials and, for the entropy, the sum of
+// e (x - max); the block merges them in fixed order; a second pass forms s1
+// per row. Both read the logits from global memory (written just before by
+// the logits kernel: L2, and L1 for the second pass). s1 is written to s1_out
+// (global) and, when given, to s1_loc (shared).
 __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, int seg, int64_t sb, int n,
-                                               const float* lg, float* s1_loc) {
+                                               float* s1_loc) {
   constexpr int H = 16, D = 64;
-  __shared__ float red[16][17], red2[16][17];
+  __shared__ float rm[16][17], rz[16][17], rt[16][17];
   __shared__ float gmax[16], ginv[16], lcls_s[16];
   const int tid = threadIdx.x;
-  if (tid < 256) {
+  // thread t takes head (t & 15) of rows (t >> 4) + 16 k: a warp reads 32
+  // consecutive floats per row pair. Up to 32 rows' loads are in flight at
+  // once (issued before the [CLS] key's dot product below, which they
+  // overlap), so a segment of up to 512 rows costs one L2 round trip.
+  constexpr int KC = 32;
+  const float* lg = p.logits + sb * H;
+  const int h = tid & 15, j = tid >> 4;
+  float x[KC];
+  auto load_chunk = [&](int r0) {
+#pragma unroll
+    for (int u = 0; u < KC; ++u) {
+      const int r = r0 + 16 * u;
+      x[u] = r < n ? __ldg(&lg[(int64_t)r * H + h]) : -INFINITY;
+    }
+  };
+  load_chunk(j);
+  {
     // l_cls,h: 16 threads per head, 4 dims each
-    const int h = tid >> 4, sub = tid & 15;
+    const int hh = tid >> 4, sub = tid & 15;
     float acc = 0.f;
     if (p.k_cls) {
-      const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + h) * D + sub * 4;
-      const __nv_bfloat16* kp = p.k_cls + ((int64_t)seg * H + h) * D + sub * 4;
+      const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + hh) * D + sub * 4;
+      const __nv_bfloat16* kp = p.k_cls + ((int64_t)seg * H + hh) * D + sub * 4;
 #pragma unroll
       for (int d = 0; d < 4; ++d) acc = fmaf(__bfloat162float(qp[d]), __bfloat162float(kp[d]), acc);
     }
 #pragma unroll
     for (int o = 8; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (sub == 0) lcls_s[h] = p.k_cls ? acc * p.scale : -INFINITY;
+    if (sub == 0) lcls_s[hh] = p.k_cls ? acc * p.scale : -INFINITY;
   }
-  // thread t takes head (t & 15) of rows (t >> 4) + 16 k: a warp reads 32
-  // consecutive floats per step
-  const int h = tid & 15, j = tid >> 4;
-  float m = -INFINITY;
-  for (int r = j; r < n; r += 16) m = fmaxf(m, lg[r * H + h]);
-  red[j][h] = m;
-  __syncthreads();
-  if (tid < 16) {
-    float mm = lcls_s[tid];
-    for (int k = 0; k < 16; ++k) mm = fmaxf(mm, red[k][tid]);
-    gmax[tid] = mm;
-  }
-  __syncthreads();
-  const float mh = gmax[h];
-  float z = 0.f, t = 0.f;  // t: sum of e (l - max), for the entropy
-  for (int r = j; r < n; r += 16) {
-    const float x = lg[r * H + h] - mh;
-    const float e = expf(x);
-    z += e;
-    t = fmaf(e, x, t);
-  }
-  red[j][h] = z;
-  red2[j][h] = t;
-  __syncthreads();
-  if (tid < 16) {
-    const bool self = lcls_s[tid] != -INFINITY;
-    const float xc = self ? lcls_s[tid] - gmax[tid] : 0.f;
-    float zz = self ? expf(xc) : 0.f;
-    float tt = zz * xc;
-    for (int k = 0; k < 16; ++k) {
-      zz += red[k][tid];
-      tt += red2[k][tid];
+  float m = -INFINITY, z = 0.f, t = 0.f;
+  for (int r0 = j;;) {
+    float cm = x[0];
+#pragma unroll
+    for (int u = 1; u < KC; ++u) cm = fmaxf(cm, x[u]);
+    if (cm > m) {
+      // the running sums move to the new max
+      if (m != -INFINITY) {
+        const float d = m - cm, f = fast_exp2(d);
+        t = f * fmaf(d, z, t);
+        z *= f;
+      }
+      m = cm;
     }
-    ginv[tid] = 1.0f / zz;
+#pragma unroll
+    for (int u = 0; u < KC; ++u) {
+      const float d = x[u] - m;
+      const float e = fast_exp2(d);  // 0 for rows past the segment (-inf)
+      z += e;
+      t = d > -INFINITY ? fmaf(e, d, t) : t;
+    }
+    r0 += 16 * KC;
+    if (r0 >= n) break;
+    load_chunk(r0);
+  }
+  rm[j][h] = m;
+  rz[j][h] = z;
+  rt[j][h] = t;
+  __syncthreads();
+  if (tid < 16) {
+    // the [CLS] key itself, then the 16 partials in order
+    float M = -INFINITY, Z = 0.f, T = 0.f;
+    merge_softmax_stats(M, Z, T, lcls_s[tid], 1.f, 0.f);
+    for (int k = 0; k < 16; ++k) merge_softmax_stats(M, Z, T, rm[k][tid], rz[k][tid], rt[k][tid]);
+    gmax[tid] = M;
+    ginv[tid] = 1.0f / Z;
     // entropy of the head's distribution a = e / Z over the keys:
-    // H = -sum a log a = log Z - (sum e (l - max)) / Z; n_eff = exp(H)
-    if (p.n_eff) p.n_eff[(int64_t)seg * H + tid] = expf(logf(zz) - tt / zz);
+    // H = -sum a ln a = ln Z - (sum e (l - max)) / Z, with sum e (l - max) =
+    // ln 2 * T in log2 units; n_eff = exp(H)
+    if (p.n_eff) p.n_eff[(int64_t)seg * H + tid] = expf(logf(Z) - 0.69314718055994531f * T / Z);
   }
   __syncthreads();
   for (int r = tid; r < n; r += blockDim.x) {
-    const float4* lp = reinterpret_cast<const float4*>(lg + r * H);
+    const float4* lp = reinterpret_cast<const float4*>(lg + (int64_t)r * H);
     float acc = 0.f;
 #pragma unroll
     for (int k = 0; k < H / 4; ++k) {
-      const float4 l = lp[k];
-      acc += expf(l.x - gmax[4 * k]) * ginv[4 * k] + expf(l.y - gmax[4 * k + 1]) * ginv[4 * k + 1] +
-             expf(l.z - gmax[4 * k + 2]) * ginv[4 * k + 2] + expf(l.w - gmax[4 * k + 3]) * ginv[4 * k + 3];
+      const float4 l = __ldg(lp + k);
+      acc += fast_exp2(l.x - gmax[4 * k]) * ginv[4 * k] + fast_exp2(l.y - gmax[4 * k + 1]) * ginv[4 * k + 1] +
+             fast_exp2(l.z - gmax[4 * k + 2]) * ginv[4 * k + 2] + fast_exp2(l.w - gmax[4 * k + 3]) * ginv[4 * k + 3];
     }
     const float v = acc * (1.0f / H);
     p.s1_out[sb + r] = v;
@@ -208,10 +254,9 @@ __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, in
   __syncthreads();
 }
 
-// 256 threads, one CTA per segment. With n <= smem_rows the segment's
-// logits ([CLS] mode), s1 and roles are staged in shared memory (one
-// coalesced pass over global memory each way); larger segments work from
-// global memory.
+// 256 threads, one CTA per segment. With n <= smem_rows the segment's s1
+// and roles are staged in shared memory; larger segments work from global
+// memory.
 __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizeParams p) {
   extern __shared__ float4 fin_smem[];
   __shared__ int tmp[40];
@@ -228,35 +273,13 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   const int n = (int)(se - sb);
   const int ra = p.bt.reg_off[seg], rb = p.bt.reg_off[seg + 1];
   const bool staged = n <= p.smem_rows;
-  // shared layout for a staged segment: [logits (CLS mode)][s1][role]
-  float* lg_loc = reinterpret_cast<float*>(fin_smem);
-  float* s1_loc = lg_loc + (p.logits ? (size_t)p.smem_rows * 16 : 0);
+  // shared layout for a staged segment: [s1][role]
+  float* s1_loc = reinterpret_cast<float*>(fin_smem);
   uint8_t* role_loc = reinterpret_cast<uint8_t*>(s1_loc + p.smem_rows);
 
   const float* s1g = p.logits ? p.s1_out : p.s1;  // the segment's s1 in global memory
   if (p.logits) {
-    const float* lg = p.logits + sb * 16;
-    if (staged) {
-      // eight independent 16-byte loads in flight per thread, then the stores
-      const float4* __restrict__ src = reinterpret_cast<const float4*>(lg);
-      const int nv = n * 4;
-      for (int base = 0; base < nv; base += 8 * 256) {
-        float4 t[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int i = base + u * 256 + tid;
-          if (i < nv) t[u] = __ldg(src + i);
-        }
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int i = base + u * 256 + tid;
-          if (i < nv) fin_smem[i] = t[u];
-        }
-      }
-      __syncthreads();
-      lg = lg_loc;
-    }
-    cls_softmax_s1(p, seg, sb, n, lg, staged ? s1_loc : nullptr);
+    cls_softmax_s1(p, seg, sb, n, staged ? s1_loc : nullptr);
   } else if (staged) {
     for (int r = tid; r < n; r += blockDim.x) s1_loc[r] = s1g[sb + r];
   }
