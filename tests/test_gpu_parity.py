@@ -77,6 +77,19 @@ def test_prune_mutual_matches_oracle(d1):
     check_prune(b, gpu, 0.5, 1.1)
 
 
+@pytest.mark.parametrize("d1", [72, 64, 80])
+def test_prune_mutual_segment_edges(d1):
+    """Mutual Stage I on segments of 5 rows (one partial key block), 133 (a
+    second 128-row tile of one row past the first), 260 (a second 256-key
+    block) and 512 (whole tiles and blocks), for each supported d1 (72 takes
+    the log-sums folded into the MMA, 64 and 80 the shared-memory ring)."""
+    b = _tiny(B=4, segs=1, P=(1, 129, 256, 508), R=4, M=(3, 40, 17, 128), stage1="mutual", d1=d1, seed=33,
+              query_bias=0.5, beta1=2.0)
+    gpu = run_prune(b, 0.5, 1.1)
+    assert gpu["status"] == 0
+    check_prune(b, gpu, 0.5, 1.1)
+
+
 @pytest.mark.parametrize("d1", [72, 64])
 def test_prune_mutual_late_large_logits(d1):
     """Keys past the first 256 of a segment with logits far above the first
