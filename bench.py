@@ -649,7 +649,7 @@ def run_ours(args, rank, world, local):
         next_rows = {
             "lambda2_budget": {"ms": lam_ms, "target_rows": K_tar, "candidates": int(ncand.item()),
                                "lambda2": float(lam.item()), "calibrated_lambda2": w.lambda2,
-                               "how": "radix select of the K-th largest s2/ref2 over the step's S1 rows"},
+                               "how": "radix select of the K-th largest s2/ref2 over the step's S1 rows (11-bit digits, grid-wide histograms; one pass of kept counts for the fp32 product rule)"},
             "register_construction": {"ms": reg_ms, "rows": meta["total_rows"], "channels": 10,
                                       "how": "in place on hidden [rows, 4096] bf16, per segment"},
             "n_eff": "computed in the Stage-I finalize of every timed step ([CLS] mode, optional output)",

@@ -82,6 +82,7 @@ WsLayout ws_layout(const occam_batch* b, int H1, int H2) {
   L.tau2 = take(B * 4);
   L.stats1_rows = rows;
   L.stats1 = take(rows * (H1 > 0 ? H1 : 1) * 8);
+  L.l2sel = take(kL2SelBytes);
   L.total = off;
   return L;
 }
@@ -1001,10 +1002,22 @@ int occam_calibrate_lambda2(const occam_batch* batch, const float* s2, const flo
   p.role = at<uint8_t>(workspace, L.role);
   p.target = target_count;
   p.keys = reinterpret_cast<uint32_t*>(at<int32_t>(workspace, L.dense));
+  p.sel = at<unsigned char>(workspace, L.l2sel);
   p.lambda2 = lambda2_out;
   p.n_candidates = n_candidates;
-  lambda2_select_kernel<<<1, 1024, 0, st>>>(p);
-  count_launch();
+  // keys and top-digit histogram, then per digit a one-CTA bucket choice and
+  // the next digit's histogram, the window of kept counts, the choice
+  OCCAM_CUDA(cudaMemsetAsync(p.sel, 0, kL2SelBytes, st));
+  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(cdiv(batch->total_rows, 256), (int64_t)num_sms() * 4));
+  l2_keys_kernel<<<grid, 256, 0, st>>>(p);
+  l2_select_kernel<<<1, 1024, 0, st>>>(p, 0);
+  l2_hist_kernel<<<grid, 256, 0, st>>>(p, 1);
+  l2_select_kernel<<<1, 1024, 0, st>>>(p, 1);
+  l2_hist_kernel<<<grid, 256, 0, st>>>(p, 2);
+  l2_select_kernel<<<1, 1024, 0, st>>>(p, 2);
+  l2_window_kernel<<<grid, 256, 0, st>>>(p);
+  l2_finish_kernel<<<1, 1024, 0, st>>>(p);
+  count_launch(8);
   return cuda_ok();
 }
 

@@ -221,6 +221,7 @@ struct WsLayout {
   size_t status, counters, role, keep1, s1, s2, ref1, dense, n1, n1_vis;
   size_t itemsHS, ppart, itemA_off, itemB_off, stats2, refpart, ref2, tau2, done, scan_state, seg_state, stats1, itemsF, itemsF8, itemsF16,
       slot_off;
+  size_t l2sel;                 // lambda2 selection scratch (kL2SelBytes)
   size_t zero_begin, zero_end;  // the accumulators every prune call zeroes (one contiguous range)
   size_t total;
   int64_t maxA, maxB, maxF, maxSlots, scan_tiles, stats1_rows;

@@ -303,103 +303,196 @@ __device__ int lambda2_kept(const Lambda2Params& p, float lam, int* s_cnt) {
   return tot;
 }
 
-// lambda2_select_kernel: one CTA of 1,024 threads. Each candidate row (a
-// visual S1 row of a sample with ref2 > 0) gets the key 2^31 | bits(s2 /
-// ref2), with an IEEE round-to-nearest fp32 quotient >= 0 whose bit pattern
-// orders like its value; every other row gets key 0, below every candidate.
-// The K-th largest key is then found most significant byte first: per byte,
-// a histogram of the keys that match the bytes chosen so far (one 256-bin
-// histogram per warp, then summed), and the bucket where the running count
-// from the top reaches K. With K <= the candidate count the result is the
-// K-th largest candidate ratio. The rule applies lambda2 as one fp32 product
+// lambda2 budget matching (App. A, Eq. 19), over all SMs. Each candidate
+// row (a visual S1 row of a sample with ref2 > 0) gets the key 2^31 |
+// bits(s2 / ref2), with an IEEE round-to-nearest fp32 quotient >= 0 whose bit
+// pattern orders like its value; every other row gets key 0, below every
+// candidate. The K-th largest key is found eleven bits at a time (bits
+// 31-21, 20-10, 9-0): a grid-wide histogram of the keys that match the digits
+// chosen so far, then one CTA picks the bucket where the running count from
+// the top reaches K. With K <= the candidate count the result is the K-th
+// largest candidate ratio. The rule applies lambda2 as one fp32 product
 // (s2 >= fl(lambda2 * ref2)), whose rounding can disagree with the
-// quotient's by an ulp or two: the ratio is then moved by single fp32 steps
-// to the largest value under which that test keeps at least K rows.
-__global__ void __launch_bounds__(1024) lambda2_select_kernel(Lambda2Params p) {
-  __shared__ uint32_t hist[32][256];
-  __shared__ uint32_t tot[256];
-  __shared__ uint32_t s_prefix, s_k;
-  __shared__ int s_cnt;
-  const int tid = threadIdx.x, warp = tid >> 5;
-  const int64_t R = p.bt.total_rows;
-  if (tid == 0) s_cnt = 0;
+// quotient's by an ulp or two: the kept counts of the ratio and its
+// neighbours up to kL2Window fp32 steps either way are taken in one more
+// grid pass, and the largest of them that keeps at least K rows is the
+// result (single steps beyond the window, should the answer lie there).
+namespace {
+struct L2Sel {
+  uint32_t prefix;  // the key's digits chosen so far
+  int32_t k;        // rank still sought among the keys matching prefix
+  int32_t done;     // the result is already written (K <= 0 or K > candidates)
+  int32_t n;        // candidates
+  unsigned long long kept[2 * kL2Window + 1];  // kept counts of lambda0 stepped by -W..W
+  uint32_t hist[3][kL2Digits];
+};
+static_assert(sizeof(L2Sel) <= kL2SelBytes, "lambda2 selection scratch");
+
+__device__ __forceinline__ L2Sel* l2sel(const Lambda2Params& p) { return reinterpret_cast<L2Sel*>(p.sel); }
+
+// the level's digit shift and the mask of the digits above it
+__device__ __forceinline__ int l2_shift(int level) { return level == 0 ? 21 : level == 1 ? 10 : 0; }
+__device__ __forceinline__ uint32_t l2_mask_above(int level) {
+  return level == 0 ? 0u : level == 1 ? 0xFFE00000u : 0xFFFFFC00u;
+}
+
+// lambda0 stepped by j fp32 steps (j < 0: down, toward 0)
+__device__ __forceinline__ float l2_step(float lam, int j) {
+  for (; j < 0; ++j) lam = nextafterf(lam, 0.f);
+  for (; j > 0; --j) lam = nextafterf(lam, __int_as_float(0x7f800000));
+  return lam;
+}
+}  // namespace
+
+// keys of every row and the histogram of their top digit
+__global__ void __launch_bounds__(256) l2_keys_kernel(Lambda2Params p) {
+  __shared__ uint32_t h[kL2Digits];
+  L2Sel* st = l2sel(p);
+  for (int i = threadIdx.x; i < kL2Digits; i += blockDim.x) h[i] = 0;
   __syncthreads();
+  const int64_t R = p.bt.total_rows;
   int cnt = 0;
-  for (int64_t r = tid; r < R; r += blockDim.x) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < R; r += (int64_t)gridDim.x * blockDim.x) {
     const int b = upper_interval(p.bt.row_off, p.bt.B, r);
     const float ref = p.ref2[b];
     uint32_t key = 0;
     if (p.keep1[r] && p.role[r] == 0 && ref > 0.f) {
       key = 0x80000000u | __float_as_uint(__fdiv_rn(p.s2[r], ref));
+      atomicAdd(&h[key >> 21], 1u);
       ++cnt;
     }
     p.keys[r] = key;
   }
-  atomicAdd(&s_cnt, cnt);
+  cnt = __reduce_add_sync(0xffffffffu, cnt);
+  if ((threadIdx.x & 31) == 0 && cnt) atomicAdd(&st->n, cnt);
   __syncthreads();
-  const int64_t n = s_cnt;
-  if (p.n_candidates && tid == 0) *p.n_candidates = (int32_t)n;
-  if (p.target <= 0 || p.target > n) {
-    // K <= 0: no lambda2 keeps nothing but +inf; K > n: 0 keeps every candidate
-    if (tid == 0) *p.lambda2 = p.target <= 0 ? __int_as_float(0x7f800000) : 0.f;
-    return;
+  for (int i = threadIdx.x; i < kL2Digits; i += blockDim.x)
+    if (h[i]) atomicAdd(&st->hist[0][i], h[i]);
+}
+
+// histogram of the level's digit over the keys that match the digits above it
+__global__ void __launch_bounds__(256) l2_hist_kernel(Lambda2Params p, int level) {
+  __shared__ uint32_t h[kL2Digits];
+  L2Sel* st = l2sel(p);
+  if (st->done) return;
+  for (int i = threadIdx.x; i < kL2Digits; i += blockDim.x) h[i] = 0;
+  __syncthreads();
+  const uint32_t prefix = st->prefix, mask = l2_mask_above(level);
+  const int shift = l2_shift(level);
+  const int64_t R = p.bt.total_rows;
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < R; r += (int64_t)gridDim.x * blockDim.x) {
+    const uint32_t key = p.keys[r];
+    if ((key & mask) == prefix && (key >> 31)) atomicAdd(&h[(key >> shift) & (kL2Digits - 1)], 1u);
   }
-  if (tid == 0) {
-    s_prefix = 0;
-    s_k = (uint32_t)p.target;
-  }
-  uint32_t mask = 0;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = tid; i < 32 * 256; i += blockDim.x) (&hist[0][0])[i] = 0;
-    __syncthreads();
-    const uint32_t prefix = s_prefix;
-    for (int64_t r = tid; r < R; r += blockDim.x) {
-      const uint32_t key = p.keys[r];
-      if ((key & mask) == prefix) atomicAdd(&hist[warp][(key >> shift) & 255u], 1u);
-    }
-    __syncthreads();
-    if (tid < 256) {
-      uint32_t t = 0;
-      for (int w = 0; w < 32; ++w) t += hist[w][tid];
-      tot[tid] = t;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      // walk from the largest byte value down to the bucket holding the K-th key
-      uint32_t k = s_k, cum = 0;
-      int d = 255;
-      for (; d > 0; --d) {
-        if (cum + tot[d] >= k) break;
-        cum += tot[d];
+  __syncthreads();
+  for (int i = threadIdx.x; i < kL2Digits; i += blockDim.x)
+    if (h[i]) atomicAdd(&st->hist[level][i], h[i]);
+}
+
+// one CTA of 1,024 threads: the bucket of the level's histogram where the
+// count from the top reaches k (thread t holds buckets 2047 - 2t and 2046 - 2t)
+__global__ void __launch_bounds__(1024) l2_select_kernel(Lambda2Params p, int level) {
+  __shared__ int tmp[40];
+  L2Sel* st = l2sel(p);
+  const int tid = threadIdx.x;
+  if (level == 0) {
+    const int n = st->n;
+    if (tid == 0 && p.n_candidates) *p.n_candidates = n;
+    if (p.target <= 0 || p.target > n) {
+      // K <= 0: no lambda2 keeps nothing but +inf; K > n: 0 keeps every candidate
+      if (tid == 0) {
+        *p.lambda2 = p.target <= 0 ? __int_as_float(0x7f800000) : 0.f;
+        st->done = 1;
       }
-      s_k = k - cum;
-      s_prefix = prefix | ((uint32_t)d << shift);
+      return;
     }
-    mask |= 255u << shift;
-    __syncthreads();
   }
-  // from the K-th largest quotient to the largest fp32 lambda2 whose product
-  // test keeps >= K rows: down while it keeps fewer (kept(0) counts every
-  // candidate), then up while the next value still keeps K (a few steps;
-  // bounded)
-  __shared__ float s_lam;
+  if (st->done) return;
+  const int k = level == 0 ? (int)p.target : st->k;
+  const uint32_t* hist = st->hist[level];
+  const int hi = kL2Digits - 1 - 2 * tid, lo = hi - 1;
+  const int chi = (int)hist[hi], clo = (int)hist[lo];
+  int total;
+  const int above = block_exclusive_scan(chi + clo, tmp, &total);
+  if (above < k && k <= above + chi + clo) {
+    const int bucket = above + chi >= k ? hi : lo;
+    const int k_rest = bucket == hi ? k - above : k - above - chi;
+    const uint32_t prefix = (level == 0 ? 0u : st->prefix) | ((uint32_t)bucket << l2_shift(level));
+    st->prefix = prefix;
+    st->k = k_rest;
+  }
+}
+
+// kept counts of the selected ratio and its neighbours, one grid pass
+__global__ void __launch_bounds__(256) l2_window_kernel(Lambda2Params p) {
+  L2Sel* st = l2sel(p);
+  if (st->done) return;
+  constexpr int NW = 2 * kL2Window + 1;
+  const float lam0 = __uint_as_float(st->prefix & 0x7fffffffu);
+  float lam[NW];
+#pragma unroll
+  for (int j = 0; j < NW; ++j) lam[j] = l2_step(lam0, j - kL2Window);
+  int c[NW];
+#pragma unroll
+  for (int j = 0; j < NW; ++j) c[j] = 0;
+  const int64_t R = p.bt.total_rows;
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < R; r += (int64_t)gridDim.x * blockDim.x) {
+    if (p.keys[r] >> 31) {
+      const int b = upper_interval(p.bt.row_off, p.bt.B, r);
+      const float s = p.s2[r], ref = p.ref2[b];
+#pragma unroll
+      for (int j = 0; j < NW; ++j) c[j] += s >= __fmul_rn(lam[j], ref) ? 1 : 0;
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < NW; ++j) {
+    const int v = __reduce_add_sync(0xffffffffu, c[j]);
+    if ((threadIdx.x & 31) == 0 && v) atomicAdd(&st->kept[j], (unsigned long long)v);
+  }
+}
+
+// one CTA of 1,024 threads: the largest lambda2 of the window whose product
+// test keeps at least K rows; beyond the window, single fp32 steps as before
+__global__ void __launch_bounds__(1024) l2_finish_kernel(Lambda2Params p) {
   __shared__ int s_kept;
-  if (tid == 0) s_lam = __uint_as_float(s_prefix & 0x7fffffffu);
+  __shared__ float s_lam;
+  L2Sel* st = l2sel(p);
+  if (st->done) return;
+  constexpr int NW = 2 * kL2Window + 1;
+  const int64_t K = p.target;
+  const float lam0 = __uint_as_float(st->prefix & 0x7fffffffu);
+  if ((int64_t)st->kept[0] < K) {
+    // below the window: down while fewer than K are kept (kept(0) counts every candidate)
+    if (threadIdx.x == 0) s_lam = l2_step(lam0, -kL2Window);
+    __syncthreads();
+    for (int it = 0; it < 64; ++it) {
+      const float lam = nextafterf(s_lam, 0.f);
+      if (lambda2_kept(p, lam, &s_kept) >= K) {
+        if (threadIdx.x == 0) s_lam = lam;
+        break;
+      }
+      if (threadIdx.x == 0) s_lam = lam;
+      __syncthreads();
+    }
+  } else if ((int64_t)st->kept[NW - 1] >= K) {
+    // above the window: up while the next value still keeps K
+    if (threadIdx.x == 0) s_lam = l2_step(lam0, kL2Window);
+    __syncthreads();
+    for (int it = 0; it < 64; ++it) {
+      const float up = nextafterf(s_lam, __int_as_float(0x7f800000));
+      if (lambda2_kept(p, up, &s_kept) < K) break;
+      if (threadIdx.x == 0) s_lam = up;
+      __syncthreads();
+    }
+  } else {
+    if (threadIdx.x == 0) {
+      int j = NW - 1;
+      while ((int64_t)st->kept[j] < K) --j;  // kept is non-increasing in lambda2; kept[0] >= K
+      s_lam = l2_step(lam0, j - kL2Window);
+    }
+  }
   __syncthreads();
-  const int K = p.target;
-  for (int it = 0; it < 64; ++it) {
-    const float lam = s_lam;
-    if (lambda2_kept(p, lam, &s_kept) >= K) break;
-    if (tid == 0) s_lam = nextafterf(lam, 0.f);
-    __syncthreads();
-  }
-  for (int it = 0; it < 64; ++it) {
-    const float up = nextafterf(s_lam, __int_as_float(0x7f800000));
-    if (lambda2_kept(p, up, &s_kept) < K) break;
-    if (tid == 0) s_lam = up;
-    __syncthreads();
-  }
-  if (tid == 0) *p.lambda2 = s_lam;
+  if (threadIdx.x == 0) *p.lambda2 = s_lam;
 }
 
 }  // namespace occam

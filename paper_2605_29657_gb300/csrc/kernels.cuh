@@ -235,9 +235,13 @@ struct Lambda2Params {
   const uint8_t* role;
   int64_t target;       // K
   uint32_t* keys;       // [total_rows] scratch
+  void* sel;            // kL2SelBytes of zeroed scratch: selection state, histograms, window counts
   float* lambda2;       // out
   int32_t* n_candidates;  // out, nullable
 };
+constexpr int kL2Digits = 2048;         // lambda2 selection: 11-bit digits
+constexpr int kL2Window = 4;            // fp32 steps either way whose kept counts are taken in one pass
+constexpr int kL2SelBytes = 32 * 1024;  // workspace scratch of the selection
 
 // mean-threshold reference (component ablation): ref[u] = mean of s over the
 // unit's candidate rows (role 0, and prev_keep where given)
@@ -318,7 +322,11 @@ int s2_fused_threads();
 // compact.cu
 __global__ void scan_kernel(ScanParams p);
 __global__ void stage_rows_kernel(StageRowsParams p);
-__global__ void lambda2_select_kernel(Lambda2Params p);
+__global__ void l2_keys_kernel(Lambda2Params p);
+__global__ void l2_hist_kernel(Lambda2Params p, int level);
+__global__ void l2_select_kernel(Lambda2Params p, int level);
+__global__ void l2_window_kernel(Lambda2Params p);
+__global__ void l2_finish_kernel(Lambda2Params p);
 __global__ void registers_kernel(RegistersParams p);
 
 // rules.cu
