@@ -438,6 +438,19 @@ def run_ours(args, rank, world, local):
     kept_total = int(out["out_off"][-1].item())
     bytes_ = algorithmic_bytes(meta, n1_total, kept_total)
     want = {k: v.clone() for k, v in call.out.items()}
+    # near-threshold rows of the two tests (band 1e-5), from one more eager
+    # call with the flags requested (outside the timed region, no gather)
+    ncall = occ.PruneCall(layout, stage1_of(batch),
+                          dict(Q_text=batch["Q_text"], K_text=batch["K_text"], K2=batch["K2"]),
+                          w.lambda1, w.lambda2, keep_registers=True,
+                          want=occ.PruneCall.OPTIONAL + occ.PruneCall.NEAR, ws=call.ws)
+    ncall()
+    torch.cuda.synchronize()
+    if ncall.status() != 0:
+        raise RuntimeError("device status after the near-threshold call")
+    near_rows = {"stage1": int(ncall.out["near1"].sum().item()), "stage2": int(ncall.out["near2"].sum().item()),
+                 "band": "|s - tau| <= 1e-5 |tau| (visual rows; S1 rows for Stage II)"}
+    del ncall
 
     def same_as_first(c, what):
         for k, v in want.items():
@@ -744,6 +757,7 @@ def run_ours(args, rank, world, local):
             "mean_n1_vis": float(out["n1_vis"].float().mean().item()),
             "mean_count_vis": float(out["count_vis"].float().mean().item()),
             "kept_rows_per_step": kept_total,
+            "near_threshold_rows": near_rows,
             "algorithmic_bytes_per_step": bytes_["step"],
             "step_algorithmic_GBps": step_gbs,
             "step_frac_of_measured_hbm": step_gbs / peak,

@@ -277,6 +277,11 @@ typedef struct occam_prune_args {
    * is unused and ref2 keeps the register reference). */
   int32_t rule;
   const int32_t* budget; /* [B] int32 device, OCCAM_RULE_BUDGET only (else unused) */
+  /* relative width of the near-threshold band of the optional outputs near1
+   * and near2: |s - tau| <= near_rel * |tau|; 0 (or negative, or NaN) means
+   * 1e-5, the band inside which a mask may legitimately differ between two
+   * correct fp32 evaluations of the scores */
+  float near_rel;
 } occam_prune_args;
 
 /* Outputs of occam_prune. Required: keep2 [total_rows] u8 (S2, registers =
@@ -288,7 +293,14 @@ typedef struct occam_prune_args {
  * ([CLS] mode only, else OCCAM_ERR_UNSUPPORTED): per segment and head the
  * effective number of attended keys of the Stage-I [CLS] attention,
  * exp(H(a)) with H(a) = -sum_i a_i log a_i over the keys {[CLS]} u rows
- * (Sec. 3.2, Observation 1). */
+ * (Sec. 3.2, Observation 1). near1, near2 [total_rows] u8 (optional):
+ * near-threshold flags of the two tests (Eq. 5 and Eq. 8), the rows whose
+ * keep decision turns on the last digits of their score. near1[v] = 1 for a
+ * visual row with |s1(v) - tau1| <= near_rel * |tau1| (tau1 = lambda1 * ref1
+ * of its segment, the same fp32 product the test uses); near2[v] = 1 for a
+ * visual S1 row with |s2(v) - tau2| <= near_rel * |tau2| (tau2 = lambda2 *
+ * ref2 of its sample); every other row 0. Under OCCAM_RULE_BUDGET there is
+ * no Stage-II threshold and near2 is all 0. */
 typedef struct occam_prune_out {
   uint8_t* keep2;
   int32_t* out_index;
@@ -302,6 +314,8 @@ typedef struct occam_prune_out {
   float* ref2;
   int32_t* n1_vis;
   float* n_eff;
+  uint8_t* near1;
+  uint8_t* near2;
 } occam_prune_out;
 
 /* The whole path in one call (Algorithm 1's pruning steps): Stage-I scores,

@@ -73,7 +73,7 @@ class CPruneArgs(ctypes.Structure):
         ("lambda1", ctypes.c_float), ("lambda2", ctypes.c_float),
         ("keep_registers", _i32), ("n_tensors", _i32),
         ("src", _p * OCCAM_MAX_GATHER), ("row_bytes", _i64 * OCCAM_MAX_GATHER), ("dst", _p * OCCAM_MAX_GATHER),
-        ("capacity_rows", _i64), ("rule", _i32), ("budget", _p),
+        ("capacity_rows", _i64), ("rule", _i32), ("budget", _p), ("near_rel", ctypes.c_float),
     ]
 
 
@@ -81,6 +81,7 @@ class CPruneOut(ctypes.Structure):
     _fields_ = [
         ("keep2", _p), ("out_index", _p), ("count_vis", _p), ("count_out", _p), ("out_off", _p),
         ("keep1", _p), ("s1", _p), ("ref1", _p), ("s2", _p), ("ref2", _p), ("n1_vis", _p), ("n_eff", _p),
+        ("near1", _p), ("near2", _p),
     ]
 
 
@@ -477,15 +478,19 @@ class PruneCall:
     built once and reused, so repeated calls marshal nothing."""
 
     OPTIONAL = ("keep1", "s1", "ref1", "s2", "ref2", "n1_vis", "n_eff")  # n_eff: [CLS] mode only
+    NEAR = ("near1", "near2")  # near-threshold flags of the two tests (opt-in through `want`)
 
     def __init__(self, layout: BatchLayout, stage1: dict, stage2: dict, lambda1: float, lambda2: float,
                  keep_registers: bool = True, gather=(), capacity_rows: int | None = None,
-                 want=OPTIONAL, ws=None, host_inputs: bool = False, rule: str = "register", budget=None):
+                 want=OPTIONAL, ws=None, host_inputs: bool = False, rule: str = "register", budget=None,
+                 near_rel: float = 0.0):
         """host_inputs: K2 and the gather tensors may be pinned host tensors,
         read in place through occam_prune_staged (S1 rows of K2 and kept rows
         only); a device staging tensor for K2 is allocated here.
         rule: "register" (the method), "mean" or "budget" (the component
-        ablation's variants); budget: [B] int32 CUDA tensor for "budget"."""
+        ablation's variants); budget: [B] int32 CUDA tensor for "budget".
+        want may name "near1" / "near2" (PruneCall.NEAR): the near-threshold
+        flags of the two tests, with relative band near_rel (0: 1e-5)."""
         bf = torch.bfloat16
         mode = OCCAM_STAGE1_CLS if stage1.get("mode", "cls") == "cls" else OCCAM_STAGE1_MUTUAL
         q = _dev_tensor(stage1["q"], bf, "q")
@@ -520,7 +525,7 @@ class PruneCall:
         )
         shapes = dict(keep1=(R, torch.uint8), s1=(R, torch.float32), ref1=(layout.S_tot, torch.float32),
                       s2=(R, torch.float32), ref2=(B, torch.float32), n1_vis=(B, torch.int32),
-                      n_eff=((layout.S_tot, H1), torch.float32))
+                      n_eff=((layout.S_tot, H1), torch.float32), near1=(R, torch.uint8), near2=(R, torch.uint8))
         if mode != OCCAM_STAGE1_CLS:
             want = tuple(k for k in want if k != "n_eff")
         for k in want:
@@ -542,6 +547,7 @@ class PruneCall:
             a.dst[i] = dst_a[i]
             a.row_bytes[i] = rb_a[i]
         a.capacity_rows = cap
+        a.near_rel = float(near_rel)
         if rule not in RULES:
             raise OccamError(OCCAM_ERR_INVALID_ARG, f"rule must be one of {sorted(RULES)}")
         a.rule = RULES[rule]
@@ -556,7 +562,7 @@ class PruneCall:
         self.args = a
         self.cout = CPruneOut(*[_ptr(o.get(k)) for k in
                                 ("keep2", "out_index", "count_vis", "count_out", "out_off", "keep1", "s1", "ref1",
-                                 "s2", "ref2", "n1_vis", "n_eff")])
+                                 "s2", "ref2", "n1_vis", "n_eff", "near1", "near2")])
         self.capacity = cap
 
     def __call__(self, stream=None) -> dict:
@@ -590,12 +596,13 @@ class PruneCall:
 def occam_prune(layout: BatchLayout, stage1: dict, stage2: dict, lambda1: float, lambda2: float,
                 keep_registers: bool = True, gather=(), capacity_rows: int | None = None,
                 want=PruneCall.OPTIONAL, ws=None, stream=None, host_inputs: bool = False,
-                rule: str = "register", budget=None) -> dict:
+                rule: str = "register", budget=None, near_rel: float = 0.0) -> dict:
     """One fused prune call; returns the output tensors and the gathered rows.
     With host_inputs, K2 and the gather tensors may be pinned host tensors
-    (occam_prune_staged). rule / budget select the rule variant (PruneCall)."""
+    (occam_prune_staged). rule / budget select the rule variant (PruneCall);
+    want may add "near1" / "near2" (PruneCall.NEAR), with band near_rel."""
     call = PruneCall(layout, stage1, stage2, lambda1, lambda2, keep_registers, gather, capacity_rows, want, ws,
-                     host_inputs, rule, budget)
+                     host_inputs, rule, budget, near_rel)
     out = dict(call(stream))
     out["gathered"] = call.gathered
     out["ws"] = call.ws

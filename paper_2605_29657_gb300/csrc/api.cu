@@ -388,7 +388,7 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
                      float lambda1, int do_threshold, float* ref1, uint8_t* keep1, int32_t* n1_vis,
                      const occam_stage1_args* a1, float* s2_zero, const Stage2Params* plan, int32_t* count_out,
                      int32_t* count_vis, cudaStream_t st, Trace trace = Trace(), float* n_eff = nullptr,
-                     int ref_mean = 0) {
+                     int ref_mean = 0, uint8_t* near1 = nullptr, float near_rel = 1e-5f) {
   const NvtxRange nvtx("stage1_finalize");
   Stage1FinalizeParams p;
   p.bt = dev_batch(b);
@@ -421,6 +421,8 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   if (plan) p.plan = *plan;
   p.zero_count_out = count_out;
   p.zero_count_vis = count_vis;
+  p.near1 = near1;
+  p.near_rel = near_rel;
   stage1_finalize_kernel<<<b->S_tot, 256, finalize_smem_bytes(p.smem_rows), st>>>(p);
   count_launch();
   trace.mark(st);
@@ -579,7 +581,8 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
                    const uint8_t* keep1, const float* s2, int keep_registers, uint8_t* keep_out, int n_tensors,
                    const void* const* src, const int64_t* row_bytes, void* const* dst, int64_t capacity,
                    int32_t* out_index, int32_t* count_out, int32_t* count_vis, int64_t* out_off,
-                   cudaStream_t st, bool do_memsets = true, Trace trace = Trace(), bool use_role = false) {
+                   cudaStream_t st, bool do_memsets = true, Trace trace = Trace(), bool use_role = false,
+                   uint8_t* near_out = nullptr, float near_rel = 1e-5f) {
   const NvtxRange nvtx(mode == 1 ? "stage2_threshold_compact" : "compact");
   ScanParams p;
   p.bt = dev_batch(b);
@@ -600,6 +603,8 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
   p.ticket = at<int32_t>(ws, L.counters) + CNT_SCAN_TICKET;
   p.ntiles = L.scan_tiles;
   p.status = at<int>(ws, L.status);
+  p.near_out = mode == 1 ? near_out : nullptr;
+  p.near_rel = near_rel;
   if (do_memsets) {
     OCCAM_CUDA(cudaMemsetAsync(p.tile_state, 0, L.scan_tiles * 8, st));
     OCCAM_CUDA(cudaMemsetAsync(p.ticket, 0, 4, st));
@@ -846,6 +851,8 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
     OCCAM_TRY(require_device(args->budget));
   }
   if (out->n_eff && args->stage1.mode != OCCAM_STAGE1_CLS) return OCCAM_ERR_UNSUPPORTED;
+  // the near-threshold band of the optional flags (0, negative or NaN: 1e-5)
+  const float near_rel = args->near_rel > 0.f ? args->near_rel : 1e-5f;
   WsLayout L;
   OCCAM_TRY(check_ws(b, args->stage1.H1, args->stage2.H2, workspace, workspace_bytes, &L));
   // memory kinds (see device_view)
@@ -893,7 +900,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   const Stage2Params plan = stage2_params(b, &a2, L, ws, s2, ref2, args->lambda2);
   OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, &args->stage1, s2,
                              &plan, out->count_out, out->count_vis, st, trace, out->n_eff,
-                             args->rule == OCCAM_RULE_MEAN ? 1 : 0));
+                             args->rule == OCCAM_RULE_MEAN ? 1 : 0, out->near1, near_rel));
   if (k2_stage) {
     // the S1 rows of K2 (only those) into the device staging tensor
     const NvtxRange nvtx("stage_k2_rows");
@@ -926,6 +933,8 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
     budget_keep_kernel<<<b->B, 1024, 0, st>>>(bp);
     count_launch();
     OCCAM_CUDA(cudaGetLastError());
+    // no Stage-II threshold under the budget rule: no near-threshold rows
+    if (out->near2) OCCAM_CUDA(cudaMemsetAsync(out->near2, 0, b->total_rows, st));
     return launch_compact(b, L, ws, 0, out->keep2, nullptr, nullptr, args->keep_registers, nullptr, args->n_tensors,
                           src, args->row_bytes, dst, args->capacity_rows, out->out_index, out->count_out,
                           out->count_vis, out->out_off, st, false, trace, true);
@@ -948,7 +957,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   }
   return launch_compact(b, L, ws, 1, nullptr, keep1, s2, args->keep_registers, out->keep2, args->n_tensors,
                         src, args->row_bytes, dst, args->capacity_rows, out->out_index,
-                        out->count_out, out->count_vis, out->out_off, st, false, trace);
+                        out->count_out, out->count_vis, out->out_off, st, false, trace, false, out->near2, near_rel);
 }
 
 int occam_prune(const occam_prune_args* args, const occam_prune_out* out, void* workspace,

@@ -80,9 +80,13 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
         k = p.keep_registers != 0;
         vis = false;
       } else {
-        k = (p.keep1[r] != 0) && (p.s2[r] >= tau2[samp]);
+        const float sv = p.s2[r], t = tau2[samp];
+        k = (p.keep1[r] != 0) && (sv >= t);
         vis = k;
+        // near-threshold flag of a visual S1 row: the same fp32 tau as the test
+        if (p.near_out) p.near_out[r] = p.keep1[r] != 0 && fabsf(sv - t) <= p.near_rel * fabsf(t) ? 1 : 0;
       }
+      if (p.near_out && reg) p.near_out[r] = 0;
       if (p.keep_out) p.keep_out[r] = k ? 1 : 0;
     }
     kmask |= (unsigned)k << i;

@@ -142,6 +142,8 @@ struct Stage1FinalizeParams {
   float* n_eff;                   // nullable, [CLS] mode: [S_tot, 16] effective number of attended keys per head
   float* s2_zero;                 // nullable: zeroed per row (Stage-II max accumulator)
   int smem_rows;                  // segments up to this many rows stage their s1 and roles in shared memory
+  uint8_t* near1 = nullptr;       // nullable: near-threshold flags of the Stage-I test
+  float near_rel = 1e-5f;         // their relative band
   const float* s1;          // nullable when keep_in is given
   const uint8_t* keep_in;   // nullable: S1 membership of visual rows given instead of tested
   float lambda1;
@@ -185,6 +187,8 @@ struct ScanParams {
   int32_t* ticket;
   int64_t ntiles;
   int* status;
+  uint8_t* near_out = nullptr;  // nullable, mode 1: near-threshold flags of the Stage-II test
+  float near_rel = 1e-5f;       // their relative band
 };
 
 struct GatherParams {

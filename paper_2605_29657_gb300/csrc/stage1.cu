@@ -414,8 +414,11 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   const int64_t list_len = p.bt.row_off[b + 1] - p.bt.row_off[b] - s_base;  // room left in the sample's list
   for (int r = a; r < z; ++r) {
     const bool reg = role[r] != 0;
-    const bool k = reg || (p.keep_in ? p.keep_in[sb + r] != 0 : (staged ? s1_loc[r] : s1g[sb + r]) >= tau);
+    const float sv = p.keep_in ? 0.f : (staged ? s1_loc[r] : s1g[sb + r]);
+    const bool k = reg || (p.keep_in ? p.keep_in[sb + r] != 0 : sv >= tau);
     if (p.keep1) p.keep1[sb + r] = k ? 1 : 0;
+    // near-threshold flag: the same fp32 tau as the test
+    if (p.near1) p.near1[sb + r] = !reg && !p.keep_in && fabsf(sv - tau) <= p.near_rel * fabsf(tau) ? 1 : 0;
     if (k) {
       if (in_bounds(pos >= 0 && pos < list_len, p.status, kSiteListPos)) list[pos] = (int32_t)(sb + r);
       ++pos;

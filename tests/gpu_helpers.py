@@ -30,24 +30,26 @@ def to_device(batch: dict, dev) -> dict:
 
 def run_prune(batch: dict, lam1: float, lam2: float, keep_registers: bool = True, dev="cuda",
               capacity_rows=None, gather=True, text_keys: bool = True, g=None, path: str = "auto",
-              host_inputs: bool = False, rule: str = "register", budget=None):
+              host_inputs: bool = False, rule: str = "register", budget=None, near: bool = False,
+              near_rel: float = 0.0):
     """path: "auto" (fused tensor-core Stage II where it fits, wider clusters
     for small batches), "narrow" (the same without the widening) or "twopass".
     host_inputs: K2, hidden and V stay in pinned host memory (occam_prune_staged).
     rule / budget: the selection rule ("register", "mean", "budget") and the
-    per-sample budget array (host ints) of the "budget" rule."""
+    per-sample budget array (host ints) of the "budget" rule. near: also
+    return the near-threshold flags near1 / near2 (band near_rel, 0: 1e-5)."""
     import paper_2605_29657_gb300 as occ
     route = {"auto": occ.OCCAM_ROUTE_AUTO, "twopass": occ.OCCAM_ROUTE_TWOPASS, "narrow": occ.OCCAM_ROUTE_NARROW}[path]
     old = occ.occam_set_stage2_route(route)
     try:
         return _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs,
-                          rule, budget)
+                          rule, budget, near, near_rel)
     finally:
         occ.occam_set_stage2_route(old)
 
 
 def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, text_keys, g, host_inputs=False,
-               rule="register", budget=None):
+               rule="register", budget=None, near=False, near_rel=0.0):
     import paper_2605_29657_gb300 as occ
 
     m = batch["meta"]
@@ -66,8 +68,10 @@ def _run_prune(batch, lam1, lam2, keep_registers, dev, capacity_rows, gather, te
     if gather:
         tensors = (g["hidden"], g["K2"].view(g["K2"].shape[0], -1), g["V"])
     bud = None if budget is None else torch.as_tensor(np.asarray(budget, np.int32)).to(dev)
+    want = occ.PruneCall.OPTIONAL + (occ.PruneCall.NEAR if near else ())
     out = occ.occam_prune(layout, st1, st2, lam1, lam2, keep_registers=keep_registers, gather=tensors,
-                          capacity_rows=capacity_rows, host_inputs=host_inputs, rule=rule, budget=bud)
+                          capacity_rows=capacity_rows, host_inputs=host_inputs, rule=rule, budget=bud, want=want,
+                          near_rel=near_rel)
     torch.cuda.synchronize()
     status = occ.occam_get_status(out["ws"])
     res = {k: v.cpu().numpy() for k, v in out.items() if isinstance(v, torch.Tensor) and k != "ws"}

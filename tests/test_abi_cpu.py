@@ -122,3 +122,37 @@ def test_selftest_arguments_checked_on_host(lib):
     assert lib.occam_selftest_wait(0, None, None) == occ._lib.OCCAM_ERR_INVALID_ARG
     assert lib.occam_selftest_wait(10 ** 6, None, None) == occ._lib.OCCAM_ERR_INVALID_ARG
     assert lib.occam_selftest_wait(2 * 10 ** 9, 0x1000, None) == occ._lib.OCCAM_ERR_INVALID_ARG
+
+
+def test_ctypes_structs_match_the_header(tmp_path):
+    """The binding's ctypes structs have the header's layout: a C program
+    compiled against include/occam.h prints every field's offset and each
+    struct's size, and ctypes must agree (an ABI drift between the two would
+    pass wrong pointers silently)."""
+    import shutil
+    import subprocess
+
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    occ = pytest.importorskip("paper_2605_29657_gb300")
+    L = occ._lib
+    structs = {"occam_batch": L.CBatch, "occam_stage1_args": L.CStage1, "occam_stage2_args": L.CStage2,
+               "occam_prune_args": L.CPruneArgs, "occam_prune_out": L.CPruneOut}
+    lines = ["#include <stdio.h>", "#include <stddef.h>", '#include "occam.h"', "int main(void) {"]
+    for cname, py in structs.items():
+        lines.append(f'  printf("{cname} size %zu\\n", sizeof({cname}));')
+        for fname, _ in py._fields_:
+            lines.append(f'  printf("{cname}.{fname} %zu\\n", offsetof({cname}, {fname}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    subprocess.run([cc, "-std=c11", "-I", os.path.join(root, "include"), str(src), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split("\n")
+    got = dict(line.rsplit(" ", 1) for line in out if line)
+    for cname, py in structs.items():
+        assert int(got[f"{cname} size"]) == ctypes.sizeof(py), cname
+        for fname, _ in py._fields_:
+            assert int(got[f"{cname}.{fname}"]) == getattr(py, fname).offset, f"{cname}.{fname}"
