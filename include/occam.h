@@ -103,7 +103,8 @@ typedef struct occam_batch {
 /* Stage-I inputs (Sec. 3.4). CLS: q = q_cls [S_tot,H1,d1]; k_cls [S_tot,H1,d1]
  * or NULL (the [CLS] key is then left out of the softmax). MUTUAL: q = Q1
  * [rows,H1,d1], k_cls ignored. K1 [rows,H1,d1]. Built for H1 = 16 with
- * d1 = 64 (CLS) and d1 in {64, 72, 80} (MUTUAL). */
+ * d1 in {64, 72, 128} (CLS) and for 1 <= H1 <= 64 with d1 in {64, 72, 80}
+ * (MUTUAL); other shapes return OCCAM_ERR_UNSUPPORTED. */
 typedef struct occam_stage1_args {
   int32_t mode; /* OCCAM_STAGE1_CLS or OCCAM_STAGE1_MUTUAL */
   int32_t H1;

@@ -133,8 +133,6 @@ size_t finalize_smem_bytes(int rows) { return ((size_t)rows * (4 + 1) + 15) & ~(
 void set_smem_attrs() {
   static std::once_flag once;
   std::call_once(once, [] {
-    cudaFuncSetAttribute(stage1_logits_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         stage1_logits_smem_bytes());
     cudaFuncSetAttribute(stage1_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)finalize_smem_bytes(kFinalizeSmemRows));
   });
@@ -263,7 +261,7 @@ int check_stage1(const occam_batch* b, const occam_stage1_args* a) {
   if (!a || !a->q || !a->K1) return OCCAM_ERR_INVALID_ARG;
   if (!aligned16(a->q) || !aligned16(a->K1) || (a->k_cls && !aligned16(a->k_cls))) return OCCAM_ERR_INVALID_ARG;
   if (a->mode == OCCAM_STAGE1_CLS) {
-    if (a->H1 != 16 || a->d1 != 64) return OCCAM_ERR_UNSUPPORTED;
+    if (a->H1 != 16 || (a->d1 != 64 && a->d1 != 72 && a->d1 != 128)) return OCCAM_ERR_UNSUPPORTED;
   } else if (a->mode == OCCAM_STAGE1_MUTUAL) {
     if (a->H1 < 1 || a->H1 > 64) return OCCAM_ERR_UNSUPPORTED;
     if (a->d1 != 64 && a->d1 != 72 && a->d1 != 80) return OCCAM_ERR_UNSUPPORTED;
@@ -349,7 +347,7 @@ int launch_stage1_scores(const occam_batch* b, const occam_stage1_args* a, const
     p.status = status;
     const int64_t tiles = cdiv(b->total_rows, 16);
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(tiles, 2 * num_sms()));
-    stage1_logits_kernel<<<grid, 256, stage1_logits_smem_bytes(), st>>>(p);
+    launch_stage1_logits(p, a->d1, grid, st);
     count_launch();
     trace.mark(st);
   } else {
@@ -397,6 +395,7 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   p.q_cls = cls ? static_cast<const __nv_bfloat16*>(a1->q) : nullptr;
   p.k_cls = cls ? static_cast<const __nv_bfloat16*>(a1->k_cls) : nullptr;
   p.scale = cls ? (float)(1.4426950408889634 / std::sqrt((double)a1->d1)) : 1.f;  // log2 units, as the logits
+  p.d1 = cls ? a1->d1 : 64;
   p.s1_out = s1;
   p.n_eff = cls ? n_eff : nullptr;
   p.s2_zero = cls ? s2_zero : nullptr;

@@ -138,6 +138,7 @@ struct Stage1FinalizeParams {
   const __nv_bfloat16* q_cls;     // [CLS] mode
   const __nv_bfloat16* k_cls;     // nullable
   float scale;  // log2(e) / sqrt(d1): [CLS] logits in log2 units
+  int d1 = 64;  // [CLS] mode: head dim of q_cls / k_cls
   float* s1_out;                  // [CLS] mode: where s1 is written
   float* n_eff;                   // nullable, [CLS] mode: [S_tot, 16] effective number of attended keys per head
   float* s2_zero;                 // nullable: zeroed per row (Stage-II max accumulator)
@@ -300,8 +301,9 @@ struct Stage2TcParams {
 };
 
 // stage1.cu
-__global__ void stage1_logits_kernel(Stage1ClsParams p);
-int stage1_logits_smem_bytes();
+// the [CLS] logits kernel for d1 = 64, 72 or 128 (stage1.cu)
+int stage1_logits_smem_bytes(int d1);
+void launch_stage1_logits(const Stage1ClsParams& p, int d1, int grid, cudaStream_t st);
 __global__ void stage1_finalize_kernel(Stage1FinalizeParams p);
 void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mq1,
                       const CUtensorMap& mk1, int sms, cudaStream_t st);

@@ -2,6 +2,8 @@
 // scores of every visual and register row, the register reference of each
 // segment, and the image-adaptive threshold S1 = {v : s1(v) >= lambda1 s1(r)} u {r}
 // (Eqs. 4-6; App. A, Eqs. 10-13).
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.cuh"
 #include "plan.cuh"
@@ -19,17 +21,46 @@ namespace occam {
 // HBM is read exactly once.
 // ============================================================================
 namespace cls {
-constexpr int H = 16, D = 64;
+constexpr int H = 16;
 constexpr int kThreads = 256;
-constexpr int kRowBytes = H * D * 2;            // 2048
 constexpr int kTileRows = 16;                   // rows per stage
-constexpr int kStageBytes = kTileRows * kRowBytes;
 constexpr int kStages = 3;
-constexpr int kSmem = kStages * kStageBytes + 64;
+template <int D>
+struct Geo {
+  static constexpr int kRowBytes = H * D * 2;   // 2048 / 2304 / 4096 for d1 = 64 / 72 / 128
+  static constexpr int kStageBytes = kTileRows * kRowBytes;
+  static constexpr int kSmem = kStages * kStageBytes + 64;
+  static constexpr int kLaneDims = D / 8;       // dims of one (row, head) per lane (8 lanes share it)
+  static_assert(D % 8 == 0 && kRowBytes % 16 == 0, "rows in whole 16-byte units");
+};
+static_assert(Geo<128>::kSmem <= 227 * 1024, "shared memory per CTA");
+
+// n consecutive bf16 values as floats: 16-byte loads when the lane's slice is
+// a whole number of them, else 2-byte loads (d1 = 72: 9 dims = 18 bytes)
+template <int N>
+__device__ __forceinline__ void load_bf16(const unsigned char* src, float (&out)[N]) {
+  if constexpr (N % 8 == 0) {
+#pragma unroll
+    for (int c = 0; c < N / 8; ++c) {
+      const uint4 raw = *reinterpret_cast<const uint4*>(src + 16 * c);
+      const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        out[8 * c + 2 * i] = bf16_lo(w[i]);
+        out[8 * c + 2 * i + 1] = bf16_hi(w[i]);
+      }
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < N; ++i) out[i] = __uint_as_float((uint32_t)reinterpret_cast<const uint16_t*>(src)[i] << 16);
+  }
+}
 }  // namespace cls
 
+template <int D>
 __global__ void __launch_bounds__(cls::kThreads) stage1_logits_kernel(Stage1ClsParams p) {
   using namespace cls;
+  constexpr int kRowBytes = Geo<D>::kRowBytes, kStageBytes = Geo<D>::kStageBytes, NL = Geo<D>::kLaneDims;
   extern __shared__ __align__(128) unsigned char smem[];
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -52,14 +83,14 @@ __global__ void __launch_bounds__(cls::kThreads) stage1_logits_kernel(Stage1ClsP
   __syncthreads();
 
   // lane layout for the dot products: 8 lanes share one (row, head); lane
-  // k = lane & 7 owns dims [8k, 8k+8) of that head. The four (row, head)
-  // slots of a warp share one row, so segment changes are warp-uniform.
+  // k = lane & 7 owns dims [k D/8, (k+1) D/8) of that head. The four (row,
+  // head) slots of a warp share one row, so segment changes are warp-uniform.
   const int slot = warp * 4 + (lane >> 3);   // 0..31
   const int my_h = slot & (H - 1);
   const int my_rr = slot >> 4;               // 0..1: row parity inside a step
   const int kv = lane & 7;
   int64_t seg_lo = 0, seg_hi = 0;            // rows of the segment q belongs to
-  float q[8];
+  float q[NL];
 
   bool timed_out = false;
   int it = 0;
@@ -84,21 +115,12 @@ __global__ void __launch_bounds__(cls::kThreads) stage1_logits_kernel(Stage1ClsP
           if (!in_bounds(sg >= 0 && sg < p.bt.S_tot, p.status, kSiteLogitsSegment)) sg = 0;
           seg_lo = p.bt.seg_off[sg];
           seg_hi = p.bt.seg_off[sg + 1];
-          const uint4 raw = *reinterpret_cast<const uint4*>(p.q_cls + ((int64_t)sg * H + my_h) * D + kv * 8);
-          const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            q[2 * i] = bf16_lo(w[i]);
-            q[2 * i + 1] = bf16_hi(w[i]);
-          }
+          load_bf16<NL>(reinterpret_cast<const unsigned char*>(p.q_cls + ((int64_t)sg * H + my_h) * D + kv * NL), q);
         }
-        const uint4 raw = *reinterpret_cast<const uint4*>(buf + rr * kRowBytes + my_h * D * 2 + kv * 16);
-        const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+        float kx[NL];
+        load_bf16<NL>(buf + rr * kRowBytes + my_h * D * 2 + kv * NL * 2, kx);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          acc = fmaf(q[2 * i], bf16_lo(w[i]), acc);
-          acc = fmaf(q[2 * i + 1], bf16_hi(w[i]), acc);
-        }
+        for (int i = 0; i < NL; ++i) acc = fmaf(q[i], kx[i], acc);
       }
       acc += __shfl_xor_sync(0xffffffffu, acc, 1);
       acc += __shfl_xor_sync(0xffffffffu, acc, 2);
@@ -121,7 +143,26 @@ __global__ void __launch_bounds__(cls::kThreads) stage1_logits_kernel(Stage1ClsP
   }
 }
 
-int stage1_logits_smem_bytes() { return cls::kSmem; }
+int stage1_logits_smem_bytes(int d1) {
+  return d1 == 128 ? cls::Geo<128>::kSmem : d1 == 72 ? cls::Geo<72>::kSmem : cls::Geo<64>::kSmem;
+}
+
+void launch_stage1_logits(const Stage1ClsParams& p, int d1, int grid, cudaStream_t st) {
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaFuncSetAttribute(stage1_logits_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, cls::Geo<64>::kSmem);
+    cudaFuncSetAttribute(stage1_logits_kernel<72>, cudaFuncAttributeMaxDynamicSharedMemorySize, cls::Geo<72>::kSmem);
+    cudaFuncSetAttribute(stage1_logits_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         cls::Geo<128>::kSmem);
+  });
+  const int smem = stage1_logits_smem_bytes(d1);
+  if (d1 == 128)
+    stage1_logits_kernel<128><<<grid, cls::kThreads, smem, st>>>(p);
+  else if (d1 == 72)
+    stage1_logits_kernel<72><<<grid, cls::kThreads, smem, st>>>(p);
+  else
+    stage1_logits_kernel<64><<<grid, cls::kThreads, smem, st>>>(p);
+}
 
 // ============================================================================
 // Stage-I finalize: per segment, the register reference ref1 = mean of s1
@@ -161,7 +202,8 @@ __device__ __forceinline__ void merge_softmax_stats(float& M, float& Z, float& T
 // (global) and, when given, to s1_loc (shared).
 __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, int seg, int64_t sb, int n,
                                                float* s1_loc) {
-  constexpr int H = 16, D = 64;
+  constexpr int H = 16;
+  const int D = p.d1;
   __shared__ float rm[16][17], rz[16][17], rt[16][17];
   __shared__ float gmax[16], ginv[16], lcls_s[16];
   const int tid = threadIdx.x;
@@ -182,14 +224,13 @@ __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, in
   };
   load_chunk(j);
   {
-    // l_cls,h: 16 threads per head, 4 dims each
+    // l_cls,h: 16 threads per head, dims sub, sub + 16, ...
     const int hh = tid >> 4, sub = tid & 15;
     float acc = 0.f;
     if (p.k_cls) {
-      const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + hh) * D + sub * 4;
-      const __nv_bfloat16* kp = p.k_cls + ((int64_t)seg * H + hh) * D + sub * 4;
-#pragma unroll
-      for (int d = 0; d < 4; ++d) acc = fmaf(__bfloat162float(qp[d]), __bfloat162float(kp[d]), acc);
+      const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + hh) * D;
+      const __nv_bfloat16* kp = p.k_cls + ((int64_t)seg * H + hh) * D;
+      for (int d = sub; d < D; d += 16) acc = fmaf(__bfloat162float(qp[d]), __bfloat162float(kp[d]), acc);
     }
 #pragma unroll
     for (int o = 8; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);

@@ -77,6 +77,18 @@ def test_prune_mutual_matches_oracle(d1):
     check_prune(b, gpu, 0.5, 1.1)
 
 
+@pytest.mark.parametrize("d1", [72, 128])
+def test_prune_cls_head_dims(d1):
+    """[CLS] mode with vision heads of 72 and 128 dims (2,304- and 4,096-byte
+    K1 rows; 72 takes 18-byte lane slices), ragged segments and tiles."""
+    b = _tiny(B=3, segs=2, P=(200, 37, 130), R=3, M=(9, 70, 129), d1=d1, seed=35)
+    for path in ("auto", "twopass"):
+        gpu = run_prune(b, 0.3, 1.2, path=path)
+        assert gpu["status"] == 0
+        rep = check_prune(b, gpu, 0.3, 1.2)
+        assert rep["kept"] > 0
+
+
 @pytest.mark.parametrize("d1", [72, 64, 80])
 def test_prune_mutual_segment_edges(d1):
     """Mutual Stage I on segments of 5 rows (one partial key block), 133 (a
