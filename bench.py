@@ -596,39 +596,54 @@ def run_ours(args, rank, world, local):
             if not torch.equal(rh["out_index"][:kept_total], call.out["out_index"][:kept_total].cpu()):
                 raise RuntimeError("host-input call differs from the device-input call in out_index")
         e_steps = max(20, min(50, args.steps // 20))
-        if world > 1:
-            dist.barrier()
-        a = torch.cuda.Event(enable_timing=True)
-        z = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        copy_stream.wait_event(a)
-        for i in range(e_steps):
-            e2e_step(i)
-        z.record(stream)
-        torch.cuda.synchronize()
-        ems, e_images = aggregate(a.elapsed_time(z), meta["B"] * e_steps, dev)
-        # the host link's own rate, measured here after the timed region: the
-        # largest scoring input copied host -> device by the copy engine
+        # the host link's own rate: the largest scoring input copied host ->
+        # device by the copy engine (best of 3), before and after the timed blocks
         big = max(copy_names, key=lambda k: host[k].numel() * host[k].element_size())
         big_bytes = host[big].numel() * host[big].element_size()
-        l0 = torch.cuda.Event(enable_timing=True)
-        l1 = torch.cuda.Event(enable_timing=True)
-        link_ms = []
+
+        def link_rate():
+            l0 = torch.cuda.Event(enable_timing=True)
+            l1 = torch.cuda.Event(enable_timing=True)
+            best = None
+            for _ in range(3):
+                l0.record(copy_stream)
+                with torch.cuda.stream(copy_stream):
+                    dins[0][big].copy_(host[big], non_blocking=True)
+                l1.record(copy_stream)
+                torch.cuda.synchronize()
+                t = l0.elapsed_time(l1)
+                best = t if best is None else min(best, t)
+            return big_bytes / (best / 1e3) / 1e9
+
+        link_before = link_rate()
+        # three timed blocks of e_steps steps; the host (its memory and link)
+        # is shared with other jobs, so the median block is reported, with all three
+        blocks = []
         for _ in range(3):
-            l0.record(copy_stream)
-            with torch.cuda.stream(copy_stream):
-                dins[0][big].copy_(host[big], non_blocking=True)
-            l1.record(copy_stream)
+            if world > 1:
+                dist.barrier()
+            a = torch.cuda.Event(enable_timing=True)
+            z = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            copy_stream.wait_event(a)
+            for i in range(e_steps):
+                e2e_step(i)
+            z.record(stream)
             torch.cuda.synchronize()
-            link_ms.append(l0.elapsed_time(l1))
-        link_gbs = big_bytes / (min(link_ms) / 1e3) / 1e9
+            blocks.append(aggregate(a.elapsed_time(z), meta["B"] * e_steps, dev))
+        link_after = link_rate()
+        ems, e_images = sorted(blocks, key=lambda bl: bl[0])[1]
+        link_gbs = max(link_before, link_after)
         step_gbs = (copied_bytes + in_place) / (ems / e_steps / 1e3) / 1e9
         e2e = {"value": e_images / (ems / 1e3), "unit": UNIT,
-               "host_link": {"h2d_gbs": link_gbs, "bytes": int(big_bytes), "tensor": big,
-                             "how": "copy-engine host->device copy from pinned memory, best of 3, after the timed region"},
+               "blocks": [bi / (bm / 1e3) for bm, bi in blocks],
+               "host_link": {"h2d_gbs": link_gbs, "before": link_before, "after": link_after, "bytes": int(big_bytes),
+                             "tensor": big,
+                             "how": "copy-engine host->device copy from pinned memory, best of 3, before and after "
+                                    "the timed blocks (the larger is h2d_gbs)"},
                "h2d_gbs_per_step": step_gbs, "frac_of_host_link": step_gbs / link_gbs,
                "h2d_bytes_per_step": int(copied_bytes + in_place), "d2h_bytes_per_step": int(d2h),
-               "steps": e_steps, "h2d_copied_bytes_per_step": int(copied_bytes),
+               "steps": e_steps, "timed_blocks": 3, "h2d_copied_bytes_per_step": int(copied_bytes),
                "h2d_read_in_place_bytes_per_step": int(in_place),
                "inputs": f"pinned host memory; {', '.join(copy_names)} copied each step (two device "
                          "input sets, the next step's copies overlapping the current step); K2, hidden, V "
