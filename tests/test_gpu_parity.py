@@ -119,6 +119,22 @@ def test_prune_mutual_late_large_logits(d1):
     check_prune(b, gpu, 0.5, 1.1)
 
 
+@pytest.mark.parametrize("B", [300, 2100])
+def test_many_samples(B):
+    """More samples than the planning CTA's 256 threads (the plan walks them
+    in chunks) and, at 2,100, more than the 2,048 whose row offsets and
+    thresholds the scan stages in shared memory; samples of 0-11 visual rows
+    and one register."""
+    rng = np.random.default_rng(B)
+    P = tuple(int(x) for x in rng.integers(0, 12, size=B))
+    M = tuple(int(x) for x in rng.integers(1, 20, size=B))
+    b = _tiny(B=B, segs=1, P=P, R=1, M=M, hidden=32, seed=50, sinks=("count", 0))
+    gpu = run_prune(b, 0.3, 1.1)
+    assert gpu["status"] == 0
+    rep = check_prune(b, gpu, 0.3, 1.1)
+    assert rep["kept"] > 0
+
+
 @pytest.mark.parametrize("name", ["llava15_b1", "llavanext_b8"])
 def test_small_workloads(name):
     w = get_config(name)
