@@ -119,6 +119,19 @@ def test_prune_mutual_late_large_logits(d1):
     check_prune(b, gpu, 0.5, 1.1)
 
 
+@pytest.mark.parametrize("lam1", [0.3, 0.0])
+def test_segment_above_finalize_staging(lam1):
+    """A [CLS] segment of 23,004 rows, above the 22,400 whose s1 and roles the
+    finalize kernel stages in shared memory (it works from global memory),
+    with a small sample beside it; at lambda1 = 0 every row enters S1 and
+    Stage II takes the two-pass path for the large sample."""
+    b = _tiny(B=2, segs=1, P=(23000, 40), R=4, M=(8, 5), hidden=32, seed=51)
+    gpu = run_prune(b, lam1, 1.1)
+    assert gpu["status"] == 0
+    rep = check_prune(b, gpu, lam1, 1.1)
+    assert rep["kept"] > 0
+
+
 @pytest.mark.parametrize("B", [300, 2100])
 def test_many_samples(B):
     """More samples than the planning CTA's 256 threads (the plan walks them
