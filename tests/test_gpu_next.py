@@ -51,11 +51,17 @@ def _lambda2_case(b, s2, ref2, keep1, K):
 
     m = b["meta"]
     layout = occ.BatchLayout.from_batch(b, "cuda")
+    _lambda2_check(layout, m["total_rows"], m["reg_idx_host"], m["row_off_host"], s2, ref2, keep1, K)
+
+
+def _lambda2_check(layout, total_rows, reg_idx, row_off, s2, ref2, keep1, K):
+    import paper_2605_29657_gb300 as occ
+
     lam, n = occ.occam_calibrate_lambda2(layout, torch.from_numpy(s2).cuda(), torch.from_numpy(ref2).cuda(),
                                          torch.from_numpy(keep1.astype(np.uint8)).cuda(), K)
     torch.cuda.synchronize()
-    is_reg = O.register_mask(m["total_rows"], m["reg_idx_host"])
-    want, n_want = O.lambda2_for_budget(s2, ref2, keep1, is_reg, m["row_off_host"], K)
+    is_reg = O.register_mask(total_rows, reg_idx)
+    want, n_want = O.lambda2_for_budget(s2, ref2, keep1, is_reg, row_off, K)
     got = lam.cpu().numpy()[0]
     assert int(n.cpu()[0]) == n_want
     assert got.tobytes() == np.float32(want).tobytes(), (K, got, want)   # bit-exact: same fp32 arithmetic
@@ -90,6 +96,29 @@ def test_lambda2_select_matches_oracle_random(seed):
     n = int(keep1.sum())
     for K in (0, 1, 2, 17, n // 2, n - 1, n, n + 5, 10 ** 9):
         _lambda2_case(b, s2, ref2, keep1, K)
+
+
+def test_lambda2_select_at_batch_scale():
+    """192,000 rows (64 samples of 2,996 visual rows and 4 registers): every
+    grid pass of the selection walks several rows per thread. Scores with
+    ties, exact zeros and a few samples without a positive reference."""
+    import paper_2605_29657_gb300 as occ
+
+    B, n = 64, 3000
+    row_off = np.arange(B + 1, dtype=np.int64) * n
+    reg_idx = np.concatenate([b * n + n - 4 + np.arange(4) for b in range(B)]).astype(np.int32)
+    layout = occ.BatchLayout(row_off, row_off.copy(), reg_idx, np.arange(B + 1) * 4, np.arange(B + 1) * 8)
+    rng = np.random.default_rng(7)
+    R = B * n
+    s2 = (rng.random(R) * rng.choice([1e-4, 1e-2, 1.0], R)).astype(np.float32)
+    s2[rng.random(R) < 0.05] = 0.0
+    s2[rng.random(R) < 0.05] = np.float32(0.5)              # ties
+    ref2 = (rng.random(B) * 0.01 + 1e-4).astype(np.float32)
+    ref2[[3, 17]] = 0.0                                     # samples without a positive reference
+    keep1 = rng.random(R) < 0.5
+    n_cand = int(np.sum(keep1 & ~O.register_mask(R, reg_idx) & (ref2[np.repeat(np.arange(B), n)] > 0)))
+    for K in (1, 1000, 34000, n_cand - 1, n_cand, n_cand + 1, 0):
+        _lambda2_check(layout, R, reg_idx, row_off, s2, ref2, keep1, K)
 
 
 def test_lambda2_select_on_oracle_scores():
