@@ -436,10 +436,12 @@ int launch_twopass(const Stage2Params& p, const WsLayout& L, int sms, const occa
   const int gB = (int)std::min<int64_t>(L.maxB, sms);
   if (gA <= 0 && gB <= 0) return OCCAM_OK;
   // both passes on the tensor cores: keys copied from K2 (and the text keys)
-  // by row with cp.async, the text queries in TMA boxes of 64 rows
-  CUtensorMap mq64;
+  // by row with cp.async, the text queries in TMA boxes of 128 rows
+  // (statistics) and 64 rows (scores)
+  CUtensorMap mq128, mq64;
+  if (!encode_map(&mq128, a->Q_text, b->total_text, (int64_t)a->H2 * 128, kStatsTile)) return OCCAM_ERR_CUDA;
   if (!encode_map(&mq64, a->Q_text, b->total_text, (int64_t)a->H2 * 128, kTextTile)) return OCCAM_ERR_CUDA;
-  if (gA > 0 && launch_stats_tc(p, mq64, gA, st) != 0) return OCCAM_ERR_CUDA;
+  if (gA > 0 && launch_stats_tc(p, mq128, gA, st) != 0) return OCCAM_ERR_CUDA;
   if (gB > 0 && launch_scores_tc(p, mq64, gB, st) != 0) return OCCAM_ERR_CUDA;
   return OCCAM_OK;
 }

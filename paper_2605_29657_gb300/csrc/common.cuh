@@ -245,7 +245,8 @@ enum {
   CNT_SLOTS = 14
 };
 
-constexpr int kTextTile = 64;    // Stage-II text rows per item
+constexpr int kTextTile = 64;    // Stage-II text rows per item of the two-pass score pass
+constexpr int kStatsTile = 128;  // Stage-II text rows per item of the two-pass statistics pass
 constexpr int kHeadGroup = 4;    // Stage-II heads per stats item
 constexpr int kStatSplits = 16;  // at most this many key ranges per (text tile, head group) in the stats pass
 constexpr int kKeyChunk = 128;   // Stage-II image keys per score item

@@ -313,7 +313,7 @@ __global__ void threshold_kernel(ThresholdParams p);
 // stage2.cu
 
 int s2_stats_smem_bytes();
-int launch_stats_tc(const Stage2Params& p, const CUtensorMap& mq64, int grid, cudaStream_t st);
+int launch_stats_tc(const Stage2Params& p, const CUtensorMap& mq128, int grid, cudaStream_t st);
 
 // stage2_tc.cu
 int fused_resident_clusters(int C);

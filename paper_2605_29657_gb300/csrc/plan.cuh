@@ -70,10 +70,9 @@ __device__ __forceinline__ void plan_stage2(const Stage2Params& p, int* tmp) {
       } else if (fused16) {
         nF16 = (M + 127) / 128 * hsg;
       } else {
-        const int tiles = (M + kTextTile - 1) / kTextTile;
         const int nch = (n1 + kKeyChunk - 1) / kKeyChunk;
-        nA = tiles * nhg * s2_stat_splits(n1, M);
-        nB = tiles * nch;
+        nA = (M + kStatsTile - 1) / kStatsTile * nhg * s2_stat_splits(n1, M);
+        nB = (M + kTextTile - 1) / kTextTile * nch;
       }
       if (M == 0) {
         set_status(p.status, OCCAM_ERR_INVALID_ARG);

@@ -7,27 +7,27 @@
 //
 // Samples the fused kernel cannot hold take two passes, so that any S1 size
 // and any text length fit:
-//   stats  (item = sample, 64 text rows, 4 heads, key range): per (j, h)
+//   stats  (item = sample, 128 text rows, 4 heads, key range): per (j, h)
 //          the softmax max and sum over the range's keys; a sample's keys
 //          are split into up to 16 ranges so that large samples still
 //          spread over the SMs (this file);
 //   scores (item = sample, 64 text rows, 128 S1 keys): stage2_scores_tc.cu.
 //
 // The statistics pass on the 5th-generation tensor cores. Per head of an
-// item, the 64 text queries are the MMA's A operand (one text row per TMEM
-// lane; M = 128, lanes 64-127 unused, their smem rows zeroed once), and the
-// range's keys come as B in blocks of 128 (S1 rows of K2 by the S1 list,
-// then the tile's text keys; zero-filled past the range), copied by three
-// loader warps with 16-byte cp.async into the 128-byte-swizzled K-major
-// layout. D = Q K^T (128 x 128 fp32) alternates between two TMEM buffers.
-// Four epilogue warps (TMEM lane quadrants 0 and 1, two column halves each)
-// keep an online max and sum per text row over their columns, in log2
-// units; at the head's last block the second half hands its pair to the
-// first through shared memory, and the first writes the merged partial.
-// Roles (320 threads): warps 0, 2, 3 load keys (warp 0 also issues the query
-// tile's TMA boxes), warp 1 issues the MMAs, warps 4, 5, 8, 9 are the
-// epilogue, warps 6 and 7 idle. Every wait is bounded; on a timeout the CTA
-// records OCCAM_ERR_TIMEOUT, lets its copies land, frees TMEM and returns.
+// item, the 128 text queries are the MMA's A operand (one text row per TMEM
+// lane, two TMA boxes of 128 rows), and the range's keys come as B in blocks
+// of 128 (S1 rows of K2 by the S1 list, then the tile's text keys;
+// zero-filled past the range), copied by seven loader warps with 16-byte
+// cp.async into the 128-byte-swizzled K-major layout. D = Q K^T (128 x 128
+// fp32) alternates between two TMEM buffers. Eight epilogue warps (the four
+// TMEM lane quadrants, two column halves each) keep an online max and sum
+// per text row over their columns, in log2 units; at the head's last block
+// the second half hands its pair to the first through shared memory, and
+// the first writes the merged partial.
+// Roles (512 threads): warps 0, 2, 3 and 12-15 load keys (warp 0 also
+// issues the query tile's TMA boxes), warp 1 issues the MMAs, warps 4-11
+// are the epilogue. Every wait is bounded; on a timeout the CTA records
+// OCCAM_ERR_TIMEOUT, lets its copies land, frees TMEM and returns.
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc5.cuh"
@@ -35,21 +35,22 @@
 namespace occam {
 
 namespace s2s {
-constexpr int QR = 128;                   // MMA M (text rows 0..63 of the tile are real)
+constexpr int QR = kStatsTile;            // MMA M: the item's text rows
 constexpr int KB = 128;                   // keys per block (MMA N)
 constexpr int QBYTES = QR * 128;          // one 64-dim K-block of the query operand
 constexpr int KBYTES = KB * 128;          // one 64-dim K-block of the key block
 constexpr int NST = 3;                    // key block stages
-constexpr int NLOAD = 96;                 // key loader threads (warps 0, 2, 3)
-constexpr int THREADS = 10 * 32;
+constexpr int NLOAD = 7 * 32;             // key loader threads (warps 0, 2, 3, 12-15)
+constexpr int NEPI = 8;                   // epilogue warps (4-11)
+constexpr int THREADS = 16 * 32;
 constexpr int KT = 64;                    // keys per range chunk (ranges are whole chunks)
 constexpr uint64_t kLimitNs = 2000000000ull;
-static_assert(kTextTile == 64, "query rows 64..127 of the MMA are padding");
+static_assert(kStatsTile == 128, "one text row per TMEM lane");
 
 struct Smem {
   uint8_t q[2][2][QBYTES];   // query tile per head: [buffer][K-block], 128-byte swizzled rows
   uint8_t k[NST][2][KBYTES]; // key block: [stage][K-block]
-  float2 part[2][64];        // the second column half's (max, sum) per text row, by head parity
+  float2 part[2][QR];        // the second column half's (max, sum) per text row, by head parity
   uint64_t qfull[2], qempty[2], kfull[NST], kempty[NST], dfull[2], dfree[2], hsync[2];
   uint32_t tmem_base;
   int abort;
@@ -89,11 +90,11 @@ __device__ __forceinline__ StatsItem decode_stats_item(const Stage2Params& p, in
   const int nhg = (p.H + kHeadGroup - 1) / kHeadGroup;
   const int nsp = s2_stat_splits(s.n_img, s.M);
   const int i = it - p.itemA_off[s.b];
-  s.j0 = (i / (nhg * nsp)) * kTextTile;
+  s.j0 = (i / (nhg * nsp)) * kStatsTile;
   const int hg = (i / nsp) % nhg;
   s.sp = i % nsp;
-  s.nq = min(kTextTile, s.M - s.j0);
-  const int n_txt = p.Kt ? min(s.j0 + kTextTile, s.M) : 0;
+  s.nq = min(kStatsTile, s.M - s.j0);
+  const int n_txt = p.Kt ? min(s.j0 + kStatsTile, s.M) : 0;
   s.total = s.n_img + n_txt;
   // the range's chunks [c0, c1) of the tile's key list (may be empty)
   const int nchunks = (s.total + KT - 1) / KT;
@@ -151,8 +152,8 @@ __global__ void __launch_bounds__(s2s::THREADS, 1)
       tc::bar_init(&sm.qfull[i], 1);
       tc::bar_init(&sm.qempty[i], 1);
       tc::bar_init(&sm.dfull[i], 1);
-      tc::bar_init(&sm.dfree[i], 4);
-      tc::bar_init(&sm.hsync[i], 2);
+      tc::bar_init(&sm.dfree[i], NEPI);
+      tc::bar_init(&sm.hsync[i], NEPI / 2);
     }
     for (int i = 0; i < NST; ++i) {
       tc::bar_init(&sm.kfull[i], NLOAD);
@@ -162,26 +163,18 @@ __global__ void __launch_bounds__(s2s::THREADS, 1)
     tc::bar_fence_init();
     tc::prefetch_map(&mapQ);
   }
-  {
-    // query rows 64..127 are never loaded: zero them once, so the unused
-    // lanes of D hold finite values
-    uint4* z4 = reinterpret_cast<uint4*>(&sm.q[0][0][0]);
-    constexpr int n16 = (int)(sizeof(sm.q) / 16);
-    for (int i = tid; i < n16; i += THREADS) z4[i] = make_uint4(0u, 0u, 0u, 0u);
-    tc::fence_proxy_async();
-  }
   if (warp == 1) tc::tmem_alloc(&sm.tmem_base, 2 * KB);
   tc::fence_before();
   __syncthreads();
   tc::fence_after();
   const uint32_t tmem = sm.tmem_base;
 
-  if (warp == 0 || warp == 2 || warp == 3) {
+  if (warp == 0 || warp == 2 || warp == 3 || warp >= 12) {
     // ------------------------------------------------------------ loaders
     // block g: 2,048 16-byte copies, copy i = (key i >> 4, K-block
     // (i >> 3) & 1, chunk i & 7) at chunk ^ (key & 7) of its 128-byte row;
     // block g - 1 is signalled once this thread's copies for it landed
-    const int lt = (warp == 0 ? 0 : warp - 1) * 32 + lane;
+    const int lt = (warp == 0 ? 0 : warp < 12 ? warp - 1 : warp - 9) * 32 + lane;
     const int64_t HD = (int64_t)p.Hkv * 128;
     uint32_t g = 0, gq = 0;
     bool ok = true, pending = false;
@@ -204,7 +197,7 @@ __global__ void __launch_bounds__(s2s::THREADS, 1)
               break;
             }
             if (lane == 0) {
-              tc::bar_expect_tx(&sm.qfull[qb], 2 * kTextTile * 128);
+              tc::bar_expect_tx(&sm.qfull[qb], 2 * QBYTES);
               tc::tma_load_2d(sm.q[qb][0], &mapQ, h * 128, (int)(s.t0 + s.j0), &sm.qfull[qb]);
               tc::tma_load_2d(sm.q[qb][1], &mapQ, h * 128 + 64, (int)(s.t0 + s.j0), &sm.qfull[qb]);
             }
@@ -283,9 +276,9 @@ __global__ void __launch_bounds__(s2s::THREADS, 1)
       }
     }
     __syncwarp();
-  } else if (warp == 4 || warp == 5 || warp == 8 || warp == 9) {
+  } else if (warp >= 4 && warp < 4 + NEPI) {
     // ------------------------------------------------------------ epilogue
-    const int quad = warp & 3, half = warp >> 3;  // text rows quad * 32 + lane, columns half * 64 ..
+    const int quad = warp & 3, half = (warp - 4) >> 2;  // text rows quad * 32 + lane, columns half * 64 ..
     const int row = quad * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
     uint32_t g = 0, gq = 0;
@@ -369,9 +362,9 @@ __global__ void __launch_bounds__(s2s::THREADS, 1)
   if (warp == 1) tc::tmem_dealloc(tmem, 2 * KB);
 }
 
-int launch_stats_tc(const Stage2Params& p, const CUtensorMap& mq64, int grid, cudaStream_t st) {
+int launch_stats_tc(const Stage2Params& p, const CUtensorMap& mq128, int grid, cudaStream_t st) {
   cudaFuncSetAttribute(s2_stats_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, s2_stats_smem_bytes());
-  s2_stats_tc_kernel<<<grid, s2s::THREADS, s2_stats_smem_bytes(), st>>>(mq64, p);
+  s2_stats_tc_kernel<<<grid, s2s::THREADS, s2_stats_smem_bytes(), st>>>(mq128, p);
   count_launch();
   return cudaGetLastError() == cudaSuccess ? 0 : 1;
 }

@@ -17,11 +17,12 @@
 // swizzled K-major layout), the 64 text queries its B operand (one TMA box
 // per 64-dim K-block), and D = K Q^T (128 x 64 fp32) lands in one of two
 // TMEM buffers. The key rows are scattered: per-copy TMA gathers (four rows
-// a copy) left this pass bound by the copy rate, while 96 threads' cp.async
-// keep two heads' key tiles in flight.
-// Roles (384 threads): warps 0, 2 and 3 load the keys (warp 0 also issues
-// the query TMA boxes), warp 1 issues the MMAs, warps 4-11 (two per TMEM
-// lane quadrant, 32 text rows each) add each head into register
+// a copy) left this pass bound by the copy rate, while 224 threads' cp.async
+// keep two heads' key tiles in flight (the copy rate grows with the number
+// of issuing warps).
+// Roles (512 threads): warps 0, 2, 3 and 12-15 load the keys (warp 0 also
+// issues the query TMA boxes), warp 1 issues the MMAs, warps 4-11 (two per
+// TMEM lane quadrant, 32 text rows each) add each head into register
 // accumulators. Operands have three stages, accumulators two. A loader
 // signals a stage once its own copies landed and, through a proxy fence,
 // are visible to the tensor cores. Every wait is bounded; on a timeout the
@@ -39,10 +40,10 @@ constexpr int TR = kTextTile;             // text rows per item (MMA N)
 constexpr int ABYTES = KR * 128;          // one 64-dim K-block of the key tile
 constexpr int BBYTES = TR * 128;          // one 64-dim K-block of the query tile
 constexpr int NST = 3;                    // operand stages
-constexpr int NLOAD = 96;                 // key loader threads (warps 0, 2, 3)
+constexpr int NLOAD = 7 * 32;             // key loader threads (warps 0, 2, 3, 12-15)
 constexpr int EPI0 = 4;                   // first softmax warp
 constexpr int NEPI = 8;
-constexpr int THREADS = (EPI0 + NEPI) * 32;
+constexpr int THREADS = 16 * 32;
 constexpr int HMAX = 64;                  // heads the statistics table holds
 constexpr uint64_t kLimitNs = 2000000000ull;
 static_assert(TR == 64, "two softmax warps of 32 rows per quadrant");
@@ -176,14 +177,14 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
     tc::fence_after();
     if (*abort) break;  // uniform: read after the barrier
 
-    if (warp == 0 || warp == 2 || warp == 3) {
+    if (warp == 0 || warp == 2 || warp == 3 || warp >= EPI0 + NEPI) {
       // ---------------------------------------------------------- loaders
       // per head: the key tile's 2 x 128 rows of 128 bytes as 2,048 16-byte
       // copies, copy i = (key i >> 4, K-block (i >> 3) & 1, chunk i & 7),
       // written where the 128-byte swizzle puts it (chunk ^ (row & 7)); then
       // stage g - 1 is signalled once this thread's copies for it landed.
       // Lane 0 of warp 0 also issues the query tile's two TMA boxes.
-      const int lt = (warp == 0 ? 0 : warp - 1) * 32 + lane;
+      const int lt = (warp == 0 ? 0 : warp < EPI0 ? warp - 1 : warp - (EPI0 + NEPI - 3)) * 32 + lane;
       const int64_t HD = (int64_t)p.Hkv * 128;
       bool ok = true;
       for (int h = 0; h < H && ok; ++h) {
@@ -245,7 +246,7 @@ __global__ void __launch_bounds__(s2t::THREADS, 1)
         }
       }
       __syncwarp();
-    } else if (warp >= EPI0) {
+    } else if (warp >= EPI0) {  // warps EPI0 .. EPI0 + NEPI - 1
       // ---------------------------------------------------------- softmax warps
       const int ew = warp - EPI0, quad = warp & 3, half = ew >> 2;
       const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
