@@ -33,6 +33,17 @@ constexpr unsigned long long kValMask = (1ull << 62) - 1;
 
 constexpr int kScanSmemSamples = 2048;  // samples whose offsets fit the scan's shared copy
 
+// Writes the byte flags of rows r0 .. r0 + 7 (byte i of w for row r0 + i) to
+// o (nullable): one 8-byte store where the rows are whole and aligned.
+__device__ __forceinline__ void store_flags8(uint8_t* o, int64_t r0, int64_t R, bool whole, uint64_t w) {
+  if (o == nullptr) return;
+  if (whole && (reinterpret_cast<uintptr_t>(o) & 7) == 0) {
+    *reinterpret_cast<uint64_t*>(o + r0) = w;
+  } else {
+    for (int i = 0; i < 8 && r0 + i < R; ++i) o[r0 + i] = (uint8_t)(w >> (8 * i));
+  }
+}
+
 __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   constexpr int PER = kScanTile / 256;  // 8 rows per thread
   __shared__ int tmp[40];
@@ -56,7 +67,35 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   const int64_t tile = s_tile;
   const int64_t R = p.bt.total_rows;
   const int64_t r_first = tile * kScanTile + (int64_t)tid * PER;
-  // flags of my rows
+  // flags of my rows. Their inputs are loaded first, all together (one
+  // memory round trip: 8-byte loads of the byte flags and 16-byte loads of
+  // s2 where the rows are whole and aligned), then tested.
+  uint64_t in_a = 0, in_b = 0;  // byte i: row r_first + i (mode 0: keep_in, role; mode 1: role, keep1)
+  float in_s[PER];              // mode 1: s2
+  const uint8_t* pa = p.mode == 0 ? p.keep_in : p.role;
+  const uint8_t* pb = p.mode == 0 ? p.role : p.keep1;
+  const bool whole = r_first + PER <= R;
+  const bool vec = whole && ((reinterpret_cast<uintptr_t>(pa) | reinterpret_cast<uintptr_t>(pb)) & 7) == 0 &&
+                   (p.mode == 0 || (reinterpret_cast<uintptr_t>(p.s2) & 15) == 0);
+  if (vec) {
+    in_a = *reinterpret_cast<const uint64_t*>(pa + r_first);
+    if (pb) in_b = *reinterpret_cast<const uint64_t*>(pb + r_first);
+    if (p.mode != 0) {
+      const float4 s0 = *reinterpret_cast<const float4*>(p.s2 + r_first);
+      const float4 s1 = *reinterpret_cast<const float4*>(p.s2 + r_first + 4);
+      in_s[0] = s0.x; in_s[1] = s0.y; in_s[2] = s0.z; in_s[3] = s0.w;
+      in_s[4] = s1.x; in_s[5] = s1.y; in_s[6] = s1.z; in_s[7] = s1.w;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      const int64_t r = r_first + i;
+      const bool ok = r < R;
+      in_a |= (uint64_t)(ok ? pa[r] : 0) << (8 * i);
+      in_b |= (uint64_t)(ok && pb ? pb[r] : 0) << (8 * i);
+      in_s[i] = ok && p.mode != 0 ? p.s2[r] : 0.f;
+    }
+  }
   unsigned kmask = 0, vmask = 0;
   int samp = -1;
   int64_t samp_end = 0;
@@ -65,32 +104,36 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
     if (!in_bounds(samp >= 0 && samp < p.bt.B, p.status, kSiteScanSample)) samp = 0;
     samp_end = row_off[samp + 1];
   }
+  uint64_t kw = 0, nw = 0;  // keep2 and near bytes of my rows
 #pragma unroll
   for (int i = 0; i < PER; ++i) {
     const int64_t r = r_first + i;
-    if (r >= R) break;
-    while (r >= samp_end) { ++samp; samp_end = row_off[samp + 1]; }
-    bool k, vis;
-    if (p.mode == 0) {
-      k = p.keep_in[r] != 0;
-      vis = k && (p.role == nullptr || p.role[r] == 0);
-    } else {
-      const bool reg = p.role[r] != 0;
-      if (reg) {
+    bool k = false, vis = false, nr = false;
+    if (r < R) {
+      while (r >= samp_end) { ++samp; samp_end = row_off[samp + 1]; }
+      if (p.mode == 0) {
+        k = (in_a >> (8 * i) & 0xffu) != 0;
+        vis = k && (p.role == nullptr || (in_b >> (8 * i) & 0xffu) == 0);
+      } else if ((in_a >> (8 * i) & 0xffu) != 0) {  // a register row
         k = p.keep_registers != 0;
-        vis = false;
       } else {
-        const float sv = p.s2[r], t = tau2[samp];
-        k = (p.keep1[r] != 0) && (sv >= t);
+        const float sv = in_s[i], t = tau2[samp];
+        const bool s1row = (in_b >> (8 * i) & 0xffu) != 0;
+        k = s1row && (sv >= t);
         vis = k;
         // near-threshold flag of a visual S1 row: the same fp32 tau as the test
-        if (p.near_out) p.near_out[r] = p.keep1[r] != 0 && fabsf(sv - t) <= p.near_rel * fabsf(t) ? 1 : 0;
+        nr = s1row && fabsf(sv - t) <= p.near_rel * fabsf(t);
       }
-      if (p.near_out && reg) p.near_out[r] = 0;
-      if (p.keep_out) p.keep_out[r] = k ? 1 : 0;
     }
+    kw |= (uint64_t)k << (8 * i);
+    nw |= (uint64_t)nr << (8 * i);
     kmask |= (unsigned)k << i;
     vmask |= (unsigned)vis << i;
+  }
+  if (p.mode != 0) {
+    // keep2 and the near flags of my rows, 8 bytes at a time where aligned
+    store_flags8(p.keep_out, r_first, R, whole, kw);
+    store_flags8(p.near_out, r_first, R, whole, nw);
   }
   const int cnt = __popc(kmask);
   int tile_total;

@@ -208,10 +208,11 @@ __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, in
   __shared__ float gmax[16], ginv[16], lcls_s[16];
   const int tid = threadIdx.x;
   // thread t takes head (t & 15) of rows (t >> 4) + 16 k: a warp reads 32
-  // consecutive floats per row pair. Up to 32 rows' loads are in flight at
+  // consecutive floats per row pair. Up to 40 rows' loads are in flight at
   // once (issued before the [CLS] key's dot product below, which they
-  // overlap), so a segment of up to 512 rows costs one L2 round trip.
-  constexpr int KC = 32;
+  // overlap), so a segment of up to 640 rows (a 576-token crop with its
+  // registers) costs one L2 round trip.
+  constexpr int KC = 40;
   const float* lg = p.logits + sb * H;
   const int h = tid & 15, j = tid >> 4;
   float x[KC];
@@ -313,6 +314,12 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   const int64_t sb = p.bt.seg_off[seg], se = p.bt.seg_off[seg + 1];
   const int n = (int)(se - sb);
   const int ra = p.bt.reg_off[seg], rb = p.bt.reg_off[seg + 1];
+  // loaded now, used after the softmax: the sample's segment range and row
+  // range (for the S1 list) and this thread's first register index
+  const int b = p.bt.seg_sample[seg];
+  const int s0 = p.bt.seg_first[b], s_next = p.bt.seg_first[b + 1];
+  const int64_t row_b = p.bt.row_off[b], row_b1 = p.bt.row_off[b + 1];
+  const int64_t reg0 = ra + tid < rb ? (int64_t)p.bt.reg_idx[ra + tid] : -1;
   const bool staged = n <= p.smem_rows;
   // shared layout for a staged segment: [s1][role]
   float* s1_loc = reinterpret_cast<float*>(fin_smem);
@@ -329,7 +336,7 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
     for (int r = tid; r < n; r += blockDim.x) role_loc[r] = 0;
     __syncthreads();
     for (int i = ra + tid; i < rb; i += blockDim.x) {
-      const int64_t reg = p.bt.reg_idx[i];
+      const int64_t reg = i == ra + tid ? reg0 : p.bt.reg_idx[i];
       if (in_bounds(reg >= sb && reg < se, p.status, kSiteRegisterRow)) role_loc[reg - sb] = 1;
     }
     __syncthreads();
@@ -338,7 +345,7 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
     for (int r = tid; r < n; r += blockDim.x) p.role[sb + r] = 0;
     __syncthreads();
     for (int i = ra + tid; i < rb; i += blockDim.x) {
-      const int64_t reg = p.bt.reg_idx[i];
+      const int64_t reg = i == ra + tid ? reg0 : p.bt.reg_idx[i];
       if (in_bounds(reg >= sb && reg < se, p.status, kSiteRegisterRow)) p.role[reg] = 1;
     }
     __syncthreads();
@@ -368,7 +375,7 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
     float v = 0.f;
     if (s1g) {
       for (int i = ra + tid; i < rb; i += blockDim.x) {
-        const int64_t row = p.bt.reg_idx[i];
+        const int64_t row = i == ra + tid ? reg0 : p.bt.reg_idx[i];
         v += staged ? s1_loc[row - sb] : s1g[row];
       }
     }
@@ -404,8 +411,6 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   // sample's earlier segments (warp 0, a window of 32 at a time). A state
   // packs the visual count (bits 31..61) and the key count (bits 0..30)
   // with an "aggregate" or "inclusive prefix" flag.
-  const int b = p.bt.seg_sample[seg];
-  const int s0 = p.bt.seg_first[b];
   constexpr unsigned long long kAgg = 1ull << 62, kPre = 2ull << 62, kLo = (1ull << 31) - 1;
   if (tid < 32) {
     const unsigned long long mine = ((unsigned long long)vis_total << 31) | (unsigned long long)total;
@@ -444,15 +449,15 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
     }
     if (tid == 0) {
       s_base = (long long)(excl & kLo);
-      if (seg + 1 == p.bt.seg_first[b + 1]) {  // the sample's last segment
+      if (seg + 1 == s_next) {  // the sample's last segment
         p.n1[b] = (int)((excl & kLo) + (unsigned long long)total);
         if (p.n1_vis) p.n1_vis[b] = (int)(((excl >> 31) & kLo) + (unsigned long long)vis_total);
       }
     }
   }
   __syncthreads();
-  int32_t* list = p.dense + p.bt.row_off[b] + s_base;
-  const int64_t list_len = p.bt.row_off[b + 1] - p.bt.row_off[b] - s_base;  // room left in the sample's list
+  int32_t* list = p.dense + row_b + s_base;
+  const int64_t list_len = row_b1 - row_b - s_base;  // room left in the sample's list
   for (int r = a; r < z; ++r) {
     const bool reg = role[r] != 0;
     const float sv = p.keep_in ? 0.f : (staged ? s1_loc[r] : s1g[sb + r]);
