@@ -549,9 +549,6 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     q8.queue = p.counters + CNT_QUEUE8;
     const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
     if (!only16 && launch_fused(8, mq, mk, mkt, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
-    // the two-pass kernels (samples the fused kernel cannot hold; often none)
-    // follow the 8-CTA launch on the second stream
-    OCCAM_TRY(launch_twopass(p, L, sms, b, a, side.stream));
     // samples too large for 8 CTAs: 16-CTA clusters, on this stream ahead of
     // the 4-CTA launch. A launch without items returns at once; it also
     // lets the 8-CTA clusters (larger items) take their SMs first, which
@@ -561,6 +558,12 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     q16.queue = p.counters + CNT_QUEUE16;
     const int ncl16 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 16));
     if (launch_fused(16, mq, mk, mkt, q16, ncl16, st) != 0) return OCCAM_ERR_CUDA;
+    // the two-pass kernels (samples the fused kernel cannot hold; often none)
+    // follow the 8-CTA launch on the second stream. They are enqueued after
+    // the 16-CTA launch: a CTA of theirs takes a whole SM, and enqueued
+    // earlier they held every SM before the 16-CTA clusters, which need 16
+    // SMs of one GPC, could be placed.
+    OCCAM_TRY(launch_twopass(p, L, sms, b, a, side.stream));
     q.queue = p.counters + CNT_QUEUE4;
     const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
     if (!only16 && launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
