@@ -47,6 +47,9 @@ CASES = [
     ("fused_c8", dict(B=2, segs=1, P=(1000, 1532), R=4, M=(130, 33), seed=25), 0.0, 1.15),
     # one sample above the fused kernel's S1 limit (two-pass), one below (fused)
     ("mixed_paths", dict(B=2, segs=1, P=(1700, 200), R=3, M=(70, 90), seed=23), 0.0, 1.1),
+    # many key ranges (the two-pass statistics pass caps them at 16) over
+    # 128-row statistics tiles with ragged last tiles (M = 200, 257)
+    ("twopass_ranges", dict(B=2, segs=1, P=(1300, 2900), R=4, M=(200, 257), seed=26), 0.0, 1.1),
 ]
 
 
