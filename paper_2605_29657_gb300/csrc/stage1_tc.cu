@@ -434,19 +434,19 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
 #pragma unroll
               for (int i = 0; i < 64; ++i) v[i] = i < lim ? v[i] : 0xff800000u;  // -inf
             }
-            // max as a tree of three-input maxima (short dependency chains,
-            // few values live beside v)
-            float t[16];
+            // max as a tree of three-input maxima (32 operations for 64
+            // values; short dependency chains)
+            float t[22];
 #pragma unroll
-            for (int i = 0; i < 16; ++i)
-              t[i] = fmaxf(tc::fmax3(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]), __uint_as_float(v[4 * i + 2])),
-                           __uint_as_float(v[4 * i + 3]));
-            float u[6];
+            for (int i = 0; i < 21; ++i)
+              t[i] = tc::fmax3(__uint_as_float(v[3 * i]), __uint_as_float(v[3 * i + 1]), __uint_as_float(v[3 * i + 2]));
+            t[21] = __uint_as_float(v[63]);
+            float u[8];
 #pragma unroll
-            for (int i = 0; i < 5; ++i) u[i] = tc::fmax3(t[3 * i], t[3 * i + 1], t[3 * i + 2]);
-            u[5] = t[15];
+            for (int i = 0; i < 7; ++i) u[i] = tc::fmax3(t[3 * i], t[3 * i + 1], t[3 * i + 2]);
+            u[7] = t[21];
             // c > 0: the max of c l is c times the max of l
-            const float mx = fmaxf(tc::fmax3(u[0], u[1], u[2]), tc::fmax3(u[3], u[4], u[5])) * c;
+            const float mx = fmaxf(tc::fmax3(u[0], u[1], u[2]), tc::fmax3(u[3], u[4], fmaxf(u[5], fmaxf(u[6], u[7])))) * c;
             if (mx != -INFINITY) {
               const float2 cc = make_float2(c, c), om = make_float2(-mx, -mx);
               float2 ap[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
