@@ -179,9 +179,8 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         const int nb = (w.n + BR - 1) / BR;
         const int nheads = PASS == 1 ? 1 : min(kMutHeadGroup, H - w.h);
         bool ok = true;
-        for (int s = 0; s < nheads * nb && ok; ++s) {
-          const int h = w.h + s / nb;
-          const int jb = s % nb;
+        // step s is block jb of head h (counters instead of a division per step)
+        for (int s = 0, h = w.h, jb = 0; s < nheads * nb && ok; ++s, jb = jb + 1 == nb ? 0 : jb + 1, h += jb == 0) {
           if (jb == 0) {
             const int ab = na & 1;
             if (!tc::bar_wait(&sm.aempty[ab], ((na >> 1) & 1) ^ 1, abort, kLimitNs)) {
@@ -235,8 +234,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         const int nb = (w.n + BR - 1) / BR;
         const int nheads = PASS == 1 ? 1 : min(kMutHeadGroup, H - w.h);
         bool ok = true;
-        for (int s = 0; s < nheads * nb; ++s, ++sg) {
-          const int jb = s % nb;
+        for (int s = 0, jb = 0; s < nheads * nb; ++s, ++sg, jb = jb + 1 == nb ? 0 : jb + 1) {
           const int ab = na & 1, bb = sg % NBB, db = sg & 1;
           if (jb == 0) ok = tc::bar_wait(FOLD ? &sm.aready[ab] : &sm.afull[ab], (na >> 1) & 1, abort, kLimitNs);
           if (ok) ok = tc::bar_wait(FOLD ? &sm.bready[bb] : &sm.bfull[bb], (sg / NBB) & 1, abort, kLimitNs);
@@ -301,16 +299,15 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       // (clamped to the segment; rows past it are replaced below)
       constexpr int KR = BR / 64;  // B rows per lane and step
       float lpre[KR];
-      auto load_l = [&](int t) {
-        const int ht = w.h + t / nb, base = (t % nb) * BR + half * (BR / 2);
+      auto load_l = [&](int ht, int tb) {  // block tb of head ht
+        const int base = tb * BR + half * (BR / 2);
 #pragma unroll
         for (int k = 0; k < KR; ++k)
           lpre[k] = __ldcg(&p.lsum[(int64_t)ht * R + sb + min(base + lane + 32 * k, n - 1)]);
       };
-      load_l(0);
+      load_l(w.h, 0);
       bool ok = true;
-      for (int s = 0; s < steps; ++s) {
-        const int jb = s % nb;
+      for (int s = 0, h = w.h, jb = 0; s < steps; ++s, jb = jb + 1 == nb ? 0 : jb + 1, h += jb == 0) {
         if (jb == 0) {
           const int ab = na & 1;
           if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.afull[ab], (na >> 1) & 1, nullptr, kLimitNs))) {
@@ -333,7 +330,10 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         float cur[KR];
 #pragma unroll
         for (int k = 0; k < KR; ++k) cur[k] = lpre[k];
-        if (s + 1 < steps) load_l(s + 1);
+        if (s + 1 < steps) {
+          if (jb + 1 == nb) load_l(h + 1, 0);
+          else load_l(h, jb + 1);
+        }
 #pragma unroll
         for (int k = 0; k < KR; ++k) {
           const int r = half * (BR / 2) + lane + 32 * k;
@@ -389,9 +389,8 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       float m = -INFINITY, z = 0.f;  // pass 1: running max / sum (log2 domain)
       float acc = 0.f;               // pass 2: attention received by this key row
       bool ok = true;
-      for (int s = 0; s < steps; ++s, ++sg) {
-        const int h = w.h + s / nb;
-        const int jb = s % nb;
+      // step s is block jb of head h (counters instead of a division per step)
+      for (int s = 0, h = w.h, jb = 0; s < steps; ++s, ++sg, jb = jb + 1 == nb ? 0 : jb + 1, h += jb == 0) {
         const int col0 = jb * BR + qtr * COLS;          // segment-relative index of this warp's column 0
         if (PASS == 2 && !FOLD) {
           // minus the log-sums of this warp's 64 query columns (past the
@@ -399,8 +398,8 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
           // of two step slots, one step ahead; the item's first step's are
           // fetched here. The slot refilled below was last read in the
           // previous step, which every lane of the warp has finished.
-          auto fetch = [&](int t) {
-            const int ht = w.h + t / nb, ct = (t % nb) * BR + qtr * COLS;
+          auto fetch = [&](int t, int ht, int tb) {  // step t = block tb of head ht
+            const int ct = tb * BR + qtr * COLS;
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
               const int qq = ct + lane * 2 + i;
@@ -412,10 +411,13 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
             }
             cp_async_commit();
           };
-          if (s == 0) fetch(0);
+          if (s == 0) fetch(0, w.h, 0);
           cp_async_wait<0>();
           __syncwarp();
-          if (s + 1 < steps) fetch(s + 1);
+          if (s + 1 < steps) {
+            if (jb + 1 == nb) fetch(s + 1, h + 1, 0);
+            else fetch(s + 1, h, jb + 1);
+          }
         }
         const int db = sg & 1;
         if (!__all_sync(0xffffffffu, tc::bar_wait(&sm.dfull[db], (sg >> 1) & 1, nullptr, kLimitNs))) {
