@@ -49,6 +49,13 @@ constexpr int NBB = 4;                    // B blocks in flight (a ring; A tiles
 static_assert(COLS == 64, "one 64-column TMEM load per softmax warp and block");
 constexpr uint64_t kLimitNs = 2000000000ull;
 
+// A decoded work item: segment, first row of its tile, first head, the
+// segment's rows and its first row in the batch.
+struct MutItem {
+  int seg, a0, h, n;
+  int64_t sb;
+};
+
 struct Smem {
   uint8_t a[2][ABYTES];     // K-block 0 per buffer
   uint8_t b[NBB][BBYTES];
@@ -57,6 +64,7 @@ struct Smem {
   float lsm[2][NEPI][COLS];  // pass 2: minus the log-sums of each softmax warp's columns (a ring of 2 steps)
   float2 part[2][QW - 1][4][32];  // partials of quarters 1.. per (item parity, quarter, quadrant, lane)
   int32_t item[8];          // the ii-th work item, by ii & 7 (-1: no more)
+  MutItem itm[8];           // ... decoded by the TMA producer for every role
   uint64_t afull[2], aempty[2], bfull[NBB], bempty[NBB], dfull[2], dfree[2], hb[2][4], inext[8], mdone;
   uint64_t aready[2], bready[NBB];  // pass 2 with the log-sums folded into the MMA: tiles completed for it
   uint32_t tmem_base;
@@ -99,12 +107,9 @@ __device__ __forceinline__ void wait_ld64(uint32_t (&v)[64]) {
 // memory (the producer runs at most a few steps ahead, so a slot is read
 // before it comes round again); buffer and phase counters run on across
 // items, so the next item's loads overlap the current item's tail.
-struct MutItem {
-  int seg, a0, h, n;
-};
 
 template <int PASS>
-__device__ __forceinline__ bool mut_item(const MutualTcParams& p, int it, MutItem& w) {
+__device__ __forceinline__ bool mut_item(const MutualTcParams& p, int it, m1::MutItem& w) {
   const int sub_n = PASS == 1 ? p.H : p.hgroups;  // heads (pass 1) or head groups (pass 2) per tile
   const int per_seg = p.tiles * sub_n;
   w.seg = it / per_seg;
@@ -112,7 +117,8 @@ __device__ __forceinline__ bool mut_item(const MutualTcParams& p, int it, MutIte
   const int tile = rem / sub_n;
   w.h = (rem - tile * sub_n) * (PASS == 1 ? 1 : kMutHeadGroup);  // first head of the item
   w.a0 = tile * m1::AR;
-  w.n = (int)(p.bt.seg_off[w.seg + 1] - p.bt.seg_off[w.seg]);
+  w.sb = p.bt.seg_off[w.seg];
+  w.n = (int)(p.bt.seg_off[w.seg + 1] - w.sb);
   return w.a0 < w.n;
 }
 
@@ -172,10 +178,11 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         do {
           it = atomicAdd(queue, 1);
         } while (it < total && !mut_item<PASS>(p, it, w));
+        if (it < total) sm.itm[ii & 7] = w;
         sm.item[ii & 7] = it < total && !*abort ? it : -1;
         tc::bar_arrive(&sm.inext[ii & 7]);
         if (it >= total || *abort) break;
-        const int64_t sb = p.bt.seg_off[w.seg];
+        const int64_t sb = w.sb;
         const int nb = (w.n + BR - 1) / BR;
         const int nheads = PASS == 1 ? 1 : min(kMutHeadGroup, H - w.h);
         bool ok = true;
@@ -229,8 +236,7 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
         }
         const int it = *reinterpret_cast<volatile int*>(&sm.item[ii & 7]);
         if (it < 0) break;
-        MutItem w;
-        mut_item<PASS>(p, it, w);
+        const MutItem w = sm.itm[ii & 7];
         const int nb = (w.n + BR - 1) / BR;
         const int nheads = PASS == 1 ? 1 : min(kMutHeadGroup, H - w.h);
         bool ok = true;
@@ -289,10 +295,9 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       }
       const int it = *reinterpret_cast<volatile int*>(&sm.item[ii & 7]);
       if (it < 0) break;
-      MutItem w;
-      mut_item<PASS>(p, it, w);
+      const MutItem w = sm.itm[ii & 7];
       const int n = w.n;
-      const int64_t sb = p.bt.seg_off[w.seg];
+      const int64_t sb = w.sb;
       const int nb = (n + BR - 1) / BR;
       const int steps = min(kMutHeadGroup, H - w.h) * nb;
       // -L of the block's query rows lane + 32 k, loaded a step ahead
@@ -378,10 +383,9 @@ __global__ void __launch_bounds__(m1::THREADS, 1)
       }
       const int it = *reinterpret_cast<volatile int*>(&sm.item[ii & 7]);
       if (it < 0) break;
-      MutItem w;
-      mut_item<PASS>(p, it, w);
+      const MutItem w = sm.itm[ii & 7];
       const int n = w.n;
-      const int64_t sb = p.bt.seg_off[w.seg];
+      const int64_t sb = w.sb;
       const int nb = (n + BR - 1) / BR;
       const int steps = (PASS == 1 ? 1 : min(kMutHeadGroup, H - w.h)) * nb;
       const bool vrow = w.a0 + row < n;
