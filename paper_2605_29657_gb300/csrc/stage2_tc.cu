@@ -495,7 +495,8 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
               fail(sm, p.status);
               break;
             }
-            tc::fence_proxy_async();
+            // (the operands arrive by TMA, in the async proxy the MMA reads
+            // through: the barrier waits above are all the ordering needed)
             tc::fence_after();
             if (g.N > 0) {
               const uint32_t qa = tc::su32(sm.q[qb]), kbase = tc::su32(sm.k[kb]);
