@@ -9,6 +9,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <utility>
 
 #include "common.cuh"
 #include "kernels.cuh"
@@ -204,6 +205,24 @@ SideStream& side_stream(cudaStream_t caller) {
   return *s;
 }
 
+// Launches kern with the programmatic stream-serialization attribute: it may
+// start before the kernel ahead of it in the stream has finished, and waits
+// for that kernel's results where it calls pdl_wait() (common.cuh).
+template <class... P, class... A>
+cudaError_t launch_pdl(void (*kern)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, A&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<A>(args)...);
+}
+
 // 2-D bf16 map over a [rows, cols] row-major tensor, 128-byte swizzle, box
 // of 64 columns x box_rows rows.
 bool encode_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, uint32_t box_rows) {
@@ -386,7 +405,7 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
                      float lambda1, int do_threshold, float* ref1, uint8_t* keep1, int32_t* n1_vis,
                      const occam_stage1_args* a1, float* s2_zero, const Stage2Params* plan, int32_t* count_out,
                      int32_t* count_vis, cudaStream_t st, Trace trace = Trace(), float* n_eff = nullptr,
-                     int ref_mean = 0, uint8_t* near1 = nullptr, float near_rel = 1e-5f) {
+                     int ref_mean = 0, uint8_t* near1 = nullptr, float near_rel = 1e-5f, bool pdl = false) {
   const NvtxRange nvtx("stage1_finalize");
   Stage1FinalizeParams p;
   p.bt = dev_batch(b);
@@ -422,7 +441,15 @@ int launch_finalize1(const occam_batch* b, const WsLayout& L, void* ws, float* s
   p.zero_count_vis = count_vis;
   p.near1 = near1;
   p.near_rel = near_rel;
-  stage1_finalize_kernel<<<b->S_tot, 256, finalize_smem_bytes(p.smem_rows), st>>>(p);
+  // pdl (the op before this launch is the Stage-I kernel, which started after
+  // the call's counters were zeroed): programmatic dependent launch, so that
+  // the finalize kernel's input-only prologue (its segment ticket, the batch
+  // offsets, the [CLS] key's own logits) overlaps the end of that kernel
+  if (pdl)
+    OCCAM_CUDA(launch_pdl(stage1_finalize_kernel, dim3((unsigned)b->S_tot), dim3(256),
+                          (size_t)finalize_smem_bytes(p.smem_rows), st, p));
+  else
+    stage1_finalize_kernel<<<b->S_tot, 256, finalize_smem_bytes(p.smem_rows), st>>>(p);
   count_launch();
   trace.mark(st);
   return cuda_ok();
@@ -615,7 +642,14 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
     OCCAM_CUDA(cudaMemsetAsync(count_out, 0, b->B * 4, st));
     if (count_vis) OCCAM_CUDA(cudaMemsetAsync(count_vis, 0, b->B * 4, st));
   }
-  scan_kernel<<<(unsigned)L.scan_tiles, 256, 0, st>>>(p);
+  // without memsets just before it, the op ahead of the scan is a kernel that
+  // started after the call's counters were zeroed: programmatic dependent
+  // launch, the ticket and the row offsets read before that kernel finishes,
+  // everything else after (pdl_wait)
+  if (!do_memsets)
+    OCCAM_CUDA(launch_pdl(scan_kernel, dim3((unsigned)L.scan_tiles), dim3(256), 0, st, p));
+  else
+    scan_kernel<<<(unsigned)L.scan_tiles, 256, 0, st>>>(p);
   count_launch();
   trace.mark(st);
   if (n_tensors > 0) {
@@ -632,7 +666,9 @@ int launch_compact(const occam_batch* b, const WsLayout& L, void* ws, int mode, 
     g.capacity = capacity;
     g.src_rows = b->total_rows;
     g.status = at<int>(ws, L.status);
-    gather_kernel<<<num_sms() * 4, 256, 0, st>>>(g);
+    // programmatic dependent launch: scheduled as the scan ends, it waits for
+    // the scan's results inside (pdl_wait)
+    OCCAM_CUDA(launch_pdl(gather_kernel, dim3((unsigned)(num_sms() * 4)), dim3(256), 0, st, g));
     count_launch();
   }
   trace.mark(st);
@@ -695,7 +731,7 @@ int occam_score_stage1(const occam_batch* batch, const occam_stage1_args* args, 
   set_smem_attrs();
   OCCAM_TRY(launch_stage1_scores(batch, args, L, workspace, s1, nullptr, st));
   OCCAM_TRY(launch_finalize1(batch, L, workspace, s1, nullptr, 0.f, 0, ref1, nullptr, nullptr, args, nullptr, nullptr,
-                             nullptr, nullptr, st));
+                             nullptr, nullptr, st, Trace(), nullptr, 0, nullptr, 1e-5f, true));
   return OCCAM_OK;
 }
 
@@ -904,7 +940,7 @@ static int prune_impl(const occam_prune_args* args, const occam_prune_out* out, 
   const Stage2Params plan = stage2_params(b, &a2, L, ws, s2, ref2, args->lambda2);
   OCCAM_TRY(launch_finalize1(b, L, ws, s1, nullptr, args->lambda1, 1, out->ref1, keep1, n1_vis, &args->stage1, s2,
                              &plan, out->count_out, out->count_vis, st, trace, out->n_eff,
-                             args->rule == OCCAM_RULE_MEAN ? 1 : 0, out->near1, near_rel));
+                             args->rule == OCCAM_RULE_MEAN ? 1 : 0, out->near1, near_rel, true));
   if (k2_stage) {
     // the S1 rows of K2 (only those) into the device staging tensor
     const NvtxRange nvtx("stage_k2_rows");

@@ -98,6 +98,16 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// Programmatic dependent launch. A kernel launched with the programmatic
+// stream-serialization attribute may start once every CTA of the kernel
+// before it in the stream has called pdl_trigger() (or exited); until it
+// calls pdl_wait() it may read only what was complete before that kernel
+// started (inputs, earlier kernels' results). pdl_wait() returns once the
+// previous kernel has finished and its writes are visible. Both are no-ops
+// for kernels launched without the attribute.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // N exclusive prefix sums over the block at once (three barriers in all, as
 // for one): excl[k] = sum of v[k] over the threads before this one, total[k]
 // = the block's sum. tmp: N * 33 ints of shared memory.

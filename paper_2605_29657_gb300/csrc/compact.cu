@@ -53,14 +53,15 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
   __shared__ float s_tau[kScanSmemSamples];
   const int tid = threadIdx.x;
   if (tid == 0) s_tile = atomicAdd(p.ticket, 1);
-  // the row offsets and (Stage-II threshold mode) the samples' thresholds,
-  // loaded while the ticket is drawn
+  // the row offsets (an input) while the ticket is drawn; then, once the
+  // kernel before this one has finished (its s2, thresholds and flags), the
+  // samples' thresholds (Stage-II threshold mode)
   const bool ro_smem = p.bt.B <= kScanSmemSamples;
-  if (ro_smem) {
+  if (ro_smem)
     for (int b = tid; b <= p.bt.B; b += blockDim.x) s_ro[b] = p.bt.row_off[b];
-    if (p.mode != 0)
-      for (int b = tid; b < p.bt.B; b += blockDim.x) s_tau[b] = p.tau2[b];
-  }
+  pdl_wait();
+  if (ro_smem && p.mode != 0)
+    for (int b = tid; b < p.bt.B; b += blockDim.x) s_tau[b] = p.tau2[b];
   const int64_t* row_off = ro_smem ? s_ro : p.bt.row_off;
   const float* tau2 = ro_smem ? s_tau : p.tau2;
   __syncthreads();
@@ -235,6 +236,7 @@ __global__ void __launch_bounds__(256) scan_kernel(ScanParams p) {
     const long long total = s_prefix + tile_total;
     for (int bb = p.bt.B; bb >= 0 && row_off[bb] >= R; --bb) p.out_off[bb] = total;
   }
+  pdl_trigger();  // the gather kernel may be scheduled (it waits for these results)
 }
 
 // A batch with no rows at all has no scan tile: its offsets are all zero.
@@ -247,6 +249,7 @@ __global__ void __launch_bounds__(256) gather_kernel(GatherParams p) {
   const int lane = threadIdx.x & 31;
   const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  pdl_wait();  // the scan's offsets and row list
   const int64_t total = min(p.out_off[p.B], p.capacity);
   const int64_t items = total * p.n_tensors;
   for (int64_t w = gw; w < items; w += nw) {

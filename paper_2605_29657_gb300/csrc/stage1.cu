@@ -96,6 +96,10 @@ __global__ void __launch_bounds__(cls::kThreads) stage1_logits_kernel(Stage1ClsP
   int it = 0;
   for (; it < ntiles; ++it) {
     const int st = it % kStages;
+    // at its last tile the CTA lets the finalize kernel start its input-only
+    // prologue (triggered late, so that waiting finalize CTAs do not hold
+    // SMs that other work in flight could use)
+    if (it == ntiles - 1) pdl_trigger();
     if (!mbar_wait(&bar[st], (it / kStages) & 1, kSpinLimit)) timed_out = true;
     if (__syncthreads_or(timed_out)) {
       timed_out = true;
@@ -191,6 +195,27 @@ __device__ __forceinline__ void merge_softmax_stats(float& M, float& Z, float& T
   }
 }
 
+// The [CLS] key's own logit per head, l_cls,h = q_cls,h . k_cls,h in log2
+// units (-inf without a [CLS] key), into lcls_s[16] (shared): 16 threads per
+// head, dims sub, sub + 16, ... It reads only inputs, so it may run before
+// the logits kernel has finished. The caller synchronizes before lcls_s is
+// read.
+__device__ __forceinline__ void cls_self_logits(const Stage1FinalizeParams& p, int seg, float* lcls_s) {
+  constexpr int H = 16;
+  const int D = p.d1;
+  const int tid = threadIdx.x;
+  const int hh = tid >> 4, sub = tid & 15;
+  float acc = 0.f;
+  if (p.k_cls) {
+    const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + hh) * D;
+    const __nv_bfloat16* kp = p.k_cls + ((int64_t)seg * H + hh) * D;
+    for (int d = sub; d < D; d += 16) acc = fmaf(__bfloat162float(qp[d]), __bfloat162float(kp[d]), acc);
+  }
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (sub == 0) lcls_s[hh] = p.k_cls ? acc * p.scale : -INFINITY;
+}
+
 // [CLS] mode (Sec. 3.4, Eq. 4; App. A, Eq. 10): per head h the softmax of the
 // [CLS] row over {k_cls} u rows(segment), s1 = mean over heads. The logits
 // come in log2 units (the logits kernel scales by log2(e) / sqrt(d1)), so
@@ -199,18 +224,17 @@ __device__ __forceinline__ void merge_softmax_stats(float& M, float& Z, float& T
 // e (x - max); the block merges them in fixed order; a second pass forms s1
 // per row. Both read the logits from global memory (written just before by
 // the logits kernel: L2, and L1 for the second pass). s1 is written to s1_out
-// (global) and, when given, to s1_loc (shared).
+// (global) and, when given, to s1_loc (shared). lcls_s: the [CLS] key's own
+// logit per head (cls_self_logits), in shared memory.
 __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, int seg, int64_t sb, int n,
-                                               float* s1_loc) {
+                                               float* s1_loc, const float* lcls_s) {
   constexpr int H = 16;
-  const int D = p.d1;
   __shared__ float rm[16][17], rz[16][17], rt[16][17];
-  __shared__ float gmax[16], ginv[16], lcls_s[16];
+  __shared__ float gmax[16], ginv[16];
   const int tid = threadIdx.x;
   // thread t takes head (t & 15) of rows (t >> 4) + 16 k: a warp reads 32
   // consecutive floats per row pair. Up to 40 rows' loads are in flight at
-  // once (issued before the [CLS] key's dot product below, which they
-  // overlap), so a segment of up to 640 rows (a 576-token crop with its
+  // once, so a segment of up to 640 rows (a 576-token crop with its
   // registers) costs one L2 round trip.
   constexpr int KC = 40;
   const float* lg = p.logits + sb * H;
@@ -224,19 +248,6 @@ __device__ __forceinline__ void cls_softmax_s1(const Stage1FinalizeParams& p, in
     }
   };
   load_chunk(j);
-  {
-    // l_cls,h: 16 threads per head, dims sub, sub + 16, ...
-    const int hh = tid >> 4, sub = tid & 15;
-    float acc = 0.f;
-    if (p.k_cls) {
-      const __nv_bfloat16* qp = p.q_cls + ((int64_t)seg * H + hh) * D;
-      const __nv_bfloat16* kp = p.k_cls + ((int64_t)seg * H + hh) * D;
-      for (int d = sub; d < D; d += 16) acc = fmaf(__bfloat162float(qp[d]), __bfloat162float(kp[d]), acc);
-    }
-#pragma unroll
-    for (int o = 8; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (sub == 0) lcls_s[hh] = p.k_cls ? acc * p.scale : -INFINITY;
-  }
   float m = -INFINITY, z = 0.f, t = 0.f;
   for (int r0 = j;;) {
     float cm = x[0];
@@ -320,6 +331,11 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
   const int s0 = p.bt.seg_first[b], s_next = p.bt.seg_first[b + 1];
   const int64_t row_b = p.bt.row_off[b], row_b1 = p.bt.row_off[b + 1];
   const int64_t reg0 = ra + tid < rb ? (int64_t)p.bt.reg_idx[ra + tid] : -1;
+  __shared__ float lcls_s[16];
+  if (p.logits) cls_self_logits(p, seg, lcls_s);
+  // everything above reads inputs only; what follows reads the previous
+  // kernel's results (logits, or s1 in mutual mode)
+  pdl_wait();
   const bool staged = n <= p.smem_rows;
   // shared layout for a staged segment: [s1][role]
   float* s1_loc = reinterpret_cast<float*>(fin_smem);
@@ -327,7 +343,7 @@ __global__ void __launch_bounds__(256) stage1_finalize_kernel(Stage1FinalizePara
 
   const float* s1g = p.logits ? p.s1_out : p.s1;  // the segment's s1 in global memory
   if (p.logits) {
-    cls_softmax_s1(p, seg, sb, n, staged ? s1_loc : nullptr);
+    cls_softmax_s1(p, seg, sb, n, staged ? s1_loc : nullptr, lcls_s);
   } else if (staged) {
     for (int r = tid; r < n; r += blockDim.x) s1_loc[r] = s1g[sb + r];
   }

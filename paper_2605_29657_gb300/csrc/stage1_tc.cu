@@ -560,6 +560,7 @@ __global__ void __launch_bounds__(256) mutual_reduce_kernel(MutualTcParams p) {
     p.s1[r] = v;
     if (p.s2_zero) p.s2_zero[r] = 0.f;
   }
+  pdl_trigger();  // the finalize kernel may start its input-only prologue
 }
 
 void launch_mutual_tc(const MutualTcParams& p, const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mq1,
