@@ -585,6 +585,8 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     q16.queue = p.counters + CNT_QUEUE16;
     const int ncl16 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 16));
     if (launch_fused(16, mq, mk, mkt, q16, ncl16, st) != 0) return OCCAM_ERR_CUDA;
+    // head-split tiles (small batches) meet right behind the 16-CTA launch
+    launch_s2_merge(q16, st);
     // the two-pass kernels (samples the fused kernel cannot hold; often none)
     // follow the 8-CTA launch on the second stream. They are enqueued after
     // the 16-CTA launch: a CTA of theirs takes a whole SM, and enqueued
@@ -596,8 +598,6 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     if (!only16 && launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
     OCCAM_CUDA(cudaEventRecord(side.join, side.stream));
     OCCAM_CUDA(cudaStreamWaitEvent(st, side.join, 0));
-    // head-split tiles (small batches) meet here
-    launch_s2_merge(q16, st);
     OCCAM_CUDA(cudaGetLastError());
     trace.mark(st);
   } else {

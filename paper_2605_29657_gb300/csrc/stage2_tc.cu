@@ -784,6 +784,7 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   }
 
   // ------------------------------------------------------------ teardown
+  pdl_trigger();  // a head-split merge behind this launch may be scheduled
   tc::fence_before();
   __syncthreads();
   if (sm.abort && tid == 0) {
@@ -828,10 +829,17 @@ __global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParam
   const int rows = min(kHsRows, g.M - g.j0);
   const float invH = 1.0f / (float)p.H;
   float rc = 0.f;
+  int row_id = 0;
+  bool is_reg = false;
   if (k < g.own_img) {
-    int row_id = p.dense[g.rbase + g.img0 + k];
+    row_id = p.dense[g.rbase + g.img0 + k];
     if (!in_bounds(row_id >= 0 && row_id < p.bt.total_rows, p.status, kSiteFusedKeyRow)) row_id = 0;
-    const bool is_reg = p.role[row_id] != 0;
+    is_reg = p.role[row_id] != 0;
+  }
+  // all of the above comes from the Stage-I finalize kernel; the fused
+  // kernel's partials (and its s2 and slot writes) only after it finished
+  pdl_wait();
+  if (k < g.own_img) {
     const float* src = p.ppart + (((int64_t)t * kHsGroups * 16 + rank) * kHsRows) * PMAX + k;
     float cmax = 0.f, rsum = 0.f;
     // eight rows at a time, every group's load issued before any add (up to
@@ -893,7 +901,19 @@ __global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParam
 
 void launch_s2_merge(const Stage2TcParams& q, cudaStream_t st) {
   if (q.ppart) {
-    s2_merge_kernel<<<kHsMaxTiles * 16, kFusedMaxOwnImg, 0, st>>>(q);
+    // launched right behind the 16-CTA fused kernel with programmatic
+    // stream serialization: its item, geometry and key-row loads overlap the
+    // end of that kernel, and it waits for the partials (pdl_wait)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kHsMaxTiles * 16);
+    cfg.blockDim = dim3(kFusedMaxOwnImg);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, s2_merge_kernel, q);
     count_launch();
   }
 }
