@@ -809,29 +809,34 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
 }
 
 // Merge of head-split tiles. CTA (t, rank) of a kHsMaxTiles x 16 grid takes
-// tile t's S1 keys of cluster rank `rank`, one key column per thread: it sums
-// the head groups' partials (in group order) row by row, takes the column
-// max over the tile's text rows into s2, and sums the register columns over
-// rows. The register sums of the CTA's columns, added in a fixed order, fill
-// the tile's partial slots of that rank. The sample's last slot writer turns
-// the slots into ref2 and tau2 as the fused kernel does.
-__global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParams p) {
+// tile t's S1 keys of cluster rank `rank`: key column k and row quarter q
+// belong to thread q * kFusedMaxOwnImg + k. A thread sums the head groups'
+// partials (in group order) for each of its rows (rows q, q + 4, ...), with
+// every load of its rows issued before the adds, and keeps their max and
+// sum; the four quarters then meet in shared memory in quarter order. The
+// column max over the tile's text rows goes to s2; the register columns'
+// sums over rows, added over the CTA's columns in a fixed order, fill the
+// tile's partial slots of that rank. The sample's last slot writer turns the
+// slots into ref2 and tau2 as the fused kernel does.
+constexpr int kMergeQ = 4;                            // row quarters per key column
+constexpr int kMergeThreads = kMergeQ * kFusedMaxOwnImg;
+__global__ void __launch_bounds__(kMergeThreads) s2_merge_kernel(Stage2TcParams p) {
   using namespace s2f;
   constexpr int NW = kFusedMaxOwnImg / 32;
   __shared__ float wsum[NW];
+  __shared__ float2 qpart[kMergeQ][kFusedMaxOwnImg];  // (column max, column sum) per row quarter
   __shared__ int s_last;
   const int t = blockIdx.x / 16, rank = blockIdx.x % 16;
   if (t >= p.counters[CNT_NHS]) return;
   const int4 it = p.itemsHS[t];
   const int nhg = it.w;
   const ItemGeom g = item_geom<16>(p, make_int4(it.x, it.y, it.z, 0), rank);
-  const int k = threadIdx.x, lane = k & 31;
+  const int k = threadIdx.x % kFusedMaxOwnImg, q = threadIdx.x / kFusedMaxOwnImg, lane = threadIdx.x & 31;
   const int rows = min(kHsRows, g.M - g.j0);
   const float invH = 1.0f / (float)p.H;
-  float rc = 0.f;
   int row_id = 0;
   bool is_reg = false;
-  if (k < g.own_img) {
+  if (q == 0 && k < g.own_img) {
     row_id = p.dense[g.rbase + g.img0 + k];
     if (!in_bounds(row_id >= 0 && row_id < p.bt.total_rows, p.status, kSiteFusedKeyRow)) row_id = 0;
     is_reg = p.role[row_id] != 0;
@@ -839,21 +844,24 @@ __global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParam
   // all of the above comes from the Stage-I finalize kernel; the fused
   // kernel's partials (and its s2 and slot writes) only after it finished
   pdl_wait();
+  float cmax = 0.f, rsum = 0.f;
   if (k < g.own_img) {
     const float* src = p.ppart + (((int64_t)t * kHsGroups * 16 + rank) * kHsRows) * PMAX + k;
-    float cmax = 0.f, rsum = 0.f;
-    // eight rows at a time, every group's load issued before any add (up to
-    // 32 loads in flight); the sums still run in group order, then row order
-    for (int r0 = 0; r0 < rows; r0 += 8) {
+    // this thread's rows q, q + 4, ..., up to eight at a time with every
+    // group's load in flight before the adds; sums in group order, then row
+    // order
+    for (int r0 = q; r0 < rows; r0 += 8 * kMergeQ) {
       float v[8][kHsGroups];
 #pragma unroll
       for (int u = 0; u < 8; ++u)
 #pragma unroll
-        for (int hg = 0; hg < kHsGroups; ++hg)
-          v[u][hg] = (r0 + u < rows && hg < nhg) ? __ldcg(src + ((int64_t)hg * 16 * kHsRows + r0 + u) * PMAX) : 0.f;
+        for (int hg = 0; hg < kHsGroups; ++hg) {
+          const int r = r0 + u * kMergeQ;
+          v[u][hg] = (r < rows && hg < nhg) ? __ldcg(src + ((int64_t)hg * 16 * kHsRows + r) * PMAX) : 0.f;
+        }
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
-        if (r0 + u < rows) {
+        if (r0 + u * kMergeQ < rows) {
           float x = v[u][0];
 #pragma unroll
           for (int hg = 1; hg < kHsGroups; ++hg) x += v[u][hg];
@@ -862,16 +870,29 @@ __global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParam
         }
       }
     }
-    if (is_reg) {
-      rc = rsum * invH;
-    } else {
-      atomicMax(reinterpret_cast<int*>(&p.s2[row_id]), __float_as_int(cmax * invH));
-    }
   }
-  rc = warp_sum_f(rc);
-  if (lane == 0) wsum[k >> 5] = rc;
+  qpart[q][k] = make_float2(cmax, rsum);
   __syncthreads();
-  if (k == 0) {
+  float rc = 0.f;
+  if (q == 0) {
+    if (k < g.own_img) {
+      float cm = qpart[0][k].x, rs = qpart[0][k].y;
+#pragma unroll
+      for (int qq = 1; qq < kMergeQ; ++qq) {
+        cm = fmaxf(cm, qpart[qq][k].x);
+        rs += qpart[qq][k].y;
+      }
+      if (is_reg) {
+        rc = rs * invH;
+      } else {
+        atomicMax(reinterpret_cast<int*>(&p.s2[row_id]), __float_as_int(cm * invH));
+      }
+    }
+    rc = warp_sum_f(rc);
+    if (lane == 0) wsum[k >> 5] = rc;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
     float acc = 0.f;
     for (int w = 0; w < NW; ++w) acc += wsum[w];
     // the tile's NPW slots of this rank: the sum in the first, zeros after
@@ -882,7 +903,7 @@ __global__ void __launch_bounds__(kFusedMaxOwnImg) s2_merge_kernel(Stage2TcParam
     s_last = atomicAdd(&p.done[g.b], NPW) == nslots - NPW;
   }
   __syncthreads();
-  if (s_last && k < 32) {
+  if (s_last && threadIdx.x < 32) {
     // the sample's last partials: ref2 = (sum of the partials) / (R M),
     // lane l taking slots l, l + 32, ... in order, then a fixed tree
     __threadfence();
@@ -906,7 +927,7 @@ void launch_s2_merge(const Stage2TcParams& q, cudaStream_t st) {
     // end of that kernel, and it waits for the partials (pdl_wait)
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(kHsMaxTiles * 16);
-    cfg.blockDim = dim3(kFusedMaxOwnImg);
+    cfg.blockDim = dim3(kMergeThreads);
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
