@@ -516,6 +516,19 @@ Stage2Params stage2_params(const occam_batch* b, const occam_stage2_args* a, con
 }
 
 // Stage II after the Stage-I finalize kernel planned it (same arguments).
+// Clusters a fused launch of C-CTA clusters makes: no more than the device
+// holds at once (a cluster must fit in one GPC). Launched clusters beyond
+// that cannot be placed until resident ones leave, and while they wait, the
+// clusters of the launch beside it on the other stream are not placed either
+// (measured: the 8-CTA clusters of the Qwen3-VL-shaped batch started only
+// when the 16-CTA launch's surplus clusters were placed). Items come from the
+// launch's queue, so fewer clusters lose no work.
+int fused_launch_clusters(int C, int64_t max_items, int sms) {
+  const int res = fused_resident_clusters(C);
+  const int64_t cap = res > 0 ? res : sms / C;
+  return (int)std::max<int64_t>(1, std::min<int64_t>(max_items, cap));
+}
+
 int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayout& L, void* ws, float* s2,
                   float* ref2, float lambda2, cudaStream_t st, Trace trace = Trace()) {
   const NvtxRange nvtx("stage2_scores");
@@ -574,7 +587,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     Stage2TcParams q8 = q;
     q8.items = p.itemsF8;
     q8.queue = p.counters + CNT_QUEUE8;
-    const int ncl8 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 8));
+    const int ncl8 = fused_launch_clusters(8, L.maxF, sms);
     if (!only16 && launch_fused(8, mq, mk, mkt, q8, ncl8, side.stream) != 0) return OCCAM_ERR_CUDA;
     // samples too large for 8 CTAs: 16-CTA clusters, on this stream ahead of
     // the 4-CTA launch. A launch without items returns at once; it also
@@ -583,7 +596,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     Stage2TcParams q16 = q;
     q16.items = p.itemsF16;
     q16.queue = p.counters + CNT_QUEUE16;
-    const int ncl16 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 16));
+    const int ncl16 = fused_launch_clusters(16, L.maxF, sms);
     if (launch_fused(16, mq, mk, mkt, q16, ncl16, st) != 0) return OCCAM_ERR_CUDA;
     // head-split tiles (small batches) meet right behind the 16-CTA launch
     launch_s2_merge(q16, st);
@@ -594,7 +607,7 @@ int launch_stage2(const occam_batch* b, const occam_stage2_args* a, const WsLayo
     // SMs of one GPC, could be placed.
     OCCAM_TRY(launch_twopass(p, L, sms, b, a, side.stream));
     q.queue = p.counters + CNT_QUEUE4;
-    const int ncl4 = (int)std::max<int64_t>(1, std::min<int64_t>(L.maxF, sms / 4));
+    const int ncl4 = fused_launch_clusters(4, L.maxF, sms);
     if (!only16 && launch_fused(4, mq, mk, mkt, q, ncl4, st) != 0) return OCCAM_ERR_CUDA;
     OCCAM_CUDA(cudaEventRecord(side.join, side.stream));
     OCCAM_CUDA(cudaStreamWaitEvent(st, side.join, 0));
