@@ -332,9 +332,12 @@ __global__ void __launch_bounds__(s2f::THREADS, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rank = (int)tc::cluster_rank();
   const int nF = p.counters[C == 16 ? CNT_NF16 : C == 8 ? CNT_NF8 : CNT_NF];
-  // no work for this cluster size (every CTA of every cluster reads the same
-  // count): leave before touching shared memory, TMEM or the cluster
-  if (nF == 0) return;
+  // no work for this cluster (every CTA of every cluster reads the same
+  // count): leave before touching shared memory, TMEM or the cluster. With
+  // nF items, the clusters numbered nF and up can never be handed one (at
+  // most nF hand-outs succeed and the first nF clusters keep drawing until
+  // the queue is empty), so they leave too, freeing their SMs at once.
+  if ((int)blockIdx.x / C >= nF) return;
   volatile int* abort = &sm.abort;
 
   if (tid == 0) {
